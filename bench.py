@@ -1,0 +1,576 @@
+#!/usr/bin/env python3
+"""Benchmark of the GB300 privacy-intent validator.
+
+Default workload: the end-to-end cross-layer configuration (10,000 intents on
+1,024 nodes x 32 label keys attached to a 512-switch random graph with 1,000
+rules per switch; per intent a node-selector conjunction, a region mask, 4
+pods placed by seeded choice among feasible nodes and 5,000 probes; 50M
+probes, hop cap 32).  One step = selector rows -> placement -> probe binding
+-> hop-synchronous walks -> per-intent verdicts, all in libpv's kernels.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload e2e|placement|flow|wan]
+
+Prints one JSON line (rank 0).  `value` is device-timed throughput with the
+inputs resident in HBM (CUDA events on the launching stream, K steps after W
+warm-ups, max over ranks); `e2e` is the same metric through the public API
+from pinned host buffers (loads, host->device copies, the step and the
+device->host read of the verdicts inside the timed region).  Under torchrun
+each rank processes its own shard (seed offset by rank): weak scaling, no
+collective on the data path.  `--impl reference` times the CPU oracle on a
+bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2602_16100_gb300 import workloads as W  # noqa: E402
+
+METRIC = "probe-hop verifications/s and pod×node selector evals/s; % of HBM peak"
+HBM_FALLBACK_GBS = 6800.0
+
+
+# ----------------------------------------------------------------------------
+# environment helpers
+# ----------------------------------------------------------------------------
+def hbm_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return HBM_FALLBACK_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu_index = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            cmd = ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200"]
+            if self.gpu_index is not None:
+                cmd += ["-i", str(self.gpu_index)]
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.result = None
+        if self.proc is None:
+            return
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out = ""
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(n)
+        if sm:
+            self.result = {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                           "samples": len(sm)}
+
+
+def source_hash(*names):
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2602_16100_gb300", "csrc", n), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(kernel: str, src_hash: str):
+    """DRAM bytes per unit from the committed ncu summary, if it was taken on
+    the current kernel source (else None)."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)[kernel]
+        return float(d["dram_bytes_per_unit"]) if d.get("source_hash") == src_hash else None
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------------------
+# workloads
+# ----------------------------------------------------------------------------
+class EndToEndBench:
+    name = "end-to-end cross-layer"
+    unit = "probe-hop verifications/s"
+
+    def __init__(self, seed):
+        self.e = W.end_to_end(seed=20260220 + seed)
+
+    def config(self):
+        e = self.e
+        return {"workload": self.name, "intents": e.intents.num_pods, "nodes": e.cluster.num_nodes,
+                "label_keys": e.cluster.num_keys, "switches": e.network.num_switches,
+                "rules_per_switch": int(np.diff(e.network.rule_offs).max()), "pods_per_intent": e.pods_per_intent,
+                "probes": len(e.probes.probes), "hop_cap": e.probes.hop_cap,
+                "l2": "inputs larger than L2 (800 MB probe array and 200 MB results per step)"}
+
+    def setup(self, v):
+        self.v = v
+        v.load_cluster(self.e.cluster)
+        v.load_network(self.e.network)
+        self.dev, self.sizes = v.alloc_end_to_end(self.e)
+
+    def step(self, stream):
+        self.v.run_end_to_end(self.dev, self.sizes, stream)
+
+    def measure_units(self):
+        import torch
+        res = self.dev["results"].view(-1, 4)
+        self.probe_hops = int(res[:, 1].to(torch.int64).sum().item())
+        self.selector_evals = self.e.intents.num_pods * self.e.cluster.num_nodes
+        self.status_hist = torch.bincount(res[:, 0].to(torch.int64), minlength=6).tolist()
+        self.pass_count = int(self.dev["pass"][: self.e.intents.num_pods].to(torch.int64).sum().item())
+        return self.probe_hops
+
+    def extra(self, secs_per_step):
+        return {"selector_evals_per_s": self.selector_evals / secs_per_step,
+                "probe_hops_per_step": self.probe_hops,
+                "status_histogram": dict(zip(W.STATUS_NAMES, self.status_hist)),
+                "intents_passed": self.pass_count}
+
+    def algorithmic_bytes(self, group):
+        e = self.e
+        I = e.intents.num_pods
+        M = len(e.probes.probes)
+        if group == "walk_hop":         # per probe-hop: 16 B probe record read + 4 B result / state written
+            return 20 * self.probe_hops
+        if group == "walk_regroup":     # per probe-hop: 8 B state read + 8 B state written
+            return 16 * self.probe_hops
+        if group == "selector":
+            return I * W.words_per_row(e.cluster.num_nodes) * 4 + len(e.intents.exprs) * 20 + I * 5
+        if group == "bind":
+            return M * 16 * 2
+        if group == "aggregate":
+            return M * 4 + I * 33
+        if group == "walk_init":
+            return M * 16
+        return 0
+
+    def traffic_unit(self, group):
+        return self.probe_hops if group in ("walk_hop", "walk_regroup") else None
+
+    # host-buffer end-to-end step through the public API
+    def setup_e2e(self, v):
+        import torch
+        e = self.e
+        self.h_probes = torch.from_numpy(e.probes.probes.view(np.uint8).reshape(-1)).pin_memory()
+        self.h_offs = torch.from_numpy(e.intents.expr_offs.astype(np.uint32).view(np.uint8)).pin_memory()
+        self.h_exprs = torch.from_numpy(e.intents.exprs.view(np.uint8).reshape(-1)).pin_memory()
+        self.h_draws = torch.from_numpy(e.place_draws.astype(np.uint64).view(np.uint8)).pin_memory()
+        self.h_pass = torch.empty(e.intents.num_pods, dtype=torch.uint8).pin_memory()
+        self.h_counts = torch.empty(e.intents.num_pods * 32, dtype=torch.uint8).pin_memory()
+        net = e.network
+        self.h2d = (self.h_probes.numel() + self.h_offs.numel() + self.h_exprs.numel() + self.h_draws.numel()
+                    + e.cluster.labels.nbytes + net.rule_offs.nbytes + net.rules.nbytes + net.switch_region.nbytes
+                    + net.port_offs.nbytes + net.port_peer.nbytes + net.host_switch.nbytes + net.host_port.nbytes
+                    + net.host_ip.nbytes)
+        self.d2h = self.h_pass.numel() + self.h_counts.numel()
+
+    def step_e2e(self, v, stream):
+        e, dev = self.e, self.dev
+        v.load_cluster(e.cluster)
+        v.load_network(e.network)
+        dev["probes"][: self.h_probes.numel()].copy_(self.h_probes, non_blocking=True)
+        dev["offs"][: self.h_offs.numel()].copy_(self.h_offs, non_blocking=True)
+        dev["exprs"][: self.h_exprs.numel()].copy_(self.h_exprs, non_blocking=True)
+        dev["draws"][: self.h_draws.numel()].copy_(self.h_draws, non_blocking=True)
+        v.run_end_to_end(dev, self.sizes, stream)
+        self.h_pass.copy_(dev["pass"][: self.h_pass.numel()], non_blocking=True)
+        self.h_counts.copy_(dev["counts"][: self.h_counts.numel()], non_blocking=True)
+
+    # oracle on a bounded sample: the first n intents, whole pipeline
+    def oracle_sample(self, n_intents):
+        import oracle
+        e = self.e
+        c = e.cluster
+        ppg, pods = e.probes_per_intent, e.pods_per_intent
+        offs = e.intents.expr_offs[: n_intents + 1].astype(np.uint32)
+        exprs = e.intents.exprs[: int(offs[-1])]
+        t0 = time.perf_counter()
+        bits, flags = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, offs, exprs)
+        assign = oracle.place_pods(bits, c.num_nodes, pods, e.place_draws[: n_intents * pods])
+        probes = oracle.bind_probes(e.probes.probes[: n_intents * ppg], ppg, pods, assign, e.network.host_ip)
+        res = oracle.verify_probes(e.network, probes, e.probes.hop_cap)
+        oracle.aggregate(bits, c.num_nodes, flags, assign, pods, res, ppg)
+        dt = time.perf_counter() - t0
+        units = int(res["hops"].astype(np.int64).sum())
+        return units, dt, f"first {n_intents} intents ({n_intents * ppg} probes), whole pipeline"
+
+    oracle_start = 2
+
+
+class PlacementBench:
+    name = "placement-scale"
+    unit = "pod×node selector evals/s"
+
+    def __init__(self, seed):
+        d = W.selector_workload(seed=20260217 + seed)
+        self.c, self.s = d["cluster"], d["selectors"]
+
+    def config(self):
+        return {"workload": self.name, "nodes": self.c.num_nodes, "label_keys": self.c.num_keys,
+                "pods": self.s.num_pods, "expressions": len(self.s.exprs),
+                "l2": "output bitsets (64 MB) rewritten each step; labels and value rows L2-resident"}
+
+    def setup(self, v):
+        from paper_2602_16100_gb300.validator import to_device, empty_device
+        self.v = v
+        v.load_cluster(self.c)
+        d = v.device
+        self.words = W.words_per_row(self.c.num_nodes)
+        self.d_offs = to_device(self.s.expr_offs.astype(np.uint32), d)
+        self.d_exprs = to_device(self.s.exprs, d)
+        self.d_assign = to_device(self.s.assign.astype(np.uint32), d)
+        self.d_bits = empty_device(self.s.num_pods * self.words * 4, d)
+        self.d_flags = empty_device(self.s.num_pods, d)
+
+    def step(self, stream):
+        self.v.eval_selectors(self.d_offs, len(self.s.exprs), self.d_exprs, self.d_assign, self.s.num_pods,
+                              words=self.words, d_bits=self.d_bits, d_flags=self.d_flags, stream=stream)
+
+    def measure_units(self):
+        return self.s.num_pods * self.c.num_nodes
+
+    def extra(self, secs_per_step):
+        return {}
+
+    def algorithmic_bytes(self, group):
+        if group != "selector":
+            return 0
+        P = self.s.num_pods
+        return P * self.words * 4 + len(self.s.exprs) * 20 + P * 4 * 2 + P + self.c.labels.nbytes
+
+    def traffic_unit(self, group):
+        return self.s.num_pods if group == "selector" else None
+
+    def oracle_sample(self, n):
+        import oracle
+        idx = np.arange(n)
+        offs = self.s.expr_offs[: n + 1].astype(np.uint32)
+        ex = self.s.exprs[: int(offs[-1])]
+        t0 = time.perf_counter()
+        oracle.eval_selectors(self.c.num_nodes, self.c.num_keys, self.c.labels, offs, ex, self.s.assign[idx])
+        dt = time.perf_counter() - t0
+        return n * self.c.num_nodes, dt, f"first {n} pods"
+
+    oracle_start = 500
+
+
+class FlowBench:
+    name = "flow-verification"
+    unit = "probe-hop verifications/s"
+
+    def __init__(self, seed):
+        d = W.fat_tree(seed=20260218 + seed)
+        self.net, self.p = d["network"], d["probes"]
+
+    def config(self):
+        return {"workload": self.name, "switches": self.net.num_switches, "hosts": self.net.num_hosts,
+                "rules_per_switch": int(np.diff(self.net.rule_offs).max()), "probes": len(self.p.probes),
+                "hop_cap": self.p.hop_cap, "l2": "inputs larger than L2 (160 MB probes, 40 MB results)"}
+
+    def setup(self, v):
+        from paper_2602_16100_gb300.validator import to_device, empty_device
+        self.v = v
+        v.load_network(self.net)
+        self.d_probes = to_device(self.p.probes, v.device)
+        self.d_out = empty_device(len(self.p.probes) * 4, v.device)
+
+    def step(self, stream):
+        self.v.verify_probes(self.d_probes, len(self.p.probes), self.p.hop_cap, d_out=self.d_out, stream=stream)
+
+    def measure_units(self):
+        import torch
+        res = self.d_out.view(-1, 4)
+        self.probe_hops = int(res[:, 1].to(torch.int64).sum().item())
+        self.hist = torch.bincount(res[:, 0].to(torch.int64), minlength=6).tolist()
+        return self.probe_hops
+
+    def extra(self, secs_per_step):
+        return {"probe_hops_per_step": self.probe_hops, "status_histogram": dict(zip(W.STATUS_NAMES, self.hist))}
+
+    def algorithmic_bytes(self, group):
+        return {"walk_hop": 20, "walk_regroup": 16}.get(group, 0) * self.probe_hops + \
+            (len(self.p.probes) * 16 if group == "walk_init" else 0)
+
+    def traffic_unit(self, group):
+        return self.probe_hops if group in ("walk_hop", "walk_regroup") else None
+
+    def oracle_sample(self, n):
+        import oracle
+        idx = np.arange(n, dtype=np.uint32)
+        t0 = time.perf_counter()
+        r = oracle.verify_probes(self.net, self.p.probes, self.p.hop_cap, idx=idx)
+        dt = time.perf_counter() - t0
+        return int(r["hops"].astype(np.int64).sum()), dt, f"first {n} probes"
+
+    oracle_start = 2000
+
+
+class WanBench:
+    name = "continuum WAN"
+    unit = "compliant-reach (mask, source) rows/s"
+
+    def __init__(self, seed):
+        self.q = W.continuum_wan(seed=20260219 + seed)
+
+    def config(self):
+        g = self.q.graph
+        return {"workload": self.name, "vertices": g.num_vertices, "edges": len(g.cols),
+                "masks": len(self.q.masks), "sources": len(self.q.sources),
+                "l2": "output rows (128 MB) rewritten each step"}
+
+    def setup(self, v):
+        from paper_2602_16100_gb300.validator import to_device, empty_device
+        self.v = v
+        d = v.device
+        self.g = v.upload_graph(self.q.graph)
+        self.d_src = to_device(self.q.sources.astype(np.uint32), d)
+        self.d_masks = to_device(self.q.masks.astype(np.uint32), d)
+        self.words = W.words_per_row(self.q.graph.num_vertices)
+        self.d_out = empty_device(len(self.q.masks) * len(self.q.sources) * self.words * 4, d)
+
+    def step(self, stream):
+        self.v.compliant_reach(self.g, len(self.q.sources), self.d_src, len(self.q.masks), self.d_masks,
+                               words=self.words, d_reach=self.d_out, stream=stream)
+
+    def measure_units(self):
+        return len(self.q.masks) * len(self.q.sources)
+
+    def extra(self, secs_per_step):
+        return {}
+
+    def algorithmic_bytes(self, group):
+        if group != "reach":
+            return 0
+        return len(self.q.masks) * len(self.q.sources) * self.words * 4 + len(self.q.graph.cols) * 4
+
+    def traffic_unit(self, group):
+        return len(self.q.masks) * len(self.q.sources) if group == "reach" else None
+
+    def oracle_sample(self, n):
+        import oracle
+        m = len(self.q.masks)
+        pairs = np.stack([np.arange(n) % m, np.arange(n) // m], 1).astype(np.uint32)
+        t0 = time.perf_counter()
+        oracle.compliant_reach(self.q.graph, self.q.sources, self.q.masks, pairs=pairs)
+        return n, time.perf_counter() - t0, f"first {n} (mask, source) rows"
+
+    oracle_start = 256
+
+
+WORKLOADS = {"e2e": EndToEndBench, "placement": PlacementBench, "flow": FlowBench, "wan": WanBench}
+SOURCES = {"walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector": ("k_selector.cu",),
+           "reach": ("k_reach.cu",)}
+
+
+def timed_oracle(wl, target_s=12.0, cap_s=40.0):
+    """Grow the sample until one run takes >= target_s seconds of CPU."""
+    n = wl.oracle_start
+    while True:
+        units, dt, desc = wl.oracle_sample(n)
+        if dt >= target_s or dt * 2 > cap_s:
+            return units, dt, desc, n
+        n = int(n * max(1.5, min(8.0, target_s / max(dt, 1e-3))))
+
+
+# ----------------------------------------------------------------------------
+# arms
+# ----------------------------------------------------------------------------
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    wl = WORKLOADS[args.workload](0)
+    # size one step to a few seconds of single-threaded CPU work (this also
+    # serves as warm-up), then time K steps on that sample
+    _, _, desc, n = timed_oracle(wl, target_s=3.0, cap_s=20.0)
+    for _ in range(max(0, args.warmup - 1)):
+        wl.oracle_sample(max(1, n // 8))
+    tot_units, tot_s = 0, 0.0
+    for _ in range(args.steps):
+        u, d, desc = wl.oracle_sample(n)
+        tot_units += u
+        tot_s += d
+    value = tot_units / tot_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": wl.unit, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
+            "data": "synthetic", "config": wl.config(),
+            "cpu_baseline": {"value": value, "unit": wl.unit, "cores": 1, "kind": "oracle", "sample": desc},
+            "e2e": {"value": value, "unit": wl.unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    from paper_2602_16100_gb300 import binding as B
+    from paper_2602_16100_gb300 import build
+    from paper_2602_16100_gb300.validator import Validator
+    if rank == 0 or world == 1:
+        build.build_library()
+    if dist:
+        dist.barrier()
+    wl = WORKLOADS[args.workload](rank)
+    v = Validator(local)
+    wl.setup(v)
+    stream = torch.cuda.current_stream()
+    for _ in range(max(args.warmup, 1)):
+        wl.step(stream)
+    v.sync(stream)
+    units = wl.measure_units()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    gpu_index = vis.split(",")[local] if vis else local
+    barrier()
+    B.pv_profile_enable(v.ctx, True)
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(gpu_index) as clk:
+        start.record(stream)
+        for _ in range(args.steps):
+            wl.step(stream)
+        stop.record(stream)
+        B.pv_profile_collect(v.ctx, stream)
+        barrier()
+    B.pv_profile_enable(v.ctx, False)
+    ms = start.elapsed_time(stop)
+    v.sync(stream)
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    secs_per_step = ms / 1e3 / args.steps
+    value = units * world / secs_per_step
+
+    # per-kernel-group device time inside the timed region
+    kernels, launches = {}, 0
+    for gi, name in enumerate(B.PV_K_NAMES):
+        kms, n = B.pv_profile_read(v.ctx, gi)
+        if n:
+            kernels[name] = {"ms_per_step": kms / args.steps, "launches_per_step": n / args.steps,
+                             "share_of_step": kms / ms}
+            launches += n
+    dom = max(kernels, key=lambda k: kernels[k]["ms_per_step"]) if kernels else None
+    peak, peak_kind = hbm_peak()
+    roofline = None
+    if dom:
+        kd = kernels[dom]
+        n_launch = kd["launches_per_step"]
+        bytes_per_launch = wl.algorithmic_bytes(dom) / max(n_launch, 1)
+        avg_launch_s = kd["ms_per_step"] / 1e3 / max(n_launch, 1)
+        achieved = bytes_per_launch / avg_launch_s / 1e9 if avg_launch_s > 0 else 0.0
+        tr_unit = committed_traffic(dom, source_hash(*SOURCES.get(dom, ("k_walk.cu",))))
+        u = wl.traffic_unit(dom)
+        traffic = tr_unit * u / max(n_launch, 1) if (tr_unit is not None and u) else None
+        roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                    "frac": achieved / peak, "peak_source": peak_kind, "traffic": traffic,
+                    "algorithmic_bytes_per_launch": bytes_per_launch, "avg_launch_ms": avg_launch_s * 1e3}
+
+    # end-to-end through the public API from pinned host buffers
+    e2e = None
+    if hasattr(wl, "setup_e2e"):
+        wl.setup_e2e(v)
+        wl.step_e2e(v, stream)
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            wl.step_e2e(v, stream)
+        barrier()
+        e_s = (time.perf_counter() - t0) / args.steps
+        if dist:
+            t = torch.tensor([e_s], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e_s = float(t.item())
+        e2e = {"value": units * world / e_s, "unit": wl.unit, "h2d_bytes_per_step": int(wl.h2d),
+               "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        u, dt, desc, _ = timed_oracle(wl)
+        cpu = {"value": u / dt, "unit": wl.unit, "cores": 1, "kind": "oracle", "sample": desc,
+               "seconds": dt}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": wl.unit, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+                "config": {**wl.config(), "parallelism": f"independent shards x{world}"},
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+                "clocks": clk.result, "kernels": kernels, **wl.extra(secs_per_step)}
+        print(json.dumps(line), flush=True)
+    v.close()
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", choices=tuple(WORKLOADS), default="e2e")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        print("note: warmup raised to 3", file=sys.stderr)
+        args.warmup = 3
+    return run_reference(args) if args.impl == "reference" else run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,306 @@
+/*
+ * pv.h -- C ABI of the GB300 privacy-intent validator library (libpv.so).
+ *
+ * The library checks, in batches on one GPU, whether a deployed
+ * configuration C = <sigma, rho> satisfies compiled privacy intents
+ * (Sec. 3.3, "Formal Model and Satisfaction"): (i) pod placements sigma
+ * against Kubernetes node selectors over the node labels lambda_N, and
+ * (ii) the realised paths of ONOS-style flow rules against per-flow
+ * permitted-jurisdiction sets over the switch labels lambda_V.  It also
+ * answers jurisdiction-masked reachability over the topology G = (V, E).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Return value: PV_OK (0) or a PV_E* code; pv_last_error() gives a
+ *    message.  Nothing throws across the ABI.
+ *  - Ownership: a pv_ctx owns all state loaded by pv_load_* (copied from
+ *    HOST pointers into library-owned device memory) and a scratch arena
+ *    that grows on demand.  Evaluation calls take CALLER-OWNED DEVICE
+ *    pointers and a CUDA stream (NULL = legacy default stream); they only
+ *    enqueue work and return before it completes.
+ *  - Device-detected errors (malformed device-resident inputs, a bounded
+ *    wait that gave up) are recorded in a device status word and returned
+ *    by the next pv_sync() on that context.  Device kernels never read or
+ *    write out of bounds on malformed inputs.
+ *  - Bitsets: item i is bit (i & 31) of 32-bit word (i >> 5) (LSB first);
+ *    rows hold words_per_row words, words_per_row >= ceil(n / 32) and a
+ *    multiple of 4 (rows are 16-byte aligned); padding bits are written 0.
+ *  - A context is not thread-safe; use one context per host thread.
+ */
+#ifndef PV_H
+#define PV_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *pv_stream; /* same type as cudaStream_t */
+typedef struct pv_ctx pv_ctx;
+
+enum {
+    PV_OK = 0,
+    PV_EINVAL = 1,    /* argument or input out of range / malformed      */
+    PV_ENOMEM = 2,    /* device or host allocation failed                */
+    PV_ECUDA = 3,     /* a CUDA runtime call failed                      */
+    PV_ESTATE = 4,    /* required pv_load_* has not been called          */
+    PV_ETIMEOUT = 5,  /* a bounded device-side wait gave up              */
+    PV_ENOTIMPL = 6
+};
+
+/* label / selector encodings (Sec. 3.3 label functions; Sec. 4.1) */
+#define PV_ABSENT 0xFFFFu          /* node does not carry the key           */
+enum { PV_IN = 0, PV_NOTIN = 1, PV_EXISTS = 2, PV_DOESNOTEXIST = 3 };
+
+/* flow-rule / topology encodings (Sec. 4.2 per-hop flow rules) */
+#define PV_ANY_PORT 0xFFFFu        /* rule.in_port wildcard                 */
+#define PV_DROP 0xFFFFu            /* rule.action: drop                     */
+#define PV_NO_HOST 0xFFFFu         /* probe.src_host: no source host        */
+#define PV_PEER_NONE (-1)          /* port_peer: unconnected port           */
+#define PV_PEER_HOST 0x40000000    /* port_peer: PV_PEER_HOST | host id     */
+#define PV_UNPLACED 0xFFFFFFFFu    /* assign[]: pod has no feasible node    */
+
+/* limits */
+#define PV_MAX_PORTS 256           /* ports per switch (port ids 0..255)    */
+#define PV_MAX_RULES 8192          /* rules per switch                      */
+#define PV_MAX_SWITCHES 65535
+#define PV_MAX_HOSTS 65535
+#define PV_MAX_HOP_CAP 255
+
+/* probe walk statuses */
+enum {
+    PV_COMPLIANT = 0,     /* delivered to the destination host, every switch permitted */
+    PV_VIOLATION = 1,     /* visited a switch whose region is not permitted             */
+    PV_DROPPED = 2,       /* table miss, drop action, or unconnected output port       */
+    PV_LOOP = 3,          /* not terminated within hop_cap switch visits                */
+    PV_MISDELIVERED = 4,  /* delivered to a host that does not own dst_ip               */
+    PV_NOSRC = 5          /* src_host is PV_NO_HOST or out of range                      */
+};
+
+/* per-pod selector flags */
+enum {
+    PV_F_ASSIGN_OK = 1,      /* assign[p] < num_nodes and that node is feasible          */
+    PV_F_EMPTY = 2,          /* no feasible node: the intent is unenforceable, fail closed */
+    PV_F_UNKNOWN_VALUE = 4,  /* an In value is carried by no node (hallucinated id)       */
+    PV_F_PASS = 8,           /* placement check passes: ASSIGN_OK and not UNKNOWN_VALUE   */
+    PV_F_BAD_EXPR = 16       /* malformed expression list: row empty, check fails         */
+};
+
+typedef struct {           /* one matchExpression, 20 bytes                             */
+    uint16_t key;          /* label key id < num_keys                                     */
+    uint8_t op;            /* PV_IN, PV_NOTIN, PV_EXISTS, PV_DOESNOTEXIST                 */
+    uint8_t nvals;         /* 1..8 for In/NotIn, 0 for Exists/DoesNotExist                */
+    uint16_t vals[8];      /* value ids (not PV_ABSENT); entries >= nvals are ignored    */
+} pv_expr;
+
+typedef struct {           /* one flow rule, 20 bytes                                    */
+    uint16_t priority;     /* higher wins; ties go to the lower input index               */
+    uint16_t in_port;      /* port id or PV_ANY_PORT                                      */
+    uint32_t src_ip, dst_ip;  /* prefix values; bits beyond the length are ignored       */
+    uint8_t src_len, dst_len; /* prefix lengths 0..32 (0 matches everything)             */
+    uint16_t dport_lo, dport_hi; /* inclusive destination-port range, lo <= hi          */
+    uint16_t action;       /* output port id or PV_DROP                                   */
+} pv_rule;
+
+typedef struct {           /* one probe packet, 16 bytes                                 */
+    uint32_t src_ip, dst_ip;
+    uint16_t dport;
+    uint16_t src_host;     /* injecting host id, or PV_NO_HOST                            */
+    uint32_t allowed_mask; /* bit r set = switches of region r are permitted              */
+} pv_probe;
+
+typedef struct {           /* one walk result, 4 bytes                                   */
+    uint8_t status;        /* PV_COMPLIANT .. PV_NOSRC                                    */
+    uint8_t hops;          /* switch visits made (hop_cap for PV_LOOP, 0 for PV_NOSRC)   */
+    uint16_t last_switch;  /* last switch visited (0xFFFF for PV_NOSRC)                   */
+} pv_result;
+
+/* ---------------------------------------------------------------------------
+ * Context.
+ * pv_create: binds the context to CUDA device `cuda_device` (the device must
+ * be current on the calling thread for every later call).  Returns PV_ECUDA
+ * if the device cannot be used.  pv_destroy frees all device state; it
+ * accepts NULL.  pv_sync waits for `stream` and returns (and clears) the
+ * first device-detected error since the previous pv_sync.
+ * ------------------------------------------------------------------------- */
+int pv_create(pv_ctx **out, int cuda_device);
+void pv_destroy(pv_ctx *ctx);
+const char *pv_last_error(const pv_ctx *ctx);
+int pv_sync(pv_ctx *ctx, pv_stream stream);
+int pv_version(void);
+
+/* ---------------------------------------------------------------------------
+ * pv_load_cluster -- the node label function lambda_N (Sec. 3.3; label
+ * schema of Sec. 5.2, e.g. location, provider, security-level, zone).
+ *
+ * labels: HOST pointer, key-major (structure of arrays):
+ *   labels[k * num_nodes + n] = value id of key k on node n, or PV_ABSENT.
+ * Copied to the device; the library also builds the per-key inventory of
+ * carried values (for the hallucinated-identifier check of Sec. 6.3) and,
+ * when it fits its memory budget, per-(key, value) node bitsets.
+ * Errors: PV_EINVAL if num_nodes == 0, num_keys == 0 or num_keys > 65535;
+ * PV_ENOMEM.  Replaces any previously loaded cluster.
+ * ------------------------------------------------------------------------- */
+int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_keys, const uint16_t *labels);
+
+/* ---------------------------------------------------------------------------
+ * pv_eval_selectors -- placement constraints Phi_C (Sec. 3.3 satisfaction
+ * (i) and worked example; Sec. 4.1 placement directives; Sec. 5.5 compute
+ * check "a pod is scheduled only onto nodes whose labels satisfy the
+ * placement constraints").
+ *
+ * For pod p, feasible(p) = { n : every expression of p matches node n },
+ * with Kubernetes matchExpressions semantics (In: key carried and value in
+ * set; NotIn: key absent or value not in set; Exists; DoesNotExist).  An
+ * empty expression list admits every node.
+ *
+ * Device inputs: d_expr_offs[num_pods + 1] (CSR offsets into d_exprs,
+ * num_exprs entries), d_assign[num_pods] or NULL (the placement sigma).
+ * Device outputs: d_bits[num_pods][words_per_row] feasible-node bitsets;
+ * d_flags[num_pods] PV_F_* bits (ASSIGN_OK and PASS need d_assign).
+ * Malformed expression lists (offsets decreasing or beyond num_exprs, key
+ * >= num_keys, unknown op, bad nvals, PV_ABSENT as a value) give an empty
+ * row and PV_F_BAD_EXPR for that pod; they are not call errors.
+ * Errors: PV_ESTATE (no cluster), PV_EINVAL (words_per_row too small or
+ * not a multiple of 4, NULL pointers with num_pods > 0).
+ * ------------------------------------------------------------------------- */
+int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_expr_offs, uint32_t num_exprs,
+                      const pv_expr *d_exprs, const uint32_t *d_assign, uint32_t *d_bits,
+                      uint32_t words_per_row, uint8_t *d_flags, pv_stream stream);
+
+/* ---------------------------------------------------------------------------
+ * pv_load_flow_tables -- the installed per-hop flow rules rho (Sec. 4.2
+ * flow scheduling module; each path becomes per-hop rules pushed to ONOS)
+ * and the switch labels lambda_V reduced to a region id per switch
+ * (Sec. 5.2 label schema, device_labels.location).
+ *
+ * HOST inputs:
+ *   rule_offs[num_switches + 1], rules[rule_offs[num_switches]]: switch s
+ *     owns rules[rule_offs[s] .. rule_offs[s+1]) in input order;
+ *   switch_region[num_switches]: region id < 32;
+ *   port_offs[num_switches + 1], port_peer[port_offs[num_switches]]: port p
+ *     of switch s (p < port_offs[s+1]-port_offs[s] <= PV_MAX_PORTS) leads to
+ *     PV_PEER_NONE, PV_PEER_HOST | h, or the switch port (s2 << 8) | p2;
+ *   host_switch[num_hosts], host_port[num_hosts]: attachment of host h;
+ *   host_ip[num_hosts]: the address host h owns.
+ * The library sorts each switch's rules by (priority desc, input index asc)
+ * on the device and compiles them for the walk kernels.
+ * Errors: PV_EINVAL for any out-of-range field (in_port / action >= the
+ * switch's port count unless wildcard/drop, prefix length > 32, lo > hi,
+ * region >= 32, offsets not monotone, more than PV_MAX_RULES rules or
+ * PV_MAX_PORTS ports on a switch, peers out of range); PV_ENOMEM.
+ * Replaces any previously loaded tables.
+ * ------------------------------------------------------------------------- */
+int pv_load_flow_tables(pv_ctx *ctx, uint32_t num_switches, const uint32_t *rule_offs, const pv_rule *rules,
+                        const uint8_t *switch_region, const uint32_t *port_offs, const int32_t *port_peer,
+                        uint32_t num_hosts, const uint16_t *host_switch, const uint16_t *host_port,
+                        const uint32_t *host_ip);
+
+/* ---------------------------------------------------------------------------
+ * pv_verify_probes -- routing constraints Phi_N on the realised paths
+ * (Sec. 3.3 satisfaction (ii): "for all v on the path"; Sec. 5.5 network
+ * check; Sec. 6.3 item 4: transit switches are checked hop by hop).
+ *
+ * Each probe starts at (host_switch[src_host], host_port[src_host]); at each
+ * visited switch s: (1) region(s) not in allowed_mask -> PV_VIOLATION;
+ * (2) first matching rule by priority (no match or drop -> PV_DROPPED);
+ * (3) the output port's peer: unconnected -> PV_DROPPED, a host ->
+ * PV_COMPLIANT if it owns dst_ip else PV_MISDELIVERED, a switch port ->
+ * next hop.  Not terminated within hop_cap visits -> PV_LOOP.
+ *
+ * Device input d_probes[num_probes] (16-byte aligned); device output
+ * d_out[num_probes].
+ * Errors: PV_ESTATE (no tables), PV_EINVAL (hop_cap 0 or > 255, NULL
+ * pointers with num_probes > 0).  Out-of-range src_host gives PV_NOSRC.
+ * ------------------------------------------------------------------------- */
+int pv_verify_probes(pv_ctx *ctx, uint32_t num_probes, const pv_probe *d_probes, uint32_t hop_cap,
+                     pv_result *d_out, pv_stream stream);
+
+/* ---------------------------------------------------------------------------
+ * pv_compliant_reach -- jurisdiction-masked reachability over G = (V, E)
+ * (Sec. 3.3 forbidden-vertex policy; Sec. 4.2 graph search over the current
+ * topology).  R(s, m) = { v : some path s -> v has every vertex, s included,
+ * in a region permitted by m }; empty when region(s) is not permitted.
+ *
+ * Device inputs: d_offs[V + 1], d_cols[num_edges] (CSR of directed edges
+ * u -> v: the out-neighbours of u are d_cols[d_offs[u] .. d_offs[u+1])),
+ * d_region[V] (< 32), d_src[num_src] (vertex ids), d_masks[num_masks].
+ * Device output: d_reach[num_masks][num_src][words_per_row] bitsets over V.
+ * Malformed CSR entries (decreasing offsets, offsets > num_edges, cols >= V,
+ * region >= 32) are
+ * skipped and reported as PV_EINVAL by the next pv_sync(); out-of-range
+ * sources give empty rows.
+ * Errors: PV_EINVAL (V == 0, V > 16384, words_per_row too small or not a
+ * multiple of 4, NULL pointers); PV_ENOMEM (scratch).
+ * ------------------------------------------------------------------------- */
+int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_offs, uint32_t num_edges,
+                       const uint32_t *d_cols, const uint8_t *d_region, uint32_t num_src, const uint32_t *d_src, uint32_t num_masks,
+                       const uint32_t *d_masks, uint32_t *d_reach, uint32_t words_per_row, pv_stream stream);
+
+/* ---------------------------------------------------------------------------
+ * End-to-end composition (Sec. 4.2 hybrid coordination: pods are placed
+ * first, then flows from their attachments are checked; Sec. 5.5: an intent
+ * passes only if all of its checks pass).  A "group" is one intent: one
+ * selector row, pods_per_group pods, probes_per_group probes.  Cluster node
+ * n is network host n.
+ *
+ * pv_place_pods: pod j of group g gets the r-th feasible node of row g in
+ *   ascending order, r = d_draws[g * pods_per_group + j] mod |feasible|, or
+ *   PV_UNPLACED if the row is empty.  d_assign[num_groups * pods_per_group].
+ * pv_bind_probes: probe k of group g = k / probes_per_group is sent from
+ *   the host of pod (k mod probes_per_group) mod pods_per_group of g:
+ *   src_host and src_ip are rewritten in place (PV_NO_HOST / 0 when that pod
+ *   is unplaced or not a host).  Needs the flow tables (host_ip).
+ * pv_aggregate_intents: d_pass[g] = 1 iff every pod of g has d_assign in
+ *   row g, d_group_flags[g] has neither PV_F_UNKNOWN_VALUE nor
+ *   PV_F_BAD_EXPR, and every probe of g is PV_COMPLIANT.
+ *   d_counts[g][8]: [0..5] probe status histogram, [6] pods placed on a
+ *   feasible node, [7] zero.
+ * Errors: PV_ESTATE, PV_EINVAL (zero group sizes, NULL pointers).
+ * ------------------------------------------------------------------------- */
+int pv_place_pods(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_group, const uint32_t *d_bits,
+                  uint32_t words_per_row, const uint64_t *d_draws, uint32_t *d_assign, pv_stream stream);
+int pv_bind_probes(pv_ctx *ctx, uint32_t num_probes, pv_probe *d_probes, uint32_t probes_per_group,
+                   uint32_t pods_per_group, const uint32_t *d_assign, pv_stream stream);
+int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_group, const uint32_t *d_bits,
+                         uint32_t words_per_row, const uint8_t *d_group_flags, const uint32_t *d_assign,
+                         uint32_t probes_per_group, const pv_result *d_results, uint8_t *d_pass,
+                         uint32_t *d_counts, pv_stream stream);
+
+/* ---------------------------------------------------------------------------
+ * Tuning knobs (no counterpart in the paper).
+ * PV_OPT_SELECTOR_KERNEL: 0 = automatic, 1 = per-node label comparison over
+ *   shared-memory label tiles, 2 = per-(key, value) node-bitset rows
+ *   (needs the rows to have been built by pv_load_cluster).
+ * PV_OPT_WALK_KERNEL: 0 = automatic, 1 = hop-synchronous regroup + staged
+ *   tables (the only kernel at present).
+ * pv_get_stat: PV_STAT_SELECTOR_ROWS_BUILT (1 if value rows exist),
+ *   PV_STAT_SCRATCH_BYTES.
+ * ------------------------------------------------------------------------- */
+enum { PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2 };
+enum { PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2 };
+int pv_set_option(pv_ctx *ctx, int option, int64_t value);
+int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value);
+
+/* ---------------------------------------------------------------------------
+ * Kernel timing (no counterpart in the paper).  While enabled, every kernel
+ * group the library launches is bracketed by CUDA events recorded on the
+ * caller's stream.  pv_profile_enable(ctx, 1) clears the totals and starts
+ * recording, (ctx, 0) stops; pv_profile_collect synchronises `stream` and
+ * folds the recorded event pairs into per-group totals; pv_profile_read
+ * returns a group's total device milliseconds and number of kernel
+ * launches.  Groups: PV_K_* below (REGROUP = histogram + scan + scatter).
+ * ------------------------------------------------------------------------- */
+enum {
+    PV_K_SELECTOR = 0, PV_K_PLACE = 1, PV_K_BIND = 2, PV_K_WALK_INIT = 3, PV_K_WALK_REGROUP = 4,
+    PV_K_WALK_HOP = 5, PV_K_AGGREGATE = 6, PV_K_REACH = 7, PV_K_COUNT = 8
+};
+int pv_profile_enable(pv_ctx *ctx, int on);
+int pv_profile_collect(pv_ctx *ctx, pv_stream stream);
+int pv_profile_read(const pv_ctx *ctx, int group, double *total_ms, uint64_t *launches);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PV_H */

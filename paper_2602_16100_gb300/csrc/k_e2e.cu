@@ -1,0 +1,178 @@
+// End-to-end composition of the validator (Sec. 4.2 hybrid coordination:
+// pods are placed first, then flows from their attachments are compiled and
+// checked; Sec. 5.5: an intent passes only if all of its checks pass).
+#include <cuda_runtime.h>
+
+#include "pv_internal.cuh"
+
+namespace {
+
+constexpr int kThreads = 256;
+
+// Warp per group: count the feasible nodes (< N) of the group's row, then for
+// each pod select the r-th set bit, r = draw mod count.
+__global__ void __launch_bounds__(kThreads) place_pods_kernel(uint32_t G, uint32_t pods, uint32_t N,
+                                                              const uint32_t *__restrict__ bits, uint32_t W,
+                                                              const uint64_t *__restrict__ draws,
+                                                              uint32_t *__restrict__ assign) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t nwords = (N + 31) / 32, tail = N & 31;
+    for (uint32_t g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g < G; g += (gridDim.x * kThreads) >> 5) {
+        const uint32_t *row = bits + (size_t)g * W;
+        auto word = [&](uint32_t w) -> uint32_t {
+            uint32_t x = row[w];
+            if (w == nwords - 1 && tail) x &= (1u << tail) - 1u;
+            return x;
+        };
+        uint32_t c = 0;
+        for (uint32_t w = lane; w < nwords; w += 32) c += __popc(word(w));
+        for (int d = 16; d > 0; d >>= 1) c += __shfl_xor_sync(PV_FULL_MASK, c, d);
+        for (uint32_t j = 0; j < pods; ++j) {
+            const size_t pod = (size_t)g * pods + j;
+            if (c == 0) {
+                if (lane == 0) assign[pod] = PV_UNPLACED;
+                continue;
+            }
+            uint32_t r = (uint32_t)(draws[pod] % c);   // rank among feasible nodes
+            uint32_t result = PV_UNPLACED;
+            for (uint32_t w0 = 0; w0 < nwords; w0 += 32) {
+                const uint32_t w = w0 + lane;
+                const uint32_t x = w < nwords ? word(w) : 0u;
+                const uint32_t pc = __popc(x);
+                uint32_t incl = pc;
+                for (int d = 1; d < 32; d <<= 1) {
+                    uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
+                    if (lane >= (uint32_t)d) incl += y;
+                }
+                const uint32_t total = __shfl_sync(PV_FULL_MASK, incl, 31);
+                if (r < total) {
+                    const uint32_t excl = incl - pc;
+                    const bool here = r >= excl && r < incl;
+                    const uint32_t who = __ffs(__ballot_sync(PV_FULL_MASK, here)) - 1;
+                    if (lane == who) {
+                        uint32_t y = x;
+                        for (uint32_t k = r - excl; k > 0; --k) y &= y - 1u;
+                        result = w * 32 + (__ffs(y) - 1);
+                    }
+                    result = __shfl_sync(PV_FULL_MASK, result, who);
+                    break;
+                }
+                r -= total;
+            }
+            if (lane == 0) assign[pod] = result;
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads) bind_probes_kernel(uint32_t M, pv_probe *__restrict__ probes,
+                                                               uint32_t ppg, uint32_t pods,
+                                                               const uint32_t *__restrict__ assign, uint32_t H,
+                                                               const uint32_t *__restrict__ host_ip) {
+    for (uint32_t k = blockIdx.x * kThreads + threadIdx.x; k < M; k += gridDim.x * kThreads) {
+        const uint32_t g = k / ppg;
+        const uint32_t pod = g * pods + (k - g * ppg) % pods;
+        const uint32_t node = assign[pod];
+        if (node < H) {
+            probes[k].src_host = (uint16_t)node;
+            probes[k].src_ip = host_ip[node];
+        } else {
+            probes[k].src_host = PV_NO_HOST;
+            probes[k].src_ip = 0;
+        }
+    }
+}
+
+// Warp per group: placement check of each pod against the group's row, probe
+// status histogram, verdict.
+__global__ void __launch_bounds__(kThreads) aggregate_kernel(uint32_t G, uint32_t pods, uint32_t N,
+                                                             const uint32_t *__restrict__ bits, uint32_t W,
+                                                             const uint8_t *__restrict__ gflags,
+                                                             const uint32_t *__restrict__ assign, uint32_t ppg,
+                                                             const pv_result *__restrict__ results,
+                                                             uint8_t *__restrict__ pass, uint32_t *__restrict__ counts) {
+    const uint32_t lane = threadIdx.x & 31;
+    for (uint32_t g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g < G; g += (gridDim.x * kThreads) >> 5) {
+        uint32_t placed = 0;
+        for (uint32_t j = lane; j < pods; j += 32) {
+            const uint32_t a = assign[(size_t)g * pods + j];
+            placed += (a < N && ((bits[(size_t)g * W + (a >> 5)] >> (a & 31)) & 1u)) ? 1u : 0u;
+        }
+        uint32_t c[6] = {0, 0, 0, 0, 0, 0};
+        const uint32_t *res = reinterpret_cast<const uint32_t *>(results + (size_t)g * ppg);
+        for (uint32_t k = lane; k < ppg; k += 32) {
+            const uint32_t st = __ldg(res + k) & 0xFFu;
+#pragma unroll
+            for (int s = 0; s < 6; ++s) c[s] += st == (uint32_t)s;
+        }
+        for (int d = 16; d > 0; d >>= 1) {
+            placed += __shfl_xor_sync(PV_FULL_MASK, placed, d);
+#pragma unroll
+            for (int s = 0; s < 6; ++s) c[s] += __shfl_xor_sync(PV_FULL_MASK, c[s], d);
+        }
+        if (lane == 0) {
+            uint32_t *out = counts + (size_t)g * 8;
+#pragma unroll
+            for (int s = 0; s < 6; ++s) out[s] = c[s];
+            out[6] = placed;
+            out[7] = 0;
+            const bool ok = placed == pods && !(gflags[g] & (PV_F_UNKNOWN_VALUE | PV_F_BAD_EXPR)) && c[0] == ppg;
+            pass[g] = ok ? 1 : 0;
+        }
+    }
+}
+
+uint32_t grid_for(const pv_ctx *ctx, size_t items, uint32_t per_block) {
+    size_t b = (items + per_block - 1) / per_block;
+    size_t cap = (size_t)ctx->num_sms * 16;
+    if (b > cap) b = cap;
+    return (uint32_t)(b ? b : 1);
+}
+
+}  // namespace
+
+extern "C" int pv_place_pods(pv_ctx *ctx, uint32_t G, uint32_t pods, const uint32_t *d_bits, uint32_t W,
+                             const uint64_t *d_draws, uint32_t *d_assign, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->cl.loaded) return pv_fail(ctx, PV_ESTATE, "pv_place_pods: no cluster loaded");
+    if (G == 0) return PV_OK;
+    if (pods == 0) return pv_fail(ctx, PV_EINVAL, "pv_place_pods: pods_per_group must be > 0");
+    if (!d_bits || !d_draws || !d_assign) return pv_fail(ctx, PV_EINVAL, "pv_place_pods: NULL device pointer");
+    if (W < (ctx->cl.num_nodes + 31) / 32) return pv_fail(ctx, PV_EINVAL, "pv_place_pods: words_per_row too small");
+    const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_PLACE);
+    place_pods_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
+        G, pods, ctx->cl.num_nodes, d_bits, W, d_draws, d_assign);
+    pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    return pv_check_launch(ctx, "place_pods_kernel");
+}
+
+extern "C" int pv_bind_probes(pv_ctx *ctx, uint32_t M, pv_probe *d_probes, uint32_t ppg, uint32_t pods,
+                              const uint32_t *d_assign, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->tb.loaded) return pv_fail(ctx, PV_ESTATE, "pv_bind_probes: no flow tables loaded");
+    if (M == 0) return PV_OK;
+    if (ppg == 0 || pods == 0) return pv_fail(ctx, PV_EINVAL, "pv_bind_probes: group sizes must be > 0");
+    if (!d_probes || !d_assign) return pv_fail(ctx, PV_EINVAL, "pv_bind_probes: NULL device pointer");
+    const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_BIND);
+    bind_probes_kernel<<<grid_for(ctx, M, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
+        M, d_probes, ppg, pods, d_assign, ctx->tb.num_hosts, ctx->tb.d_host_ip);
+    pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    return pv_check_launch(ctx, "bind_probes_kernel");
+}
+
+extern "C" int pv_aggregate_intents(pv_ctx *ctx, uint32_t G, uint32_t pods, const uint32_t *d_bits, uint32_t W,
+                                    const uint8_t *d_gflags, const uint32_t *d_assign, uint32_t ppg,
+                                    const pv_result *d_results, uint8_t *d_pass, uint32_t *d_counts,
+                                    pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->cl.loaded) return pv_fail(ctx, PV_ESTATE, "pv_aggregate_intents: no cluster loaded");
+    if (G == 0) return PV_OK;
+    if (pods == 0) return pv_fail(ctx, PV_EINVAL, "pv_aggregate_intents: pods_per_group must be > 0");
+    if (!d_bits || !d_gflags || !d_assign || !d_pass || !d_counts || (ppg && !d_results))
+        return pv_fail(ctx, PV_EINVAL, "pv_aggregate_intents: NULL device pointer");
+    if (W < (ctx->cl.num_nodes + 31) / 32) return pv_fail(ctx, PV_EINVAL, "pv_aggregate_intents: words_per_row too small");
+    const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_AGGREGATE);
+    aggregate_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
+        G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts);
+    pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    return pv_check_launch(ctx, "aggregate_kernel");
+}

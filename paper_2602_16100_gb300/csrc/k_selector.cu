@@ -1,0 +1,464 @@
+// Placement constraints Phi_C: node-label loading and batched node-selector
+// evaluation (Sec. 3.3 satisfaction (i); Sec. 4.1 placement directives;
+// Sec. 5.5 compute check; Sec. 6.3 hallucinated identifiers; Sec. 5.3
+// fail-closed unenforceable intents).
+//
+// Two exact kernels compute the same feasible-node bitsets:
+//  * sel_cmp_kernel: label columns of a node tile are staged in shared
+//    memory; a warp per pod sweeps 32 nodes at a time, tests each
+//    expression against the node's value and emits one bitset word per
+//    sweep with __ballot_sync.
+//  * sel_rows_kernel: pv_load_cluster builds, for every (key, carried
+//    value), the bitset of nodes carrying it, plus one "key present" row
+//    per key.  An In expression is then the OR of its values' rows, NotIn
+//    its complement, Exists / DoesNotExist the present row or its
+//    complement, and a pod's row the AND over its expressions -- 32 nodes
+//    per word operation, rows read from L2 with 128-bit loads.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <vector>
+
+#include "pv_internal.cuh"
+
+namespace {
+
+constexpr uint32_t kInvWords = 2048;                  // 65536 value ids / 32
+constexpr uint64_t kRowBudgetBytes = 2ull << 30;      // value-row memory budget
+constexpr uint32_t kMaxKeys = 4096;
+
+__host__ __device__ inline uint32_t words_for(uint32_t n) { return ((n + 127) / 128) * 4; }
+
+// ---------------------------------------------------------------------------
+// loading
+// ---------------------------------------------------------------------------
+__global__ void build_inventory_kernel(uint32_t N, uint32_t K, const uint16_t *__restrict__ labels,
+                                       uint32_t *__restrict__ inv) {
+    size_t total = (size_t)N * K;
+    for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < total; i += (size_t)gridDim.x * blockDim.x) {
+        uint32_t k = (uint32_t)(i / N);
+        uint16_t v = labels[i];
+        if (v != PV_ABSENT) atomicOr(&inv[(size_t)k * kInvWords + (v >> 5)], 1u << (v & 31));
+    }
+}
+
+// One block (1024 threads) per key: exclusive prefix popcount over the key's
+// 2048 inventory words; count[k] = number of carried values.
+__global__ void __launch_bounds__(1024) inventory_rank_kernel(const uint32_t *__restrict__ inv,
+                                                              uint32_t *__restrict__ rank,
+                                                              uint32_t *__restrict__ count) {
+    __shared__ uint32_t s_warp[32];
+    const uint32_t k = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const uint32_t *w = inv + (size_t)k * kInvWords;
+    uint32_t a = __popc(w[2 * t]), b = __popc(w[2 * t + 1]);
+    uint32_t x = a + b, incl = x;
+    for (int d = 1; d < 32; d <<= 1) {
+        uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
+        if (lane >= (uint32_t)d) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        uint32_t v = s_warp[lane], vi = v;
+        for (int d = 1; d < 32; d <<= 1) {
+            uint32_t y = __shfl_up_sync(PV_FULL_MASK, vi, d);
+            if (lane >= (uint32_t)d) vi += y;
+        }
+        s_warp[lane] = vi - v;
+        if (lane == 31) count[k] = vi;
+    }
+    __syncthreads();
+    uint32_t excl = s_warp[warp] + incl - x;
+    rank[(size_t)k * kInvWords + 2 * t] = excl;
+    rank[(size_t)k * kInvWords + 2 * t + 1] = excl + a;
+}
+
+// Single block: key_base = exclusive scan of count[0..K), key_base[K] = total.
+__global__ void __launch_bounds__(1024) key_base_kernel(uint32_t K, const uint32_t *__restrict__ count,
+                                                        uint32_t *__restrict__ base) {
+    __shared__ uint32_t s_carry;
+    __shared__ uint32_t s_warp[32];
+    const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    if (t == 0) s_carry = 0;
+    __syncthreads();
+    for (uint32_t c0 = 0; c0 < K; c0 += 1024) {
+        uint32_t i = c0 + t;
+        uint32_t x = i < K ? count[i] : 0, incl = x;
+        for (int d = 1; d < 32; d <<= 1) {
+            uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
+            if (lane >= (uint32_t)d) incl += y;
+        }
+        if (lane == 31) s_warp[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            uint32_t v = s_warp[lane], vi = v;
+            for (int d = 1; d < 32; d <<= 1) {
+                uint32_t y = __shfl_up_sync(PV_FULL_MASK, vi, d);
+                if (lane >= (uint32_t)d) vi += y;
+            }
+            s_warp[lane] = vi - v;
+        }
+        __syncthreads();
+        uint32_t excl = s_carry + s_warp[warp] + incl - x;
+        if (i < K) base[i] = excl;
+        __syncthreads();
+        if (t == 1023) s_carry = excl + x;
+        __syncthreads();
+    }
+    if (t == 0) base[K] = s_carry;
+}
+
+__device__ __forceinline__ uint32_t value_row(const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
+                                              const uint32_t *__restrict__ key_base, uint32_t k, uint32_t v,
+                                              bool *carried) {
+    uint32_t w = inv[(size_t)k * kInvWords + (v >> 5)];
+    uint32_t bit = v & 31;
+    *carried = (w >> bit) & 1u;
+    return key_base[k] + rank[(size_t)k * kInvWords + (v >> 5)] + __popc(w & ((1u << bit) - 1u));
+}
+
+// Value rows and present rows.  One warp covers 32 consecutive nodes of one
+// key; present rows are written with a ballot, value rows with atomicOr.
+__global__ void build_rows_kernel(uint32_t N, uint32_t K, const uint16_t *__restrict__ labels,
+                                  const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
+                                  const uint32_t *__restrict__ key_base, uint32_t num_value_rows,
+                                  uint32_t row_words, uint32_t *__restrict__ rows) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t words = (N + 31) / 32;
+    const size_t total_warps = (size_t)K * words;
+    const size_t gw = (blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5;
+    const size_t nw = ((size_t)gridDim.x * blockDim.x) >> 5;
+    for (size_t i = gw; i < total_warps; i += nw) {
+        uint32_t k = (uint32_t)(i / words), wd = (uint32_t)(i % words);
+        uint32_t n = wd * 32 + lane;
+        uint16_t v = n < N ? labels[(size_t)k * N + n] : (uint16_t)PV_ABSENT;
+        uint32_t pres = __ballot_sync(PV_FULL_MASK, v != PV_ABSENT);
+        if (lane == 0) rows[((size_t)num_value_rows + k) * row_words + wd] = pres;
+        if (v != PV_ABSENT) {
+            bool carried;
+            uint32_t r = value_row(inv, rank, key_base, k, v, &carried);
+            atomicOr(&rows[(size_t)r * row_words + wd], 1u << lane);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// expression checks shared by both kernels
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ bool expr_valid(const pv_expr &x, uint32_t K) {
+    if (x.key >= K) return false;
+    if (x.op == PV_IN || x.op == PV_NOTIN) {
+        if (x.nvals < 1 || x.nvals > 8) return false;
+        for (int j = 0; j < 8; ++j)
+            if (j < x.nvals && x.vals[j] == PV_ABSENT) return false;
+        return true;
+    }
+    if (x.op == PV_EXISTS || x.op == PV_DOESNOTEXIST) return x.nvals == 0;
+    return false;
+}
+
+// Lane-parallel validation and hallucinated-value scan of pod p's list.
+// Returns bit0 = bad, bit1 = unknown value.
+__device__ __forceinline__ uint32_t pod_prescan(uint32_t lo, uint32_t hi, uint32_t num_exprs,
+                                                const pv_expr *__restrict__ exprs, uint32_t K,
+                                                const uint32_t *__restrict__ inv, uint32_t lane) {
+    bool bad = hi < lo || hi > num_exprs;
+    bool unknown = false;
+    if (!bad) {
+        for (uint32_t e = lo + lane; e < hi; e += 32) {
+            pv_expr x = exprs[e];
+            if (!expr_valid(x, K)) {
+                bad = true;
+                continue;
+            }
+            if (x.op == PV_IN)
+                for (int j = 0; j < 8; ++j)
+                    if (j < x.nvals) {
+                        uint32_t v = x.vals[j];
+                        if (!((inv[(size_t)x.key * kInvWords + (v >> 5)] >> (v & 31)) & 1u)) unknown = true;
+                    }
+        }
+    }
+    bad = __any_sync(PV_FULL_MASK, bad);
+    unknown = __any_sync(PV_FULL_MASK, unknown);
+    return (bad ? 1u : 0u) | (unknown ? 2u : 0u);
+}
+
+__device__ __forceinline__ uint8_t pod_flags(bool nonempty, bool unknown, bool has_assign, bool assign_ok) {
+    uint8_t f = 0;
+    if (!nonempty) f |= PV_F_EMPTY;
+    if (unknown) f |= PV_F_UNKNOWN_VALUE;
+    if (has_assign && assign_ok) {
+        f |= PV_F_ASSIGN_OK;
+        if (!unknown) f |= PV_F_PASS;
+    }
+    return f;
+}
+
+// ---------------------------------------------------------------------------
+// kernel 1: per-node comparison over shared-memory label tiles
+// ---------------------------------------------------------------------------
+constexpr int kCmpThreads = 512;
+constexpr int kCmpWarps = kCmpThreads / 32;
+constexpr int kCmpPods = 128;   // pods per block
+constexpr int kCmpCache = 8;    // expressions cached per warp
+
+__global__ void __launch_bounds__(kCmpThreads) sel_cmp_kernel(
+    uint32_t N, uint32_t K, const uint16_t *__restrict__ labels, uint32_t tile, uint32_t P,
+    const uint32_t *__restrict__ offs, uint32_t num_exprs, const pv_expr *__restrict__ exprs,
+    const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits, uint32_t W, uint8_t *__restrict__ flags,
+    const uint32_t *__restrict__ inv) {
+    extern __shared__ uint16_t s_lab[];   // [K][tile]
+    __shared__ uint8_t s_state[kCmpPods]; // bit0 nonempty, bit1 assign ok, bit2 bad, bit3 unknown
+    __shared__ pv_expr s_ex[kCmpWarps][kCmpCache];
+    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint32_t p0 = blockIdx.x * kCmpPods;
+    if (p0 >= P) return;
+    const uint32_t np = min((uint32_t)kCmpPods, P - p0);
+    const uint32_t nvalid_words = (N + 31) / 32;
+
+    // per-pod validation / unknown scan (warp per pod)
+    for (uint32_t pl = warp; pl < np; pl += kCmpWarps) {
+        uint32_t p = p0 + pl;
+        uint32_t r = pod_prescan(offs[p], offs[p + 1], num_exprs, exprs, K, inv, lane);
+        if (lane == 0) s_state[pl] = (uint8_t)(((r & 1u) ? 4u : 0u) | ((r & 2u) ? 8u : 0u));
+    }
+
+    for (uint32_t n0 = 0; n0 < N; n0 += tile) {
+        const uint32_t tn = min(tile, N - n0);
+        __syncthreads();
+        for (uint32_t i = threadIdx.x; i < K * tile; i += kCmpThreads) {
+            uint32_t k = i / tile, j = i - k * tile;
+            s_lab[i] = j < tn ? labels[(size_t)k * N + n0 + j] : (uint16_t)PV_ABSENT;
+        }
+        __syncthreads();
+        const uint32_t groups = (tn + 31) / 32;
+        for (uint32_t pl = warp; pl < np; pl += kCmpWarps) {
+            const uint32_t p = p0 + pl;
+            const uint8_t st = s_state[pl];
+            uint32_t *row = bits + (size_t)p * W + (n0 >> 5);
+            if (st & 4u) {
+                for (uint32_t g = lane; g < groups; g += 32) row[g] = 0;
+                continue;
+            }
+            const uint32_t lo = offs[p], E = offs[p + 1] - lo;
+            const bool cached = E <= (uint32_t)kCmpCache;
+            if (cached) {
+                if (lane < E) s_ex[warp][lane] = exprs[lo + lane];
+                __syncwarp();
+            }
+            const uint32_t a = assign ? assign[p] : PV_UNPLACED;
+            bool any = false, aok = false;
+            for (uint32_t gb = 0; gb < groups; gb += 32) {
+                uint32_t mine = 0;
+                const uint32_t gend = min(groups, gb + 32);
+                for (uint32_t g = gb; g < gend; ++g) {
+                    const uint32_t j = g * 32 + lane;   // node offset within the tile
+                    bool ok = j < tn;
+                    for (uint32_t e = 0; e < E; ++e) {
+                        const pv_expr &x = cached ? s_ex[warp][e] : exprs[lo + e];
+                        const uint16_t v = s_lab[(uint32_t)x.key * tile + j];
+                        const bool present = v != PV_ABSENT;
+                        bool inset = false;
+                        const uint32_t nv = x.nvals;
+                        for (uint32_t q = 0; q < nv; ++q) inset |= (v == x.vals[q]);
+                        bool m;
+                        switch (x.op) {
+                        case PV_IN: m = present && inset; break;
+                        case PV_NOTIN: m = !present || !inset; break;
+                        case PV_EXISTS: m = present; break;
+                        default: m = !present; break;
+                        }
+                        ok = ok && m;
+                    }
+                    const uint32_t w = __ballot_sync(PV_FULL_MASK, ok);
+                    if (lane == g - gb) mine = w;
+                    const uint32_t node_base = n0 + g * 32;
+                    if (a >= node_base && a < node_base + 32) aok = (w >> (a - node_base)) & 1u;
+                }
+                if (lane < gend - gb) row[gb + lane] = mine;
+                any = any || __any_sync(PV_FULL_MASK, mine != 0);
+            }
+            __syncwarp();
+            if (lane == 0) s_state[pl] = st | (any ? 1u : 0u) | (aok ? 2u : 0u);
+        }
+    }
+    __syncthreads();
+    // padding words and flags
+    for (uint32_t pl = warp; pl < np; pl += kCmpWarps) {
+        const uint32_t p = p0 + pl;
+        for (uint32_t w = nvalid_words + lane; w < W; w += 32) bits[(size_t)p * W + w] = 0;
+        if (lane == 0) {
+            const uint8_t st = s_state[pl];
+            flags[p] = (st & 4u) ? (uint8_t)PV_F_BAD_EXPR
+                                 : pod_flags(st & 1u, st & 8u, assign != nullptr, st & 2u);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// kernel 2: per-(key, value) node-bitset rows
+// ---------------------------------------------------------------------------
+constexpr int kRowsThreads = 256;
+
+__global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
+    uint32_t N, uint32_t K, uint32_t P, const uint32_t *__restrict__ offs, uint32_t num_exprs,
+    const pv_expr *__restrict__ exprs, const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits,
+    uint32_t W, uint8_t *__restrict__ flags, const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
+    const uint32_t *__restrict__ key_base, const uint32_t *__restrict__ rows, uint32_t row_words,
+    uint32_t num_value_rows) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t gw = (blockIdx.x * kRowsThreads + threadIdx.x) >> 5;
+    const uint32_t nw = (gridDim.x * kRowsThreads) >> 5;
+    const uint32_t full_words = N >> 5, tail_bits = N & 31;
+    for (uint32_t p = gw; p < P; p += nw) {
+        const uint32_t lo = offs[p], hi = offs[p + 1];
+        const uint32_t pre = pod_prescan(lo, hi, num_exprs, exprs, K, inv, lane);
+        uint4 *out = reinterpret_cast<uint4 *>(bits + (size_t)p * W);
+        if (pre & 1u) {
+            for (uint32_t q = lane; q < W / 4; q += 32) out[q] = make_uint4(0, 0, 0, 0);
+            if (lane == 0) flags[p] = PV_F_BAD_EXPR;
+            continue;
+        }
+        const uint32_t a = assign ? assign[p] : PV_UNPLACED;
+        bool any = false, aok = false;
+        for (uint32_t q = lane; q < W / 4; q += 32) {
+            const uint32_t w0 = q * 4;
+            uint4 acc = make_uint4(~0u, ~0u, ~0u, ~0u);
+            const bool in_rows = w0 < row_words;
+            for (uint32_t e = lo; e < hi; ++e) {
+                const pv_expr &x = exprs[e];
+                const uint32_t k = x.key, op = x.op;
+                uint4 r;
+                if (op == PV_IN || op == PV_NOTIN) {
+                    r = make_uint4(0, 0, 0, 0);
+                    const uint32_t nv = x.nvals;
+                    for (uint32_t j = 0; j < nv; ++j) {
+                        bool carried;
+                        const uint32_t row = value_row(inv, rank, key_base, k, x.vals[j], &carried);
+                        if (carried && in_rows) {
+                            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(rows + (size_t)row * row_words + w0));
+                            r.x |= v.x; r.y |= v.y; r.z |= v.z; r.w |= v.w;
+                        }
+                    }
+                } else {
+                    r = in_rows ? __ldg(reinterpret_cast<const uint4 *>(rows + ((size_t)num_value_rows + k) * row_words + w0))
+                                : make_uint4(0, 0, 0, 0);
+                }
+                if (op == PV_NOTIN || op == PV_DOESNOTEXIST) { r.x = ~r.x; r.y = ~r.y; r.z = ~r.z; r.w = ~r.w; }
+                acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
+            }
+            // clear bits of nodes >= N
+            uint32_t *aw = &acc.x;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t w = w0 + i;
+                if (w > full_words || (w == full_words && tail_bits == 0)) aw[i] = 0;
+                else if (w == full_words) aw[i] &= (1u << tail_bits) - 1u;
+            }
+            out[q] = acc;
+            any = any || (acc.x | acc.y | acc.z | acc.w) != 0;
+            if (a < N && (a >> 5) >= w0 && (a >> 5) < w0 + 4) aok = (aw[(a >> 5) - w0] >> (a & 31)) & 1u;
+        }
+        any = __any_sync(PV_FULL_MASK, any);
+        aok = __any_sync(PV_FULL_MASK, aok);
+        if (lane == 0) flags[p] = pod_flags(any, pre & 2u, assign != nullptr, aok);
+    }
+}
+
+}  // namespace
+
+// -----------------------------------------------------------------------------
+// C ABI
+// -----------------------------------------------------------------------------
+extern "C" int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_keys, const uint16_t *labels) {
+    if (!ctx) return PV_EINVAL;
+    if (num_nodes == 0 || num_keys == 0 || !labels)
+        return pv_fail(ctx, PV_EINVAL, "pv_load_cluster: empty cluster or NULL labels");
+    if (num_keys > kMaxKeys) return pv_fail(ctx, PV_EINVAL, "pv_load_cluster: num_keys > %u", kMaxKeys);
+    PV_TRY_CUDA(ctx, cudaSetDevice(ctx->device), "cudaSetDevice");
+    PV_TRY_CUDA(ctx, cudaDeviceSynchronize(), "pv_load_cluster sync");
+    pv_free_cluster(ctx->cl);
+    pv_cluster_state &c = ctx->cl;
+    const size_t nl = (size_t)num_nodes * num_keys;
+    int rc;
+    if ((rc = pv_device_alloc(ctx, (void **)&c.d_labels, nl * 2, "labels")) ||
+        (rc = pv_device_alloc(ctx, (void **)&c.d_inv, (size_t)num_keys * kInvWords * 4, "inventory")) ||
+        (rc = pv_device_alloc(ctx, (void **)&c.d_inv_rank, (size_t)num_keys * kInvWords * 4, "inventory rank")) ||
+        (rc = pv_device_alloc(ctx, (void **)&c.d_key_base, ((size_t)num_keys + 1) * 4 * 2, "key base"))) {
+        pv_free_cluster(c);
+        return rc;
+    }
+    uint32_t *d_count = c.d_key_base + (num_keys + 1);
+    PV_TRY_CUDA(ctx, cudaMemcpy(c.d_labels, labels, nl * 2, cudaMemcpyHostToDevice), "labels upload");
+    PV_TRY_CUDA(ctx, cudaMemset(c.d_inv, 0, (size_t)num_keys * kInvWords * 4), "inventory clear");
+    build_inventory_kernel<<<ctx->num_sms * 8, 256>>>(num_nodes, num_keys, c.d_labels, c.d_inv);
+    inventory_rank_kernel<<<num_keys, 1024>>>(c.d_inv, c.d_inv_rank, d_count);
+    key_base_kernel<<<1, 1024>>>(num_keys, d_count, c.d_key_base);
+    if ((rc = pv_check_launch(ctx, "inventory kernels"))) { pv_free_cluster(c); return rc; }
+    uint32_t nvr = 0;
+    PV_TRY_CUDA(ctx, cudaMemcpy(&nvr, c.d_key_base + num_keys, 4, cudaMemcpyDeviceToHost), "value count");
+    c.num_nodes = num_nodes;
+    c.num_keys = num_keys;
+    c.row_words = words_for(num_nodes);
+    c.num_value_rows = nvr;
+    const uint64_t row_bytes = ((uint64_t)nvr + num_keys) * c.row_words * 4;
+    if (row_bytes <= kRowBudgetBytes) {
+        if (pv_device_alloc(ctx, (void **)&c.d_rows, row_bytes, "value rows") == PV_OK) {
+            PV_TRY_CUDA(ctx, cudaMemset(c.d_rows, 0, row_bytes), "value rows clear");
+            build_rows_kernel<<<ctx->num_sms * 8, 256>>>(num_nodes, num_keys, c.d_labels, c.d_inv, c.d_inv_rank,
+                                                          c.d_key_base, nvr, c.row_words, c.d_rows);
+            if ((rc = pv_check_launch(ctx, "value rows"))) { pv_free_cluster(c); return rc; }
+            c.rows_built = true;
+        } else {
+            ctx->err.clear();   // rows are optional; fall back to the comparison kernel
+        }
+    }
+    PV_TRY_CUDA(ctx, cudaDeviceSynchronize(), "pv_load_cluster");
+    c.loaded = true;
+    return PV_OK;
+}
+
+extern "C" int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_expr_offs, uint32_t num_exprs,
+                                 const pv_expr *d_exprs, const uint32_t *d_assign, uint32_t *d_bits,
+                                 uint32_t words_per_row, uint8_t *d_flags, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    const pv_cluster_state &c = ctx->cl;
+    if (!c.loaded) return pv_fail(ctx, PV_ESTATE, "pv_eval_selectors: no cluster loaded");
+    if (num_pods == 0) return PV_OK;
+    if (!d_expr_offs || !d_bits || !d_flags || (num_exprs > 0 && !d_exprs))
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: NULL device pointer");
+    if (words_per_row % 4 != 0 || words_per_row < (c.num_nodes + 31) / 32)
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: words_per_row must be >= ceil(N/32) and a multiple of 4");
+    if (((uintptr_t)d_bits & 15) != 0) return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: d_bits must be 16-byte aligned");
+    int which = ctx->opt_selector;
+    if (which == 0) which = c.rows_built ? 2 : 1;
+    if (which == 2 && !c.rows_built)
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: value rows were not built for this cluster");
+    cudaStream_t st = (cudaStream_t)stream;
+    if (which == 2) {
+        uint32_t blocks = std::min<uint32_t>((num_pods + 7) / 8, (uint32_t)ctx->num_sms * 16);
+        const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
+        sel_rows_kernel<<<blocks, kRowsThreads, 0, st>>>(c.num_nodes, c.num_keys, num_pods, d_expr_offs, num_exprs,
+                                                         d_exprs, d_assign, d_bits, words_per_row, d_flags, c.d_inv,
+                                                         c.d_inv_rank, c.d_key_base, c.d_rows, c.row_words,
+                                                         c.num_value_rows);
+        pv_prof_stop(ctx, st, pr, 1);
+        return pv_check_launch(ctx, "sel_rows_kernel");
+    }
+    // tile: as many nodes (multiple of 32) as fit 96 KB of label columns
+    const size_t budget = 96 * 1024;
+    uint32_t tile = (uint32_t)(budget / (2ull * c.num_keys)) / 32 * 32;
+    if (tile < 32) return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: too many keys for the comparison kernel");
+    tile = min(tile, ((c.num_nodes + 31) / 32) * 32);
+    const size_t smem = (size_t)tile * c.num_keys * 2;
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(sel_cmp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                "sel_cmp_kernel smem");
+    const uint32_t blocks = (num_pods + kCmpPods - 1) / kCmpPods;
+    const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
+    sel_cmp_kernel<<<blocks, kCmpThreads, smem, st>>>(c.num_nodes, c.num_keys, c.d_labels, tile, num_pods,
+                                                      d_expr_offs, num_exprs, d_exprs, d_assign, d_bits,
+                                                      words_per_row, d_flags, c.d_inv);
+    pv_prof_stop(ctx, st, pr, 1);
+    return pv_check_launch(ctx, "sel_cmp_kernel");
+}

@@ -1,0 +1,236 @@
+// Context management, error reporting and the scratch arena of libpv.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <new>
+
+#include "pv_internal.cuh"
+
+#define PV_VERSION 100
+
+int pv_fail(pv_ctx *ctx, int code, const char *fmt, ...) {
+    if (ctx) {
+        char buf[512];
+        va_list ap;
+        va_start(ap, fmt);
+        vsnprintf(buf, sizeof buf, fmt, ap);
+        va_end(ap);
+        ctx->err = buf;
+    }
+    return code;
+}
+
+int pv_cuda_fail(pv_ctx *ctx, cudaError_t e, const char *what) {
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();
+        return pv_fail(ctx, PV_ENOMEM, "%s: out of device memory", what);
+    }
+    return pv_fail(ctx, PV_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int pv_device_alloc(pv_ctx *ctx, void **p, size_t bytes, const char *what) {
+    *p = nullptr;
+    if (bytes == 0) bytes = 16;
+    cudaError_t e = cudaMalloc(p, bytes);
+    if (e != cudaSuccess) {
+        *p = nullptr;
+        return pv_cuda_fail(ctx, e, what);
+    }
+    return PV_OK;
+}
+
+void pv_device_free(void *p) {
+    if (p) cudaFree(p);
+}
+
+int pv_check_launch(pv_ctx *ctx, const char *what) {
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return pv_cuda_fail(ctx, e, what);
+    return PV_OK;
+}
+
+void *pv_scratch(pv_ctx *ctx, size_t bytes) {
+    if (bytes <= ctx->scratch_bytes && ctx->scratch) return ctx->scratch;
+    size_t want = bytes + bytes / 4 + (1u << 20);
+    if (ctx->scratch) {
+        cudaDeviceSynchronize();
+        cudaFree(ctx->scratch);
+        ctx->scratch = nullptr;
+        ctx->scratch_bytes = 0;
+    }
+    void *p = nullptr;
+    if (pv_device_alloc(ctx, &p, want, "scratch arena") != PV_OK) return nullptr;
+    ctx->scratch = p;
+    ctx->scratch_bytes = want;
+    return p;
+}
+
+void pv_free_cluster(pv_cluster_state &c) {
+    pv_free_ptr(c.d_labels);
+    pv_free_ptr(c.d_inv);
+    pv_free_ptr(c.d_inv_rank);
+    pv_free_ptr(c.d_key_base);
+    pv_free_ptr(c.d_rows);
+    c = pv_cluster_state();
+}
+
+void pv_free_tables(pv_table_state &t) {
+    pv_free_ptr(t.d_tab_offs);
+    pv_free_ptr(t.d_rule_a);
+    pv_free_ptr(t.d_rule_b);
+    pv_free_ptr(t.d_region);
+    pv_free_ptr(t.d_port_offs);
+    pv_free_ptr(t.d_port_peer);
+    pv_free_ptr(t.d_host_switch);
+    pv_free_ptr(t.d_host_port);
+    pv_free_ptr(t.d_host_ip);
+    t = pv_table_state();
+}
+
+int pv_prof_start(pv_ctx *ctx, cudaStream_t st, int group) {
+    pv_prof_state &p = ctx->prof;
+    if (!p.on) return -1;
+    if (p.used * 2 + 2 > p.pool.size()) {
+        for (int i = 0; i < 2; ++i) {
+            cudaEvent_t e;
+            if (cudaEventCreate(&e) != cudaSuccess) return -1;
+            p.pool.push_back(e);
+        }
+        p.group.push_back(0);
+        p.nlaunch.push_back(0);
+    }
+    const size_t i = p.used++;
+    p.group[i] = group;
+    p.nlaunch[i] = 0;
+    cudaEventRecord(p.pool[2 * i], st);
+    return (int)i;
+}
+
+void pv_prof_stop(pv_ctx *ctx, cudaStream_t st, int pair, uint32_t launches) {
+    if (pair < 0) return;
+    pv_prof_state &p = ctx->prof;
+    p.nlaunch[pair] = launches;
+    cudaEventRecord(p.pool[2 * (size_t)pair + 1], st);
+}
+
+extern "C" int pv_profile_enable(pv_ctx *ctx, int on) {
+    if (!ctx) return PV_EINVAL;
+    pv_prof_state &p = ctx->prof;
+    if (on) {
+        for (int g = 0; g < PV_K_COUNT; ++g) {
+            p.ms[g] = 0;
+            p.launches[g] = 0;
+        }
+        p.used = 0;
+    }
+    p.on = on != 0;
+    return PV_OK;
+}
+
+extern "C" int pv_profile_collect(pv_ctx *ctx, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    pv_prof_state &p = ctx->prof;
+    PV_TRY_CUDA(ctx, cudaStreamSynchronize((cudaStream_t)stream), "pv_profile_collect");
+    for (size_t i = 0; i < p.used; ++i) {
+        float ms = 0;
+        PV_TRY_CUDA(ctx, cudaEventElapsedTime(&ms, p.pool[2 * i], p.pool[2 * i + 1]), "event elapsed");
+        p.ms[p.group[i]] += ms;
+        p.launches[p.group[i]] += p.nlaunch[i];
+    }
+    p.used = 0;
+    return PV_OK;
+}
+
+extern "C" int pv_profile_read(const pv_ctx *ctx, int group, double *total_ms, uint64_t *launches) {
+    if (!ctx || group < 0 || group >= PV_K_COUNT) return PV_EINVAL;
+    if (total_ms) *total_ms = ctx->prof.ms[group];
+    if (launches) *launches = ctx->prof.launches[group];
+    return PV_OK;
+}
+
+extern "C" int pv_version(void) { return PV_VERSION; }
+
+extern "C" int pv_create(pv_ctx **out, int cuda_device) {
+    if (!out) return PV_EINVAL;
+    *out = nullptr;
+    pv_ctx *ctx = new (std::nothrow) pv_ctx();
+    if (!ctx) return PV_ENOMEM;
+    int ndev = 0;
+    cudaError_t e = cudaGetDeviceCount(&ndev);
+    if (e != cudaSuccess || cuda_device < 0 || cuda_device >= ndev) {
+        delete ctx;
+        return PV_ECUDA;
+    }
+    e = cudaSetDevice(cuda_device);
+    if (e != cudaSuccess) {
+        delete ctx;
+        return PV_ECUDA;
+    }
+    ctx->device = cuda_device;
+    cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, cuda_device);
+    int smem = 0;
+    cudaDeviceGetAttribute(&smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, cuda_device);
+    ctx->max_smem_optin = (size_t)smem;
+    if (pv_device_alloc(ctx, (void **)&ctx->d_status, sizeof(int32_t), "status word") != PV_OK ||
+        cudaMemset(ctx->d_status, 0, sizeof(int32_t)) != cudaSuccess) {
+        pv_device_free(ctx->d_status);
+        delete ctx;
+        return PV_ENOMEM;
+    }
+    *out = ctx;
+    return PV_OK;
+}
+
+extern "C" void pv_destroy(pv_ctx *ctx) {
+    if (!ctx) return;
+    cudaDeviceSynchronize();
+    pv_free_cluster(ctx->cl);
+    pv_free_tables(ctx->tb);
+    for (cudaEvent_t e : ctx->prof.pool) cudaEventDestroy(e);
+    pv_device_free(ctx->scratch);
+    pv_device_free(ctx->d_status);
+    delete ctx;
+}
+
+extern "C" const char *pv_last_error(const pv_ctx *ctx) {
+    if (!ctx) return "null context";
+    return ctx->err.c_str();
+}
+
+extern "C" int pv_sync(pv_ctx *ctx, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    PV_TRY_CUDA(ctx, cudaStreamSynchronize((cudaStream_t)stream), "pv_sync");
+    int32_t st = 0;
+    PV_TRY_CUDA(ctx, cudaMemcpy(&st, ctx->d_status, sizeof st, cudaMemcpyDeviceToHost), "pv_sync status");
+    if (st != 0) {
+        PV_TRY_CUDA(ctx, cudaMemset(ctx->d_status, 0, sizeof(int32_t)), "pv_sync reset");
+        if (st == PV_ETIMEOUT) return pv_fail(ctx, PV_ETIMEOUT, "a bounded device-side wait gave up");
+        return pv_fail(ctx, st, "device-detected error %d (malformed device-resident input)", (int)st);
+    }
+    return PV_OK;
+}
+
+extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
+    if (!ctx) return PV_EINVAL;
+    switch (option) {
+    case PV_OPT_SELECTOR_KERNEL:
+        if (value < 0 || value > 2) return pv_fail(ctx, PV_EINVAL, "selector kernel must be 0, 1 or 2");
+        ctx->opt_selector = (int)value;
+        return PV_OK;
+    case PV_OPT_WALK_KERNEL:
+        if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "walk kernel must be 0 or 1");
+        ctx->opt_walk = (int)value;
+        return PV_OK;
+    default:
+        return pv_fail(ctx, PV_EINVAL, "unknown option %d", option);
+    }
+}
+
+extern "C" int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value) {
+    if (!ctx || !value) return PV_EINVAL;
+    switch (stat) {
+    case PV_STAT_SELECTOR_ROWS_BUILT: *value = ctx->cl.rows_built ? 1 : 0; return PV_OK;
+    case PV_STAT_SCRATCH_BYTES: *value = (int64_t)ctx->scratch_bytes; return PV_OK;
+    default: return PV_EINVAL;
+    }
+}

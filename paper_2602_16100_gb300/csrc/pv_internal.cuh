@@ -1,0 +1,115 @@
+// Internal declarations of libpv (not part of the C ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "pv.h"
+
+#define PV_FULL_MASK 0xFFFFFFFFu
+
+// -----------------------------------------------------------------------------
+// context
+// -----------------------------------------------------------------------------
+struct pv_cluster_state {
+    bool loaded = false;
+    uint32_t num_nodes = 0, num_keys = 0;
+    uint16_t *d_labels = nullptr;     // [K][N]
+    uint32_t *d_inv = nullptr;        // [K][2048]: bit v = some node carries value v of key k
+    uint32_t *d_inv_rank = nullptr;   // [K][2048]: set bits of the key's inventory before word w
+    uint32_t *d_key_base = nullptr;   // [K + 1]: first value row of key k; [K] = number of value rows
+    // per-(key, value) node bitsets, then one "present" row per key
+    bool rows_built = false;
+    uint32_t row_words = 0;           // words per value row (multiple of 4)
+    uint32_t num_value_rows = 0;
+    uint32_t *d_rows = nullptr;       // [num_value_rows + K][row_words]
+};
+
+struct pv_table_state {
+    bool loaded = false;
+    uint32_t num_switches = 0, num_hosts = 0;
+    uint32_t max_rules_padded = 0;    // largest per-switch table, in rules (multiple of 32)
+    uint32_t *d_tab_offs = nullptr;   // [S + 1] start of each switch's compiled table (multiple of 32)
+    uint4 *d_rule_a = nullptr;        // [total padded] {src & m, m_src, dst & m, m_dst}
+    uint2 *d_rule_b = nullptr;        // [total padded] {lo | hi << 16, inval | inmask << 8 | action << 16}
+    uint8_t *d_region = nullptr;      // [S]
+    uint32_t *d_port_offs = nullptr;  // [S + 1]
+    int32_t *d_port_peer = nullptr;   // [ports]
+    uint16_t *d_host_switch = nullptr, *d_host_port = nullptr;
+    uint32_t *d_host_ip = nullptr;
+};
+
+struct pv_prof_state {
+    bool on = false;
+    std::vector<cudaEvent_t> pool;     // event pairs: [2i] start, [2i+1] stop
+    std::vector<int> group;            // group of pair i
+    std::vector<uint32_t> nlaunch;     // kernel launches inside pair i
+    size_t used = 0;                   // pairs recorded since the last collect
+    double ms[PV_K_COUNT] = {};
+    uint64_t launches[PV_K_COUNT] = {};
+};
+
+struct pv_ctx {
+    int device = 0;
+    pv_prof_state prof;
+    int num_sms = 0;
+    size_t max_smem_optin = 0;
+    std::string err;
+    int32_t *d_status = nullptr;      // first device-detected error (0 = none)
+    int opt_selector = 0, opt_walk = 0;
+    void *scratch = nullptr;
+    size_t scratch_bytes = 0;
+    pv_cluster_state cl;
+    pv_table_state tb;
+};
+
+// -----------------------------------------------------------------------------
+// host helpers (pv_api.cu)
+// -----------------------------------------------------------------------------
+int pv_fail(pv_ctx *ctx, int code, const char *fmt, ...);
+int pv_cuda_fail(pv_ctx *ctx, cudaError_t e, const char *what);
+// Returns a device pointer to at least `bytes` of context scratch (grows the
+// arena; growing synchronises the device).  nullptr on failure (error set).
+void *pv_scratch(pv_ctx *ctx, size_t bytes);
+int pv_device_alloc(pv_ctx *ctx, void **p, size_t bytes, const char *what);
+void pv_device_free(void *p);
+int pv_check_launch(pv_ctx *ctx, const char *what);
+// Kernel-group timing: no-ops unless profiling is enabled.  Returns the pair
+// index to pass to pv_prof_stop (or -1).
+int pv_prof_start(pv_ctx *ctx, cudaStream_t st, int group);
+void pv_prof_stop(pv_ctx *ctx, cudaStream_t st, int pair, uint32_t launches);
+
+#define PV_TRY_CUDA(ctx, call, what)                          \
+    do {                                                      \
+        cudaError_t _e = (call);                              \
+        if (_e != cudaSuccess) return pv_cuda_fail(ctx, _e, what); \
+    } while (0)
+
+// -----------------------------------------------------------------------------
+// device helpers
+// -----------------------------------------------------------------------------
+// Records the first device-detected error code in the context status word.
+__device__ __forceinline__ void pv_device_error(int32_t *status, int32_t code) {
+    atomicCAS(status, 0, code);
+}
+
+__host__ __device__ __forceinline__ uint32_t pv_div_up(uint32_t a, uint32_t b) { return (a + b - 1) / b; }
+
+// Prefix mask with the top `len` bits set; len in 0..32 (len 0 -> 0, never a
+// shift by 32).
+__host__ __device__ __forceinline__ uint32_t pv_prefix_mask(uint32_t len) {
+    return len == 0 ? 0u : (0xFFFFFFFFu << (32u - len));
+}
+
+// Allocation free-list helpers shared by the loaders.
+template <typename T>
+inline void pv_free_ptr(T *&p) {
+    if (p) pv_device_free((void *)p);
+    p = nullptr;
+}
+
+void pv_free_cluster(pv_cluster_state &c);
+void pv_free_tables(pv_table_state &t);

@@ -1,0 +1,140 @@
+"""User-facing wrapper over the C ABI: owns a pv_ctx, moves numpy arrays to
+device byte tensors and back, and chains the end-to-end pipeline.
+
+Every computation runs in libpv's CUDA kernels; this module only allocates
+torch device buffers, copies, and calls the binding.
+"""
+from __future__ import annotations
+
+from typing import Optional
+
+import numpy as np
+import torch
+
+from . import binding as B
+from . import workloads as W
+
+
+def to_device(a: np.ndarray, device) -> torch.Tensor:
+    """Byte tensor on `device` holding the bytes of the numpy array."""
+    a = np.ascontiguousarray(a)
+    return torch.from_numpy(a.view(np.uint8).reshape(-1).copy()).to(device)
+
+
+def empty_device(nbytes: int, device) -> torch.Tensor:
+    return torch.empty(max(16, int(nbytes)), dtype=torch.uint8, device=device)
+
+
+def to_numpy(t: torch.Tensor, dtype, shape=None) -> np.ndarray:
+    a = t.detach().cpu().numpy().view(dtype)
+    return a.reshape(shape) if shape is not None else a
+
+
+class Validator:
+    """One GPU validator context (not thread-safe)."""
+
+    def __init__(self, device: int = 0):
+        self.device = torch.device("cuda", device)
+        torch.cuda.set_device(self.device)
+        self.ctx = B.pv_create(device)
+        self.num_nodes = 0
+        self.num_hosts = 0
+
+    def close(self):
+        if self.ctx is not None:
+            B.pv_destroy(self.ctx)
+            self.ctx = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    # -- options -------------------------------------------------------------
+    def set_option(self, option: int, value: int):
+        B.pv_set_option(self.ctx, option, value)
+
+    def sync(self, stream=None):
+        B.pv_sync(self.ctx, stream)
+
+    # -- loads (host arrays) -------------------------------------------------
+    def load_cluster(self, cluster: W.Cluster):
+        B.pv_load_cluster(self.ctx, cluster.num_nodes, cluster.num_keys, cluster.labels)
+        self.num_nodes = cluster.num_nodes
+
+    def load_network(self, net: W.Network):
+        B.pv_load_flow_tables(self.ctx, net.num_switches, net.rule_offs, net.rules, net.switch_region,
+                              net.port_offs, net.port_peer, net.num_hosts, net.host_switch, net.host_port,
+                              net.host_ip)
+        self.num_hosts = net.num_hosts
+
+    # -- evaluation (device tensors) -----------------------------------------
+    def eval_selectors(self, d_offs, num_exprs, d_exprs, d_assign, num_pods, words=None, d_bits=None,
+                       d_flags=None, stream=None):
+        words = words or W.words_per_row(self.num_nodes)
+        if d_bits is None:
+            d_bits = empty_device(num_pods * words * 4, self.device)
+        if d_flags is None:
+            d_flags = empty_device(num_pods, self.device)
+        B.pv_eval_selectors(self.ctx, num_pods, d_offs, num_exprs, d_exprs, d_assign, d_bits, words, d_flags, stream)
+        return d_bits, d_flags
+
+    def verify_probes(self, d_probes, num_probes, hop_cap, d_out=None, stream=None):
+        if d_out is None:
+            d_out = empty_device(num_probes * 4, self.device)
+        B.pv_verify_probes(self.ctx, num_probes, d_probes, hop_cap, d_out, stream)
+        return d_out
+
+    def compliant_reach(self, graph_dev, num_src, d_src, num_masks, d_masks, words=None, d_reach=None,
+                        stream=None):
+        V, d_offs, E, d_cols, d_region = graph_dev
+        words = words or W.words_per_row(V)
+        if d_reach is None:
+            d_reach = empty_device(num_masks * num_src * words * 4, self.device)
+        B.pv_compliant_reach(self.ctx, V, d_offs, E, d_cols, d_region, num_src, d_src, num_masks, d_masks, d_reach,
+                             words, stream)
+        return d_reach
+
+    def upload_graph(self, g: W.Graph):
+        return (g.num_vertices, to_device(g.offs.astype(np.uint32), self.device), len(g.cols),
+                to_device(g.cols.astype(np.uint32), self.device), to_device(g.region.astype(np.uint8), self.device))
+
+    # -- end-to-end ------------------------------------------------------------
+    def run_end_to_end(self, dev: dict, e2e_sizes: dict, stream=None) -> dict:
+        """Selector rows -> seeded placement -> probe binding -> walks ->
+        per-intent verdict, all on the device.  ``dev`` holds the device
+        inputs (offs, exprs, draws, probes) and output buffers."""
+        I, pods, ppg = e2e_sizes["intents"], e2e_sizes["pods"], e2e_sizes["probes_per_intent"]
+        words = W.words_per_row(self.num_nodes)
+        M = I * ppg
+        B.pv_eval_selectors(self.ctx, I, dev["offs"], e2e_sizes["num_exprs"], dev["exprs"], None, dev["bits"], words,
+                            dev["flags"], stream)
+        B.pv_place_pods(self.ctx, I, pods, dev["bits"], words, dev["draws"], dev["assign"], stream)
+        B.pv_bind_probes(self.ctx, M, dev["probes"], ppg, pods, dev["assign"], stream)
+        B.pv_verify_probes(self.ctx, M, dev["probes"], e2e_sizes["hop_cap"], dev["results"], stream)
+        B.pv_aggregate_intents(self.ctx, I, pods, dev["bits"], words, dev["flags"], dev["assign"], ppg,
+                               dev["results"], dev["pass"], dev["counts"], stream)
+        return dev
+
+    def alloc_end_to_end(self, e: W.EndToEnd) -> tuple:
+        """Device buffers for an end-to-end workload (inputs uploaded)."""
+        I, pods, ppg = e.intents.num_pods, e.pods_per_intent, e.probes_per_intent
+        words = W.words_per_row(e.cluster.num_nodes)
+        M = I * ppg
+        d = self.device
+        dev = {
+            "offs": to_device(e.intents.expr_offs.astype(np.uint32), d),
+            "exprs": to_device(e.intents.exprs, d),
+            "draws": to_device(e.place_draws.astype(np.uint64), d),
+            "probes": to_device(e.probes.probes, d),
+            "bits": empty_device(I * words * 4, d),
+            "flags": empty_device(I, d),
+            "assign": empty_device(I * pods * 4, d),
+            "results": empty_device(M * 4, d),
+            "pass": empty_device(I, d),
+            "counts": empty_device(I * 8 * 4, d),
+        }
+        sizes = {"intents": I, "pods": pods, "probes_per_intent": ppg, "num_exprs": len(e.intents.exprs),
+                 "hop_cap": e.probes.hop_cap}
+        return dev, sizes

@@ -10,3 +10,17 @@ if ROOT not in sys.path:
 
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a) and the built library")
+
+
+@pytest.fixture(scope="session")
+def validator():
+    """One GPU validator context for the GPU tests (library built first)."""
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2602_16100_gb300 import build
+    from paper_2602_16100_gb300.validator import Validator
+    build.build_library()
+    v = Validator(0)
+    yield v
+    v.close()

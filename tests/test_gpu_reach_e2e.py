@@ -1,0 +1,138 @@
+"""GPU parity of compliant reach and the end-to-end pipeline against the
+oracle (bit-exact): random directed and symmetric graphs with ragged vertex
+counts, malformed CSR reported by pv_sync, the continuum-WAN workload on
+sampled (mask, source) rows, and the end-to-end cross-layer pipeline
+(selectors -> placement -> binding -> walks -> verdicts)."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2602_16100_gb300 import binding as B
+from paper_2602_16100_gb300 import workloads as W
+from paper_2602_16100_gb300.validator import to_device, to_numpy
+from gpu_util import sample
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu_reach(v, g, src, masks, words=None):
+    dev = v.device
+    words = words or W.words_per_row(g.num_vertices)
+    out = v.compliant_reach(v.upload_graph(g), len(src), to_device(src.astype(np.uint32), dev), len(masks),
+                            to_device(masks.astype(np.uint32), dev), words=words)
+    v.sync()
+    return to_numpy(out, np.uint32, (len(masks), len(src), words))
+
+
+@pytest.mark.parametrize("V,E,seed", [(1, 0, 1), (37, 90, 2), (200, 900, 3), (1000, 3000, 4), (4097, 12000, 5)])
+def test_random_digraphs(validator, V, E, seed):
+    g = W.random_digraph(seed, V, E, num_regions=6)
+    st = W.Stream(seed, "reach-test")
+    src = st.ints(0, V - 1, 150).astype(np.uint32)
+    masks = (st.u64(9) % np.uint64(64)).astype(np.uint32)
+    masks[0] = 0xFFFFFFFF
+    masks[1] = 0
+    gr = _gpu_reach(validator, g, src, masks)
+    orr = oracle.compliant_reach(g, src, masks)
+    assert (gr == orr).all()
+
+
+def test_symmetric_wan_small_all_sources(validator):
+    q = W.continuum_wan(seed=7, num_vertices=700, num_masks=8, num_regions=12, mask_pop=(2, 8))
+    gr = _gpu_reach(validator, q.graph, q.sources, q.masks, words=W.words_per_row(700) + 4)
+    orr = oracle.compliant_reach(q.graph, q.sources, q.masks, words=W.words_per_row(700) + 4)
+    assert (gr == orr).all()
+
+
+def test_malformed_csr_is_reported(validator):
+    g = W.random_digraph(3, 50, 200)
+    cols = g.cols.copy()
+    cols[7] = 50                      # out of range neighbour: skipped, reported
+    bad = W.Graph(50, g.offs, cols, g.region)
+    dev = validator.device
+    src = np.arange(50, dtype=np.uint32)
+    masks = np.array([0xFFFFFFFF], np.uint32)
+    out = validator.compliant_reach(validator.upload_graph(bad), 50, to_device(src, dev), 1, to_device(masks, dev))
+    with pytest.raises(B.PVError) as e:
+        validator.sync()
+    assert e.value.code == B.PV_EINVAL
+    validator.sync()                  # error was cleared
+    # skipping the bad edge gives the oracle's answer (it never enters it either)
+    got = to_numpy(out, np.uint32, (1, 50, W.words_per_row(50)))
+    assert (got == oracle.compliant_reach(bad, src, masks)).all()
+    with pytest.raises(B.PVError):
+        B.pv_compliant_reach(validator.ctx, 0, 0, 0, 0, 0, 1, 0, 1, 0, 0, 4)
+
+
+def test_continuum_wan_full_size_sampled(validator):
+    q = W.continuum_wan()
+    gr = _gpu_reach(validator, q.graph, q.sources, q.masks)
+    st = W.Stream(11, "reach-sample")
+    pairs = np.stack([st.ints(0, len(q.masks) - 1, 600), st.ints(0, len(q.sources) - 1, 600)], 1).astype(np.uint32)
+    orr = oracle.compliant_reach(q.graph, q.sources, q.masks, pairs=pairs)
+    for i, (m, s) in enumerate(pairs):
+        assert (gr[m, s] == orr[i]).all(), (m, s)
+
+
+def _run_e2e(v, e):
+    v.load_cluster(e.cluster)
+    v.load_network(e.network)
+    dev, sizes = v.alloc_end_to_end(e)
+    v.run_end_to_end(dev, sizes)
+    v.sync()
+    I, pods, ppg = sizes["intents"], sizes["pods"], sizes["probes_per_intent"]
+    words = W.words_per_row(e.cluster.num_nodes)
+    return {
+        "bits": to_numpy(dev["bits"], np.uint32, (I, words)),
+        "flags": to_numpy(dev["flags"], np.uint8),
+        "assign": to_numpy(dev["assign"], np.uint32),
+        "probes": to_numpy(dev["probes"], W.PROBE_DTYPE),
+        "results": to_numpy(dev["results"], W.RESULT_DTYPE),
+        "pass": to_numpy(dev["pass"], np.uint8),
+        "counts": to_numpy(dev["counts"], np.uint32, (I, 8)),
+    }
+
+
+def _oracle_e2e(e, idx_probes=None):
+    c = e.cluster
+    bits, flags = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, e.intents.expr_offs, e.intents.exprs)
+    assign = oracle.place_pods(bits, c.num_nodes, e.pods_per_intent, e.place_draws)
+    probes = oracle.bind_probes(e.probes.probes, e.probes_per_intent, e.pods_per_intent, assign, e.network.host_ip)
+    return bits, flags, assign, probes
+
+
+def test_end_to_end_small(validator):
+    e = W.end_to_end(seed=21, num_switches=64, num_intents=300, probes_per_intent=200, rules_per_switch=200)
+    g = _run_e2e(validator, e)
+    bits, flags, assign, probes = _oracle_e2e(e)
+    assert (g["bits"] == bits).all() and (g["flags"] == flags).all() and (g["assign"] == assign).all()
+    assert (g["probes"] == probes).all()
+    res = oracle.verify_probes(e.network, probes, e.probes.hop_cap)
+    assert (g["results"] == res).all()
+    passed, counts = oracle.aggregate(bits, e.cluster.num_nodes, flags, assign, e.pods_per_intent, res,
+                                      e.probes_per_intent)
+    assert (g["pass"] == passed).all() and (g["counts"] == counts).all()
+
+
+def test_end_to_end_full_size_sampled(validator):
+    """The full end-to-end workload (10,000 intents, 50M probes) in the
+    benchmark's launch configuration; the oracle checks every selector row,
+    placement and binding, and walks a sample of probes; per-intent verdicts
+    are checked on intents whose probes were all sampled."""
+    e = W.end_to_end()
+    g = _run_e2e(validator, e)
+    bits, flags, assign, probes = _oracle_e2e(e)
+    assert (g["bits"] == bits).all() and (g["flags"] == flags).all() and (g["assign"] == assign).all()
+    assert (g["probes"] == probes).all()
+    idx = sample(len(probes), 20000, seed=3)
+    res = oracle.verify_probes(e.network, probes, e.probes.hop_cap, idx=idx)
+    assert (g["results"][idx] == res).all()
+    ppg = e.probes_per_intent
+    for i in (0, 4321, e.intents.num_pods - 1):
+        sl = slice(i * ppg, (i + 1) * ppg)
+        r_i = oracle.verify_probes(e.network, probes, e.probes.hop_cap, idx=np.arange(i * ppg, (i + 1) * ppg))
+        assert (g["results"][sl] == r_i).all()
+        p_i, c_i = oracle.aggregate(bits[i:i + 1], e.cluster.num_nodes, flags[i:i + 1],
+                                    assign[i * e.pods_per_intent:(i + 1) * e.pods_per_intent], e.pods_per_intent,
+                                    r_i, ppg)
+        assert g["pass"][i] == p_i[0] and (g["counts"][i] == c_i[0]).all()

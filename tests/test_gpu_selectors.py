@@ -1,0 +1,139 @@
+"""GPU parity of node-selector evaluation against the oracle (bit-exact):
+both kernels (label-tile comparison and per-value bitset rows), ragged node
+counts spanning several tiles, absent labels, hallucinated values,
+DoesNotExist, malformed expressions, empty inputs, and the placement-scale
+workload (100,000 pods x 5,000 nodes) on sampled pods."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2602_16100_gb300 import binding as B
+from paper_2602_16100_gb300 import workloads as W
+from paper_2602_16100_gb300.validator import empty_device, to_device, to_numpy
+from gpu_util import sample, sub_selectors
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu_eval(v, cluster, sel, kernel, words=None):
+    v.load_cluster(cluster)
+    v.set_option(B.PV_OPT_SELECTOR_KERNEL, kernel)
+    d = v.device
+    words = words or W.words_per_row(cluster.num_nodes)
+    d_assign = None if sel.assign is None else to_device(sel.assign.astype(np.uint32), d)
+    bits, flags = v.eval_selectors(to_device(sel.expr_offs.astype(np.uint32), d), len(sel.exprs),
+                                   to_device(sel.exprs, d), d_assign, sel.num_pods, words=words)
+    v.sync()
+    v.set_option(B.PV_OPT_SELECTOR_KERNEL, 0)
+    return (to_numpy(bits, np.uint32, (sel.num_pods, words)), to_numpy(flags, np.uint8))
+
+
+def _oracle_eval(cluster, sel, words=None):
+    return oracle.eval_selectors(cluster.num_nodes, cluster.num_keys, cluster.labels, sel.expr_offs, sel.exprs,
+                                 sel.assign, words=words)
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_tiny_workload(validator, kernel):
+    d = W.tiny()
+    gb, gf = _gpu_eval(validator, d["cluster"], d["selectors"], kernel)
+    ob, of = _oracle_eval(d["cluster"], d["selectors"])
+    assert (gb == ob).all() and (gf == of).all()
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+@pytest.mark.parametrize("n,k,p_absent,p_unknown,dne", [
+    (1000, 16, 0.0, 0.0, False),      # ragged: 1000 = 31.25 words
+    (4097, 64, 0.1, 0.02, True),      # spans several label tiles and one extra word
+    (33, 5, 0.5, 0.1, True),
+    (32, 3, 0.0, 0.0, False),
+    (7001, 24, 0.05, 0.0, True),
+])
+def test_random_workloads(validator, kernel, n, k, p_absent, p_unknown, dne):
+    d = W.selector_workload(seed=n + k, num_nodes=n, num_keys=k, num_values=40, num_pods=3000,
+                            p_absent=p_absent, p_unknown=p_unknown, with_doesnotexist=dne)
+    gb, gf = _gpu_eval(validator, d["cluster"], d["selectors"], kernel)
+    ob, of = _oracle_eval(d["cluster"], d["selectors"])
+    assert (gf == of).all()
+    assert (gb == ob).all()
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_wide_rows_and_malformed_lists(validator, kernel):
+    d = W.selector_workload(seed=3, num_nodes=300, num_keys=6, num_values=9, num_pods=400, p_absent=0.2)
+    sel = d["selectors"]
+    ex = sel.exprs.copy()
+    ex[5]["key"] = 99                 # key out of range
+    ex[17]["op"] = 9                  # unknown operator
+    ex[40]["nvals"] = 0
+    ex[41]["op"], ex[41]["nvals"] = W.OP_EXISTS, 2
+    ex[60]["vals"][0] = W.ABSENT
+    offs = sel.expr_offs.copy()
+    bad_sel = W.Selectors(sel.num_pods, offs, ex, sel.assign)
+    words = W.words_per_row(300) + 8  # caller-chosen wider rows: padding must be zero
+    gb, gf = _gpu_eval(validator, d["cluster"], bad_sel, kernel, words=words)
+    ob, of = _oracle_eval(d["cluster"], bad_sel, words=words)
+    assert (gf == of).all() and (gb == ob).all()
+    assert (of & W.F_BAD_EXPR).sum() >= 5
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_offsets_beyond_expression_count(validator, kernel):
+    d = W.selector_workload(seed=5, num_nodes=64, num_keys=4, num_values=5, num_pods=10)
+    sel = d["selectors"]
+    offs = sel.expr_offs.copy()
+    offs[3] = offs[4] + 1             # decreasing at pod 3
+    offs[-1] = len(sel.exprs)         # valid end; also try a too-large count below
+    s2 = W.Selectors(sel.num_pods, offs, sel.exprs, sel.assign)
+    gb, gf = _gpu_eval(validator, d["cluster"], s2, kernel)
+    ob, of = _oracle_eval(d["cluster"], s2)
+    assert (gf == of).all() and (gb == ob).all()
+
+
+def test_empty_and_invalid_calls(validator):
+    d = W.selector_workload(seed=1, num_nodes=50, num_keys=4, num_pods=4)
+    validator.load_cluster(d["cluster"])
+    dev = validator.device
+    offs = to_device(d["selectors"].expr_offs.astype(np.uint32), dev)
+    ex = to_device(d["selectors"].exprs, dev)
+    bits = empty_device(4 * 4 * 4, dev)
+    flags = empty_device(4, dev)
+    B.pv_eval_selectors(validator.ctx, 0, offs, 0, ex, None, bits, 4, flags)   # no pods: no-op
+    with pytest.raises(B.PVError) as e:
+        B.pv_eval_selectors(validator.ctx, 4, offs, len(d["selectors"].exprs), ex, None, bits, 2, flags)
+    assert e.value.code == B.PV_EINVAL
+    with pytest.raises(B.PVError):
+        B.pv_eval_selectors(validator.ctx, 4, offs, len(d["selectors"].exprs), ex, None, bits, 6, flags)
+    with pytest.raises(B.PVError) as e:
+        B.pv_load_cluster(validator.ctx, 0, 4, np.zeros(0, np.uint16))
+    assert e.value.code == B.PV_EINVAL
+
+
+def test_placement_scale_sampled(validator):
+    """Full placement-scale workload in the benchmark's launch configuration;
+    the oracle recomputes a sample of pods (both ends included)."""
+    d = W.selector_workload()
+    c, sel = d["cluster"], d["selectors"]
+    validator.load_cluster(c)
+    assert B.pv_get_stat(validator.ctx, B.PV_STAT_SELECTOR_ROWS_BUILT) == 1
+    dev = validator.device
+    words = W.words_per_row(c.num_nodes)
+    bits, flags = validator.eval_selectors(to_device(sel.expr_offs.astype(np.uint32), dev), len(sel.exprs),
+                                           to_device(sel.exprs, dev), to_device(sel.assign.astype(np.uint32), dev),
+                                           sel.num_pods, words=words)
+    validator.sync()
+    gb = to_numpy(bits, np.uint32, (sel.num_pods, words))
+    gf = to_numpy(flags, np.uint8)
+    idx = sample(sel.num_pods, 3000, seed=1)
+    offs, ex, asg = sub_selectors(sel, idx)
+    ob, of = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, offs, ex, asg, words=words)
+    assert (gb[idx] == ob).all() and (gf[idx] == of).all()
+    # the comparison kernel agrees on the same sample
+    validator.set_option(B.PV_OPT_SELECTOR_KERNEL, 1)
+    bits1, flags1 = validator.eval_selectors(to_device(offs, dev), len(ex), to_device(ex, dev),
+                                             to_device(asg, dev), len(idx), words=words)
+    validator.sync()
+    validator.set_option(B.PV_OPT_SELECTOR_KERNEL, 0)
+    assert (to_numpy(bits1, np.uint32, (len(idx), words)) == ob).all()
+    assert (to_numpy(flags1, np.uint8) == of).all()
