@@ -131,8 +131,8 @@ class EndToEndBench:
     name = "end-to-end cross-layer"
     unit = "probe-hop verifications/s"
 
-    def __init__(self, seed):
-        self.e = W.end_to_end(seed=20260220 + seed)
+    def __init__(self, seed, intents=None):
+        self.e = W.end_to_end(seed=20260220 + seed, **({"num_intents": intents} if intents else {}))
 
     def config(self):
         e = self.e
@@ -236,6 +236,9 @@ class EndToEndBench:
 
     oracle_start = 2
 
+    def oracle_max(self):
+        return self.e.intents.num_pods
+
 
 class PlacementBench:
     name = "placement-scale"
@@ -293,6 +296,9 @@ class PlacementBench:
 
     oracle_start = 500
 
+    def oracle_max(self):
+        return self.s.num_pods
+
 
 class FlowBench:
     name = "flow-verification"
@@ -343,6 +349,9 @@ class FlowBench:
         return int(r["hops"].astype(np.int64).sum()), dt, f"first {n} probes"
 
     oracle_start = 2000
+
+    def oracle_max(self):
+        return len(self.p.probes)
 
 
 class WanBench:
@@ -396,6 +405,9 @@ class WanBench:
 
     oracle_start = 256
 
+    def oracle_max(self):
+        return len(self.q.masks) * len(self.q.sources)
+
 
 WORKLOADS = {"e2e": EndToEndBench, "placement": PlacementBench, "flow": FlowBench, "wan": WanBench}
 SOURCES = {"walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector": ("k_selector.cu",),
@@ -404,12 +416,12 @@ SOURCES = {"walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector
 
 def timed_oracle(wl, target_s=12.0, cap_s=40.0):
     """Grow the sample until one run takes >= target_s seconds of CPU."""
-    n = wl.oracle_start
+    n = min(wl.oracle_start, wl.oracle_max())
     while True:
         units, dt, desc = wl.oracle_sample(n)
-        if dt >= target_s or dt * 2 > cap_s:
+        if dt >= target_s or dt * 2 > cap_s or n >= wl.oracle_max():
             return units, dt, desc, n
-        n = int(n * max(1.5, min(8.0, target_s / max(dt, 1e-3))))
+        n = min(wl.oracle_max(), int(n * max(1.5, min(8.0, target_s / max(dt, 1e-3)))))
 
 
 # ----------------------------------------------------------------------------
@@ -458,7 +470,7 @@ def run_ours(args):
         build.build_library()
     if dist:
         dist.barrier()
-    wl = WORKLOADS[args.workload](rank)
+    wl = WORKLOADS[args.workload](rank, **({"intents": args.intents} if args.intents else {}))
     v = Validator(local)
     wl.setup(v)
     stream = torch.cuda.current_stream()
@@ -565,7 +577,11 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", choices=tuple(WORKLOADS), default="e2e")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--intents", type=int, default=None,
+                    help="end-to-end only: fewer intents (a smaller case for profiling, not a bench line)")
     args = ap.parse_args()
+    if args.intents and args.workload != "e2e":
+        ap.error("--intents applies to the end-to-end workload only")
     if args.warmup < 3:
         print("note: warmup raised to 3", file=sys.stderr)
         args.warmup = 3

@@ -273,13 +273,19 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  * PV_OPT_SELECTOR_KERNEL: 0 = automatic, 1 = per-node label comparison over
  *   shared-memory label tiles, 2 = per-(key, value) node-bitset rows
  *   (needs the rows to have been built by pv_load_cluster).
- * PV_OPT_WALK_KERNEL: 0 = automatic, 1 = hop-synchronous regroup + staged
- *   tables (the only kernel at present).
+ * PV_OPT_WALK_KERNEL: 0 = automatic, 1 = linear first-match scan of the
+ *   staged table, 2 = indexed first match (per-dport-bucket candidate lists
+ *   and destination-interval maps built by pv_load_flow_tables; needs every
+ *   switch's index to fit shared memory).
  * pv_get_stat: PV_STAT_SELECTOR_ROWS_BUILT (1 if value rows exist),
- *   PV_STAT_SCRATCH_BYTES.
+ *   PV_STAT_SCRATCH_BYTES, PV_STAT_WALK_INDEX_FITS (1 if kernel 2 is
+ *   usable), PV_STAT_WALK_INDEX_BYTES (largest per-switch table + index).
  * ------------------------------------------------------------------------- */
 enum { PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2 };
-enum { PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2 };
+enum {
+    PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,
+    PV_STAT_WALK_INDEX_BYTES = 4
+};
 int pv_set_option(pv_ctx *ctx, int option, int64_t value);
 int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value);
 

@@ -129,6 +129,287 @@ __global__ void __launch_bounds__(1024) compile_tables_kernel(const uint32_t *__
 }
 
 // ---------------------------------------------------------------------------
+// load: first-match index
+// ---------------------------------------------------------------------------
+// A switch's blob (sections 16-byte aligned):
+//   header   uint4 {npad, n_items, n_segs, n_bnd}
+//   A[npad] uint4, B[npad] uint2     rules in first-match order (as above)
+//   boff[kBuckets + 1] u32           item range of each destination-port bucket
+//   items[n_items] u16               per bucket, in first-match order: a rule
+//                                    position, or kSegItem | segment id
+//   segs[n_segs] uint2               {first boundary, number of boundaries}
+//   bnd[n_bnd] u32, win[n_bnd] u32   per segment: ascending elementary-interval
+//                                    starts (the first is 0) and the interval's
+//                                    winner (kWinFound | action, or 0 = none)
+// Exactness.  A header whose dport lies in bucket k can only match rules whose
+// port range meets bucket k; bucket k's list keeps the first-match order, so
+// its first hit is the first match of the whole table.  A segment is a run of
+// consecutive rules that constrain nothing but the destination prefix (any
+// in_port, no source prefix, full port range); every rule's address range is
+// a union of the segment's elementary intervals (each range contributes its
+// start and end + 1 as boundaries), so within a segment the first match of
+// address d is the precomputed winner of d's interval.
+constexpr uint32_t kBuckets = 64;           // dport >> kBucketShift
+constexpr uint32_t kBucketShift = 10;
+constexpr uint32_t kMinSegment = 4;         // shorter destination-only runs stay plain items
+constexpr uint32_t kMaxSegment = 4096;      // longer runs are split (in order: still exact)
+constexpr uint32_t kMaxSegments = PV_MAX_RULES / kMinSegment;
+constexpr uint32_t kSegItem = 0x8000u;
+constexpr uint32_t kWinFound = 0x80000000u;
+constexpr uint32_t kKeyCap = 2 * kMaxSegment + 8;   // boundaries of one segment (+ slack)
+constexpr uint32_t kSortCap = 16384;                // power of two >= 2 * kMaxSegment + 1
+constexpr size_t kIndexSmem = (size_t)kSortCap * 4 + (size_t)kKeyCap * 8 + PV_MAX_RULES * 2 + kMaxSegments * 8;
+
+__host__ __device__ inline uint32_t up16(uint32_t b) { return (b + 15u) & ~15u; }
+
+struct BlobLayout {
+    uint32_t a, b, boff, items, segs, bnd, win, total;
+    __host__ __device__ BlobLayout(uint32_t npad, uint32_t n_items, uint32_t n_segs, uint32_t n_bnd) {
+        a = 16;
+        b = a + npad * 16;
+        boff = b + npad * 8;
+        items = boff + up16((kBuckets + 1) * 4);
+        segs = items + up16(n_items * 2);
+        bnd = segs + up16(n_segs * 8);
+        win = bnd + up16(n_bnd * 4);
+        total = win + up16(n_bnd * 4);
+    }
+};
+
+__device__ __forceinline__ bool rule_dst_only(uint4 a, uint2 b) {
+    return a.y == 0 && b.x == 0xFFFF0000u && ((b.y >> 8) & 0xFFu) == 0;
+}
+
+// In-place exclusive scan of v[0..n) by the whole block; returns the total.
+__device__ uint32_t block_exclusive_scan(uint32_t *v, uint32_t n, uint32_t *s_warp) {
+    const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
+    const uint32_t per = (n + nt - 1) / nt, b0 = t * per;
+    uint32_t local = 0;
+    for (uint32_t i = 0; i < per; ++i)
+        if (b0 + i < n) local += v[b0 + i];
+    uint32_t incl = local;
+    for (int d = 1; d < 32; d <<= 1) {
+        const uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
+        if (lane >= (uint32_t)d) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        const uint32_t x = lane < nt / 32 ? s_warp[lane] : 0u;
+        uint32_t xi = x;
+        for (int d = 1; d < 32; d <<= 1) {
+            const uint32_t y = __shfl_up_sync(PV_FULL_MASK, xi, d);
+            if (lane >= (uint32_t)d) xi += y;
+        }
+        s_warp[lane] = xi - x;
+        if (lane == 31) s_warp[32] = xi;
+    }
+    __syncthreads();
+    uint32_t run = s_warp[warp] + incl - local;
+    for (uint32_t i = 0; i < per; ++i)
+        if (b0 + i < n) {
+            const uint32_t x = v[b0 + i];
+            v[b0 + i] = run;
+            run += x;
+        }
+    const uint32_t total = s_warp[32];
+    __syncthreads();
+    return total;
+}
+
+// Pass 1 (kFill = false) writes sizes[s] = {n_items, n_segs, n_bnd}; pass 2
+// writes the blob at blob_offs[s].  One 1024-thread block per switch.
+template <bool kFill>
+__global__ void __launch_bounds__(1024) index_build_kernel(const uint32_t *__restrict__ rule_offs,
+                                                           const uint32_t *__restrict__ tab_offs,
+                                                           const uint4 *__restrict__ A, const uint2 *__restrict__ B,
+                                                           uint32_t *__restrict__ sizes,
+                                                           const uint64_t *__restrict__ blob_offs,
+                                                           uint8_t *__restrict__ blob) {
+    extern __shared__ __align__(16) uint32_t s_mem[];
+    uint32_t *s_keys = s_mem;                                      // [kSortCap]
+    uint32_t *s_win = s_keys + kSortCap;                           // [kKeyCap]
+    uint32_t *s_pos = s_win + kKeyCap;                             // [kKeyCap]
+    int16_t *s_cls = reinterpret_cast<int16_t *>(s_pos + kKeyCap);  // [PV_MAX_RULES]
+    uint32_t *s_segs = reinterpret_cast<uint32_t *>(s_cls + PV_MAX_RULES);  // [kMaxSegments][2]
+    __shared__ uint32_t s_warp[33];
+    __shared__ uint32_t s_nsegs;
+    const uint32_t s = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
+    const uint32_t n = rule_offs[s + 1] - rule_offs[s];
+    const uint32_t t0 = tab_offs[s], npad = tab_offs[s + 1] - t0;
+    const uint4 *a = A + t0;
+    const uint2 *b = B + t0;
+
+    // 1. destination-only runs -> segments
+    if (t == 0) {
+        uint32_t seg = 0, i = 0;
+        while (i < n) {
+            if (!rule_dst_only(a[i], b[i])) {
+                s_cls[i++] = -1;
+                continue;
+            }
+            uint32_t j = i;
+            while (j < n && rule_dst_only(a[j], b[j])) ++j;
+            if (j - i < kMinSegment) {
+                for (uint32_t k = i; k < j; ++k) s_cls[k] = -1;
+            } else {
+                for (uint32_t k0 = i; k0 < j; k0 += kMaxSegment) {
+                    const uint32_t k1 = min(j, k0 + kMaxSegment);
+                    s_segs[2 * seg] = k0;
+                    s_segs[2 * seg + 1] = k1;
+                    for (uint32_t k = k0; k < k1; ++k) s_cls[k] = (int16_t)seg;
+                    ++seg;
+                }
+            }
+            i = j;
+        }
+        s_nsegs = seg;
+    }
+    __syncthreads();
+    const uint32_t nsegs = s_nsegs;
+    uint8_t *out = nullptr;
+    BlobLayout L(npad, 0, 0, 0);
+    if (kFill) {
+        out = blob + blob_offs[s];
+        L = BlobLayout(npad, sizes[3 * s], sizes[3 * s + 1], sizes[3 * s + 2]);
+    }
+
+    // 2. bucket lists
+    auto in_bucket = [&](uint32_t i, uint32_t k) -> bool {
+        if (i >= n) return false;
+        const int c = s_cls[i];
+        if (c >= 0) return s_segs[2 * c] == i;   // segment token at its first rule
+        const uint32_t lo = b[i].x & 0xFFFFu, hi = b[i].x >> 16;
+        return lo <= ((k << kBucketShift) | ((1u << kBucketShift) - 1u)) && hi >= (k << kBucketShift);
+    };
+    for (uint32_t k = warp; k < kBuckets; k += nt / 32) {
+        uint32_t cnt = 0;
+        for (uint32_t c0 = 0; c0 < n; c0 += 32) cnt += __popc(__ballot_sync(PV_FULL_MASK, in_bucket(c0 + lane, k)));
+        if (lane == 0) s_pos[k] = cnt;
+    }
+    __syncthreads();
+    const uint32_t n_items = block_exclusive_scan(s_pos, kBuckets, s_warp);
+    if (kFill) {
+        uint32_t *boff = reinterpret_cast<uint32_t *>(out + L.boff);
+        uint16_t *items = reinterpret_cast<uint16_t *>(out + L.items);
+        for (uint32_t k = t; k < kBuckets; k += nt) boff[k] = s_pos[k];
+        if (t == 0) boff[kBuckets] = n_items;
+        for (uint32_t k = warp; k < kBuckets; k += nt / 32) {
+            uint32_t base = s_pos[k];
+            for (uint32_t c0 = 0; c0 < n; c0 += 32) {
+                const uint32_t i = c0 + lane;
+                const bool inc = in_bucket(i, k);
+                const uint32_t m = __ballot_sync(PV_FULL_MASK, inc);
+                if (inc) {
+                    const int c = s_cls[i];
+                    items[base + __popc(m & ((1u << lane) - 1u))] = (uint16_t)(c >= 0 ? (kSegItem | (uint32_t)c) : i);
+                }
+                base += __popc(m);
+            }
+        }
+    }
+    __syncthreads();
+
+    // 3. per segment: sorted unique boundaries, interval winners, merged runs
+    uint32_t n_bnd = 0;
+    for (uint32_t j = 0; j < nsegs; ++j) {
+        const uint32_t k0 = s_segs[2 * j], k1 = s_segs[2 * j + 1], m = k1 - k0;
+        const uint32_t nk = 2 * m + 1;
+        uint32_t npow = 1;
+        while (npow < nk) npow <<= 1;
+        for (uint32_t x = t; x < npow; x += nt) {
+            uint32_t key = 0xFFFFFFFFu;
+            if (x == 0) {
+                key = 0;
+            } else if (x < nk) {
+                const uint4 r = a[k0 + (x - 1) / 2];
+                if (x & 1u) {
+                    key = r.z;
+                } else {
+                    const uint64_t end1 = (uint64_t)r.z + (uint64_t)(~r.w) + 1ull;
+                    key = end1 < (1ull << 32) ? (uint32_t)end1 : 0u;
+                }
+            }
+            s_keys[x] = key;
+        }
+        __syncthreads();
+        for (uint32_t kk = 2; kk <= npow; kk <<= 1)
+            for (uint32_t jj = kk >> 1; jj > 0; jj >>= 1) {
+                for (uint32_t i = t; i < npow; i += nt) {
+                    const uint32_t ixj = i ^ jj;
+                    if (ixj > i) {
+                        const uint32_t p = s_keys[i], q = s_keys[ixj];
+                        if ((p > q) == ((i & kk) == 0)) {
+                            s_keys[i] = q;
+                            s_keys[ixj] = p;
+                        }
+                    }
+                }
+                __syncthreads();
+            }
+        for (uint32_t x = t; x < nk; x += nt) s_pos[x] = (x == 0 || s_keys[x] != s_keys[x - 1]) ? 1u : 0u;
+        __syncthreads();
+        for (uint32_t x = t; x < nk; x += nt) s_win[x] = s_keys[x];   // keep sorted copy
+        __syncthreads();
+        const uint32_t K = block_exclusive_scan(s_pos, nk, s_warp);
+        for (uint32_t x = t; x < nk; x += nt)
+            if (x == 0 || s_win[x] != s_win[x - 1]) s_keys[s_pos[x]] = s_win[x];
+        __syncthreads();
+        // winners of the K elementary intervals
+        for (uint32_t x = t; x < K; x += nt) {
+            const uint32_t d = s_keys[x];
+            uint32_t w = 0;
+            for (uint32_t r = k0; r < k1; ++r) {
+                const uint4 ar = a[r];
+                if (((d ^ ar.z) & ar.w) == 0) {
+                    w = kWinFound | (b[r].y >> 16);
+                    break;
+                }
+            }
+            s_win[x] = w;
+        }
+        __syncthreads();
+        // merge adjacent intervals with the same winner
+        for (uint32_t x = t; x < K; x += nt) s_pos[x] = (x == 0 || s_win[x] != s_win[x - 1]) ? 1u : 0u;
+        __syncthreads();
+        // keep flags must be read before the scan overwrites them
+        uint32_t keep_mask = 0;
+        for (uint32_t x = t, q = 0; x < K && q < 32; x += nt, ++q)
+            if (s_pos[x]) keep_mask |= 1u << q;
+        __syncthreads();
+        const uint32_t K2 = block_exclusive_scan(s_pos, K, s_warp);
+        if (kFill) {
+            uint2 *segs = reinterpret_cast<uint2 *>(out + L.segs);
+            uint32_t *bnd = reinterpret_cast<uint32_t *>(out + L.bnd);
+            uint32_t *win = reinterpret_cast<uint32_t *>(out + L.win);
+            if (t == 0) segs[j] = make_uint2(n_bnd, K2);
+            for (uint32_t x = t, q = 0; x < K; x += nt, ++q)
+                if ((keep_mask >> q) & 1u) {
+                    bnd[n_bnd + s_pos[x]] = s_keys[x];
+                    win[n_bnd + s_pos[x]] = s_win[x];
+                }
+        }
+        n_bnd += K2;
+        __syncthreads();
+    }
+
+    // 4. header and rules
+    if (kFill) {
+        if (t == 0) *reinterpret_cast<uint4 *>(out) = make_uint4(npad, n_items, nsegs, n_bnd);
+        uint4 *oa = reinterpret_cast<uint4 *>(out + L.a);
+        uint2 *ob = reinterpret_cast<uint2 *>(out + L.b);
+        for (uint32_t i = t; i < npad; i += nt) {
+            oa[i] = a[i];
+            ob[i] = b[i];
+        }
+    } else if (t == 0) {
+        sizes[3 * s] = n_items;
+        sizes[3 * s + 1] = nsegs;
+        sizes[3 * s + 2] = n_bnd;
+    }
+}
+
+// ---------------------------------------------------------------------------
 // walk kernels
 // ---------------------------------------------------------------------------
 // Every thread of the block calls this; threads with want append one slot of
@@ -288,10 +569,8 @@ struct HopArgs {
     uint32_t hop, cap;
     const uint32_t *seg;
     uint32_t S, H;
-    const uint32_t *tab_offs;
-    const uint4 *rule_a;
-    const uint2 *rule_b;
-    uint32_t max_pad;
+    const uint8_t *blob;
+    const uint64_t *blob_offs;
     const uint8_t *region;
     const uint32_t *port_offs;
     const int32_t *port_peer;
@@ -303,10 +582,92 @@ struct HopArgs {
     int32_t *status;
 };
 
+// Linear first match: 32 consecutive rules per warp step.
+// Both first-match routines return kWinFound | action, or 0 for a table miss.
+__device__ __forceinline__ uint32_t first_match_linear(const uint8_t *sm, uint32_t npad, uint32_t lane, uint32_t src,
+                                                       uint32_t dst, uint32_t dport, uint32_t in_port) {
+    const BlobLayout L(npad, 0, 0, 0);
+    const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
+    const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
+    for (uint32_t base = 0; base < npad; base += 32) {
+        const uint4 a = sA[base + lane];
+        const uint2 b = sB[base + lane];
+        const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ b.y) & ((b.y >> 8) & 0xFFu));
+        const bool hit = diff == 0 && dport >= (b.x & 0xFFFFu) && dport <= (b.x >> 16);
+        const uint32_t m = __ballot_sync(PV_FULL_MASK, hit);
+        if (m) return kWinFound | __shfl_sync(PV_FULL_MASK, b.y >> 16, __ffs(m) - 1);
+    }
+    return 0u;
+}
+
+// Winner of the elementary interval holding dst: the warp narrows the range
+// 32-ways per step (bnd ascending, bnd[0] = 0 <= dst).
+__device__ __forceinline__ uint32_t segment_lookup(const uint32_t *bnd, const uint32_t *win, uint32_t cnt,
+                                                   uint32_t dst, uint32_t lane) {
+    uint32_t lo = 0, len = cnt;
+    while (len > 32) {
+        const uint32_t stride = (len + 31) / 32;
+        const bool le = lane * stride < len && bnd[lo + lane * stride] <= dst;
+        const uint32_t c = __popc(__ballot_sync(PV_FULL_MASK, le));
+        lo += (c - 1) * stride;
+        len = min(stride, len - (c - 1) * stride);
+    }
+    const bool le = lane < len && bnd[lo + lane] <= dst;
+    const uint32_t c = __popc(__ballot_sync(PV_FULL_MASK, le));
+    return win[lo + c - 1];
+}
+
+// Indexed first match: walk the dport bucket's candidate list in first-match
+// order, 32 items per step; segment items are answered by interval lookup.
+__device__ __forceinline__ uint32_t first_match_indexed(const uint8_t *sm, const uint4 hdr, uint32_t lane,
+                                                        uint32_t src, uint32_t dst, uint32_t dport, uint32_t in_port) {
+    const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
+    const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
+    const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
+    const uint32_t *boff = reinterpret_cast<const uint32_t *>(sm + L.boff);
+    const uint16_t *items = reinterpret_cast<const uint16_t *>(sm + L.items);
+    const uint2 *segs = reinterpret_cast<const uint2 *>(sm + L.segs);
+    const uint32_t *bnd = reinterpret_cast<const uint32_t *>(sm + L.bnd);
+    const uint32_t *win = reinterpret_cast<const uint32_t *>(sm + L.win);
+    const uint32_t k = dport >> kBucketShift;
+    const uint32_t i0 = boff[k], i1 = boff[k + 1];
+    for (uint32_t c0 = i0; c0 < i1; c0 += 32) {
+        const uint32_t idx = c0 + lane;
+        const uint32_t it = idx < i1 ? items[idx] : 0xFFFFu;
+        const bool valid = it != 0xFFFFu;
+        const bool is_seg = valid && (it & kSegItem);
+        bool hit = false;
+        uint32_t action = 0;
+        if (valid && !is_seg) {
+            const uint4 a = sA[it];
+            const uint2 b = sB[it];
+            const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ b.y) & ((b.y >> 8) & 0xFFu));
+            hit = diff == 0 && dport >= (b.x & 0xFFFFu) && dport <= (b.x >> 16);
+            action = b.y >> 16;
+        }
+        uint32_t G = __ballot_sync(PV_FULL_MASK, hit);
+        uint32_t Sg = __ballot_sync(PV_FULL_MASK, is_seg);
+        while (true) {
+            const uint32_t pg = G ? (uint32_t)__ffs(G) - 1 : 32u;
+            const uint32_t ps = Sg ? (uint32_t)__ffs(Sg) - 1 : 32u;
+            if (ps < pg) {
+                const uint2 sd = segs[__shfl_sync(PV_FULL_MASK, it, ps) & 0x7FFFu];
+                const uint32_t w = segment_lookup(bnd + sd.x, win + sd.x, sd.y, dst, lane);
+                if (w & kWinFound) return w;
+                Sg &= Sg - 1u;
+            } else if (pg < 32u) {
+                return kWinFound | __shfl_sync(PV_FULL_MASK, action, pg);
+            } else {
+                break;
+            }
+        }
+    }
+    return 0u;
+}
+
+template <bool kIndexed>
 __global__ void __launch_bounds__(kHopThreads) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
-    uint4 *sA = reinterpret_cast<uint4 *>(s_raw);
-    uint2 *sB = reinterpret_cast<uint2 *>(s_raw + (size_t)g.max_pad * 16);
     __shared__ uint64_t s_bar;
     __shared__ uint32_t s_tmp[40];
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -328,23 +689,23 @@ __global__ void __launch_bounds__(kHopThreads) walk_hop_kernel(HopArgs g) {
         }
         const uint32_t s = lo;
         const uint32_t seg_end = min(r1, g.seg[s + 1]);
-        const uint32_t t0 = g.tab_offs[s], npad = g.tab_offs[s + 1] - t0;
+        const uint8_t *src_blob = g.blob + g.blob_offs[s];
+        const uint4 hdr = __ldg(reinterpret_cast<const uint4 *>(src_blob));
+        const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
+        const uint32_t bytes = kIndexed ? L.total : L.boff;   // header + rules (+ index)
         __syncthreads();   // everyone is done with the previous table
-        if (npad > 0) {
-            if (threadIdx.x == 0) {
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                mbar_arrive_expect_tx(&s_bar, npad * 24u);
-                bulk_g2s(sA, g.rule_a + t0, npad * 16u, &s_bar);
-                bulk_g2s(sB, g.rule_b + t0, npad * 8u, &s_bar);
-            }
-            const bool ok = mbar_wait_bounded(&s_bar, parity);
-            if (__syncthreads_or(!ok)) {
-                if (threadIdx.x == 0) pv_device_error(g.status, PV_ETIMEOUT);
-                mbar_wait_bounded(&s_bar, parity);   // let copies in flight land
-                return;
-            }
-            parity ^= 1u;
+        if (threadIdx.x == 0) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            mbar_arrive_expect_tx(&s_bar, bytes);
+            bulk_g2s(s_raw, src_blob, bytes, &s_bar);
         }
+        const bool ok = mbar_wait_bounded(&s_bar, parity);
+        if (__syncthreads_or(!ok)) {
+            if (threadIdx.x == 0) pv_device_error(g.status, PV_ETIMEOUT);
+            mbar_wait_bounded(&s_bar, parity);   // let copies in flight land
+            return;
+        }
+        parity ^= 1u;
         const uint32_t reg = g.region[s];
         const uint32_t pbase = g.port_offs[s], nports = g.port_offs[s + 1] - pbase;
         for (uint32_t rb = pos; rb < seg_end; rb += 32 * kHopWarps) {
@@ -363,23 +724,10 @@ __global__ void __launch_bounds__(kHopThreads) walk_hop_kernel(HopArgs g) {
                     status = PV_VIOLATION;
                 } else {
                     const uint32_t src = pr.x, dst = pr.y, dport = pr.z & 0xFFFFu;
-                    uint32_t act = PV_DROP;
-                    bool found = false;
-                    for (uint32_t base = 0; base < npad; base += 32) {
-                        const uint4 a = sA[base + lane];
-                        const uint2 b = sB[base + lane];
-                        const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) |
-                                              ((in_port ^ b.y) & ((b.y >> 8) & 0xFFu));
-                        const bool hit = diff == 0 && dport >= (b.x & 0xFFFFu) && dport <= (b.x >> 16);
-                        const uint32_t m = __ballot_sync(PV_FULL_MASK, hit);
-                        if (m) {
-                            const int l = __ffs(m) - 1;
-                            act = __shfl_sync(PV_FULL_MASK, b.y >> 16, l);
-                            found = true;
-                            break;
-                        }
-                    }
-                    if (!found || act == PV_DROP || act >= nports) {
+                    const uint32_t fm = kIndexed ? first_match_indexed(s_raw, hdr, lane, src, dst, dport, in_port)
+                                                 : first_match_linear(s_raw, hdr.x, lane, src, dst, dport, in_port);
+                    const uint32_t act = fm & 0xFFFFu;
+                    if (!(fm & kWinFound) || act == PV_DROP || act >= nports) {
                         status = PV_DROPPED;
                     } else {
                         const int32_t peer = g.port_peer[pbase + act];
@@ -481,12 +829,24 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     pv_free_tables(ctx->tb);
     pv_table_state &t = ctx->tb;
     const uint32_t T = tab[S];
-    uint32_t *d_rule_offs = nullptr;
+    uint32_t *d_rule_offs = nullptr, *d_tab_offs = nullptr, *d_sizes = nullptr;
     pv_rule *d_raw = nullptr;
+    uint4 *d_rule_a = nullptr;
+    uint2 *d_rule_b = nullptr;
+    auto free_temps = [&]() {
+        pv_device_free(d_rule_offs);
+        pv_device_free(d_raw);
+        pv_device_free(d_tab_offs);
+        pv_device_free(d_rule_a);
+        pv_device_free(d_rule_b);
+        pv_device_free(d_sizes);
+    };
     int rc;
-    if ((rc = pv_device_alloc(ctx, (void **)&t.d_tab_offs, (S + 1) * 4, "table offsets")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_rule_a, (size_t)T * 16, "rules A")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_rule_b, (size_t)T * 8, "rules B")) ||
+    if ((rc = pv_device_alloc(ctx, (void **)&d_tab_offs, (S + 1) * 4, "table offsets")) ||
+        (rc = pv_device_alloc(ctx, (void **)&d_rule_a, (size_t)T * 16, "rules A")) ||
+        (rc = pv_device_alloc(ctx, (void **)&d_rule_b, (size_t)T * 8, "rules B")) ||
+        (rc = pv_device_alloc(ctx, (void **)&d_sizes, (size_t)S * 12, "index sizes")) ||
+        (rc = pv_device_alloc(ctx, (void **)&t.d_blob_offs, ((size_t)S + 1) * 8, "blob offsets")) ||
         (rc = pv_device_alloc(ctx, (void **)&t.d_region, S, "regions")) ||
         (rc = pv_device_alloc(ctx, (void **)&t.d_port_offs, (S + 1) * 4, "port offsets")) ||
         (rc = pv_device_alloc(ctx, (void **)&t.d_port_peer, (size_t)P * 4, "port peers")) ||
@@ -495,13 +855,12 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         (rc = pv_device_alloc(ctx, (void **)&t.d_host_ip, (size_t)H * 4, "host ip")) ||
         (rc = pv_device_alloc(ctx, (void **)&d_rule_offs, (S + 1) * 4, "rule offsets")) ||
         (rc = pv_device_alloc(ctx, (void **)&d_raw, (size_t)R * sizeof(pv_rule), "raw rules"))) {
-        pv_device_free(d_rule_offs);
-        pv_device_free(d_raw);
+        free_temps();
         pv_free_tables(t);
         return rc;
     }
     cudaError_t e = cudaSuccess;
-    e = e ? e : cudaMemcpy(t.d_tab_offs, tab.data(), (S + 1) * 4, cudaMemcpyHostToDevice);
+    e = e ? e : cudaMemcpy(d_tab_offs, tab.data(), (S + 1) * 4, cudaMemcpyHostToDevice);
     e = e ? e : cudaMemcpy(t.d_region, switch_region, S, cudaMemcpyHostToDevice);
     e = e ? e : cudaMemcpy(t.d_port_offs, port_offs, (S + 1) * 4, cudaMemcpyHostToDevice);
     if (P) e = e ? e : cudaMemcpy(t.d_port_peer, port_peer, (size_t)P * 4, cudaMemcpyHostToDevice);
@@ -517,12 +876,48 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         for (uint32_t s = 0; s < S; ++s) maxn = std::max(maxn, rule_offs[s + 1] - rule_offs[s]);
         uint32_t npow = 1;
         while (npow < maxn) npow <<= 1;
-        compile_tables_kernel<<<S, 1024, npow * 4>>>(d_rule_offs, d_raw, t.d_tab_offs, t.d_rule_a, t.d_rule_b);
+        compile_tables_kernel<<<S, 1024, npow * 4>>>(d_rule_offs, d_raw, d_tab_offs, d_rule_a, d_rule_b);
+        e = cudaGetLastError();
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(index_build_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kIndexSmem);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(index_build_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)kIndexSmem);
+        if (e == cudaSuccess) {
+            index_build_kernel<false><<<S, 1024, kIndexSmem>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
+                                                               nullptr, nullptr);
+            e = cudaGetLastError();
+        }
+    }
+    // blob layout from the index sizes
+    std::vector<uint32_t> sizes((size_t)S * 3);
+    std::vector<uint64_t> boffs(S + 1, 0);
+    if (e == cudaSuccess) e = cudaMemcpy(sizes.data(), d_sizes, (size_t)S * 12, cudaMemcpyDeviceToHost);
+    uint32_t max_blob = 0, max_linear = 0;
+    if (e == cudaSuccess) {
+        for (uint32_t s = 0; s < S; ++s) {
+            const uint32_t npad = tab[s + 1] - tab[s];
+            const BlobLayout L(npad, sizes[3 * s], sizes[3 * s + 1], sizes[3 * s + 2]);
+            boffs[s + 1] = boffs[s] + L.total;
+            max_blob = std::max(max_blob, L.total);
+            max_linear = std::max(max_linear, L.boff);
+        }
+        e = cudaMemcpy(t.d_blob_offs, boffs.data(), ((size_t)S + 1) * 8, cudaMemcpyHostToDevice);
+    }
+    if (e == cudaSuccess) {
+        rc = pv_device_alloc(ctx, (void **)&t.d_blob, boffs[S], "flow table blobs");
+        if (rc) {
+            free_temps();
+            pv_free_tables(t);
+            return rc;
+        }
+        index_build_kernel<true><<<S, 1024, kIndexSmem>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
+                                                          t.d_blob_offs, t.d_blob);
         e = cudaGetLastError();
         if (e == cudaSuccess) e = cudaDeviceSynchronize();
     }
-    pv_device_free(d_rule_offs);
-    pv_device_free(d_raw);
+    free_temps();
     if (e != cudaSuccess) {
         pv_free_tables(t);
         return pv_cuda_fail(ctx, e, "pv_load_flow_tables");
@@ -530,13 +925,21 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     t.num_switches = S;
     t.num_hosts = H;
     t.max_rules_padded = max_pad;
-    const size_t smem = (size_t)max_pad * 24;
-    if (smem > ctx->max_smem_optin - 1024) {
+    t.max_blob_bytes = max_blob;
+    t.max_linear_bytes = max_linear;
+    const size_t smem_cap = ctx->max_smem_optin - 1024;
+    t.index_fits = max_blob <= smem_cap;
+    if (max_linear > smem_cap) {
         pv_free_tables(t);
-        return pv_fail(ctx, PV_EINVAL, "largest flow table needs %zu bytes of shared memory", smem);
+        return pv_fail(ctx, PV_EINVAL, "largest flow table needs %u bytes of shared memory", max_linear);
     }
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)max_linear),
                 "walk_hop_kernel smem");
+    if (t.index_fits)
+        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)max_blob),
+                    "walk_hop_kernel smem");
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           (int)(2 * kSmemHistMax * 4)),
                 "walk_scatter_kernel smem");
@@ -575,19 +978,25 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     pv_prof_stop(ctx, st, pr, 1);
     const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
-    const size_t hop_smem = (size_t)t.max_rules_padded * 24;
+    int which = ctx->opt_walk;
+    if (which == 0) which = t.index_fits ? 2 : 1;
+    if (which == 2 && !t.index_fits)
+        return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: the first-match index does not fit shared memory");
+    const bool indexed = which == 2;
+    const size_t hop_smem = indexed ? t.max_blob_bytes : t.max_linear_bytes;
     int hop_blocks_per_sm = 0;
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, walk_hop_kernel, kHopThreads, hop_smem);
+    if (indexed)
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, walk_hop_kernel<true>, kHopThreads, hop_smem);
+    else
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, walk_hop_kernel<false>, kHopThreads, hop_smem);
     const uint32_t hop_grid = (uint32_t)ctx->num_sms * (uint32_t)std::max(1, hop_blocks_per_sm);
     HopArgs g;
     g.cap = hop_cap;
     g.seg = seg;
     g.S = S;
     g.H = t.num_hosts;
-    g.tab_offs = t.d_tab_offs;
-    g.rule_a = t.d_rule_a;
-    g.rule_b = t.d_rule_b;
-    g.max_pad = t.max_rules_padded;
+    g.blob = t.d_blob;
+    g.blob_offs = t.d_blob_offs;
     g.region = t.d_region;
     g.port_offs = t.d_port_offs;
     g.port_peer = t.d_port_peer;
@@ -609,7 +1018,10 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
         g.next_list = nxt;
         g.next_count = counts + h + 1;
         pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
-        walk_hop_kernel<<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+        if (indexed)
+            walk_hop_kernel<true><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+        else
+            walk_hop_kernel<false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         pv_prof_stop(ctx, st, pr, 1);
     }
     return pv_check_launch(ctx, "probe walk kernels");

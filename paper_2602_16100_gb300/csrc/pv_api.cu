@@ -75,9 +75,8 @@ void pv_free_cluster(pv_cluster_state &c) {
 }
 
 void pv_free_tables(pv_table_state &t) {
-    pv_free_ptr(t.d_tab_offs);
-    pv_free_ptr(t.d_rule_a);
-    pv_free_ptr(t.d_rule_b);
+    pv_free_ptr(t.d_blob);
+    pv_free_ptr(t.d_blob_offs);
     pv_free_ptr(t.d_region);
     pv_free_ptr(t.d_port_offs);
     pv_free_ptr(t.d_port_peer);
@@ -218,7 +217,7 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         ctx->opt_selector = (int)value;
         return PV_OK;
     case PV_OPT_WALK_KERNEL:
-        if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "walk kernel must be 0 or 1");
+        if (value < 0 || value > 2) return pv_fail(ctx, PV_EINVAL, "walk kernel must be 0, 1 or 2");
         ctx->opt_walk = (int)value;
         return PV_OK;
     default:
@@ -231,6 +230,8 @@ extern "C" int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value) {
     switch (stat) {
     case PV_STAT_SELECTOR_ROWS_BUILT: *value = ctx->cl.rows_built ? 1 : 0; return PV_OK;
     case PV_STAT_SCRATCH_BYTES: *value = (int64_t)ctx->scratch_bytes; return PV_OK;
+    case PV_STAT_WALK_INDEX_FITS: *value = ctx->tb.index_fits ? 1 : 0; return PV_OK;
+    case PV_STAT_WALK_INDEX_BYTES: *value = (int64_t)ctx->tb.max_blob_bytes; return PV_OK;
     default: return PV_EINVAL;
     }
 }

@@ -32,9 +32,13 @@ struct pv_table_state {
     bool loaded = false;
     uint32_t num_switches = 0, num_hosts = 0;
     uint32_t max_rules_padded = 0;    // largest per-switch table, in rules (multiple of 32)
-    uint32_t *d_tab_offs = nullptr;   // [S + 1] start of each switch's compiled table (multiple of 32)
-    uint4 *d_rule_a = nullptr;        // [total padded] {src & m, m_src, dst & m, m_dst}
-    uint2 *d_rule_b = nullptr;        // [total padded] {lo | hi << 16, inval | inmask << 8 | action << 16}
+    // One blob per switch (16-byte aligned): header, compiled rules in first-
+    // match order, then the first-match index (see k_walk.cu).
+    uint8_t *d_blob = nullptr;
+    uint64_t *d_blob_offs = nullptr;  // [S + 1] byte offsets
+    uint32_t max_blob_bytes = 0;      // largest blob (indexed kernel stages it whole)
+    uint32_t max_linear_bytes = 0;    // largest header + rules prefix (linear-scan kernel)
+    bool index_fits = false;          // every blob fits shared memory
     uint8_t *d_region = nullptr;      // [S]
     uint32_t *d_port_offs = nullptr;  // [S + 1]
     int32_t *d_port_peer = nullptr;   // [ports]

@@ -22,7 +22,9 @@ def to_device(a: np.ndarray, device) -> torch.Tensor:
 
 
 def empty_device(nbytes: int, device) -> torch.Tensor:
-    return torch.empty(max(16, int(nbytes)), dtype=torch.uint8, device=device)
+    """Uninitialised device byte buffer (torch allocations are 512-byte
+    aligned, which the 16-byte alignment rules of the C ABI need)."""
+    return torch.empty(max(1, int(nbytes)), dtype=torch.uint8, device=device)
 
 
 def to_numpy(t: torch.Tensor, dtype, shape=None) -> np.ndarray:

@@ -16,10 +16,17 @@ from netbuild import ip, make_net, probe, rule
 pytestmark = pytest.mark.gpu
 
 
-def _gpu_walk(v, net, probes, cap):
+KERNELS = [1, 2]   # linear first-match scan, indexed first match
+
+
+def _gpu_walk(v, net, probes, cap, kernel=0):
     v.load_network(net)
-    out = v.verify_probes(to_device(probes, v.device), len(probes), cap)
-    v.sync()
+    v.set_option(B.PV_OPT_WALK_KERNEL, kernel)
+    try:
+        out = v.verify_probes(to_device(probes, v.device), len(probes), cap)
+        v.sync()
+    finally:
+        v.set_option(B.PV_OPT_WALK_KERNEL, 0)
     return to_numpy(out, W.RESULT_DTYPE)
 
 
@@ -28,7 +35,8 @@ def _same(a, b):
         (a["last_switch"] == b["last_switch"]).all()
 
 
-def test_worked_cases(validator):
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_worked_cases(validator, kernel):
     A, Bh, C = ip(10, 0, 0, 1), ip(10, 0, 2, 1), ip(10, 0, 2, 2)
     rules = [[rule(100, Bh, 24, 1), rule(100, A, 32, 0)],
              [rule(100, Bh, 24, 1), rule(100, A, 24, 0), rule(150, Bh, 32, W.DROP, lo=7, hi=7)],
@@ -38,34 +46,37 @@ def test_worked_cases(validator):
                          probe(0, A, C, 3), probe(W.NO_HOST, A, Bh, 3), probe(7, A, Bh, 3),
                          probe(0, A, ip(99, 0, 0, 0), 3)])
     for cap in (1, 2, 3, 16, 255):
-        g = _gpu_walk(validator, net, pr, cap)
+        g = _gpu_walk(validator, net, pr, cap, kernel)
         o = oracle.verify_probes(net, pr, cap)
         assert _same(g, o), cap
     g = _gpu_walk(validator, net, pr, 16)
     assert g["status"][0] == W.ST_VIOLATION and g["last_switch"][0] == 1
 
 
-def test_tiny(validator):
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_tiny(validator, kernel):
     d = W.tiny()
-    g = _gpu_walk(validator, d["network"], d["probes"].probes, d["probes"].hop_cap)
+    g = _gpu_walk(validator, d["network"], d["probes"].probes, d["probes"].hop_cap, kernel)
     o = oracle.verify_probes(d["network"], d["probes"].probes, d["probes"].hop_cap)
     assert _same(g, o)
 
 
 @pytest.mark.parametrize("k,rules,cap,mask_all", [(4, 100, 8, False), (4, 100, 8, True), (8, 600, 32, False),
                                                   (8, 600, 5, True), (6, 2000, 255, True)])
-def test_fat_trees(validator, k, rules, cap, mask_all):
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_fat_trees(validator, k, rules, cap, mask_all, kernel):
     d = W.fat_tree(seed=k * 31 + rules, k=k, rules_per_switch=rules, num_probes=20011, hop_cap=cap)
     pr = d["probes"].probes.copy()
     if mask_all:
         pr["allowed_mask"] = 0xFFFFFFFF
-    g = _gpu_walk(validator, d["network"], pr, cap)
+    g = _gpu_walk(validator, d["network"], pr, cap, kernel)
     o = oracle.verify_probes(d["network"], pr, cap)
     assert _same(g, o)
     assert len(np.unique(o["status"])) >= 3
 
 
-def test_random_graph_network(validator):
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_random_graph_network(validator, kernel):
     e = W.end_to_end(seed=4, num_switches=40, num_intents=20, probes_per_intent=500, rules_per_switch=150)
     pr = e.probes.probes.copy()
     H = e.network.num_hosts
@@ -73,7 +84,7 @@ def test_random_graph_network(validator):
     ok = pr["src_host"] < H
     pr["src_ip"][ok] = e.network.host_ip[pr["src_host"][ok]]
     for cap in (1, 32):
-        g = _gpu_walk(validator, e.network, pr, cap)
+        g = _gpu_walk(validator, e.network, pr, cap, kernel)
         o = oracle.verify_probes(e.network, pr, cap)
         assert _same(g, o)
 
@@ -102,12 +113,81 @@ def test_empty_and_invalid_calls(validator):
                               net.port_peer, net.num_hosts, net.host_switch, net.host_port, net.host_ip)
 
 
-def test_flow_verification_full_size_sampled(validator):
+def _index_stress_network(seed, S=6, rules=700):
+    """Ring of switches whose tables interleave destination-only runs with
+    general rules: nested prefixes (/0 to /32) over a few addresses, priority
+    ties, port ranges straddling the 1024-port bucket edges, in_port rules
+    with full port ranges."""
+    st = W.Stream(seed, "index-stress")
+    hosts_per = 2
+    H = S * hosts_per
+    host_ip = np.array([ip(10, s, h, 1) for s in range(S) for h in range(hosts_per)], np.uint32)
+    nports = [hosts_per + 2] * S
+    links = [(s, hosts_per, (s + 1) % S, hosts_per + 1) for s in range(S)]
+    hosts = [(s, h, int(host_ip[s * hosts_per + h])) for s in range(S) for h in range(hosts_per)]
+    tables = []
+    for s in range(S):
+        n = rules
+        r = np.zeros(n, W.RULE_DTYPE)
+        dst_only = st.floats(n) < 0.6
+        # priorities in runs so destination-only rules form contiguous segments
+        r["priority"] = (np.arange(n) // st.ints(1, 40, 1)[0]) % 9 + st.ints(0, 1, n)
+        base = host_ip[st.ints(0, H - 1, n)].astype(np.uint64)
+        base ^= (st.u64(n) & np.uint64(0x00FF00FF)) * (st.floats(n) < 0.3)
+        lens = np.array([0, 8, 12, 16, 20, 24, 28, 31, 32])[st.ints(0, 8, n)]
+        m = np.where(lens == 0, 0, (0xFFFFFFFF << (32 - lens)) & 0xFFFFFFFF).astype(np.uint64)
+        r["dst_ip"] = (base & m).astype(np.uint32)
+        r["dst_len"] = lens
+        edge = st.ints(1, 63, n) * 1024
+        lo = np.clip(edge - st.ints(0, 3, n), 0, 65535)
+        hi = np.clip(edge + st.ints(-1, 900, n), 0, 65535)
+        r["dport_lo"] = np.where(dst_only, 0, np.minimum(lo, hi))
+        r["dport_hi"] = np.where(dst_only, 65535, np.maximum(lo, hi))
+        src_rule = (~dst_only) & (st.floats(n) < 0.5)
+        r["src_len"] = np.where(src_rule, st.ints(1, 32, n), 0)
+        r["src_ip"] = np.where(src_rule, host_ip[st.ints(0, H - 1, n)], 0)
+        inp = (~dst_only) & (st.floats(n) < 0.3)
+        r["in_port"] = np.where(inp, st.ints(0, nports[s] - 1, n), W.ANY_PORT)
+        full = (~dst_only) & (st.floats(n) < 0.2)                 # general rule with full port range
+        r["dport_lo"] = np.where(full, 0, r["dport_lo"])
+        r["dport_hi"] = np.where(full, 65535, r["dport_hi"])
+        act = st.ints(0, nports[s], n)
+        r["action"] = np.where(act == nports[s], W.DROP, act)
+        tables.append([r[i:i + 1] for i in range(n)])
+    return make_net(nports, links, hosts, st.ints(0, 3, S).astype(np.uint8), tables), host_ip
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_index_stress_tables(validator, seed):
+    net, host_ip = _index_stress_network(seed)
+    st = W.Stream(seed, "index-stress-probes")
+    M = 20000
+    pr = np.zeros(M, W.PROBE_DTYPE)
+    src = st.ints(0, net.num_hosts - 1, M)
+    pr["src_host"] = src
+    pr["src_ip"] = np.where(st.floats(M) < 0.8, host_ip[src], st.u64(M) & np.uint64(0xFFFFFFFF))
+    pr["dst_ip"] = np.where(st.floats(M) < 0.7, host_ip[st.ints(0, net.num_hosts - 1, M)],
+                            st.u64(M) & np.uint64(0xFFFFFFFF))
+    edges = st.ints(0, 64, M) * 1024 + st.ints(-2, 2, M)
+    pr["dport"] = np.where(st.floats(M) < 0.5, np.clip(edges, 0, 65535), st.ints(0, 65535, M))
+    pr["allowed_mask"] = 0xF
+    validator.load_network(net)
+    assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_INDEX_FITS) == 1
+    o = oracle.verify_probes(net, pr, 24)
+    for kernel in KERNELS:
+        g = _gpu_walk(validator, net, pr, 24, kernel)
+        assert _same(g, o), kernel
+    # every first match along the way also agrees hop by hop with the oracle's
+    assert len(np.unique(o["status"])) >= 3
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_flow_verification_full_size_sampled(validator, kernel):
     """The full flow-verification workload in the benchmark's launch
     configuration; the oracle walks a sample of probes."""
     d = W.fat_tree()
     net, P = d["network"], d["probes"]
-    g = _gpu_walk(validator, net, P.probes, P.hop_cap)
+    g = _gpu_walk(validator, net, P.probes, P.hop_cap, kernel)
     idx = sample(len(P.probes), 20000, seed=2)
     o = oracle.verify_probes(net, P.probes, P.hop_cap, idx=idx)
     assert _same(g[idx], o)
