@@ -277,11 +277,14 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  *   staged table, 2 = indexed first match (per-dport-bucket candidate lists
  *   and destination-interval maps built by pv_load_flow_tables; needs every
  *   switch's index to fit shared memory).
+ * PV_OPT_WALK_LANE_MAX: with kernel 2, a batch of 32 probes is resolved one
+ *   probe per lane when its longest candidate list has at most this many
+ *   items (default 96), else one probe at a time by the whole warp.
  * pv_get_stat: PV_STAT_SELECTOR_ROWS_BUILT (1 if value rows exist),
  *   PV_STAT_SCRATCH_BYTES, PV_STAT_WALK_INDEX_FITS (1 if kernel 2 is
  *   usable), PV_STAT_WALK_INDEX_BYTES (largest per-switch table + index).
  * ------------------------------------------------------------------------- */
-enum { PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2 };
+enum { PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3 };
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,
     PV_STAT_WALK_INDEX_BYTES = 4

@@ -32,7 +32,7 @@
 
 namespace {
 
-constexpr int kHopThreads = 512;
+constexpr int kHopThreads = 256;
 constexpr int kHopWarps = kHopThreads / 32;
 constexpr int kGridThreads = 256;
 constexpr uint32_t kSmemHistMax = 12288;     // switches for shared-memory histograms
@@ -412,41 +412,34 @@ __global__ void __launch_bounds__(1024) index_build_kernel(const uint32_t *__res
 // ---------------------------------------------------------------------------
 // walk kernels
 // ---------------------------------------------------------------------------
-// Every thread of the block calls this; threads with want append one slot of
-// the shared output list.  Returns the slot (undefined when !want).
-__device__ __forceinline__ uint32_t block_append(bool want, uint32_t *count, uint32_t *s_tmp) {
-    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+// Live lists are written in per-block slices: block b of the producing kernel
+// owns list[desc[b].x .. desc[b].x + desc[b].y); consumers take one slice
+// per block.  Warps reserve slots of their block's slice with shared-memory
+// atomics, so producing a list needs neither a global counter nor barriers.
+// Entry: x = probe id, y = location (switch << 8 | in_port).
+__device__ __forceinline__ uint32_t warp_reserve(bool want, uint32_t *s_count) {
+    const uint32_t lane = threadIdx.x & 31;
     const uint32_t m = __ballot_sync(PV_FULL_MASK, want);
-    const uint32_t rank = __popc(m & ((1u << lane) - 1u));
-    if (lane == 0) s_tmp[warp] = __popc(m);
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        uint32_t run = 0;
-        for (uint32_t w = 0; w < nwarps; ++w) {
-            uint32_t c = s_tmp[w];
-            s_tmp[w] = run;
-            run += c;
-        }
-        s_tmp[32] = run ? atomicAdd(count, run) : 0;
-    }
-    __syncthreads();
-    const uint32_t pos = s_tmp[32] + s_tmp[warp] + rank;
-    __syncthreads();
-    return pos;
+    uint32_t base = 0;
+    if (lane == 0 && m) base = atomicAdd(s_count, (uint32_t)__popc(m));
+    base = __shfl_sync(PV_FULL_MASK, base, 0);
+    return base + __popc(m & ((1u << lane) - 1u));
 }
 
-// Live list entry: x = probe id, y = location (switch << 8 | in_port).
 __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
     uint32_t M, const pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
     const uint16_t *__restrict__ host_port, pv_result *__restrict__ out, uint2 *__restrict__ list,
-    uint32_t *__restrict__ count) {
-    __shared__ uint32_t s_tmp[40];
-    const uint32_t stride = gridDim.x * kGridThreads;
-    for (uint32_t base = blockIdx.x * kGridThreads; base < M; base += stride) {
+    uint2 *__restrict__ desc) {
+    __shared__ uint32_t s_count;
+    const uint32_t c0 = (uint32_t)(((uint64_t)M * blockIdx.x) / gridDim.x);
+    const uint32_t c1 = (uint32_t)(((uint64_t)M * (blockIdx.x + 1)) / gridDim.x);
+    if (threadIdx.x == 0) s_count = 0;
+    __syncthreads();
+    for (uint32_t base = c0; base < c1; base += kGridThreads) {
         const uint32_t i = base + threadIdx.x;
         bool live = false;
         uint32_t loc = 0;
-        if (i < M) {
+        if (i < c1) {
             const uint32_t h = probes[i].src_host;
             if (h < H) {
                 live = true;
@@ -459,22 +452,26 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
                 out[i] = r;
             }
         }
-        const uint32_t pos = block_append(live, count, s_tmp);
-        if (live) list[pos] = make_uint2(i, loc);
+        const uint32_t slot = warp_reserve(live, &s_count);
+        if (live) list[c0 + slot] = make_uint2(i, loc);
     }
+    __syncthreads();
+    if (threadIdx.x == 0) desc[blockIdx.x] = make_uint2(c0, s_count);
 }
 
+// One block per list slice: per-switch histogram of the live probes.
 __global__ void __launch_bounds__(kGridThreads) walk_hist_kernel(const uint2 *__restrict__ list,
-                                                                 const uint32_t *__restrict__ count_ptr,
-                                                                 uint32_t S, uint32_t *__restrict__ hist) {
+                                                                 const uint2 *__restrict__ desc, uint32_t S,
+                                                                 uint32_t *__restrict__ hist) {
     extern __shared__ uint32_t s_hist[];
-    const uint32_t n = *count_ptr;
+    const uint2 d = desc[blockIdx.x];
+    if (d.y == 0) return;
     const bool use_smem = S <= kSmemHistMax;
     if (use_smem) {
         for (uint32_t j = threadIdx.x; j < S; j += kGridThreads) s_hist[j] = 0;
         __syncthreads();
     }
-    for (uint32_t i = blockIdx.x * kGridThreads + threadIdx.x; i < n; i += gridDim.x * kGridThreads) {
+    for (uint32_t i = d.x + threadIdx.x; i < d.x + d.y; i += kGridThreads) {
         const uint32_t s = list[i].y >> 8;
         if (use_smem) atomicAdd(&s_hist[s], 1u);
         else atomicAdd(&hist[s], 1u);
@@ -527,17 +524,16 @@ __global__ void __launch_bounds__(1024) walk_scan_kernel(uint32_t S, uint32_t *_
     if (t == 0) seg[S] = s_carry;
 }
 
-// Block-aggregated counting-sort scatter: each block reserves, per switch,
-// one contiguous run of its items with a single atomicAdd.
+// One block per list slice: block-aggregated counting-sort scatter (one
+// atomicAdd per (block, switch) reserves a contiguous run).
 __global__ void __launch_bounds__(kGridThreads) walk_scatter_kernel(const uint2 *__restrict__ list,
-                                                                    const uint32_t *__restrict__ count_ptr,
-                                                                    uint32_t S, uint32_t *__restrict__ cursor,
+                                                                    const uint2 *__restrict__ desc, uint32_t S,
+                                                                    uint32_t *__restrict__ cursor,
                                                                     uint2 *__restrict__ sorted) {
     extern __shared__ uint32_t s_cnt[];   // [S] counts, then [S] bases
-    const uint32_t n = *count_ptr;
-    const uint32_t per = (n + gridDim.x - 1) / gridDim.x;
-    const uint32_t b0 = min(n, blockIdx.x * per), b1 = min(n, b0 + per);
-    if (b0 >= b1) return;
+    const uint2 d = desc[blockIdx.x];
+    if (d.y == 0) return;
+    const uint32_t b0 = d.x, b1 = d.x + d.y;
     if (S > kSmemHistMax) {
         for (uint32_t i = b0 + threadIdx.x; i < b1; i += kGridThreads) {
             const uint2 e = list[i];
@@ -565,7 +561,6 @@ __global__ void __launch_bounds__(kGridThreads) walk_scatter_kernel(const uint2 
 
 struct HopArgs {
     const uint2 *sorted;
-    const uint32_t *counts;
     uint32_t hop, cap;
     const uint32_t *seg;
     uint32_t S, H;
@@ -578,8 +573,9 @@ struct HopArgs {
     const pv_probe *probes;
     pv_result *out;
     uint2 *next_list;
-    uint32_t *next_count;
+    uint2 *next_desc;
     int32_t *status;
+    uint32_t lane_max;   // longest candidate list handled one probe per lane
 };
 
 // Linear first match: 32 consecutive rules per warp step.
@@ -665,17 +661,88 @@ __device__ __forceinline__ uint32_t first_match_indexed(const uint8_t *sm, const
     return 0u;
 }
 
+// Scalar first match for one probe per lane: the bucket's candidate list in
+// order, segments by binary search over their interval starts.
+__device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const BlobLayout &L, uint32_t src,
+                                                     uint32_t dst, uint32_t dport, uint32_t in_port) {
+    const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
+    const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
+    const uint32_t *boff = reinterpret_cast<const uint32_t *>(sm + L.boff);
+    const uint16_t *items = reinterpret_cast<const uint16_t *>(sm + L.items);
+    const uint2 *segs = reinterpret_cast<const uint2 *>(sm + L.segs);
+    const uint32_t *bnd = reinterpret_cast<const uint32_t *>(sm + L.bnd);
+    const uint32_t *win = reinterpret_cast<const uint32_t *>(sm + L.win);
+    const uint32_t k = dport >> kBucketShift;
+    const uint32_t i1 = boff[k + 1];
+    for (uint32_t i = boff[k]; i < i1; ++i) {
+        const uint32_t it = items[i];
+        if (it & kSegItem) {
+            const uint2 sd = segs[it & 0x7FFFu];
+            const uint32_t *b = bnd + sd.x;
+            uint32_t lo = 0, len = sd.y;   // b[0] = 0 <= dst; answer in [lo, lo + len)
+            while (len > 1) {
+                const uint32_t half = len >> 1;
+                lo = b[lo + half] <= dst ? lo + half : lo;
+                len -= half;
+            }
+            const uint32_t w = win[sd.x + lo];
+            if (w & kWinFound) return w;
+        } else {
+            const uint4 a = sA[it];
+            const uint2 bb = sB[it];
+            const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
+            if (diff == 0 && dport >= (bb.x & 0xFFFFu) && dport <= (bb.x >> 16)) return kWinFound | (bb.y >> 16);
+        }
+    }
+    return 0u;
+}
+
+// Outcome of one hop at a permitted (or forbidden) switch given the first
+// match fm (kWinFound | action, or 0): a terminal status, or 0xFF (alive)
+// with the next location.
+__device__ __forceinline__ void hop_outcome(const HopArgs &g, bool allowed, uint32_t fm, uint32_t dst, uint32_t pbase,
+                                            uint32_t nports, uint32_t *status, uint32_t *next) {
+    *next = 0;
+    if (!allowed) {
+        *status = PV_VIOLATION;
+        return;
+    }
+    const uint32_t act = fm & 0xFFFFu;
+    if (!(fm & kWinFound) || act == PV_DROP || act >= nports) {
+        *status = PV_DROPPED;
+        return;
+    }
+    const int32_t peer = g.port_peer[pbase + act];
+    if (peer < 0) {
+        *status = PV_DROPPED;
+    } else if (peer & PV_PEER_HOST) {
+        const uint32_t q = (uint32_t)(peer & ~PV_PEER_HOST);
+        *status = (q < g.H && g.host_ip[q] == dst) ? PV_COMPLIANT : PV_MISDELIVERED;
+    } else if (g.hop + 1 >= g.cap) {
+        *status = PV_LOOP;
+    } else {
+        *status = 0xFFu;
+        *next = (uint32_t)peer;
+    }
+}
+
 template <bool kIndexed>
-__global__ void __launch_bounds__(kHopThreads) walk_hop_kernel(HopArgs g) {
+__global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
     __shared__ uint64_t s_bar;
-    __shared__ uint32_t s_tmp[40];
+    __shared__ uint32_t s_count;
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const uint32_t n = g.counts[g.hop];
+    const uint32_t n = g.seg[g.S];   // live probes this hop
     const uint32_t r0 = (uint32_t)(((uint64_t)n * blockIdx.x) / gridDim.x);
     const uint32_t r1 = (uint32_t)(((uint64_t)n * (blockIdx.x + 1)) / gridDim.x);
-    if (r0 >= r1) return;
-    if (threadIdx.x == 0) mbar_init(&s_bar, 1);
+    if (r0 >= r1) {
+        if (threadIdx.x == 0) g.next_desc[blockIdx.x] = make_uint2(r0, 0);
+        return;
+    }
+    if (threadIdx.x == 0) {
+        mbar_init(&s_bar, 1);
+        s_count = 0;
+    }
     __syncthreads();
     uint32_t parity = 0;
     uint32_t pos = r0;
@@ -701,66 +768,82 @@ __global__ void __launch_bounds__(kHopThreads) walk_hop_kernel(HopArgs g) {
         }
         const bool ok = mbar_wait_bounded(&s_bar, parity);
         if (__syncthreads_or(!ok)) {
-            if (threadIdx.x == 0) pv_device_error(g.status, PV_ETIMEOUT);
+            if (threadIdx.x == 0) {
+                pv_device_error(g.status, PV_ETIMEOUT);
+                g.next_desc[blockIdx.x] = make_uint2(r0, 0);
+            }
             mbar_wait_bounded(&s_bar, parity);   // let copies in flight land
             return;
         }
         parity ^= 1u;
         const uint32_t reg = g.region[s];
         const uint32_t pbase = g.port_offs[s], nports = g.port_offs[s + 1] - pbase;
-        for (uint32_t rb = pos; rb < seg_end; rb += 32 * kHopWarps) {
-            const uint32_t wb = rb + warp * 32;
-            const uint32_t cnt = wb < seg_end ? min(32u, seg_end - wb) : 0u;
-            bool my_live = false;
-            uint2 my_entry = make_uint2(0, 0);
-            for (uint32_t j = 0; j < cnt; ++j) {
-                const uint2 e = g.sorted[wb + j];
-                const uint32_t pid = e.x, in_port = e.y & 0xFFu;
+        for (uint32_t wb = pos + warp * 32; wb < seg_end; wb += 32 * kHopWarps) {
+            const uint32_t cnt = min(32u, seg_end - wb);
+            // lane j fetches probe j of this warp's batch; records are then
+            // broadcast one at a time with shuffles
+            uint2 e = make_uint2(0, 0);
+            uint4 pr = make_uint4(0, 0, 0, 0);
+            if (lane < cnt) {
+                e = g.sorted[wb + lane];
                 // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
-                const uint4 pr = __ldg(reinterpret_cast<const uint4 *>(g.probes) + pid);
-                uint32_t status = 0xFFu;   // alive
-                uint32_t next = 0;
-                if (reg >= 32 || !((pr.w >> reg) & 1u)) {
-                    status = PV_VIOLATION;
-                } else {
-                    const uint32_t src = pr.x, dst = pr.y, dport = pr.z & 0xFFFFu;
-                    const uint32_t fm = kIndexed ? first_match_indexed(s_raw, hdr, lane, src, dst, dport, in_port)
-                                                 : first_match_linear(s_raw, hdr.x, lane, src, dst, dport, in_port);
-                    const uint32_t act = fm & 0xFFFFu;
-                    if (!(fm & kWinFound) || act == PV_DROP || act >= nports) {
-                        status = PV_DROPPED;
-                    } else {
-                        const int32_t peer = g.port_peer[pbase + act];
-                        if (peer < 0) {
-                            status = PV_DROPPED;
-                        } else if (peer & PV_PEER_HOST) {
-                            const uint32_t q = (uint32_t)(peer & ~PV_PEER_HOST);
-                            status = (q < g.H && g.host_ip[q] == dst) ? PV_COMPLIANT : PV_MISDELIVERED;
-                        } else if (g.hop + 1 >= g.cap) {
-                            status = PV_LOOP;
-                        } else {
-                            next = (uint32_t)peer;
-                        }
-                    }
+                pr = __ldg(reinterpret_cast<const uint4 *>(g.probes) + e.x);
+            }
+            uint32_t my_status = 0xFFu, my_next = 0;
+            // lane-per-probe when every candidate list of the batch is short
+            bool lane_mode = false;
+            if (kIndexed) {
+                const uint32_t *boff = reinterpret_cast<const uint32_t *>(s_raw + L.boff);
+                uint32_t len = 0;
+                if (lane < cnt) {
+                    const uint32_t k = (pr.z & 0xFFFFu) >> kBucketShift;
+                    len = boff[k + 1] - boff[k];
                 }
-                if (status != 0xFFu) {
-                    if (lane == 0) {
-                        pv_result r;
-                        r.status = (uint8_t)status;
-                        r.hops = (uint8_t)(g.hop + 1);
-                        r.last_switch = (uint16_t)s;
-                        g.out[pid] = r;
+                lane_mode = __reduce_max_sync(PV_FULL_MASK, len) <= g.lane_max;
+            }
+            if (lane_mode) {
+                if (lane < cnt) {
+                    const uint32_t mask = pr.w;
+                    uint32_t fm = 0;
+                    const bool allowed = reg < 32 && ((mask >> reg) & 1u);
+                    if (allowed) fm = first_match_lane(s_raw, L, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu);
+                    hop_outcome(g, allowed, fm, pr.y, pbase, nports, &my_status, &my_next);
+                }
+            } else {
+                for (uint32_t j = 0; j < cnt; ++j) {
+                    const uint32_t in_port = __shfl_sync(PV_FULL_MASK, e.y, j) & 0xFFu;
+                    const uint32_t src = __shfl_sync(PV_FULL_MASK, pr.x, j);
+                    const uint32_t dst = __shfl_sync(PV_FULL_MASK, pr.y, j);
+                    const uint32_t dport = __shfl_sync(PV_FULL_MASK, pr.z, j) & 0xFFFFu;
+                    const uint32_t mask = __shfl_sync(PV_FULL_MASK, pr.w, j);
+                    const bool allowed = reg < 32 && ((mask >> reg) & 1u);
+                    uint32_t fm = 0;
+                    if (allowed)
+                        fm = kIndexed ? first_match_indexed(s_raw, hdr, lane, src, dst, dport, in_port)
+                                      : first_match_linear(s_raw, hdr.x, lane, src, dst, dport, in_port);
+                    uint32_t status, next;
+                    hop_outcome(g, allowed, fm, dst, pbase, nports, &status, &next);
+                    if (lane == j) {
+                        my_status = status;
+                        my_next = next;
                     }
-                } else if (lane == j) {
-                    my_live = true;
-                    my_entry = make_uint2(pid, next);
                 }
             }
-            const uint32_t slot = block_append(my_live, g.next_count, s_tmp);
-            if (my_live) g.next_list[slot] = my_entry;
+            if (lane < cnt && my_status != 0xFFu) {
+                pv_result r;
+                r.status = (uint8_t)my_status;
+                r.hops = (uint8_t)(g.hop + 1);
+                r.last_switch = (uint16_t)s;
+                g.out[e.x] = r;
+            }
+            const bool live = lane < cnt && my_status == 0xFFu;
+            const uint32_t slot = warp_reserve(live, &s_count);
+            if (live) g.next_list[r0 + slot] = make_uint2(e.x, my_next);
         }
         pos = seg_end;
     }
+    __syncthreads();
+    if (threadIdx.x == 0) g.next_desc[blockIdx.x] = make_uint2(r0, s_count);
 }
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -957,27 +1040,6 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     if (!d_probes || !d_out) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: NULL device pointer");
     if (((uintptr_t)d_probes & 15) != 0) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: d_probes must be 16-byte aligned");
     const uint32_t S = t.num_switches;
-    const size_t o_a = 0, o_b = align256((size_t)M * 8), o_sorted = o_b + align256((size_t)M * 8);
-    const size_t o_hist = o_sorted + align256((size_t)M * 8);
-    const size_t o_seg = o_hist + align256((size_t)S * 4);
-    const size_t o_cur = o_seg + align256((size_t)(S + 1) * 4);
-    const size_t o_cnt = o_cur + align256((size_t)S * 4);
-    const size_t total = o_cnt + align256((size_t)(hop_cap + 2) * 4);
-    uint8_t *base = (uint8_t *)pv_scratch(ctx, total);
-    if (!base) return PV_ENOMEM;
-    uint2 *listA = (uint2 *)(base + o_a), *listB = (uint2 *)(base + o_b), *sorted = (uint2 *)(base + o_sorted);
-    uint32_t *hist = (uint32_t *)(base + o_hist), *seg = (uint32_t *)(base + o_seg);
-    uint32_t *cursor = (uint32_t *)(base + o_cur), *counts = (uint32_t *)(base + o_cnt);
-    cudaStream_t st = (cudaStream_t)stream;
-    PV_TRY_CUDA(ctx, cudaMemsetAsync(counts, 0, (size_t)(hop_cap + 2) * 4, st), "counts clear");
-    PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
-    const uint32_t grid = (uint32_t)ctx->num_sms * 8;
-    int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
-    walk_init_kernel<<<grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port, d_out,
-                                                    listA, counts);
-    pv_prof_stop(ctx, st, pr, 1);
-    const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
-    const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
     int which = ctx->opt_walk;
     if (which == 0) which = t.index_fits ? 2 : 1;
     if (which == 2 && !t.index_fits)
@@ -990,6 +1052,28 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     else
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, walk_hop_kernel<false>, kHopThreads, hop_smem);
     const uint32_t hop_grid = (uint32_t)ctx->num_sms * (uint32_t)std::max(1, hop_blocks_per_sm);
+    const uint32_t init_grid = (uint32_t)ctx->num_sms * 8;
+    const uint32_t max_desc = std::max(hop_grid, init_grid);
+    const size_t o_a = 0, o_b = align256((size_t)M * 8), o_sorted = o_b + align256((size_t)M * 8);
+    const size_t o_hist = o_sorted + align256((size_t)M * 8);
+    const size_t o_seg = o_hist + align256((size_t)S * 4);
+    const size_t o_cur = o_seg + align256((size_t)(S + 1) * 4);
+    const size_t o_desc = o_cur + align256((size_t)S * 4);
+    const size_t total = o_desc + 2 * align256((size_t)max_desc * 8);
+    uint8_t *base = (uint8_t *)pv_scratch(ctx, total);
+    if (!base) return PV_ENOMEM;
+    uint2 *listA = (uint2 *)(base + o_a), *listB = (uint2 *)(base + o_b), *sorted = (uint2 *)(base + o_sorted);
+    uint32_t *hist = (uint32_t *)(base + o_hist), *seg = (uint32_t *)(base + o_seg);
+    uint32_t *cursor = (uint32_t *)(base + o_cur);
+    uint2 *descA = (uint2 *)(base + o_desc), *descB = (uint2 *)(base + o_desc + align256((size_t)max_desc * 8));
+    cudaStream_t st = (cudaStream_t)stream;
+    PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
+    int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
+    walk_init_kernel<<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port,
+                                                         d_out, listA, descA);
+    pv_prof_stop(ctx, st, pr, 1);
+    const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
+    const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
     HopArgs g;
     g.cap = hop_cap;
     g.seg = seg;
@@ -1004,25 +1088,29 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     g.probes = d_probes;
     g.out = d_out;
     g.status = ctx->d_status;
-    g.counts = counts;
+    g.lane_max = (uint32_t)ctx->opt_walk_lane_max;
+    uint32_t in_slices = init_grid;
     for (uint32_t h = 0; h < hop_cap; ++h) {
         uint2 *cur = (h & 1) ? listB : listA;
         uint2 *nxt = (h & 1) ? listA : listB;
+        uint2 *dcur = (h & 1) ? descB : descA;
+        uint2 *dnxt = (h & 1) ? descA : descB;
         pr = pv_prof_start(ctx, st, PV_K_WALK_REGROUP);
-        walk_hist_kernel<<<grid, kGridThreads, hist_smem, st>>>(cur, counts + h, S, hist);
+        walk_hist_kernel<<<in_slices, kGridThreads, hist_smem, st>>>(cur, dcur, S, hist);
         walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
-        walk_scatter_kernel<<<grid, kGridThreads, scat_smem, st>>>(cur, counts + h, S, cursor, sorted);
+        walk_scatter_kernel<<<in_slices, kGridThreads, scat_smem, st>>>(cur, dcur, S, cursor, sorted);
         pv_prof_stop(ctx, st, pr, 3);
         g.sorted = sorted;
         g.hop = h;
         g.next_list = nxt;
-        g.next_count = counts + h + 1;
+        g.next_desc = dnxt;
         pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
         if (indexed)
             walk_hop_kernel<true><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         else
             walk_hop_kernel<false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         pv_prof_stop(ctx, st, pr, 1);
+        in_slices = hop_grid;
     }
     return pv_check_launch(ctx, "probe walk kernels");
 }

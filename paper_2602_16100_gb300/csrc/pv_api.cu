@@ -220,6 +220,10 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         if (value < 0 || value > 2) return pv_fail(ctx, PV_EINVAL, "walk kernel must be 0, 1 or 2");
         ctx->opt_walk = (int)value;
         return PV_OK;
+    case PV_OPT_WALK_LANE_MAX:
+        if (value < 0 || value > 65535) return pv_fail(ctx, PV_EINVAL, "lane-mode list length must be 0..65535");
+        ctx->opt_walk_lane_max = (int)value;
+        return PV_OK;
     default:
         return pv_fail(ctx, PV_EINVAL, "unknown option %d", option);
     }

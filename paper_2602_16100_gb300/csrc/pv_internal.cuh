@@ -64,6 +64,7 @@ struct pv_ctx {
     std::string err;
     int32_t *d_status = nullptr;      // first device-detected error (0 = none)
     int opt_selector = 0, opt_walk = 0;
+    int opt_walk_lane_max = 96;
     void *scratch = nullptr;
     size_t scratch_bytes = 0;
     pv_cluster_state cl;

@@ -53,10 +53,14 @@ def test_worked_cases(validator, kernel):
     assert g["status"][0] == W.ST_VIOLATION and g["last_switch"][0] == 1
 
 
-@pytest.mark.parametrize("kernel", KERNELS)
-def test_tiny(validator, kernel):
+@pytest.mark.parametrize("kernel,lane_max", [(1, 96), (2, 0), (2, 96), (2, 65535)])
+def test_tiny(validator, kernel, lane_max):
     d = W.tiny()
-    g = _gpu_walk(validator, d["network"], d["probes"].probes, d["probes"].hop_cap, kernel)
+    validator.set_option(B.PV_OPT_WALK_LANE_MAX, lane_max)
+    try:
+        g = _gpu_walk(validator, d["network"], d["probes"].probes, d["probes"].hop_cap, kernel)
+    finally:
+        validator.set_option(B.PV_OPT_WALK_LANE_MAX, 96)
     o = oracle.verify_probes(d["network"], d["probes"].probes, d["probes"].hop_cap)
     assert _same(g, o)
 
@@ -177,6 +181,14 @@ def test_index_stress_tables(validator, seed):
     for kernel in KERNELS:
         g = _gpu_walk(validator, net, pr, 24, kernel)
         assert _same(g, o), kernel
+    # indexed kernel with every batch warp-cooperative, and every batch one probe per lane
+    for lane_max in (0, 65535):
+        validator.set_option(B.PV_OPT_WALK_LANE_MAX, lane_max)
+        try:
+            g = _gpu_walk(validator, net, pr, 24, 2)
+        finally:
+            validator.set_option(B.PV_OPT_WALK_LANE_MAX, 96)
+        assert _same(g, o), lane_max
     # every first match along the way also agrees hop by hop with the oracle's
     assert len(np.unique(o["status"])) >= 3
 
