@@ -426,10 +426,12 @@ __device__ __forceinline__ uint32_t warp_reserve(bool want, uint32_t *s_count) {
     return base + __popc(m & ((1u << lane) - 1u));
 }
 
+// First visit of every probe: NOSRC for an absent source host, VIOLATION at
+// the attachment switch when its region is not permitted, otherwise listed.
 __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
     uint32_t M, const pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
-    const uint16_t *__restrict__ host_port, pv_result *__restrict__ out, uint2 *__restrict__ list,
-    uint2 *__restrict__ desc) {
+    const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
+    uint2 *__restrict__ list, uint2 *__restrict__ desc) {
     __shared__ uint32_t s_count;
     const uint32_t c0 = (uint32_t)(((uint64_t)M * blockIdx.x) / gridDim.x);
     const uint32_t c1 = (uint32_t)(((uint64_t)M * (blockIdx.x + 1)) / gridDim.x);
@@ -440,12 +442,23 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
         bool live = false;
         uint32_t loc = 0;
         if (i < c1) {
-            const uint32_t h = probes[i].src_host;
+            // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
+            const uint4 pr = __ldg(reinterpret_cast<const uint4 *>(probes) + i);
+            const uint32_t h = pr.z >> 16;
+            pv_result r;
             if (h < H) {
-                live = true;
-                loc = ((uint32_t)host_switch[h] << 8) | host_port[h];
+                const uint32_t s = host_switch[h];
+                const uint32_t reg = region[s];
+                if (reg < 32 && ((pr.w >> reg) & 1u)) {
+                    live = true;
+                    loc = (s << 8) | host_port[h];
+                } else {
+                    r.status = PV_VIOLATION;
+                    r.hops = 1;
+                    r.last_switch = (uint16_t)s;
+                    out[i] = r;
+                }
             } else {
-                pv_result r;
                 r.status = PV_NOSRC;
                 r.hops = 0;
                 r.last_switch = 0xFFFF;
@@ -661,10 +674,13 @@ __device__ __forceinline__ uint32_t first_match_indexed(const uint8_t *sm, const
     return 0u;
 }
 
-// Scalar first match for one probe per lane: the bucket's candidate list in
-// order, segments by binary search over their interval starts.
-__device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const BlobLayout &L, uint32_t src,
-                                                     uint32_t dst, uint32_t dport, uint32_t in_port) {
+// Scalar first match, one probe per lane (called by all 32 lanes; inactive
+// lanes return 0): each lane walks its bucket's candidate list in order.
+// Plain rules are tested until a hit or a segment token; the warp then
+// reconverges and the lanes parked on a segment token run their interval
+// binary searches together (a segment miss resumes the walk after the token).
+__device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const BlobLayout &L, bool active,
+                                                     uint32_t src, uint32_t dst, uint32_t dport, uint32_t in_port) {
     const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
     const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
     const uint32_t *boff = reinterpret_cast<const uint32_t *>(sm + L.boff);
@@ -673,11 +689,33 @@ __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const Bl
     const uint32_t *bnd = reinterpret_cast<const uint32_t *>(sm + L.bnd);
     const uint32_t *win = reinterpret_cast<const uint32_t *>(sm + L.win);
     const uint32_t k = dport >> kBucketShift;
-    const uint32_t i1 = boff[k + 1];
-    for (uint32_t i = boff[k]; i < i1; ++i) {
-        const uint32_t it = items[i];
-        if (it & kSegItem) {
-            const uint2 sd = segs[it & 0x7FFFu];
+    uint32_t i = active ? boff[k] : 0u, i1 = active ? boff[k + 1] : 0u;
+    uint32_t result = 0;
+    bool done = !active;
+    while (__any_sync(PV_FULL_MASK, !done)) {
+        uint32_t seg = 0xFFFFFFFFu;
+        if (!done) {
+            for (; i < i1; ++i) {
+                const uint32_t it = items[i];
+                if (it & kSegItem) {
+                    seg = it & 0x7FFFu;
+                    break;
+                }
+                const uint4 a = sA[it];
+                const uint2 bb = sB[it];
+                const uint32_t diff =
+                    ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
+                if (diff == 0 && dport >= (bb.x & 0xFFFFu) && dport <= (bb.x >> 16)) {
+                    result = kWinFound | (bb.y >> 16);
+                    done = true;
+                    break;
+                }
+            }
+            if (!done && seg == 0xFFFFFFFFu) done = true;   // list exhausted: table miss
+        }
+        __syncwarp();
+        if (seg != 0xFFFFFFFFu) {
+            const uint2 sd = segs[seg];
             const uint32_t *b = bnd + sd.x;
             uint32_t lo = 0, len = sd.y;   // b[0] = 0 <= dst; answer in [lo, lo + len)
             while (len > 1) {
@@ -686,27 +724,29 @@ __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const Bl
                 len -= half;
             }
             const uint32_t w = win[sd.x + lo];
-            if (w & kWinFound) return w;
-        } else {
-            const uint4 a = sA[it];
-            const uint2 bb = sB[it];
-            const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
-            if (diff == 0 && dport >= (bb.x & 0xFFFFu) && dport <= (bb.x >> 16)) return kWinFound | (bb.y >> 16);
+            if (w & kWinFound) {
+                result = w;
+                done = true;
+            } else {
+                ++i;
+            }
         }
     }
-    return 0u;
+    return result;
 }
 
-// Outcome of one hop at a permitted (or forbidden) switch given the first
-// match fm (kWinFound | action, or 0): a terminal status, or 0xFF (alive)
-// with the next location.
-__device__ __forceinline__ void hop_outcome(const HopArgs &g, bool allowed, uint32_t fm, uint32_t dst, uint32_t pbase,
-                                            uint32_t nports, uint32_t *status, uint32_t *next) {
+// Outcome of one hop at a permitted switch given the first match fm
+// (kWinFound | action, or 0): a terminal status, kViolationNext (the next
+// switch is outside the probe's jurisdictions: the walk ends there, one hop
+// later), or kAlive with the next location.  Checking the next switch's
+// region here, when the probe is handed on, is the region check of the next
+// visit done early, so live lists only hold probes permitted where they are.
+constexpr uint32_t kAlive = 0xFFu;
+constexpr uint32_t kViolationNext = 0xFEu;
+
+__device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t fm, uint32_t dst, uint32_t mask,
+                                            uint32_t pbase, uint32_t nports, uint32_t *status, uint32_t *next) {
     *next = 0;
-    if (!allowed) {
-        *status = PV_VIOLATION;
-        return;
-    }
     const uint32_t act = fm & 0xFFFFu;
     if (!(fm & kWinFound) || act == PV_DROP || act >= nports) {
         *status = PV_DROPPED;
@@ -721,7 +761,8 @@ __device__ __forceinline__ void hop_outcome(const HopArgs &g, bool allowed, uint
     } else if (g.hop + 1 >= g.cap) {
         *status = PV_LOOP;
     } else {
-        *status = 0xFFu;
+        const uint32_t r2 = g.region[(uint32_t)peer >> 8];
+        *status = (r2 < 32 && ((mask >> r2) & 1u)) ? kAlive : kViolationNext;
         *next = (uint32_t)peer;
     }
 }
@@ -776,7 +817,6 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             return;
         }
         parity ^= 1u;
-        const uint32_t reg = g.region[s];
         const uint32_t pbase = g.port_offs[s], nports = g.port_offs[s + 1] - pbase;
         for (uint32_t wb = pos + warp * 32; wb < seg_end; wb += 32 * kHopWarps) {
             const uint32_t cnt = min(32u, seg_end - wb);
@@ -789,8 +829,9 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
                 pr = __ldg(reinterpret_cast<const uint4 *>(g.probes) + e.x);
             }
-            uint32_t my_status = 0xFFu, my_next = 0;
-            // lane-per-probe when every candidate list of the batch is short
+            uint32_t my_status = kAlive, my_next = 0;
+            // Every listed probe is permitted at s (checked when it was handed
+            // on).  Lane-per-probe when every candidate list of the batch is short.
             bool lane_mode = false;
             if (kIndexed) {
                 const uint32_t *boff = reinterpret_cast<const uint32_t *>(s_raw + L.boff);
@@ -802,13 +843,8 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 lane_mode = __reduce_max_sync(PV_FULL_MASK, len) <= g.lane_max;
             }
             if (lane_mode) {
-                if (lane < cnt) {
-                    const uint32_t mask = pr.w;
-                    uint32_t fm = 0;
-                    const bool allowed = reg < 32 && ((mask >> reg) & 1u);
-                    if (allowed) fm = first_match_lane(s_raw, L, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu);
-                    hop_outcome(g, allowed, fm, pr.y, pbase, nports, &my_status, &my_next);
-                }
+                const uint32_t fm = first_match_lane(s_raw, L, lane < cnt, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu);
+                if (lane < cnt) hop_outcome(g, fm, pr.y, pr.w, pbase, nports, &my_status, &my_next);
             } else {
                 for (uint32_t j = 0; j < cnt; ++j) {
                     const uint32_t in_port = __shfl_sync(PV_FULL_MASK, e.y, j) & 0xFFu;
@@ -816,27 +852,25 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                     const uint32_t dst = __shfl_sync(PV_FULL_MASK, pr.y, j);
                     const uint32_t dport = __shfl_sync(PV_FULL_MASK, pr.z, j) & 0xFFFFu;
                     const uint32_t mask = __shfl_sync(PV_FULL_MASK, pr.w, j);
-                    const bool allowed = reg < 32 && ((mask >> reg) & 1u);
-                    uint32_t fm = 0;
-                    if (allowed)
-                        fm = kIndexed ? first_match_indexed(s_raw, hdr, lane, src, dst, dport, in_port)
-                                      : first_match_linear(s_raw, hdr.x, lane, src, dst, dport, in_port);
+                    const uint32_t fm = kIndexed ? first_match_indexed(s_raw, hdr, lane, src, dst, dport, in_port)
+                                                 : first_match_linear(s_raw, hdr.x, lane, src, dst, dport, in_port);
                     uint32_t status, next;
-                    hop_outcome(g, allowed, fm, dst, pbase, nports, &status, &next);
+                    hop_outcome(g, fm, dst, mask, pbase, nports, &status, &next);
                     if (lane == j) {
                         my_status = status;
                         my_next = next;
                     }
                 }
             }
-            if (lane < cnt && my_status != 0xFFu) {
+            if (lane < cnt && my_status != kAlive) {
+                const bool at_next = my_status == kViolationNext;
                 pv_result r;
-                r.status = (uint8_t)my_status;
-                r.hops = (uint8_t)(g.hop + 1);
-                r.last_switch = (uint16_t)s;
+                r.status = (uint8_t)(at_next ? (uint32_t)PV_VIOLATION : my_status);
+                r.hops = (uint8_t)(g.hop + (at_next ? 2u : 1u));
+                r.last_switch = (uint16_t)(at_next ? (my_next >> 8) : s);
                 g.out[e.x] = r;
             }
-            const bool live = lane < cnt && my_status == 0xFFu;
+            const bool live = lane < cnt && my_status == kAlive;
             const uint32_t slot = warp_reserve(live, &s_count);
             if (live) g.next_list[r0 + slot] = make_uint2(e.x, my_next);
         }
@@ -1070,7 +1104,7 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
     walk_init_kernel<<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port,
-                                                         d_out, listA, descA);
+                                                         t.d_region, d_out, listA, descA);
     pv_prof_stop(ctx, st, pr, 1);
     const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
