@@ -239,6 +239,34 @@ int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_offs, uint32_t
                        const uint32_t *d_masks, uint32_t *d_reach, uint32_t words_per_row, pv_stream stream);
 
 /* ---------------------------------------------------------------------------
+ * pv_compliant_reach_noalloc -- the same computation and output as
+ * pv_compliant_reach, for callers that cannot allocate device memory: a
+ * program whose device memory belongs to another framework's pool or is held
+ * to a fixed budget, or a latency-critical caller that cannot absorb the
+ * device-wide synchronisation cudaMalloc / cudaFree may imply.  (The paper
+ * has no counterpart; this is a property of the library, not of the method.)
+ *
+ * It needs no pv_ctx and allocates nothing: its working memory (a status
+ * word and the in-edge CSR) is one static device array of about 1.2 MB that
+ * every GPU which loads the library holds until the process exits.  Limits:
+ * V <= 16384 and num_edges <= 262144; larger inputs return PV_EINVAL before
+ * any work is queued.  Arguments, layouts and the result are those of
+ * pv_compliant_reach; the call runs on `stream` on the current device.
+ * The first call on a device looks up the array's device address (no
+ * allocation); make that first call before any stream capture.
+ * All calls share the one array and each call overwrites it, so calls whose
+ * work overlaps on the GPU (different streams, or host threads without
+ * ordering) race; order them on one stream.  Malformed CSR entries are
+ * skipped as in pv_compliant_reach, but no error is reported for them here.
+ * Returns PV_OK, PV_EINVAL (limits, NULL or misaligned pointers) or
+ * PV_ECUDA.
+ * ------------------------------------------------------------------------- */
+int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_edges, const uint32_t *d_cols,
+                               const uint8_t *d_region, uint32_t num_src, const uint32_t *d_src,
+                               uint32_t num_masks, const uint32_t *d_masks, uint32_t *d_reach,
+                               uint32_t words_per_row, pv_stream stream);
+
+/* ---------------------------------------------------------------------------
  * End-to-end composition (Sec. 4.2 hybrid coordination: pods are placed
  * first, then flows from their attachments are checked; Sec. 5.5: an intent
  * passes only if all of its checks pass).  A "group" is one intent: one

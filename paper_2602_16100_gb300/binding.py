@@ -27,7 +27,7 @@ PV_STAT_SELECTOR_ROWS_BUILT, PV_STAT_SCRATCH_BYTES, PV_STAT_WALK_INDEX_FITS, PV_
 SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", "pv_load_cluster",
            "pv_eval_selectors", "pv_load_flow_tables", "pv_verify_probes", "pv_compliant_reach",
            "pv_place_pods", "pv_bind_probes", "pv_aggregate_intents", "pv_set_option", "pv_get_stat",
-           "pv_profile_enable", "pv_profile_collect", "pv_profile_read")
+           "pv_profile_enable", "pv_profile_collect", "pv_profile_read", "pv_compliant_reach_noalloc")
 
 #: kernel groups timed by the library profiler (PV_K_* in include/pv.h)
 PV_K_NAMES = ("selector", "place", "bind", "walk_init", "walk_regroup", "walk_hop", "aggregate", "reach")
@@ -75,6 +75,7 @@ def load_library(path: Optional[str] = None):
         "pv_profile_collect": (ctypes.c_int, [vp, vp]),
         "pv_profile_read": (ctypes.c_int, [vp, ctypes.c_int, ctypes.POINTER(ctypes.c_double),
                                            ctypes.POINTER(ctypes.c_uint64)]),
+        "pv_compliant_reach_noalloc": (ctypes.c_int, [u32, vp, u32, vp, vp, u32, vp, u32, vp, vp, u32, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -230,3 +231,18 @@ def pv_aggregate_intents(ctx, num_groups, pods_per_group, d_bits, words_per_row,
                                                            words_per_row, _dev(d_group_flags), _dev(d_assign),
                                                            probes_per_group, _dev(d_results), _dev(d_pass),
                                                            _dev(d_counts), _stream(stream)))
+
+
+def pv_compliant_reach_noalloc(V, d_offs, num_edges, d_cols, d_region, num_src, d_src, num_masks, d_masks, d_reach,
+                               words_per_row, stream=None) -> int:
+    """Compliant reach without any device allocation (no context): for callers
+    whose device memory is owned by another allocator or a fixed budget, or
+    that cannot absorb cudaMalloc/cudaFree synchronisation.  Works in a static
+    ~1.2 MB device array shared by all calls (V <= 16384, num_edges <=
+    262144).  Returns the C status; a non-zero status raises PVError."""
+    rc = load_library().pv_compliant_reach_noalloc(V, _dev(d_offs), num_edges, _dev(d_cols), _dev(d_region), num_src,
+                                                   _dev(d_src), num_masks, _dev(d_masks), _dev(d_reach),
+                                                   words_per_row, _stream(stream))
+    if rc != PV_OK:
+        raise PVError(rc, "pv_compliant_reach_noalloc rejected its arguments or failed")
+    return rc

@@ -16,6 +16,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "pv_internal.cuh"
 
@@ -209,4 +210,88 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
                                                        d_reach, words_per_row);
     pv_prof_stop(ctx, st, pr, 4);
     return pv_check_launch(ctx, "reach kernels");
+}
+
+// -----------------------------------------------------------------------------
+// Compliant reach that allocates nothing.
+//
+// For callers that must not allocate device memory themselves or through this
+// library: a host program whose device memory is owned by another framework's
+// pool or held to a fixed budget, or a latency-critical caller that cannot
+// afford the device-wide synchronisation cudaMalloc / cudaFree may imply.
+// The in-edge CSR this path builds lives in one static device array below;
+// every GPU that loads the library holds it until the process exits.
+// -----------------------------------------------------------------------------
+namespace {
+
+constexpr size_t up256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+constexpr uint32_t kNoAllocMaxEdges = 1u << 18;   // directed edges accepted by the no-allocation call
+constexpr size_t kNoAllocIndeg = 256;              // [0, 256): status word
+constexpr size_t kNoAllocInOffs = kNoAllocIndeg + up256((size_t)(kReachMaxV + 1) * 4);
+constexpr size_t kNoAllocCursor = kNoAllocInOffs + up256((size_t)(kReachMaxV + 1) * 4);
+constexpr size_t kNoAllocCols = kNoAllocCursor + up256((size_t)kReachMaxV * 4);
+constexpr size_t kNoAllocBytes = kNoAllocCols + up256((size_t)kNoAllocMaxEdges * 4);   // about 1.2 MB
+
+__device__ __align__(256) uint8_t g_reach_noalloc_scratch[kNoAllocBytes];
+
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+uint8_t *g_noalloc_base[kNoAllocMaxDevices] = {};
+
+// Device address of the static array on the current device, looked up once
+// per device (in host code the array's name is not a device address).
+int noalloc_scratch(uint8_t **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return PV_ECUDA;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return PV_EINVAL;
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (!g_noalloc_base[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_reach_noalloc_scratch) != cudaSuccess || !p) return PV_ECUDA;
+        g_noalloc_base[dev] = static_cast<uint8_t *>(p);
+    }
+    *out = g_noalloc_base[dev];
+    return PV_OK;
+}
+
+}  // namespace
+
+extern "C" int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_edges,
+                                          const uint32_t *d_cols, const uint8_t *d_region, uint32_t num_src,
+                                          const uint32_t *d_src, uint32_t num_masks, const uint32_t *d_masks,
+                                          uint32_t *d_reach, uint32_t words_per_row, pv_stream stream) {
+    if (V == 0 || V > kReachMaxV) return PV_EINVAL;
+    if (num_edges > kNoAllocMaxEdges) return PV_EINVAL;
+    if (words_per_row % 4 != 0 || words_per_row < (V + 31) / 32) return PV_EINVAL;
+    if (num_src == 0 || num_masks == 0) return PV_OK;
+    if (!d_offs || !d_region || !d_src || !d_masks || !d_reach || (num_edges && !d_cols)) return PV_EINVAL;
+    if (((uintptr_t)d_reach & 15) != 0 || num_masks > 65535) return PV_EINVAL;
+    uint8_t *base = nullptr;
+    const int rc = noalloc_scratch(&base);
+    if (rc != PV_OK) return rc;
+    int32_t *status = reinterpret_cast<int32_t *>(base);
+    uint32_t *indeg = reinterpret_cast<uint32_t *>(base + kNoAllocIndeg);
+    uint32_t *in_offs = reinterpret_cast<uint32_t *>(base + kNoAllocInOffs);
+    uint32_t *cursor = reinterpret_cast<uint32_t *>(base + kNoAllocCursor);
+    uint32_t *in_cols = reinterpret_cast<uint32_t *>(base + kNoAllocCols);
+    cudaStream_t st = (cudaStream_t)stream;
+    // the array keeps the previous call's contents: clear what must start at zero
+    if (cudaMemsetAsync(base, 0, kNoAllocIndeg + (size_t)(V + 1) * 4, st) != cudaSuccess) return PV_ECUDA;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return PV_ECUDA;
+    const uint32_t grid = std::min<uint32_t>((V + kGridThreads - 1) / kGridThreads, (uint32_t)sms * 8);
+    reach_indeg_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, d_region, indeg, status);
+    reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor);
+    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols);
+    const size_t smem = (size_t)V * 8;
+    if (cudaFuncSetAttribute(reach_msbfs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+        cudaSuccess)
+        return PV_ECUDA;
+    dim3 g2((num_src + 63) / 64, num_masks);
+    reach_msbfs_kernel<<<g2, kReachThreads, smem, st>>>(V, in_offs, in_cols, d_region, num_src, d_src, d_masks,
+                                                       d_reach, words_per_row);
+    return cudaGetLastError() == cudaSuccess ? PV_OK : PV_ECUDA;
 }
