@@ -124,6 +124,14 @@ def committed_traffic(kernel: str, src_hash: str):
         return None
 
 
+def _walk_entries(v):
+    """Probe-hop entries the hop kernel processed in the last walk (the sum
+    over hops of the live probes; a probe judged at a hand-off is counted in
+    its result's hops but never entered at the next switch)."""
+    from paper_2602_16100_gb300 import binding as B
+    return int(B.pv_get_stat(v.ctx, B.PV_STAT_WALK_LIVE_TOTAL))
+
+
 # ----------------------------------------------------------------------------
 # workloads
 # ----------------------------------------------------------------------------
@@ -158,11 +166,12 @@ class EndToEndBench:
         self.selector_evals = self.e.intents.num_pods * self.e.cluster.num_nodes
         self.status_hist = torch.bincount(res[:, 0].to(torch.int64), minlength=6).tolist()
         self.pass_count = int(self.dev["pass"][: self.e.intents.num_pods].to(torch.int64).sum().item())
+        self.hop_entries = _walk_entries(self.v)
         return self.probe_hops
 
     def extra(self, secs_per_step):
         return {"selector_evals_per_s": self.selector_evals / secs_per_step,
-                "probe_hops_per_step": self.probe_hops,
+                "probe_hops_per_step": self.probe_hops, "hop_kernel_entries_per_step": self.hop_entries,
                 "status_histogram": dict(zip(W.STATUS_NAMES, self.status_hist)),
                 "intents_passed": self.pass_count}
 
@@ -170,10 +179,10 @@ class EndToEndBench:
         e = self.e
         I = e.intents.num_pods
         M = len(e.probes.probes)
-        if group == "walk_hop":         # per probe-hop: 16 B probe record read + 4 B result / state written
-            return 20 * self.probe_hops
-        if group == "walk_regroup":     # per probe-hop: 8 B state read + 8 B state written
-            return 16 * self.probe_hops
+        if group == "walk_hop":         # per hop entry: 16 B probe record read + 4 B result / state written
+            return 20 * self.hop_entries
+        if group == "walk_regroup":     # per hop entry: 8 B state read + 8 B state written
+            return 16 * self.hop_entries
         if group == "selector":
             return I * W.words_per_row(e.cluster.num_nodes) * 4 + len(e.intents.exprs) * 20 + I * 5
         if group == "bind":
@@ -185,36 +194,35 @@ class EndToEndBench:
         return 0
 
     def traffic_unit(self, group):
-        return self.probe_hops if group in ("walk_hop", "walk_regroup") else None
+        return self.hop_entries if group in ("walk_hop", "walk_regroup") else None
 
     # host-buffer end-to-end step through the public API
-    def setup_e2e(self, v):
+    def setup_e2e(self, v, chunks=2):
         import torch
         e = self.e
-        self.h_probes = torch.from_numpy(e.probes.probes.view(np.uint8).reshape(-1)).pin_memory()
-        self.h_offs = torch.from_numpy(e.intents.expr_offs.astype(np.uint32).view(np.uint8)).pin_memory()
-        self.h_exprs = torch.from_numpy(e.intents.exprs.view(np.uint8).reshape(-1)).pin_memory()
-        self.h_draws = torch.from_numpy(e.place_draws.astype(np.uint64).view(np.uint8)).pin_memory()
-        self.h_pass = torch.empty(e.intents.num_pods, dtype=torch.uint8).pin_memory()
-        self.h_counts = torch.empty(e.intents.num_pods * 32, dtype=torch.uint8).pin_memory()
+        pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1).copy()).pin_memory()
+        self.host = {"offs": pin(e.intents.expr_offs.astype(np.uint32)), "exprs": pin(e.intents.exprs),
+                     "draws": pin(e.place_draws.astype(np.uint64)), "probes": pin(e.probes.probes),
+                     "pass": torch.empty(e.intents.num_pods, dtype=torch.uint8).pin_memory(),
+                     "counts": torch.empty(e.intents.num_pods * 32, dtype=torch.uint8).pin_memory()}
+        self.copy_stream = torch.cuda.Stream()
+        self.chunks = chunks
         net = e.network
-        self.h2d = (self.h_probes.numel() + self.h_offs.numel() + self.h_exprs.numel() + self.h_draws.numel()
+        self.h2d = (sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "probes"))
                     + e.cluster.labels.nbytes + net.rule_offs.nbytes + net.rules.nbytes + net.switch_region.nbytes
                     + net.port_offs.nbytes + net.port_peer.nbytes + net.host_switch.nbytes + net.host_port.nbytes
                     + net.host_ip.nbytes)
-        self.d2h = self.h_pass.numel() + self.h_counts.numel()
+        self.d2h = self.host["pass"].numel() + self.host["counts"].numel()
 
     def step_e2e(self, v, stream):
-        e, dev = self.e, self.dev
+        """Every input from host memory: cluster labels and flow tables
+        through the loaders, intents and probes copied (the probe upload
+        overlapped with verification, `chunks` intent ranges), verdicts and
+        counters copied back."""
+        e = self.e
         v.load_cluster(e.cluster)
         v.load_network(e.network)
-        dev["probes"][: self.h_probes.numel()].copy_(self.h_probes, non_blocking=True)
-        dev["offs"][: self.h_offs.numel()].copy_(self.h_offs, non_blocking=True)
-        dev["exprs"][: self.h_exprs.numel()].copy_(self.h_exprs, non_blocking=True)
-        dev["draws"][: self.h_draws.numel()].copy_(self.h_draws, non_blocking=True)
-        v.run_end_to_end(dev, self.sizes, stream)
-        self.h_pass.copy_(dev["pass"][: self.h_pass.numel()], non_blocking=True)
-        self.h_counts.copy_(dev["counts"][: self.h_counts.numel()], non_blocking=True)
+        v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks)
 
     # oracle on a bounded sample: the first n intents, whole pipeline
     def oracle_sample(self, n_intents):
@@ -328,17 +336,19 @@ class FlowBench:
         res = self.d_out.view(-1, 4)
         self.probe_hops = int(res[:, 1].to(torch.int64).sum().item())
         self.hist = torch.bincount(res[:, 0].to(torch.int64), minlength=6).tolist()
+        self.hop_entries = _walk_entries(self.v)
         return self.probe_hops
 
     def extra(self, secs_per_step):
-        return {"probe_hops_per_step": self.probe_hops, "status_histogram": dict(zip(W.STATUS_NAMES, self.hist))}
+        return {"probe_hops_per_step": self.probe_hops, "hop_kernel_entries_per_step": self.hop_entries,
+                "status_histogram": dict(zip(W.STATUS_NAMES, self.hist))}
 
     def algorithmic_bytes(self, group):
-        return {"walk_hop": 20, "walk_regroup": 16}.get(group, 0) * self.probe_hops + \
+        return {"walk_hop": 20, "walk_regroup": 16}.get(group, 0) * self.hop_entries + \
             (len(self.p.probes) * 16 if group == "walk_init" else 0)
 
     def traffic_unit(self, group):
-        return self.probe_hops if group in ("walk_hop", "walk_regroup") else None
+        return self.hop_entries if group in ("walk_hop", "walk_regroup") else None
 
     def oracle_sample(self, n):
         import oracle
@@ -465,12 +475,15 @@ def run_ours(args):
     torch.cuda.set_device(local)
     from paper_2602_16100_gb300 import binding as B
     from paper_2602_16100_gb300 import build
+    from paper_2602_16100_gb300 import sharding as SH
     from paper_2602_16100_gb300.validator import Validator
     if rank == 0 or world == 1:
         build.build_library()
     if dist:
         dist.barrier()
-    wl = WORKLOADS[args.workload](rank, **({"intents": args.intents} if args.intents else {}))
+    # weak scaling: every rank verifies its own batch of the same shape (the
+    # units are independent; no collective on the data path)
+    wl = WORKLOADS[args.workload](SH.shard_seed(0, rank), **({"intents": args.intents} if args.intents else {}))
     v = Validator(local)
     wl.setup(v)
     stream = torch.cuda.current_stream()
@@ -500,10 +513,7 @@ def run_ours(args):
     B.pv_profile_enable(v.ctx, False)
     ms = start.elapsed_time(stop)
     v.sync(stream)
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = SH.max_over_ranks(ms, dist, "cuda")
     secs_per_step = ms / 1e3 / args.steps
     value = units * world / secs_per_step
 
@@ -534,7 +544,7 @@ def run_ours(args):
     # end-to-end through the public API from pinned host buffers
     e2e = None
     if hasattr(wl, "setup_e2e"):
-        wl.setup_e2e(v)
+        wl.setup_e2e(v, args.e2e_chunks)
         wl.step_e2e(v, stream)
         barrier()
         t0 = time.perf_counter()
@@ -542,12 +552,9 @@ def run_ours(args):
             wl.step_e2e(v, stream)
         barrier()
         e_s = (time.perf_counter() - t0) / args.steps
-        if dist:
-            t = torch.tensor([e_s], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e_s = float(t.item())
+        e_s = SH.max_over_ranks(e_s, dist, "cuda")
         e2e = {"value": units * world / e_s, "unit": wl.unit, "h2d_bytes_per_step": int(wl.h2d),
-               "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3}
+               "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3, "upload_chunks": args.e2e_chunks}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -577,6 +584,8 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", choices=tuple(WORKLOADS), default="e2e")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-chunks", type=int, default=2,
+                    help="intent ranges whose probe upload overlaps verification in the host-buffer step")
     ap.add_argument("--intents", type=int, default=None,
                     help="end-to-end only: fewer intents (a smaller case for profiling, not a bench line)")
     args = ap.parse_args()

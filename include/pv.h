@@ -139,7 +139,7 @@ int pv_version(void);
  * Copied to the device; the library also builds the per-key inventory of
  * carried values (for the hallucinated-identifier check of Sec. 6.3) and,
  * when it fits its memory budget, per-(key, value) node bitsets.
- * Errors: PV_EINVAL if num_nodes == 0, num_keys == 0 or num_keys > 65535;
+ * Errors: PV_EINVAL if num_nodes == 0, num_keys == 0 or num_keys > 4096;
  * PV_ENOMEM.  Replaces any previously loaded cluster.
  * ------------------------------------------------------------------------- */
 int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_keys, const uint16_t *labels);
@@ -308,14 +308,24 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  * PV_OPT_WALK_LANE_MAX: with kernel 2, a batch of 32 probes is resolved one
  *   probe per lane when its longest candidate list has at most this many
  *   items (default 96), else one probe at a time by the whole warp.
+ * PV_OPT_TEST_STALL_STAGING: failure-injection switch for tests (0 or 1).
+ *   When 1, each hop block's table-staging barrier expects 16 bytes more
+ *   than its copy delivers, so its bounded wait runs out (after 50 ms rather
+ *   than the normal 2 s); the walk then reports PV_ETIMEOUT through pv_sync
+ *   and the context stays usable.  Never set it outside a test.
  * pv_get_stat: PV_STAT_SELECTOR_ROWS_BUILT (1 if value rows exist),
  *   PV_STAT_SCRATCH_BYTES, PV_STAT_WALK_INDEX_FITS (1 if kernel 2 is
- *   usable), PV_STAT_WALK_INDEX_BYTES (largest per-switch table + index).
+ *   usable), PV_STAT_WALK_INDEX_BYTES (largest per-switch table + index),
+ *   PV_STAT_WALK_LIVE_TOTAL (probe-hop entries the last pv_verify_probes
+ *   processed: the sum over its hops of the probes still walking; reading it
+ *   synchronises with the device).
  * ------------------------------------------------------------------------- */
-enum { PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3 };
+enum {
+    PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4
+};
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,
-    PV_STAT_WALK_INDEX_BYTES = 4
+    PV_STAT_WALK_INDEX_BYTES = 4, PV_STAT_WALK_LIVE_TOTAL = 5
 };
 int pv_set_option(pv_ctx *ctx, int option, int64_t value);
 int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value);

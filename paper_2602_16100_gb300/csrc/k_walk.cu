@@ -34,6 +34,7 @@ namespace {
 
 constexpr int kHopThreads = 256;
 constexpr int kHopWarps = kHopThreads / 32;
+constexpr uint32_t kMinPerBlock = 512;       // live probes per active hop block
 constexpr int kGridThreads = 256;
 constexpr uint32_t kSmemHistMax = 12288;     // switches for shared-memory histograms
 constexpr uint32_t kWaitLimit = 1u << 24;    // bounded mbarrier polls
@@ -60,6 +61,17 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
         "l"(src), "r"(bytes), "r"(smem_u32(bar))
         : "memory");
 }
+// Same copy, asking L2 to keep the source lines (evict_last): the flow-table
+// blobs are re-read every hop while the probe lists stream through L2.
+__device__ __forceinline__ void bulk_g2s_keep(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile(
+        "{\n\t.reg .b64 pol;\n\t"
+        "createpolicy.fractional.L2::evict_last.b64 pol, 1.0;\n\t"
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], pol;\n\t}"
+        ::"r"(smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar))
+        : "memory");
+}
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
@@ -71,22 +83,44 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
-    for (uint32_t it = 0; it < kWaitLimit; ++it)
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+// Waits for the phase with the given parity; gives up after limit_ns
+// nanoseconds of the global timer (or kWaitLimit polls, whichever is first).
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity, uint64_t limit_ns) {
+    const uint64_t t0 = global_ns();
+    for (uint32_t it = 0; it < kWaitLimit; ++it) {
         if (mbar_try_wait(bar, parity)) return true;
+        if (global_ns() - t0 > limit_ns) break;
+    }
     return false;
 }
 
 // ---------------------------------------------------------------------------
 // load: per-switch stable priority sort + compile
 // ---------------------------------------------------------------------------
+// Also validates every rule of the switch against its port count; the lowest
+// offending global rule index goes to *bad (0xFFFFFFFF when all are valid).
 __global__ void __launch_bounds__(1024) compile_tables_kernel(const uint32_t *__restrict__ rule_offs,
                                                               const pv_rule *__restrict__ raw,
+                                                              const uint32_t *__restrict__ port_offs,
                                                               const uint32_t *__restrict__ tab_offs,
-                                                              uint4 *__restrict__ A, uint2 *__restrict__ B) {
+                                                              uint4 *__restrict__ A, uint2 *__restrict__ B,
+                                                              uint32_t *__restrict__ bad) {
     extern __shared__ uint32_t s_keys[];
     const uint32_t s = blockIdx.x, t = threadIdx.x;
     const uint32_t base = rule_offs[s], n = rule_offs[s + 1] - base;
+    const uint32_t nports = port_offs[s + 1] - port_offs[s];
+    for (uint32_t i = t; i < n; i += blockDim.x) {
+        const pv_rule r = raw[base + i];
+        const bool ok = (r.in_port == PV_ANY_PORT || r.in_port < nports) &&
+                        (r.action == PV_DROP || r.action < nports) && r.src_len <= 32 && r.dst_len <= 32 &&
+                        r.dport_lo <= r.dport_hi;
+        if (!ok) atomicMin(bad, base + i);
+    }
     uint32_t npow = 1;
     while (npow < n) npow <<= 1;
     for (uint32_t i = t; i < npow; i += blockDim.x)
@@ -113,7 +147,8 @@ __global__ void __launch_bounds__(1024) compile_tables_kernel(const uint32_t *__
         uint2 b;
         if (i < n) {
             const pv_rule r = raw[base + (s_keys[i] & 0xFFFFu)];
-            const uint32_t ms = pv_prefix_mask(r.src_len), md = pv_prefix_mask(r.dst_len);
+            const uint32_t ms = pv_prefix_mask(min(32u, (uint32_t)r.src_len));
+            const uint32_t md = pv_prefix_mask(min(32u, (uint32_t)r.dst_len));
             a = make_uint4(r.src_ip & ms, ms, r.dst_ip & md, md);
             const bool any = r.in_port == PV_ANY_PORT;
             b.x = (uint32_t)r.dport_lo | ((uint32_t)r.dport_hi << 16);
@@ -158,7 +193,8 @@ constexpr uint32_t kSegItem = 0x8000u;
 constexpr uint32_t kWinFound = 0x80000000u;
 constexpr uint32_t kKeyCap = 2 * kMaxSegment + 8;   // boundaries of one segment (+ slack)
 constexpr uint32_t kSortCap = 16384;                // power of two >= 2 * kMaxSegment + 1
-constexpr size_t kIndexSmem = (size_t)kSortCap * 4 + (size_t)kKeyCap * 8 + PV_MAX_RULES * 2 + kMaxSegments * 8;
+constexpr size_t kIndexSmem = (size_t)kSortCap * 4 + (size_t)kKeyCap * 8 + PV_MAX_RULES * 2 + kMaxSegments * 8 +
+                              (size_t)kMaxSegment * 10;
 
 __host__ __device__ inline uint32_t up16(uint32_t b) { return (b + 15u) & ~15u; }
 
@@ -232,6 +268,8 @@ __global__ void __launch_bounds__(1024) index_build_kernel(const uint32_t *__res
     uint32_t *s_pos = s_win + kKeyCap;                             // [kKeyCap]
     int16_t *s_cls = reinterpret_cast<int16_t *>(s_pos + kKeyCap);  // [PV_MAX_RULES]
     uint32_t *s_segs = reinterpret_cast<uint32_t *>(s_cls + PV_MAX_RULES);  // [kMaxSegments][2]
+    uint2 *s_rules = reinterpret_cast<uint2 *>(s_segs + 2 * kMaxSegments);  // [kMaxSegment] {value, mask}
+    uint16_t *s_act = reinterpret_cast<uint16_t *>(s_rules + kMaxSegment);   // [kMaxSegment]
     __shared__ uint32_t s_warp[33];
     __shared__ uint32_t s_nsegs;
     const uint32_t s = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
@@ -355,14 +393,22 @@ __global__ void __launch_bounds__(1024) index_build_kernel(const uint32_t *__res
         for (uint32_t x = t; x < nk; x += nt)
             if (x == 0 || s_win[x] != s_win[x - 1]) s_keys[s_pos[x]] = s_win[x];
         __syncthreads();
+        // the segment's prefixes and actions, staged so the winner scan below
+        // reads them as shared-memory broadcasts
+        for (uint32_t r = t; r < m; r += nt) {
+            const uint4 ar = a[k0 + r];
+            s_rules[r] = make_uint2(ar.z, ar.w);
+            s_act[r] = (uint16_t)(b[k0 + r].y >> 16);
+        }
+        __syncthreads();
         // winners of the K elementary intervals
         for (uint32_t x = t; x < K; x += nt) {
             const uint32_t d = s_keys[x];
             uint32_t w = 0;
-            for (uint32_t r = k0; r < k1; ++r) {
-                const uint4 ar = a[r];
-                if (((d ^ ar.z) & ar.w) == 0) {
-                    w = kWinFound | (b[r].y >> 16);
+            for (uint32_t r = 0; r < m; ++r) {
+                const uint2 ar = s_rules[r];
+                if (((d ^ ar.x) & ar.y) == 0) {
+                    w = kWinFound | s_act[r];
                     break;
                 }
             }
@@ -589,6 +635,9 @@ struct HopArgs {
     uint2 *next_desc;
     int32_t *status;
     uint32_t lane_max;   // longest candidate list handled one probe per lane
+    uint32_t wait_extra; // bytes the staging barrier expects beyond the copy (0; > 0 only in failure tests)
+    uint64_t wait_ns;    // bound on each staging wait
+    uint32_t *hop_live;  // [cap]: live probes processed at each hop (statistics)
 };
 
 // Linear first match: 32 consecutive rules per warp step.
@@ -774,8 +823,12 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     __shared__ uint32_t s_count;
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t n = g.seg[g.S];   // live probes this hop
-    const uint32_t r0 = (uint32_t)(((uint64_t)n * blockIdx.x) / gridDim.x);
-    const uint32_t r1 = (uint32_t)(((uint64_t)n * (blockIdx.x + 1)) / gridDim.x);
+    if (blockIdx.x == 0 && threadIdx.x == 0) g.hop_live[g.hop] = n;
+    // only as many blocks as give each at least kMinPerBlock probes: a block
+    // stages a whole switch table, which small shares would not repay
+    const uint32_t active = max(1u, min(gridDim.x, (n + kMinPerBlock - 1) / kMinPerBlock));
+    const uint32_t r0 = blockIdx.x < active ? (uint32_t)(((uint64_t)n * blockIdx.x) / active) : n;
+    const uint32_t r1 = blockIdx.x < active ? (uint32_t)(((uint64_t)n * (blockIdx.x + 1)) / active) : n;
     if (r0 >= r1) {
         if (threadIdx.x == 0) g.next_desc[blockIdx.x] = make_uint2(r0, 0);
         return;
@@ -804,16 +857,18 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
         __syncthreads();   // everyone is done with the previous table
         if (threadIdx.x == 0) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            mbar_arrive_expect_tx(&s_bar, bytes);
-            bulk_g2s(s_raw, src_blob, bytes, &s_bar);
+            mbar_arrive_expect_tx(&s_bar, bytes + g.wait_extra);
+            bulk_g2s_keep(s_raw, src_blob, bytes, &s_bar);
         }
-        const bool ok = mbar_wait_bounded(&s_bar, parity);
+        const bool ok = mbar_wait_bounded(&s_bar, parity, g.wait_ns);
         if (__syncthreads_or(!ok)) {
+            // give up: record the timeout, leave an empty slice for the next
+            // hop, let the copy in flight land (bounded again), return
             if (threadIdx.x == 0) {
                 pv_device_error(g.status, PV_ETIMEOUT);
                 g.next_desc[blockIdx.x] = make_uint2(r0, 0);
             }
-            mbar_wait_bounded(&s_bar, parity);   // let copies in flight land
+            mbar_wait_bounded(&s_bar, parity, g.wait_ns);
             return;
         }
         parity ^= 1u;
@@ -913,17 +968,8 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     const uint32_t R = rule_offs[S], P = port_offs[S];
     if (R && !rules) return pv_fail(ctx, PV_EINVAL, "NULL rules");
     if (P && !port_peer) return pv_fail(ctx, PV_EINVAL, "NULL port_peer");
+    // per-rule fields are checked on the device by compile_tables_kernel
     for (uint32_t s = 0; s < S; ++s) {
-        const uint32_t np = port_offs[s + 1] - port_offs[s];
-        for (uint32_t i = rule_offs[s]; i < rule_offs[s + 1]; ++i) {
-            const pv_rule &r = rules[i];
-            if (r.in_port != PV_ANY_PORT && r.in_port >= np)
-                return pv_fail(ctx, PV_EINVAL, "rule %u: in_port %u >= %u ports", i, r.in_port, np);
-            if (r.action != PV_DROP && r.action >= np)
-                return pv_fail(ctx, PV_EINVAL, "rule %u: action %u >= %u ports", i, r.action, np);
-            if (r.src_len > 32 || r.dst_len > 32) return pv_fail(ctx, PV_EINVAL, "rule %u: prefix length > 32", i);
-            if (r.dport_lo > r.dport_hi) return pv_fail(ctx, PV_EINVAL, "rule %u: dport_lo > dport_hi", i);
-        }
         for (uint32_t p = port_offs[s]; p < port_offs[s + 1]; ++p) {
             const int32_t peer = port_peer[p];
             if (peer == PV_PEER_NONE) continue;
@@ -962,7 +1008,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     if ((rc = pv_device_alloc(ctx, (void **)&d_tab_offs, (S + 1) * 4, "table offsets")) ||
         (rc = pv_device_alloc(ctx, (void **)&d_rule_a, (size_t)T * 16, "rules A")) ||
         (rc = pv_device_alloc(ctx, (void **)&d_rule_b, (size_t)T * 8, "rules B")) ||
-        (rc = pv_device_alloc(ctx, (void **)&d_sizes, (size_t)S * 12, "index sizes")) ||
+        (rc = pv_device_alloc(ctx, (void **)&d_sizes, (size_t)S * 12 + 4, "index sizes")) ||
         (rc = pv_device_alloc(ctx, (void **)&t.d_blob_offs, ((size_t)S + 1) * 8, "blob offsets")) ||
         (rc = pv_device_alloc(ctx, (void **)&t.d_region, S, "regions")) ||
         (rc = pv_device_alloc(ctx, (void **)&t.d_port_offs, (S + 1) * 4, "port offsets")) ||
@@ -993,8 +1039,13 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         for (uint32_t s = 0; s < S; ++s) maxn = std::max(maxn, rule_offs[s + 1] - rule_offs[s]);
         uint32_t npow = 1;
         while (npow < maxn) npow <<= 1;
-        compile_tables_kernel<<<S, 1024, npow * 4>>>(d_rule_offs, d_raw, d_tab_offs, d_rule_a, d_rule_b);
-        e = cudaGetLastError();
+        uint32_t *d_bad = d_sizes + (size_t)S * 3;   // lowest invalid rule index
+        e = cudaMemset(d_bad, 0xFF, 4);
+        if (e == cudaSuccess) {
+            compile_tables_kernel<<<S, 1024, npow * 4>>>(d_rule_offs, d_raw, t.d_port_offs, d_tab_offs, d_rule_a,
+                                                         d_rule_b, d_bad);
+            e = cudaGetLastError();
+        }
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(index_build_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)kIndexSmem);
@@ -1007,10 +1058,22 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
             e = cudaGetLastError();
         }
     }
-    // blob layout from the index sizes
-    std::vector<uint32_t> sizes((size_t)S * 3);
+    // blob layout from the index sizes (and the device-side rule validation)
+    std::vector<uint32_t> sizes((size_t)S * 3 + 1);
     std::vector<uint64_t> boffs(S + 1, 0);
-    if (e == cudaSuccess) e = cudaMemcpy(sizes.data(), d_sizes, (size_t)S * 12, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemcpy(sizes.data(), d_sizes, (size_t)S * 12 + 4, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && sizes[(size_t)S * 3] != 0xFFFFFFFFu) {
+        const uint32_t i = sizes[(size_t)S * 3];
+        const uint32_t s = (uint32_t)(std::upper_bound(rule_offs, rule_offs + S + 1, i) - rule_offs) - 1;
+        const pv_rule &r = rules[i];
+        free_temps();
+        pv_free_tables(t);
+        return pv_fail(ctx, PV_EINVAL,
+                       "rule %u (switch %u, %u ports): in_port %u, action %u, prefix lengths %u/%u, dport %u..%u "
+                       "out of range",
+                       i, s, port_offs[s + 1] - port_offs[s], r.in_port, r.action, r.src_len, r.dst_len,
+                       r.dport_lo, r.dport_hi);
+    }
     uint32_t max_blob = 0, max_linear = 0;
     if (e == cudaSuccess) {
         for (uint32_t s = 0; s < S; ++s) {
@@ -1123,6 +1186,10 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     g.out = d_out;
     g.status = ctx->d_status;
     g.lane_max = (uint32_t)ctx->opt_walk_lane_max;
+    g.hop_live = ctx->d_walk_live;
+    ctx->last_walk_cap = hop_cap;
+    g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
+    g.wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
     uint32_t in_slices = init_grid;
     for (uint32_t h = 0; h < hop_cap; ++h) {
         uint2 *cur = (h & 1) ? listB : listA;

@@ -171,8 +171,12 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
     cudaDeviceGetAttribute(&smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, cuda_device);
     ctx->max_smem_optin = (size_t)smem;
     if (pv_device_alloc(ctx, (void **)&ctx->d_status, sizeof(int32_t), "status word") != PV_OK ||
-        cudaMemset(ctx->d_status, 0, sizeof(int32_t)) != cudaSuccess) {
+        cudaMemset(ctx->d_status, 0, sizeof(int32_t)) != cudaSuccess ||
+        pv_device_alloc(ctx, (void **)&ctx->d_walk_live, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t),
+                        "walk statistics") != PV_OK ||
+        cudaMemset(ctx->d_walk_live, 0, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t)) != cudaSuccess) {
         pv_device_free(ctx->d_status);
+        pv_device_free(ctx->d_walk_live);
         delete ctx;
         return PV_ENOMEM;
     }
@@ -188,6 +192,7 @@ extern "C" void pv_destroy(pv_ctx *ctx) {
     for (cudaEvent_t e : ctx->prof.pool) cudaEventDestroy(e);
     pv_device_free(ctx->scratch);
     pv_device_free(ctx->d_status);
+    pv_device_free(ctx->d_walk_live);
     delete ctx;
 }
 
@@ -224,6 +229,10 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         if (value < 0 || value > 65535) return pv_fail(ctx, PV_EINVAL, "lane-mode list length must be 0..65535");
         ctx->opt_walk_lane_max = (int)value;
         return PV_OK;
+    case PV_OPT_TEST_STALL_STAGING:
+        if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "stall-staging test switch must be 0 or 1");
+        ctx->opt_test_stall_staging = (int)value;
+        return PV_OK;
     default:
         return pv_fail(ctx, PV_EINVAL, "unknown option %d", option);
     }
@@ -236,6 +245,17 @@ extern "C" int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value) {
     case PV_STAT_SCRATCH_BYTES: *value = (int64_t)ctx->scratch_bytes; return PV_OK;
     case PV_STAT_WALK_INDEX_FITS: *value = ctx->tb.index_fits ? 1 : 0; return PV_OK;
     case PV_STAT_WALK_INDEX_BYTES: *value = (int64_t)ctx->tb.max_blob_bytes; return PV_OK;
+    case PV_STAT_WALK_LIVE_TOTAL: {
+        uint32_t live[PV_MAX_HOP_CAP + 1];
+        const uint32_t cap = ctx->last_walk_cap;
+        if (cap && cudaMemcpy(live, ctx->d_walk_live, cap * sizeof(uint32_t), cudaMemcpyDeviceToHost) !=
+                       cudaSuccess)
+            return PV_ECUDA;
+        int64_t sum = 0;
+        for (uint32_t h = 0; h < cap; ++h) sum += live[h];
+        *value = sum;
+        return PV_OK;
+    }
     default: return PV_EINVAL;
     }
 }

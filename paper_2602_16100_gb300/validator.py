@@ -119,6 +119,58 @@ class Validator:
                                dev["results"], dev["pass"], dev["counts"], stream)
         return dev
 
+    def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
+                                 chunks: int = 2) -> dict:
+        """The end-to-end pipeline on inputs in pinned HOST memory, the probe
+        upload overlapped with the pipeline: the intents are cut into
+        `chunks` ranges (independent units), range c's probes are copied on
+        `copy_stream` while range c-1 is verified on `stream`; the per-intent
+        verdicts and counters come back into ``host["pass"]`` and
+        ``host["counts"]`` on `stream` (not synchronised).
+
+        ``host`` holds pinned byte tensors "offs", "exprs", "draws", "probes"
+        (inputs, as alloc_end_to_end lays them out) and "pass", "counts"
+        (outputs); ``dev`` the device buffers of alloc_end_to_end."""
+        I, pods, ppg = e2e_sizes["intents"], e2e_sizes["pods"], e2e_sizes["probes_per_intent"]
+        words = W.words_per_row(self.num_nodes)
+        ctx = self.ctx
+        # the previous step's kernels must be done with the device inputs
+        copy_stream.wait_stream(stream)
+        with torch.cuda.stream(copy_stream):
+            for k in ("offs", "exprs", "draws"):
+                n = host[k].numel()
+                dev[k][:n].copy_(host[k], non_blocking=True)
+        chunks = max(1, min(int(chunks), max(1, I // 4)))
+        # range edges on multiples of 4 intents (keeps every slice 16-byte aligned)
+        edges = [0] + [((I * c) // chunks) & ~3 for c in range(1, chunks)] + [I]
+        P = W.PROBE_DTYPE.itemsize
+        for lo, hi in zip(edges[:-1], edges[1:]):
+            if hi <= lo:
+                continue
+            n = hi - lo
+            with torch.cuda.stream(copy_stream):
+                dev["probes"][lo * ppg * P:hi * ppg * P].copy_(host["probes"][lo * ppg * P:hi * ppg * P],
+                                                                non_blocking=True)
+                ready = torch.cuda.Event()
+                ready.record(copy_stream)
+            stream.wait_event(ready)
+            bits = dev["bits"][lo * words * 4:]
+            flags = dev["flags"][lo:]
+            assign = dev["assign"][lo * pods * 4:]
+            probes = dev["probes"][lo * ppg * P:]
+            results = dev["results"][lo * ppg * 4:]
+            B.pv_eval_selectors(ctx, n, dev["offs"][lo * 4:], e2e_sizes["num_exprs"], dev["exprs"], None, bits,
+                                words, flags, stream)
+            B.pv_place_pods(ctx, n, pods, bits, words, dev["draws"][lo * pods * 8:], assign, stream)
+            B.pv_bind_probes(ctx, n * ppg, probes, ppg, pods, assign, stream)
+            B.pv_verify_probes(ctx, n * ppg, probes, e2e_sizes["hop_cap"], results, stream)
+            B.pv_aggregate_intents(ctx, n, pods, bits, words, flags, assign, ppg, results, dev["pass"][lo:],
+                                   dev["counts"][lo * 32:], stream)
+        with torch.cuda.stream(stream):
+            host["pass"].copy_(dev["pass"][: host["pass"].numel()], non_blocking=True)
+            host["counts"].copy_(dev["counts"][: host["counts"].numel()], non_blocking=True)
+        return host
+
     def alloc_end_to_end(self, e: W.EndToEnd) -> tuple:
         """Device buffers for an end-to-end workload (inputs uploaded)."""
         I, pods, ppg = e.intents.num_pods, e.pods_per_intent, e.probes_per_intent

@@ -136,3 +136,40 @@ def test_end_to_end_full_size_sampled(validator):
                                     assign[i * e.pods_per_intent:(i + 1) * e.pods_per_intent], e.pods_per_intent,
                                     r_i, ppg)
         assert g["pass"][i] == p_i[0] and (g["counts"][i] == c_i[0]).all()
+
+
+def _pinned(a):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1).copy()).pin_memory()
+
+
+@pytest.mark.parametrize("chunks", [1, 3, 7])
+def test_end_to_end_pipelined_from_host(validator, chunks):
+    """Host-buffer pipeline (probe upload of range c overlapped with the
+    verification of range c-1) gives the oracle's verdicts; the device
+    input buffers are zeroed first, so only the host copies can supply them."""
+    import torch
+    e = W.end_to_end(seed=22, num_switches=64, num_intents=301, probes_per_intent=120, rules_per_switch=200)
+    validator.load_cluster(e.cluster)
+    validator.load_network(e.network)
+    dev, sizes = validator.alloc_end_to_end(e)
+    for k in ("offs", "exprs", "draws", "probes"):
+        dev[k].zero_()
+    I = e.intents.num_pods
+    host = {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
+            "draws": _pinned(e.place_draws.astype(np.uint64)), "probes": _pinned(e.probes.probes),
+            "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
+            "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
+    stream = torch.cuda.current_stream()
+    validator.run_end_to_end_from_host(host, dev, sizes, stream, torch.cuda.Stream(), chunks)
+    stream.synchronize()
+    validator.sync()
+    bits, flags, assign, probes = _oracle_e2e(e)
+    res = oracle.verify_probes(e.network, probes, e.probes.hop_cap)
+    passed, counts = oracle.aggregate(bits, e.cluster.num_nodes, flags, assign, e.pods_per_intent, res,
+                                      e.probes_per_intent)
+    words = W.words_per_row(e.cluster.num_nodes)
+    assert (to_numpy(dev["bits"], np.uint32, (I, words)) == bits).all()
+    assert (to_numpy(dev["results"], W.RESULT_DTYPE) == res).all()
+    assert (host["pass"].numpy() == passed).all()
+    assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()

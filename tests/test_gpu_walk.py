@@ -193,6 +193,45 @@ def test_index_stress_tables(validator, seed):
     assert len(np.unique(o["status"])) >= 3
 
 
+def test_walk_live_total_counts_hop_entries(validator):
+    """PV_STAT_WALK_LIVE_TOTAL: probes entered at a switch, summed over hops.
+    A probe whose next switch (its first one included) lies outside its mask
+    is judged before it enters that switch, so it counts one entry fewer
+    than its result's hops."""
+    d = W.fat_tree(seed=5, k=4, rules_per_switch=100, num_probes=7000, hop_cap=8)
+    net, pr = d["network"], d["probes"].probes
+    g = _gpu_walk(validator, net, pr, 8)
+    o = oracle.verify_probes(net, pr, 8)
+    assert _same(g, o)
+    ran = o["status"] != W.ST_NOSRC
+    want = int(o["hops"][ran].astype(np.int64).sum()) - int((o["status"] == W.ST_VIOLATION).sum())
+    assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) == want
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_stalled_staging_wait_times_out_and_context_recovers(validator, kernel):
+    """A staging barrier that expects bytes no copy delivers: each hop block's
+    bounded wait runs out, pv_sync reports PV_ETIMEOUT, and the same context
+    then walks correctly (no fault, no hang)."""
+    d = W.fat_tree(seed=3, k=4, rules_per_switch=100, num_probes=5000, hop_cap=8)
+    net, pr = d["network"], d["probes"].probes
+    validator.load_network(net)
+    dev = validator.device
+    d_pr = to_device(pr, dev)
+    validator.set_option(B.PV_OPT_WALK_KERNEL, kernel)
+    validator.set_option(B.PV_OPT_TEST_STALL_STAGING, 1)
+    try:
+        validator.verify_probes(d_pr, len(pr), 8)
+        with pytest.raises(B.PVError) as e:
+            validator.sync()
+        assert e.value.code == B.PV_ETIMEOUT
+    finally:
+        validator.set_option(B.PV_OPT_TEST_STALL_STAGING, 0)
+        validator.set_option(B.PV_OPT_WALK_KERNEL, 0)
+    g = _gpu_walk(validator, net, pr, 8, kernel)
+    assert _same(g, oracle.verify_probes(net, pr, 8))
+
+
 @pytest.mark.parametrize("kernel", KERNELS)
 def test_flow_verification_full_size_sampled(validator, kernel):
     """The full flow-verification workload in the benchmark's launch
