@@ -230,7 +230,10 @@ int pv_verify_probes(pv_ctx *ctx, uint32_t num_probes, const pv_probe *d_probes,
  * Malformed CSR entries (decreasing offsets, offsets > num_edges, cols >= V,
  * region >= 32) are
  * skipped and reported as PV_EINVAL by the next pv_sync(); out-of-range
- * sources give empty rows.
+ * sources give empty rows.  When every remaining edge has its reverse (and
+ * no vertex has more than 64 out-edges) the rows are taken from the
+ * connected components of the permitted subgraph, which on such a graph is
+ * the same set (PV_OPT_REACH_KERNEL).
  * Errors: PV_EINVAL (V == 0, V > 16384, words_per_row too small or not a
  * multiple of 4, NULL pointers); PV_ENOMEM (scratch).
  * ------------------------------------------------------------------------- */
@@ -308,6 +311,9 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  * PV_OPT_WALK_LANE_MAX: with kernel 2, a batch of 32 probes is resolved one
  *   probe per lane when its longest candidate list has at most this many
  *   items (default 96), else one probe at a time by the whole warp.
+ * PV_OPT_REACH_KERNEL: 0 = automatic (on a symmetric graph, rows are the
+ *   connected components of the permitted subgraph; otherwise multi-source
+ *   pull sweeps), 1 = sweeps always.  Both give the same rows.
  * PV_OPT_TEST_STALL_STAGING: failure-injection switch for tests (0 or 1).
  *   When 1, each hop block's table-staging barrier expects 16 bytes more
  *   than its copy delivers, so its bounded wait runs out (after 50 ms rather
@@ -318,14 +324,17 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  *   usable), PV_STAT_WALK_INDEX_BYTES (largest per-switch table + index),
  *   PV_STAT_WALK_LIVE_TOTAL (probe-hop entries the last pv_verify_probes
  *   processed: the sum over its hops of the probes still walking; reading it
- *   synchronises with the device).
+ *   synchronises with the device), PV_STAT_REACH_COMPONENTS (1 if the last
+ *   pv_compliant_reach found its graph symmetric and wrote the rows from
+ *   components; synchronises).
  * ------------------------------------------------------------------------- */
 enum {
-    PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4
+    PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4,
+    PV_OPT_REACH_KERNEL = 5
 };
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,
-    PV_STAT_WALK_INDEX_BYTES = 4, PV_STAT_WALK_LIVE_TOTAL = 5
+    PV_STAT_WALK_INDEX_BYTES = 4, PV_STAT_WALK_LIVE_TOTAL = 5, PV_STAT_REACH_COMPONENTS = 6
 };
 int pv_set_option(pv_ctx *ctx, int option, int64_t value);
 int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value);

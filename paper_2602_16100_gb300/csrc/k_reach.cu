@@ -13,6 +13,16 @@
 // extends every search by at least one level).  The vertex-major words are
 // transposed with __ballot_sync into the caller's source-major bitset rows,
 // written with 128-bit stores.
+//
+// Symmetric graphs (every edge u -> v has its reverse v -> u) take an exact
+// shortcut: there a path s -> v inside the permitted vertices exists iff s
+// and v lie in the same connected component of the subgraph induced by the
+// permitted vertices, so R(s, m) is that component (or empty when s itself
+// is not permitted).  One block labels the components of one mask with a
+// lock-free union-find in shared memory, materialises the bitset of each
+// component its sources fall in, and copies those rows out: the output
+// write is the whole cost.  A device-side check decides per call which of
+// the two paths runs; both are launched and the other one returns at once.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -53,7 +63,8 @@ __global__ void reach_indeg_kernel(uint32_t V, uint32_t E, const uint32_t *__res
 // Single block: in_offs = exclusive scan of indeg (V+1 entries); cursor copy.
 __global__ void __launch_bounds__(1024) reach_scan_kernel(uint32_t V, const uint32_t *__restrict__ indeg,
                                                           uint32_t *__restrict__ in_offs,
-                                                          uint32_t *__restrict__ cursor) {
+                                                          uint32_t *__restrict__ cursor, const uint32_t *asym) {
+    if (asym && *(volatile const uint32_t *)asym == 0) return;   // symmetric: in-edges unused
     __shared__ uint32_t s_warp[32];
     __shared__ uint32_t s_carry;
     const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5;
@@ -92,7 +103,8 @@ __global__ void __launch_bounds__(1024) reach_scan_kernel(uint32_t V, const uint
 
 __global__ void reach_fill_kernel(uint32_t V, uint32_t E, const uint32_t *__restrict__ offs,
                                   const uint32_t *__restrict__ cols, uint32_t *__restrict__ cursor,
-                                  uint32_t *__restrict__ in_cols) {
+                                  uint32_t *__restrict__ in_cols, const uint32_t *asym) {
+    if (asym && *(volatile const uint32_t *)asym == 0) return;   // symmetric: in-edges unused
     for (uint32_t u = blockIdx.x * blockDim.x + threadIdx.x; u < V; u += gridDim.x * blockDim.x) {
         const uint32_t a = offs[u], b = offs[u + 1];
         if (b < a || b > E) continue;
@@ -103,16 +115,259 @@ __global__ void reach_fill_kernel(uint32_t V, uint32_t E, const uint32_t *__rest
     }
 }
 
-__global__ void __launch_bounds__(kReachThreads) reach_msbfs_kernel(
-    uint32_t V, const uint32_t *__restrict__ in_offs, const uint32_t *__restrict__ in_cols,
-    const uint8_t *__restrict__ region, uint32_t num_src, const uint32_t *__restrict__ src,
-    const uint32_t *__restrict__ masks, uint32_t *__restrict__ reach, uint32_t W) {
-    extern __shared__ uint64_t s_vis[];                 // [V]
-    __shared__ uint32_t s_allow[kReachMaxV / 32];
-    const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5;
+// Symmetry check of the caller's out-edge CSR, one warp per vertex:
+// *asym != 0 unless every edge u -> v (v < V, both lists well formed) has
+// its reverse v -> u.  Vertices whose list is longer than kSymScanMax make
+// the graph count as asymmetric (the sweep path then runs; still exact).
+// The same pass lists each undirected edge once, as pairs[] = u << 16 | v
+// with v < u (*npairs of them, in no particular order).
+constexpr uint32_t kSymScanMax = 64;
+
+__global__ void reach_symcheck_kernel(uint32_t V, uint32_t E, const uint32_t *__restrict__ offs,
+                                      const uint32_t *__restrict__ cols, uint32_t *asym, uint32_t *pairs,
+                                      uint32_t *npairs) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t nwarps = gridDim.x * (blockDim.x / 32);
+    for (uint32_t u = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32; u < V; u += nwarps) {
+        // warp-uniform early exit (lane 0's read decides for the warp)
+        if (__shfl_sync(PV_FULL_MASK, *(volatile uint32_t *)asym, 0)) return;
+        const uint32_t a = offs[u], b = offs[u + 1];
+        if (b < a || b > E) continue;
+        if (b - a > kSymScanMax) {
+            if (lane == 0) atomicOr(asym, 1u);
+            return;
+        }
+        for (uint32_t e0 = a; e0 < b; e0 += 32) {
+            const uint32_t e = e0 + lane;
+            uint32_t v = V;
+            bool ok = true;
+            if (e < b) {
+                v = cols[e];
+                if (v < V && v != u) {
+                    const uint32_t c = offs[v], d = offs[v + 1];
+                    bool found = false;
+                    if (!(d < c || d > E) && d - c <= kSymScanMax)
+                        for (uint32_t f = c; f < d && !found; ++f) found = cols[f] == u;
+                    ok = found;
+                }
+            }
+            if (__any_sync(PV_FULL_MASK, !ok)) {
+                if (lane == 0) atomicOr(asym, 1u);
+                return;
+            }
+            const bool keep = v < u;   // v < V too
+            const uint32_t bal = __ballot_sync(PV_FULL_MASK, keep);
+            uint32_t base = 0;
+            if (lane == 0 && bal) base = atomicAdd(npairs, (uint32_t)__popc(bal));
+            base = __shfl_sync(PV_FULL_MASK, base, 0);
+            if (keep) pairs[base + __popc(bal & ((1u << lane) - 1u))] = (u << 16) | v;
+        }
+    }
+}
+
+// Union-find over shared memory with parent[x] <= x at all times: roots are
+// hooked under smaller roots by compare-and-swap, finds halve paths (a
+// racing write only ever stores an ancestor).  A failed hook means the root
+// gained a parent, so the next attempt starts from a smaller root: at most
+// 2V attempts.
+__device__ __forceinline__ uint32_t uf_find(volatile uint32_t *parent, uint32_t x) {
+    for (;;) {
+        const uint32_t p = parent[x];
+        if (p == x) return x;
+        const uint32_t gp = parent[p];
+        if (gp != p) parent[x] = gp;
+        x = gp;
+    }
+}
+
+__device__ __forceinline__ void uf_union(volatile uint32_t *parent, uint32_t a, uint32_t b, uint32_t limit) {
+    for (uint32_t it = 0; it < limit; ++it) {
+        a = uf_find(parent, a);
+        b = uf_find(parent, b);
+        if (a == b) return;
+        if (a < b) {
+            const uint32_t x = a;
+            a = b;
+            b = x;
+        }
+        if (atomicCAS(const_cast<uint32_t *>(parent + a), a, b) == a) return;
+    }
+}
+
+constexpr int kCompThreads = 512;
+constexpr uint32_t kNoComp = 0xFFFFFFFFu;
+constexpr uint16_t kNoLabel = 0xFFFF;
+constexpr uint16_t kSlotNone = 0xFFFF, kSlotWanted = 0xFFFE, kSlotOverflow = 0xFFFD;
+
+__host__ __device__ inline uint32_t up16u(uint32_t x) { return (x + 15u) & ~15u; }
+
+// Component labels of one mask per block: lab[m][v] = the smallest vertex
+// of v's component in the permitted subgraph, kNoLabel for a vertex whose
+// region the mask does not permit.  Before the union pass every permitted
+// vertex points at its smallest permitted neighbour below it (a valid
+// forest of the same components, so most unions then find one root).
+constexpr int kLabelThreads = 1024;
+
+__global__ void __launch_bounds__(kLabelThreads) reach_labels_kernel(
+    uint32_t V, const uint32_t *__restrict__ pairs, const uint32_t *__restrict__ npairs,
+    const uint8_t *__restrict__ region, const uint32_t *__restrict__ masks, uint16_t *__restrict__ lab,
+    const uint32_t *asym) {
+    if (*(volatile const uint32_t *)asym) return;       // not symmetric: the sweep kernel runs
+    extern __shared__ __align__(16) uint8_t s_dyn[];
+    volatile uint32_t *parent = reinterpret_cast<uint32_t *>(s_dyn);              // [V]
+    uint32_t *s_allow = reinterpret_cast<uint32_t *>(s_dyn + up16u(V * 4));        // [ceil(V / 32)]
+    const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
+    const uint32_t m = blockIdx.x, mask = masks[m];
+    auto allowed = [&](uint32_t v) { return (s_allow[v >> 5] >> (v & 31)) & 1u; };
+    // every vertex its own root; permitted-vertex bitmap
+    for (uint32_t v0 = 0; v0 < V; v0 += nt) {
+        const uint32_t v = v0 + t;
+        bool ok = false;
+        if (v < V) {
+            const uint32_t r = region[v];
+            ok = r < 32 && ((mask >> r) & 1u);
+            parent[v] = v;
+        }
+        const uint32_t bal = __ballot_sync(PV_FULL_MASK, ok);
+        if (lane == 0 && v0 + warp * 32 < V) s_allow[(v0 >> 5) + warp] = bal;
+    }
+    __syncthreads();
+    // each permitted vertex under its smallest permitted neighbour
+    const uint32_t np = *npairs;
+    for (uint32_t i = 4 * t; i < np; i += 4 * nt) {
+        const uint4 q = *reinterpret_cast<const uint4 *>(pairs + i);
+        const uint32_t pq[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t u = pq[k] >> 16, v = pq[k] & 0xFFFFu;   // v < u
+            if (i + k < np && allowed(u) && allowed(v)) atomicMin(const_cast<uint32_t *>(parent + u), v);
+        }
+    }
+    __syncthreads();
+    // union the endpoints of every undirected edge inside the permitted
+    // vertices (the pair list holds each once; four pairs per load)
+    for (uint32_t i = 4 * t; i < np; i += 4 * nt) {
+        const uint4 q = *reinterpret_cast<const uint4 *>(pairs + i);
+        const uint32_t pq[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t u = pq[k] >> 16, v = pq[k] & 0xFFFFu;
+            if (i + k < np && allowed(u) && allowed(v)) uf_union(parent, u, v, 2 * V + 2);
+        }
+    }
+    __syncthreads();
+    uint16_t *out = lab + (size_t)m * V;
+    for (uint32_t v = t; v < V; v += nt) out[v] = allowed(v) ? (uint16_t)uf_find(parent, v) : kNoLabel;
+}
+
+struct RowSmem {   // dynamic shared-memory layout of reach_rows_kernel
+    uint32_t slot, slot_comp, rows, total;
+    __host__ __device__ RowSmem(uint32_t V, uint32_t W, uint32_t cap) {
+        slot = up16u(V * 4);
+        slot_comp = slot + up16u(V * 2);
+        rows = slot_comp + up16u(cap * 4);
+        total = rows + cap * W * 4;
+    }
+};
+
+// The bitset row of component c (all v < V with lab[v] == c; words past V
+// are zero), W / 4 uint4s written by one warp to dst (shared or global).
+__device__ __forceinline__ void comp_row(const uint32_t *lab, uint32_t V, uint32_t W, uint32_t c, uint4 *dst,
+                                         uint32_t lane) {
+    const uint32_t groups = W / 4;
+    for (uint32_t g0 = 0; g0 < groups; g0 += 32) {
+        uint4 mine = make_uint4(0, 0, 0, 0);
+        const uint32_t n = min(32u, groups - g0);
+        for (uint32_t i = 0; i < n; ++i) {
+            const uint32_t base = (g0 + i) * 128 + lane;
+            uint32_t bits[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const uint32_t v = base + 32 * k;
+                bits[k] = __ballot_sync(PV_FULL_MASK, v < V && lab[v] == c);
+            }
+            if (lane == i) mine = make_uint4(bits[0], bits[1], bits[2], bits[3]);
+        }
+        if (lane < n) dst[g0 + lane] = mine;
+    }
+}
+
+// Rows of one mask for a slice of sources: R(s, m) = the bitset of s's
+// component (empty when s is not permitted or out of range).  The
+// components the slice's sources fall in get a shared-memory row each
+// (first come, up to cap), built in one pass over the vertices; each output
+// row is then a 128-bit copy, or, past cap, built from ballots directly.
+__global__ void __launch_bounds__(kCompThreads) reach_rows_kernel(
+    uint32_t V, const uint16_t *__restrict__ lab_all, uint32_t num_src, const uint32_t *__restrict__ src,
+    uint32_t *__restrict__ reach, uint32_t W, uint32_t src_per_block, uint32_t cap, const uint32_t *asym) {
+    if (*(volatile const uint32_t *)asym) return;
+    extern __shared__ __align__(16) uint8_t s_dyn[];
+    const RowSmem L(V, W, cap);
+    uint32_t *s_lab = reinterpret_cast<uint32_t *>(s_dyn);
+    uint16_t *s_slot = reinterpret_cast<uint16_t *>(s_dyn + L.slot);
+    uint32_t *s_slot_comp = reinterpret_cast<uint32_t *>(s_dyn + L.slot_comp);
+    uint4 *s_rows = reinterpret_cast<uint4 *>(s_dyn + L.rows);
+    __shared__ uint32_t s_nslots;
+    const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x, nw = nt / 32;
     const uint32_t m = blockIdx.y;
-    const uint32_t j0 = blockIdx.x * 64, nb = min(64u, num_src - j0);
-    const uint32_t mask = masks[m];
+    const uint32_t j0 = blockIdx.x * src_per_block, j1 = min(num_src, j0 + src_per_block);
+    const uint16_t *lab = lab_all + (size_t)m * V;
+    for (uint32_t v = t; v < V; v += nt) {
+        const uint16_t l = lab[v];
+        s_lab[v] = l == kNoLabel ? kNoComp : l;
+        s_slot[v] = kSlotNone;
+    }
+    if (t == 0) s_nslots = 0;
+    __syncthreads();
+    for (uint32_t j = j0 + t; j < j1; j += nt) {
+        const uint32_t s = src[j];
+        if (s < V && s_lab[s] != kNoComp) s_slot[s_lab[s]] = kSlotWanted;
+    }
+    __syncthreads();
+    for (uint32_t v = t; v < V; v += nt)
+        if (s_slot[v] == kSlotWanted) {
+            const uint32_t k = atomicAdd(&s_nslots, 1u);
+            s_slot[v] = k < cap ? (uint16_t)k : kSlotOverflow;
+            if (k < cap) s_slot_comp[k] = v;
+        }
+    __syncthreads();
+    const uint32_t nsl = min(s_nslots, cap);
+    // slot rows: cleared, then every word written once by the lanes of the
+    // slot's component among its 32 vertices
+    for (uint32_t q = t; q < nsl * (W / 4); q += nt) s_rows[q] = make_uint4(0, 0, 0, 0);
+    __syncthreads();
+    uint32_t *s_words = reinterpret_cast<uint32_t *>(s_rows);
+    for (uint32_t v0 = warp * 32; v0 < V; v0 += nt) {
+        const uint32_t v = v0 + lane;
+        const uint32_t c = v < V ? s_lab[v] : kNoComp;
+        const uint32_t k = c != kNoComp ? s_slot[c] : kSlotNone;
+        const uint32_t peers = __match_any_sync(PV_FULL_MASK, k);
+        if (k < cap && lane == (uint32_t)(__ffs(peers) - 1)) s_words[(size_t)k * W + (v0 >> 5)] = peers;
+    }
+    __syncthreads();
+    for (uint32_t j = j0 + warp; j < j1; j += nw) {
+        const uint32_t s = src[j];
+        const uint32_t c = s < V ? s_lab[s] : kNoComp;
+        uint4 *out = reinterpret_cast<uint4 *>(reach + ((size_t)m * num_src + j) * W);
+        if (c == kNoComp) {
+            for (uint32_t q = lane; q < W / 4; q += 32) out[q] = make_uint4(0, 0, 0, 0);
+        } else if (s_slot[c] < cap) {
+            const uint4 *row = s_rows + (size_t)s_slot[c] * (W / 4);
+            for (uint32_t q = lane; q < W / 4; q += 32) out[q] = row[q];
+        } else {
+            comp_row(s_lab, V, W, c, out, lane);
+        }
+    }
+}
+
+// One work item of the sweep kernel: mask m, sources j0 .. j0 + 63.
+__device__ __forceinline__ void msbfs_item(uint32_t V, const uint32_t *__restrict__ in_offs,
+                                           const uint32_t *__restrict__ in_cols, const uint8_t *__restrict__ region,
+                                           uint32_t num_src, const uint32_t *__restrict__ src, uint32_t mask,
+                                           uint32_t *__restrict__ reach, uint32_t W, uint32_t m, uint32_t j0,
+                                           uint64_t *s_vis, uint32_t *s_allow) {
+    const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const uint32_t nb = min(64u, num_src - j0);
     volatile uint64_t *vis = s_vis;
     for (uint32_t v0 = 0; v0 < V; v0 += kReachThreads) {
         const uint32_t v = v0 + t;
@@ -172,6 +427,25 @@ __global__ void __launch_bounds__(kReachThreads) reach_msbfs_kernel(
     }
 }
 
+
+__global__ void __launch_bounds__(kReachThreads) reach_msbfs_kernel(
+    uint32_t V, const uint32_t *__restrict__ in_offs, const uint32_t *__restrict__ in_cols,
+    const uint8_t *__restrict__ region, uint32_t num_src, const uint32_t *__restrict__ src, uint32_t num_masks,
+    const uint32_t *__restrict__ masks, uint32_t *__restrict__ reach, uint32_t W, const uint32_t *asym) {
+    // the component path has written the rows of a symmetric graph
+    if (asym && *(volatile const uint32_t *)asym == 0) return;
+    extern __shared__ uint64_t s_vis[];                 // [V]
+    __shared__ uint32_t s_allow[kReachMaxV / 32];
+    const uint32_t nbatch = (num_src + 63) / 64;
+    const uint64_t items = (uint64_t)nbatch * num_masks;   // (mask, source batch) pairs
+    for (uint64_t item = blockIdx.x; item < items; item += gridDim.x) {
+        const uint32_t m = (uint32_t)(item / nbatch);
+        msbfs_item(V, in_offs, in_cols, region, num_src, src, masks[m], reach, W, m,
+                   (uint32_t)(item % nbatch) * 64, s_vis, s_allow);
+        __syncthreads();
+    }
+}
+
 }  // namespace
 
 extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_offs, uint32_t num_edges,
@@ -190,25 +464,87 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
     const size_t o_indeg = 0, o_in_offs = align256((size_t)(V + 1) * 4);
     const size_t o_cursor = o_in_offs + align256((size_t)(V + 1) * 4);
     const size_t o_cols = o_cursor + align256((size_t)V * 4);
-    const size_t total = o_cols + align256((size_t)num_edges * 4 + 4);
+    const size_t o_pairs = o_cols + align256((size_t)num_edges * 4 + 4);   // undirected pairs (+ count)
+    const size_t o_lab = o_pairs + align256((size_t)num_edges * 4 + 16) + 256;   // component labels
+    const bool comp = ctx->opt_reach == 0;
+    const size_t total = o_lab + (comp ? align256((size_t)num_masks * V * 2) : 0);
     uint8_t *base = (uint8_t *)pv_scratch(ctx, total);
     if (!base) return PV_ENOMEM;
     uint32_t *indeg = (uint32_t *)(base + o_indeg), *in_offs = (uint32_t *)(base + o_in_offs);
     uint32_t *cursor = (uint32_t *)(base + o_cursor), *in_cols = (uint32_t *)(base + o_cols);
+    uint32_t *pairs = (uint32_t *)(base + o_pairs);
+    uint32_t *npairs = (uint32_t *)(base + o_pairs + align256((size_t)num_edges * 4 + 16));
     cudaStream_t st = (cudaStream_t)stream;
+    // component path: row-slot cache sized to keep 3 blocks per SM when the
+    // fixed part allows it, at least one slot otherwise, none if even that
+    // does not fit (rows then come straight from the ballots)
+    uint32_t cap = 0;
+    size_t rows_smem = 0;
+    const size_t lab_smem = up16u(V * 4) + up16u(((V + 31) / 32) * 4);
+    const size_t limit = ctx->max_smem_optin - 1024;
+    if (comp) {
+        const size_t fixed = RowSmem(V, words_per_row, 0).total;
+        const size_t row = (size_t)words_per_row * 4 + 4;
+        const size_t budget = std::max<size_t>(72 * 1024, fixed + 16 * row);
+        if (fixed + row <= limit) cap = (uint32_t)std::min<size_t>((std::min(budget, limit) - fixed) / row, 0xFFF0);
+        rows_smem = RowSmem(V, words_per_row, cap).total;
+        if (rows_smem > limit) {
+            cap = 0;
+            rows_smem = RowSmem(V, words_per_row, 0).total;
+        }
+        if (rows_smem > limit) return pv_fail(ctx, PV_EINVAL, "pv_compliant_reach: words_per_row too large");
+    }
+    uint16_t *lab = (uint16_t *)(base + o_lab);   // [num_masks][V] (component path only)
     PV_TRY_CUDA(ctx, cudaMemsetAsync(indeg, 0, (size_t)(V + 1) * 4, st), "indeg clear");
+    if (comp) {
+        PV_TRY_CUDA(ctx, cudaMemsetAsync(ctx->d_reach_asym, 0, 4, st), "symmetry flag clear");
+        PV_TRY_CUDA(ctx, cudaMemsetAsync(npairs, 0, 4, st), "pair count clear");
+    }
+    ctx->last_reach_comp = comp;
+    const uint32_t *sym_flag = comp ? ctx->d_reach_asym : nullptr;
     const uint32_t grid = std::min<uint32_t>((V + kGridThreads - 1) / kGridThreads, (uint32_t)ctx->num_sms * 8);
     const int pr = pv_prof_start(ctx, st, PV_K_REACH);
+    uint32_t launches = 4;
     reach_indeg_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, d_region, indeg, ctx->d_status);
-    reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor);
-    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols);
+    if (comp) {
+        const uint32_t wgrid = std::min<uint32_t>((V + kGridThreads / 32 - 1) / (kGridThreads / 32),
+                                                  (uint32_t)ctx->num_sms * 8);
+        reach_symcheck_kernel<<<wgrid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, ctx->d_reach_asym, pairs,
+                                                              npairs);
+        launches += 3;
+    }
+    reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor, sym_flag);
+    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, sym_flag);
+    if (comp) {
+        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(reach_labels_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)lab_smem),
+                    "labels smem");
+        reach_labels_kernel<<<num_masks, kLabelThreads, lab_smem, st>>>(V, pairs, npairs, d_region, d_masks, lab,
+                                                                         ctx->d_reach_asym);
+        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(reach_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                              (int)rows_smem),
+                    "rows smem");
+        int per_sm = 1;
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reach_rows_kernel, kCompThreads, rows_smem);
+        // one wave of resident blocks over masks x source slices
+        const uint64_t want = (uint64_t)std::max(per_sm, 1) * ctx->num_sms;
+        const uint32_t slices = (uint32_t)std::max<uint64_t>(1, std::min<uint64_t>(num_src, want / num_masks));
+        const uint32_t spb = (num_src + slices - 1) / slices;
+        dim3 gc((num_src + spb - 1) / spb, num_masks);
+        reach_rows_kernel<<<gc, kCompThreads, rows_smem, st>>>(V, lab, num_src, d_src, d_reach, words_per_row, spb,
+                                                               cap, ctx->d_reach_asym);
+    }
     const size_t smem = (size_t)V * 8;
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(reach_msbfs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
                 "reach smem");
-    dim3 g2((num_src + 63) / 64, num_masks);
-    reach_msbfs_kernel<<<g2, kReachThreads, smem, st>>>(V, in_offs, in_cols, d_region, num_src, d_src, d_masks,
-                                                       d_reach, words_per_row);
-    pv_prof_stop(ctx, st, pr, 4);
+    int bfs_per_sm = 1;
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bfs_per_sm, reach_msbfs_kernel, kReachThreads, smem);
+    const uint64_t items = (uint64_t)((num_src + 63) / 64) * num_masks;
+    const uint32_t g2 = (uint32_t)std::min<uint64_t>(items, (uint64_t)std::max(bfs_per_sm, 1) * ctx->num_sms);
+    reach_msbfs_kernel<<<g2, kReachThreads, smem, st>>>(V, in_offs, in_cols, d_region, num_src, d_src, num_masks,
+                                                       d_masks, d_reach, words_per_row,
+                                                       comp ? ctx->d_reach_asym : nullptr);
+    pv_prof_stop(ctx, st, pr, launches);
     return pv_check_launch(ctx, "reach kernels");
 }
 
@@ -284,14 +620,15 @@ extern "C" int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, ui
         return PV_ECUDA;
     const uint32_t grid = std::min<uint32_t>((V + kGridThreads - 1) / kGridThreads, (uint32_t)sms * 8);
     reach_indeg_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, d_region, indeg, status);
-    reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor);
-    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols);
+    reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor, nullptr);
+    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, nullptr);
     const size_t smem = (size_t)V * 8;
     if (cudaFuncSetAttribute(reach_msbfs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
         cudaSuccess)
         return PV_ECUDA;
-    dim3 g2((num_src + 63) / 64, num_masks);
-    reach_msbfs_kernel<<<g2, kReachThreads, smem, st>>>(V, in_offs, in_cols, d_region, num_src, d_src, d_masks,
-                                                       d_reach, words_per_row);
+    const uint64_t items = (uint64_t)((num_src + 63) / 64) * num_masks;
+    const uint32_t g2 = (uint32_t)std::min<uint64_t>(items, (uint64_t)sms * 4);
+    reach_msbfs_kernel<<<g2, kReachThreads, smem, st>>>(V, in_offs, in_cols, d_region, num_src, d_src, num_masks,
+                                                       d_masks, d_reach, words_per_row, nullptr);
     return cudaGetLastError() == cudaSuccess ? PV_OK : PV_ECUDA;
 }

@@ -174,9 +174,11 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
         cudaMemset(ctx->d_status, 0, sizeof(int32_t)) != cudaSuccess ||
         pv_device_alloc(ctx, (void **)&ctx->d_walk_live, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t),
                         "walk statistics") != PV_OK ||
-        cudaMemset(ctx->d_walk_live, 0, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t)) != cudaSuccess) {
+        cudaMemset(ctx->d_walk_live, 0, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t)) != cudaSuccess ||
+        pv_device_alloc(ctx, (void **)&ctx->d_reach_asym, sizeof(uint32_t), "reach symmetry flag") != PV_OK) {
         pv_device_free(ctx->d_status);
         pv_device_free(ctx->d_walk_live);
+        pv_device_free(ctx->d_reach_asym);
         delete ctx;
         return PV_ENOMEM;
     }
@@ -193,6 +195,7 @@ extern "C" void pv_destroy(pv_ctx *ctx) {
     pv_device_free(ctx->scratch);
     pv_device_free(ctx->d_status);
     pv_device_free(ctx->d_walk_live);
+    pv_device_free(ctx->d_reach_asym);
     delete ctx;
 }
 
@@ -233,6 +236,10 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "stall-staging test switch must be 0 or 1");
         ctx->opt_test_stall_staging = (int)value;
         return PV_OK;
+    case PV_OPT_REACH_KERNEL:
+        if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "reach kernel must be 0 or 1");
+        ctx->opt_reach = (int)value;
+        return PV_OK;
     default:
         return pv_fail(ctx, PV_EINVAL, "unknown option %d", option);
     }
@@ -254,6 +261,14 @@ extern "C" int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value) {
         int64_t sum = 0;
         for (uint32_t h = 0; h < cap; ++h) sum += live[h];
         *value = sum;
+        return PV_OK;
+    }
+    case PV_STAT_REACH_COMPONENTS: {
+        uint32_t asym = 1;
+        if (ctx->last_reach_comp &&
+            cudaMemcpy(&asym, ctx->d_reach_asym, sizeof asym, cudaMemcpyDeviceToHost) != cudaSuccess)
+            return PV_ECUDA;
+        *value = (ctx->last_reach_comp && asym == 0) ? 1 : 0;
         return PV_OK;
     }
     default: return PV_EINVAL;

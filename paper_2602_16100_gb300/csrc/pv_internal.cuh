@@ -68,6 +68,9 @@ struct pv_ctx {
     int opt_test_stall_staging = 0;   // failure test: staging waits expect bytes that never come
     uint32_t *d_walk_live = nullptr;  // [PV_MAX_HOP_CAP + 1] live probes per hop of the last walk
     uint32_t last_walk_cap = 0;       // hop cap of the last walk
+    int opt_reach = 0;                // 0: components on symmetric graphs, 1: sweeps only
+    uint32_t *d_reach_asym = nullptr; // != 0: the last reach call's graph is not symmetric
+    bool last_reach_comp = false;     // the last reach call launched the component path
     void *scratch = nullptr;
     size_t scratch_bytes = 0;
     pv_cluster_state cl;

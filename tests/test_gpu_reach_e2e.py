@@ -44,6 +44,87 @@ def test_symmetric_wan_small_all_sources(validator):
     assert (gr == orr).all()
 
 
+def _symmetric(V, pairs, region):
+    """CSR with both directions of every pair (host-side test helper)."""
+    a = np.concatenate([pairs[:, 0], pairs[:, 1]]).astype(np.int64)
+    b = np.concatenate([pairs[:, 1], pairs[:, 0]]).astype(np.int64)
+    ab = np.unique(a * V + b)                       # sorted, no duplicate edges
+    a, b = ab // V, ab % V
+    offs = np.zeros(V + 1, np.int64)
+    np.add.at(offs, a + 1, 1)
+    return W.Graph(V, np.cumsum(offs).astype(np.uint32), b.astype(np.uint32), region.astype(np.uint8))
+
+
+def _reach_both(v, g, src, masks, words=None):
+    """Rows from the automatic path and from the sweeps alone, and whether
+    the automatic path took the component shortcut."""
+    auto = _gpu_reach(v, g, src, masks, words)
+    used = B.pv_get_stat(v.ctx, B.PV_STAT_REACH_COMPONENTS)
+    v.set_option(B.PV_OPT_REACH_KERNEL, 1)
+    try:
+        sweeps = _gpu_reach(v, g, src, masks, words)
+        assert B.pv_get_stat(v.ctx, B.PV_STAT_REACH_COMPONENTS) == 0
+    finally:
+        v.set_option(B.PV_OPT_REACH_KERNEL, 0)
+    return auto, sweeps, used
+
+
+@pytest.mark.parametrize("V,E,seed", [(1, 0, 1), (37, 40, 2), (1000, 2500, 3), (4097, 9000, 4), (16384, 30000, 5)])
+def test_symmetric_graphs_take_components(validator, V, E, seed):
+    st = W.Stream(seed, "sym-reach")
+    pairs = np.stack([st.ints(0, V - 1, E), st.ints(0, V - 1, E)], 1)
+    g = _symmetric(V, pairs, st.ints(0, 7, V))
+    src = st.ints(0, V - 1, 300).astype(np.uint32)
+    src[:3] = [0, V - 1, V + 5]                      # ends and an out-of-range source
+    masks = (st.u64(7) % np.uint64(256)).astype(np.uint32)
+    masks[0], masks[1] = 0xFFFFFFFF, 0
+    auto, sweeps, used = _reach_both(validator, g, src, masks)
+    assert used == 1
+    orr = oracle.compliant_reach(g, src, masks)
+    assert (auto == orr).all() and (sweeps == orr).all()
+
+
+def test_many_small_components_overflow_row_cache(validator):
+    """Every source in its own or a two-vertex component: far more distinct
+    components per block than row slots; plus padded rows (words_per_row
+    well above ceil(V/32)) that shrink the cache."""
+    V = 4096
+    pairs = np.stack([np.arange(0, V, 2), np.arange(1, V, 2)], 1)[::2]
+    g = _symmetric(V, pairs, np.arange(V) % 5)
+    src = np.arange(V, dtype=np.uint32)[::-1].copy()
+    masks = np.array([0xFFFFFFFF, 0b10110, 0b1], np.uint32)
+    orr = oracle.compliant_reach(g, src, masks)
+    auto, _, used = _reach_both(validator, g, src, masks)
+    assert used == 1 and (auto == orr).all()
+    words = W.words_per_row(V) + 1200
+    auto, _, used = _reach_both(validator, g, src, masks, words)
+    assert used == 1 and (auto == oracle.compliant_reach(g, src, masks, words=words)).all()
+
+
+def test_asymmetric_or_high_degree_graphs_take_sweeps(validator):
+    st = W.Stream(9, "asym-reach")
+    V = 600
+    pairs = np.stack([st.ints(0, V - 1, 1500), st.ints(0, V - 1, 1500)], 1)
+    g = _symmetric(V, pairs, st.ints(0, 5, V))
+    # drop one reverse edge: one direction of the first non-loop pair remains
+    k = int(np.nonzero(g.cols[: g.offs[-1]] != np.repeat(np.arange(V), np.diff(g.offs)))[0][0])
+    u = int(np.searchsorted(g.offs, k, side="right") - 1)
+    cols = np.delete(g.cols, k)
+    offs = g.offs.copy()
+    offs[u + 1:] -= 1
+    one_way = W.Graph(V, offs, cols, g.region)
+    # a hub with more out-edges than the symmetry check scans
+    hub = np.stack([np.zeros(100, np.int64), np.arange(1, 101)], 1)
+    star = _symmetric(V, np.concatenate([pairs, hub]), g.region)
+    src = np.arange(0, V, 3, dtype=np.uint32)
+    masks = np.array([0xFFFFFFFF, 0b111, 0b101010], np.uint32)
+    for graph in (one_way, star):
+        auto, sweeps, used = _reach_both(validator, graph, src, masks)
+        assert used == 0
+        orr = oracle.compliant_reach(graph, src, masks)
+        assert (auto == orr).all() and (sweeps == orr).all()
+
+
 def test_malformed_csr_is_reported(validator):
     g = W.random_digraph(3, 50, 200)
     cols = g.cols.copy()
