@@ -224,6 +224,35 @@ class EndToEndBench:
         v.load_network(e.network)
         v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks)
 
+    def e2e_phases(self, v, stream, reps=3):
+        """Each part of the host-buffer step alone (diagnostic, after the
+        timed region): the two table loads, the input upload, the device
+        pipeline on resident inputs."""
+        import torch
+        e = self.e
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            v.load_cluster(e.cluster)
+            v.load_network(e.network)
+        torch.cuda.synchronize()
+        load = (time.perf_counter() - t0) / reps
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            with torch.cuda.stream(self.copy_stream):
+                for k in ("offs", "exprs", "draws", "probes"):
+                    self.dev[k][: self.host[k].numel()].copy_(self.host[k], non_blocking=True)
+        torch.cuda.synchronize()
+        upload = (time.perf_counter() - t0) / reps
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            self.v.run_end_to_end(self.dev, self.sizes, stream)
+        torch.cuda.synchronize()
+        dev = (time.perf_counter() - t0) / reps
+        up_bytes = sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "probes"))
+        return {"load_tables_ms": load * 1e3, "upload_inputs_ms": upload * 1e3,
+                "upload_gbs": up_bytes / upload / 1e9, "device_pipeline_ms": dev * 1e3}
+
     # oracle on a bounded sample: the first n intents, whole pipeline
     def oracle_sample(self, n_intents):
         import oracle
@@ -555,6 +584,8 @@ def run_ours(args):
         e_s = SH.max_over_ranks(e_s, dist, "cuda")
         e2e = {"value": units * world / e_s, "unit": wl.unit, "h2d_bytes_per_step": int(wl.h2d),
                "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3, "upload_chunks": args.e2e_chunks}
+        if hasattr(wl, "e2e_phases"):
+            e2e["phases"] = wl.e2e_phases(v, stream)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

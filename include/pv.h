@@ -311,6 +311,12 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  * PV_OPT_WALK_LANE_MAX: with kernel 2, a batch of 32 probes is resolved one
  *   probe per lane when its longest candidate list has at most this many
  *   items (default 96), else one probe at a time by the whole warp.
+ * PV_OPT_WALK_CYCLES: 0 (default) = a probe found back at a (switch,
+ *   in_port) it already held is in a forwarding cycle (its header is fixed,
+ *   so its walk repeats); it walks only to the cycle position of hop
+ *   hop_cap - 1 and is finished there with the PV_LOOP result the full walk
+ *   gives (checkpoints at hops 4, 8, 16, ...); 1 = walk every hop to the cap.
+ *   Both give the same results; PV_STAT_WALK_LIVE_TOTAL differs.
  * PV_OPT_REACH_KERNEL: 0 = automatic (on a symmetric graph, rows are the
  *   connected components of the permitted subgraph; otherwise multi-source
  *   pull sweeps), 1 = sweeps always.  Both give the same rows.
@@ -330,7 +336,7 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  * ------------------------------------------------------------------------- */
 enum {
     PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4,
-    PV_OPT_REACH_KERNEL = 5
+    PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6
 };
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,

@@ -518,6 +518,21 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
     if (threadIdx.x == 0) desc[blockIdx.x] = make_uint2(c0, s_count);
 }
 
+// A live-list entry is uint2 {probe id, loc}: loc bits 0..7 in_port, 8..23
+// switch, 24..31 the hop at which a probe caught in a forwarding cycle is
+// finished (plus one; 0 = not known to cycle).
+__device__ __forceinline__ uint32_t entry_switch(uint32_t loc) { return (loc >> 8) & 0xFFFFu; }
+
+// Forwarding-cycle shortcut.  For a fixed header the next location depends
+// only on the current one (first match, action, port map, region check), so
+// once a probe is back at a location it visited, its walk repeats with that
+// period until the hop cap: it ends LOOP, hops = cap, at the switch it holds
+// at hop cap - 1.  Locations are compared with a checkpoint taken at hops 4,
+// 8, 16, ... (Brent's cycle detection); with period p found at hop h the
+// probe walks only (cap - 1 - h) mod p more hops and is then finished with
+// exactly the result the full walk gives.
+constexpr uint32_t kCycleCheckFrom = 4;
+
 // One block per list slice: per-switch histogram of the live probes.
 __global__ void __launch_bounds__(kGridThreads) walk_hist_kernel(const uint2 *__restrict__ list,
                                                                  const uint2 *__restrict__ desc, uint32_t S,
@@ -531,7 +546,7 @@ __global__ void __launch_bounds__(kGridThreads) walk_hist_kernel(const uint2 *__
         __syncthreads();
     }
     for (uint32_t i = d.x + threadIdx.x; i < d.x + d.y; i += kGridThreads) {
-        const uint32_t s = list[i].y >> 8;
+        const uint32_t s = entry_switch(list[i].y);
         if (use_smem) atomicAdd(&s_hist[s], 1u);
         else atomicAdd(&hist[s], 1u);
     }
@@ -542,18 +557,21 @@ __global__ void __launch_bounds__(kGridThreads) walk_hist_kernel(const uint2 *__
     }
 }
 
-// Single block: seg[s] = exclusive prefix of hist, seg[S] = total;
-// cursor[s] = seg[s]; hist cleared for the next hop.
+// Single block: seg[s] = exclusive prefix of hist, seg[S] = total,
+// seg[S + 1] = switches holding at least one probe; cursor[s] = seg[s];
+// hist cleared for the next hop.
 __global__ void __launch_bounds__(1024) walk_scan_kernel(uint32_t S, uint32_t *__restrict__ hist,
                                                          uint32_t *__restrict__ seg, uint32_t *__restrict__ cursor) {
     __shared__ uint32_t s_warp[32];
     __shared__ uint32_t s_carry;
     const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    uint32_t nonempty = 0;
     if (t == 0) s_carry = 0;
     __syncthreads();
     for (uint32_t c0 = 0; c0 < S; c0 += 1024) {
         const uint32_t i = c0 + t;
         const uint32_t x = i < S ? hist[i] : 0;
+        nonempty += (uint32_t)__syncthreads_count(x > 0);
         uint32_t incl = x;
         for (int d = 1; d < 32; d <<= 1) {
             uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
@@ -580,7 +598,10 @@ __global__ void __launch_bounds__(1024) walk_scan_kernel(uint32_t S, uint32_t *_
         if (t == 1023) s_carry = excl + x;
         __syncthreads();
     }
-    if (t == 0) seg[S] = s_carry;
+    if (t == 0) {
+        seg[S] = s_carry;
+        seg[S + 1] = nonempty;
+    }
 }
 
 // One block per list slice: block-aggregated counting-sort scatter (one
@@ -596,14 +617,14 @@ __global__ void __launch_bounds__(kGridThreads) walk_scatter_kernel(const uint2 
     if (S > kSmemHistMax) {
         for (uint32_t i = b0 + threadIdx.x; i < b1; i += kGridThreads) {
             const uint2 e = list[i];
-            sorted[atomicAdd(&cursor[e.y >> 8], 1u)] = e;
+            sorted[atomicAdd(&cursor[entry_switch(e.y)], 1u)] = e;
         }
         return;
     }
     uint32_t *s_base = s_cnt + S;
     for (uint32_t j = threadIdx.x; j < S; j += kGridThreads) s_cnt[j] = 0;
     __syncthreads();
-    for (uint32_t i = b0 + threadIdx.x; i < b1; i += kGridThreads) atomicAdd(&s_cnt[list[i].y >> 8], 1u);
+    for (uint32_t i = b0 + threadIdx.x; i < b1; i += kGridThreads) atomicAdd(&s_cnt[entry_switch(list[i].y)], 1u);
     __syncthreads();
     for (uint32_t j = threadIdx.x; j < S; j += kGridThreads) {
         const uint32_t c = s_cnt[j];
@@ -613,7 +634,7 @@ __global__ void __launch_bounds__(kGridThreads) walk_scatter_kernel(const uint2 
     __syncthreads();
     for (uint32_t i = b0 + threadIdx.x; i < b1; i += kGridThreads) {
         const uint2 e = list[i];
-        const uint32_t s = e.y >> 8;
+        const uint32_t s = entry_switch(e.y);
         sorted[s_base[s] + atomicAdd(&s_cnt[s], 1u)] = e;
     }
 }
@@ -638,6 +659,8 @@ struct HopArgs {
     uint32_t wait_extra; // bytes the staging barrier expects beyond the copy (0; > 0 only in failure tests)
     uint64_t wait_ns;    // bound on each staging wait
     uint32_t *hop_live;  // [cap]: live probes processed at each hop (statistics)
+    uint32_t *ck;        // [M]: cycle-detection checkpoint location per probe
+    uint32_t cycles;     // 1: finish probes caught in forwarding cycles early
 };
 
 // Linear first match: 32 consecutive rules per warp step.
@@ -824,9 +847,11 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t n = g.seg[g.S];   // live probes this hop
     if (blockIdx.x == 0 && threadIdx.x == 0) g.hop_live[g.hop] = n;
-    // only as many blocks as give each at least kMinPerBlock probes: a block
-    // stages a whole switch table, which small shares would not repay
-    const uint32_t active = max(1u, min(gridDim.x, (n + kMinPerBlock - 1) / kMinPerBlock));
+    // blocks: enough for kMinPerBlock probes each (a block stages a whole
+    // switch table, which small shares would not repay), but at least one per
+    // switch holding probes (else few blocks stage many tables one by one)
+    const uint32_t want = max((n + kMinPerBlock - 1) / kMinPerBlock, g.seg[g.S + 1]);
+    const uint32_t active = max(1u, min(gridDim.x, want));
     const uint32_t r0 = blockIdx.x < active ? (uint32_t)(((uint64_t)n * blockIdx.x) / active) : n;
     const uint32_t r1 = blockIdx.x < active ? (uint32_t)(((uint64_t)n * (blockIdx.x + 1)) / active) : n;
     if (r0 >= r1) {
@@ -884,7 +909,11 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
                 pr = __ldg(reinterpret_cast<const uint4 *>(g.probes) + e.x);
             }
-            uint32_t my_status = kAlive, my_next = 0;
+            // a probe in a known forwarding cycle that has reached its finish hop
+            const uint32_t fin = e.y >> 24;
+            const bool fin_now = lane < cnt && fin != 0 && fin - 1 == g.hop;
+            const uint32_t fin_lanes = __ballot_sync(PV_FULL_MASK, fin_now);
+            uint32_t my_status = fin_now ? (uint32_t)PV_LOOP : kAlive, my_next = 0;
             // Every listed probe is permitted at s (checked when it was handed
             // on).  Lane-per-probe when every candidate list of the batch is short.
             bool lane_mode = false;
@@ -898,10 +927,12 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 lane_mode = __reduce_max_sync(PV_FULL_MASK, len) <= g.lane_max;
             }
             if (lane_mode) {
-                const uint32_t fm = first_match_lane(s_raw, L, lane < cnt, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu);
-                if (lane < cnt) hop_outcome(g, fm, pr.y, pr.w, pbase, nports, &my_status, &my_next);
+                const bool act = lane < cnt && !fin_now;
+                const uint32_t fm = first_match_lane(s_raw, L, act, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu);
+                if (act) hop_outcome(g, fm, pr.y, pr.w, pbase, nports, &my_status, &my_next);
             } else {
                 for (uint32_t j = 0; j < cnt; ++j) {
+                    if ((fin_lanes >> j) & 1u) continue;
                     const uint32_t in_port = __shfl_sync(PV_FULL_MASK, e.y, j) & 0xFFu;
                     const uint32_t src = __shfl_sync(PV_FULL_MASK, pr.x, j);
                     const uint32_t dst = __shfl_sync(PV_FULL_MASK, pr.y, j);
@@ -921,13 +952,27 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 const bool at_next = my_status == kViolationNext;
                 pv_result r;
                 r.status = (uint8_t)(at_next ? (uint32_t)PV_VIOLATION : my_status);
-                r.hops = (uint8_t)(g.hop + (at_next ? 2u : 1u));
+                r.hops = (uint8_t)(fin_now ? g.cap : g.hop + (at_next ? 2u : 1u));
                 r.last_switch = (uint16_t)(at_next ? (my_next >> 8) : s);
                 g.out[e.x] = r;
             }
             const bool live = lane < cnt && my_status == kAlive;
+            uint32_t nloc = my_next;
+            if (live) {
+                uint32_t nfin = fin;
+                const uint32_t h1 = g.hop + 1;   // hop of the next visit (< cap)
+                if (g.cycles && nfin == 0 && h1 >= kCycleCheckFrom) {
+                    if ((h1 & (h1 - 1u)) == 0) {
+                        g.ck[e.x] = my_next;   // new checkpoint
+                    } else if (g.ck[e.x] == my_next) {
+                        const uint32_t period = h1 - (1u << (31 - __clz(h1)));
+                        nfin = h1 + (g.cap - 1u - h1) % period + 1u;
+                    }
+                }
+                nloc = my_next | (nfin << 24);
+            }
             const uint32_t slot = warp_reserve(live, &s_count);
-            if (live) g.next_list[r0 + slot] = make_uint2(e.x, my_next);
+            if (live) g.next_list[r0 + slot] = make_uint2(e.x, nloc);
         }
         pos = seg_end;
     }
@@ -1154,9 +1199,11 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     const size_t o_a = 0, o_b = align256((size_t)M * 8), o_sorted = o_b + align256((size_t)M * 8);
     const size_t o_hist = o_sorted + align256((size_t)M * 8);
     const size_t o_seg = o_hist + align256((size_t)S * 4);
-    const size_t o_cur = o_seg + align256((size_t)(S + 1) * 4);
+    const size_t o_cur = o_seg + align256((size_t)(S + 2) * 4);
     const size_t o_desc = o_cur + align256((size_t)S * 4);
-    const size_t total = o_desc + 2 * align256((size_t)max_desc * 8);
+    const size_t o_ck = o_desc + 2 * align256((size_t)max_desc * 8);
+    const bool cycles = ctx->opt_walk_cycles == 0 && hop_cap > kCycleCheckFrom;
+    const size_t total = o_ck + (cycles ? align256((size_t)M * 4) : 0);
     uint8_t *base = (uint8_t *)pv_scratch(ctx, total);
     if (!base) return PV_ENOMEM;
     uint2 *listA = (uint2 *)(base + o_a), *listB = (uint2 *)(base + o_b), *sorted = (uint2 *)(base + o_sorted);
@@ -1187,6 +1234,8 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     g.status = ctx->d_status;
     g.lane_max = (uint32_t)ctx->opt_walk_lane_max;
     g.hop_live = ctx->d_walk_live;
+    g.ck = (uint32_t *)(base + o_ck);
+    g.cycles = cycles ? 1u : 0u;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
     g.wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;

@@ -200,12 +200,66 @@ def test_walk_live_total_counts_hop_entries(validator):
     than its result's hops."""
     d = W.fat_tree(seed=5, k=4, rules_per_switch=100, num_probes=7000, hop_cap=8)
     net, pr = d["network"], d["probes"].probes
-    g = _gpu_walk(validator, net, pr, 8)
     o = oracle.verify_probes(net, pr, 8)
-    assert _same(g, o)
     ran = o["status"] != W.ST_NOSRC
     want = int(o["hops"][ran].astype(np.int64).sum()) - int((o["status"] == W.ST_VIOLATION).sum())
-    assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) == want
+    validator.set_option(B.PV_OPT_WALK_CYCLES, 1)      # every hop walked
+    try:
+        g = _gpu_walk(validator, net, pr, 8)
+        assert _same(g, o)
+        assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) == want
+    finally:
+        validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
+    g = _gpu_walk(validator, net, pr, 8)                # cycles finished early
+    assert _same(g, o)
+    assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) <= want
+
+
+def _cycle_network():
+    """Disjoint components, each a tail of t switches leading into a ring of
+    R switches (every switch forwards everything to its next port), one host
+    at the tail's head; one ring holds a switch of region 1.  Periods 1 (a
+    switch cabled to itself) to 40, cycle entry after 0 to 20 hops."""
+    nports, links, hosts, region, rules = [], [], [], [], []
+    combos = [(t, R) for t in (0, 1, 3, 5, 9, 20) for R in (1, 2, 3, 5, 8, 9, 13, 40)]
+    for c, (t, R) in enumerate(combos):
+        base = len(nports)
+        n = t + R
+        for i in range(n):
+            nports.append(3)                   # 0: in, 1: out, 2: host (head only)
+            region.append(1 if (c % 7 == 3 and i == t + R // 2) else 0)
+            rules.append([rule(100, 0, 0, 1)])  # everything out of port 1
+        for i in range(n - 1):
+            links.append((base + i, 1, base + i + 1, 0))
+        links.append((base + n - 1, 1, base + t, 0))   # close the ring
+        hosts.append((base, 2, ip(10, c, 0, 1)))
+    return make_net(nports, links, hosts, region, rules), len(combos)
+
+
+def test_forwarding_cycles_finish_with_the_full_walk_result(validator):
+    net, C = _cycle_network()
+    pr = np.concatenate([probe(h, ip(10, h, 0, 1), ip(99, 0, 0, 1), m, dport=h)
+                         for h in range(C) for m in (1, 3)])
+    for cap in (1, 2, 3, 4, 5, 7, 8, 9, 15, 16, 17, 31, 32, 33, 64, 100, 254, 255):
+        o = oracle.verify_probes(net, pr, cap)
+        for cyc in (0, 1):
+            validator.set_option(B.PV_OPT_WALK_CYCLES, cyc)
+            try:
+                for kernel in KERNELS:
+                    assert _same(_gpu_walk(validator, net, pr, cap, kernel), o), (cap, cyc, kernel)
+            finally:
+                validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
+        if cap == 255:
+            assert (o["status"] == W.ST_LOOP).sum() > C and (o["status"] == W.ST_VIOLATION).any()
+    # the shortcut does less work on the long cap
+    validator.set_option(B.PV_OPT_WALK_CYCLES, 1)
+    try:
+        _gpu_walk(validator, net, pr, 255)
+        full = B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL)
+    finally:
+        validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
+    _gpu_walk(validator, net, pr, 255)
+    assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) < full // 2
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
