@@ -184,8 +184,8 @@ __global__ void __launch_bounds__(1024) compile_tables_kernel(const uint32_t *__
 // a union of the segment's elementary intervals (each range contributes its
 // start and end + 1 as boundaries), so within a segment the first match of
 // address d is the precomputed winner of d's interval.
-constexpr uint32_t kBuckets = 64;           // dport >> kBucketShift
-constexpr uint32_t kBucketShift = 10;
+constexpr uint32_t kBuckets = 256;          // dport >> kBucketShift
+constexpr uint32_t kBucketShift = 8;
 constexpr uint32_t kMinSegment = 4;         // shorter destination-only runs stay plain items
 constexpr uint32_t kMaxSegment = 4096;      // longer runs are split (in order: still exact)
 constexpr uint32_t kMaxSegments = PV_MAX_RULES / kMinSegment;

@@ -17,6 +17,7 @@ pytestmark = pytest.mark.gpu
 
 
 KERNELS = [1, 2]   # linear first-match scan, indexed first match
+BUCKET = 256       # destination ports per bucket of the first-match index
 
 
 def _gpu_walk(v, net, probes, cap, kernel=0):
@@ -120,8 +121,8 @@ def test_empty_and_invalid_calls(validator):
 def _index_stress_network(seed, S=6, rules=700):
     """Ring of switches whose tables interleave destination-only runs with
     general rules: nested prefixes (/0 to /32) over a few addresses, priority
-    ties, port ranges straddling the 1024-port bucket edges, in_port rules
-    with full port ranges."""
+    ties, port ranges straddling the index's destination-port bucket edges,
+    in_port rules with full port ranges."""
     st = W.Stream(seed, "index-stress")
     hosts_per = 2
     H = S * hosts_per
@@ -142,7 +143,7 @@ def _index_stress_network(seed, S=6, rules=700):
         m = np.where(lens == 0, 0, (0xFFFFFFFF << (32 - lens)) & 0xFFFFFFFF).astype(np.uint64)
         r["dst_ip"] = (base & m).astype(np.uint32)
         r["dst_len"] = lens
-        edge = st.ints(1, 63, n) * 1024
+        edge = st.ints(1, 255, n) * BUCKET
         lo = np.clip(edge - st.ints(0, 3, n), 0, 65535)
         hi = np.clip(edge + st.ints(-1, 900, n), 0, 65535)
         r["dport_lo"] = np.where(dst_only, 0, np.minimum(lo, hi))
@@ -172,7 +173,7 @@ def test_index_stress_tables(validator, seed):
     pr["src_ip"] = np.where(st.floats(M) < 0.8, host_ip[src], st.u64(M) & np.uint64(0xFFFFFFFF))
     pr["dst_ip"] = np.where(st.floats(M) < 0.7, host_ip[st.ints(0, net.num_hosts - 1, M)],
                             st.u64(M) & np.uint64(0xFFFFFFFF))
-    edges = st.ints(0, 64, M) * 1024 + st.ints(-2, 2, M)
+    edges = st.ints(0, 256, M) * BUCKET + st.ints(-2, 2, M)
     pr["dport"] = np.where(st.floats(M) < 0.5, np.clip(edges, 0, 65535), st.ints(0, 65535, M))
     pr["allowed_mask"] = 0xF
     validator.load_network(net)
