@@ -278,16 +278,24 @@ __global__ void __launch_bounds__(1024) index_build_kernel(const uint32_t *__res
     const uint4 *a = A + t0;
     const uint2 *b = B + t0;
 
-    // 1. destination-only runs -> segments
+    // 1. destination-only runs -> segments.  The rules are classified and
+    //    their port ranges staged in parallel (s_keys is free until the
+    //    segment sort of step 3); one thread then walks the flags.
+    for (uint32_t i = t; i < n; i += nt) {
+        const uint2 bi = b[i];
+        s_cls[i] = rule_dst_only(a[i], bi) ? 1 : -1;
+        s_keys[i] = bi.x;   // dport lo | hi << 16
+    }
+    __syncthreads();
     if (t == 0) {
         uint32_t seg = 0, i = 0;
         while (i < n) {
-            if (!rule_dst_only(a[i], b[i])) {
-                s_cls[i++] = -1;
+            if (s_cls[i] < 0) {
+                ++i;
                 continue;
             }
             uint32_t j = i;
-            while (j < n && rule_dst_only(a[j], b[j])) ++j;
+            while (j < n && s_cls[j] > 0) ++j;
             if (j - i < kMinSegment) {
                 for (uint32_t k = i; k < j; ++k) s_cls[k] = -1;
             } else {
@@ -317,7 +325,7 @@ __global__ void __launch_bounds__(1024) index_build_kernel(const uint32_t *__res
         if (i >= n) return false;
         const int c = s_cls[i];
         if (c >= 0) return s_segs[2 * c] == i;   // segment token at its first rule
-        const uint32_t lo = b[i].x & 0xFFFFu, hi = b[i].x >> 16;
+        const uint32_t lo = s_keys[i] & 0xFFFFu, hi = s_keys[i] >> 16;
         return lo <= ((k << kBucketShift) | ((1u << kBucketShift) - 1u)) && hi >= (k << kBucketShift);
     };
     for (uint32_t k = warp; k < kBuckets; k += nt / 32) {
