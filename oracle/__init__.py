@@ -162,3 +162,51 @@ def aggregate(bits, num_nodes, group_flags, assign, pods_per_group, results, pro
                              _p(bits), ctypes.c_uint32(W), _p(gf), _p(assign), ctypes.c_uint32(probes_per_group),
                              _p(results), _p(passed), _p(counts))
     return passed, counts
+
+
+def _policy_arrays(pol):
+    return [np.ascontiguousarray(x) for x in (pol.forbid_offs.astype(np.uint32), pol.forbid.astype(np.uint16),
+                                              pol.must_offs.astype(np.uint32), pol.must.astype(np.uint16),
+                                              pol.concrete.astype(np.uint8))]
+
+
+def verify_constrained(net, probes, hop_cap, pol, probe_policy=None, probes_per_policy=0, idx=None):
+    """Walk with path constraints; returns (RESULT records, waypoint hit bits)."""
+    lib = _load()
+    probes = np.ascontiguousarray(probes)
+    ix = None if idx is None else np.ascontiguousarray(idx, np.uint32)
+    n = len(probes) if ix is None else len(ix)
+    out = np.zeros(n, _RESULT)
+    hits = np.zeros(n, np.uint32)
+    arr = [np.ascontiguousarray(x) for x in (net.rule_offs.astype(np.uint32), net.rules,
+                                             net.switch_region.astype(np.uint8), net.port_offs.astype(np.uint32),
+                                             net.port_peer.astype(np.int32), net.host_switch.astype(np.uint16),
+                                             net.host_port.astype(np.uint16), net.host_ip.astype(np.uint32))]
+    pp = None if probe_policy is None else np.ascontiguousarray(probe_policy, np.uint32)
+    fo, fb, mo, mg, _ = _policy_arrays(pol)
+    lib.oracle_verify_constrained(_p(arr[0]), _p(arr[1]), _p(arr[2]), _p(arr[3]), _p(arr[4]),
+                                  ctypes.c_uint32(net.num_hosts), _p(arr[5]), _p(arr[6]), _p(arr[7]), _p(probes),
+                                  _p(pp), ctypes.c_uint32(probes_per_policy), ctypes.c_uint32(pol.num_policies),
+                                  _p(fo), _p(fb), _p(mo), _p(mg), _p(ix), ctypes.c_uint32(n),
+                                  ctypes.c_uint32(hop_cap), _p(out), _p(hits))
+    return out, hits
+
+
+def aggregate_constrained(bits, num_nodes, group_flags, assign, pods_per_group, results, probes_per_group, hits,
+                          pol, group_policy=None):
+    bits = np.ascontiguousarray(bits, np.uint32)
+    G, W = bits.shape
+    gf = np.ascontiguousarray(group_flags, np.uint8)
+    assign = np.ascontiguousarray(assign, np.uint32)
+    results = np.ascontiguousarray(results)
+    hits = np.ascontiguousarray(hits, np.uint32)
+    gp = None if group_policy is None else np.ascontiguousarray(group_policy, np.uint32)
+    _, _, mo, _, cc = _policy_arrays(pol)
+    passed = np.zeros(G, np.uint8)
+    counts = np.zeros((G, 8), np.uint32)
+    _load().oracle_aggregate_constrained(ctypes.c_uint32(G), ctypes.c_uint32(pods_per_group),
+                                         ctypes.c_uint32(num_nodes), _p(bits), ctypes.c_uint32(W), _p(gf),
+                                         _p(assign), ctypes.c_uint32(probes_per_group), _p(results), _p(hits),
+                                         _p(gp), ctypes.c_uint32(pol.num_policies), _p(mo), _p(cc), _p(passed),
+                                         _p(counts))
+    return passed, counts

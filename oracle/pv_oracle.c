@@ -26,6 +26,11 @@
  *  - Compliant reach: the set of vertices reachable from a source over
  *    vertices whose region is permitted (Sec. 3.3 forbidden-vertex policy
  *    over G = (V, E); Sec. 4.2 graph search over the topology).
+ *  - Path constraints (Sec. 4.2 constraint object; Sec. 5.3 waypoint
+ *    intent; Sec. 5.5 network checks): forbidden switches are judged like
+ *    forbidden jurisdictions, required waypoints must be on the path; a
+ *    constraint naming no concrete flow is a no-op policy and fails
+ *    (Sec. 6.3, failure mode 2).
  *  - An intent passes only if all its checks pass (Sec. 5.5, validator
  *    check definition).
  *
@@ -36,7 +41,9 @@
  * Parity pins: selectors against a string-keyed brute force and the paper's
  * 5-worker label table; first-match against a sort-then-scan formulation and
  * hand cases; walks against hand-built topologies, a recursive path trace
- * and path invariants; reach against simple-path enumeration, union-find
+ * and path invariants; constrained walks against a path recorded without
+ * constraints and judged afterwards, and a hand-built waypoint case; reach
+ * against simple-path enumeration, union-find
  * components and monotonicity/symmetry; placement/aggregation by
  * composition and invariants.
  */
@@ -407,5 +414,128 @@ void oracle_aggregate(uint32_t num_groups, uint32_t pods_per_group, uint32_t num
             ok = ok && st == OR_COMPLIANT;
         }
         pass[g] = (uint8_t)ok;
+    }
+}
+
+/* ------------------------------------------------------------------------
+ * Path constraints of a flow set (Sec. 4.2: the constraint object handed to
+ * the flow scheduler names forbidden switches and must_go switches; Sec.
+ * 5.3, networking intent: the realised path must include the waypoint;
+ * Sec. 5.5: network checks assert that realised paths avoid forbidden
+ * switches and include required waypoints).
+ *
+ * Policy p: forbidden switches forbid[forbid_offs[p] .. forbid_offs[p+1]),
+ * required waypoints must[must_offs[p] .. must_offs[p+1]) (at most 32).
+ * Probe k follows policy probe_policy[k] (or k / probes_per_policy when
+ * probe_policy is NULL); a policy index >= num_policies means none.
+ *
+ * The walk is walk_one's with one more check at every switch visit: a
+ * forbidden switch is judged exactly like a switch outside the probe's
+ * jurisdictions (VIOLATION there, the walk stops).  Reading: a visit counts
+ * toward the waypoints only once it has passed these checks.  hits[k] bit i
+ * is set iff must[must_offs[p] + i] was visited.
+ * ---------------------------------------------------------------------- */
+static int in_list(const uint16_t *list, uint32_t n, uint32_t s) {
+    for (uint32_t i = 0; i < n; ++i)
+        if (list[i] == s) return 1;
+    return 0;
+}
+
+static or_result walk_constrained(const uint32_t *rule_offs, const or_rule *rules, const uint8_t *switch_region,
+                                  const uint32_t *port_offs, const int32_t *port_peer, uint32_t num_hosts,
+                                  const uint16_t *host_switch, const uint16_t *host_port, const uint32_t *host_ip,
+                                  const or_probe *pr, uint32_t hop_cap, const uint16_t *forbid, uint32_t nforbid,
+                                  const uint16_t *must, uint32_t nmust, uint32_t *hits) {
+    or_result res;
+    *hits = 0;
+    if (pr->src_host >= num_hosts) {
+        res.status = OR_NOSRC; res.hops = 0; res.last_switch = 0xFFFF;
+        return res;
+    }
+    uint32_t s = host_switch[pr->src_host];
+    uint32_t in_port = host_port[pr->src_host];
+    uint32_t last = s;
+    for (uint32_t h = 0; h < hop_cap; ++h) {
+        last = s;
+        res.hops = (uint8_t)(h + 1);
+        res.last_switch = (uint16_t)s;
+        uint32_t region = switch_region[s];
+        if (region >= 32 || !((pr->allowed_mask >> region) & 1u) || in_list(forbid, nforbid, s)) {
+            res.status = OR_VIOLATION;
+            return res;
+        }
+        for (uint32_t i = 0; i < nmust; ++i)
+            if (must[i] == s) *hits |= 1u << i;
+        uint32_t r0 = rule_offs[s], nr = rule_offs[s + 1] - r0;
+        int32_t m = oracle_first_match(rules + r0, nr, in_port, pr->src_ip, pr->dst_ip, pr->dport);
+        if (m < 0 || rules[r0 + m].action == OR_DROP) { res.status = OR_DROPPED; return res; }
+        uint32_t port = rules[r0 + m].action;
+        uint32_t nports = port_offs[s + 1] - port_offs[s];
+        if (port >= nports) { res.status = OR_DROPPED; return res; }
+        int32_t peer = port_peer[port_offs[s] + port];
+        if (peer < 0) { res.status = OR_DROPPED; return res; }
+        if (peer & OR_HOST_BIT) {
+            uint32_t q = (uint32_t)(peer & ~OR_HOST_BIT);
+            res.status = (q < num_hosts && host_ip[q] == pr->dst_ip) ? OR_COMPLIANT : OR_MISDELIVERED;
+            return res;
+        }
+        s = (uint32_t)peer >> 8;
+        in_port = (uint32_t)peer & 0xFFu;
+    }
+    res.status = OR_LOOP;
+    res.hops = (uint8_t)hop_cap;
+    res.last_switch = (uint16_t)last;
+    return res;
+}
+
+void oracle_verify_constrained(const uint32_t *rule_offs, const or_rule *rules, const uint8_t *switch_region,
+                               const uint32_t *port_offs, const int32_t *port_peer, uint32_t num_hosts,
+                               const uint16_t *host_switch, const uint16_t *host_port, const uint32_t *host_ip,
+                               const or_probe *probes, const uint32_t *probe_policy, uint32_t probes_per_policy,
+                               uint32_t num_policies, const uint32_t *forbid_offs, const uint16_t *forbid,
+                               const uint32_t *must_offs, const uint16_t *must, const uint32_t *idx, uint32_t count,
+                               uint32_t hop_cap, or_result *out, uint32_t *hits) {
+    for (uint32_t i = 0; i < count; ++i) {
+        uint32_t k = idx ? idx[i] : i;
+        uint32_t p = probe_policy ? probe_policy[k] : (probes_per_policy ? k / probes_per_policy : 0xFFFFFFFFu);
+        const uint16_t *fb = NULL, *mg = NULL;
+        uint32_t nf = 0, nm = 0;
+        if (p < num_policies) {
+            fb = forbid + forbid_offs[p];
+            nf = forbid_offs[p + 1] - forbid_offs[p];
+            mg = must + must_offs[p];
+            nm = must_offs[p + 1] - must_offs[p];
+        }
+        out[i] = walk_constrained(rule_offs, rules, switch_region, port_offs, port_peer, num_hosts, host_switch,
+                                  host_port, host_ip, &probes[k], hop_cap, fb, nf, mg, nm, &hits[i]);
+    }
+}
+
+/* Per-intent verdict with path constraints (Sec. 5.5: an intent passes only
+ * if all its checks pass).  On top of oracle_aggregate's checks, group g's
+ * policy p = group_policy[g] (or g when group_policy is NULL; p >=
+ * num_policies: none) must be concrete (Sec. 6.3, failure mode 2: a
+ * constraint object without a concrete src/dst applies to no flow, a no-op
+ * policy, and the intent is reported as not enforced) and every probe of g
+ * must have visited all of p's waypoints.  counts[g][7] = probes of g that
+ * missed a waypoint. */
+void oracle_aggregate_constrained(uint32_t num_groups, uint32_t pods_per_group, uint32_t num_nodes,
+                                  const uint32_t *bits, uint32_t words_per_row, const uint8_t *group_flags,
+                                  const uint32_t *assign, uint32_t probes_per_group, const or_result *results,
+                                  const uint32_t *hits, const uint32_t *group_policy, uint32_t num_policies,
+                                  const uint32_t *must_offs, const uint8_t *concrete, uint8_t *pass,
+                                  uint32_t *counts) {
+    oracle_aggregate(num_groups, pods_per_group, num_nodes, bits, words_per_row, group_flags, assign,
+                     probes_per_group, results, pass, counts);
+    for (uint32_t g = 0; g < num_groups; ++g) {
+        uint32_t p = group_policy ? group_policy[g] : g;
+        if (p >= num_policies) continue;
+        uint32_t nm = must_offs[p + 1] - must_offs[p];
+        uint32_t full = nm >= 32 ? 0xFFFFFFFFu : ((1u << nm) - 1u);
+        uint32_t missed = 0;
+        for (uint32_t k = 0; k < probes_per_group; ++k)
+            if (hits[(size_t)g * probes_per_group + k] != full) missed += 1;
+        counts[(size_t)g * 8 + 7] = missed;
+        if (!concrete[p] || missed) pass[g] = 0;
     }
 }

@@ -191,6 +191,16 @@ class EndToEnd:
     probes_per_intent: int
 
 
+@dataclasses.dataclass
+class PathPolicies:
+    num_policies: int
+    forbid_offs: np.ndarray       # u32 [P + 1]
+    forbid: np.ndarray            # u16: forbidden switches of each policy
+    must_offs: np.ndarray         # u32 [P + 1]
+    must: np.ndarray              # u16: required waypoints of each policy (<= 32)
+    concrete: np.ndarray          # u8 [P]: 1 if the constraint names a concrete (src, dst) flow
+
+
 # ----------------------------------------------------------------------------
 # helpers shared by the recipes
 # ----------------------------------------------------------------------------
@@ -789,3 +799,29 @@ def end_to_end(seed: int = 20260220, num_switches: int = 512, avg_degree: float 
     pr["allowed_mask"] = np.repeat(masks, probes_per_intent)
     return EndToEnd(cluster, intents, masks, pods_per_intent, draws, net, Probes(pr, hop_cap),
                     probes_per_intent)
+
+
+def path_policies(seed: int, net: Network, num_policies: int, forbid_max: int = 2, must_max: int = 3,
+                  hubs: int = 16, p_noop: float = 0.03) -> PathPolicies:
+    """Path-constraint objects for a network: per policy up to forbid_max
+    distinct forbidden switches drawn uniformly, U[0, must_max] waypoints
+    drawn among the `hubs` switches with the most ports (the backbone that
+    many paths cross), and with probability p_noop no concrete (src, dst)
+    flow (the constraint applies to nothing)."""
+    st = Stream(seed, "path-policies")
+    S = net.num_switches
+    hub = np.argsort(-np.diff(net.port_offs.astype(np.int64)), kind="stable")[: min(hubs, S)]
+    want_f = st.ints(0, forbid_max, num_policies)
+    nm = st.ints(0, min(must_max, len(hub)), num_policies)
+    fkeys = st.u64(num_policies * max(forbid_max, 1)).reshape(num_policies, max(forbid_max, 1))
+    mkeys = st.u64(num_policies * len(hub)).reshape(num_policies, len(hub))
+    forbid_lists = [np.unique((fkeys[p, : want_f[p]] % np.uint64(S)).astype(np.int64)) for p in range(num_policies)]
+    must_lists = [hub[np.argsort(mkeys[p], kind="stable")[: nm[p]]] for p in range(num_policies)]
+    fo = np.zeros(num_policies + 1, np.uint32)
+    fo[1:] = np.cumsum([len(f) for f in forbid_lists])
+    mo = np.zeros(num_policies + 1, np.uint32)
+    mo[1:] = np.cumsum(nm)
+    forbid = np.concatenate(forbid_lists).astype(np.uint16) if num_policies else np.zeros(0, np.uint16)
+    must = np.concatenate(must_lists).astype(np.uint16) if num_policies else np.zeros(0, np.uint16)
+    concrete = (st.floats(num_policies) >= p_noop).astype(np.uint8)
+    return PathPolicies(num_policies, fo, forbid, mo, must, concrete)

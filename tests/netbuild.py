@@ -109,3 +109,44 @@ def trace_walk(net, pr, cap):
     q = ev[1]
     ok = q < net.num_hosts and int(net.host_ip[q]) == hdr[1]
     return ((W.ST_COMPLIANT if ok else W.ST_MISDELIVERED), len(path), path[-1]), path
+
+
+def trace_walk_constrained(net, pr, cap, forbid, must):
+    """trace_walk's recorded path judged against a path constraint: the first
+    visited switch outside the jurisdictions or in `forbid` is a violation;
+    waypoint bit i is set iff must[i] is among the switches visited before
+    the walk ended (a violating switch does not count)."""
+    (status, hops, last), path = trace_walk(net, pr, 10 ** 6 if cap is None else cap)
+    pr = pr.reshape(-1)[0] if hasattr(pr, "reshape") else pr
+    if status == W.ST_NOSRC:
+        return (status, hops, last), 0
+    full_path, _ = _trace_path(net, pr, cap)
+    mask = int(pr["allowed_mask"])
+    for i, s in enumerate(full_path):
+        reg = int(net.switch_region[s])
+        if reg >= 32 or not (mask >> reg) & 1 or s in set(int(x) for x in forbid):
+            hit = sum(1 << j for j, m in enumerate(must) if int(m) in set(full_path[:i]))
+            return (W.ST_VIOLATION, i + 1, s), hit
+    hit = sum(1 << j for j, m in enumerate(must) if int(m) in set(full_path))
+    return (status, hops, last), hit
+
+
+def _trace_path(net, pr, cap):
+    """Switches visited ignoring every constraint, up to cap visits."""
+    src_host = int(pr["src_host"])
+    hdr = (int(pr["src_ip"]), int(pr["dst_ip"]), int(pr["dport"]))
+    s, p, path = int(net.host_switch[src_host]), int(net.host_port[src_host]), []
+    while len(path) < cap:
+        path.append(s)
+        rs = net.rules[net.rule_offs[s]:net.rule_offs[s + 1]]
+        i = first_match_sorted(rs, p, *hdr)
+        if i < 0 or int(rs[i]["action"]) == W.DROP:
+            break
+        port = int(rs[i]["action"])
+        if port >= int(net.port_offs[s + 1] - net.port_offs[s]):
+            break
+        peer = int(net.port_peer[net.port_offs[s] + port])
+        if peer < 0 or peer & W.HOST_BIT:
+            break
+        s, p = peer >> 8, peer & 0xFF
+    return path, None
