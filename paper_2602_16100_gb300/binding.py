@@ -29,7 +29,8 @@ PV_OPT_REACH_KERNEL, PV_OPT_WALK_CYCLES = 5, 6
 SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", "pv_load_cluster",
            "pv_eval_selectors", "pv_load_flow_tables", "pv_verify_probes", "pv_compliant_reach",
            "pv_place_pods", "pv_bind_probes", "pv_aggregate_intents", "pv_set_option", "pv_get_stat",
-           "pv_profile_enable", "pv_profile_collect", "pv_profile_read", "pv_compliant_reach_noalloc")
+           "pv_profile_enable", "pv_profile_collect", "pv_profile_read", "pv_compliant_reach_noalloc",
+           "pv_load_path_policies", "pv_verify_probes_constrained", "pv_aggregate_constrained")
 
 #: kernel groups timed by the library profiler (PV_K_* in include/pv.h)
 PV_K_NAMES = ("selector", "place", "bind", "walk_init", "walk_regroup", "walk_hop", "aggregate", "reach")
@@ -78,6 +79,9 @@ def load_library(path: Optional[str] = None):
         "pv_profile_read": (ctypes.c_int, [vp, ctypes.c_int, ctypes.POINTER(ctypes.c_double),
                                            ctypes.POINTER(ctypes.c_uint64)]),
         "pv_compliant_reach_noalloc": (ctypes.c_int, [u32, vp, u32, vp, vp, u32, vp, u32, vp, vp, u32, vp]),
+        "pv_load_path_policies": (ctypes.c_int, [vp, u32, vp, vp, vp, vp, vp]),
+        "pv_verify_probes_constrained": (ctypes.c_int, [vp, u32, vp, u32, vp, u32, vp, vp, vp]),
+        "pv_aggregate_constrained": (ctypes.c_int, [vp, u32, u32, vp, u32, vp, vp, u32, vp, vp, vp, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -207,6 +211,30 @@ def pv_load_flow_tables(ctx, num_switches, rule_offs, rules, switch_region, port
 def pv_verify_probes(ctx, num_probes, d_probes, hop_cap, d_out, stream=None) -> int:
     return _check(ctx, load_library().pv_verify_probes(ctx, num_probes, _dev(d_probes), hop_cap, _dev(d_out),
                                                        _stream(stream)))
+
+
+def pv_load_path_policies(ctx, num_policies, forbid_offs, forbid, must_offs, must, concrete) -> int:
+    a = [np.ascontiguousarray(forbid_offs, np.uint32), np.ascontiguousarray(forbid, np.uint16),
+         np.ascontiguousarray(must_offs, np.uint32), np.ascontiguousarray(must, np.uint16),
+         np.ascontiguousarray(concrete, np.uint8)]
+    return _check(ctx, load_library().pv_load_path_policies(ctx, num_policies, *[_host(x) for x in a]))
+
+
+def pv_verify_probes_constrained(ctx, num_probes, d_probes, hop_cap, d_probe_policy, probes_per_policy, d_out,
+                                 d_waypoints, stream=None) -> int:
+    return _check(ctx, load_library().pv_verify_probes_constrained(ctx, num_probes, _dev(d_probes), hop_cap,
+                                                                   _dev(d_probe_policy), probes_per_policy,
+                                                                   _dev(d_out), _dev(d_waypoints), _stream(stream)))
+
+
+def pv_aggregate_constrained(ctx, num_groups, pods_per_group, d_bits, words_per_row, d_group_flags, d_assign,
+                             probes_per_group, d_results, d_waypoints, d_group_policy, d_pass, d_counts,
+                             stream=None) -> int:
+    return _check(ctx, load_library().pv_aggregate_constrained(ctx, num_groups, pods_per_group, _dev(d_bits),
+                                                               words_per_row, _dev(d_group_flags), _dev(d_assign),
+                                                               probes_per_group, _dev(d_results),
+                                                               _dev(d_waypoints), _dev(d_group_policy),
+                                                               _dev(d_pass), _dev(d_counts), _stream(stream)))
 
 
 def pv_compliant_reach(ctx, V, d_offs, num_edges, d_cols, d_region, num_src, d_src, num_masks, d_masks, d_reach,

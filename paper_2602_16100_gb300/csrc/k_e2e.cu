@@ -89,7 +89,11 @@ __global__ void __launch_bounds__(kThreads) aggregate_kernel(uint32_t G, uint32_
                                                              const uint8_t *__restrict__ gflags,
                                                              const uint32_t *__restrict__ assign, uint32_t ppg,
                                                              const pv_result *__restrict__ results,
-                                                             uint8_t *__restrict__ pass, uint32_t *__restrict__ counts) {
+                                                             uint8_t *__restrict__ pass, uint32_t *__restrict__ counts,
+                                                             const uint32_t *__restrict__ hits,
+                                                             const uint32_t *__restrict__ group_pol, uint32_t num_pol,
+                                                             const uint4 *__restrict__ pol_hdr,
+                                                             const uint8_t *__restrict__ concrete) {
     const uint32_t lane = threadIdx.x & 31;
     for (uint32_t g = (blockIdx.x * kThreads + threadIdx.x) >> 5; g < G; g += (gridDim.x * kThreads) >> 5) {
         uint32_t placed = 0;
@@ -104,7 +108,21 @@ __global__ void __launch_bounds__(kThreads) aggregate_kernel(uint32_t G, uint32_
 #pragma unroll
             for (int s = 0; s < 6; ++s) c[s] += st == (uint32_t)s;
         }
+        // path constraints: every probe must have entered all waypoints of the
+        // group's policy, and the policy must name a concrete flow
+        uint32_t missed = 0;
+        bool policy_ok = true;
+        if (pol_hdr) {
+            const uint32_t p = group_pol ? group_pol[g] : g;
+            if (p < num_pol) {
+                const uint32_t nm = pol_hdr[p].w;
+                const uint32_t full = nm >= 32 ? 0xFFFFFFFFu : ((1u << nm) - 1u);
+                for (uint32_t k = lane; k < ppg; k += 32) missed += hits[(size_t)g * ppg + k] != full;
+                policy_ok = concrete[p] != 0;
+            }
+        }
         for (int d = 16; d > 0; d >>= 1) {
+            missed += __shfl_xor_sync(PV_FULL_MASK, missed, d);
             placed += __shfl_xor_sync(PV_FULL_MASK, placed, d);
 #pragma unroll
             for (int s = 0; s < 6; ++s) c[s] += __shfl_xor_sync(PV_FULL_MASK, c[s], d);
@@ -114,8 +132,9 @@ __global__ void __launch_bounds__(kThreads) aggregate_kernel(uint32_t G, uint32_
 #pragma unroll
             for (int s = 0; s < 6; ++s) out[s] = c[s];
             out[6] = placed;
-            out[7] = 0;
-            const bool ok = placed == pods && !(gflags[g] & (PV_F_UNKNOWN_VALUE | PV_F_BAD_EXPR)) && c[0] == ppg;
+            out[7] = missed;
+            const bool ok = placed == pods && !(gflags[g] & (PV_F_UNKNOWN_VALUE | PV_F_BAD_EXPR)) && c[0] == ppg &&
+                            policy_ok && missed == 0;
             pass[g] = ok ? 1 : 0;
         }
     }
@@ -172,7 +191,30 @@ extern "C" int pv_aggregate_intents(pv_ctx *ctx, uint32_t G, uint32_t pods, cons
     if (W < (ctx->cl.num_nodes + 31) / 32) return pv_fail(ctx, PV_EINVAL, "pv_aggregate_intents: words_per_row too small");
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_AGGREGATE);
     aggregate_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
-        G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts);
+        G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts, nullptr,
+        nullptr, 0, nullptr, nullptr);
+    pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    return pv_check_launch(ctx, "aggregate_kernel");
+}
+
+extern "C" int pv_aggregate_constrained(pv_ctx *ctx, uint32_t G, uint32_t pods, const uint32_t *d_bits, uint32_t W,
+                                        const uint8_t *d_gflags, const uint32_t *d_assign, uint32_t ppg,
+                                        const pv_result *d_results, const uint32_t *d_waypoints,
+                                        const uint32_t *d_group_policy, uint8_t *d_pass, uint32_t *d_counts,
+                                        pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->cl.loaded) return pv_fail(ctx, PV_ESTATE, "pv_aggregate_constrained: no cluster loaded");
+    if (!ctx->pol.loaded) return pv_fail(ctx, PV_ESTATE, "pv_aggregate_constrained: no path policies loaded");
+    if (G == 0) return PV_OK;
+    if (pods == 0) return pv_fail(ctx, PV_EINVAL, "pv_aggregate_constrained: pods_per_group must be > 0");
+    if (!d_bits || !d_gflags || !d_assign || !d_pass || !d_counts || (ppg && (!d_results || !d_waypoints)))
+        return pv_fail(ctx, PV_EINVAL, "pv_aggregate_constrained: NULL device pointer");
+    if (W < (ctx->cl.num_nodes + 31) / 32)
+        return pv_fail(ctx, PV_EINVAL, "pv_aggregate_constrained: words_per_row too small");
+    const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_AGGREGATE);
+    aggregate_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
+        G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts,
+        d_waypoints, d_group_policy, ctx->pol.num, ctx->pol.d_hdr, ctx->pol.d_concrete);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
     return pv_check_launch(ctx, "aggregate_kernel");
 }

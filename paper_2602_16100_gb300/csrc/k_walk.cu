@@ -480,12 +480,40 @@ __device__ __forceinline__ uint32_t warp_reserve(bool want, uint32_t *s_count) {
     return base + __popc(m & ((1u << lane) - 1u));
 }
 
+// Path constraints of the walk (Sec. 4.2 constraint object; Sec. 5.3 and
+// Sec. 5.5 waypoint and forbidden-switch checks).  Probe k follows policy
+// probe_pol[k] (or k / per when probe_pol is null); an index >= num means
+// none.  A forbidden switch is judged like a forbidden jurisdiction (checked
+// when the probe is handed to it, so it never enters); hits[k] bit i is set
+// once the probe has entered waypoint i of its policy.
+struct PolicyArgs {
+    const uint4 *hdr;          // [num] {forbid offset, count, waypoint offset, count}
+    const uint16_t *sw;        // switch ids
+    uint32_t num;
+    const uint32_t *probe_pol; // [M] or null
+    uint32_t per;              // probes per policy when probe_pol is null
+    uint32_t *hits;            // [M] waypoint bits (output)
+};
+
+__device__ __forceinline__ uint4 policy_of(const PolicyArgs &pa, uint32_t k) {
+    const uint32_t p = pa.probe_pol ? pa.probe_pol[k] : (pa.per ? k / pa.per : 0xFFFFFFFFu);
+    return p < pa.num ? pa.hdr[p] : make_uint4(0, 0, 0, 0);
+}
+
+__device__ __forceinline__ bool switch_listed(const uint16_t *list, uint32_t n, uint32_t s) {
+    for (uint32_t i = 0; i < n; ++i)
+        if (list[i] == s) return true;
+    return false;
+}
+
 // First visit of every probe: NOSRC for an absent source host, VIOLATION at
-// the attachment switch when its region is not permitted, otherwise listed.
+// the attachment switch when its region is not permitted (or, with path
+// constraints, the switch is forbidden to the probe), otherwise listed.
+template <bool kPolicy>
 __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
     uint32_t M, const pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
     const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
-    uint2 *__restrict__ list, uint2 *__restrict__ desc) {
+    uint2 *__restrict__ list, uint2 *__restrict__ desc, PolicyArgs pa) {
     __shared__ uint32_t s_count;
     const uint32_t c0 = (uint32_t)(((uint64_t)M * blockIdx.x) / gridDim.x);
     const uint32_t c1 = (uint32_t)(((uint64_t)M * (blockIdx.x + 1)) / gridDim.x);
@@ -500,10 +528,16 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
             const uint4 pr = __ldg(reinterpret_cast<const uint4 *>(probes) + i);
             const uint32_t h = pr.z >> 16;
             pv_result r;
+            if (kPolicy) pa.hits[i] = 0;
             if (h < H) {
                 const uint32_t s = host_switch[h];
                 const uint32_t reg = region[s];
-                if (reg < 32 && ((pr.w >> reg) & 1u)) {
+                bool ok = reg < 32 && ((pr.w >> reg) & 1u);
+                if (kPolicy && ok) {
+                    const uint4 ph = policy_of(pa, i);
+                    ok = !switch_listed(pa.sw + ph.x, ph.y, s);
+                }
+                if (ok) {
                     live = true;
                     loc = (s << 8) | host_port[h];
                 } else {
@@ -669,6 +703,7 @@ struct HopArgs {
     uint32_t *hop_live;  // [cap]: live probes processed at each hop (statistics)
     uint32_t *ck;        // [M]: cycle-detection checkpoint location per probe
     uint32_t cycles;     // 1: finish probes caught in forwarding cycles early
+    PolicyArgs pa;       // path constraints (used by the kPolicy kernels)
 };
 
 // Linear first match: 32 consecutive rules per warp step.
@@ -847,7 +882,7 @@ __device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t fm, uint3
     }
 }
 
-template <bool kIndexed>
+template <bool kIndexed, bool kPolicy>
 __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
     __shared__ uint64_t s_bar;
@@ -955,6 +990,15 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                         my_next = next;
                     }
                 }
+            }
+            if (kPolicy && lane < cnt && !fin_now) {
+                const uint4 ph = policy_of(g.pa, e.x);
+                uint32_t bits = 0;   // waypoints of the probe's policy at this switch
+                for (uint32_t i = 0; i < ph.w; ++i)
+                    if (g.pa.sw[ph.z + i] == s) bits |= 1u << i;
+                if (bits) g.pa.hits[e.x] |= bits;
+                if (my_status == kAlive && switch_listed(g.pa.sw + ph.x, ph.y, my_next >> 8))
+                    my_status = kViolationNext;   // the next switch is forbidden to this flow
             }
             if (lane < cnt && my_status != kAlive) {
                 const bool at_next = my_status == kViolationNext;
@@ -1166,13 +1210,20 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         pv_free_tables(t);
         return pv_fail(ctx, PV_EINVAL, "largest flow table needs %u bytes of shared memory", max_linear);
     }
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           (int)max_linear),
                 "walk_hop_kernel smem");
-    if (t.index_fits)
-        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              (int)max_blob),
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)max_linear),
+                "walk_hop_kernel smem");
+    if (t.index_fits) {
+        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<true, false>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_blob),
                     "walk_hop_kernel smem");
+        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<true, true>,
+                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_blob),
+                    "walk_hop_kernel smem");
+    }
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           (int)(2 * kSmemHistMax * 4)),
                 "walk_scatter_kernel smem");
@@ -1180,10 +1231,14 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     return PV_OK;
 }
 
-extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap,
-                                pv_result *d_out, pv_stream stream) {
-    if (!ctx) return PV_EINVAL;
+namespace {
+
+// The walk of pv_verify_probes; with pa, under the path constraints of
+// pv_verify_probes_constrained.
+int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap, pv_result *d_out,
+                const PolicyArgs *pa, pv_stream stream) {
     const pv_table_state &t = ctx->tb;
+    const bool pol = pa != nullptr;
     if (!t.loaded) return pv_fail(ctx, PV_ESTATE, "pv_verify_probes: no flow tables loaded");
     if (hop_cap == 0 || hop_cap > PV_MAX_HOP_CAP) return pv_fail(ctx, PV_EINVAL, "hop_cap must be 1..255");
     if (M == 0) return PV_OK;
@@ -1197,10 +1252,9 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     const bool indexed = which == 2;
     const size_t hop_smem = indexed ? t.max_blob_bytes : t.max_linear_bytes;
     int hop_blocks_per_sm = 0;
-    if (indexed)
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, walk_hop_kernel<true>, kHopThreads, hop_smem);
-    else
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, walk_hop_kernel<false>, kHopThreads, hop_smem);
+    const void *hop_fn = indexed ? (pol ? (const void *)walk_hop_kernel<true, true> : (const void *)walk_hop_kernel<true, false>)
+                                 : (pol ? (const void *)walk_hop_kernel<false, true> : (const void *)walk_hop_kernel<false, false>);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, hop_fn, kHopThreads, hop_smem);
     const uint32_t hop_grid = (uint32_t)ctx->num_sms * (uint32_t)std::max(1, hop_blocks_per_sm);
     const uint32_t init_grid = (uint32_t)ctx->num_sms * 8;
     const uint32_t max_desc = std::max(hop_grid, init_grid);
@@ -1221,8 +1275,14 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     cudaStream_t st = (cudaStream_t)stream;
     PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
-    walk_init_kernel<<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port,
-                                                         t.d_region, d_out, listA, descA);
+    const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, nullptr};
+    if (pol)
+        walk_init_kernel<true><<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch,
+                                                                   t.d_host_port, t.d_region, d_out, listA, descA, *pa);
+    else
+        walk_init_kernel<false><<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch,
+                                                                    t.d_host_port, t.d_region, d_out, listA, descA,
+                                                                    no_policy);
     pv_prof_stop(ctx, st, pr, 1);
     const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
@@ -1244,6 +1304,7 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
     g.hop_live = ctx->d_walk_live;
     g.ck = (uint32_t *)(base + o_ck);
     g.cycles = cycles ? 1u : 0u;
+    g.pa = pol ? *pa : no_policy;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
     g.wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
@@ -1263,12 +1324,84 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
         g.next_list = nxt;
         g.next_desc = dnxt;
         pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
-        if (indexed)
-            walk_hop_kernel<true><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+        if (indexed && pol)
+            walk_hop_kernel<true, true><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+        else if (indexed)
+            walk_hop_kernel<true, false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+        else if (pol)
+            walk_hop_kernel<false, true><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         else
-            walk_hop_kernel<false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+            walk_hop_kernel<false, false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         pv_prof_stop(ctx, st, pr, 1);
         in_slices = hop_grid;
     }
     return pv_check_launch(ctx, "probe walk kernels");
+}
+
+}  // namespace
+
+extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap,
+                                pv_result *d_out, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    return walk_probes(ctx, M, d_probes, hop_cap, d_out, nullptr, stream);
+}
+
+extern "C" int pv_verify_probes_constrained(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap,
+                                            const uint32_t *d_probe_policy, uint32_t probes_per_policy,
+                                            pv_result *d_out, uint32_t *d_waypoints, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->pol.loaded) return pv_fail(ctx, PV_ESTATE, "pv_verify_probes_constrained: no path policies loaded");
+    if (M && !d_waypoints) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes_constrained: NULL waypoint output");
+    const PolicyArgs pa = {ctx->pol.d_hdr, ctx->pol.d_sw, ctx->pol.num, d_probe_policy, probes_per_policy,
+                           d_waypoints};
+    return walk_probes(ctx, M, d_probes, hop_cap, d_out, &pa, stream);
+}
+
+extern "C" int pv_load_path_policies(pv_ctx *ctx, uint32_t num_policies, const uint32_t *forbid_offs,
+                                     const uint16_t *forbid, const uint32_t *must_offs, const uint16_t *must,
+                                     const uint8_t *concrete) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->tb.loaded) return pv_fail(ctx, PV_ESTATE, "pv_load_path_policies: load the flow tables first");
+    if (num_policies == 0 || !forbid_offs || !must_offs || !concrete)
+        return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: need num_policies > 0 and offset arrays");
+    if (forbid_offs[0] != 0 || must_offs[0] != 0)
+        return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: offsets must start at 0");
+    const uint32_t S = ctx->tb.num_switches;
+    std::vector<uint4> hdr(num_policies);
+    const uint32_t nf = forbid_offs[num_policies], nm = must_offs[num_policies];
+    if ((nf && !forbid) || (nm && !must)) return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: NULL switch list");
+    if ((uint64_t)nf + nm > 0xFFFFFFFFull) return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: lists too long");
+    for (uint32_t p = 0; p < num_policies; ++p) {
+        if (forbid_offs[p + 1] < forbid_offs[p] || must_offs[p + 1] < must_offs[p])
+            return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: policy %u: decreasing offsets", p);
+        const uint32_t fl = forbid_offs[p + 1] - forbid_offs[p], ml = must_offs[p + 1] - must_offs[p];
+        if (ml > 32) return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: policy %u has %u > 32 waypoints", p, ml);
+        hdr[p] = make_uint4(forbid_offs[p], fl, nf + must_offs[p], ml);
+    }
+    std::vector<uint16_t> sw((size_t)nf + nm);
+    for (uint32_t i = 0; i < nf; ++i) sw[i] = forbid[i];
+    for (uint32_t i = 0; i < nm; ++i) sw[(size_t)nf + i] = must[i];
+    for (size_t i = 0; i < sw.size(); ++i)
+        if (sw[i] >= S)
+            return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: switch id %u >= %u switches", (unsigned)sw[i], S);
+    pv_policy_state p;
+    int rc;
+    if ((rc = pv_device_alloc(ctx, (void **)&p.d_hdr, (size_t)num_policies * 16, "policy headers")) ||
+        (rc = pv_device_alloc(ctx, (void **)&p.d_sw, std::max<size_t>(sw.size(), 1) * 2, "policy switches")) ||
+        (rc = pv_device_alloc(ctx, (void **)&p.d_concrete, num_policies, "policy flags"))) {
+        pv_free_policies(p);
+        return rc;
+    }
+    cudaError_t e = cudaMemcpy(p.d_hdr, hdr.data(), (size_t)num_policies * 16, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && !sw.empty()) e = cudaMemcpy(p.d_sw, sw.data(), sw.size() * 2, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(p.d_concrete, concrete, num_policies, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) {
+        pv_free_policies(p);
+        return pv_cuda_fail(ctx, e, "pv_load_path_policies");
+    }
+    p.loaded = true;
+    p.num = num_policies;
+    pv_free_policies(ctx->pol);
+    ctx->pol = p;
+    return PV_OK;
 }

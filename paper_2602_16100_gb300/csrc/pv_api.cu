@@ -74,6 +74,13 @@ void pv_free_cluster(pv_cluster_state &c) {
     c = pv_cluster_state();
 }
 
+void pv_free_policies(pv_policy_state &p) {
+    pv_free_ptr(p.d_hdr);
+    pv_free_ptr(p.d_sw);
+    pv_free_ptr(p.d_concrete);
+    p = pv_policy_state();
+}
+
 void pv_free_tables(pv_table_state &t) {
     pv_free_ptr(t.d_blob);
     pv_free_ptr(t.d_blob_offs);
@@ -191,6 +198,7 @@ extern "C" void pv_destroy(pv_ctx *ctx) {
     cudaDeviceSynchronize();
     pv_free_cluster(ctx->cl);
     pv_free_tables(ctx->tb);
+    pv_free_policies(ctx->pol);
     for (cudaEvent_t e : ctx->prof.pool) cudaEventDestroy(e);
     pv_device_free(ctx->scratch);
     pv_device_free(ctx->d_status);

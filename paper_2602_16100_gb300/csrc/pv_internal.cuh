@@ -46,6 +46,16 @@ struct pv_table_state {
     uint32_t *d_host_ip = nullptr;
 };
 
+// Path constraints of flow sets (pv_load_path_policies): per policy
+// {forbidden offset, count, waypoint offset, count} into one switch list.
+struct pv_policy_state {
+    bool loaded = false;
+    uint32_t num = 0;
+    uint4 *d_hdr = nullptr;        // [num]
+    uint16_t *d_sw = nullptr;      // forbidden and waypoint switch ids
+    uint8_t *d_concrete = nullptr; // [num]: the constraint names a concrete flow
+};
+
 struct pv_prof_state {
     bool on = false;
     std::vector<cudaEvent_t> pool;     // event pairs: [2i] start, [2i+1] stop
@@ -76,6 +86,7 @@ struct pv_ctx {
     size_t scratch_bytes = 0;
     pv_cluster_state cl;
     pv_table_state tb;
+    pv_policy_state pol;
 };
 
 // -----------------------------------------------------------------------------
@@ -125,3 +136,4 @@ inline void pv_free_ptr(T *&p) {
 
 void pv_free_cluster(pv_cluster_state &c);
 void pv_free_tables(pv_table_state &t);
+void pv_free_policies(pv_policy_state &p);

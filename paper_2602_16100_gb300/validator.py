@@ -88,6 +88,21 @@ class Validator:
         B.pv_verify_probes(self.ctx, num_probes, d_probes, hop_cap, d_out, stream)
         return d_out
 
+    def load_policies(self, pol: W.PathPolicies):
+        B.pv_load_path_policies(self.ctx, pol.num_policies, pol.forbid_offs, pol.forbid, pol.must_offs, pol.must,
+                                pol.concrete)
+
+    def verify_constrained(self, d_probes, num_probes, hop_cap, d_probe_policy=None, probes_per_policy=0,
+                           d_out=None, d_waypoints=None, stream=None):
+        """Walk under the loaded path constraints; returns (results, waypoint bits)."""
+        if d_out is None:
+            d_out = empty_device(num_probes * 4, self.device)
+        if d_waypoints is None:
+            d_waypoints = empty_device(num_probes * 4, self.device)
+        B.pv_verify_probes_constrained(self.ctx, num_probes, d_probes, hop_cap, d_probe_policy, probes_per_policy,
+                                       d_out, d_waypoints, stream)
+        return d_out, d_waypoints
+
     def compliant_reach(self, graph_dev, num_src, d_src, num_masks, d_masks, words=None, d_reach=None,
                         stream=None):
         V, d_offs, E, d_cols, d_region = graph_dev

@@ -1,0 +1,152 @@
+"""GPU parity of the path-constraint checks against the oracle (bit-exact
+status, hops, last switch and waypoint bits): the backup-switch waypoint
+case, random networks and policies under both first-match kernels, hop caps
+that do and do not reach the forwarding-cycle shortcut, per-probe and
+strided policy indices, the constrained end-to-end verdict, invalid calls,
+and the full end-to-end workload with a policy per intent on sampled probes."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2602_16100_gb300 import binding as B
+from paper_2602_16100_gb300 import workloads as W
+from paper_2602_16100_gb300.validator import empty_device, to_device, to_numpy
+from gpu_util import sample
+from test_oracle_policies import _backup_switch_net, _policies
+from netbuild import probe
+
+pytestmark = pytest.mark.gpu
+
+
+def _walk(v, net, pol, pr, cap, probe_policy=None, per=0, kernel=0):
+    v.load_network(net)
+    v.load_policies(pol)
+    dev = v.device
+    dpp = None if probe_policy is None else to_device(np.asarray(probe_policy, np.uint32), dev)
+    v.set_option(B.PV_OPT_WALK_KERNEL, kernel)
+    try:
+        out, hits = v.verify_constrained(to_device(pr, dev), len(pr), cap, dpp, per)
+        v.sync()
+    finally:
+        v.set_option(B.PV_OPT_WALK_KERNEL, 0)
+    return to_numpy(out, W.RESULT_DTYPE), to_numpy(hits, np.uint32)
+
+
+@pytest.mark.parametrize("via_backup", [True, False])
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_backup_switch_waypoint(validator, via_backup, kernel):
+    net, H2, H4 = _backup_switch_net(via_backup)
+    pol = _policies([[], [8], [5]], [[8], [8], [8, 5]])
+    pr = np.concatenate([probe(0, H2, H4, 1)] * 4)
+    pp = np.array([0, 1, 2, 9], np.uint32)
+    g, gh = _walk(validator, net, pol, pr, 16, pp, kernel=kernel)
+    o, oh = oracle.verify_constrained(net, pr, 16, pol, probe_policy=pp)
+    assert (g == o).all() and (gh == oh).all()
+
+
+@pytest.mark.parametrize("seed,cap", [(0, 24), (1, 32), (2, 3), (3, 255)])
+@pytest.mark.parametrize("kernel", [1, 2])
+def test_random_policies(validator, seed, cap, kernel):
+    e = W.end_to_end(seed=60 + seed, num_switches=80, num_intents=50, probes_per_intent=200, rules_per_switch=200,
+                     hop_cap=cap)
+    net = e.network
+    pol = W.path_policies(seed, net, 50, forbid_max=3, must_max=4, hubs=10)
+    pr = e.probes.probes.copy()
+    st = W.Stream(seed, "gpu-policy-probes")
+    H = net.num_hosts
+    pr["src_host"] = st.ints(0, H - 1, len(pr))
+    pr["src_ip"] = net.host_ip[pr["src_host"]]
+    pr["src_host"][::23] = W.NO_HOST
+    pr["allowed_mask"][::3] = 0xFFFFFFFF
+    g, gh = _walk(validator, net, pol, pr, cap, per=200, kernel=kernel)
+    o, oh = oracle.verify_constrained(net, pr, cap, pol, probes_per_policy=200)
+    assert (g == o).all() and (gh == oh).all()
+    assert (oh != 0).any() and (o["status"] == W.ST_VIOLATION).any()
+    # explicit policy indices, some past the table (no constraint: the plain walk)
+    pp = (np.arange(len(pr)) % 57).astype(np.uint32)
+    g2, gh2 = _walk(validator, net, pol, pr, cap, pp, kernel=kernel)
+    o2, oh2 = oracle.verify_constrained(net, pr, cap, pol, probe_policy=pp)
+    assert (g2 == o2).all() and (gh2 == oh2).all()
+    plain = pp >= 50
+    assert (o2[plain] == oracle.verify_probes(net, pr[plain], cap)).all() and not oh2[plain].any()
+
+
+def test_constrained_end_to_end(validator):
+    e = W.end_to_end(seed=25, num_switches=64, num_intents=300, probes_per_intent=100, rules_per_switch=200)
+    pol = W.path_policies(7, e.network, 300, forbid_max=1, must_max=2, hubs=6, p_noop=0.1)
+    v = validator
+    v.load_cluster(e.cluster)
+    v.load_network(e.network)
+    v.load_policies(pol)
+    dev, sizes = v.alloc_end_to_end(e)
+    I, pods, ppg = sizes["intents"], sizes["pods"], sizes["probes_per_intent"]
+    words = W.words_per_row(e.cluster.num_nodes)
+    B.pv_eval_selectors(v.ctx, I, dev["offs"], sizes["num_exprs"], dev["exprs"], None, dev["bits"], words,
+                        dev["flags"])
+    B.pv_place_pods(v.ctx, I, pods, dev["bits"], words, dev["draws"], dev["assign"])
+    B.pv_bind_probes(v.ctx, I * ppg, dev["probes"], ppg, pods, dev["assign"])
+    hits = empty_device(I * ppg * 4, v.device)
+    B.pv_verify_probes_constrained(v.ctx, I * ppg, dev["probes"], sizes["hop_cap"], None, ppg, dev["results"], hits)
+    B.pv_aggregate_constrained(v.ctx, I, pods, dev["bits"], words, dev["flags"], dev["assign"], ppg, dev["results"],
+                               hits, None, dev["pass"], dev["counts"])
+    v.sync()
+    c = e.cluster
+    bits, flags = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, e.intents.expr_offs, e.intents.exprs)
+    assign = oracle.place_pods(bits, c.num_nodes, pods, e.place_draws)
+    probes = oracle.bind_probes(e.probes.probes, ppg, pods, assign, e.network.host_ip)
+    res, oh = oracle.verify_constrained(e.network, probes, e.probes.hop_cap, pol, probes_per_policy=ppg)
+    passed, counts = oracle.aggregate_constrained(bits, c.num_nodes, flags, assign, pods, res, ppg, oh, pol)
+    assert (to_numpy(dev["results"], W.RESULT_DTYPE) == res).all()
+    assert (to_numpy(hits, np.uint32) == oh).all()
+    assert (to_numpy(dev["pass"], np.uint8)[:I] == passed).all()
+    assert (to_numpy(dev["counts"], np.uint32, (I, 8)) == counts).all()
+    assert counts[:, 7].any()
+
+
+def test_invalid_policy_calls(validator):
+    d = W.tiny()
+    net = d["network"]
+    fresh = B.pv_create(validator.device.index)
+    try:
+        with pytest.raises(B.PVError) as e:     # no flow tables yet
+            B.pv_load_path_policies(fresh, 1, np.array([0, 0], np.uint32), np.zeros(0, np.uint16),
+                                    np.array([0, 1], np.uint32), np.array([1], np.uint16), np.ones(1, np.uint8))
+        assert e.value.code == B.PV_ESTATE
+    finally:
+        B.pv_destroy(fresh)
+    validator.load_network(net)
+    S = net.num_switches
+    bad = [(np.array([0, 0], np.uint32), np.zeros(0, np.uint16), np.array([0, 33], np.uint32),
+            np.zeros(33, np.uint16)),                                           # > 32 waypoints
+           (np.array([0, 1], np.uint32), np.array([S], np.uint16), np.array([0, 0], np.uint32),
+            np.zeros(0, np.uint16)),                                            # switch out of range
+           (np.array([0, 2, 1], np.uint32), np.zeros(2, np.uint16), np.array([0, 0, 0], np.uint32),
+            np.zeros(0, np.uint16))]                                            # decreasing offsets
+    for fo, f, mo, m in bad:
+        with pytest.raises(B.PVError) as e:
+            B.pv_load_path_policies(validator.ctx, len(fo) - 1, fo, f, mo, m, np.ones(len(fo) - 1, np.uint8))
+        assert e.value.code == B.PV_EINVAL
+    pr = to_device(d["probes"].probes, validator.device)
+    out = empty_device(4 * len(d["probes"].probes), validator.device)
+    validator.load_policies(_policies([[1]], [[2]]))
+    with pytest.raises(B.PVError):                                              # NULL waypoint output
+        B.pv_verify_probes_constrained(validator.ctx, 10, pr, 16, None, 10, out, None)
+
+
+def test_full_size_end_to_end_policies_sampled(validator):
+    """The full end-to-end workload (10,000 intents, 50M probes) with one
+    policy per intent; the oracle walks a sample of probes."""
+    e = W.end_to_end()
+    pol = W.path_policies(11, e.network, e.intents.num_pods)
+    v = validator
+    v.load_network(e.network)
+    v.load_policies(pol)
+    pr = e.probes.probes.copy()
+    st = W.Stream(12, "full-policy-probes")
+    pr["src_host"] = st.ints(0, e.network.num_hosts - 1, len(pr))
+    pr["src_ip"] = e.network.host_ip[pr["src_host"]]
+    g, gh = _walk(v, e.network, pol, pr, e.probes.hop_cap, per=e.probes_per_intent)
+    idx = sample(len(pr), 20000, seed=5)
+    o, oh = oracle.verify_constrained(e.network, pr, e.probes.hop_cap, pol, probes_per_policy=e.probes_per_intent,
+                                      idx=idx)
+    assert (g[idx] == o).all() and (gh[idx] == oh).all()
