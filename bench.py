@@ -139,8 +139,12 @@ class EndToEndBench:
     name = "end-to-end cross-layer"
     unit = "probe-hop verifications/s"
 
-    def __init__(self, seed, intents=None):
+    def __init__(self, seed, intents=None, policies=False):
         self.e = W.end_to_end(seed=20260220 + seed, **({"num_intents": intents} if intents else {}))
+        # path constraints (forbidden switches, waypoints), one policy per intent
+        self.pol = W.path_policies(20260221 + seed, self.e.network, self.e.intents.num_pods) if policies else None
+        if policies:
+            self.name = "end-to-end cross-layer with path constraints"
 
     def config(self):
         e = self.e
@@ -148,13 +152,17 @@ class EndToEndBench:
                 "label_keys": e.cluster.num_keys, "switches": e.network.num_switches,
                 "rules_per_switch": int(np.diff(e.network.rule_offs).max()), "pods_per_intent": e.pods_per_intent,
                 "probes": len(e.probes.probes), "hop_cap": e.probes.hop_cap,
-                "l2": "inputs larger than L2 (800 MB probe array and 200 MB results per step)"}
+                "l2": "inputs larger than L2 (800 MB probe array and 200 MB results per step)",
+                **({"path_policies": self.pol.num_policies, "forbidden_switches": len(self.pol.forbid),
+                    "waypoints": len(self.pol.must)} if self.pol is not None else {})}
 
     def setup(self, v):
         self.v = v
         v.load_cluster(self.e.cluster)
         v.load_network(self.e.network)
-        self.dev, self.sizes = v.alloc_end_to_end(self.e)
+        if self.pol is not None:
+            v.load_policies(self.pol)
+        self.dev, self.sizes = v.alloc_end_to_end(self.e, with_policies=self.pol is not None)
 
     def step(self, stream):
         self.v.run_end_to_end(self.dev, self.sizes, stream)
@@ -222,6 +230,8 @@ class EndToEndBench:
         e = self.e
         v.load_cluster(e.cluster)
         v.load_network(e.network)
+        if self.pol is not None:
+            v.load_policies(self.pol)
         v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks)
 
     def e2e_phases(self, v, stream, reps=3):
@@ -235,6 +245,8 @@ class EndToEndBench:
         for _ in range(reps):
             v.load_cluster(e.cluster)
             v.load_network(e.network)
+            if self.pol is not None:
+                v.load_policies(self.pol)
         torch.cuda.synchronize()
         load = (time.perf_counter() - t0) / reps
         t0 = time.perf_counter()
@@ -265,8 +277,12 @@ class EndToEndBench:
         bits, flags = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, offs, exprs)
         assign = oracle.place_pods(bits, c.num_nodes, pods, e.place_draws[: n_intents * pods])
         probes = oracle.bind_probes(e.probes.probes[: n_intents * ppg], ppg, pods, assign, e.network.host_ip)
-        res = oracle.verify_probes(e.network, probes, e.probes.hop_cap)
-        oracle.aggregate(bits, c.num_nodes, flags, assign, pods, res, ppg)
+        if self.pol is None:
+            res = oracle.verify_probes(e.network, probes, e.probes.hop_cap)
+            oracle.aggregate(bits, c.num_nodes, flags, assign, pods, res, ppg)
+        else:
+            res, hits = oracle.verify_constrained(e.network, probes, e.probes.hop_cap, self.pol, probes_per_policy=ppg)
+            oracle.aggregate_constrained(bits, c.num_nodes, flags, assign, pods, res, ppg, hits, self.pol)
         dt = time.perf_counter() - t0
         units = int(res["hops"].astype(np.int64).sum())
         return units, dt, f"first {n_intents} intents ({n_intents * ppg} probes), whole pipeline"
@@ -448,7 +464,8 @@ class WanBench:
         return len(self.q.masks) * len(self.q.sources)
 
 
-WORKLOADS = {"e2e": EndToEndBench, "placement": PlacementBench, "flow": FlowBench, "wan": WanBench}
+WORKLOADS = {"e2e": EndToEndBench,
+             "e2e_policies": lambda seed, **kw: EndToEndBench(seed, policies=True, **kw), "placement": PlacementBench, "flow": FlowBench, "wan": WanBench}
 SOURCES = {"walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector": ("k_selector.cu",),
            "reach": ("k_reach.cu",)}
 
@@ -620,7 +637,7 @@ def main():
     ap.add_argument("--intents", type=int, default=None,
                     help="end-to-end only: fewer intents (a smaller case for profiling, not a bench line)")
     args = ap.parse_args()
-    if args.intents and args.workload != "e2e":
+    if args.intents and not args.workload.startswith("e2e"):
         ap.error("--intents applies to the end-to-end workload only")
     if args.warmup < 3:
         print("note: warmup raised to 3", file=sys.stderr)

@@ -317,27 +317,28 @@ int pv_aggregate_intents(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_gro
  *   (decreasing offsets, > 32 waypoints, switch id out of range), PV_ENOMEM.
  * pv_verify_probes_constrained: pv_verify_probes with path constraints.
  *   Probe k follows policy d_probe_policy[k] (device, or NULL: policy
- *   k / probes_per_policy); an index >= num_policies means none.  A forbidden
+ *   first_policy + k / probes_per_policy, so a slice of a larger batch can
+ *   keep its policies); an index >= num_policies means none.  A forbidden
  *   switch is judged like a switch outside the probe's jurisdictions
  *   (PV_VIOLATION there; the walk stops).  Device output d_waypoints[M]: bit
  *   i set iff the probe entered waypoint i of its policy (a switch it was
  *   refused does not count).  Errors: as pv_verify_probes; PV_ESTATE (no
  *   policies), PV_EINVAL (NULL d_waypoints).
  * pv_aggregate_constrained: pv_aggregate_intents plus, for group g with
- *   policy p = d_group_policy[g] (device, or NULL: p = g; p >= num_policies:
- *   none): g fails unless concrete[p] and every probe of g has all of p's
+ *   policy p = d_group_policy[g] (device, or NULL: p = first_policy + g;
+ *   p >= num_policies: none): g fails unless concrete[p] and every probe of g has all of p's
  *   waypoint bits; d_counts[g][7] = probes of g that missed a waypoint.
  * ------------------------------------------------------------------------- */
 int pv_load_path_policies(pv_ctx *ctx, uint32_t num_policies, const uint32_t *forbid_offs, const uint16_t *forbid,
                           const uint32_t *must_offs, const uint16_t *must, const uint8_t *concrete);
 int pv_verify_probes_constrained(pv_ctx *ctx, uint32_t num_probes, const pv_probe *d_probes, uint32_t hop_cap,
-                                 const uint32_t *d_probe_policy, uint32_t probes_per_policy, pv_result *d_out,
-                                 uint32_t *d_waypoints, pv_stream stream);
+                                 const uint32_t *d_probe_policy, uint32_t probes_per_policy, uint32_t first_policy,
+                                 pv_result *d_out, uint32_t *d_waypoints, pv_stream stream);
 int pv_aggregate_constrained(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_group, const uint32_t *d_bits,
                              uint32_t words_per_row, const uint8_t *d_group_flags, const uint32_t *d_assign,
                              uint32_t probes_per_group, const pv_result *d_results, const uint32_t *d_waypoints,
-                             const uint32_t *d_group_policy, uint8_t *d_pass, uint32_t *d_counts,
-                             pv_stream stream);
+                             const uint32_t *d_group_policy, uint32_t first_policy, uint8_t *d_pass,
+                             uint32_t *d_counts, pv_stream stream);
 
 /* ---------------------------------------------------------------------------
  * Tuning knobs (no counterpart in the paper).

@@ -80,8 +80,9 @@ def load_library(path: Optional[str] = None):
                                            ctypes.POINTER(ctypes.c_uint64)]),
         "pv_compliant_reach_noalloc": (ctypes.c_int, [u32, vp, u32, vp, vp, u32, vp, u32, vp, vp, u32, vp]),
         "pv_load_path_policies": (ctypes.c_int, [vp, u32, vp, vp, vp, vp, vp]),
-        "pv_verify_probes_constrained": (ctypes.c_int, [vp, u32, vp, u32, vp, u32, vp, vp, vp]),
-        "pv_aggregate_constrained": (ctypes.c_int, [vp, u32, u32, vp, u32, vp, vp, u32, vp, vp, vp, vp, vp, vp]),
+        "pv_verify_probes_constrained": (ctypes.c_int, [vp, u32, vp, u32, vp, u32, u32, vp, vp, vp]),
+        "pv_aggregate_constrained": (ctypes.c_int, [vp, u32, u32, vp, u32, vp, vp, u32, vp, vp, vp, u32, vp, vp,
+                                                    vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -221,20 +222,22 @@ def pv_load_path_policies(ctx, num_policies, forbid_offs, forbid, must_offs, mus
 
 
 def pv_verify_probes_constrained(ctx, num_probes, d_probes, hop_cap, d_probe_policy, probes_per_policy, d_out,
-                                 d_waypoints, stream=None) -> int:
+                                 d_waypoints, stream=None, first_policy=0) -> int:
     return _check(ctx, load_library().pv_verify_probes_constrained(ctx, num_probes, _dev(d_probes), hop_cap,
                                                                    _dev(d_probe_policy), probes_per_policy,
-                                                                   _dev(d_out), _dev(d_waypoints), _stream(stream)))
+                                                                   first_policy, _dev(d_out), _dev(d_waypoints),
+                                                                   _stream(stream)))
 
 
 def pv_aggregate_constrained(ctx, num_groups, pods_per_group, d_bits, words_per_row, d_group_flags, d_assign,
                              probes_per_group, d_results, d_waypoints, d_group_policy, d_pass, d_counts,
-                             stream=None) -> int:
+                             stream=None, first_policy=0) -> int:
     return _check(ctx, load_library().pv_aggregate_constrained(ctx, num_groups, pods_per_group, _dev(d_bits),
                                                                words_per_row, _dev(d_group_flags), _dev(d_assign),
                                                                probes_per_group, _dev(d_results),
                                                                _dev(d_waypoints), _dev(d_group_policy),
-                                                               _dev(d_pass), _dev(d_counts), _stream(stream)))
+                                                               first_policy, _dev(d_pass), _dev(d_counts),
+                                                               _stream(stream)))
 
 
 def pv_compliant_reach(ctx, V, d_offs, num_edges, d_cols, d_region, num_src, d_src, num_masks, d_masks, d_reach,

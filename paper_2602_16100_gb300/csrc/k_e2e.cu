@@ -91,7 +91,8 @@ __global__ void __launch_bounds__(kThreads) aggregate_kernel(uint32_t G, uint32_
                                                              const pv_result *__restrict__ results,
                                                              uint8_t *__restrict__ pass, uint32_t *__restrict__ counts,
                                                              const uint32_t *__restrict__ hits,
-                                                             const uint32_t *__restrict__ group_pol, uint32_t num_pol,
+                                                             const uint32_t *__restrict__ group_pol,
+                                                             uint32_t first_pol, uint32_t num_pol,
                                                              const uint4 *__restrict__ pol_hdr,
                                                              const uint8_t *__restrict__ concrete) {
     const uint32_t lane = threadIdx.x & 31;
@@ -113,7 +114,7 @@ __global__ void __launch_bounds__(kThreads) aggregate_kernel(uint32_t G, uint32_
         uint32_t missed = 0;
         bool policy_ok = true;
         if (pol_hdr) {
-            const uint32_t p = group_pol ? group_pol[g] : g;
+            const uint32_t p = group_pol ? group_pol[g] : first_pol + g;
             if (p < num_pol) {
                 const uint32_t nm = pol_hdr[p].w;
                 const uint32_t full = nm >= 32 ? 0xFFFFFFFFu : ((1u << nm) - 1u);
@@ -192,7 +193,7 @@ extern "C" int pv_aggregate_intents(pv_ctx *ctx, uint32_t G, uint32_t pods, cons
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_AGGREGATE);
     aggregate_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
         G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts, nullptr,
-        nullptr, 0, nullptr, nullptr);
+        nullptr, 0, 0, nullptr, nullptr);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
     return pv_check_launch(ctx, "aggregate_kernel");
 }
@@ -200,8 +201,8 @@ extern "C" int pv_aggregate_intents(pv_ctx *ctx, uint32_t G, uint32_t pods, cons
 extern "C" int pv_aggregate_constrained(pv_ctx *ctx, uint32_t G, uint32_t pods, const uint32_t *d_bits, uint32_t W,
                                         const uint8_t *d_gflags, const uint32_t *d_assign, uint32_t ppg,
                                         const pv_result *d_results, const uint32_t *d_waypoints,
-                                        const uint32_t *d_group_policy, uint8_t *d_pass, uint32_t *d_counts,
-                                        pv_stream stream) {
+                                        const uint32_t *d_group_policy, uint32_t first_policy, uint8_t *d_pass,
+                                        uint32_t *d_counts, pv_stream stream) {
     if (!ctx) return PV_EINVAL;
     if (!ctx->cl.loaded) return pv_fail(ctx, PV_ESTATE, "pv_aggregate_constrained: no cluster loaded");
     if (!ctx->pol.loaded) return pv_fail(ctx, PV_ESTATE, "pv_aggregate_constrained: no path policies loaded");
@@ -214,7 +215,7 @@ extern "C" int pv_aggregate_constrained(pv_ctx *ctx, uint32_t G, uint32_t pods, 
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_AGGREGATE);
     aggregate_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
         G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts,
-        d_waypoints, d_group_policy, ctx->pol.num, ctx->pol.d_hdr, ctx->pol.d_concrete);
+        d_waypoints, d_group_policy, first_policy, ctx->pol.num, ctx->pol.d_hdr, ctx->pol.d_concrete);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
     return pv_check_launch(ctx, "aggregate_kernel");
 }

@@ -482,7 +482,7 @@ __device__ __forceinline__ uint32_t warp_reserve(bool want, uint32_t *s_count) {
 
 // Path constraints of the walk (Sec. 4.2 constraint object; Sec. 5.3 and
 // Sec. 5.5 waypoint and forbidden-switch checks).  Probe k follows policy
-// probe_pol[k] (or k / per when probe_pol is null); an index >= num means
+// probe_pol[k] (or first + k / per when probe_pol is null); an index >= num means
 // none.  A forbidden switch is judged like a forbidden jurisdiction (checked
 // when the probe is handed to it, so it never enters); hits[k] bit i is set
 // once the probe has entered waypoint i of its policy.
@@ -492,11 +492,12 @@ struct PolicyArgs {
     uint32_t num;
     const uint32_t *probe_pol; // [M] or null
     uint32_t per;              // probes per policy when probe_pol is null
+    uint32_t first;            // policy of probe 0 when probe_pol is null
     uint32_t *hits;            // [M] waypoint bits (output)
 };
 
 __device__ __forceinline__ uint4 policy_of(const PolicyArgs &pa, uint32_t k) {
-    const uint32_t p = pa.probe_pol ? pa.probe_pol[k] : (pa.per ? k / pa.per : 0xFFFFFFFFu);
+    const uint32_t p = pa.probe_pol ? pa.probe_pol[k] : (pa.per ? pa.first + k / pa.per : 0xFFFFFFFFu);
     return p < pa.num ? pa.hdr[p] : make_uint4(0, 0, 0, 0);
 }
 
@@ -1275,7 +1276,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     cudaStream_t st = (cudaStream_t)stream;
     PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
-    const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, nullptr};
+    const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, 0, nullptr};
     if (pol)
         walk_init_kernel<true><<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch,
                                                                    t.d_host_port, t.d_region, d_out, listA, descA, *pa);
@@ -1348,12 +1349,13 @@ extern "C" int pv_verify_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probe
 
 extern "C" int pv_verify_probes_constrained(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap,
                                             const uint32_t *d_probe_policy, uint32_t probes_per_policy,
-                                            pv_result *d_out, uint32_t *d_waypoints, pv_stream stream) {
+                                            uint32_t first_policy, pv_result *d_out, uint32_t *d_waypoints,
+                                            pv_stream stream) {
     if (!ctx) return PV_EINVAL;
     if (!ctx->pol.loaded) return pv_fail(ctx, PV_ESTATE, "pv_verify_probes_constrained: no path policies loaded");
     if (M && !d_waypoints) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes_constrained: NULL waypoint output");
     const PolicyArgs pa = {ctx->pol.d_hdr, ctx->pol.d_sw, ctx->pol.num, d_probe_policy, probes_per_policy,
-                           d_waypoints};
+                           first_policy, d_waypoints};
     return walk_probes(ctx, M, d_probes, hop_cap, d_out, &pa, stream);
 }
 

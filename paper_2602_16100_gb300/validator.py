@@ -129,10 +129,27 @@ class Validator:
                             dev["flags"], stream)
         B.pv_place_pods(self.ctx, I, pods, dev["bits"], words, dev["draws"], dev["assign"], stream)
         B.pv_bind_probes(self.ctx, M, dev["probes"], ppg, pods, dev["assign"], stream)
-        B.pv_verify_probes(self.ctx, M, dev["probes"], e2e_sizes["hop_cap"], dev["results"], stream)
-        B.pv_aggregate_intents(self.ctx, I, pods, dev["bits"], words, dev["flags"], dev["assign"], ppg,
-                               dev["results"], dev["pass"], dev["counts"], stream)
+        self._walk_and_verdict(dev, e2e_sizes, 0, I, stream)
         return dev
+
+    def _walk_and_verdict(self, dev, e2e_sizes, lo, hi, stream):
+        """Walks and verdicts of intents [lo, hi); under the loaded path
+        policies (policy i for intent i) when ``dev`` holds a "hits" buffer."""
+        ppg, pods, n = e2e_sizes["probes_per_intent"], e2e_sizes["pods"], hi - lo
+        words = W.words_per_row(self.num_nodes)
+        P = W.PROBE_DTYPE.itemsize
+        probes, results = dev["probes"][lo * ppg * P:], dev["results"][lo * ppg * 4:]
+        bits, flags, assign = dev["bits"][lo * words * 4:], dev["flags"][lo:], dev["assign"][lo * pods * 4:]
+        if "hits" in dev:
+            hits = dev["hits"][lo * ppg * 4:]
+            B.pv_verify_probes_constrained(self.ctx, n * ppg, probes, e2e_sizes["hop_cap"], None, ppg, results,
+                                           hits, stream, first_policy=lo)
+            B.pv_aggregate_constrained(self.ctx, n, pods, bits, words, flags, assign, ppg, results, hits, None,
+                                       dev["pass"][lo:], dev["counts"][lo * 32:], stream, first_policy=lo)
+        else:
+            B.pv_verify_probes(self.ctx, n * ppg, probes, e2e_sizes["hop_cap"], results, stream)
+            B.pv_aggregate_intents(self.ctx, n, pods, bits, words, flags, assign, ppg, results, dev["pass"][lo:],
+                                   dev["counts"][lo * 32:], stream)
 
     def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
                                  chunks: int = 2) -> dict:
@@ -173,21 +190,20 @@ class Validator:
             flags = dev["flags"][lo:]
             assign = dev["assign"][lo * pods * 4:]
             probes = dev["probes"][lo * ppg * P:]
-            results = dev["results"][lo * ppg * 4:]
             B.pv_eval_selectors(ctx, n, dev["offs"][lo * 4:], e2e_sizes["num_exprs"], dev["exprs"], None, bits,
                                 words, flags, stream)
             B.pv_place_pods(ctx, n, pods, bits, words, dev["draws"][lo * pods * 8:], assign, stream)
             B.pv_bind_probes(ctx, n * ppg, probes, ppg, pods, assign, stream)
-            B.pv_verify_probes(ctx, n * ppg, probes, e2e_sizes["hop_cap"], results, stream)
-            B.pv_aggregate_intents(ctx, n, pods, bits, words, flags, assign, ppg, results, dev["pass"][lo:],
-                                   dev["counts"][lo * 32:], stream)
+            self._walk_and_verdict(dev, e2e_sizes, lo, hi, stream)
         with torch.cuda.stream(stream):
             host["pass"].copy_(dev["pass"][: host["pass"].numel()], non_blocking=True)
             host["counts"].copy_(dev["counts"][: host["counts"].numel()], non_blocking=True)
         return host
 
-    def alloc_end_to_end(self, e: W.EndToEnd) -> tuple:
-        """Device buffers for an end-to-end workload (inputs uploaded)."""
+    def alloc_end_to_end(self, e: W.EndToEnd, with_policies: bool = False) -> tuple:
+        """Device buffers for an end-to-end workload (inputs uploaded); with
+        with_policies, a waypoint-bit buffer that makes the pipeline check the
+        loaded path policies (policy i for intent i)."""
         I, pods, ppg = e.intents.num_pods, e.pods_per_intent, e.probes_per_intent
         words = W.words_per_row(e.cluster.num_nodes)
         M = I * ppg
@@ -204,6 +220,8 @@ class Validator:
             "pass": empty_device(I, d),
             "counts": empty_device(I * 8 * 4, d),
         }
+        if with_policies:
+            dev["hits"] = empty_device(M * 4, d)
         sizes = {"intents": I, "pods": pods, "probes_per_intent": ppg, "num_exprs": len(e.intents.exprs),
                  "hop_cap": e.probes.hop_cap}
         return dev, sizes

@@ -150,3 +150,36 @@ def test_full_size_end_to_end_policies_sampled(validator):
     o, oh = oracle.verify_constrained(e.network, pr, e.probes.hop_cap, pol, probes_per_policy=e.probes_per_intent,
                                       idx=idx)
     assert (g[idx] == o).all() and (gh[idx] == oh).all()
+
+
+@pytest.mark.parametrize("chunks", [1, 3])
+def test_constrained_pipeline_from_host(validator, chunks):
+    """The host-buffer pipeline with path policies, cut into intent chunks
+    (each chunk keeps its intents' policies through first_policy)."""
+    import torch
+    from test_gpu_reach_e2e import _pinned
+    e = W.end_to_end(seed=26, num_switches=64, num_intents=203, probes_per_intent=80, rules_per_switch=200)
+    pol = W.path_policies(8, e.network, 203, forbid_max=1, must_max=2, hubs=6, p_noop=0.1)
+    v = validator
+    v.load_cluster(e.cluster)
+    v.load_network(e.network)
+    v.load_policies(pol)
+    dev, sizes = v.alloc_end_to_end(e, with_policies=True)
+    I, pods, ppg = sizes["intents"], sizes["pods"], sizes["probes_per_intent"]
+    host = {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
+            "draws": _pinned(e.place_draws.astype(np.uint64)), "probes": _pinned(e.probes.probes),
+            "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
+            "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
+    stream = torch.cuda.current_stream()
+    v.run_end_to_end_from_host(host, dev, sizes, stream, torch.cuda.Stream(), chunks)
+    stream.synchronize()
+    v.sync()
+    c = e.cluster
+    bits, flags = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, e.intents.expr_offs, e.intents.exprs)
+    assign = oracle.place_pods(bits, c.num_nodes, pods, e.place_draws)
+    probes = oracle.bind_probes(e.probes.probes, ppg, pods, assign, e.network.host_ip)
+    res, oh = oracle.verify_constrained(e.network, probes, e.probes.hop_cap, pol, probes_per_policy=ppg)
+    passed, counts = oracle.aggregate_constrained(bits, c.num_nodes, flags, assign, pods, res, ppg, oh, pol)
+    assert (to_numpy(dev["hits"], np.uint32) == oh).all()
+    assert (host["pass"].numpy() == passed).all()
+    assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
