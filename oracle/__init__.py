@@ -41,6 +41,7 @@ def _load():
         _lib = ctypes.CDLL(_LIB)
         _lib.oracle_first_match.restype = ctypes.c_int32
         _lib.oracle_eval_selectors.restype = ctypes.c_int
+        _lib.oracle_eval_selector_terms.restype = ctypes.c_int
         _lib.oracle_compliant_reach.restype = ctypes.c_int
     return _lib
 
@@ -77,6 +78,27 @@ def eval_selectors(num_nodes, num_keys, labels, expr_offs, exprs, assign=None, w
     rc = lib.oracle_eval_selectors(ctypes.c_uint32(num_nodes), ctypes.c_uint32(num_keys), _p(labels),
                                    ctypes.c_uint32(P), _p(offs), ctypes.c_uint32(len(exprs)), _p(exprs),
                                    _p(a), _p(bits), ctypes.c_uint32(W), _p(flags))
+    if rc != 0:
+        raise MemoryError("oracle inventory allocation failed")
+    return bits, flags
+
+
+def eval_selector_terms(num_nodes, num_keys, labels, pod_terms, term_offs, exprs, assign=None, words=None):
+    """Multi-term selectors: returns (bits [P, W] uint32, flags [P] uint8)."""
+    lib = _load()
+    W = words or words_per_row(num_nodes)
+    labels = np.ascontiguousarray(labels, np.uint16)
+    pt = np.ascontiguousarray(pod_terms, np.uint32)
+    to = np.ascontiguousarray(term_offs, np.uint32)
+    exprs = np.ascontiguousarray(exprs)
+    P = len(pt) - 1
+    bits = np.zeros((P, W), np.uint32)
+    flags = np.zeros(P, np.uint8)
+    asg = None if assign is None else np.ascontiguousarray(assign, np.uint32)
+    rc = lib.oracle_eval_selector_terms(ctypes.c_uint32(num_nodes), ctypes.c_uint32(num_keys), _p(labels),
+                                        ctypes.c_uint32(P), _p(pt), ctypes.c_uint32(len(to) - 1), _p(to),
+                                        ctypes.c_uint32(len(exprs)), _p(exprs), _p(asg), _p(bits),
+                                        ctypes.c_uint32(W), _p(flags))
     if rc != 0:
         raise MemoryError("oracle inventory allocation failed")
     return bits, flags

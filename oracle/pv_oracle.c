@@ -13,7 +13,8 @@
  *  - Placement constraints are Kubernetes node selectors / affinities
  *    (Sec. 3.3 worked example; Sec. 4.1 "Placement Directives"): the
  *    matchExpressions operators In, NotIn, Exists, DoesNotExist, ANDed
- *    within one pod.  An equality nodeSelector is In with one value.
+ *    within one pod (or within one selector term, the terms ORed, for the
+ *    node-affinity form).  An equality nodeSelector is In with one value.
  *  - Hallucinated identifiers (Sec. 6.3, failure mode 3): a value referenced
  *    by an In expression that no node carries fails the check.
  *  - Unenforceable intents fail closed (Sec. 5.3, intent examples table): a
@@ -279,6 +280,70 @@ void oracle_verify_probes(uint32_t num_switches, const uint32_t *rule_offs, cons
         out[i] = walk_one(num_switches, rule_offs, rules, switch_region, port_offs, port_peer, num_hosts,
                           host_switch, host_port, host_ip, pr, hop_cap);
     }
+}
+
+/* Multi-term node selectors (Sec. 3.3 and Sec. 4.1: placement constraints
+ * are node selectors / affinities): the Kubernetes required node-affinity
+ * form, a list of selector terms that are ORed, each term a list of
+ * expressions that are ANDed:
+ *     feasible(p) = union over p's terms t of { n : every expression of t
+ *                   matches node n }.
+ * Readings: a pod with no terms has no affinity and admits every node; a
+ * term with no expressions matches no node (Kubernetes: an empty selector
+ * term matches nothing); an In value carried by no node anywhere in the pod
+ * sets UNKNOWN (the inventory check of Sec. 6.3 covers every referenced
+ * label); a malformed term range or expression makes the pod BAD with an
+ * empty row.  Pod p's terms are pod_terms[p] .. pod_terms[p+1]) of
+ * term_offs, term t's expressions term_offs[t] .. term_offs[t+1]).  Flags
+ * as oracle_eval_selectors. */
+int oracle_eval_selector_terms(uint32_t num_nodes, uint32_t num_keys, const uint16_t *labels, uint32_t num_pods,
+                               const uint32_t *pod_terms, uint32_t num_terms, const uint32_t *term_offs,
+                               uint32_t num_exprs, const or_expr *exprs, const uint32_t *assign, uint32_t *bits,
+                               uint32_t words_per_row, uint8_t *flags) {
+    uint8_t *inv = build_inventory(num_nodes, num_keys, labels);
+    if (!inv) return -1;
+    for (uint32_t p = 0; p < num_pods; ++p) {
+        uint32_t *row = bits + (size_t)p * words_per_row;
+        memset(row, 0, (size_t)words_per_row * 4);
+        uint32_t t0 = pod_terms[p], t1 = pod_terms[p + 1];
+        int bad = t1 < t0 || t1 > num_terms;
+        for (uint32_t t = t0; !bad && t < t1; ++t) {
+            uint32_t lo = term_offs[t], hi = term_offs[t + 1];
+            if (hi < lo || hi > num_exprs) { bad = 1; break; }
+            for (uint32_t e = lo; e < hi; ++e)
+                if (!expr_is_valid(&exprs[e], num_keys)) { bad = 1; break; }
+        }
+        if (bad) { flags[p] = OR_F_BAD; continue; }
+        uint32_t count = 0;
+        for (uint32_t n = 0; n < num_nodes; ++n) {
+            int ok = t0 == t1;   /* no terms: no affinity */
+            for (uint32_t t = t0; t < t1 && !ok; ++t) {
+                uint32_t lo = term_offs[t], hi = term_offs[t + 1];
+                int all = hi > lo;   /* an empty term matches nothing */
+                for (uint32_t e = lo; e < hi && all; ++e)
+                    all = expr_matches(&exprs[e], labels[(size_t)exprs[e].key * num_nodes + n]);
+                ok = all;
+            }
+            if (ok) { row[n >> 5] |= 1u << (n & 31); ++count; }
+        }
+        int unknown = 0;
+        for (uint32_t t = t0; t < t1; ++t)
+            for (uint32_t e = term_offs[t]; e < term_offs[t + 1]; ++e)
+                if (exprs[e].op == OR_OP_IN)
+                    for (int j = 0; j < exprs[e].nvals; ++j)
+                        if (!inv[(size_t)exprs[e].key * 65536u + exprs[e].vals[j]]) unknown = 1;
+        uint8_t f = 0;
+        if (count == 0) f |= OR_F_EMPTY;
+        if (unknown) f |= OR_F_UNKNOWN;
+        if (assign) {
+            uint32_t a = assign[p];
+            if (a < num_nodes && ((row[a >> 5] >> (a & 31)) & 1u)) f |= OR_F_ASSIGN_OK;
+            if ((f & OR_F_ASSIGN_OK) && !unknown) f |= OR_F_PASS;
+        }
+        flags[p] = f;
+    }
+    free(inv);
+    return 0;
 }
 
 /* ------------------------------------------------------------------------

@@ -142,6 +142,15 @@ class Selectors:
 
 
 @dataclasses.dataclass
+class SelectorTerms:
+    num_pods: int
+    pod_terms: np.ndarray         # u32 [num_pods + 1]: terms of each pod (ORed)
+    term_offs: np.ndarray         # u32 [num_terms + 1]: expressions of each term (ANDed)
+    exprs: np.ndarray             # EXPR_DTYPE [num_exprs]
+    assign: np.ndarray            # u32 [num_pods]
+
+
+@dataclasses.dataclass
 class Network:
     num_switches: int
     rule_offs: np.ndarray         # u32 [S + 1]
@@ -518,6 +527,32 @@ def selector_workload(seed: int = 20260217, num_nodes: int = 5000, num_keys: int
     exprs["vals"] = vals
     assign = st.ints(0, N - 1, P).astype(np.uint32)
     return dict(cluster=cluster, selectors=Selectors(P, offs, exprs, assign))
+
+
+def selector_terms(seed: int = 20260222, num_nodes: int = 5000, num_keys: int = 64, num_values: int = 256,
+                   num_pods: int = 100_000, max_terms: int = 3, max_exprs: int = 4, p_empty_term: float = 0.0,
+                   **kw):
+    """Pods with the node-affinity form: U[0, max_terms] selector terms each
+    (ORed); every term is one pod of selector_workload's recipe (U[1,
+    max_exprs] expressions on distinct keys, ANDed), or, with probability
+    p_empty_term, a term without expressions.  One uniform assignment per pod."""
+    st = Stream(seed, "selector-terms")
+    nterm = st.ints(0, max_terms, num_pods)
+    T = int(nterm.sum())
+    d = selector_workload(seed=seed + 1, num_nodes=num_nodes, num_keys=num_keys, num_values=num_values,
+                          num_pods=max(T, 1), max_exprs=max_exprs, **kw)
+    c, sel = d["cluster"], d["selectors"]
+    lens = np.diff(sel.expr_offs.astype(np.int64))[:T]
+    lens = np.where(st.floats(T) < p_empty_term, 0, lens)
+    keep = np.concatenate([np.arange(sel.expr_offs[t], sel.expr_offs[t] + lens[t]) for t in range(T)]) \
+        if T else np.zeros(0, np.int64)
+    term_offs = np.zeros(T + 1, np.uint32)
+    term_offs[1:] = np.cumsum(lens)
+    pod_terms = np.zeros(num_pods + 1, np.uint32)
+    pod_terms[1:] = np.cumsum(nterm)
+    assign = st.ints(0, num_nodes - 1, num_pods).astype(np.uint32)
+    return dict(cluster=c, terms=SelectorTerms(num_pods, pod_terms, term_offs,
+                                               sel.exprs[keep.astype(np.int64)].copy(), assign))
 
 
 # ----------------------------------------------------------------------------
