@@ -353,6 +353,69 @@ class PlacementBench:
         return self.s.num_pods
 
 
+class PlacementTermsBench:
+    name = "placement-scale, multi-term node affinity"
+    unit = "pod×node selector evals/s"
+
+    def __init__(self, seed):
+        d = W.selector_terms(seed=20260222 + seed)
+        self.c, self.t = d["cluster"], d["terms"]
+
+    def config(self):
+        return {"workload": self.name, "nodes": self.c.num_nodes, "label_keys": self.c.num_keys,
+                "pods": self.t.num_pods, "terms": len(self.t.term_offs) - 1, "expressions": len(self.t.exprs),
+                "l2": "output bitsets (64 MB) rewritten each step; labels and value rows L2-resident"}
+
+    def setup(self, v):
+        from paper_2602_16100_gb300.validator import to_device, empty_device
+        self.v = v
+        v.load_cluster(self.c)
+        d = v.device
+        self.words = W.words_per_row(self.c.num_nodes)
+        self.d_pt = to_device(self.t.pod_terms.astype(np.uint32), d)
+        self.d_to = to_device(self.t.term_offs.astype(np.uint32), d)
+        self.d_exprs = to_device(self.t.exprs, d)
+        self.d_assign = to_device(self.t.assign.astype(np.uint32), d)
+        self.d_bits = empty_device(self.t.num_pods * self.words * 4, d)
+        self.d_flags = empty_device(self.t.num_pods, d)
+
+    def step(self, stream):
+        from paper_2602_16100_gb300 import binding as B
+        B.pv_eval_selector_terms(self.v.ctx, self.t.num_pods, self.d_pt, len(self.t.term_offs) - 1, self.d_to,
+                                 len(self.t.exprs), self.d_exprs, self.d_assign, self.d_bits, self.words,
+                                 self.d_flags, stream)
+
+    def measure_units(self):
+        return self.t.num_pods * self.c.num_nodes
+
+    def extra(self, secs_per_step):
+        return {}
+
+    def algorithmic_bytes(self, group):
+        if group != "selector":
+            return 0
+        P, T = self.t.num_pods, len(self.t.term_offs) - 1
+        return P * self.words * 4 + len(self.t.exprs) * 20 + T * 4 + P * 4 * 2 + P + self.c.labels.nbytes
+
+    def traffic_unit(self, group):
+        return self.t.num_pods if group == "selector" else None
+
+    def oracle_sample(self, n):
+        import oracle
+        pt = self.t.pod_terms[: n + 1].astype(np.uint32)
+        to = self.t.term_offs[: int(pt[-1]) + 1].astype(np.uint32)
+        ex = self.t.exprs[: int(to[-1])]
+        t0 = time.perf_counter()
+        oracle.eval_selector_terms(self.c.num_nodes, self.c.num_keys, self.c.labels, pt, to, ex, self.t.assign[:n])
+        dt = time.perf_counter() - t0
+        return n * self.c.num_nodes, dt, f"first {n} pods"
+
+    oracle_start = 500
+
+    def oracle_max(self):
+        return self.t.num_pods
+
+
 class FlowBench:
     name = "flow-verification"
     unit = "probe-hop verifications/s"
@@ -464,7 +527,7 @@ class WanBench:
         return len(self.q.masks) * len(self.q.sources)
 
 
-WORKLOADS = {"e2e": EndToEndBench,
+WORKLOADS = {"e2e": EndToEndBench, "placement_terms": PlacementTermsBench,
              "e2e_policies": lambda seed, **kw: EndToEndBench(seed, policies=True, **kw), "placement": PlacementBench, "flow": FlowBench, "wan": WanBench}
 SOURCES = {"walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector": ("k_selector.cu",),
            "reach": ("k_reach.cu",)}

@@ -170,6 +170,31 @@ int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_expr_off
                       uint32_t words_per_row, uint8_t *d_flags, pv_stream stream);
 
 /* ---------------------------------------------------------------------------
+ * pv_eval_selector_terms -- the node-affinity form of placement constraints
+ * (Sec. 3.3 and Sec. 4.1: node selectors / affinities): Kubernetes required
+ * node affinity, a list of selector terms that are ORed, each term a list of
+ * expressions that are ANDed (the same pv_expr semantics as above):
+ *     feasible(p) = union over p's terms t of { n : every expression of t
+ *                   matches node n }.
+ * A pod with no terms admits every node; a term with no expressions matches
+ * no node (Kubernetes: an empty selector term matches nothing).
+ *
+ * Device inputs: d_pod_terms[num_pods + 1] (CSR: pod p's terms are
+ * pod_terms[p] .. pod_terms[p+1]), d_term_offs[num_terms + 1] (CSR into
+ * d_exprs), d_exprs[num_exprs], d_assign[num_pods] or NULL.  Outputs and
+ * flags as pv_eval_selectors; an In value carried by no node in any term
+ * sets PV_F_UNKNOWN_VALUE; a malformed term range or expression gives an
+ * empty row and PV_F_BAD_EXPR.  Needs the per-(key, value) rows
+ * (PV_STAT_SELECTOR_ROWS_BUILT).
+ * Errors: PV_ESTATE (no cluster), PV_EINVAL (words_per_row, alignment, NULL
+ * pointers, rows not built).
+ * ------------------------------------------------------------------------- */
+int pv_eval_selector_terms(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_pod_terms, uint32_t num_terms,
+                           const uint32_t *d_term_offs, uint32_t num_exprs, const pv_expr *d_exprs,
+                           const uint32_t *d_assign, uint32_t *d_bits, uint32_t words_per_row, uint8_t *d_flags,
+                           pv_stream stream);
+
+/* ---------------------------------------------------------------------------
  * pv_load_flow_tables -- the installed per-hop flow rules rho (Sec. 4.2
  * flow scheduling module; each path becomes per-hop rules pushed to ONOS)
  * and the switch labels lambda_V reduced to a region id per switch

@@ -30,7 +30,8 @@ SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", 
            "pv_eval_selectors", "pv_load_flow_tables", "pv_verify_probes", "pv_compliant_reach",
            "pv_place_pods", "pv_bind_probes", "pv_aggregate_intents", "pv_set_option", "pv_get_stat",
            "pv_profile_enable", "pv_profile_collect", "pv_profile_read", "pv_compliant_reach_noalloc",
-           "pv_load_path_policies", "pv_verify_probes_constrained", "pv_aggregate_constrained")
+           "pv_load_path_policies", "pv_verify_probes_constrained", "pv_aggregate_constrained",
+           "pv_eval_selector_terms")
 
 #: kernel groups timed by the library profiler (PV_K_* in include/pv.h)
 PV_K_NAMES = ("selector", "place", "bind", "walk_init", "walk_regroup", "walk_hop", "aggregate", "reach")
@@ -80,6 +81,7 @@ def load_library(path: Optional[str] = None):
                                            ctypes.POINTER(ctypes.c_uint64)]),
         "pv_compliant_reach_noalloc": (ctypes.c_int, [u32, vp, u32, vp, vp, u32, vp, u32, vp, vp, u32, vp]),
         "pv_load_path_policies": (ctypes.c_int, [vp, u32, vp, vp, vp, vp, vp]),
+        "pv_eval_selector_terms": (ctypes.c_int, [vp, u32, vp, u32, vp, u32, vp, vp, vp, u32, vp, vp]),
         "pv_verify_probes_constrained": (ctypes.c_int, [vp, u32, vp, u32, vp, u32, u32, vp, vp, vp]),
         "pv_aggregate_constrained": (ctypes.c_int, [vp, u32, u32, vp, u32, vp, vp, u32, vp, vp, vp, u32, vp, vp,
                                                     vp]),
@@ -212,6 +214,14 @@ def pv_load_flow_tables(ctx, num_switches, rule_offs, rules, switch_region, port
 def pv_verify_probes(ctx, num_probes, d_probes, hop_cap, d_out, stream=None) -> int:
     return _check(ctx, load_library().pv_verify_probes(ctx, num_probes, _dev(d_probes), hop_cap, _dev(d_out),
                                                        _stream(stream)))
+
+
+def pv_eval_selector_terms(ctx, num_pods, d_pod_terms, num_terms, d_term_offs, num_exprs, d_exprs, d_assign, d_bits,
+                           words_per_row, d_flags, stream=None) -> int:
+    return _check(ctx, load_library().pv_eval_selector_terms(ctx, num_pods, _dev(d_pod_terms), num_terms,
+                                                             _dev(d_term_offs), num_exprs, _dev(d_exprs),
+                                                             _dev(d_assign), _dev(d_bits), words_per_row,
+                                                             _dev(d_flags), _stream(stream)))
 
 
 def pv_load_path_policies(ctx, num_policies, forbid_offs, forbid, must_offs, must, concrete) -> int:

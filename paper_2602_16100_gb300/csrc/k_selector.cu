@@ -301,6 +301,47 @@ __global__ void __launch_bounds__(kCmpThreads) sel_cmp_kernel(
 // ---------------------------------------------------------------------------
 constexpr int kRowsThreads = 256;
 
+// Four words (128 nodes from word w0) of the node set matching expression x:
+// In = OR of its values' rows, NotIn its complement, Exists the key's
+// present row, DoesNotExist its complement.  Words past the rows read 0
+// before the complement.
+__device__ __forceinline__ uint4 expr_rows4(const pv_expr &x, uint32_t w0, bool in_rows,
+                                            const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
+                                            const uint32_t *__restrict__ key_base, const uint32_t *__restrict__ rows,
+                                            uint32_t row_words, uint32_t num_value_rows) {
+    const uint32_t k = x.key, op = x.op;
+    uint4 r;
+    if (op == PV_IN || op == PV_NOTIN) {
+        r = make_uint4(0, 0, 0, 0);
+        const uint32_t nv = x.nvals;
+        for (uint32_t j = 0; j < nv; ++j) {
+            bool carried;
+            const uint32_t row = value_row(inv, rank, key_base, k, x.vals[j], &carried);
+            if (carried && in_rows) {
+                const uint4 v = __ldg(reinterpret_cast<const uint4 *>(rows + (size_t)row * row_words + w0));
+                r.x |= v.x; r.y |= v.y; r.z |= v.z; r.w |= v.w;
+            }
+        }
+    } else {
+        r = in_rows ? __ldg(reinterpret_cast<const uint4 *>(rows + ((size_t)num_value_rows + k) * row_words + w0))
+                    : make_uint4(0, 0, 0, 0);
+    }
+    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) { r.x = ~r.x; r.y = ~r.y; r.z = ~r.z; r.w = ~r.w; }
+    return r;
+}
+
+// Clears the bits of nodes >= N in the four words from w0.
+__device__ __forceinline__ void clip_rows4(uint4 &acc, uint32_t w0, uint32_t N) {
+    const uint32_t full_words = N >> 5, tail_bits = N & 31;
+    uint32_t *aw = &acc.x;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint32_t w = w0 + i;
+        if (w > full_words || (w == full_words && tail_bits == 0)) aw[i] = 0;
+        else if (w == full_words) aw[i] &= (1u << tail_bits) - 1u;
+    }
+}
+
 __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
     uint32_t N, uint32_t K, uint32_t P, const uint32_t *__restrict__ offs, uint32_t num_exprs,
     const pv_expr *__restrict__ exprs, const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits,
@@ -310,7 +351,6 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
     const uint32_t lane = threadIdx.x & 31;
     const uint32_t gw = (blockIdx.x * kRowsThreads + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * kRowsThreads) >> 5;
-    const uint32_t full_words = N >> 5, tail_bits = N & 31;
     for (uint32_t p = gw; p < P; p += nw) {
         const uint32_t lo = offs[p], hi = offs[p + 1];
         const uint32_t pre = pod_prescan(lo, hi, num_exprs, exprs, K, inv, lane);
@@ -327,37 +367,67 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
             uint4 acc = make_uint4(~0u, ~0u, ~0u, ~0u);
             const bool in_rows = w0 < row_words;
             for (uint32_t e = lo; e < hi; ++e) {
-                const pv_expr &x = exprs[e];
-                const uint32_t k = x.key, op = x.op;
-                uint4 r;
-                if (op == PV_IN || op == PV_NOTIN) {
-                    r = make_uint4(0, 0, 0, 0);
-                    const uint32_t nv = x.nvals;
-                    for (uint32_t j = 0; j < nv; ++j) {
-                        bool carried;
-                        const uint32_t row = value_row(inv, rank, key_base, k, x.vals[j], &carried);
-                        if (carried && in_rows) {
-                            const uint4 v = __ldg(reinterpret_cast<const uint4 *>(rows + (size_t)row * row_words + w0));
-                            r.x |= v.x; r.y |= v.y; r.z |= v.z; r.w |= v.w;
-                        }
-                    }
-                } else {
-                    r = in_rows ? __ldg(reinterpret_cast<const uint4 *>(rows + ((size_t)num_value_rows + k) * row_words + w0))
-                                : make_uint4(0, 0, 0, 0);
-                }
-                if (op == PV_NOTIN || op == PV_DOESNOTEXIST) { r.x = ~r.x; r.y = ~r.y; r.z = ~r.z; r.w = ~r.w; }
+                const uint4 r = expr_rows4(exprs[e], w0, in_rows, inv, rank, key_base, rows, row_words,
+                                           num_value_rows);
                 acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
             }
-            // clear bits of nodes >= N
-            uint32_t *aw = &acc.x;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint32_t w = w0 + i;
-                if (w > full_words || (w == full_words && tail_bits == 0)) aw[i] = 0;
-                else if (w == full_words) aw[i] &= (1u << tail_bits) - 1u;
-            }
+            clip_rows4(acc, w0, N);
+            const uint32_t *aw = &acc.x;
             out[q] = acc;
             any = any || (acc.x | acc.y | acc.z | acc.w) != 0;
+            if (a < N && (a >> 5) >= w0 && (a >> 5) < w0 + 4) aok = (aw[(a >> 5) - w0] >> (a & 31)) & 1u;
+        }
+        any = __any_sync(PV_FULL_MASK, any);
+        aok = __any_sync(PV_FULL_MASK, aok);
+        if (lane == 0) flags[p] = pod_flags(any, pre & 2u, assign != nullptr, aok);
+    }
+}
+
+// Multi-term selectors (Kubernetes required node affinity): a pod's row is
+// the OR over its terms of the AND over each term's expressions.  A pod
+// without terms admits every node; a term without expressions matches none.
+// Warp per pod; every term's list is validated and scanned for values no
+// node carries, as in sel_rows_kernel.
+__global__ void __launch_bounds__(kRowsThreads) sel_terms_kernel(
+    uint32_t N, uint32_t K, uint32_t P, const uint32_t *__restrict__ pod_terms, uint32_t num_terms,
+    const uint32_t *__restrict__ term_offs, uint32_t num_exprs, const pv_expr *__restrict__ exprs,
+    const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits, uint32_t W, uint8_t *__restrict__ flags,
+    const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank, const uint32_t *__restrict__ key_base,
+    const uint32_t *__restrict__ rows, uint32_t row_words, uint32_t num_value_rows) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t gw = (blockIdx.x * kRowsThreads + threadIdx.x) >> 5;
+    const uint32_t nw = (gridDim.x * kRowsThreads) >> 5;
+    for (uint32_t p = gw; p < P; p += nw) {
+        const uint32_t t0 = pod_terms[p], t1 = pod_terms[p + 1];
+        uint32_t pre = (t1 < t0 || t1 > num_terms) ? 1u : 0u;
+        for (uint32_t t = t0; t < t1 && !(pre & 1u); ++t)
+            pre |= pod_prescan(term_offs[t], term_offs[t + 1], num_exprs, exprs, K, inv, lane);
+        uint4 *out = reinterpret_cast<uint4 *>(bits + (size_t)p * W);
+        if (pre & 1u) {
+            for (uint32_t q = lane; q < W / 4; q += 32) out[q] = make_uint4(0, 0, 0, 0);
+            if (lane == 0) flags[p] = PV_F_BAD_EXPR;
+            continue;
+        }
+        const uint32_t a = assign ? assign[p] : PV_UNPLACED;
+        bool any = false, aok = false;
+        for (uint32_t q = lane; q < W / 4; q += 32) {
+            const uint32_t w0 = q * 4;
+            const bool in_rows = w0 < row_words;
+            uint4 res = t0 == t1 ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
+            for (uint32_t t = t0; t < t1; ++t) {
+                const uint32_t lo = term_offs[t], hi = term_offs[t + 1];
+                uint4 acc = hi > lo ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
+                for (uint32_t e = lo; e < hi; ++e) {
+                    const uint4 r = expr_rows4(exprs[e], w0, in_rows, inv, rank, key_base, rows, row_words,
+                                               num_value_rows);
+                    acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
+                }
+                res.x |= acc.x; res.y |= acc.y; res.z |= acc.z; res.w |= acc.w;
+            }
+            clip_rows4(res, w0, N);
+            const uint32_t *aw = &res.x;
+            out[q] = res;
+            any = any || (res.x | res.y | res.z | res.w) != 0;
             if (a < N && (a >> 5) >= w0 && (a >> 5) < w0 + 4) aok = (aw[(a >> 5) - w0] >> (a & 31)) & 1u;
         }
         any = __any_sync(PV_FULL_MASK, any);
@@ -461,4 +531,32 @@ extern "C" int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t 
                                                       words_per_row, d_flags, c.d_inv);
     pv_prof_stop(ctx, st, pr, 1);
     return pv_check_launch(ctx, "sel_cmp_kernel");
+}
+
+extern "C" int pv_eval_selector_terms(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_pod_terms, uint32_t num_terms,
+                                      const uint32_t *d_term_offs, uint32_t num_exprs, const pv_expr *d_exprs,
+                                      const uint32_t *d_assign, uint32_t *d_bits, uint32_t words_per_row,
+                                      uint8_t *d_flags, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    const pv_cluster_state &c = ctx->cl;
+    if (!c.loaded) return pv_fail(ctx, PV_ESTATE, "pv_eval_selector_terms: no cluster loaded");
+    if (num_pods == 0) return PV_OK;
+    if (!d_pod_terms || !d_bits || !d_flags || (num_terms > 0 && !d_term_offs) || (num_exprs > 0 && !d_exprs))
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selector_terms: NULL device pointer");
+    if (words_per_row % 4 != 0 || words_per_row < (c.num_nodes + 31) / 32)
+        return pv_fail(ctx, PV_EINVAL,
+                       "pv_eval_selector_terms: words_per_row must be >= ceil(N/32) and a multiple of 4");
+    if (((uintptr_t)d_bits & 15) != 0)
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selector_terms: d_bits must be 16-byte aligned");
+    if (!c.rows_built)
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selector_terms: value rows were not built for this cluster");
+    cudaStream_t st = (cudaStream_t)stream;
+    const uint32_t blocks = std::min<uint32_t>((num_pods + 7) / 8, (uint32_t)ctx->num_sms * 16);
+    const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
+    sel_terms_kernel<<<blocks, kRowsThreads, 0, st>>>(c.num_nodes, c.num_keys, num_pods, d_pod_terms, num_terms,
+                                                      d_term_offs, num_exprs, d_exprs, d_assign, d_bits,
+                                                      words_per_row, d_flags, c.d_inv, c.d_inv_rank, c.d_key_base,
+                                                      c.d_rows, c.row_words, c.num_value_rows);
+    pv_prof_stop(ctx, st, pr, 1);
+    return pv_check_launch(ctx, "sel_terms_kernel");
 }
