@@ -232,3 +232,43 @@ def aggregate_constrained(bits, num_nodes, group_flags, assign, pods_per_group, 
                                          _p(gp), ctypes.c_uint32(pol.num_policies), _p(mo), _p(cc), _p(passed),
                                          _p(counts))
     return passed, counts
+
+
+def schedule_paths(net, requests, pol=None, weights=None, max_len=64):
+    """Scheduled paths: (visits [R, max_len] u32, lengths [R] u8, status [R] u8)."""
+    assert 1 <= max_len <= 255
+    lib = _load()
+    req = np.ascontiguousarray(requests)
+    R = len(req)
+    hops = np.zeros((R, max_len), np.uint32)
+    ln = np.zeros(R, np.uint8)
+    st = np.zeros(R, np.uint8)
+    arr = [np.ascontiguousarray(x) for x in (net.switch_region.astype(np.uint8), net.port_offs.astype(np.uint32),
+                                             net.port_peer.astype(np.int32), net.host_switch.astype(np.uint16),
+                                             net.host_port.astype(np.uint16))]
+    w = None if weights is None else np.ascontiguousarray(weights, np.uint16)
+    if pol is None:
+        P, fo, fb, mo, mg = 0, None, None, None, None
+    else:
+        P = pol.num_policies
+        fo, fb, mo, mg, _ = _policy_arrays(pol)
+    lib.oracle_schedule_paths(ctypes.c_uint32(net.num_switches), _p(arr[0]), _p(arr[1]), _p(arr[2]),
+                              ctypes.c_uint32(net.num_hosts), _p(arr[3]), _p(arr[4]), _p(w), ctypes.c_uint32(P),
+                              _p(fo), _p(fb), _p(mo), _p(mg), ctypes.c_uint32(R), _p(req), ctypes.c_uint32(max_len),
+                              _p(hops), _p(ln), _p(st))
+    return hops, ln, st
+
+
+def compile_path_rules(net, requests, hops, lengths, status, priority=65535):
+    """Per-hop rules: (rules [R * max_len] RULE records, rule_switch [R * max_len] u16)."""
+    req = np.ascontiguousarray(requests)
+    R, L = hops.shape
+    rules = np.zeros(R * L, net.rules.dtype)
+    rsw = np.zeros(R * L, np.uint16)
+    hip = np.ascontiguousarray(net.host_ip, np.uint32)
+    _load().oracle_compile_path_rules(ctypes.c_uint32(R), _p(req), _p(hip), ctypes.c_uint32(L),
+                                      _p(np.ascontiguousarray(hops, np.uint32)),
+                                      _p(np.ascontiguousarray(lengths, np.uint8)),
+                                      _p(np.ascontiguousarray(status, np.uint8)), ctypes.c_uint16(priority),
+                                      _p(rules), _p(rsw))
+    return rules, rsw

@@ -604,3 +604,167 @@ void oracle_aggregate_constrained(uint32_t num_groups, uint32_t pods_per_group, 
         if (!concrete[p] || missed) pass[g] = 0;
     }
 }
+
+/* ------------------------------------------------------------------------
+ * Path scheduler (Sec. 4.2: the flow scheduling module computes paths that
+ * respect the constraint object with graph algorithms -- weighted Dijkstra,
+ * BFS when no weights are given -- and turns each path into per-hop flow
+ * rules).
+ *
+ * Request r: from host src to host dst, over switches whose region the mask
+ * permits and that its policy (index >= num_policies: none) does not forbid,
+ * through the policy's waypoints in their listed order.  The path is the
+ * concatenation of shortest segments src switch -> waypoint 1 -> ... -> dst
+ * switch.  Link u --port p--> v costs w[port_offs[u] + p] (a weight of 0
+ * counts as 1; all 1 when w is NULL, i.e. breadth-first hop counts).
+ *
+ * Readings: a shortest segment is made canonical by walking back from its
+ * end and taking, at every switch v, the predecessor link (u, p) with the
+ * smallest u, then the smallest p, among those on some shortest path; the
+ * path is a list of visits (switch, in_port, out_port), in_port of the
+ * first visit = the source host's port, out_port of the last = the
+ * destination host's port.  Status: 0 OK; 1 NOSRC (a host id out of
+ * range); 2 BLOCKED (an endpoint or waypoint switch is not permitted, or a
+ * segment has no path); 3 TOO_LONG (more than max_len visits); 4 REPEAT (a
+ * (switch, in_port) pair recurs: per-hop rules that match on the header and
+ * in_port cannot realise the path).  Visits are encoded switch << 16 |
+ * in_port << 8 | out_port.
+ * ---------------------------------------------------------------------- */
+typedef struct { uint16_t src_host, dst_host; uint32_t allowed_mask, policy, reserved; } or_path_req;
+
+static uint32_t link_w(const uint16_t *w, uint32_t i) { return w && w[i] ? w[i] : 1u; }   /* 0 counts as 1 */
+
+static int switch_ok(const uint8_t *region, uint32_t mask, const uint16_t *forbid, uint32_t nforbid, uint32_t s) {
+    return region[s] < 32 && ((mask >> region[s]) & 1u) && !in_list(forbid, nforbid, s);
+}
+
+/* Dijkstra from a over permitted switches (simple O(S^2) selection). */
+static void dijkstra(uint32_t S, const uint32_t *port_offs, const int32_t *port_peer, const uint16_t *w,
+                     const uint8_t *ok, uint32_t a, uint32_t *dist, uint8_t *done) {
+    for (uint32_t v = 0; v < S; ++v) { dist[v] = 0xFFFFFFFFu; done[v] = 0; }
+    dist[a] = 0;
+    for (;;) {
+        uint32_t u = S, best = 0xFFFFFFFFu;
+        for (uint32_t v = 0; v < S; ++v)
+            if (!done[v] && dist[v] < best) { best = dist[v]; u = v; }
+        if (u == S) return;
+        done[u] = 1;
+        for (uint32_t p = 0; p < port_offs[u + 1] - port_offs[u]; ++p) {
+            int32_t peer = port_peer[port_offs[u] + p];
+            if (peer < 0 || (peer & OR_HOST_BIT)) continue;
+            uint32_t v = (uint32_t)peer >> 8;
+            if (v >= S || !ok[v]) continue;
+            uint32_t c = dist[u] + link_w(w, port_offs[u] + p);
+            if (c < dist[v]) dist[v] = c;
+        }
+    }
+}
+
+void oracle_schedule_paths(uint32_t S, const uint8_t *switch_region, const uint32_t *port_offs,
+                           const int32_t *port_peer, uint32_t num_hosts, const uint16_t *host_switch,
+                           const uint16_t *host_port, const uint16_t *weights, uint32_t num_policies,
+                           const uint32_t *forbid_offs, const uint16_t *forbid, const uint32_t *must_offs,
+                           const uint16_t *must, uint32_t num_req, const or_path_req *req, uint32_t max_len,
+                           uint32_t *hops, uint8_t *len, uint8_t *status) {
+    uint32_t *dist = malloc((size_t)S * 4);
+    uint8_t *done = malloc(S), *ok = malloc(S);
+    uint32_t *seg = malloc((size_t)(S + 1) * 4 * 2);
+    for (uint32_t r = 0; r < num_req; ++r) {
+        uint32_t *out = hops + (size_t)r * max_len;
+        len[r] = 0;
+        const or_path_req *q = &req[r];
+        if (q->src_host >= num_hosts || q->dst_host >= num_hosts) { status[r] = 1; continue; }
+        const uint16_t *fb = NULL, *mg = NULL;
+        uint32_t nf = 0, nm = 0;
+        if (q->policy < num_policies) {
+            fb = forbid + forbid_offs[q->policy];
+            nf = forbid_offs[q->policy + 1] - forbid_offs[q->policy];
+            mg = must + must_offs[q->policy];
+            nm = must_offs[q->policy + 1] - must_offs[q->policy];
+        }
+        for (uint32_t s = 0; s < S; ++s) ok[s] = (uint8_t)switch_ok(switch_region, q->allowed_mask, fb, nf, s);
+        uint32_t cur = host_switch[q->src_host], dst = host_switch[q->dst_host];
+        int st = 0;
+        if (!ok[cur] || !ok[dst]) st = 2;
+        for (uint32_t i = 0; i < nm && !st; ++i)
+            if (!ok[mg[i]]) st = 2;
+        /* visits: (switch, in_port) with out_port filled when the next link is chosen */
+        uint32_t n = 1, vsw[256], vin[256], vout[256];
+        vsw[0] = cur; vin[0] = host_port[q->src_host]; vout[0] = 0;
+        for (uint32_t i = 0; i <= nm && !st; ++i) {
+            uint32_t tgt = i < nm ? mg[i] : dst;
+            if (tgt == cur) continue;
+            dijkstra(S, port_offs, port_peer, weights, ok, cur, dist, done);
+            if (dist[tgt] == 0xFFFFFFFFu) { st = 2; break; }
+            /* canonical walk back: seg holds (u, p) pairs from tgt to cur */
+            uint32_t k = 0, v = tgt;
+            while (v != cur) {
+                uint32_t bu = S, bp = 0, bq = 0;
+                for (uint32_t u = 0; u < S && bu == S; ++u) {
+                    if (!ok[u] || dist[u] == 0xFFFFFFFFu) continue;
+                    for (uint32_t p = 0; p < port_offs[u + 1] - port_offs[u]; ++p) {
+                        int32_t peer = port_peer[port_offs[u] + p];
+                        if (peer < 0 || (peer & OR_HOST_BIT) || ((uint32_t)peer >> 8) != v) continue;
+                        if (dist[u] + link_w(weights, port_offs[u] + p) == dist[v]) {
+                            bu = u; bp = p; bq = (uint32_t)peer & 0xFFu;
+                            break;
+                        }
+                    }
+                }
+                seg[2 * k] = bu << 8 | bp;
+                seg[2 * k + 1] = v << 8 | bq;
+                ++k;
+                v = bu;
+            }
+            while (k > 0 && !st) {
+                --k;
+                uint32_t p = seg[2 * k] & 0xFFu, v2 = seg[2 * k + 1] >> 8, q2 = seg[2 * k + 1] & 0xFFu;
+                if (n >= max_len) { st = 3; break; }
+                vout[n - 1] = p;
+                vsw[n] = v2; vin[n] = q2; vout[n] = 0;
+                ++n;
+            }
+            cur = tgt;
+        }
+        if (!st) {
+            vout[n - 1] = host_port[q->dst_host];
+            for (uint32_t i = 0; i < n && !st; ++i)
+                for (uint32_t j = i + 1; j < n; ++j)
+                    if (vsw[i] == vsw[j] && vin[i] == vin[j]) { st = 4; break; }
+        }
+        status[r] = (uint8_t)st;
+        if (!st) {
+            len[r] = (uint8_t)n;
+            for (uint32_t i = 0; i < n; ++i) out[i] = vsw[i] << 16 | vin[i] << 8 | vout[i];
+        }
+    }
+    free(dist); free(done); free(ok); free(seg);
+}
+
+/* Per-hop rules of the scheduled paths (Sec. 4.2: each path becomes per-hop
+ * flow rules): visit i of an OK request becomes, at its switch, the rule
+ * {priority, in_port, src /32, dst /32, any port, action out_port}, in slot
+ * r * max_len + i; rule_switch of the slot = its switch, 0xFFFF for unused
+ * slots. */
+void oracle_compile_path_rules(uint32_t num_req, const or_path_req *req, const uint32_t *host_ip, uint32_t max_len,
+                               const uint32_t *hops, const uint8_t *len, const uint8_t *status, uint16_t priority,
+                               or_rule *rules, uint16_t *rule_switch) {
+    for (uint32_t r = 0; r < num_req; ++r)
+        for (uint32_t i = 0; i < max_len; ++i) {
+            size_t k = (size_t)r * max_len + i;
+            memset(&rules[k], 0, sizeof(or_rule));
+            rule_switch[k] = 0xFFFF;
+            if (status[r] != 0 || i >= len[r]) continue;
+            uint32_t h = hops[k];
+            rules[k].priority = priority;
+            rules[k].in_port = (uint16_t)((h >> 8) & 0xFFu);
+            rules[k].src_ip = host_ip[req[r].src_host];
+            rules[k].src_len = 32;
+            rules[k].dst_ip = host_ip[req[r].dst_host];
+            rules[k].dst_len = 32;
+            rules[k].dport_lo = 0;
+            rules[k].dport_hi = 0xFFFF;
+            rules[k].action = (uint16_t)(h & 0xFFu);
+            rule_switch[k] = (uint16_t)(h >> 16);
+        }
+}

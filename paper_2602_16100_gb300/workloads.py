@@ -126,6 +126,13 @@ class Stream:
 # ----------------------------------------------------------------------------
 # containers
 # ----------------------------------------------------------------------------
+# path request of the scheduler: {src_host, dst_host, allowed_mask, policy, reserved}
+PATH_REQ_DTYPE = np.dtype([("src_host", "<u2"), ("dst_host", "<u2"), ("allowed_mask", "<u4"), ("policy", "<u4"),
+                           ("reserved", "<u4")])
+NO_POLICY = 0xFFFFFFFF
+PATH_OK, PATH_NOSRC, PATH_BLOCKED, PATH_TOO_LONG, PATH_REPEAT = 0, 1, 2, 3, 4
+
+
 @dataclasses.dataclass
 class Cluster:
     num_nodes: int
@@ -860,3 +867,37 @@ def path_policies(seed: int, net: Network, num_policies: int, forbid_max: int = 
     must = np.concatenate(must_lists).astype(np.uint16) if num_policies else np.zeros(0, np.uint16)
     concrete = (st.floats(num_policies) >= p_noop).astype(np.uint8)
     return PathPolicies(num_policies, fo, forbid, mo, must, concrete)
+
+
+def path_requests(seed: int, net: Network, num_requests: int, num_policies: int = 0, extra_regions=(2, 8),
+                  p_no_policy: float = 0.3, bad_hosts: int = 0) -> np.ndarray:
+    """Scheduler requests with distinct (src, dst) host pairs: the mask
+    permits the two endpoints' regions plus U[extra_regions] others; the
+    policy is uniform over num_policies (or none with probability
+    p_no_policy); the first bad_hosts requests name an absent host."""
+    st = Stream(seed, "path-requests")
+    H = net.num_hosts
+    assert num_requests <= H * (H - 1)
+    pairs = np.unique(st.u64(num_requests * 4) % np.uint64(H * H))
+    pairs = pairs[(pairs // H) != (pairs % H)]
+    pairs = pairs[st.permutation(len(pairs))][:num_requests]
+    assert len(pairs) == num_requests
+    req = np.zeros(num_requests, PATH_REQ_DTYPE)
+    req["src_host"] = pairs // H
+    req["dst_host"] = pairs % H
+    reg = net.switch_region.astype(np.uint64)
+    own = (np.uint64(1) << reg[net.host_switch[req["src_host"]]]) | (np.uint64(1) << reg[net.host_switch[req["dst_host"]]])
+    nreg = int(reg.max()) + 1
+    extra = np.zeros(num_requests, np.uint64)
+    k = st.ints(extra_regions[0], extra_regions[1], num_requests)
+    keys = st.u64(num_requests * nreg).reshape(num_requests, nreg)
+    for r in range(num_requests):
+        for g in np.argsort(keys[r], kind="stable")[: k[r]]:
+            extra[r] |= np.uint64(1) << np.uint64(g)
+    req["allowed_mask"] = ((own | extra) & np.uint64(0xFFFFFFFF)).astype(np.uint32)
+    pol = st.ints(0, max(num_policies - 1, 0), num_requests).astype(np.uint32)
+    none = (st.floats(num_requests) < p_no_policy) | (num_policies == 0)
+    req["policy"] = np.where(none, NO_POLICY, pol)
+    if bad_hosts:
+        req["dst_host"][:bad_hosts] = 0xFFFF
+    return req
