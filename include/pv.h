@@ -115,6 +115,14 @@ typedef struct {           /* one walk result, 4 bytes                          
     uint8_t hops;          /* switch visits made (hop_cap for PV_LOOP, 0 for PV_NOSRC)   */
     uint16_t last_switch;  /* last switch visited (0xFFFF for PV_NOSRC)                   */
 } pv_result;
+typedef struct {           /* one path request of the scheduler, 16 bytes                */
+    uint16_t src_host;     /* source host id                                             */
+    uint16_t dst_host;     /* destination host id                                        */
+    uint32_t allowed_mask; /* permitted regions (bit r = region r)                       */
+    uint32_t policy;       /* path policy index (>= loaded policies: none)               */
+    uint32_t reserved;     /* 0                                                          */
+} pv_path_req;
+enum { PV_PATH_OK = 0, PV_PATH_NOSRC = 1, PV_PATH_BLOCKED = 2, PV_PATH_TOO_LONG = 3, PV_PATH_REPEAT = 4 };
 
 /* ---------------------------------------------------------------------------
  * Context.
@@ -364,6 +372,48 @@ int pv_aggregate_constrained(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per
                              uint32_t probes_per_group, const pv_result *d_results, const uint32_t *d_waypoints,
                              const uint32_t *d_group_policy, uint32_t first_policy, uint8_t *d_pass,
                              uint32_t *d_counts, pv_stream stream);
+
+/* ---------------------------------------------------------------------------
+ * Path scheduling -- the enforcement side (Sec. 4.2: the flow scheduling
+ * module computes paths respecting the constraint object with weighted
+ * Dijkstra, breadth-first when no weights are given, and turns each path
+ * into per-hop flow rules).
+ *
+ * pv_schedule_paths: request r asks for a path from host src_host to host
+ *   dst_host over switches whose region allowed_mask permits and that its
+ *   policy (pv_load_path_policies; none when the index is out of range or no
+ *   policies are loaded) does not forbid, through the policy's waypoints in
+ *   their listed order.  The path is the concatenation of shortest segments
+ *   src switch -> waypoint 1 -> ... -> dst switch; link u --port p--> costs
+ *   d_link_weights[port_offs[u] + p] (device, 0 counts as 1; NULL: 1 each).
+ *   A segment is made canonical by walking back from its end and taking, at
+ *   every switch, the predecessor link with the smallest source switch, then
+ *   the smallest source port, among those on a shortest path.  Device
+ *   outputs: d_visits[r][max_len] = switch << 16 | in_port << 8 | out_port
+ *   for the d_len[r] visits (in_port of the first = the source host's port,
+ *   out_port of the last = the destination host's port), d_status[r] =
+ *   PV_PATH_OK, NOSRC (a host id out of range), BLOCKED (an endpoint or
+ *   waypoint not permitted, or no path), TOO_LONG (more than max_len visits),
+ *   REPEAT (a (switch, in_port) pair recurs: rules matching header and
+ *   in_port cannot realise it).  Needs <= 16,384 switches.
+ * pv_compile_path_rules: visit i of an OK request becomes, at its switch,
+ *   the rule {priority, in_port, src /32, dst /32, ports 0..65535, out_port}
+ *   in d_rules[r * max_len + i], d_rule_switch[...] = its switch (0xFFFF for
+ *   unused slots).
+ * pv_install_path_rules: adds the compiled rules ahead of each switch's
+ *   loaded rules (they win priority ties) and reloads the tables
+ *   (synchronous, like pv_load_flow_tables; slots with switch 0xFFFF or out
+ *   of range are skipped).
+ * Errors: PV_ESTATE (no tables), PV_EINVAL (max_len not 1..255, NULL
+ * pointers, too many switches), PV_ENOMEM.
+ * ------------------------------------------------------------------------- */
+int pv_schedule_paths(pv_ctx *ctx, uint32_t num_requests, const pv_path_req *d_requests,
+                      const uint16_t *d_link_weights, uint32_t max_len, uint32_t *d_visits, uint8_t *d_len,
+                      uint8_t *d_status, pv_stream stream);
+int pv_compile_path_rules(pv_ctx *ctx, uint32_t num_requests, const pv_path_req *d_requests, uint32_t max_len,
+                          const uint32_t *d_visits, const uint8_t *d_len, const uint8_t *d_status,
+                          uint16_t priority, pv_rule *d_rules, uint16_t *d_rule_switch, pv_stream stream);
+int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rules, const uint16_t *d_rule_switch);
 
 /* ---------------------------------------------------------------------------
  * Tuning knobs (no counterpart in the paper).

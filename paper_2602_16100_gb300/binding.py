@@ -31,7 +31,7 @@ SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", 
            "pv_place_pods", "pv_bind_probes", "pv_aggregate_intents", "pv_set_option", "pv_get_stat",
            "pv_profile_enable", "pv_profile_collect", "pv_profile_read", "pv_compliant_reach_noalloc",
            "pv_load_path_policies", "pv_verify_probes_constrained", "pv_aggregate_constrained",
-           "pv_eval_selector_terms")
+           "pv_eval_selector_terms", "pv_schedule_paths", "pv_compile_path_rules", "pv_install_path_rules")
 
 #: kernel groups timed by the library profiler (PV_K_* in include/pv.h)
 PV_K_NAMES = ("selector", "place", "bind", "walk_init", "walk_regroup", "walk_hop", "aggregate", "reach")
@@ -82,6 +82,9 @@ def load_library(path: Optional[str] = None):
         "pv_compliant_reach_noalloc": (ctypes.c_int, [u32, vp, u32, vp, vp, u32, vp, u32, vp, vp, u32, vp]),
         "pv_load_path_policies": (ctypes.c_int, [vp, u32, vp, vp, vp, vp, vp]),
         "pv_eval_selector_terms": (ctypes.c_int, [vp, u32, vp, u32, vp, u32, vp, vp, vp, u32, vp, vp]),
+        "pv_schedule_paths": (ctypes.c_int, [vp, u32, vp, vp, u32, vp, vp, vp, vp]),
+        "pv_compile_path_rules": (ctypes.c_int, [vp, u32, vp, u32, vp, vp, vp, ctypes.c_uint16, vp, vp, vp]),
+        "pv_install_path_rules": (ctypes.c_int, [vp, u32, vp, vp]),
         "pv_verify_probes_constrained": (ctypes.c_int, [vp, u32, vp, u32, vp, u32, u32, vp, vp, vp]),
         "pv_aggregate_constrained": (ctypes.c_int, [vp, u32, u32, vp, u32, vp, vp, u32, vp, vp, vp, u32, vp, vp,
                                                     vp]),
@@ -222,6 +225,24 @@ def pv_eval_selector_terms(ctx, num_pods, d_pod_terms, num_terms, d_term_offs, n
                                                              _dev(d_term_offs), num_exprs, _dev(d_exprs),
                                                              _dev(d_assign), _dev(d_bits), words_per_row,
                                                              _dev(d_flags), _stream(stream)))
+
+
+def pv_schedule_paths(ctx, num_requests, d_requests, d_link_weights, max_len, d_visits, d_len, d_status,
+                      stream=None) -> int:
+    return _check(ctx, load_library().pv_schedule_paths(ctx, num_requests, _dev(d_requests), _dev(d_link_weights),
+                                                        max_len, _dev(d_visits), _dev(d_len), _dev(d_status),
+                                                        _stream(stream)))
+
+
+def pv_compile_path_rules(ctx, num_requests, d_requests, max_len, d_visits, d_len, d_status, priority, d_rules,
+                          d_rule_switch, stream=None) -> int:
+    return _check(ctx, load_library().pv_compile_path_rules(ctx, num_requests, _dev(d_requests), max_len,
+                                                            _dev(d_visits), _dev(d_len), _dev(d_status), priority,
+                                                            _dev(d_rules), _dev(d_rule_switch), _stream(stream)))
+
+
+def pv_install_path_rules(ctx, num_slots, d_rules, d_rule_switch) -> int:
+    return _check(ctx, load_library().pv_install_path_rules(ctx, num_slots, _dev(d_rules), _dev(d_rule_switch)))
 
 
 def pv_load_path_policies(ctx, num_policies, forbid_offs, forbid, must_offs, must, concrete) -> int:

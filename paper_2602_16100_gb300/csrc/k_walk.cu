@@ -1228,6 +1228,47 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           (int)(2 * kSmemHistMax * 4)),
                 "walk_scatter_kernel smem");
+    // links into each switch, sorted by (source switch, source port)
+    {
+        std::vector<uint32_t> in_offs(S + 1, 0), links;
+        for (uint32_t u = 0; u < S; ++u)
+            for (uint32_t p = port_offs[u]; p < port_offs[u + 1]; ++p) {
+                const int32_t peer = port_peer[p];
+                if (peer >= 0 && !(peer & PV_PEER_HOST)) ++in_offs[((uint32_t)peer >> 8) + 1];
+            }
+        for (uint32_t v = 0; v < S; ++v) in_offs[v + 1] += in_offs[v];
+        links.resize(std::max<uint32_t>(in_offs[S], 1));
+        std::vector<uint32_t> cur(in_offs.begin(), in_offs.end() - 1);
+        for (uint32_t u = 0; u < S; ++u)   // ascending u, then p: each list ends up sorted
+            for (uint32_t p = port_offs[u]; p < port_offs[u + 1]; ++p) {
+                const int32_t peer = port_peer[p];
+                if (peer < 0 || (peer & PV_PEER_HOST)) continue;
+                const uint32_t v = (uint32_t)peer >> 8;
+                links[cur[v]++] = u << 16 | (p - port_offs[u]) << 8 | ((uint32_t)peer & 0xFFu);
+            }
+        int rc2;
+        if ((rc2 = pv_device_alloc(ctx, (void **)&t.d_in_offs, (S + 1) * 4, "in-link offsets")) ||
+            (rc2 = pv_device_alloc(ctx, (void **)&t.d_in_links, links.size() * 4, "in-links"))) {
+            pv_free_tables(t);
+            return rc2;
+        }
+        cudaError_t e2 = cudaMemcpy(t.d_in_offs, in_offs.data(), (S + 1) * 4, cudaMemcpyHostToDevice);
+        if (e2 == cudaSuccess) e2 = cudaMemcpy(t.d_in_links, links.data(), links.size() * 4, cudaMemcpyHostToDevice);
+        if (e2 != cudaSuccess) {
+            pv_free_tables(t);
+            return pv_cuda_fail(ctx, e2, "in-links upload");
+        }
+    }
+    // host copy for rule installation
+    pv_table_host &h = ctx->tbh;
+    h.rule_offs.assign(rule_offs, rule_offs + S + 1);
+    h.rules.assign(rules, rules + R);
+    h.region.assign(switch_region, switch_region + S);
+    h.port_offs.assign(port_offs, port_offs + S + 1);
+    h.port_peer.assign(port_peer, port_peer + P);
+    h.host_switch.assign(host_switch, host_switch + H);
+    h.host_port.assign(host_port, host_port + H);
+    h.host_ip.assign(host_ip, host_ip + H);
     t.loaded = true;
     return PV_OK;
 }

@@ -90,6 +90,8 @@ void pv_free_tables(pv_table_state &t) {
     pv_free_ptr(t.d_host_switch);
     pv_free_ptr(t.d_host_port);
     pv_free_ptr(t.d_host_ip);
+    pv_free_ptr(t.d_in_offs);
+    pv_free_ptr(t.d_in_links);
     t = pv_table_state();
 }
 

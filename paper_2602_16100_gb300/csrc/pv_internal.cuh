@@ -44,6 +44,20 @@ struct pv_table_state {
     int32_t *d_port_peer = nullptr;   // [ports]
     uint16_t *d_host_switch = nullptr, *d_host_port = nullptr;
     uint32_t *d_host_ip = nullptr;
+    // switch-to-switch links into each switch, sorted by (source switch,
+    // source port): u << 16 | p << 8 | q for port p of u cabled to port q
+    uint32_t *d_in_offs = nullptr;    // [S + 1]
+    uint32_t *d_in_links = nullptr;   // [links]
+};
+
+// Host copy of the loaded flow tables (the path scheduler's rule
+// installation merges into it and reloads).
+struct pv_table_host {
+    std::vector<uint32_t> rule_offs, port_offs, host_ip;
+    std::vector<pv_rule> rules;
+    std::vector<uint8_t> region;
+    std::vector<int32_t> port_peer;
+    std::vector<uint16_t> host_switch, host_port;
 };
 
 // Path constraints of flow sets (pv_load_path_policies): per policy
@@ -86,6 +100,7 @@ struct pv_ctx {
     size_t scratch_bytes = 0;
     pv_cluster_state cl;
     pv_table_state tb;
+    pv_table_host tbh;
     pv_policy_state pol;
 };
 

@@ -99,3 +99,26 @@ def test_create_without_gpu_fails_cleanly():
 def test_missing_library_raises(tmp_path):
     with pytest.raises(RuntimeError):
         B.load_library(str(tmp_path / "nope.so"))
+
+
+def test_path_request_layout_matches_header(tmp_path):
+    src = tmp_path / "req.c"
+    src.write_text(r'''
+#include <stddef.h>
+#include <stdio.h>
+#include "pv.h"
+int main(void) {
+  printf("%zu %zu %zu %zu %zu\n", sizeof(pv_path_req), offsetof(pv_path_req, dst_host),
+         offsetof(pv_path_req, allowed_mask), offsetof(pv_path_req, policy), offsetof(pv_path_req, reserved));
+  printf("%d %d %d %d %d\n", PV_PATH_OK, PV_PATH_NOSRC, PV_PATH_BLOCKED, PV_PATH_TOO_LONG, PV_PATH_REPEAT);
+  return 0;
+}
+''')
+    exe = tmp_path / "req"
+    subprocess.check_call(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)])
+    lines = subprocess.check_output([str(exe)], text=True).split("\n")
+    f = W.PATH_REQ_DTYPE.fields
+    assert [int(x) for x in lines[0].split()] == [W.PATH_REQ_DTYPE.itemsize, f["dst_host"][1], f["allowed_mask"][1],
+                                                  f["policy"][1], f["reserved"][1]]
+    assert [int(x) for x in lines[1].split()] == [W.PATH_OK, W.PATH_NOSRC, W.PATH_BLOCKED, W.PATH_TOO_LONG,
+                                                  W.PATH_REPEAT]
