@@ -416,6 +416,81 @@ class PlacementTermsBench:
         return self.t.num_pods
 
 
+class ScheduleBench:
+    name = "path scheduling on the end-to-end network"
+    unit = "scheduled paths/s"
+    max_len = 64
+
+    def __init__(self, seed):
+        e = W.end_to_end(seed=20260220 + seed, num_intents=8, probes_per_intent=1)
+        self.net = e.network
+        self.pol = W.path_policies(20260223 + seed, self.net, 10_000)
+        self.req = W.path_requests(20260224 + seed, self.net, 10_000, num_policies=10_000, extra_regions=(6, 14))
+        self.weights = W.Stream(20260225 + seed, "link-weights").ints(1, 16, int(self.net.port_offs[-1])).astype(
+            np.uint16)
+
+    def config(self):
+        return {"workload": self.name, "switches": self.net.num_switches, "requests": len(self.req),
+                "path_policies": self.pol.num_policies, "waypoints": len(self.pol.must),
+                "forbidden_switches": len(self.pol.forbid), "max_len": self.max_len, "weights": "U[1,16] per link",
+                "l2": "working set L2-resident (small graph); every step recomputes all paths and rules"}
+
+    def setup(self, v):
+        from paper_2602_16100_gb300.validator import to_device, empty_device
+        self.v = v
+        v.load_network(self.net)
+        v.load_policies(self.pol)
+        d = v.device
+        R, L = len(self.req), self.max_len
+        self.d_req = to_device(self.req, d)
+        self.d_w = to_device(self.weights, d)
+        self.d_vis = empty_device(R * L * 4, d)
+        self.d_len = empty_device(R, d)
+        self.d_st = empty_device(R, d)
+        self.d_rules = empty_device(R * L * W.RULE_DTYPE.itemsize, d)
+        self.d_rsw = empty_device(R * L * 2, d)
+
+    def step(self, stream):
+        from paper_2602_16100_gb300 import binding as B
+        R, L = len(self.req), self.max_len
+        B.pv_schedule_paths(self.v.ctx, R, self.d_req, self.d_w, L, self.d_vis, self.d_len, self.d_st, stream)
+        B.pv_compile_path_rules(self.v.ctx, R, self.d_req, L, self.d_vis, self.d_len, self.d_st, 65535,
+                                self.d_rules, self.d_rsw, stream)
+
+    def measure_units(self):
+        import torch
+        st = self.d_st.to(torch.int64)
+        self.hist = torch.bincount(st, minlength=5).tolist()
+        self.mean_len = float(self.d_len.to(torch.float64).sum().item()) / max(1, self.hist[0])
+        return len(self.req)
+
+    def extra(self, secs_per_step):
+        return {"status_histogram": dict(zip(("ok", "nosrc", "blocked", "too_long", "repeat"), self.hist)),
+                "mean_visits_of_ok_paths": self.mean_len}
+
+    def algorithmic_bytes(self, group):
+        if group != "schedule":
+            return 0
+        R, L = len(self.req), self.max_len
+        # requests in, visits / lengths / statuses out, rules and their switches out
+        return R * (16 + 2) + int(self.hist[0] * self.mean_len) * 4 + R * L * (W.RULE_DTYPE.itemsize + 2)
+
+    def traffic_unit(self, group):
+        return None
+
+    def oracle_sample(self, n):
+        import oracle
+        t0 = time.perf_counter()
+        hops, ln, st = oracle.schedule_paths(self.net, self.req[:n], self.pol, self.weights, self.max_len)
+        oracle.compile_path_rules(self.net, self.req[:n], hops, ln, st)
+        return n, time.perf_counter() - t0, f"first {n} requests"
+
+    oracle_start = 50
+
+    def oracle_max(self):
+        return len(self.req)
+
+
 class FlowBench:
     name = "flow-verification"
     unit = "probe-hop verifications/s"
@@ -527,9 +602,9 @@ class WanBench:
         return len(self.q.masks) * len(self.q.sources)
 
 
-WORKLOADS = {"e2e": EndToEndBench, "placement_terms": PlacementTermsBench,
+WORKLOADS = {"e2e": EndToEndBench, "placement_terms": PlacementTermsBench, "schedule": ScheduleBench,
              "e2e_policies": lambda seed, **kw: EndToEndBench(seed, policies=True, **kw), "placement": PlacementBench, "flow": FlowBench, "wan": WanBench}
-SOURCES = {"walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector": ("k_selector.cu",),
+SOURCES = {"schedule": ("k_sched.cu",), "walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector": ("k_selector.cu",),
            "reach": ("k_reach.cu",)}
 
 

@@ -472,7 +472,7 @@ int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value);
  * ------------------------------------------------------------------------- */
 enum {
     PV_K_SELECTOR = 0, PV_K_PLACE = 1, PV_K_BIND = 2, PV_K_WALK_INIT = 3, PV_K_WALK_REGROUP = 4,
-    PV_K_WALK_HOP = 5, PV_K_AGGREGATE = 6, PV_K_REACH = 7, PV_K_COUNT = 8
+    PV_K_WALK_HOP = 5, PV_K_AGGREGATE = 6, PV_K_REACH = 7, PV_K_SCHEDULE = 8, PV_K_COUNT = 9
 };
 int pv_profile_enable(pv_ctx *ctx, int on);
 int pv_profile_collect(pv_ctx *ctx, pv_stream stream);

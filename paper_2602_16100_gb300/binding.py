@@ -34,7 +34,7 @@ SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", 
            "pv_eval_selector_terms", "pv_schedule_paths", "pv_compile_path_rules", "pv_install_path_rules")
 
 #: kernel groups timed by the library profiler (PV_K_* in include/pv.h)
-PV_K_NAMES = ("selector", "place", "bind", "walk_init", "walk_regroup", "walk_hop", "aggregate", "reach")
+PV_K_NAMES = ("selector", "place", "bind", "walk_init", "walk_regroup", "walk_hop", "aggregate", "reach", "schedule")
 
 _lib = None
 

@@ -251,7 +251,9 @@ extern "C" int pv_schedule_paths(pv_ctx *ctx, uint32_t num_requests, const pv_pa
     int per_sm = 1;
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sched_paths_kernel, kSchedThreads, smem);
     const uint32_t grid = std::min<uint32_t>(num_requests, (uint32_t)std::max(per_sm, 1) * ctx->num_sms);
+    const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_SCHEDULE);
     sched_paths_kernel<<<grid, kSchedThreads, smem, (cudaStream_t)stream>>>(a);
+    pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
     return pv_check_launch(ctx, "sched_paths_kernel");
 }
 
@@ -268,9 +270,11 @@ extern "C" int pv_compile_path_rules(pv_ctx *ctx, uint32_t num_requests, const p
         return pv_fail(ctx, PV_EINVAL, "pv_compile_path_rules: NULL device pointer");
     const size_t total = (size_t)num_requests * max_len;
     const uint32_t grid = (uint32_t)std::min<size_t>((total + 255) / 256, (size_t)ctx->num_sms * 8);
+    const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_SCHEDULE);
     compile_path_rules_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(num_requests, d_requests, t.d_host_ip,
                                                                       t.num_hosts, max_len, d_visits, d_len,
                                                                       d_status, priority, d_rules, d_rule_switch);
+    pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
     return pv_check_launch(ctx, "compile_path_rules_kernel");
 }
 
