@@ -433,6 +433,10 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  *   hop_cap - 1 and is finished there with the PV_LOOP result the full walk
  *   gives (checkpoints at hops 4, 8, 16, ...); 1 = walk every hop to the cap.
  *   Both give the same results; PV_STAT_WALK_LIVE_TOTAL differs.
+ * PV_OPT_WALK_TAIL_HOP: with the indexed kernel, the walk's hops from this
+ *   one on (default 8; 0 = none) run in a single launch, one thread per
+ *   probe still walking, tables read from L2 instead of staged per switch.
+ *   Same results.
  * PV_OPT_REACH_KERNEL: 0 = automatic (on a symmetric graph, rows are the
  *   connected components of the permitted subgraph; otherwise multi-source
  *   pull sweeps), 1 = sweeps always.  Both give the same rows.
@@ -452,7 +456,7 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  * ------------------------------------------------------------------------- */
 enum {
     PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4,
-    PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6
+    PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6, PV_OPT_WALK_TAIL_HOP = 7
 };
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,

@@ -23,7 +23,7 @@ PV_OK, PV_EINVAL, PV_ENOMEM, PV_ECUDA, PV_ESTATE, PV_ETIMEOUT, PV_ENOTIMPL = ran
 PV_OPT_SELECTOR_KERNEL, PV_OPT_WALK_KERNEL, PV_OPT_WALK_LANE_MAX, PV_OPT_TEST_STALL_STAGING = 1, 2, 3, 4
 PV_STAT_SELECTOR_ROWS_BUILT, PV_STAT_SCRATCH_BYTES, PV_STAT_WALK_INDEX_FITS, PV_STAT_WALK_INDEX_BYTES = 1, 2, 3, 4
 PV_STAT_WALK_LIVE_TOTAL, PV_STAT_REACH_COMPONENTS = 5, 6
-PV_OPT_REACH_KERNEL, PV_OPT_WALK_CYCLES = 5, 6
+PV_OPT_REACH_KERNEL, PV_OPT_WALK_CYCLES, PV_OPT_WALK_TAIL_HOP = 5, 6, 7
 
 #: every entry point declared in include/pv.h
 SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", "pv_load_cluster",

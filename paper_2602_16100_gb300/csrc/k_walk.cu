@@ -860,7 +860,7 @@ __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const Bl
 constexpr uint32_t kAlive = 0xFFu;
 constexpr uint32_t kViolationNext = 0xFEu;
 
-__device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t fm, uint32_t dst, uint32_t mask,
+__device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t hop, uint32_t fm, uint32_t dst, uint32_t mask,
                                             uint32_t pbase, uint32_t nports, uint32_t *status, uint32_t *next) {
     *next = 0;
     const uint32_t act = fm & 0xFFFFu;
@@ -874,7 +874,7 @@ __device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t fm, uint3
     } else if (peer & PV_PEER_HOST) {
         const uint32_t q = (uint32_t)(peer & ~PV_PEER_HOST);
         *status = (q < g.H && g.host_ip[q] == dst) ? PV_COMPLIANT : PV_MISDELIVERED;
-    } else if (g.hop + 1 >= g.cap) {
+    } else if (hop + 1 >= g.cap) {
         *status = PV_LOOP;
     } else {
         const uint32_t r2 = g.region[(uint32_t)peer >> 8];
@@ -973,7 +973,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             if (lane_mode) {
                 const bool act = lane < cnt && !fin_now;
                 const uint32_t fm = first_match_lane(s_raw, L, act, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu);
-                if (act) hop_outcome(g, fm, pr.y, pr.w, pbase, nports, &my_status, &my_next);
+                if (act) hop_outcome(g, g.hop, fm, pr.y, pr.w, pbase, nports, &my_status, &my_next);
             } else {
                 for (uint32_t j = 0; j < cnt; ++j) {
                     if ((fin_lanes >> j) & 1u) continue;
@@ -985,7 +985,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                     const uint32_t fm = kIndexed ? first_match_indexed(s_raw, hdr, lane, src, dst, dport, in_port)
                                                  : first_match_linear(s_raw, hdr.x, lane, src, dst, dport, in_port);
                     uint32_t status, next;
-                    hop_outcome(g, fm, dst, mask, pbase, nports, &status, &next);
+                    hop_outcome(g, g.hop, fm, dst, mask, pbase, nports, &status, &next);
                     if (lane == j) {
                         my_status = status;
                         my_next = next;
@@ -1031,6 +1031,117 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     }
     __syncthreads();
     if (threadIdx.x == 0) g.next_desc[blockIdx.x] = make_uint2(r0, s_count);
+}
+
+// First match of one probe by one thread, reading the switch's blob from
+// global memory (L2-resident tables): the per-lane walk of first_match_lane
+// without its warp phases.
+__device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict__ blob, const BlobLayout &L,
+                                                       uint32_t src, uint32_t dst, uint32_t dport,
+                                                       uint32_t in_port) {
+    const uint4 *A = reinterpret_cast<const uint4 *>(blob + L.a);
+    const uint2 *Bv = reinterpret_cast<const uint2 *>(blob + L.b);
+    const uint32_t *boff = reinterpret_cast<const uint32_t *>(blob + L.boff);
+    const uint16_t *items = reinterpret_cast<const uint16_t *>(blob + L.items);
+    const uint2 *segs = reinterpret_cast<const uint2 *>(blob + L.segs);
+    const uint32_t *bnd = reinterpret_cast<const uint32_t *>(blob + L.bnd);
+    const uint32_t *win = reinterpret_cast<const uint32_t *>(blob + L.win);
+    const uint32_t k = dport >> kBucketShift;
+    const uint32_t i1 = __ldg(boff + k + 1);
+    for (uint32_t i = __ldg(boff + k); i < i1; ++i) {
+        const uint32_t it = __ldg(items + i);
+        if (it & kSegItem) {
+            const uint2 sd = __ldg(segs + (it & 0x7FFFu));
+            uint32_t lo = 0, len = sd.y;   // bnd[sd.x] = 0 <= dst
+            while (len > 1) {
+                const uint32_t half = len >> 1;
+                lo = __ldg(bnd + sd.x + lo + half) <= dst ? lo + half : lo;
+                len -= half;
+            }
+            const uint32_t w = __ldg(win + sd.x + lo);
+            if (w & kWinFound) return w;
+            continue;
+        }
+        const uint4 a = __ldg(A + it);
+        const uint2 bb = __ldg(Bv + it);
+        const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
+        if (diff == 0 && dport >= (bb.x & 0xFFFFu) && dport <= (bb.x >> 16)) return kWinFound | (bb.y >> 16);
+    }
+    return 0u;
+}
+
+// The walk's last hops, first_hop .. cap - 1, in one launch: one thread per
+// probe still walking (the unsorted list the last hop kernel wrote, read
+// through its per-block slices), each thread taking its probe hop after hop
+// to the end with the tables read from L2.  Few probes are left by then, so
+// regrouping them by switch every hop would cost more in launches than the
+// table staging saves.  Results, cycle finishing, path constraints and the
+// per-hop live counts are those of walk_hop_kernel.
+template <bool kPolicy>
+__global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *__restrict__ list,
+                                                        const uint2 *__restrict__ desc, uint32_t nslices,
+                                                        uint32_t first_hop) {
+    const uint32_t lane = threadIdx.x & 31;
+    for (uint32_t sl = blockIdx.x; sl < nslices; sl += gridDim.x) {
+        const uint2 d = desc[sl];
+        for (uint32_t base = d.x; base < d.x + d.y; base += blockDim.x) {
+            const uint32_t i = base + threadIdx.x;
+            bool active = i < d.x + d.y;
+            uint2 e = make_uint2(0, 0);
+            uint4 pr = make_uint4(0, 0, 0, 0);
+            if (active) {
+                e = list[i];
+                pr = __ldg(reinterpret_cast<const uint4 *>(g.probes) + e.x);
+            }
+            uint32_t loc = e.y;
+            for (uint32_t h = first_hop; h < g.cap; ++h) {
+                const uint32_t live = __ballot_sync(PV_FULL_MASK, active);
+                if (!live) break;
+                if (lane == 0) atomicAdd(&g.hop_live[h], (uint32_t)__popc(live));
+                if (!active) continue;
+                const uint32_t s = (loc >> 8) & 0xFFFFu, in_port = loc & 0xFFu, fin = loc >> 24;
+                uint32_t *out = reinterpret_cast<uint32_t *>(g.out) + e.x;   // {status, hops, last_switch}
+                if (fin != 0 && fin - 1 == h) {   // finished at its cycle position
+                    *out = (uint32_t)PV_LOOP | g.cap << 8 | s << 16;
+                    active = false;
+                    continue;
+                }
+                const uint8_t *blob = g.blob + g.blob_offs[s];
+                const uint4 hdr = __ldg(reinterpret_cast<const uint4 *>(blob));
+                const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
+                const uint32_t fm = first_match_thread(blob, L, pr.x, pr.y, pr.z & 0xFFFFu, in_port);
+                const uint32_t pbase = g.port_offs[s], nports = g.port_offs[s + 1] - pbase;
+                uint32_t status, next;
+                hop_outcome(g, h, fm, pr.y, pr.w, pbase, nports, &status, &next);
+                if (kPolicy) {
+                    const uint4 ph = policy_of(g.pa, e.x);
+                    uint32_t bits = 0;
+                    for (uint32_t k = 0; k < ph.w; ++k)
+                        if (g.pa.sw[ph.z + k] == s) bits |= 1u << k;
+                    if (bits) g.pa.hits[e.x] |= bits;
+                    if (status == kAlive && switch_listed(g.pa.sw + ph.x, ph.y, next >> 8)) status = kViolationNext;
+                }
+                if (status != kAlive) {
+                    const bool at_next = status == kViolationNext;
+                    *out = (at_next ? (uint32_t)PV_VIOLATION : status) | (h + (at_next ? 2u : 1u)) << 8 |
+                           (at_next ? (next >> 8) : s) << 16;
+                    active = false;
+                    continue;
+                }
+                uint32_t nfin = fin;
+                const uint32_t h1 = h + 1;
+                if (g.cycles && nfin == 0 && h1 >= kCycleCheckFrom) {
+                    if ((h1 & (h1 - 1u)) == 0) {
+                        g.ck[e.x] = next;
+                    } else if (g.ck[e.x] == next) {
+                        const uint32_t period = h1 - (1u << (31 - __clz(h1)));
+                        nfin = h1 + (g.cap - 1u - h1) % period + 1u;
+                    }
+                }
+                loc = next | (nfin << 24);
+            }
+        }
+    }
 }
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1351,7 +1462,10 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
     g.wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
     uint32_t in_slices = init_grid;
-    for (uint32_t h = 0; h < hop_cap; ++h) {
+    // hops from tail_hop on run in one walk_tail_kernel launch (indexed tables only)
+    const uint32_t opt_tail = (uint32_t)ctx->opt_walk_tail_hop;
+    const uint32_t tail_hop = (indexed && opt_tail > 0 && opt_tail < hop_cap) ? opt_tail : hop_cap;
+    for (uint32_t h = 0; h < tail_hop; ++h) {
         uint2 *cur = (h & 1) ? listB : listA;
         uint2 *nxt = (h & 1) ? listA : listB;
         uint2 *dcur = (h & 1) ? descB : descA;
@@ -1376,6 +1490,20 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
             walk_hop_kernel<false, false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         pv_prof_stop(ctx, st, pr, 1);
         in_slices = hop_grid;
+    }
+    if (tail_hop < hop_cap) {
+        const uint32_t h = tail_hop - 1;   // the last regrouped hop wrote this list
+        uint2 *lst = (h & 1) ? listA : listB;
+        uint2 *dsc = (h & 1) ? descA : descB;
+        PV_TRY_CUDA(ctx, cudaMemsetAsync(ctx->d_walk_live + tail_hop, 0, (hop_cap - tail_hop) * sizeof(uint32_t), st),
+                    "tail live counts");
+        g.hop = tail_hop;
+        pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
+        if (pol)
+            walk_tail_kernel<true><<<hop_grid, 256, 0, st>>>(g, lst, dsc, hop_grid, tail_hop);
+        else
+            walk_tail_kernel<false><<<hop_grid, 256, 0, st>>>(g, lst, dsc, hop_grid, tail_hop);
+        pv_prof_stop(ctx, st, pr, 1);
     }
     return pv_check_launch(ctx, "probe walk kernels");
 }

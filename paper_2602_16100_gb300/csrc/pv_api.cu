@@ -250,6 +250,10 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "walk cycle option must be 0 or 1");
         ctx->opt_walk_cycles = (int)value;
         return PV_OK;
+    case PV_OPT_WALK_TAIL_HOP:
+        if (value < 0 || value > PV_MAX_HOP_CAP) return pv_fail(ctx, PV_EINVAL, "tail hop must be 0..255");
+        ctx->opt_walk_tail_hop = (int)value;
+        return PV_OK;
     case PV_OPT_REACH_KERNEL:
         if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "reach kernel must be 0 or 1");
         ctx->opt_reach = (int)value;

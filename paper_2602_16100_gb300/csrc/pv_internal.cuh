@@ -89,7 +89,8 @@ struct pv_ctx {
     int32_t *d_status = nullptr;      // first device-detected error (0 = none)
     int opt_selector = 0, opt_walk = 0;
     int opt_walk_lane_max = 96;
-    int opt_walk_cycles = 0;          // 0: finish probes in forwarding cycles early, 1: walk to the cap
+    int opt_walk_cycles = 0;
+    int opt_walk_tail_hop = 8;        // hops from here on run in one tail launch (0: never)          // 0: finish probes in forwarding cycles early, 1: walk to the cap
     int opt_test_stall_staging = 0;   // failure test: staging waits expect bytes that never come
     uint32_t *d_walk_live = nullptr;  // [PV_MAX_HOP_CAP + 1] live probes per hop of the last walk
     uint32_t last_walk_cap = 0;       // hop cap of the last walk

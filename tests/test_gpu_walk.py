@@ -194,6 +194,41 @@ def test_index_stress_tables(validator, seed):
     assert len(np.unique(o["status"])) >= 3
 
 
+@pytest.mark.parametrize("tail", [0, 1, 5, 8])
+def test_tail_launch_agrees(validator, tail):
+    """The last hops in one launch (one thread per probe, tables from L2)
+    give the results of the hop-by-hop walk, from any switch-over hop, with
+    and without path constraints; the live counts still add up."""
+    e = W.end_to_end(seed=33, num_switches=70, num_intents=40, probes_per_intent=400, rules_per_switch=200)
+    net = e.network
+    pr = e.probes.probes.copy()
+    st = W.Stream(33, "tail-probes")
+    pr["src_host"] = st.ints(0, net.num_hosts - 1, len(pr))
+    pr["src_ip"] = net.host_ip[pr["src_host"]]
+    o = oracle.verify_probes(net, pr, 32)
+    validator.set_option(B.PV_OPT_WALK_TAIL_HOP, tail)
+    try:
+        g = _gpu_walk(validator, net, pr, 32, 2)
+        assert _same(g, o)
+        validator.set_option(B.PV_OPT_WALK_CYCLES, 1)
+        g = _gpu_walk(validator, net, pr, 32, 2)
+        assert _same(g, o)
+        ran = o["status"] != W.ST_NOSRC
+        want = int(o["hops"][ran].astype(np.int64).sum()) - int((o["status"] == W.ST_VIOLATION).sum())
+        assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) == want
+        validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
+        from paper_2602_16100_gb300.validator import to_device as td
+        pol = W.path_policies(3, net, 40, forbid_max=2, must_max=3, hubs=8)
+        validator.load_policies(pol)
+        out, hits = validator.verify_constrained(td(pr, validator.device), len(pr), 32, None, 400)
+        validator.sync()
+        oc, oh = oracle.verify_constrained(net, pr, 32, pol, probes_per_policy=400)
+        assert (to_numpy(out, W.RESULT_DTYPE) == oc).all() and (to_numpy(hits, np.uint32) == oh).all()
+    finally:
+        validator.set_option(B.PV_OPT_WALK_TAIL_HOP, 8)
+        validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
+
+
 def test_walk_live_total_counts_hop_entries(validator):
     """PV_STAT_WALK_LIVE_TOTAL: probes entered at a switch, summed over hops.
     A probe whose next switch (its first one included) lies outside its mask
