@@ -154,7 +154,7 @@ class EndToEndBench:
                 "label_keys": e.cluster.num_keys, "switches": e.network.num_switches,
                 "rules_per_switch": int(np.diff(e.network.rule_offs).max()), "pods_per_intent": e.pods_per_intent,
                 "probes": len(e.probes.probes), "hop_cap": e.probes.hop_cap,
-                "l2": "inputs larger than L2 (800 MB probe array and 200 MB results per step)",
+                "l2": "inputs larger than L2 (400 MB of flows in, 800 MB of probe records built and 200 MB of results per step)",
                 **({"path_policies": self.pol.num_policies, "forbidden_switches": len(self.pol.forbid),
                     "waypoints": len(self.pol.must)} if self.pol is not None else {})}
 
@@ -211,30 +211,35 @@ class EndToEndBench:
         import torch
         e = self.e
         pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1).copy()).pin_memory()
+        from paper_2602_16100_gb300.validator import flows_of
         self.host = {"offs": pin(e.intents.expr_offs.astype(np.uint32)), "exprs": pin(e.intents.exprs),
-                     "draws": pin(e.place_draws.astype(np.uint64)), "probes": pin(e.probes.probes),
+                     "draws": pin(e.place_draws.astype(np.uint64)), "masks": pin(e.intent_mask.astype(np.uint32)),
+                     "flows": pin(flows_of(e)),
                      "pass": torch.empty(e.intents.num_pods, dtype=torch.uint8).pin_memory(),
                      "counts": torch.empty(e.intents.num_pods * 32, dtype=torch.uint8).pin_memory()}
         self.copy_stream = torch.cuda.Stream()
         self.chunks = chunks
         net = e.network
-        self.h2d = (sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "probes"))
+        self.h2d = (sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "masks", "flows"))
                     + e.cluster.labels.nbytes + net.rule_offs.nbytes + net.rules.nbytes + net.switch_region.nbytes
                     + net.port_offs.nbytes + net.port_peer.nbytes + net.host_switch.nbytes + net.host_port.nbytes
                     + net.host_ip.nbytes)
         self.d2h = self.host["pass"].numel() + self.host["counts"].numel()
 
     def step_e2e(self, v, stream):
-        """Every input from host memory: cluster labels and flow tables
-        through the loaders, intents and probes copied (the probe upload
-        overlapped with verification, `chunks` intent ranges), verdicts and
-        counters copied back."""
+        """Every input from host memory: intents (selectors, placement draws,
+        masks) and their flows copied (8 B per flow), the cluster labels and
+        flow tables loaded meanwhile, verification of `chunks` intent ranges
+        as their flows arrive, verdicts and counters copied back."""
         e = self.e
-        v.load_cluster(e.cluster)
-        v.load_network(e.network)
-        if self.pol is not None:
-            v.load_policies(self.pol)
-        v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks)
+
+        def loads():
+            v.load_cluster(e.cluster)
+            v.load_network(e.network)
+            if self.pol is not None:
+                v.load_policies(self.pol)
+
+        v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks, loads)
 
     def e2e_phases(self, v, stream, reps=3):
         """Each part of the host-buffer step alone (diagnostic, after the
@@ -254,7 +259,7 @@ class EndToEndBench:
         t0 = time.perf_counter()
         for _ in range(reps):
             with torch.cuda.stream(self.copy_stream):
-                for k in ("offs", "exprs", "draws", "probes"):
+                for k in ("offs", "exprs", "draws", "masks", "flows"):
                     self.dev[k][: self.host[k].numel()].copy_(self.host[k], non_blocking=True)
         torch.cuda.synchronize()
         upload = (time.perf_counter() - t0) / reps
@@ -263,7 +268,7 @@ class EndToEndBench:
             self.v.run_end_to_end(self.dev, self.sizes, stream)
         torch.cuda.synchronize()
         dev = (time.perf_counter() - t0) / reps
-        up_bytes = sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "probes"))
+        up_bytes = sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "masks", "flows"))
         return {"load_tables_ms": load * 1e3, "upload_inputs_ms": upload * 1e3,
                 "upload_gbs": up_bytes / upload / 1e9, "device_pipeline_ms": dev * 1e3}
 

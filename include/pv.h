@@ -115,6 +115,11 @@ typedef struct {           /* one walk result, 4 bytes                          
     uint8_t hops;          /* switch visits made (hop_cap for PV_LOOP, 0 for PV_NOSRC)   */
     uint16_t last_switch;  /* last switch visited (0xFFFF for PV_NOSRC)                   */
 } pv_result;
+typedef struct {           /* one flow of an intent, 8 bytes                             */
+    uint32_t dst_ip;       /* destination address                                        */
+    uint16_t dport;        /* destination port                                           */
+    uint16_t reserved;     /* 0                                                          */
+} pv_flow;
 typedef struct {           /* one path request of the scheduler, 16 bytes                */
     uint16_t src_host;     /* source host id                                             */
     uint16_t dst_host;     /* destination host id                                        */
@@ -316,6 +321,10 @@ int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_
  *   the host of pod (k mod probes_per_group) mod pods_per_group of g:
  *   src_host and src_ip are rewritten in place (PV_NO_HOST / 0 when that pod
  *   is unplaced or not a host).  Needs the flow tables (host_ip).
+ * pv_bind_flows: the same binding from the compact form of an intent's
+ *   flows: d_flows[k] = {dst_ip, dport} and the group's jurisdiction mask
+ *   d_group_mask[g] give the whole probe record d_probes[k] (16-byte
+ *   aligned), its source bound as above.
  * pv_aggregate_intents: d_pass[g] = 1 iff every pod of g has d_assign in
  *   row g, d_group_flags[g] has neither PV_F_UNKNOWN_VALUE nor
  *   PV_F_BAD_EXPR, and every probe of g is PV_COMPLIANT.
@@ -323,6 +332,9 @@ int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_
  *   feasible node, [7] zero.
  * Errors: PV_ESTATE, PV_EINVAL (zero group sizes, NULL pointers).
  * ------------------------------------------------------------------------- */
+int pv_bind_flows(pv_ctx *ctx, uint32_t num_probes, const pv_flow *d_flows, uint32_t probes_per_group,
+                  uint32_t pods_per_group, const uint32_t *d_assign, const uint32_t *d_group_mask,
+                  pv_probe *d_probes, pv_stream stream);
 int pv_place_pods(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_group, const uint32_t *d_bits,
                   uint32_t words_per_row, const uint64_t *d_draws, uint32_t *d_assign, pv_stream stream);
 int pv_bind_probes(pv_ctx *ctx, uint32_t num_probes, pv_probe *d_probes, uint32_t probes_per_group,

@@ -165,6 +165,45 @@ extern "C" int pv_place_pods(pv_ctx *ctx, uint32_t G, uint32_t pods, const uint3
     return pv_check_launch(ctx, "place_pods_kernel");
 }
 
+// Probe records from compact flows: {src_ip, dst_ip, dport | src_host << 16,
+// mask}, the source bound as in bind_probes_kernel.
+__global__ void __launch_bounds__(kThreads) bind_flows_kernel(uint32_t M, const uint2 *__restrict__ flows,
+                                                              uint32_t ppg, uint32_t pods,
+                                                              const uint32_t *__restrict__ assign,
+                                                              const uint32_t *__restrict__ group_mask, uint32_t H,
+                                                              const uint32_t *__restrict__ host_ip,
+                                                              uint4 *__restrict__ probes) {
+    for (uint32_t k = blockIdx.x * kThreads + threadIdx.x; k < M; k += gridDim.x * kThreads) {
+        const uint32_t g = k / ppg;
+        const uint32_t node = assign[g * pods + (k - g * ppg) % pods];
+        const uint2 f = __ldg(flows + k);
+        const bool placed = node < H;
+        probes[k] = make_uint4(placed ? host_ip[node] : 0u, f.x,
+                               (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16, group_mask[g]);
+    }
+}
+
+extern "C" int pv_bind_flows(pv_ctx *ctx, uint32_t M, const pv_flow *d_flows, uint32_t ppg, uint32_t pods,
+                             const uint32_t *d_assign, const uint32_t *d_group_mask, pv_probe *d_probes,
+                             pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->tb.loaded) return pv_fail(ctx, PV_ESTATE, "pv_bind_flows: no flow tables loaded");
+    if (M == 0) return PV_OK;
+    if (ppg == 0 || pods == 0) return pv_fail(ctx, PV_EINVAL, "pv_bind_flows: group sizes must be > 0");
+    if (!d_flows || !d_assign || !d_group_mask || !d_probes)
+        return pv_fail(ctx, PV_EINVAL, "pv_bind_flows: NULL device pointer");
+    if (((uintptr_t)d_probes & 15) != 0 || ((uintptr_t)d_flows & 7) != 0)
+        return pv_fail(ctx, PV_EINVAL, "pv_bind_flows: d_probes must be 16-byte and d_flows 8-byte aligned");
+    pv_use_begin(ctx, (cudaStream_t)stream);
+    const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_BIND);
+    bind_flows_kernel<<<grid_for(ctx, M, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
+        M, reinterpret_cast<const uint2 *>(d_flows), ppg, pods, d_assign, d_group_mask, ctx->tb.num_hosts,
+        ctx->tb.d_host_ip, reinterpret_cast<uint4 *>(d_probes));
+    pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    pv_mark_use(ctx, (cudaStream_t)stream);
+    return pv_check_launch(ctx, "bind_flows_kernel");
+}
+
 extern "C" int pv_bind_probes(pv_ctx *ctx, uint32_t M, pv_probe *d_probes, uint32_t ppg, uint32_t pods,
                               const uint32_t *d_assign, pv_stream stream) {
     if (!ctx) return PV_EINVAL;
@@ -172,10 +211,12 @@ extern "C" int pv_bind_probes(pv_ctx *ctx, uint32_t M, pv_probe *d_probes, uint3
     if (M == 0) return PV_OK;
     if (ppg == 0 || pods == 0) return pv_fail(ctx, PV_EINVAL, "pv_bind_probes: group sizes must be > 0");
     if (!d_probes || !d_assign) return pv_fail(ctx, PV_EINVAL, "pv_bind_probes: NULL device pointer");
+    pv_use_begin(ctx, (cudaStream_t)stream);
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_BIND);
     bind_probes_kernel<<<grid_for(ctx, M, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
         M, d_probes, ppg, pods, d_assign, ctx->tb.num_hosts, ctx->tb.d_host_ip);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    pv_mark_use(ctx, (cudaStream_t)stream);
     return pv_check_launch(ctx, "bind_probes_kernel");
 }
 
@@ -190,11 +231,13 @@ extern "C" int pv_aggregate_intents(pv_ctx *ctx, uint32_t G, uint32_t pods, cons
     if (!d_bits || !d_gflags || !d_assign || !d_pass || !d_counts || (ppg && !d_results))
         return pv_fail(ctx, PV_EINVAL, "pv_aggregate_intents: NULL device pointer");
     if (W < (ctx->cl.num_nodes + 31) / 32) return pv_fail(ctx, PV_EINVAL, "pv_aggregate_intents: words_per_row too small");
+    pv_use_begin(ctx, (cudaStream_t)stream);
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_AGGREGATE);
     aggregate_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
         G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts, nullptr,
         nullptr, 0, 0, nullptr, nullptr);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    pv_mark_use(ctx, (cudaStream_t)stream);
     return pv_check_launch(ctx, "aggregate_kernel");
 }
 
@@ -212,10 +255,12 @@ extern "C" int pv_aggregate_constrained(pv_ctx *ctx, uint32_t G, uint32_t pods, 
         return pv_fail(ctx, PV_EINVAL, "pv_aggregate_constrained: NULL device pointer");
     if (W < (ctx->cl.num_nodes + 31) / 32)
         return pv_fail(ctx, PV_EINVAL, "pv_aggregate_constrained: words_per_row too small");
+    pv_use_begin(ctx, (cudaStream_t)stream);
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_AGGREGATE);
     aggregate_kernel<<<grid_for(ctx, (size_t)G * 32, kThreads), kThreads, 0, (cudaStream_t)stream>>>(
         G, pods, ctx->cl.num_nodes, d_bits, W, d_gflags, d_assign, ppg, d_results, d_pass, d_counts,
         d_waypoints, d_group_policy, first_policy, ctx->pol.num, ctx->pol.d_hdr, ctx->pol.d_concrete);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    pv_mark_use(ctx, (cudaStream_t)stream);
     return pv_check_launch(ctx, "aggregate_kernel");
 }

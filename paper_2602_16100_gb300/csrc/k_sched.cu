@@ -251,9 +251,11 @@ extern "C" int pv_schedule_paths(pv_ctx *ctx, uint32_t num_requests, const pv_pa
     int per_sm = 1;
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sched_paths_kernel, kSchedThreads, smem);
     const uint32_t grid = std::min<uint32_t>(num_requests, (uint32_t)std::max(per_sm, 1) * ctx->num_sms);
+    pv_use_begin(ctx, (cudaStream_t)stream);
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_SCHEDULE);
     sched_paths_kernel<<<grid, kSchedThreads, smem, (cudaStream_t)stream>>>(a);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    pv_mark_use(ctx, (cudaStream_t)stream);
     return pv_check_launch(ctx, "sched_paths_kernel");
 }
 
@@ -270,11 +272,13 @@ extern "C" int pv_compile_path_rules(pv_ctx *ctx, uint32_t num_requests, const p
         return pv_fail(ctx, PV_EINVAL, "pv_compile_path_rules: NULL device pointer");
     const size_t total = (size_t)num_requests * max_len;
     const uint32_t grid = (uint32_t)std::min<size_t>((total + 255) / 256, (size_t)ctx->num_sms * 8);
+    pv_use_begin(ctx, (cudaStream_t)stream);
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_SCHEDULE);
     compile_path_rules_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(num_requests, d_requests, t.d_host_ip,
                                                                       t.num_hosts, max_len, d_visits, d_len,
                                                                       d_status, priority, d_rules, d_rule_switch);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
+    pv_mark_use(ctx, (cudaStream_t)stream);
     return pv_check_launch(ctx, "compile_path_rules_kernel");
 }
 
@@ -286,13 +290,23 @@ extern "C" int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_r
     if (!d_rules || !d_rule_switch) return pv_fail(ctx, PV_EINVAL, "pv_install_path_rules: NULL device pointer");
     std::vector<pv_rule> add(num_slots);
     std::vector<uint16_t> sw(num_slots);
-    PV_TRY_CUDA(ctx, cudaDeviceSynchronize(), "pv_install_path_rules sync");
-    PV_TRY_CUDA(ctx, cudaMemcpy(add.data(), d_rules, (size_t)num_slots * sizeof(pv_rule), cudaMemcpyDeviceToHost),
-                "path rules download");
-    PV_TRY_CUDA(ctx, cudaMemcpy(sw.data(), d_rule_switch, (size_t)num_slots * 2, cudaMemcpyDeviceToHost),
-                "path rule switches download");
+    // the compiled rules come from an evaluation call: wait for it, then read
+    // them and the loaded rules on the load stream
+    if (int rc0 = pv_load_begin(ctx)) return rc0;
+    cudaStream_t ls = ctx->load_stream;
     const pv_table_host h = ctx->tbh;   // copy: the reload below replaces ctx->tbh
     const uint32_t S = (uint32_t)h.region.size();
+    std::vector<pv_rule> base(h.rule_offs[S]);
+    PV_TRY_CUDA(ctx, cudaMemcpyAsync(add.data(), d_rules, (size_t)num_slots * sizeof(pv_rule),
+                                     cudaMemcpyDeviceToHost, ls),
+                "path rules download");
+    PV_TRY_CUDA(ctx, cudaMemcpyAsync(sw.data(), d_rule_switch, (size_t)num_slots * 2, cudaMemcpyDeviceToHost, ls),
+                "path rule switches download");
+    if (!base.empty())
+        PV_TRY_CUDA(ctx, cudaMemcpyAsync(base.data(), ctx->tb.d_raw, base.size() * sizeof(pv_rule),
+                                         cudaMemcpyDeviceToHost, ls),
+                    "loaded rules download");
+    PV_TRY_CUDA(ctx, cudaStreamSynchronize(ls), "pv_install_path_rules");
     std::vector<uint32_t> count(S, 0);
     for (uint32_t k = 0; k < num_slots; ++k)
         if (sw[k] < S) ++count[sw[k]];
@@ -303,7 +317,7 @@ extern "C" int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_r
     for (uint32_t k = 0; k < num_slots; ++k)   // new rules first, in slot order: they win priority ties
         if (sw[k] < S) rules[cur[sw[k]]++] = add[k];
     for (uint32_t s = 0; s < S; ++s)
-        for (uint32_t i = h.rule_offs[s]; i < h.rule_offs[s + 1]; ++i) rules[cur[s]++] = h.rules[i];
+        for (uint32_t i = h.rule_offs[s]; i < h.rule_offs[s + 1]; ++i) rules[cur[s]++] = base[i];
     return pv_load_flow_tables(ctx, S, offs.data(), rules.data(), h.region.data(), h.port_offs.data(),
                                h.port_peer.data(), (uint32_t)h.host_ip.size(), h.host_switch.data(),
                                h.host_port.data(), h.host_ip.data());

@@ -446,47 +446,47 @@ extern "C" int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_key
     if (num_nodes == 0 || num_keys == 0 || !labels)
         return pv_fail(ctx, PV_EINVAL, "pv_load_cluster: empty cluster or NULL labels");
     if (num_keys > kMaxKeys) return pv_fail(ctx, PV_EINVAL, "pv_load_cluster: num_keys > %u", kMaxKeys);
-    PV_TRY_CUDA(ctx, cudaSetDevice(ctx->device), "cudaSetDevice");
-    PV_TRY_CUDA(ctx, cudaDeviceSynchronize(), "pv_load_cluster sync");
-    pv_free_cluster(ctx->cl);
+    if (int rc0 = pv_load_begin(ctx)) return rc0;
+    pv_free_cluster(ctx, ctx->cl);
+    cudaStream_t ls = ctx->load_stream;
     pv_cluster_state &c = ctx->cl;
     const size_t nl = (size_t)num_nodes * num_keys;
     int rc;
-    if ((rc = pv_device_alloc(ctx, (void **)&c.d_labels, nl * 2, "labels")) ||
-        (rc = pv_device_alloc(ctx, (void **)&c.d_inv, (size_t)num_keys * kInvWords * 4, "inventory")) ||
-        (rc = pv_device_alloc(ctx, (void **)&c.d_inv_rank, (size_t)num_keys * kInvWords * 4, "inventory rank")) ||
-        (rc = pv_device_alloc(ctx, (void **)&c.d_key_base, ((size_t)num_keys + 1) * 4 * 2, "key base"))) {
-        pv_free_cluster(c);
+    if ((rc = pv_pool_alloc(ctx, (void **)&c.d_labels, nl * 2, "labels")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&c.d_inv, (size_t)num_keys * kInvWords * 4, "inventory")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&c.d_inv_rank, (size_t)num_keys * kInvWords * 4, "inventory rank")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&c.d_key_base, ((size_t)num_keys + 1) * 4 * 2, "key base"))) {
+        pv_free_cluster(ctx, c);
         return rc;
     }
     uint32_t *d_count = c.d_key_base + (num_keys + 1);
-    PV_TRY_CUDA(ctx, cudaMemcpy(c.d_labels, labels, nl * 2, cudaMemcpyHostToDevice), "labels upload");
-    PV_TRY_CUDA(ctx, cudaMemset(c.d_inv, 0, (size_t)num_keys * kInvWords * 4), "inventory clear");
-    build_inventory_kernel<<<ctx->num_sms * 8, 256>>>(num_nodes, num_keys, c.d_labels, c.d_inv);
-    inventory_rank_kernel<<<num_keys, 1024>>>(c.d_inv, c.d_inv_rank, d_count);
-    key_base_kernel<<<1, 1024>>>(num_keys, d_count, c.d_key_base);
-    if ((rc = pv_check_launch(ctx, "inventory kernels"))) { pv_free_cluster(c); return rc; }
+    PV_TRY_CUDA(ctx, cudaMemcpyAsync(c.d_labels, labels, nl * 2, cudaMemcpyHostToDevice, ls), "labels upload");
+    PV_TRY_CUDA(ctx, cudaMemsetAsync(c.d_inv, 0, (size_t)num_keys * kInvWords * 4, ls), "inventory clear");
+    build_inventory_kernel<<<ctx->num_sms * 8, 256, 0, ls>>>(num_nodes, num_keys, c.d_labels, c.d_inv);
+    inventory_rank_kernel<<<num_keys, 1024, 0, ls>>>(c.d_inv, c.d_inv_rank, d_count);
+    key_base_kernel<<<1, 1024, 0, ls>>>(num_keys, d_count, c.d_key_base);
+    if ((rc = pv_check_launch(ctx, "inventory kernels"))) { pv_free_cluster(ctx, c); return rc; }
     uint32_t nvr = 0;
-    PV_TRY_CUDA(ctx, cudaMemcpy(&nvr, c.d_key_base + num_keys, 4, cudaMemcpyDeviceToHost), "value count");
+    PV_TRY_CUDA(ctx, cudaMemcpyAsync(&nvr, c.d_key_base + num_keys, 4, cudaMemcpyDeviceToHost, ls), "value count");
+    PV_TRY_CUDA(ctx, cudaStreamSynchronize(ls), "value count");
     c.num_nodes = num_nodes;
     c.num_keys = num_keys;
     c.row_words = words_for(num_nodes);
     c.num_value_rows = nvr;
     const uint64_t row_bytes = ((uint64_t)nvr + num_keys) * c.row_words * 4;
     if (row_bytes <= kRowBudgetBytes) {
-        if (pv_device_alloc(ctx, (void **)&c.d_rows, row_bytes, "value rows") == PV_OK) {
-            PV_TRY_CUDA(ctx, cudaMemset(c.d_rows, 0, row_bytes), "value rows clear");
-            build_rows_kernel<<<ctx->num_sms * 8, 256>>>(num_nodes, num_keys, c.d_labels, c.d_inv, c.d_inv_rank,
+        if (pv_pool_alloc(ctx, (void **)&c.d_rows, row_bytes, "value rows") == PV_OK) {
+            PV_TRY_CUDA(ctx, cudaMemsetAsync(c.d_rows, 0, row_bytes, ls), "value rows clear");
+            build_rows_kernel<<<ctx->num_sms * 8, 256, 0, ls>>>(num_nodes, num_keys, c.d_labels, c.d_inv, c.d_inv_rank,
                                                           c.d_key_base, nvr, c.row_words, c.d_rows);
-            if ((rc = pv_check_launch(ctx, "value rows"))) { pv_free_cluster(c); return rc; }
+            if ((rc = pv_check_launch(ctx, "value rows"))) { pv_free_cluster(ctx, c); return rc; }
             c.rows_built = true;
         } else {
             ctx->err.clear();   // rows are optional; fall back to the comparison kernel
         }
     }
-    PV_TRY_CUDA(ctx, cudaDeviceSynchronize(), "pv_load_cluster");
     c.loaded = true;
-    return PV_OK;
+    return pv_load_end(ctx);
 }
 
 extern "C" int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_expr_offs, uint32_t num_exprs,
@@ -508,12 +508,14 @@ extern "C" int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t 
     cudaStream_t st = (cudaStream_t)stream;
     if (which == 2) {
         uint32_t blocks = std::min<uint32_t>((num_pods + 7) / 8, (uint32_t)ctx->num_sms * 16);
+        pv_use_begin(ctx, st);
         const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
         sel_rows_kernel<<<blocks, kRowsThreads, 0, st>>>(c.num_nodes, c.num_keys, num_pods, d_expr_offs, num_exprs,
                                                          d_exprs, d_assign, d_bits, words_per_row, d_flags, c.d_inv,
                                                          c.d_inv_rank, c.d_key_base, c.d_rows, c.row_words,
                                                          c.num_value_rows);
         pv_prof_stop(ctx, st, pr, 1);
+        pv_mark_use(ctx, st);
         return pv_check_launch(ctx, "sel_rows_kernel");
     }
     // tile: as many nodes (multiple of 32) as fit 96 KB of label columns
@@ -525,11 +527,13 @@ extern "C" int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t 
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(sel_cmp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
                 "sel_cmp_kernel smem");
     const uint32_t blocks = (num_pods + kCmpPods - 1) / kCmpPods;
+    pv_use_begin(ctx, st);
     const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
     sel_cmp_kernel<<<blocks, kCmpThreads, smem, st>>>(c.num_nodes, c.num_keys, c.d_labels, tile, num_pods,
                                                       d_expr_offs, num_exprs, d_exprs, d_assign, d_bits,
                                                       words_per_row, d_flags, c.d_inv);
     pv_prof_stop(ctx, st, pr, 1);
+    pv_mark_use(ctx, st);
     return pv_check_launch(ctx, "sel_cmp_kernel");
 }
 
@@ -552,11 +556,13 @@ extern "C" int pv_eval_selector_terms(pv_ctx *ctx, uint32_t num_pods, const uint
         return pv_fail(ctx, PV_EINVAL, "pv_eval_selector_terms: value rows were not built for this cluster");
     cudaStream_t st = (cudaStream_t)stream;
     const uint32_t blocks = std::min<uint32_t>((num_pods + 7) / 8, (uint32_t)ctx->num_sms * 16);
+    pv_use_begin(ctx, st);
     const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
     sel_terms_kernel<<<blocks, kRowsThreads, 0, st>>>(c.num_nodes, c.num_keys, num_pods, d_pod_terms, num_terms,
                                                       d_term_offs, num_exprs, d_exprs, d_assign, d_bits,
                                                       words_per_row, d_flags, c.d_inv, c.d_inv_rank, c.d_key_base,
                                                       c.d_rows, c.row_words, c.num_value_rows);
     pv_prof_stop(ctx, st, pr, 1);
+    pv_mark_use(ctx, st);
     return pv_check_launch(ctx, "sel_terms_kernel");
 }

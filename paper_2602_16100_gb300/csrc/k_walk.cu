@@ -1196,63 +1196,61 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         if (host_switch[h] >= S || host_port[h] >= port_offs[host_switch[h] + 1] - port_offs[host_switch[h]])
             return pv_fail(ctx, PV_EINVAL, "host %u attachment out of range", h);
 
-    PV_TRY_CUDA(ctx, cudaSetDevice(ctx->device), "cudaSetDevice");
-    PV_TRY_CUDA(ctx, cudaDeviceSynchronize(), "pv_load_flow_tables sync");
-    pv_free_tables(ctx->tb);
+    if (int rc0 = pv_load_begin(ctx)) return rc0;
+    pv_free_tables(ctx, ctx->tb);
+    cudaStream_t ls = ctx->load_stream;
     pv_table_state &t = ctx->tb;
     const uint32_t T = tab[S];
     uint32_t *d_rule_offs = nullptr, *d_tab_offs = nullptr, *d_sizes = nullptr;
-    pv_rule *d_raw = nullptr;
     uint4 *d_rule_a = nullptr;
     uint2 *d_rule_b = nullptr;
     auto free_temps = [&]() {
-        pv_device_free(d_rule_offs);
-        pv_device_free(d_raw);
-        pv_device_free(d_tab_offs);
-        pv_device_free(d_rule_a);
-        pv_device_free(d_rule_b);
-        pv_device_free(d_sizes);
+        pv_pool_free(ctx, d_rule_offs);
+        pv_pool_free(ctx, d_tab_offs);
+        pv_pool_free(ctx, d_rule_a);
+        pv_pool_free(ctx, d_rule_b);
+        pv_pool_free(ctx, d_sizes);
     };
     int rc;
-    if ((rc = pv_device_alloc(ctx, (void **)&d_tab_offs, (S + 1) * 4, "table offsets")) ||
-        (rc = pv_device_alloc(ctx, (void **)&d_rule_a, (size_t)T * 16, "rules A")) ||
-        (rc = pv_device_alloc(ctx, (void **)&d_rule_b, (size_t)T * 8, "rules B")) ||
-        (rc = pv_device_alloc(ctx, (void **)&d_sizes, (size_t)S * 12 + 4, "index sizes")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_blob_offs, ((size_t)S + 1) * 8, "blob offsets")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_region, S, "regions")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_port_offs, (S + 1) * 4, "port offsets")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_port_peer, (size_t)P * 4, "port peers")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_host_switch, (size_t)H * 2, "host switch")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_host_port, (size_t)H * 2, "host port")) ||
-        (rc = pv_device_alloc(ctx, (void **)&t.d_host_ip, (size_t)H * 4, "host ip")) ||
-        (rc = pv_device_alloc(ctx, (void **)&d_rule_offs, (S + 1) * 4, "rule offsets")) ||
-        (rc = pv_device_alloc(ctx, (void **)&d_raw, (size_t)R * sizeof(pv_rule), "raw rules"))) {
+    if ((rc = pv_pool_alloc(ctx, (void **)&d_tab_offs, (S + 1) * 4, "table offsets")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&d_rule_a, (size_t)T * 16, "rules A")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&d_rule_b, (size_t)T * 8, "rules B")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&d_sizes, (size_t)S * 12 + 4, "index sizes")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_blob_offs, ((size_t)S + 1) * 8, "blob offsets")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_region, S, "regions")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_port_offs, (S + 1) * 4, "port offsets")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_port_peer, (size_t)P * 4, "port peers")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_host_switch, (size_t)H * 2, "host switch")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_host_port, (size_t)H * 2, "host port")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_host_ip, (size_t)H * 4, "host ip")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&d_rule_offs, (S + 1) * 4, "rule offsets")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_raw, (size_t)R * sizeof(pv_rule), "raw rules"))) {
         free_temps();
-        pv_free_tables(t);
+        pv_free_tables(ctx, t);
         return rc;
     }
     cudaError_t e = cudaSuccess;
-    e = e ? e : cudaMemcpy(d_tab_offs, tab.data(), (S + 1) * 4, cudaMemcpyHostToDevice);
-    e = e ? e : cudaMemcpy(t.d_region, switch_region, S, cudaMemcpyHostToDevice);
-    e = e ? e : cudaMemcpy(t.d_port_offs, port_offs, (S + 1) * 4, cudaMemcpyHostToDevice);
-    if (P) e = e ? e : cudaMemcpy(t.d_port_peer, port_peer, (size_t)P * 4, cudaMemcpyHostToDevice);
+    e = e ? e : cudaMemcpyAsync(d_tab_offs, tab.data(), (S + 1) * 4, cudaMemcpyHostToDevice, ls);
+    e = e ? e : cudaMemcpyAsync(t.d_region, switch_region, S, cudaMemcpyHostToDevice, ls);
+    e = e ? e : cudaMemcpyAsync(t.d_port_offs, port_offs, (S + 1) * 4, cudaMemcpyHostToDevice, ls);
+    if (P) e = e ? e : cudaMemcpyAsync(t.d_port_peer, port_peer, (size_t)P * 4, cudaMemcpyHostToDevice, ls);
     if (H) {
-        e = e ? e : cudaMemcpy(t.d_host_switch, host_switch, (size_t)H * 2, cudaMemcpyHostToDevice);
-        e = e ? e : cudaMemcpy(t.d_host_port, host_port, (size_t)H * 2, cudaMemcpyHostToDevice);
-        e = e ? e : cudaMemcpy(t.d_host_ip, host_ip, (size_t)H * 4, cudaMemcpyHostToDevice);
+        e = e ? e : cudaMemcpyAsync(t.d_host_switch, host_switch, (size_t)H * 2, cudaMemcpyHostToDevice, ls);
+        e = e ? e : cudaMemcpyAsync(t.d_host_port, host_port, (size_t)H * 2, cudaMemcpyHostToDevice, ls);
+        e = e ? e : cudaMemcpyAsync(t.d_host_ip, host_ip, (size_t)H * 4, cudaMemcpyHostToDevice, ls);
     }
-    e = e ? e : cudaMemcpy(d_rule_offs, rule_offs, (S + 1) * 4, cudaMemcpyHostToDevice);
-    if (R) e = e ? e : cudaMemcpy(d_raw, rules, (size_t)R * sizeof(pv_rule), cudaMemcpyHostToDevice);
+    e = e ? e : cudaMemcpyAsync(d_rule_offs, rule_offs, (S + 1) * 4, cudaMemcpyHostToDevice, ls);
+    if (R) e = e ? e : cudaMemcpyAsync(t.d_raw, rules, (size_t)R * sizeof(pv_rule), cudaMemcpyHostToDevice, ls);
     if (e == cudaSuccess) {
         uint32_t maxn = 0;
         for (uint32_t s = 0; s < S; ++s) maxn = std::max(maxn, rule_offs[s + 1] - rule_offs[s]);
         uint32_t npow = 1;
         while (npow < maxn) npow <<= 1;
         uint32_t *d_bad = d_sizes + (size_t)S * 3;   // lowest invalid rule index
-        e = cudaMemset(d_bad, 0xFF, 4);
+        e = cudaMemsetAsync(d_bad, 0xFF, 4, ls);
         if (e == cudaSuccess) {
-            compile_tables_kernel<<<S, 1024, npow * 4>>>(d_rule_offs, d_raw, t.d_port_offs, d_tab_offs, d_rule_a,
-                                                         d_rule_b, d_bad);
+            compile_tables_kernel<<<S, 1024, npow * 4, ls>>>(d_rule_offs, t.d_raw, t.d_port_offs, d_tab_offs,
+                                                             d_rule_a, d_rule_b, d_bad);
             e = cudaGetLastError();
         }
         if (e == cudaSuccess)
@@ -1262,7 +1260,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
             e = cudaFuncSetAttribute(index_build_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                      (int)kIndexSmem);
         if (e == cudaSuccess) {
-            index_build_kernel<false><<<S, 1024, kIndexSmem>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
+            index_build_kernel<false><<<S, 1024, kIndexSmem, ls>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
                                                                nullptr, nullptr);
             e = cudaGetLastError();
         }
@@ -1270,13 +1268,14 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     // blob layout from the index sizes (and the device-side rule validation)
     std::vector<uint32_t> sizes((size_t)S * 3 + 1);
     std::vector<uint64_t> boffs(S + 1, 0);
-    if (e == cudaSuccess) e = cudaMemcpy(sizes.data(), d_sizes, (size_t)S * 12 + 4, cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sizes.data(), d_sizes, (size_t)S * 12 + 4, cudaMemcpyDeviceToHost, ls);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(ls);
     if (e == cudaSuccess && sizes[(size_t)S * 3] != 0xFFFFFFFFu) {
         const uint32_t i = sizes[(size_t)S * 3];
         const uint32_t s = (uint32_t)(std::upper_bound(rule_offs, rule_offs + S + 1, i) - rule_offs) - 1;
         const pv_rule &r = rules[i];
         free_temps();
-        pv_free_tables(t);
+        pv_free_tables(ctx, t);
         return pv_fail(ctx, PV_EINVAL,
                        "rule %u (switch %u, %u ports): in_port %u, action %u, prefix lengths %u/%u, dport %u..%u "
                        "out of range",
@@ -1292,23 +1291,23 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
             max_blob = std::max(max_blob, L.total);
             max_linear = std::max(max_linear, L.boff);
         }
-        e = cudaMemcpy(t.d_blob_offs, boffs.data(), ((size_t)S + 1) * 8, cudaMemcpyHostToDevice);
+        e = cudaMemcpyAsync(t.d_blob_offs, boffs.data(), ((size_t)S + 1) * 8, cudaMemcpyHostToDevice, ls);
     }
     if (e == cudaSuccess) {
-        rc = pv_device_alloc(ctx, (void **)&t.d_blob, boffs[S], "flow table blobs");
+        rc = pv_pool_alloc(ctx, (void **)&t.d_blob, boffs[S], "flow table blobs");
         if (rc) {
             free_temps();
-            pv_free_tables(t);
+            pv_free_tables(ctx, t);
             return rc;
         }
-        index_build_kernel<true><<<S, 1024, kIndexSmem>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
+        index_build_kernel<true><<<S, 1024, kIndexSmem, ls>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
                                                           t.d_blob_offs, t.d_blob);
         e = cudaGetLastError();
-        if (e == cudaSuccess) e = cudaDeviceSynchronize();
+        if (e == cudaSuccess) e = cudaStreamSynchronize(ls);
     }
     free_temps();
     if (e != cudaSuccess) {
-        pv_free_tables(t);
+        pv_free_tables(ctx, t);
         return pv_cuda_fail(ctx, e, "pv_load_flow_tables");
     }
     t.num_switches = S;
@@ -1319,7 +1318,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     const size_t smem_cap = ctx->max_smem_optin - 1024;
     t.index_fits = max_blob <= smem_cap;
     if (max_linear > smem_cap) {
-        pv_free_tables(t);
+        pv_free_tables(ctx, t);
         return pv_fail(ctx, PV_EINVAL, "largest flow table needs %u bytes of shared memory", max_linear);
     }
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1358,22 +1357,23 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
                 links[cur[v]++] = u << 16 | (p - port_offs[u]) << 8 | ((uint32_t)peer & 0xFFu);
             }
         int rc2;
-        if ((rc2 = pv_device_alloc(ctx, (void **)&t.d_in_offs, (S + 1) * 4, "in-link offsets")) ||
-            (rc2 = pv_device_alloc(ctx, (void **)&t.d_in_links, links.size() * 4, "in-links"))) {
-            pv_free_tables(t);
+        if ((rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_offs, (S + 1) * 4, "in-link offsets")) ||
+            (rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_links, links.size() * 4, "in-links"))) {
+            pv_free_tables(ctx, t);
             return rc2;
         }
-        cudaError_t e2 = cudaMemcpy(t.d_in_offs, in_offs.data(), (S + 1) * 4, cudaMemcpyHostToDevice);
-        if (e2 == cudaSuccess) e2 = cudaMemcpy(t.d_in_links, links.data(), links.size() * 4, cudaMemcpyHostToDevice);
+        cudaError_t e2 = cudaMemcpyAsync(t.d_in_offs, in_offs.data(), (S + 1) * 4, cudaMemcpyHostToDevice, ls);
+        if (e2 == cudaSuccess)
+            e2 = cudaMemcpyAsync(t.d_in_links, links.data(), links.size() * 4, cudaMemcpyHostToDevice, ls);
+
         if (e2 != cudaSuccess) {
-            pv_free_tables(t);
+            pv_free_tables(ctx, t);
             return pv_cuda_fail(ctx, e2, "in-links upload");
         }
     }
     // host copy for rule installation
     pv_table_host &h = ctx->tbh;
     h.rule_offs.assign(rule_offs, rule_offs + S + 1);
-    h.rules.assign(rules, rules + R);
     h.region.assign(switch_region, switch_region + S);
     h.port_offs.assign(port_offs, port_offs + S + 1);
     h.port_peer.assign(port_peer, port_peer + P);
@@ -1381,7 +1381,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     h.host_port.assign(host_port, host_port + H);
     h.host_ip.assign(host_ip, host_ip + H);
     t.loaded = true;
-    return PV_OK;
+    return pv_load_end(ctx);
 }
 
 namespace {
@@ -1426,6 +1426,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     uint32_t *cursor = (uint32_t *)(base + o_cur);
     uint2 *descA = (uint2 *)(base + o_desc), *descB = (uint2 *)(base + o_desc + align256((size_t)max_desc * 8));
     cudaStream_t st = (cudaStream_t)stream;
+    pv_use_begin(ctx, st);
     PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
     const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, 0, nullptr};
@@ -1505,6 +1506,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
             walk_tail_kernel<false><<<hop_grid, 256, 0, st>>>(g, lst, dsc, hop_grid, tail_hop);
         pv_prof_stop(ctx, st, pr, 1);
     }
+    pv_mark_use(ctx, st);
     return pv_check_launch(ctx, "probe walk kernels");
 }
 
@@ -1555,24 +1557,26 @@ extern "C" int pv_load_path_policies(pv_ctx *ctx, uint32_t num_policies, const u
     for (size_t i = 0; i < sw.size(); ++i)
         if (sw[i] >= S)
             return pv_fail(ctx, PV_EINVAL, "pv_load_path_policies: switch id %u >= %u switches", (unsigned)sw[i], S);
+    if (int rc0 = pv_load_begin(ctx)) return rc0;
+    cudaStream_t ls = ctx->load_stream;
     pv_policy_state p;
     int rc;
-    if ((rc = pv_device_alloc(ctx, (void **)&p.d_hdr, (size_t)num_policies * 16, "policy headers")) ||
-        (rc = pv_device_alloc(ctx, (void **)&p.d_sw, std::max<size_t>(sw.size(), 1) * 2, "policy switches")) ||
-        (rc = pv_device_alloc(ctx, (void **)&p.d_concrete, num_policies, "policy flags"))) {
-        pv_free_policies(p);
+    if ((rc = pv_pool_alloc(ctx, (void **)&p.d_hdr, (size_t)num_policies * 16, "policy headers")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&p.d_sw, std::max<size_t>(sw.size(), 1) * 2, "policy switches")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&p.d_concrete, num_policies, "policy flags"))) {
+        pv_free_policies(ctx, p);
         return rc;
     }
-    cudaError_t e = cudaMemcpy(p.d_hdr, hdr.data(), (size_t)num_policies * 16, cudaMemcpyHostToDevice);
-    if (e == cudaSuccess && !sw.empty()) e = cudaMemcpy(p.d_sw, sw.data(), sw.size() * 2, cudaMemcpyHostToDevice);
-    if (e == cudaSuccess) e = cudaMemcpy(p.d_concrete, concrete, num_policies, cudaMemcpyHostToDevice);
+    cudaError_t e = cudaMemcpyAsync(p.d_hdr, hdr.data(), (size_t)num_policies * 16, cudaMemcpyHostToDevice, ls);
+    if (e == cudaSuccess && !sw.empty()) e = cudaMemcpyAsync(p.d_sw, sw.data(), sw.size() * 2, cudaMemcpyHostToDevice, ls);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(p.d_concrete, concrete, num_policies, cudaMemcpyHostToDevice, ls);
     if (e != cudaSuccess) {
-        pv_free_policies(p);
+        pv_free_policies(ctx, p);
         return pv_cuda_fail(ctx, e, "pv_load_path_policies");
     }
     p.loaded = true;
     p.num = num_policies;
-    pv_free_policies(ctx->pol);
+    pv_free_policies(ctx, ctx->pol);
     ctx->pol = p;
-    return PV_OK;
+    return pv_load_end(ctx);
 }

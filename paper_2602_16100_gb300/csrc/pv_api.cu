@@ -43,6 +43,36 @@ void pv_device_free(void *p) {
     if (p) cudaFree(p);
 }
 
+int pv_pool_alloc(pv_ctx *ctx, void **p, size_t bytes, const char *what) {
+    *p = nullptr;
+    if (bytes == 0) bytes = 16;
+    cudaError_t e = cudaMallocFromPoolAsync(p, bytes, ctx->pool, ctx->load_stream);
+    if (e != cudaSuccess) {
+        *p = nullptr;
+        return pv_cuda_fail(ctx, e, what);
+    }
+    return PV_OK;
+}
+
+void pv_pool_free(pv_ctx *ctx, void *p) {
+    if (p) cudaFreeAsync(p, ctx->load_stream);
+}
+
+int pv_load_begin(pv_ctx *ctx) {
+    PV_TRY_CUDA(ctx, cudaSetDevice(ctx->device), "cudaSetDevice");
+    PV_TRY_CUDA(ctx, cudaEventSynchronize(ctx->last_use), "waiting for the last use of the loaded state");
+    return PV_OK;
+}
+
+int pv_load_end(pv_ctx *ctx) {
+    PV_TRY_CUDA(ctx, cudaEventRecord(ctx->load_done, ctx->load_stream), "load");
+    return pv_check_launch(ctx, "load kernels");
+}
+
+void pv_use_begin(pv_ctx *ctx, cudaStream_t st) { cudaStreamWaitEvent(st, ctx->load_done, 0); }
+
+void pv_mark_use(pv_ctx *ctx, cudaStream_t st) { cudaEventRecord(ctx->last_use, st); }
+
 int pv_check_launch(pv_ctx *ctx, const char *what) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return pv_cuda_fail(ctx, e, what);
@@ -65,33 +95,34 @@ void *pv_scratch(pv_ctx *ctx, size_t bytes) {
     return p;
 }
 
-void pv_free_cluster(pv_cluster_state &c) {
-    pv_free_ptr(c.d_labels);
-    pv_free_ptr(c.d_inv);
-    pv_free_ptr(c.d_inv_rank);
-    pv_free_ptr(c.d_key_base);
-    pv_free_ptr(c.d_rows);
+void pv_free_cluster(pv_ctx *ctx, pv_cluster_state &c) {
+    pv_free_ptr(ctx, c.d_labels);
+    pv_free_ptr(ctx, c.d_inv);
+    pv_free_ptr(ctx, c.d_inv_rank);
+    pv_free_ptr(ctx, c.d_key_base);
+    pv_free_ptr(ctx, c.d_rows);
     c = pv_cluster_state();
 }
 
-void pv_free_policies(pv_policy_state &p) {
-    pv_free_ptr(p.d_hdr);
-    pv_free_ptr(p.d_sw);
-    pv_free_ptr(p.d_concrete);
+void pv_free_policies(pv_ctx *ctx, pv_policy_state &p) {
+    pv_free_ptr(ctx, p.d_hdr);
+    pv_free_ptr(ctx, p.d_sw);
+    pv_free_ptr(ctx, p.d_concrete);
     p = pv_policy_state();
 }
 
-void pv_free_tables(pv_table_state &t) {
-    pv_free_ptr(t.d_blob);
-    pv_free_ptr(t.d_blob_offs);
-    pv_free_ptr(t.d_region);
-    pv_free_ptr(t.d_port_offs);
-    pv_free_ptr(t.d_port_peer);
-    pv_free_ptr(t.d_host_switch);
-    pv_free_ptr(t.d_host_port);
-    pv_free_ptr(t.d_host_ip);
-    pv_free_ptr(t.d_in_offs);
-    pv_free_ptr(t.d_in_links);
+void pv_free_tables(pv_ctx *ctx, pv_table_state &t) {
+    pv_free_ptr(ctx, t.d_blob);
+    pv_free_ptr(ctx, t.d_blob_offs);
+    pv_free_ptr(ctx, t.d_region);
+    pv_free_ptr(ctx, t.d_port_offs);
+    pv_free_ptr(ctx, t.d_port_peer);
+    pv_free_ptr(ctx, t.d_host_switch);
+    pv_free_ptr(ctx, t.d_host_port);
+    pv_free_ptr(ctx, t.d_host_ip);
+    pv_free_ptr(ctx, t.d_in_offs);
+    pv_free_ptr(ctx, t.d_in_links);
+    pv_free_ptr(ctx, t.d_raw);
     t = pv_table_state();
 }
 
@@ -179,6 +210,21 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
     int smem = 0;
     cudaDeviceGetAttribute(&smem, cudaDevAttrMaxSharedMemoryPerBlockOptin, cuda_device);
     ctx->max_smem_optin = (size_t)smem;
+    cudaMemPoolProps props = {};
+    props.allocType = cudaMemAllocationTypePinned;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = cuda_device;
+    uint64_t keep = ~0ull;   // keep freed blocks for the next load
+    if (cudaStreamCreateWithFlags(&ctx->load_stream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaMemPoolCreate(&ctx->pool, &props) != cudaSuccess ||
+        cudaMemPoolSetAttribute(ctx->pool, cudaMemPoolAttrReleaseThreshold, &keep) != cudaSuccess ||
+        cudaEventCreateWithFlags(&ctx->last_use, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&ctx->load_done, cudaEventDisableTiming) != cudaSuccess) {
+        if (ctx->load_stream) cudaStreamDestroy(ctx->load_stream);
+        if (ctx->pool) cudaMemPoolDestroy(ctx->pool);
+        delete ctx;
+        return PV_ECUDA;
+    }
     if (pv_device_alloc(ctx, (void **)&ctx->d_status, sizeof(int32_t), "status word") != PV_OK ||
         cudaMemset(ctx->d_status, 0, sizeof(int32_t)) != cudaSuccess ||
         pv_device_alloc(ctx, (void **)&ctx->d_walk_live, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t),
@@ -188,6 +234,10 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
         pv_device_free(ctx->d_status);
         pv_device_free(ctx->d_walk_live);
         pv_device_free(ctx->d_reach_asym);
+        cudaEventDestroy(ctx->last_use);
+        cudaEventDestroy(ctx->load_done);
+        cudaStreamDestroy(ctx->load_stream);
+        cudaMemPoolDestroy(ctx->pool);
         delete ctx;
         return PV_ENOMEM;
     }
@@ -198,9 +248,14 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
 extern "C" void pv_destroy(pv_ctx *ctx) {
     if (!ctx) return;
     cudaDeviceSynchronize();
-    pv_free_cluster(ctx->cl);
-    pv_free_tables(ctx->tb);
-    pv_free_policies(ctx->pol);
+    pv_free_cluster(ctx, ctx->cl);
+    pv_free_tables(ctx, ctx->tb);
+    pv_free_policies(ctx, ctx->pol);
+    cudaStreamSynchronize(ctx->load_stream);
+    cudaEventDestroy(ctx->last_use);
+    cudaEventDestroy(ctx->load_done);
+    cudaStreamDestroy(ctx->load_stream);
+    cudaMemPoolDestroy(ctx->pool);
     for (cudaEvent_t e : ctx->prof.pool) cudaEventDestroy(e);
     pv_device_free(ctx->scratch);
     pv_device_free(ctx->d_status);

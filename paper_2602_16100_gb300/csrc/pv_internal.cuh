@@ -48,13 +48,14 @@ struct pv_table_state {
     // source port): u << 16 | p << 8 | q for port p of u cabled to port q
     uint32_t *d_in_offs = nullptr;    // [S + 1]
     uint32_t *d_in_links = nullptr;   // [links]
+    pv_rule *d_raw = nullptr;         // [rules] as loaded (for rule installation)
 };
 
-// Host copy of the loaded flow tables (the path scheduler's rule
-// installation merges into it and reloads).
+// Host copy of the loaded flow tables except the rules, which stay on the
+// device (the path scheduler's rule installation merges into them and
+// reloads).
 struct pv_table_host {
     std::vector<uint32_t> rule_offs, port_offs, host_ip;
-    std::vector<pv_rule> rules;
     std::vector<uint8_t> region;
     std::vector<int32_t> port_peer;
     std::vector<uint16_t> host_switch, host_port;
@@ -82,6 +83,13 @@ struct pv_prof_state {
 
 struct pv_ctx {
     int device = 0;
+    // Loads run on their own stream with memory from the context's pool, so
+    // they wait only for the evaluation work that may still read the state
+    // they replace (last_use), not for copies or kernels on other streams.
+    cudaStream_t load_stream = nullptr;
+    cudaMemPool_t pool = nullptr;
+    cudaEvent_t last_use = nullptr;   // recorded by every call that reads loaded state
+    cudaEvent_t load_done = nullptr;  // recorded at the end of every load (its device work)
     pv_prof_state prof;
     int num_sms = 0;
     size_t max_smem_optin = 0;
@@ -115,6 +123,18 @@ int pv_cuda_fail(pv_ctx *ctx, cudaError_t e, const char *what);
 void *pv_scratch(pv_ctx *ctx, size_t bytes);
 int pv_device_alloc(pv_ctx *ctx, void **p, size_t bytes, const char *what);
 void pv_device_free(void *p);
+// Loaded-state memory: stream-ordered on the context's load stream and pool.
+int pv_pool_alloc(pv_ctx *ctx, void **p, size_t bytes, const char *what);
+void pv_pool_free(pv_ctx *ctx, void *p);
+// A load begins by waiting for the last evaluation call that may read the
+// state it replaces; it ends by recording load_done on its stream and
+// returns without waiting for its device work.
+int pv_load_begin(pv_ctx *ctx);
+int pv_load_end(pv_ctx *ctx);
+// Evaluation calls order their stream after the last load (pv_use_begin)
+// and mark their use of the loaded state (pv_mark_use).
+void pv_use_begin(pv_ctx *ctx, cudaStream_t st);
+void pv_mark_use(pv_ctx *ctx, cudaStream_t st);
 int pv_check_launch(pv_ctx *ctx, const char *what);
 // Kernel-group timing: no-ops unless profiling is enabled.  Returns the pair
 // index to pass to pv_prof_stop (or -1).
@@ -143,13 +163,13 @@ __host__ __device__ __forceinline__ uint32_t pv_prefix_mask(uint32_t len) {
     return len == 0 ? 0u : (0xFFFFFFFFu << (32u - len));
 }
 
-// Allocation free-list helpers shared by the loaders.
+// Releases loaded-state memory in the load stream's order.
 template <typename T>
-inline void pv_free_ptr(T *&p) {
-    if (p) pv_device_free((void *)p);
+inline void pv_free_ptr(pv_ctx *ctx, T *&p) {
+    if (p) pv_pool_free(ctx, (void *)p);
     p = nullptr;
 }
 
-void pv_free_cluster(pv_cluster_state &c);
-void pv_free_tables(pv_table_state &t);
-void pv_free_policies(pv_policy_state &p);
+void pv_free_cluster(pv_ctx *ctx, pv_cluster_state &c);
+void pv_free_tables(pv_ctx *ctx, pv_table_state &t);
+void pv_free_policies(pv_ctx *ctx, pv_policy_state &p);

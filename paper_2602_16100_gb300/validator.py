@@ -32,6 +32,14 @@ def to_numpy(t: torch.Tensor, dtype, shape=None) -> np.ndarray:
     return a.reshape(shape) if shape is not None else a
 
 
+def flows_of(e: W.EndToEnd) -> np.ndarray:
+    """The compact flows {dst_ip, dport} of an end-to-end workload's probes."""
+    f = np.zeros(len(e.probes.probes), W.FLOW_DTYPE)
+    f["dst_ip"] = e.probes.probes["dst_ip"]
+    f["dport"] = e.probes.probes["dport"]
+    return f
+
+
 class Validator:
     """One GPU validator context (not thread-safe)."""
 
@@ -128,7 +136,7 @@ class Validator:
         B.pv_eval_selectors(self.ctx, I, dev["offs"], e2e_sizes["num_exprs"], dev["exprs"], None, dev["bits"], words,
                             dev["flags"], stream)
         B.pv_place_pods(self.ctx, I, pods, dev["bits"], words, dev["draws"], dev["assign"], stream)
-        B.pv_bind_probes(self.ctx, M, dev["probes"], ppg, pods, dev["assign"], stream)
+        B.pv_bind_flows(self.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], dev["probes"], stream)
         self._walk_and_verdict(dev, e2e_sizes, 0, I, stream)
         return dev
 
@@ -152,40 +160,48 @@ class Validator:
                                    dev["counts"][lo * 32:], stream)
 
     def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
-                                 chunks: int = 2) -> dict:
-        """The end-to-end pipeline on inputs in pinned HOST memory, the probe
-        upload overlapped with the pipeline: the intents are cut into
-        `chunks` ranges (independent units), range c's probes are copied on
-        `copy_stream` while range c-1 is verified on `stream`; the per-intent
-        verdicts and counters come back into ``host["pass"]`` and
-        ``host["counts"]`` on `stream` (not synchronised).
+                                 chunks: int = 2, loads=None) -> dict:
+        """The end-to-end pipeline on inputs in pinned HOST memory.
+        ``loads()``, if given, runs first (the table loads: their copies go
+        out ahead of the inputs, and their device work, which the evaluation
+        calls wait for on the device, overlaps the upload); every input
+        upload is then enqueued on `copy_stream`, the flows cut into `chunks`
+        intent ranges (independent units), and range c is verified on
+        `stream` as soon as its flows have arrived.  The per-intent verdicts and
+        counters come back into ``host["pass"]`` and ``host["counts"]`` on
+        `stream` (not synchronised).
 
-        ``host`` holds pinned byte tensors "offs", "exprs", "draws", "probes"
-        (inputs, as alloc_end_to_end lays them out) and "pass", "counts"
-        (outputs); ``dev`` the device buffers of alloc_end_to_end."""
+        ``host`` holds pinned byte tensors "offs", "exprs", "draws", "masks",
+        "flows" (inputs, as alloc_end_to_end lays them out: 8-byte flows, the
+        probe records are built on the device) and "pass", "counts" (outputs);
+        ``dev`` the device buffers of alloc_end_to_end."""
         I, pods, ppg = e2e_sizes["intents"], e2e_sizes["pods"], e2e_sizes["probes_per_intent"]
         words = W.words_per_row(self.num_nodes)
         ctx = self.ctx
-        # the previous step's kernels must be done with the device inputs
-        copy_stream.wait_stream(stream)
-        with torch.cuda.stream(copy_stream):
-            for k in ("offs", "exprs", "draws"):
-                n = host[k].numel()
-                dev[k][:n].copy_(host[k], non_blocking=True)
         chunks = max(1, min(int(chunks), max(1, I // 4)))
         # range edges on multiples of 4 intents (keeps every slice 16-byte aligned)
         edges = [0] + [((I * c) // chunks) & ~3 for c in range(1, chunks)] + [I]
         P = W.PROBE_DTYPE.itemsize
-        for lo, hi in zip(edges[:-1], edges[1:]):
-            if hi <= lo:
-                continue
+        F = W.FLOW_DTYPE.itemsize
+        ranges = [(lo, hi) for lo, hi in zip(edges[:-1], edges[1:]) if hi > lo]
+        if loads is not None:
+            loads()
+        # the previous step's kernels must be done with the device inputs
+        copy_stream.wait_stream(stream)
+        ready = []
+        with torch.cuda.stream(copy_stream):
+            for k in ("offs", "exprs", "draws", "masks"):
+                n = host[k].numel()
+                dev[k][:n].copy_(host[k], non_blocking=True)
+            for lo, hi in ranges:
+                dev["flows"][lo * ppg * F:hi * ppg * F].copy_(host["flows"][lo * ppg * F:hi * ppg * F],
+                                                               non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(copy_stream)
+                ready.append(ev)
+        for (lo, hi), ev in zip(ranges, ready):
             n = hi - lo
-            with torch.cuda.stream(copy_stream):
-                dev["probes"][lo * ppg * P:hi * ppg * P].copy_(host["probes"][lo * ppg * P:hi * ppg * P],
-                                                                non_blocking=True)
-                ready = torch.cuda.Event()
-                ready.record(copy_stream)
-            stream.wait_event(ready)
+            stream.wait_event(ev)
             bits = dev["bits"][lo * words * 4:]
             flags = dev["flags"][lo:]
             assign = dev["assign"][lo * pods * 4:]
@@ -193,7 +209,8 @@ class Validator:
             B.pv_eval_selectors(ctx, n, dev["offs"][lo * 4:], e2e_sizes["num_exprs"], dev["exprs"], None, bits,
                                 words, flags, stream)
             B.pv_place_pods(ctx, n, pods, bits, words, dev["draws"][lo * pods * 8:], assign, stream)
-            B.pv_bind_probes(ctx, n * ppg, probes, ppg, pods, assign, stream)
+            B.pv_bind_flows(ctx, n * ppg, dev["flows"][lo * ppg * F:], ppg, pods, assign, dev["masks"][lo * 4:],
+                            probes, stream)
             self._walk_and_verdict(dev, e2e_sizes, lo, hi, stream)
         with torch.cuda.stream(stream):
             host["pass"].copy_(dev["pass"][: host["pass"].numel()], non_blocking=True)
@@ -213,6 +230,8 @@ class Validator:
             "exprs": to_device(e.intents.exprs, d),
             "draws": to_device(e.place_draws.astype(np.uint64), d),
             "probes": to_device(e.probes.probes, d),
+            "flows": to_device(flows_of(e), d),
+            "masks": to_device(e.intent_mask.astype(np.uint32), d),
             "bits": empty_device(I * words * 4, d),
             "flags": empty_device(I, d),
             "assign": empty_device(I * pods * 4, d),

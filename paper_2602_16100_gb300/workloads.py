@@ -126,6 +126,8 @@ class Stream:
 # ----------------------------------------------------------------------------
 # containers
 # ----------------------------------------------------------------------------
+# compact flow of an intent: {dst_ip, dport, reserved}
+FLOW_DTYPE = np.dtype([("dst_ip", "<u4"), ("dport", "<u2"), ("reserved", "<u2")])
 # path request of the scheduler: {src_host, dst_host, allowed_mask, policy, reserved}
 PATH_REQ_DTYPE = np.dtype([("src_host", "<u2"), ("dst_host", "<u2"), ("allowed_mask", "<u4"), ("policy", "<u4"),
                            ("reserved", "<u4")])

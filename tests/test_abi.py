@@ -108,6 +108,7 @@ def test_path_request_layout_matches_header(tmp_path):
 #include <stdio.h>
 #include "pv.h"
 int main(void) {
+  printf("%zu %zu %zu\n", sizeof(pv_flow), offsetof(pv_flow, dport), offsetof(pv_flow, reserved));
   printf("%zu %zu %zu %zu %zu\n", sizeof(pv_path_req), offsetof(pv_path_req, dst_host),
          offsetof(pv_path_req, allowed_mask), offsetof(pv_path_req, policy), offsetof(pv_path_req, reserved));
   printf("%d %d %d %d %d\n", PV_PATH_OK, PV_PATH_NOSRC, PV_PATH_BLOCKED, PV_PATH_TOO_LONG, PV_PATH_REPEAT);
@@ -117,6 +118,9 @@ int main(void) {
     exe = tmp_path / "req"
     subprocess.check_call(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)])
     lines = subprocess.check_output([str(exe)], text=True).split("\n")
+    ff = W.FLOW_DTYPE.fields
+    assert [int(x) for x in lines[0].split()] == [W.FLOW_DTYPE.itemsize, ff["dport"][1], ff["reserved"][1]]
+    lines = lines[1:]
     f = W.PATH_REQ_DTYPE.fields
     assert [int(x) for x in lines[0].split()] == [W.PATH_REQ_DTYPE.itemsize, f["dst_host"][1], f["allowed_mask"][1],
                                                   f["policy"][1], f["reserved"][1]]

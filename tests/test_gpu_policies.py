@@ -10,7 +10,7 @@ import pytest
 import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
-from paper_2602_16100_gb300.validator import empty_device, to_device, to_numpy
+from paper_2602_16100_gb300.validator import flows_of, empty_device, to_device, to_numpy
 from gpu_util import sample
 from test_oracle_policies import _backup_switch_net, _policies
 from netbuild import probe
@@ -167,7 +167,8 @@ def test_constrained_pipeline_from_host(validator, chunks):
     dev, sizes = v.alloc_end_to_end(e, with_policies=True)
     I, pods, ppg = sizes["intents"], sizes["pods"], sizes["probes_per_intent"]
     host = {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
-            "draws": _pinned(e.place_draws.astype(np.uint64)), "probes": _pinned(e.probes.probes),
+            "draws": _pinned(e.place_draws.astype(np.uint64)), "masks": _pinned(e.intent_mask.astype(np.uint32)),
+            "flows": _pinned(flows_of(e)),
             "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
             "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
     stream = torch.cuda.current_stream()

@@ -9,7 +9,7 @@ import pytest
 import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
-from paper_2602_16100_gb300.validator import to_device, to_numpy
+from paper_2602_16100_gb300.validator import flows_of, to_device, to_numpy
 from gpu_util import sample
 
 pytestmark = pytest.mark.gpu
@@ -234,15 +234,18 @@ def test_end_to_end_pipelined_from_host(validator, chunks):
     validator.load_cluster(e.cluster)
     validator.load_network(e.network)
     dev, sizes = validator.alloc_end_to_end(e)
-    for k in ("offs", "exprs", "draws", "probes"):
+    for k in ("offs", "exprs", "draws", "masks", "flows", "probes"):
         dev[k].zero_()
     I = e.intents.num_pods
     host = {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
-            "draws": _pinned(e.place_draws.astype(np.uint64)), "probes": _pinned(e.probes.probes),
+            "draws": _pinned(e.place_draws.astype(np.uint64)), "masks": _pinned(e.intent_mask.astype(np.uint32)),
+            "flows": _pinned(flows_of(e)),
             "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
             "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
     stream = torch.cuda.current_stream()
-    validator.run_end_to_end_from_host(host, dev, sizes, stream, torch.cuda.Stream(), chunks)
+    # with 3 chunks the tables are reloaded while the inputs upload
+    loads = (lambda: (validator.load_cluster(e.cluster), validator.load_network(e.network))) if chunks == 3 else None
+    validator.run_end_to_end_from_host(host, dev, sizes, stream, torch.cuda.Stream(), chunks, loads)
     stream.synchronize()
     validator.sync()
     bits, flags, assign, probes = _oracle_e2e(e)
