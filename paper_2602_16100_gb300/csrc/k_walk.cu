@@ -188,13 +188,32 @@ constexpr uint32_t kBuckets = 256;          // dport >> kBucketShift
 constexpr uint32_t kBucketShift = 8;
 constexpr uint32_t kMinSegment = 4;         // shorter destination-only runs stay plain items
 constexpr uint32_t kMaxSegment = 4096;      // longer runs are split (in order: still exact)
-constexpr uint32_t kMaxSegments = PV_MAX_RULES / kMinSegment;
 constexpr uint32_t kSegItem = 0x8000u;
 constexpr uint32_t kWinFound = 0x80000000u;
-constexpr uint32_t kKeyCap = 2 * kMaxSegment + 8;   // boundaries of one segment (+ slack)
-constexpr uint32_t kSortCap = 16384;                // power of two >= 2 * kMaxSegment + 1
-constexpr size_t kIndexSmem = (size_t)kSortCap * 4 + (size_t)kKeyCap * 8 + PV_MAX_RULES * 2 + kMaxSegments * 8 +
-                              (size_t)kMaxSegment * 10;
+constexpr int kIndexThreads = 512;
+
+// Shared-memory layout of index_build_kernel, sized for the largest table
+// of a load (max_rules rules): sort keys (also the staged port ranges),
+// interval winners, scan positions, rule classes, segment bounds, and one
+// segment's prefixes and actions.
+struct IndexSmem {
+    uint32_t sort_cap, key_cap, rules_cap, segs_cap, seg_cap;
+    size_t bytes;
+    __host__ __device__ IndexSmem() : sort_cap(0), key_cap(0), rules_cap(0), segs_cap(0), seg_cap(0), bytes(0) {}
+    __host__ __device__ explicit IndexSmem(uint32_t max_rules) {
+        const uint32_t n = max_rules < 1 ? 1 : max_rules;
+        seg_cap = n < kMaxSegment ? n : kMaxSegment;
+        const uint32_t need = 2 * seg_cap + 1 > n ? 2 * seg_cap + 1 : n;
+        sort_cap = 1;
+        while (sort_cap < need) sort_cap <<= 1;
+        key_cap = 2 * seg_cap + 8 > kBuckets + 8 ? 2 * seg_cap + 8 : kBuckets + 8;
+        key_cap = (key_cap + 1) & ~1u;
+        rules_cap = (n + 7) & ~7u;
+        segs_cap = n / kMinSegment + n / kMaxSegment + 2;   // runs of >= 4, long runs split
+        bytes = (size_t)sort_cap * 4 + (size_t)key_cap * 8 + (size_t)rules_cap * 2 + (size_t)segs_cap * 8 +
+                (size_t)seg_cap * 10;
+    }
+};
 
 __host__ __device__ inline uint32_t up16(uint32_t b) { return (b + 15u) & ~15u; }
 
@@ -256,20 +275,20 @@ __device__ uint32_t block_exclusive_scan(uint32_t *v, uint32_t n, uint32_t *s_wa
 // Pass 1 (kFill = false) writes sizes[s] = {n_items, n_segs, n_bnd}; pass 2
 // writes the blob at blob_offs[s].  One 1024-thread block per switch.
 template <bool kFill>
-__global__ void __launch_bounds__(1024) index_build_kernel(const uint32_t *__restrict__ rule_offs,
+__global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32_t *__restrict__ rule_offs,
                                                            const uint32_t *__restrict__ tab_offs,
                                                            const uint4 *__restrict__ A, const uint2 *__restrict__ B,
                                                            uint32_t *__restrict__ sizes,
                                                            const uint64_t *__restrict__ blob_offs,
-                                                           uint8_t *__restrict__ blob) {
+                                                           uint8_t *__restrict__ blob, IndexSmem sm) {
     extern __shared__ __align__(16) uint32_t s_mem[];
-    uint32_t *s_keys = s_mem;                                      // [kSortCap]
-    uint32_t *s_win = s_keys + kSortCap;                           // [kKeyCap]
-    uint32_t *s_pos = s_win + kKeyCap;                             // [kKeyCap]
-    int16_t *s_cls = reinterpret_cast<int16_t *>(s_pos + kKeyCap);  // [PV_MAX_RULES]
-    uint32_t *s_segs = reinterpret_cast<uint32_t *>(s_cls + PV_MAX_RULES);  // [kMaxSegments][2]
-    uint2 *s_rules = reinterpret_cast<uint2 *>(s_segs + 2 * kMaxSegments);  // [kMaxSegment] {value, mask}
-    uint16_t *s_act = reinterpret_cast<uint16_t *>(s_rules + kMaxSegment);   // [kMaxSegment]
+    uint32_t *s_keys = s_mem;                                            // [sort_cap]
+    uint32_t *s_win = s_keys + sm.sort_cap;                              // [key_cap]
+    uint32_t *s_pos = s_win + sm.key_cap;                                // [key_cap]
+    int16_t *s_cls = reinterpret_cast<int16_t *>(s_pos + sm.key_cap);     // [rules_cap]
+    uint32_t *s_segs = reinterpret_cast<uint32_t *>(s_cls + sm.rules_cap);  // [segs_cap][2]
+    uint2 *s_rules = reinterpret_cast<uint2 *>(s_segs + 2 * sm.segs_cap);   // [seg_cap] {value, mask}
+    uint16_t *s_act = reinterpret_cast<uint16_t *>(s_rules + sm.seg_cap);    // [seg_cap]
     __shared__ uint32_t s_warp[33];
     __shared__ uint32_t s_nsegs;
     const uint32_t s = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
@@ -1241,9 +1260,10 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     }
     e = e ? e : cudaMemcpyAsync(d_rule_offs, rule_offs, (S + 1) * 4, cudaMemcpyHostToDevice, ls);
     if (R) e = e ? e : cudaMemcpyAsync(t.d_raw, rules, (size_t)R * sizeof(pv_rule), cudaMemcpyHostToDevice, ls);
+    uint32_t maxn = 0;
+    for (uint32_t s = 0; s < S; ++s) maxn = std::max(maxn, rule_offs[s + 1] - rule_offs[s]);
+    const IndexSmem ism(maxn);
     if (e == cudaSuccess) {
-        uint32_t maxn = 0;
-        for (uint32_t s = 0; s < S; ++s) maxn = std::max(maxn, rule_offs[s + 1] - rule_offs[s]);
         uint32_t npow = 1;
         while (npow < maxn) npow <<= 1;
         uint32_t *d_bad = d_sizes + (size_t)S * 3;   // lowest invalid rule index
@@ -1255,13 +1275,13 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         }
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(index_build_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)kIndexSmem);
+                                     (int)ism.bytes);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(index_build_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)kIndexSmem);
+                                     (int)ism.bytes);
         if (e == cudaSuccess) {
-            index_build_kernel<false><<<S, 1024, kIndexSmem, ls>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
-                                                               nullptr, nullptr);
+            index_build_kernel<false><<<S, kIndexThreads, ism.bytes, ls>>>(d_rule_offs, d_tab_offs, d_rule_a,
+                                                                           d_rule_b, d_sizes, nullptr, nullptr, ism);
             e = cudaGetLastError();
         }
     }
@@ -1300,8 +1320,8 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
             pv_free_tables(ctx, t);
             return rc;
         }
-        index_build_kernel<true><<<S, 1024, kIndexSmem, ls>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b, d_sizes,
-                                                          t.d_blob_offs, t.d_blob);
+        index_build_kernel<true><<<S, kIndexThreads, ism.bytes, ls>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b,
+                                                                      d_sizes, t.d_blob_offs, t.d_blob, ism);
         e = cudaGetLastError();
         if (e == cudaSuccess) e = cudaStreamSynchronize(ls);
     }

@@ -162,6 +162,46 @@ def _index_stress_network(seed, S=6, rules=700):
     return make_net(nports, links, hosts, st.ints(0, 3, S).astype(np.uint8), tables), host_ip
 
 
+def test_long_destination_runs_split_into_segments(validator):
+    """A destination-only run longer than the 4,096-rule segment limit is
+    indexed as consecutive segments (first-match order kept), behind a few
+    general rules; both kernels against the oracle."""
+    S, hosts_per = 3, 2
+    host_ip = np.array([ip(10, s, h, 1) for s in range(S) for h in range(hosts_per)], np.uint32)
+    links = [(s, hosts_per, (s + 1) % S, hosts_per + 1) for s in range(S)]
+    hosts = [(s, h, int(host_ip[s * hosts_per + h])) for s in range(S) for h in range(hosts_per)]
+    st = W.Stream(41, "long-runs")
+    tables = []
+    for s in range(S):
+        n_run = 4300
+        t = [rule(200, int(host_ip[(s + 1) % S * hosts_per]), 32, W.DROP, lo=80, hi=80)]     # general rule first
+        # /32 routes to many addresses (most unused) and the real hosts, then defaults
+        addrs = (st.u64(n_run) & np.uint64(0x0003FFFF)).astype(np.uint32) | np.uint32(ip(10, 0, 0, 0))
+        for i, a in enumerate(addrs):
+            t.append(rule(100, int(a), 32, int(st.ints(0, hosts_per + 1, 1)[0])))
+        for h in range(S * hosts_per):
+            own = h // hosts_per == s
+            t.append(rule(100, int(host_ip[h]), 32, h % hosts_per if own else hosts_per))
+        t.append(rule(50, 0, 0, hosts_per))
+        tables.append(t)
+    net = make_net([hosts_per + 2] * S, links, hosts, [0] * S, tables)
+    M = 6000
+    pr = np.zeros(M, W.PROBE_DTYPE)
+    src = st.ints(0, S * hosts_per - 1, M)
+    pr["src_host"], pr["src_ip"] = src, host_ip[src]
+    pick = st.floats(M)
+    pr["dst_ip"] = np.where(pick < 0.5, host_ip[st.ints(0, S * hosts_per - 1, M)],
+                            (st.u64(M) & np.uint64(0x0003FFFF)).astype(np.uint32) | np.uint32(ip(10, 0, 0, 0)))
+    pr["dport"] = np.where(st.floats(M) < 0.3, 80, st.ints(0, 65535, M))
+    pr["allowed_mask"] = 1
+    validator.load_network(net)
+    o = oracle.verify_probes(net, pr, 16)
+    kernels = [1, 2] if B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_INDEX_FITS) else [1]
+    for kernel in kernels:
+        assert _same(_gpu_walk(validator, net, pr, 16, kernel), o), kernel
+    assert len(np.unique(o["status"])) >= 3
+
+
 @pytest.mark.parametrize("seed", [1, 2, 3])
 def test_index_stress_tables(validator, seed):
     net, host_ip = _index_stress_network(seed)
