@@ -420,26 +420,47 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
         for (uint32_t x = t; x < nk; x += nt)
             if (x == 0 || s_win[x] != s_win[x - 1]) s_keys[s_pos[x]] = s_win[x];
         __syncthreads();
-        // the segment's prefixes and actions, staged so the winner scan below
-        // reads them as shared-memory broadcasts
+        // the segment's prefixes and actions, staged in shared memory
         for (uint32_t r = t; r < m; r += nt) {
             const uint4 ar = a[k0 + r];
             s_rules[r] = make_uint2(ar.z, ar.w);
             s_act[r] = (uint16_t)(b[k0 + r].y >> 16);
         }
         __syncthreads();
-        // winners of the K elementary intervals
-        for (uint32_t x = t; x < K; x += nt) {
-            const uint32_t d = s_keys[x];
-            uint32_t w = 0;
-            for (uint32_t r = 0; r < m; ++r) {
-                const uint2 ar = s_rules[r];
-                if (((d ^ ar.x) & ar.y) == 0) {
-                    w = kWinFound | s_act[r];
-                    break;
-                }
+        // winners of the K elementary intervals: the first rule (in
+        // first-match order) whose address range contains the interval.
+        // Each rule's range [v, v + size) starts and ends on boundaries, so
+        // it covers intervals ia .. ib - 1 exactly; the smallest rule index
+        // covering an interval wins.
+        for (uint32_t x = t; x < K; x += nt) s_win[x] = 0xFFFFFFFFu;
+        __syncthreads();
+        for (uint32_t r = t; r < m; r += nt) {
+            const uint2 ar = s_rules[r];
+            const uint64_t end1 = (uint64_t)ar.x + (uint64_t)(~ar.y) + 1ull;   // exclusive end
+            uint32_t lo = 0, hi = K;   // first x with s_keys[x] >= ar.x
+            while (lo < hi) {
+                const uint32_t mid = (lo + hi) >> 1;
+                if (s_keys[mid] < ar.x) lo = mid + 1;
+                else hi = mid;
             }
-            s_win[x] = w;
+            const uint32_t ia = lo;
+            uint32_t ib = K;
+            if (end1 < (1ull << 32)) {
+                lo = ia;
+                hi = K;
+                while (lo < hi) {
+                    const uint32_t mid = (lo + hi) >> 1;
+                    if (s_keys[mid] < (uint32_t)end1) lo = mid + 1;
+                    else hi = mid;
+                }
+                ib = lo;
+            }
+            for (uint32_t x = ia; x < ib; ++x) atomicMin(&s_win[x], r);
+        }
+        __syncthreads();
+        for (uint32_t x = t; x < K; x += nt) {
+            const uint32_t r = s_win[x];
+            s_win[x] = r == 0xFFFFFFFFu ? 0u : (kWinFound | s_act[r]);
         }
         __syncthreads();
         // merge adjacent intervals with the same winner
