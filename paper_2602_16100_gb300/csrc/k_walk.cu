@@ -550,11 +550,17 @@ __device__ __forceinline__ bool switch_listed(const uint16_t *list, uint32_t n, 
 // First visit of every probe: NOSRC for an absent source host, VIOLATION at
 // the attachment switch when its region is not permitted (or, with path
 // constraints, the switch is forbidden to the probe), otherwise listed.
+// It also counts the listed probes per switch into hist (the first hop's
+// histogram; per block in shared memory when S <= kSmemHistMax).
 template <bool kPolicy>
 __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
     uint32_t M, const pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
     const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
-    uint2 *__restrict__ list, uint2 *__restrict__ desc, PolicyArgs pa) {
+    uint2 *__restrict__ list, uint2 *__restrict__ desc, PolicyArgs pa, uint32_t S, uint32_t *__restrict__ hist) {
+    extern __shared__ uint32_t s_hist[];   // [S] when S <= kSmemHistMax
+    const bool smem_hist = S <= kSmemHistMax;
+    if (smem_hist)
+        for (uint32_t j = threadIdx.x; j < S; j += kGridThreads) s_hist[j] = 0;
     __shared__ uint32_t s_count;
     const uint32_t c0 = (uint32_t)(((uint64_t)M * blockIdx.x) / gridDim.x);
     const uint32_t c1 = (uint32_t)(((uint64_t)M * (blockIdx.x + 1)) / gridDim.x);
@@ -595,10 +601,16 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
             }
         }
         const uint32_t slot = warp_reserve(live, &s_count);
-        if (live) list[c0 + slot] = make_uint2(i, loc);
+        if (live) {
+            list[c0 + slot] = make_uint2(i, loc);
+            atomicAdd(smem_hist ? &s_hist[loc >> 8] : &hist[loc >> 8], 1u);
+        }
     }
     __syncthreads();
     if (threadIdx.x == 0) desc[blockIdx.x] = make_uint2(c0, s_count);
+    if (smem_hist)
+        for (uint32_t j = threadIdx.x; j < S; j += kGridThreads)
+            if (s_hist[j]) atomicAdd(&hist[j], s_hist[j]);
 }
 
 // A live-list entry is uint2 {probe id, loc}: loc bits 0..7 in_port, 8..23
@@ -745,6 +757,8 @@ struct HopArgs {
     uint32_t *ck;        // [M]: cycle-detection checkpoint location per probe
     uint32_t cycles;     // 1: finish probes caught in forwarding cycles early
     PolicyArgs pa;       // path constraints (used by the kPolicy kernels)
+    uint32_t *hist_next; // per-switch counts of the next hop's list (null: a separate pass counts)
+    uint32_t hist_off;   // byte offset of the block's count array in dynamic shared memory
 };
 
 // Linear first match: 32 consecutive rules per warp step.
@@ -946,6 +960,9 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
         mbar_init(&s_bar, 1);
         s_count = 0;
     }
+    uint32_t *s_hist = reinterpret_cast<uint32_t *>(s_raw + g.hist_off);   // [S] when g.hist_next
+    if (g.hist_next)
+        for (uint32_t j = threadIdx.x; j < g.S; j += kHopThreads) s_hist[j] = 0;
     __syncthreads();
     uint32_t parity = 0;
     uint32_t pos = r0;
@@ -1065,12 +1082,18 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 nloc = my_next | (nfin << 24);
             }
             const uint32_t slot = warp_reserve(live, &s_count);
-            if (live) g.next_list[r0 + slot] = make_uint2(e.x, nloc);
+            if (live) {
+                g.next_list[r0 + slot] = make_uint2(e.x, nloc);
+                if (g.hist_next) atomicAdd(&s_hist[entry_switch(nloc)], 1u);
+            }
         }
         pos = seg_end;
     }
     __syncthreads();
     if (threadIdx.x == 0) g.next_desc[blockIdx.x] = make_uint2(r0, s_count);
+    if (g.hist_next)
+        for (uint32_t j = threadIdx.x; j < g.S; j += kHopThreads)
+            if (s_hist[j]) atomicAdd(&g.hist_next[j], s_hist[j]);
 }
 
 // First match of one probe by one thread, reading the switch's blob from
@@ -1444,10 +1467,17 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     if (which == 2 && !t.index_fits)
         return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: the first-match index does not fit shared memory");
     const bool indexed = which == 2;
-    const size_t hop_smem = indexed ? t.max_blob_bytes : t.max_linear_bytes;
+    const size_t table_smem = indexed ? t.max_blob_bytes : t.max_linear_bytes;
+    // the next hop's per-switch counts ride in the hop kernel's shared memory
+    // after the staged table, when they fit
+    const size_t hist_off = (table_smem + 15) & ~(size_t)15;
+    const bool fuse_hist = S <= kSmemHistMax && hist_off + (size_t)S * 4 <= ctx->max_smem_optin - 1024;
+    const size_t hop_smem = fuse_hist ? hist_off + (size_t)S * 4 : table_smem;
     int hop_blocks_per_sm = 0;
     const void *hop_fn = indexed ? (pol ? (const void *)walk_hop_kernel<true, true> : (const void *)walk_hop_kernel<true, false>)
                                  : (pol ? (const void *)walk_hop_kernel<false, true> : (const void *)walk_hop_kernel<false, false>);
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(hop_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)hop_smem),
+                "walk_hop_kernel smem");
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, hop_fn, kHopThreads, hop_smem);
     const uint32_t hop_grid = (uint32_t)ctx->num_sms * (uint32_t)std::max(1, hop_blocks_per_sm);
     const uint32_t init_grid = (uint32_t)ctx->num_sms * 8;
@@ -1471,13 +1501,14 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
     const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, 0, nullptr};
+    const size_t init_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     if (pol)
-        walk_init_kernel<true><<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch,
-                                                                   t.d_host_port, t.d_region, d_out, listA, descA, *pa);
+        walk_init_kernel<true><<<init_grid, kGridThreads, init_smem, st>>>(
+            M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, *pa, S, hist);
     else
-        walk_init_kernel<false><<<init_grid, kGridThreads, 0, st>>>(M, d_probes, t.num_hosts, t.d_host_switch,
-                                                                    t.d_host_port, t.d_region, d_out, listA, descA,
-                                                                    no_policy);
+        walk_init_kernel<false><<<init_grid, kGridThreads, init_smem, st>>>(
+            M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, no_policy, S,
+            hist);
     pv_prof_stop(ctx, st, pr, 1);
     const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
@@ -1500,6 +1531,8 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.ck = (uint32_t *)(base + o_ck);
     g.cycles = cycles ? 1u : 0u;
     g.pa = pol ? *pa : no_policy;
+    g.hist_next = nullptr;
+    g.hist_off = (uint32_t)hist_off;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
     g.wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
@@ -1513,10 +1546,14 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         uint2 *dcur = (h & 1) ? descB : descA;
         uint2 *dnxt = (h & 1) ? descA : descB;
         pr = pv_prof_start(ctx, st, PV_K_WALK_REGROUP);
-        walk_hist_kernel<<<in_slices, kGridThreads, hist_smem, st>>>(cur, dcur, S, hist);
+        // hop 0's counts come from the init kernel, later hops' from the
+        // previous hop kernel when fused
+        const bool counted = h == 0 || fuse_hist;
+        if (!counted) walk_hist_kernel<<<in_slices, kGridThreads, hist_smem, st>>>(cur, dcur, S, hist);
         walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
         walk_scatter_kernel<<<in_slices, kGridThreads, scat_smem, st>>>(cur, dcur, S, cursor, sorted);
-        pv_prof_stop(ctx, st, pr, 3);
+        pv_prof_stop(ctx, st, pr, counted ? 2 : 3);
+        g.hist_next = (fuse_hist && h + 1 < tail_hop) ? hist : nullptr;
         g.sorted = sorted;
         g.hop = h;
         g.next_list = nxt;
