@@ -325,6 +325,11 @@ int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_
  *   flows: d_flows[k] = {dst_ip, dport} and the group's jurisdiction mask
  *   d_group_mask[g] give the whole probe record d_probes[k] (16-byte
  *   aligned), its source bound as above.
+ * pv_verify_flows: pv_bind_flows followed by pv_verify_probes in one call:
+ *   the walk's first kernel binds each flow, writes its record to d_probes
+ *   (read by the later hops) and starts its walk, so the records are not
+ *   read back; same results as the two calls.  pv_verify_flows_constrained
+ *   is the same with the path constraints of pv_verify_probes_constrained.
  * pv_aggregate_intents: d_pass[g] = 1 iff every pod of g has d_assign in
  *   row g, d_group_flags[g] has neither PV_F_UNKNOWN_VALUE nor
  *   PV_F_BAD_EXPR, and every probe of g is PV_COMPLIANT.
@@ -335,6 +340,14 @@ int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_
 int pv_bind_flows(pv_ctx *ctx, uint32_t num_probes, const pv_flow *d_flows, uint32_t probes_per_group,
                   uint32_t pods_per_group, const uint32_t *d_assign, const uint32_t *d_group_mask,
                   pv_probe *d_probes, pv_stream stream);
+int pv_verify_flows(pv_ctx *ctx, uint32_t num_probes, const pv_flow *d_flows, uint32_t probes_per_group,
+                    uint32_t pods_per_group, const uint32_t *d_assign, const uint32_t *d_group_mask, uint32_t hop_cap,
+                    pv_probe *d_probes, pv_result *d_out, pv_stream stream);
+int pv_verify_flows_constrained(pv_ctx *ctx, uint32_t num_probes, const pv_flow *d_flows, uint32_t probes_per_group,
+                                uint32_t pods_per_group, const uint32_t *d_assign, const uint32_t *d_group_mask,
+                                uint32_t hop_cap, const uint32_t *d_probe_policy, uint32_t probes_per_policy,
+                                uint32_t first_policy, pv_probe *d_probes, pv_result *d_out, uint32_t *d_waypoints,
+                                pv_stream stream);
 int pv_place_pods(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_group, const uint32_t *d_bits,
                   uint32_t words_per_row, const uint64_t *d_draws, uint32_t *d_assign, pv_stream stream);
 int pv_bind_probes(pv_ctx *ctx, uint32_t num_probes, pv_probe *d_probes, uint32_t probes_per_group,

@@ -551,12 +551,23 @@ __device__ __forceinline__ bool switch_listed(const uint16_t *list, uint32_t n, 
 // the attachment switch when its region is not permitted (or, with path
 // constraints, the switch is forbidden to the probe), otherwise listed.
 // It also counts the listed probes per switch into hist (the first hop's
-// histogram; per block in shared memory when S <= kSmemHistMax).
-template <bool kPolicy>
+// histogram; per block in shared memory when S <= kSmemHistMax).  With
+// kBind, the probe records are first built from compact flows and the
+// placement (the binding of pv_bind_flows) and written for the later hops.
+struct BindArgs {
+    const uint2 *flows;          // [M] {dst_ip, dport}
+    uint32_t ppg, pods;          // probes and pods per group
+    const uint32_t *assign;      // [groups * pods]
+    const uint32_t *group_mask;  // [groups]
+    const uint32_t *host_ip;     // [H]
+};
+
+template <bool kPolicy, bool kBind>
 __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
-    uint32_t M, const pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
+    uint32_t M, pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
     const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
-    uint2 *__restrict__ list, uint2 *__restrict__ desc, PolicyArgs pa, uint32_t S, uint32_t *__restrict__ hist) {
+    uint2 *__restrict__ list, uint2 *__restrict__ desc, PolicyArgs pa, uint32_t S, uint32_t *__restrict__ hist,
+    BindArgs ba) {
     extern __shared__ uint32_t s_hist[];   // [S] when S <= kSmemHistMax
     const bool smem_hist = S <= kSmemHistMax;
     if (smem_hist)
@@ -572,7 +583,18 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
         uint32_t loc = 0;
         if (i < c1) {
             // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
-            const uint4 pr = __ldg(reinterpret_cast<const uint4 *>(probes) + i);
+            uint4 pr;
+            if (kBind) {
+                const uint32_t grp = i / ba.ppg;
+                const uint32_t node = ba.assign[grp * ba.pods + (i - grp * ba.ppg) % ba.pods];
+                const uint2 f = __ldg(ba.flows + i);
+                const bool placed = node < H;
+                pr = make_uint4(placed ? ba.host_ip[node] : 0u, f.x,
+                                (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16, ba.group_mask[grp]);
+                reinterpret_cast<uint4 *>(probes)[i] = pr;
+            } else {
+                pr = __ldg(reinterpret_cast<const uint4 *>(probes) + i);
+            }
             const uint32_t h = pr.z >> 16;
             pv_result r;
             if (kPolicy) pa.hits[i] = 0;
@@ -1453,7 +1475,7 @@ namespace {
 // The walk of pv_verify_probes; with pa, under the path constraints of
 // pv_verify_probes_constrained.
 int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap, pv_result *d_out,
-                const PolicyArgs *pa, pv_stream stream) {
+                const PolicyArgs *pa, pv_stream stream, const BindArgs *ba = nullptr) {
     const pv_table_state &t = ctx->tb;
     const bool pol = pa != nullptr;
     if (!t.loaded) return pv_fail(ctx, PV_ESTATE, "pv_verify_probes: no flow tables loaded");
@@ -1502,13 +1524,26 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
     const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, 0, nullptr};
     const size_t init_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
-    if (pol)
-        walk_init_kernel<true><<<init_grid, kGridThreads, init_smem, st>>>(
-            M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, *pa, S, hist);
+    const BindArgs no_bind = {nullptr, 1, 1, nullptr, nullptr, nullptr};
+    pv_probe *probes_rw = const_cast<pv_probe *>(d_probes);   // written only when binding
+    const PolicyArgs &pa0 = pol ? *pa : no_policy;
+    const BindArgs &ba0 = ba ? *ba : no_bind;
+    if (pol && ba)
+        walk_init_kernel<true, true><<<init_grid, kGridThreads, init_smem, st>>>(
+            M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, pa0, S, hist,
+            ba0);
+    else if (pol)
+        walk_init_kernel<true, false><<<init_grid, kGridThreads, init_smem, st>>>(
+            M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, pa0, S, hist,
+            ba0);
+    else if (ba)
+        walk_init_kernel<false, true><<<init_grid, kGridThreads, init_smem, st>>>(
+            M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, pa0, S, hist,
+            ba0);
     else
-        walk_init_kernel<false><<<init_grid, kGridThreads, init_smem, st>>>(
-            M, d_probes, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, no_policy, S,
-            hist);
+        walk_init_kernel<false, false><<<init_grid, kGridThreads, init_smem, st>>>(
+            M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, pa0, S, hist,
+            ba0);
     pv_prof_stop(ctx, st, pr, 1);
     const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
@@ -1606,6 +1641,37 @@ extern "C" int pv_verify_probes_constrained(pv_ctx *ctx, uint32_t M, const pv_pr
     const PolicyArgs pa = {ctx->pol.d_hdr, ctx->pol.d_sw, ctx->pol.num, d_probe_policy, probes_per_policy,
                            first_policy, d_waypoints};
     return walk_probes(ctx, M, d_probes, hop_cap, d_out, &pa, stream);
+}
+
+extern "C" int pv_verify_flows(pv_ctx *ctx, uint32_t M, const pv_flow *d_flows, uint32_t ppg, uint32_t pods,
+                               const uint32_t *d_assign, const uint32_t *d_group_mask, uint32_t hop_cap,
+                               pv_probe *d_probes, pv_result *d_out, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (M && (!d_flows || !d_assign || !d_group_mask))
+        return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: NULL device pointer");
+    if (M && (ppg == 0 || pods == 0)) return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: group sizes must be > 0");
+    if (((uintptr_t)d_flows & 7) != 0) return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: d_flows must be 8-byte aligned");
+    const BindArgs ba = {reinterpret_cast<const uint2 *>(d_flows), ppg, pods, d_assign, d_group_mask, ctx->tb.d_host_ip};
+    return walk_probes(ctx, M, d_probes, hop_cap, d_out, nullptr, stream, &ba);
+}
+
+extern "C" int pv_verify_flows_constrained(pv_ctx *ctx, uint32_t M, const pv_flow *d_flows, uint32_t ppg,
+                                           uint32_t pods, const uint32_t *d_assign, const uint32_t *d_group_mask,
+                                           uint32_t hop_cap, const uint32_t *d_probe_policy,
+                                           uint32_t probes_per_policy, uint32_t first_policy, pv_probe *d_probes,
+                                           pv_result *d_out, uint32_t *d_waypoints, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (!ctx->pol.loaded) return pv_fail(ctx, PV_ESTATE, "pv_verify_flows_constrained: no path policies loaded");
+    if (M && (!d_flows || !d_assign || !d_group_mask || !d_waypoints))
+        return pv_fail(ctx, PV_EINVAL, "pv_verify_flows_constrained: NULL device pointer");
+    if (M && (ppg == 0 || pods == 0))
+        return pv_fail(ctx, PV_EINVAL, "pv_verify_flows_constrained: group sizes must be > 0");
+    if (((uintptr_t)d_flows & 7) != 0)
+        return pv_fail(ctx, PV_EINVAL, "pv_verify_flows_constrained: d_flows must be 8-byte aligned");
+    const BindArgs ba = {reinterpret_cast<const uint2 *>(d_flows), ppg, pods, d_assign, d_group_mask, ctx->tb.d_host_ip};
+    const PolicyArgs pa = {ctx->pol.d_hdr, ctx->pol.d_sw, ctx->pol.num, d_probe_policy, probes_per_policy,
+                           first_policy, d_waypoints};
+    return walk_probes(ctx, M, d_probes, hop_cap, d_out, &pa, stream, &ba);
 }
 
 extern "C" int pv_load_path_policies(pv_ctx *ctx, uint32_t num_policies, const uint32_t *forbid_offs,

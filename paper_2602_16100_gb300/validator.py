@@ -136,26 +136,28 @@ class Validator:
         B.pv_eval_selectors(self.ctx, I, dev["offs"], e2e_sizes["num_exprs"], dev["exprs"], None, dev["bits"], words,
                             dev["flags"], stream)
         B.pv_place_pods(self.ctx, I, pods, dev["bits"], words, dev["draws"], dev["assign"], stream)
-        B.pv_bind_flows(self.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], dev["probes"], stream)
         self._walk_and_verdict(dev, e2e_sizes, 0, I, stream)
         return dev
 
     def _walk_and_verdict(self, dev, e2e_sizes, lo, hi, stream):
-        """Walks and verdicts of intents [lo, hi); under the loaded path
-        policies (policy i for intent i) when ``dev`` holds a "hits" buffer."""
+        """Binding, walks and verdicts of intents [lo, hi) (one fused call
+        binds the flows and walks them); under the loaded path policies
+        (policy i for intent i) when ``dev`` holds a "hits" buffer."""
         ppg, pods, n = e2e_sizes["probes_per_intent"], e2e_sizes["pods"], hi - lo
         words = W.words_per_row(self.num_nodes)
-        P = W.PROBE_DTYPE.itemsize
+        P, F = W.PROBE_DTYPE.itemsize, W.FLOW_DTYPE.itemsize
         probes, results = dev["probes"][lo * ppg * P:], dev["results"][lo * ppg * 4:]
+        flows, masks = dev["flows"][lo * ppg * F:], dev["masks"][lo * 4:]
         bits, flags, assign = dev["bits"][lo * words * 4:], dev["flags"][lo:], dev["assign"][lo * pods * 4:]
+        cap = e2e_sizes["hop_cap"]
         if "hits" in dev:
             hits = dev["hits"][lo * ppg * 4:]
-            B.pv_verify_probes_constrained(self.ctx, n * ppg, probes, e2e_sizes["hop_cap"], None, ppg, results,
-                                           hits, stream, first_policy=lo)
+            B.pv_verify_flows_constrained(self.ctx, n * ppg, flows, ppg, pods, assign, masks, cap, None, ppg, lo,
+                                          probes, results, hits, stream)
             B.pv_aggregate_constrained(self.ctx, n, pods, bits, words, flags, assign, ppg, results, hits, None,
                                        dev["pass"][lo:], dev["counts"][lo * 32:], stream, first_policy=lo)
         else:
-            B.pv_verify_probes(self.ctx, n * ppg, probes, e2e_sizes["hop_cap"], results, stream)
+            B.pv_verify_flows(self.ctx, n * ppg, flows, ppg, pods, assign, masks, cap, probes, results, stream)
             B.pv_aggregate_intents(self.ctx, n, pods, bits, words, flags, assign, ppg, results, dev["pass"][lo:],
                                    dev["counts"][lo * 32:], stream)
 
@@ -205,12 +207,9 @@ class Validator:
             bits = dev["bits"][lo * words * 4:]
             flags = dev["flags"][lo:]
             assign = dev["assign"][lo * pods * 4:]
-            probes = dev["probes"][lo * ppg * P:]
             B.pv_eval_selectors(ctx, n, dev["offs"][lo * 4:], e2e_sizes["num_exprs"], dev["exprs"], None, bits,
                                 words, flags, stream)
             B.pv_place_pods(ctx, n, pods, bits, words, dev["draws"][lo * pods * 8:], assign, stream)
-            B.pv_bind_flows(ctx, n * ppg, dev["flows"][lo * ppg * F:], ppg, pods, assign, dev["masks"][lo * 4:],
-                            probes, stream)
             self._walk_and_verdict(dev, e2e_sizes, lo, hi, stream)
         with torch.cuda.stream(stream):
             host["pass"].copy_(dev["pass"][: host["pass"].numel()], non_blocking=True)

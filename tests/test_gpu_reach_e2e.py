@@ -9,7 +9,7 @@ import pytest
 import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
-from paper_2602_16100_gb300.validator import flows_of, to_device, to_numpy
+from paper_2602_16100_gb300.validator import empty_device, flows_of, to_device, to_numpy
 from gpu_util import sample
 
 pytestmark = pytest.mark.gpu
@@ -257,3 +257,31 @@ def test_end_to_end_pipelined_from_host(validator, chunks):
     assert (to_numpy(dev["results"], W.RESULT_DTYPE) == res).all()
     assert (host["pass"].numpy() == passed).all()
     assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
+
+
+def test_flow_binding_and_fused_walk(validator):
+    """pv_bind_flows builds the oracle's bound probe records from 8-byte
+    flows; pv_verify_flows (binding inside the walk's first kernel) gives the
+    records and results of pv_bind_flows followed by pv_verify_probes."""
+    e = W.end_to_end(seed=27, num_switches=64, num_intents=120, probes_per_intent=90, rules_per_switch=150)
+    v = validator
+    v.load_cluster(e.cluster)
+    v.load_network(e.network)
+    dev, sizes = v.alloc_end_to_end(e)
+    I, pods, ppg = sizes["intents"], sizes["pods"], sizes["probes_per_intent"]
+    words = W.words_per_row(e.cluster.num_nodes)
+    B.pv_eval_selectors(v.ctx, I, dev["offs"], sizes["num_exprs"], dev["exprs"], None, dev["bits"], words, dev["flags"])
+    B.pv_place_pods(v.ctx, I, pods, dev["bits"], words, dev["draws"], dev["assign"])
+    M = I * ppg
+    p1 = empty_device(M * 16, v.device)
+    B.pv_bind_flows(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], p1)
+    r1 = empty_device(M * 4, v.device)
+    B.pv_verify_probes(v.ctx, M, p1, sizes["hop_cap"], r1)
+    p2 = empty_device(M * 16, v.device)
+    r2 = empty_device(M * 4, v.device)
+    B.pv_verify_flows(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], sizes["hop_cap"], p2, r2)
+    v.sync()
+    _, _, assign, probes = _oracle_e2e(e)
+    assert (to_numpy(p1, W.PROBE_DTYPE) == probes).all() and (to_numpy(p2, W.PROBE_DTYPE) == probes).all()
+    res = oracle.verify_probes(e.network, probes, e.probes.hop_cap)
+    assert (to_numpy(r1, W.RESULT_DTYPE) == res).all() and (to_numpy(r2, W.RESULT_DTYPE) == res).all()
