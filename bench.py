@@ -126,6 +126,24 @@ def committed_traffic(kernel: str, src_hash: str):
         return None
 
 
+def walk_statistics(v):
+    """Counters of the last walk run with PV_OPT_WALK_STATS: first matches,
+    index rule tests and interval lookups (the work the indexed kernels do),
+    the depth a scan in first-match order reaches (the work a linear scan
+    does), and index/scan disagreements (0)."""
+    from paper_2602_16100_gb300 import binding as B
+    g = lambda k: int(B.pv_get_stat(v.ctx, k))
+    fm = g(B.PV_STAT_WALK_FIRST_MATCHES)
+    d = {"first_matches": fm, "index_rule_tests": g(B.PV_STAT_WALK_RULE_TESTS),
+         "interval_lookups": g(B.PV_STAT_WALK_INTERVAL_LOOKUPS), "scan_depth": g(B.PV_STAT_WALK_SCAN_DEPTH),
+         "index_mismatches": g(B.PV_STAT_WALK_INDEX_MISMATCHES)}
+    n = max(fm, 1)
+    d.update({"index_rule_tests_per_first_match": d["index_rule_tests"] / n,
+              "interval_lookups_per_first_match": d["interval_lookups"] / n,
+              "scan_rules_per_first_match": d["scan_depth"] / n})
+    return d
+
+
 def _walk_entries(v):
     """Probe-hop entries the hop kernel processed in the last walk (the sum
     over hops of the live probes; a probe judged at a hand-off is counted in
@@ -140,6 +158,7 @@ def _walk_entries(v):
 class EndToEndBench:
     name = "end-to-end cross-layer"
     unit = "probe-hop verifications/s"
+    walks = True
 
     def __init__(self, seed, intents=None, policies=False):
         self.e = W.end_to_end(seed=20260220 + seed, **({"num_intents": intents} if intents else {}))
@@ -501,6 +520,7 @@ class ScheduleBench:
 class FlowBench:
     name = "flow-verification"
     unit = "probe-hop verifications/s"
+    walks = True
 
     def __init__(self, seed):
         d = W.fat_tree(seed=20260218 + seed)
@@ -714,6 +734,15 @@ def run_ours(args):
     B.pv_profile_enable(v.ctx, False)
     prof_ms = p0.elapsed_time(p1)
     v.sync(stream)
+    # first-match statistics of one more step, run with the library's
+    # counting kernels (a diagnostic pass, outside both timed regions)
+    walk_stats = None
+    if getattr(wl, "walks", False):
+        B.pv_set_option(v.ctx, B.PV_OPT_WALK_STATS, 1)
+        wl.step(stream)
+        v.sync(stream)
+        B.pv_set_option(v.ctx, B.PV_OPT_WALK_STATS, 0)
+        walk_stats = walk_statistics(v)
     ms = SH.max_over_ranks(ms, dist, "cuda")
     secs_per_step = ms / 1e3 / args.steps
     value = units * world / secs_per_step
@@ -773,6 +802,11 @@ def run_ours(args):
                 "config": {**wl.config(), "parallelism": f"independent shards x{world}"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
                 "clocks": clk.result, "kernels": kernels, **wl.extra(secs_per_step)}
+        if walk_stats:
+            ws = dict(walk_stats)
+            ws["rule_tests_per_s"] = (ws["index_rule_tests"] + ws["interval_lookups"]) / secs_per_step
+            ws["scan_equivalent_rules_per_s"] = ws["scan_depth"] / secs_per_step
+            line["walk_statistics"] = ws
         print(json.dumps(line), flush=True)
     v.close()
     if dist:

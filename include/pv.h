@@ -465,6 +465,18 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  * PV_OPT_REACH_KERNEL: 0 = automatic (on a symmetric graph, rows are the
  *   connected components of the permitted subgraph; otherwise multi-source
  *   pull sweeps), 1 = sweeps always.  Both give the same rows.
+ * PV_OPT_WALK_STATS: 0 (default) or 1 = walks run counting versions of the
+ *   hop kernels (same results, slower: a diagnostic, not a timed path).
+ *   For every first match they also scan the switch's compiled rules in
+ *   first-match order and record, for the walk: first matches resolved,
+ *   index rule tests (candidate rules whose match was evaluated; the linear
+ *   kernel evaluates 32 per step), interval lookups (destination-only rule
+ *   runs answered by interval search), the scan depth (rules the ordered
+ *   scan tests before its first hit, every rule of the switch on a miss), and
+ *   index mismatches (first matches where the scan and the kernel disagree;
+ *   0 unless the index is wrong).  Read them with pv_get_stat
+ *   (PV_STAT_WALK_FIRST_MATCHES .. PV_STAT_WALK_INDEX_MISMATCHES; each read
+ *   synchronises with the device).
  * PV_OPT_TEST_STALL_STAGING: failure-injection switch for tests (0 or 1).
  *   When 1, each hop block's table-staging barrier expects 16 bytes more
  *   than its copy delivers, so its bounded wait runs out (after 50 ms rather
@@ -481,11 +493,13 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  * ------------------------------------------------------------------------- */
 enum {
     PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4,
-    PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6, PV_OPT_WALK_TAIL_HOP = 7
+    PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6, PV_OPT_WALK_TAIL_HOP = 7, PV_OPT_WALK_STATS = 8
 };
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,
-    PV_STAT_WALK_INDEX_BYTES = 4, PV_STAT_WALK_LIVE_TOTAL = 5, PV_STAT_REACH_COMPONENTS = 6
+    PV_STAT_WALK_INDEX_BYTES = 4, PV_STAT_WALK_LIVE_TOTAL = 5, PV_STAT_REACH_COMPONENTS = 6,
+    PV_STAT_WALK_FIRST_MATCHES = 7, PV_STAT_WALK_RULE_TESTS = 8, PV_STAT_WALK_INTERVAL_LOOKUPS = 9,
+    PV_STAT_WALK_SCAN_DEPTH = 10, PV_STAT_WALK_INDEX_MISMATCHES = 11
 };
 int pv_set_option(pv_ctx *ctx, int option, int64_t value);
 int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value);

@@ -290,10 +290,11 @@ extern "C" int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_r
     if (!d_rules || !d_rule_switch) return pv_fail(ctx, PV_EINVAL, "pv_install_path_rules: NULL device pointer");
     std::vector<pv_rule> add(num_slots);
     std::vector<uint16_t> sw(num_slots);
-    // the compiled rules come from an evaluation call: wait for it, then read
-    // them and the loaded rules on the load stream
+    // the compiled rules come from an evaluation call: the load stream waits
+    // for it, then reads them and the loaded rules
     if (int rc0 = pv_load_begin(ctx)) return rc0;
     cudaStream_t ls = ctx->load_stream;
+    PV_TRY_CUDA(ctx, cudaStreamWaitEvent(ls, ctx->last_use, 0), "pv_install_path_rules");
     const pv_table_host h = ctx->tbh;   // copy: the reload below replaces ctx->tbh
     const uint32_t S = (uint32_t)h.region.size();
     std::vector<pv_rule> base(h.rule_offs[S]);

@@ -447,9 +447,8 @@ extern "C" int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_key
         return pv_fail(ctx, PV_EINVAL, "pv_load_cluster: empty cluster or NULL labels");
     if (num_keys > kMaxKeys) return pv_fail(ctx, PV_EINVAL, "pv_load_cluster: num_keys > %u", kMaxKeys);
     if (int rc0 = pv_load_begin(ctx)) return rc0;
-    pv_free_cluster(ctx, ctx->cl);
     cudaStream_t ls = ctx->load_stream;
-    pv_cluster_state &c = ctx->cl;
+    pv_cluster_state c;   // the new state (the loaded one stays in use until it is complete)
     const size_t nl = (size_t)num_nodes * num_keys;
     int rc;
     if ((rc = pv_pool_alloc(ctx, (void **)&c.d_labels, nl * 2, "labels")) ||
@@ -467,8 +466,12 @@ extern "C" int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_key
     key_base_kernel<<<1, 1024, 0, ls>>>(num_keys, d_count, c.d_key_base);
     if ((rc = pv_check_launch(ctx, "inventory kernels"))) { pv_free_cluster(ctx, c); return rc; }
     uint32_t nvr = 0;
-    PV_TRY_CUDA(ctx, cudaMemcpyAsync(&nvr, c.d_key_base + num_keys, 4, cudaMemcpyDeviceToHost, ls), "value count");
-    PV_TRY_CUDA(ctx, cudaStreamSynchronize(ls), "value count");
+    cudaError_t e = cudaMemcpyAsync(&nvr, c.d_key_base + num_keys, 4, cudaMemcpyDeviceToHost, ls);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(ls);
+    if (e != cudaSuccess) {
+        pv_free_cluster(ctx, c);
+        return pv_cuda_fail(ctx, e, "value count");
+    }
     c.num_nodes = num_nodes;
     c.num_keys = num_keys;
     c.row_words = words_for(num_nodes);
@@ -476,7 +479,10 @@ extern "C" int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_key
     const uint64_t row_bytes = ((uint64_t)nvr + num_keys) * c.row_words * 4;
     if (row_bytes <= kRowBudgetBytes) {
         if (pv_pool_alloc(ctx, (void **)&c.d_rows, row_bytes, "value rows") == PV_OK) {
-            PV_TRY_CUDA(ctx, cudaMemsetAsync(c.d_rows, 0, row_bytes, ls), "value rows clear");
+            if ((e = cudaMemsetAsync(c.d_rows, 0, row_bytes, ls)) != cudaSuccess) {
+                pv_free_cluster(ctx, c);
+                return pv_cuda_fail(ctx, e, "value rows clear");
+            }
             build_rows_kernel<<<ctx->num_sms * 8, 256, 0, ls>>>(num_nodes, num_keys, c.d_labels, c.d_inv, c.d_inv_rank,
                                                           c.d_key_base, nvr, c.row_words, c.d_rows);
             if ((rc = pv_check_launch(ctx, "value rows"))) { pv_free_cluster(ctx, c); return rc; }
@@ -486,6 +492,10 @@ extern "C" int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_key
         }
     }
     c.loaded = true;
+    pv_retire_begin(ctx);
+    pv_free_cluster(ctx, ctx->cl);
+    pv_retire_end(ctx);
+    ctx->cl = c;
     return pv_load_end(ctx);
 }
 

@@ -781,12 +781,56 @@ struct HopArgs {
     PolicyArgs pa;       // path constraints (used by the kPolicy kernels)
     uint32_t *hist_next; // per-switch counts of the next hop's list (null: a separate pass counts)
     uint32_t hist_off;   // byte offset of the block's count array in dynamic shared memory
+    unsigned long long *stats;   // [PV_WALK_STATS] counters of the statistics kernels (kStats)
 };
+
+// Walk statistics (kStats kernels): first matches resolved, index rule
+// tests, interval lookups, the rules a scan in first-match order tests
+// before its first hit (all of the switch's rules on a miss), and first
+// matches where that scan and the kernel disagree.
+enum { kStFirstMatches = 0, kStRuleTests, kStLookups, kStLinearDepth, kStMismatch, kStCount };
+
+// First match by a plain scan of the compiled rules in first-match order
+// (smem or global): the statistics kernels' reference for depth and result.
+// *depth = position of the hit + 1, or the number of rules on a miss.
+__device__ __forceinline__ uint32_t scan_first_match(const uint4 *A, const uint2 *Bv, uint32_t npad, uint32_t src,
+                                                     uint32_t dst, uint32_t dport, uint32_t in_port,
+                                                     uint32_t *depth) {
+    for (uint32_t r = 0; r < npad; ++r) {
+        const uint2 b = Bv[r];
+        if (b.x == 1u) {   // padding (lo 1 > hi 0): the table has r rules
+            *depth = r;
+            return 0u;
+        }
+        const uint4 a = A[r];
+        const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ b.y) & ((b.y >> 8) & 0xFFu));
+        if (diff == 0 && dport >= (b.x & 0xFFFFu) && dport <= (b.x >> 16)) {
+            *depth = r + 1;
+            return kWinFound | (b.y >> 16);
+        }
+    }
+    *depth = npad;
+    return 0u;
+}
+
+// Adds one thread's statistics to the walk's counters (one atomic per warp
+// and counter).
+__device__ __forceinline__ void flush_stats(unsigned long long *stats, const uint32_t (&c)[kStCount]) {
+    const uint32_t lane = threadIdx.x & 31;
+#pragma unroll
+    for (int i = 0; i < kStCount; ++i) {
+        unsigned long long v = c[i];
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(PV_FULL_MASK, v, o);
+        if (lane == 0 && v) atomicAdd(stats + i, v);
+    }
+}
 
 // Linear first match: 32 consecutive rules per warp step.
 // Both first-match routines return kWinFound | action, or 0 for a table miss.
+template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_linear(const uint8_t *sm, uint32_t npad, uint32_t lane, uint32_t src,
-                                                       uint32_t dst, uint32_t dport, uint32_t in_port) {
+                                                       uint32_t dst, uint32_t dport, uint32_t in_port,
+                                                       uint32_t &tests) {
     const BlobLayout L(npad, 0, 0, 0);
     const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
     const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
@@ -796,6 +840,7 @@ __device__ __forceinline__ uint32_t first_match_linear(const uint8_t *sm, uint32
         const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ b.y) & ((b.y >> 8) & 0xFFu));
         const bool hit = diff == 0 && dport >= (b.x & 0xFFFFu) && dport <= (b.x >> 16);
         const uint32_t m = __ballot_sync(PV_FULL_MASK, hit);
+        if (kStats) tests += 32;
         if (m) return kWinFound | __shfl_sync(PV_FULL_MASK, b.y >> 16, __ffs(m) - 1);
     }
     return 0u;
@@ -820,8 +865,10 @@ __device__ __forceinline__ uint32_t segment_lookup(const uint32_t *bnd, const ui
 
 // Indexed first match: walk the dport bucket's candidate list in first-match
 // order, 32 items per step; segment items are answered by interval lookup.
+template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_indexed(const uint8_t *sm, const uint4 hdr, uint32_t lane,
-                                                        uint32_t src, uint32_t dst, uint32_t dport, uint32_t in_port) {
+                                                        uint32_t src, uint32_t dst, uint32_t dport, uint32_t in_port,
+                                                        uint32_t &tests, uint32_t &lookups) {
     const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
     const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
     const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
@@ -848,12 +895,14 @@ __device__ __forceinline__ uint32_t first_match_indexed(const uint8_t *sm, const
         }
         uint32_t G = __ballot_sync(PV_FULL_MASK, hit);
         uint32_t Sg = __ballot_sync(PV_FULL_MASK, is_seg);
+        if (kStats) tests += __popc(__ballot_sync(PV_FULL_MASK, valid && !is_seg));
         while (true) {
             const uint32_t pg = G ? (uint32_t)__ffs(G) - 1 : 32u;
             const uint32_t ps = Sg ? (uint32_t)__ffs(Sg) - 1 : 32u;
             if (ps < pg) {
                 const uint2 sd = segs[__shfl_sync(PV_FULL_MASK, it, ps) & 0x7FFFu];
                 const uint32_t w = segment_lookup(bnd + sd.x, win + sd.x, sd.y, dst, lane);
+                if (kStats) ++lookups;
                 if (w & kWinFound) return w;
                 Sg &= Sg - 1u;
             } else if (pg < 32u) {
@@ -871,8 +920,10 @@ __device__ __forceinline__ uint32_t first_match_indexed(const uint8_t *sm, const
 // Plain rules are tested until a hit or a segment token; the warp then
 // reconverges and the lanes parked on a segment token run their interval
 // binary searches together (a segment miss resumes the walk after the token).
+template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const BlobLayout &L, bool active,
-                                                     uint32_t src, uint32_t dst, uint32_t dport, uint32_t in_port) {
+                                                     uint32_t src, uint32_t dst, uint32_t dport, uint32_t in_port,
+                                                     uint32_t &tests, uint32_t &lookups) {
     const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
     const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
     const uint32_t *boff = reinterpret_cast<const uint32_t *>(sm + L.boff);
@@ -893,6 +944,7 @@ __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const Bl
                     seg = it & 0x7FFFu;
                     break;
                 }
+                if (kStats) ++tests;
                 const uint4 a = sA[it];
                 const uint2 bb = sB[it];
                 const uint32_t diff =
@@ -916,6 +968,7 @@ __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const Bl
                 len -= half;
             }
             const uint32_t w = win[sd.x + lo];
+            if (kStats) ++lookups;
             if (w & kWinFound) {
                 result = w;
                 done = true;
@@ -959,7 +1012,7 @@ __device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t hop, uint
     }
 }
 
-template <bool kIndexed, bool kPolicy>
+template <bool kIndexed, bool kPolicy, bool kStats>
 __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
     __shared__ uint64_t s_bar;
@@ -988,6 +1041,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     __syncthreads();
     uint32_t parity = 0;
     uint32_t pos = r0;
+    uint32_t stc[kStCount] = {};
     while (pos < r1) {
         // switch owning position pos: last s with seg[s] <= pos
         uint32_t lo = 0, hi = g.S;   // seg[lo] <= pos < seg[hi]
@@ -1036,7 +1090,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             const uint32_t fin = e.y >> 24;
             const bool fin_now = lane < cnt && fin != 0 && fin - 1 == g.hop;
             const uint32_t fin_lanes = __ballot_sync(PV_FULL_MASK, fin_now);
-            uint32_t my_status = fin_now ? (uint32_t)PV_LOOP : kAlive, my_next = 0;
+            uint32_t my_status = fin_now ? (uint32_t)PV_LOOP : kAlive, my_next = 0, my_fm = 0;
             // Every listed probe is permitted at s (checked when it was handed
             // on).  Lane-per-probe when every candidate list of the batch is short.
             bool lane_mode = false;
@@ -1051,7 +1105,9 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             }
             if (lane_mode) {
                 const bool act = lane < cnt && !fin_now;
-                const uint32_t fm = first_match_lane(s_raw, L, act, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu);
+                const uint32_t fm = first_match_lane<kStats>(s_raw, L, act, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu,
+                                                             stc[kStRuleTests], stc[kStLookups]);
+                my_fm = fm;
                 if (act) hop_outcome(g, g.hop, fm, pr.y, pr.w, pbase, nports, &my_status, &my_next);
             } else {
                 for (uint32_t j = 0; j < cnt; ++j) {
@@ -1061,15 +1117,31 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                     const uint32_t dst = __shfl_sync(PV_FULL_MASK, pr.y, j);
                     const uint32_t dport = __shfl_sync(PV_FULL_MASK, pr.z, j) & 0xFFFFu;
                     const uint32_t mask = __shfl_sync(PV_FULL_MASK, pr.w, j);
-                    const uint32_t fm = kIndexed ? first_match_indexed(s_raw, hdr, lane, src, dst, dport, in_port)
-                                                 : first_match_linear(s_raw, hdr.x, lane, src, dst, dport, in_port);
+                    uint32_t tests = 0, lookups = 0;
+                    const uint32_t fm =
+                        kIndexed ? first_match_indexed<kStats>(s_raw, hdr, lane, src, dst, dport, in_port, tests, lookups)
+                                 : first_match_linear<kStats>(s_raw, hdr.x, lane, src, dst, dport, in_port, tests);
                     uint32_t status, next;
                     hop_outcome(g, g.hop, fm, dst, mask, pbase, nports, &status, &next);
                     if (lane == j) {
                         my_status = status;
                         my_next = next;
+                        my_fm = fm;
+                        if (kStats) {
+                            stc[kStRuleTests] += tests;
+                            stc[kStLookups] += lookups;
+                        }
                     }
                 }
+            }
+            if (kStats && lane < cnt && !fin_now) {
+                uint32_t depth = 0;
+                const uint32_t ref = scan_first_match(reinterpret_cast<const uint4 *>(s_raw + L.a),
+                                                      reinterpret_cast<const uint2 *>(s_raw + L.b), hdr.x, pr.x,
+                                                      pr.y, pr.z & 0xFFFFu, e.y & 0xFFu, &depth);
+                ++stc[kStFirstMatches];
+                stc[kStLinearDepth] += depth;
+                stc[kStMismatch] += ref != my_fm ? 1u : 0u;
             }
             if (kPolicy && lane < cnt && !fin_now) {
                 const uint4 ph = policy_of(g.pa, e.x);
@@ -1111,6 +1183,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
         }
         pos = seg_end;
     }
+    if (kStats) flush_stats(g.stats, stc);
     __syncthreads();
     if (threadIdx.x == 0) g.next_desc[blockIdx.x] = make_uint2(r0, s_count);
     if (g.hist_next)
@@ -1121,9 +1194,10 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
 // First match of one probe by one thread, reading the switch's blob from
 // global memory (L2-resident tables): the per-lane walk of first_match_lane
 // without its warp phases.
+template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict__ blob, const BlobLayout &L,
                                                        uint32_t src, uint32_t dst, uint32_t dport,
-                                                       uint32_t in_port) {
+                                                       uint32_t in_port, uint32_t &tests, uint32_t &lookups) {
     const uint4 *A = reinterpret_cast<const uint4 *>(blob + L.a);
     const uint2 *Bv = reinterpret_cast<const uint2 *>(blob + L.b);
     const uint32_t *boff = reinterpret_cast<const uint32_t *>(blob + L.boff);
@@ -1144,9 +1218,11 @@ __device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict
                 len -= half;
             }
             const uint32_t w = __ldg(win + sd.x + lo);
+            if (kStats) ++lookups;
             if (w & kWinFound) return w;
             continue;
         }
+        if (kStats) ++tests;
         const uint4 a = __ldg(A + it);
         const uint2 bb = __ldg(Bv + it);
         const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
@@ -1162,11 +1238,12 @@ __device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict
 // regrouping them by switch every hop would cost more in launches than the
 // table staging saves.  Results, cycle finishing, path constraints and the
 // per-hop live counts are those of walk_hop_kernel.
-template <bool kPolicy>
+template <bool kPolicy, bool kStats>
 __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *__restrict__ list,
                                                         const uint2 *__restrict__ desc, uint32_t nslices,
                                                         uint32_t first_hop) {
     const uint32_t lane = threadIdx.x & 31;
+    uint32_t stc[kStCount] = {};
     for (uint32_t sl = blockIdx.x; sl < nslices; sl += gridDim.x) {
         const uint2 d = desc[sl];
         for (uint32_t base = d.x; base < d.x + d.y; base += blockDim.x) {
@@ -1194,7 +1271,17 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                 const uint8_t *blob = g.blob + g.blob_offs[s];
                 const uint4 hdr = __ldg(reinterpret_cast<const uint4 *>(blob));
                 const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
-                const uint32_t fm = first_match_thread(blob, L, pr.x, pr.y, pr.z & 0xFFFFu, in_port);
+                const uint32_t fm = first_match_thread<kStats>(blob, L, pr.x, pr.y, pr.z & 0xFFFFu, in_port,
+                                                               stc[kStRuleTests], stc[kStLookups]);
+                if (kStats) {
+                    uint32_t depth = 0;
+                    const uint32_t ref = scan_first_match(reinterpret_cast<const uint4 *>(blob + L.a),
+                                                          reinterpret_cast<const uint2 *>(blob + L.b), hdr.x, pr.x,
+                                                          pr.y, pr.z & 0xFFFFu, in_port, &depth);
+                    ++stc[kStFirstMatches];
+                    stc[kStLinearDepth] += depth;
+                    stc[kStMismatch] += ref != fm ? 1u : 0u;
+                }
                 const uint32_t pbase = g.port_offs[s], nports = g.port_offs[s + 1] - pbase;
                 uint32_t status, next;
                 hop_outcome(g, h, fm, pr.y, pr.w, pbase, nports, &status, &next);
@@ -1227,6 +1314,7 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
             }
         }
     }
+    if (kStats) flush_stats(g.stats, stc);
 }
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
@@ -1282,9 +1370,8 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
             return pv_fail(ctx, PV_EINVAL, "host %u attachment out of range", h);
 
     if (int rc0 = pv_load_begin(ctx)) return rc0;
-    pv_free_tables(ctx, ctx->tb);
     cudaStream_t ls = ctx->load_stream;
-    pv_table_state &t = ctx->tb;
+    pv_table_state t;   // the new tables (the loaded ones stay in use until these are complete)
     const uint32_t T = tab[S];
     uint32_t *d_rule_offs = nullptr, *d_tab_offs = nullptr, *d_sizes = nullptr;
     uint4 *d_rule_a = nullptr;
@@ -1326,6 +1413,48 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     }
     e = e ? e : cudaMemcpyAsync(d_rule_offs, rule_offs, (S + 1) * 4, cudaMemcpyHostToDevice, ls);
     if (R) e = e ? e : cudaMemcpyAsync(t.d_raw, rules, (size_t)R * sizeof(pv_rule), cudaMemcpyHostToDevice, ls);
+    if (e != cudaSuccess) {
+        free_temps();
+        pv_free_tables(ctx, t);
+        return pv_cuda_fail(ctx, e, "pv_load_flow_tables uploads");
+    }
+    // links into each switch, sorted by (source switch, source port); uploaded
+    // here, ahead of the index-size read-back, so no pageable copy (which
+    // waits for the stream) follows the index fill
+    {
+        std::vector<uint32_t> in_offs(S + 1, 0), links;
+        for (uint32_t u = 0; u < S; ++u)
+            for (uint32_t p = port_offs[u]; p < port_offs[u + 1]; ++p) {
+                const int32_t peer = port_peer[p];
+                if (peer >= 0 && !(peer & PV_PEER_HOST)) ++in_offs[((uint32_t)peer >> 8) + 1];
+            }
+        for (uint32_t v = 0; v < S; ++v) in_offs[v + 1] += in_offs[v];
+        links.resize(std::max<uint32_t>(in_offs[S], 1));
+        std::vector<uint32_t> cur(in_offs.begin(), in_offs.end() - 1);
+        for (uint32_t u = 0; u < S; ++u)   // ascending u, then p: each list ends up sorted
+            for (uint32_t p = port_offs[u]; p < port_offs[u + 1]; ++p) {
+                const int32_t peer = port_peer[p];
+                if (peer < 0 || (peer & PV_PEER_HOST)) continue;
+                const uint32_t v = (uint32_t)peer >> 8;
+                links[cur[v]++] = u << 16 | (p - port_offs[u]) << 8 | ((uint32_t)peer & 0xFFu);
+            }
+        int rc2;
+        if ((rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_offs, (S + 1) * 4, "in-link offsets")) ||
+            (rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_links, links.size() * 4, "in-links"))) {
+            free_temps();
+            pv_free_tables(ctx, t);
+            return rc2;
+        }
+        cudaError_t e2 = cudaMemcpyAsync(t.d_in_offs, in_offs.data(), (S + 1) * 4, cudaMemcpyHostToDevice, ls);
+        if (e2 == cudaSuccess)
+            e2 = cudaMemcpyAsync(t.d_in_links, links.data(), links.size() * 4, cudaMemcpyHostToDevice, ls);
+
+        if (e2 != cudaSuccess) {
+            free_temps();
+            pv_free_tables(ctx, t);
+            return pv_cuda_fail(ctx, e2, "in-links upload");
+        }
+    }
     uint32_t maxn = 0;
     for (uint32_t s = 0; s < S; ++s) maxn = std::max(maxn, rule_offs[s + 1] - rule_offs[s]);
     const IndexSmem ism(maxn);
@@ -1389,7 +1518,6 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         index_build_kernel<true><<<S, kIndexThreads, ism.bytes, ls>>>(d_rule_offs, d_tab_offs, d_rule_a, d_rule_b,
                                                                       d_sizes, t.d_blob_offs, t.d_blob, ism);
         e = cudaGetLastError();
-        if (e == cudaSuccess) e = cudaStreamSynchronize(ls);
     }
     free_temps();
     if (e != cudaSuccess) {
@@ -1407,56 +1535,9 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         pv_free_tables(ctx, t);
         return pv_fail(ctx, PV_EINVAL, "largest flow table needs %u bytes of shared memory", max_linear);
     }
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)max_linear),
-                "walk_hop_kernel smem");
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)max_linear),
-                "walk_hop_kernel smem");
-    if (t.index_fits) {
-        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<true, false>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_blob),
-                    "walk_hop_kernel smem");
-        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_hop_kernel<true, true>,
-                                              cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_blob),
-                    "walk_hop_kernel smem");
-    }
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           (int)(2 * kSmemHistMax * 4)),
                 "walk_scatter_kernel smem");
-    // links into each switch, sorted by (source switch, source port)
-    {
-        std::vector<uint32_t> in_offs(S + 1, 0), links;
-        for (uint32_t u = 0; u < S; ++u)
-            for (uint32_t p = port_offs[u]; p < port_offs[u + 1]; ++p) {
-                const int32_t peer = port_peer[p];
-                if (peer >= 0 && !(peer & PV_PEER_HOST)) ++in_offs[((uint32_t)peer >> 8) + 1];
-            }
-        for (uint32_t v = 0; v < S; ++v) in_offs[v + 1] += in_offs[v];
-        links.resize(std::max<uint32_t>(in_offs[S], 1));
-        std::vector<uint32_t> cur(in_offs.begin(), in_offs.end() - 1);
-        for (uint32_t u = 0; u < S; ++u)   // ascending u, then p: each list ends up sorted
-            for (uint32_t p = port_offs[u]; p < port_offs[u + 1]; ++p) {
-                const int32_t peer = port_peer[p];
-                if (peer < 0 || (peer & PV_PEER_HOST)) continue;
-                const uint32_t v = (uint32_t)peer >> 8;
-                links[cur[v]++] = u << 16 | (p - port_offs[u]) << 8 | ((uint32_t)peer & 0xFFu);
-            }
-        int rc2;
-        if ((rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_offs, (S + 1) * 4, "in-link offsets")) ||
-            (rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_links, links.size() * 4, "in-links"))) {
-            pv_free_tables(ctx, t);
-            return rc2;
-        }
-        cudaError_t e2 = cudaMemcpyAsync(t.d_in_offs, in_offs.data(), (S + 1) * 4, cudaMemcpyHostToDevice, ls);
-        if (e2 == cudaSuccess)
-            e2 = cudaMemcpyAsync(t.d_in_links, links.data(), links.size() * 4, cudaMemcpyHostToDevice, ls);
-
-        if (e2 != cudaSuccess) {
-            pv_free_tables(ctx, t);
-            return pv_cuda_fail(ctx, e2, "in-links upload");
-        }
-    }
     // host copy for rule installation
     pv_table_host &h = ctx->tbh;
     h.rule_offs.assign(rule_offs, rule_offs + S + 1);
@@ -1467,6 +1548,10 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     h.host_port.assign(host_port, host_port + H);
     h.host_ip.assign(host_ip, host_ip + H);
     t.loaded = true;
+    pv_retire_begin(ctx);
+    pv_free_tables(ctx, ctx->tb);
+    pv_retire_end(ctx);
+    ctx->tb = t;
     return pv_load_end(ctx);
 }
 
@@ -1474,6 +1559,18 @@ namespace {
 
 // The walk of pv_verify_probes; with pa, under the path constraints of
 // pv_verify_probes_constrained.
+using HopKernel = void (*)(HopArgs);
+using TailKernel = void (*)(HopArgs, const uint2 *, const uint2 *, uint32_t, uint32_t);
+
+HopKernel pick_hop_kernel(bool indexed, bool pol, bool stats) {
+    if (stats) {
+        if (indexed) return pol ? walk_hop_kernel<true, true, true> : walk_hop_kernel<true, false, true>;
+        return pol ? walk_hop_kernel<false, true, true> : walk_hop_kernel<false, false, true>;
+    }
+    if (indexed) return pol ? walk_hop_kernel<true, true, false> : walk_hop_kernel<true, false, false>;
+    return pol ? walk_hop_kernel<false, true, false> : walk_hop_kernel<false, false, false>;
+}
+
 int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap, pv_result *d_out,
                 const PolicyArgs *pa, pv_stream stream, const BindArgs *ba = nullptr) {
     const pv_table_state &t = ctx->tb;
@@ -1496,11 +1593,14 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     const bool fuse_hist = S <= kSmemHistMax && hist_off + (size_t)S * 4 <= ctx->max_smem_optin - 1024;
     const size_t hop_smem = fuse_hist ? hist_off + (size_t)S * 4 : table_smem;
     int hop_blocks_per_sm = 0;
-    const void *hop_fn = indexed ? (pol ? (const void *)walk_hop_kernel<true, true> : (const void *)walk_hop_kernel<true, false>)
-                                 : (pol ? (const void *)walk_hop_kernel<false, true> : (const void *)walk_hop_kernel<false, false>);
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(hop_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)hop_smem),
+    const bool stats = ctx->opt_walk_stats != 0;
+    const HopKernel hop_fn = pick_hop_kernel(indexed, pol, stats);
+    const TailKernel tail_fn = pol ? (stats ? walk_tail_kernel<true, true> : walk_tail_kernel<true, false>)
+                                   : (stats ? walk_tail_kernel<false, true> : walk_tail_kernel<false, false>);
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute((const void *)hop_fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)hop_smem),
                 "walk_hop_kernel smem");
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, hop_fn, kHopThreads, hop_smem);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, (const void *)hop_fn, kHopThreads, hop_smem);
     const uint32_t hop_grid = (uint32_t)ctx->num_sms * (uint32_t)std::max(1, hop_blocks_per_sm);
     const uint32_t init_grid = (uint32_t)ctx->num_sms * 8;
     const uint32_t max_desc = std::max(hop_grid, init_grid);
@@ -1521,6 +1621,9 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     cudaStream_t st = (cudaStream_t)stream;
     pv_use_begin(ctx, st);
     PV_TRY_CUDA(ctx, cudaMemsetAsync(hist, 0, (size_t)S * 4, st), "hist clear");
+    if (stats)
+        PV_TRY_CUDA(ctx, cudaMemsetAsync(ctx->d_walk_stats, 0, PV_WALK_STATS * sizeof(unsigned long long), st),
+                    "walk statistics clear");
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
     const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, 0, nullptr};
     const size_t init_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
@@ -1568,6 +1671,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.pa = pol ? *pa : no_policy;
     g.hist_next = nullptr;
     g.hist_off = (uint32_t)hist_off;
+    g.stats = ctx->d_walk_stats;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
     g.wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
@@ -1594,14 +1698,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         g.next_list = nxt;
         g.next_desc = dnxt;
         pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
-        if (indexed && pol)
-            walk_hop_kernel<true, true><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
-        else if (indexed)
-            walk_hop_kernel<true, false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
-        else if (pol)
-            walk_hop_kernel<false, true><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
-        else
-            walk_hop_kernel<false, false><<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+        hop_fn<<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         pv_prof_stop(ctx, st, pr, 1);
         in_slices = hop_grid;
     }
@@ -1613,10 +1710,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
                     "tail live counts");
         g.hop = tail_hop;
         pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
-        if (pol)
-            walk_tail_kernel<true><<<hop_grid, 256, 0, st>>>(g, lst, dsc, hop_grid, tail_hop);
-        else
-            walk_tail_kernel<false><<<hop_grid, 256, 0, st>>>(g, lst, dsc, hop_grid, tail_hop);
+        tail_fn<<<hop_grid, 256, 0, st>>>(g, lst, dsc, hop_grid, tail_hop);
         pv_prof_stop(ctx, st, pr, 1);
     }
     pv_mark_use(ctx, st);
@@ -1720,7 +1814,9 @@ extern "C" int pv_load_path_policies(pv_ctx *ctx, uint32_t num_policies, const u
     }
     p.loaded = true;
     p.num = num_policies;
+    pv_retire_begin(ctx);
     pv_free_policies(ctx, ctx->pol);
+    pv_retire_end(ctx);
     ctx->pol = p;
     return pv_load_end(ctx);
 }

@@ -55,14 +55,22 @@ int pv_pool_alloc(pv_ctx *ctx, void **p, size_t bytes, const char *what) {
 }
 
 void pv_pool_free(pv_ctx *ctx, void *p) {
-    if (p) cudaFreeAsync(p, ctx->load_stream);
+    if (p) cudaFreeAsync(p, ctx->retiring ? ctx->retire_stream : ctx->load_stream);
 }
 
 int pv_load_begin(pv_ctx *ctx) {
     PV_TRY_CUDA(ctx, cudaSetDevice(ctx->device), "cudaSetDevice");
-    PV_TRY_CUDA(ctx, cudaEventSynchronize(ctx->last_use), "waiting for the last use of the loaded state");
     return PV_OK;
 }
+
+void pv_retire_begin(pv_ctx *ctx) {
+    cudaEventRecord(ctx->retire_from, ctx->load_stream);
+    cudaStreamWaitEvent(ctx->retire_stream, ctx->retire_from, 0);
+    cudaStreamWaitEvent(ctx->retire_stream, ctx->last_use, 0);
+    ctx->retiring = true;
+}
+
+void pv_retire_end(pv_ctx *ctx) { ctx->retiring = false; }
 
 int pv_load_end(pv_ctx *ctx) {
     PV_TRY_CUDA(ctx, cudaEventRecord(ctx->load_done, ctx->load_stream), "load");
@@ -215,12 +223,21 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
     props.location.type = cudaMemLocationTypeDevice;
     props.location.id = cuda_device;
     uint64_t keep = ~0ull;   // keep freed blocks for the next load
+    int no_reuse_deps = 0;
     if (cudaStreamCreateWithFlags(&ctx->load_stream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&ctx->retire_stream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&ctx->retire_from, cudaEventDisableTiming) != cudaSuccess ||
         cudaMemPoolCreate(&ctx->pool, &props) != cudaSuccess ||
         cudaMemPoolSetAttribute(ctx->pool, cudaMemPoolAttrReleaseThreshold, &keep) != cudaSuccess ||
+        // no reuse that would make the load stream wait for the retire stream
+        // (and so for evaluation work): blocks freed there are reused once done
+        cudaMemPoolSetAttribute(ctx->pool, cudaMemPoolReuseAllowInternalDependencies, &no_reuse_deps) !=
+            cudaSuccess ||
         cudaEventCreateWithFlags(&ctx->last_use, cudaEventDisableTiming) != cudaSuccess ||
         cudaEventCreateWithFlags(&ctx->load_done, cudaEventDisableTiming) != cudaSuccess) {
         if (ctx->load_stream) cudaStreamDestroy(ctx->load_stream);
+        if (ctx->retire_stream) cudaStreamDestroy(ctx->retire_stream);
+        if (ctx->retire_from) cudaEventDestroy(ctx->retire_from);
         if (ctx->pool) cudaMemPoolDestroy(ctx->pool);
         delete ctx;
         return PV_ECUDA;
@@ -230,13 +247,19 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
         pv_device_alloc(ctx, (void **)&ctx->d_walk_live, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t),
                         "walk statistics") != PV_OK ||
         cudaMemset(ctx->d_walk_live, 0, (PV_MAX_HOP_CAP + 1) * sizeof(uint32_t)) != cudaSuccess ||
-        pv_device_alloc(ctx, (void **)&ctx->d_reach_asym, sizeof(uint32_t), "reach symmetry flag") != PV_OK) {
+        pv_device_alloc(ctx, (void **)&ctx->d_reach_asym, sizeof(uint32_t), "reach symmetry flag") != PV_OK ||
+        pv_device_alloc(ctx, (void **)&ctx->d_walk_stats, PV_WALK_STATS * sizeof(unsigned long long),
+                        "walk statistics counters") != PV_OK ||
+        cudaMemset(ctx->d_walk_stats, 0, PV_WALK_STATS * sizeof(unsigned long long)) != cudaSuccess) {
         pv_device_free(ctx->d_status);
         pv_device_free(ctx->d_walk_live);
+        pv_device_free(ctx->d_walk_stats);
         pv_device_free(ctx->d_reach_asym);
         cudaEventDestroy(ctx->last_use);
         cudaEventDestroy(ctx->load_done);
+        cudaEventDestroy(ctx->retire_from);
         cudaStreamDestroy(ctx->load_stream);
+        cudaStreamDestroy(ctx->retire_stream);
         cudaMemPoolDestroy(ctx->pool);
         delete ctx;
         return PV_ENOMEM;
@@ -252,14 +275,18 @@ extern "C" void pv_destroy(pv_ctx *ctx) {
     pv_free_tables(ctx, ctx->tb);
     pv_free_policies(ctx, ctx->pol);
     cudaStreamSynchronize(ctx->load_stream);
+    cudaStreamSynchronize(ctx->retire_stream);
     cudaEventDestroy(ctx->last_use);
     cudaEventDestroy(ctx->load_done);
+    cudaEventDestroy(ctx->retire_from);
     cudaStreamDestroy(ctx->load_stream);
+    cudaStreamDestroy(ctx->retire_stream);
     cudaMemPoolDestroy(ctx->pool);
     for (cudaEvent_t e : ctx->prof.pool) cudaEventDestroy(e);
     pv_device_free(ctx->scratch);
     pv_device_free(ctx->d_status);
     pv_device_free(ctx->d_walk_live);
+    pv_device_free(ctx->d_walk_stats);
     pv_device_free(ctx->d_reach_asym);
     delete ctx;
 }
@@ -313,6 +340,10 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "reach kernel must be 0 or 1");
         ctx->opt_reach = (int)value;
         return PV_OK;
+    case PV_OPT_WALK_STATS:
+        if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "walk statistics switch must be 0 or 1");
+        ctx->opt_walk_stats = (int)value;
+        return PV_OK;
     default:
         return pv_fail(ctx, PV_EINVAL, "unknown option %d", option);
     }
@@ -342,6 +373,16 @@ extern "C" int pv_get_stat(const pv_ctx *ctx, int stat, int64_t *value) {
             cudaMemcpy(&asym, ctx->d_reach_asym, sizeof asym, cudaMemcpyDeviceToHost) != cudaSuccess)
             return PV_ECUDA;
         *value = (ctx->last_reach_comp && asym == 0) ? 1 : 0;
+        return PV_OK;
+    }
+    case PV_STAT_WALK_FIRST_MATCHES:
+    case PV_STAT_WALK_RULE_TESTS:
+    case PV_STAT_WALK_INTERVAL_LOOKUPS:
+    case PV_STAT_WALK_SCAN_DEPTH:
+    case PV_STAT_WALK_INDEX_MISMATCHES: {
+        unsigned long long c[PV_WALK_STATS];
+        if (cudaMemcpy(c, ctx->d_walk_stats, sizeof c, cudaMemcpyDeviceToHost) != cudaSuccess) return PV_ECUDA;
+        *value = (int64_t)c[stat - PV_STAT_WALK_FIRST_MATCHES];
         return PV_OK;
     }
     default: return PV_EINVAL;

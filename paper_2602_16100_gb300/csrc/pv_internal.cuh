@@ -10,6 +10,7 @@
 #include "pv.h"
 
 #define PV_FULL_MASK 0xFFFFFFFFu
+#define PV_WALK_STATS 8   // walk statistics counters (5 used)
 
 // -----------------------------------------------------------------------------
 // context
@@ -87,6 +88,13 @@ struct pv_ctx {
     // they wait only for the evaluation work that may still read the state
     // they replace (last_use), not for copies or kernels on other streams.
     cudaStream_t load_stream = nullptr;
+    // The state a load replaces is freed on the retire stream, after the last
+    // evaluation call that may read it (last_use) and the load's own work
+    // before the replacement (retire_from); the load stream never waits for
+    // evaluation work.
+    cudaStream_t retire_stream = nullptr;
+    cudaEvent_t retire_from = nullptr;
+    bool retiring = false;            // pv_pool_free frees on the retire stream
     cudaMemPool_t pool = nullptr;
     cudaEvent_t last_use = nullptr;   // recorded by every call that reads loaded state
     cudaEvent_t load_done = nullptr;  // recorded at the end of every load (its device work)
@@ -98,7 +106,9 @@ struct pv_ctx {
     int opt_selector = 0, opt_walk = 0;
     int opt_walk_lane_max = 96;
     int opt_walk_cycles = 0;
-    int opt_walk_tail_hop = 8;        // hops from here on run in one tail launch (0: never)          // 0: finish probes in forwarding cycles early, 1: walk to the cap
+    int opt_walk_tail_hop = 8;        // hops from here on run in one tail launch (0: never)
+    int opt_walk_stats = 0;           // 1: walks run the statistics kernels
+    unsigned long long *d_walk_stats = nullptr;   // [PV_WALK_STATS] counters of the last statistics walk
     int opt_test_stall_staging = 0;   // failure test: staging waits expect bytes that never come
     uint32_t *d_walk_live = nullptr;  // [PV_MAX_HOP_CAP + 1] live probes per hop of the last walk
     uint32_t last_walk_cap = 0;       // hop cap of the last walk
@@ -126,10 +136,17 @@ void pv_device_free(void *p);
 // Loaded-state memory: stream-ordered on the context's load stream and pool.
 int pv_pool_alloc(pv_ctx *ctx, void **p, size_t bytes, const char *what);
 void pv_pool_free(pv_ctx *ctx, void *p);
-// A load begins by waiting for the last evaluation call that may read the
-// state it replaces; it ends by recording load_done on its stream and
-// returns without waiting for its device work.
+// A load builds its new state in fresh memory on the load stream, without
+// waiting for the evaluation calls still reading the state it replaces.
+// Between pv_retire_begin and pv_retire_end, pv_pool_free frees on the
+// retire stream, which first waits (on the device) for the last of those
+// calls and for the load stream's work so far.  pv_load_end records
+// load_done on the load stream (the new state is complete) and returns
+// without waiting for the load's device work.  A load that fails leaves
+// the previous state loaded.
 int pv_load_begin(pv_ctx *ctx);
+void pv_retire_begin(pv_ctx *ctx);
+void pv_retire_end(pv_ctx *ctx);
 int pv_load_end(pv_ctx *ctx);
 // Evaluation calls order their stream after the last load (pv_use_begin)
 // and mark their use of the loaded state (pv_mark_use).

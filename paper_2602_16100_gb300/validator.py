@@ -161,6 +161,8 @@ class Validator:
             B.pv_aggregate_intents(self.ctx, n, pods, bits, words, flags, assign, ppg, results, dev["pass"][lo:],
                                    dev["counts"][lo * 32:], stream)
 
+    _INPUTS = ("offs", "exprs", "draws", "masks", "flows")
+
     def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
                                  chunks: int = 2, loads=None) -> dict:
         """The end-to-end pipeline on inputs in pinned HOST memory.
@@ -176,7 +178,12 @@ class Validator:
         ``host`` holds pinned byte tensors "offs", "exprs", "draws", "masks",
         "flows" (inputs, as alloc_end_to_end lays them out: 8-byte flows, the
         probe records are built on the device) and "pass", "counts" (outputs);
-        ``dev`` the device buffers of alloc_end_to_end."""
+        ``dev`` the device buffers of alloc_end_to_end.
+
+        Consecutive calls alternate between two sets of device input buffers,
+        so a call's uploads wait only for the call two back (the last one to
+        read that set), not for the previous call's kernels: the uploads of
+        one batch overlap the verification of the one before."""
         I, pods, ppg = e2e_sizes["intents"], e2e_sizes["pods"], e2e_sizes["probes_per_intent"]
         words = W.words_per_row(self.num_nodes)
         ctx = self.ctx
@@ -188,8 +195,18 @@ class Validator:
         ranges = [(lo, hi) for lo, hi in zip(edges[:-1], edges[1:]) if hi > lo]
         if loads is not None:
             loads()
-        # the previous step's kernels must be done with the device inputs
-        copy_stream.wait_stream(stream)
+        if "_inputs" not in dev:   # the second input set, and each set's last reader
+            dev["_inputs"] = [{k: dev[k] for k in self._INPUTS},
+                              {k: torch.empty_like(dev[k]) for k in self._INPUTS}]
+            dev["_read"] = [None, None]
+            dev["_slot"] = [0]
+        k_slot = dev["_slot"][0]
+        dev["_slot"][0] ^= 1
+        read = dev["_read"]
+        dev = {**dev, **dev["_inputs"][k_slot]}
+        # the kernels that last read this input set must be done with it
+        if read[k_slot] is not None:
+            copy_stream.wait_event(read[k_slot])
         ready = []
         with torch.cuda.stream(copy_stream):
             for k in ("offs", "exprs", "draws", "masks"):
@@ -211,6 +228,9 @@ class Validator:
                                 words, flags, stream)
             B.pv_place_pods(ctx, n, pods, bits, words, dev["draws"][lo * pods * 8:], assign, stream)
             self._walk_and_verdict(dev, e2e_sizes, lo, hi, stream)
+        done = torch.cuda.Event()
+        done.record(stream)
+        read[k_slot] = done
         with torch.cuda.stream(stream):
             host["pass"].copy_(dev["pass"][: host["pass"].numel()], non_blocking=True)
             host["counts"].copy_(dev["counts"][: host["counts"].numel()], non_blocking=True)

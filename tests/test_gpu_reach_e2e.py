@@ -259,6 +259,70 @@ def test_end_to_end_pipelined_from_host(validator, chunks):
     assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
 
 
+def test_back_to_back_host_steps_each_with_its_own_tables(validator):
+    """Three host-buffer steps enqueued back to back with no synchronisation,
+    each loading its own cluster and flow tables and verifying its own batch
+    (batches A, B, A): the alternating input buffers and the loads that
+    retire the replaced state only after its last use give every step the
+    oracle's verdicts for its batch."""
+    import torch
+    kw = dict(num_switches=48, num_intents=160, probes_per_intent=90, rules_per_switch=150)
+    ea, eb = W.end_to_end(seed=31, **kw), W.end_to_end(seed=32, **kw)
+    big = ea if len(ea.intents.exprs) >= len(eb.intents.exprs) else eb
+    v = validator
+    v.load_cluster(big.cluster)
+    dev, _ = v.alloc_end_to_end(big)
+
+    def sizes(e):
+        return {"intents": e.intents.num_pods, "pods": e.pods_per_intent, "probes_per_intent": e.probes_per_intent,
+                "num_exprs": len(e.intents.exprs), "hop_cap": e.probes.hop_cap}
+
+    def host(e):
+        I = e.intents.num_pods
+        return {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
+                "draws": _pinned(e.place_draws.astype(np.uint64)), "masks": _pinned(e.intent_mask.astype(np.uint32)),
+                "flows": _pinned(flows_of(e)), "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
+                "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
+
+    stream, cs = torch.cuda.current_stream(), torch.cuda.Stream()
+    steps = [(ea, host(ea)), (eb, host(eb)), (ea, host(ea))]
+    for e, h in steps:
+        v.run_end_to_end_from_host(h, dev, sizes(e), stream, cs, 2,
+                                   lambda e=e: (v.load_cluster(e.cluster), v.load_network(e.network)))
+    stream.synchronize()
+    v.sync()
+    for e, h in steps:
+        bits, flags, assign, probes = _oracle_e2e(e)
+        res = oracle.verify_probes(e.network, probes, e.probes.hop_cap)
+        passed, counts = oracle.aggregate(bits, e.cluster.num_nodes, flags, assign, e.pods_per_intent, res,
+                                          e.probes_per_intent)
+        I = e.intents.num_pods
+        assert (h["pass"].numpy() == passed).all()
+        assert (h["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
+    c = [h["counts"].numpy() for _, h in steps]
+    assert (c[0] == c[2]).all() and not (c[0] == c[1]).all()   # the batches differ; A twice alike
+
+
+def test_failed_table_load_keeps_the_loaded_tables(validator):
+    """A load that fails validation leaves the previously loaded tables in
+    place: walks after it give the same results as before it."""
+    d = W.tiny()
+    net, pr = d["network"], d["probes"].probes
+    v = validator
+    v.load_network(net)
+    first = to_numpy(v.verify_probes(to_device(pr, v.device), len(pr), 16), W.RESULT_DTYPE)
+    bad = net.rules.copy()
+    bad[5]["dst_len"] = 40
+    with pytest.raises(B.PVError) as e:
+        B.pv_load_flow_tables(v.ctx, net.num_switches, net.rule_offs, bad, net.switch_region, net.port_offs,
+                              net.port_peer, net.num_hosts, net.host_switch, net.host_port, net.host_ip)
+    assert e.value.code == B.PV_EINVAL
+    again = to_numpy(v.verify_probes(to_device(pr, v.device), len(pr), 16), W.RESULT_DTYPE)
+    v.sync()
+    assert (again == first).all()
+    assert (first == oracle.verify_probes(net, pr, 16)).all()
+
+
 def test_flow_binding_and_fused_walk(validator):
     """pv_bind_flows builds the oracle's bound probe records from 8-byte
     flows; pv_verify_flows (binding inside the walk's first kernel) gives the

@@ -373,3 +373,83 @@ def test_flow_verification_full_size_sampled(validator, kernel):
     o = oracle.verify_probes(net, P.probes, P.hop_cap, idx=idx)
     assert _same(g[idx], o)
     assert (g["status"] <= W.ST_MISDELIVERED).all()
+
+
+def _scan_totals(net, probes, cap):
+    """(first matches, summed scan depth) of the walk's definition: at every
+    visit to a permitted switch the first match is taken by scanning the
+    switch's rules in first-match order (priority descending, then input
+    order); the depth is the hit's position + 1, or the rule count on a
+    miss.  Every hop is walked (no cycle shortcut)."""
+    per = []
+    for s in range(net.num_switches):
+        rs = net.rules[net.rule_offs[s]:net.rule_offs[s + 1]]
+        order = sorted(range(len(rs)), key=lambda i: (-int(rs[i]["priority"]), i))
+        r = rs[order]
+        lens = lambda L: np.where(L == 0, 0, (0xFFFFFFFF << (32 - L.astype(np.int64))) & 0xFFFFFFFF)
+        per.append((r, lens(r["src_len"]), lens(r["dst_len"])))
+    n_fm = depth = 0
+    for pr in probes:
+        h = int(pr["src_host"])
+        if h >= net.num_hosts:
+            continue
+        s, p = int(net.host_switch[h]), int(net.host_port[h])
+        src, dst, dport, mask = int(pr["src_ip"]), int(pr["dst_ip"]), int(pr["dport"]), int(pr["allowed_mask"])
+        for _ in range(cap):
+            reg = int(net.switch_region[s])
+            if reg >= 32 or not (mask >> reg) & 1:
+                break
+            r, ms, md = per[s]
+            hit = (((r["in_port"] == W.ANY_PORT) | (r["in_port"] == p))
+                   & ((src & ms) == (r["src_ip"].astype(np.int64) & ms))
+                   & ((dst & md) == (r["dst_ip"].astype(np.int64) & md))
+                   & (r["dport_lo"] <= dport) & (dport <= r["dport_hi"]))
+            j = int(np.argmax(hit)) if hit.any() else -1
+            n_fm += 1
+            depth += j + 1 if j >= 0 else len(r)
+            if j < 0 or int(r[j]["action"]) == W.DROP:
+                break
+            port = int(r[j]["action"])
+            if port >= int(net.port_offs[s + 1] - net.port_offs[s]):
+                break
+            peer = int(net.port_peer[net.port_offs[s] + port])
+            if peer < 0 or peer & W.HOST_BIT:
+                break
+            s, p = peer >> 8, peer & 0xFF
+    return n_fm, depth
+
+
+@pytest.mark.parametrize("kernel,tail", [(1, 0), (2, 0), (2, 3)])
+def test_walk_statistics_count_first_matches_and_scan_depth(validator, kernel, tail):
+    """PV_OPT_WALK_STATS: the counting kernels give the same results; their
+    first-match count and ordered-scan depth equal those of the walk's
+    definition recomputed here; the index never disagrees with the scan and
+    tests no more candidates than the scan passes."""
+    d = W.fat_tree(seed=9, k=4, rules_per_switch=120, num_probes=2500, hop_cap=8)
+    net, pr = d["network"], d["probes"].probes
+    o = oracle.verify_probes(net, pr, 8)
+    want_fm, want_depth = _scan_totals(net, pr, 8)
+    v = validator
+    v.set_option(B.PV_OPT_WALK_CYCLES, 1)
+    v.set_option(B.PV_OPT_WALK_TAIL_HOP, tail)
+    v.set_option(B.PV_OPT_WALK_STATS, 1)
+    try:
+        g = _gpu_walk(v, net, pr, 8, kernel)
+        stat = lambda k: B.pv_get_stat(v.ctx, k)
+        fm, tests, looks = stat(B.PV_STAT_WALK_FIRST_MATCHES), stat(B.PV_STAT_WALK_RULE_TESTS), \
+            stat(B.PV_STAT_WALK_INTERVAL_LOOKUPS)
+        depth, bad = stat(B.PV_STAT_WALK_SCAN_DEPTH), stat(B.PV_STAT_WALK_INDEX_MISMATCHES)
+    finally:
+        v.set_option(B.PV_OPT_WALK_STATS, 0)
+        v.set_option(B.PV_OPT_WALK_TAIL_HOP, 8)
+        v.set_option(B.PV_OPT_WALK_CYCLES, 0)
+    assert _same(g, o)
+    assert (fm, depth, bad) == (want_fm, want_depth, 0)
+    assert want_fm > 1000 and tests > 0
+    if kernel == 1:
+        assert looks == 0 and tests % 32 == 0 and tests >= depth
+    else:
+        assert looks > 0 and tests + looks <= depth
+    # the default kernels leave the counters of the last statistics walk alone
+    g2 = _gpu_walk(v, net, pr, 8, kernel)
+    assert _same(g2, o) and B.pv_get_stat(v.ctx, B.PV_STAT_WALK_FIRST_MATCHES) == fm
