@@ -191,11 +191,14 @@ constexpr uint32_t kMaxSegment = 4096;      // longer runs are split (in order: 
 constexpr uint32_t kSegItem = 0x8000u;
 constexpr uint32_t kWinFound = 0x80000000u;
 constexpr int kIndexThreads = 512;
+static_assert(kIndexThreads / 32 == 16, "bucket fill counts are laid out for 16 warps");
 
 // Shared-memory layout of index_build_kernel, sized for the largest table
 // of a load (max_rules rules): sort keys (also the staged port ranges),
-// interval winners, scan positions, rule classes, segment bounds, and one
-// segment's prefixes and actions.
+// interval winners (also the bucket pairs' rule offsets), scan positions,
+// rule classes, segment bounds, one segment's prefixes and actions, and the
+// bucket fill's per-warp counts and cursors.
+constexpr uint32_t kIndexWarps = 512 / 32;
 struct IndexSmem {
     uint32_t sort_cap, key_cap, rules_cap, segs_cap, seg_cap;
     size_t bytes;
@@ -212,6 +215,8 @@ struct IndexSmem {
         segs_cap = n / kMinSegment + n / kMaxSegment + 2;   // runs of >= 4, long runs split
         bytes = (size_t)sort_cap * 4 + (size_t)key_cap * 8 + (size_t)rules_cap * 2 + (size_t)segs_cap * 8 +
                 (size_t)seg_cap * 10;
+        bytes = (bytes + 15) & ~(size_t)15;
+        bytes += (size_t)kIndexWarps * kBuckets * 2 + (size_t)kBuckets * 4;
     }
 };
 
@@ -289,8 +294,12 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
     uint32_t *s_segs = reinterpret_cast<uint32_t *>(s_cls + sm.rules_cap);  // [segs_cap][2]
     uint2 *s_rules = reinterpret_cast<uint2 *>(s_segs + 2 * sm.segs_cap);   // [seg_cap] {value, mask}
     uint16_t *s_act = reinterpret_cast<uint16_t *>(s_rules + sm.seg_cap);    // [seg_cap]
+    uint8_t *s_tail = reinterpret_cast<uint8_t *>(s_mem) +
+                      (((size_t)sm.sort_cap * 4 + (size_t)sm.key_cap * 8 + (size_t)sm.rules_cap * 2 +
+                        (size_t)sm.segs_cap * 8 + (size_t)sm.seg_cap * 10 + 15) & ~(size_t)15);
+    uint16_t *s_wcnt = reinterpret_cast<uint16_t *>(s_tail);                        // [16][kBuckets]
+    uint32_t *s_cur = reinterpret_cast<uint32_t *>(s_tail + kIndexWarps * kBuckets * 2);  // [kBuckets]
     __shared__ uint32_t s_warp[33];
-    __shared__ uint32_t s_nsegs;
     const uint32_t s = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
     const uint32_t n = rule_offs[s + 1] - rule_offs[s];
     const uint32_t t0 = tab_offs[s], npad = tab_offs[s + 1] - t0;
@@ -298,40 +307,58 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
     const uint2 *b = B + t0;
 
     // 1. destination-only runs -> segments.  The rules are classified and
-    //    their port ranges staged in parallel (s_keys is free until the
-    //    segment sort of step 3); one thread then walks the flags.
+    //    their port ranges staged (s_keys is free until the segment sort of
+    //    step 3); block scans then number the runs of destination-only rules
+    //    and their segments (runs shorter than kMinSegment stay plain rules,
+    //    longer ones are cut every kMaxSegment rules).
     for (uint32_t i = t; i < n; i += nt) {
         const uint2 bi = b[i];
         s_cls[i] = rule_dst_only(a[i], bi) ? 1 : -1;
         s_keys[i] = bi.x;   // dport lo | hi << 16
     }
     __syncthreads();
-    if (t == 0) {
-        uint32_t seg = 0, i = 0;
-        while (i < n) {
-            if (s_cls[i] < 0) {
-                ++i;
-                continue;
-            }
-            uint32_t j = i;
-            while (j < n && s_cls[j] > 0) ++j;
-            if (j - i < kMinSegment) {
-                for (uint32_t k = i; k < j; ++k) s_cls[k] = -1;
-            } else {
-                for (uint32_t k0 = i; k0 < j; k0 += kMaxSegment) {
-                    const uint32_t k1 = min(j, k0 + kMaxSegment);
-                    s_segs[2 * seg] = k0;
-                    s_segs[2 * seg + 1] = k1;
-                    for (uint32_t k = k0; k < k1; ++k) s_cls[k] = (int16_t)seg;
-                    ++seg;
-                }
-            }
-            i = j;
-        }
-        s_nsegs = seg;
+    auto run_start = [&](uint32_t i) { return s_cls[i] > 0 && (i == 0 || s_cls[i - 1] < 0); };
+    for (uint32_t i = t; i < n; i += nt) s_pos[i] = run_start(i) ? 1u : 0u;
+    __syncthreads();
+    const uint32_t R = block_exclusive_scan(s_pos, n, s_warp);   // s_pos[i]: runs starting before i
+    uint32_t *s_run = s_win;                                     // [2R]: start, end of each run
+    for (uint32_t i = t; i < n; i += nt) {
+        if (s_cls[i] < 0) continue;
+        const bool st = run_start(i);
+        const uint32_t r = s_pos[i] + (st ? 1u : 0u) - 1u;
+        if (st) s_run[2 * r] = i;
+        if (i + 1 == n || s_cls[i + 1] < 0) s_run[2 * r + 1] = i + 1;
     }
     __syncthreads();
-    const uint32_t nsegs = s_nsegs;
+    for (uint32_t r = t; r < R; r += nt) {
+        const uint32_t len = s_run[2 * r + 1] - s_run[2 * r];
+        s_pos[r] = len < kMinSegment ? 0u : (len + kMaxSegment - 1) / kMaxSegment;
+    }
+    __syncthreads();
+    const uint32_t nsegs = block_exclusive_scan(s_pos, R, s_warp);   // s_pos[r]: first segment of run r
+    for (uint32_t r = t; r < R; r += nt) {
+        const uint32_t r0 = s_run[2 * r], r1 = s_run[2 * r + 1];
+        if (r1 - r0 < kMinSegment) continue;
+        uint32_t seg = s_pos[r];
+        for (uint32_t k0 = r0; k0 < r1; k0 += kMaxSegment, ++seg) {
+            s_segs[2 * seg] = k0;
+            s_segs[2 * seg + 1] = min(r1, k0 + kMaxSegment);
+        }
+    }
+    // each rule's class: its segment, or -1 (a thread reads and writes only
+    // its own rules' flags from here on)
+    for (uint32_t i = t; i < n; i += nt) {
+        if (s_cls[i] < 0) continue;
+        uint32_t lo = 0, hi = R;   // the run holding i: last start <= i
+        while (hi - lo > 1) {
+            const uint32_t mid = (lo + hi) >> 1;
+            if (s_run[2 * mid] <= i) lo = mid;
+            else hi = mid;
+        }
+        const uint32_t r0 = s_run[2 * lo], r1 = s_run[2 * lo + 1];
+        s_cls[i] = r1 - r0 < kMinSegment ? (int16_t)-1 : (int16_t)(s_pos[lo] + (i - r0) / kMaxSegment);
+    }
+    __syncthreads();
     uint8_t *out = nullptr;
     BlobLayout L(npad, 0, 0, 0);
     if (kFill) {
@@ -339,38 +366,79 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
         L = BlobLayout(npad, sizes[3 * s], sizes[3 * s + 1], sizes[3 * s + 2]);
     }
 
-    // 2. bucket lists
-    auto in_bucket = [&](uint32_t i, uint32_t k) -> bool {
-        if (i >= n) return false;
+    // 2. bucket lists.  Rule i puts one item into each bucket its port range
+    //    meets (a segment's token, at the segment's first rule, goes into
+    //    every bucket); the items of rule i take pair positions poff[i] ..
+    //    poff[i] + nb(i) - 1, so pairs run in rule order, and a stable
+    //    counting sort of the pairs by bucket leaves each bucket's items in
+    //    first-match order.
+    auto bucket_range = [&](uint32_t i, uint32_t *b0) -> uint32_t {   // number of buckets
         const int c = s_cls[i];
-        if (c >= 0) return s_segs[2 * c] == i;   // segment token at its first rule
-        const uint32_t lo = s_keys[i] & 0xFFFFu, hi = s_keys[i] >> 16;
-        return lo <= ((k << kBucketShift) | ((1u << kBucketShift) - 1u)) && hi >= (k << kBucketShift);
+        if (c >= 0) {
+            *b0 = 0;
+            return s_segs[2 * c] == i ? kBuckets : 0u;
+        }
+        const uint32_t pr = s_keys[i];
+        *b0 = (pr & 0xFFFFu) >> kBucketShift;
+        return ((pr >> 16) >> kBucketShift) - *b0 + 1u;
     };
-    for (uint32_t k = warp; k < kBuckets; k += nt / 32) {
-        uint32_t cnt = 0;
-        for (uint32_t c0 = 0; c0 < n; c0 += 32) cnt += __popc(__ballot_sync(PV_FULL_MASK, in_bucket(c0 + lane, k)));
-        if (lane == 0) s_pos[k] = cnt;
+    uint32_t *s_poff = s_win;   // [n]: first pair of rule i (s_win is free until step 3)
+    for (uint32_t k = t; k < kBuckets; k += nt) s_pos[k] = 0;
+    for (uint32_t x = t; x < kIndexWarps * kBuckets; x += nt) s_wcnt[x] = 0;
+    __syncthreads();
+    for (uint32_t i = t; i < n; i += nt) {
+        uint32_t b0;
+        const uint32_t nb = bucket_range(i, &b0);
+        s_poff[i] = nb;
+        for (uint32_t k = b0; k < b0 + nb; ++k) atomicAdd(&s_pos[k], 1u);
     }
     __syncthreads();
-    const uint32_t n_items = block_exclusive_scan(s_pos, kBuckets, s_warp);
+    const uint32_t n_items = block_exclusive_scan(s_pos, kBuckets, s_warp);   // s_pos[k] = first item of bucket k
     if (kFill) {
         uint32_t *boff = reinterpret_cast<uint32_t *>(out + L.boff);
         uint16_t *items = reinterpret_cast<uint16_t *>(out + L.items);
-        for (uint32_t k = t; k < kBuckets; k += nt) boff[k] = s_pos[k];
+        for (uint32_t k = t; k < kBuckets; k += nt) {
+            boff[k] = s_pos[k];
+            s_cur[k] = s_pos[k];
+        }
         if (t == 0) boff[kBuckets] = n_items;
-        for (uint32_t k = warp; k < kBuckets; k += nt / 32) {
-            uint32_t base = s_pos[k];
-            for (uint32_t c0 = 0; c0 < n; c0 += 32) {
-                const uint32_t i = c0 + lane;
-                const bool inc = in_bucket(i, k);
-                const uint32_t m = __ballot_sync(PV_FULL_MASK, inc);
-                if (inc) {
-                    const int c = s_cls[i];
-                    items[base + __popc(m & ((1u << lane) - 1u))] = (uint16_t)(c >= 0 ? (kSegItem | (uint32_t)c) : i);
+        block_exclusive_scan(s_poff, n, s_warp);
+        const uint32_t lt = (1u << lane) - 1u;
+        for (uint32_t c0 = 0; c0 < n_items; c0 += nt) {
+            const uint32_t p = c0 + t;
+            const bool on = p < n_items;
+            uint32_t k = 0xFFFFFFFFu, i = 0;
+            if (on) {
+                uint32_t lo = 0, hi = n;   // rule of pair p: last i with poff[i] <= p
+                while (hi - lo > 1) {
+                    const uint32_t mid = (lo + hi) >> 1;
+                    if (s_poff[mid] <= p) lo = mid;
+                    else hi = mid;
                 }
-                base += __popc(m);
+                i = lo;
+                uint32_t b0;
+                bucket_range(i, &b0);
+                k = b0 + (p - s_poff[i]);
             }
+            // rank among this warp's pairs of the same bucket (lanes run in
+            // pair order), then this warp's count per bucket for the others
+            const uint32_t peers = __match_any_sync(PV_FULL_MASK, k);
+            const uint32_t rank = __popc(peers & lt);
+            const bool leader = (peers & lt) == 0;
+            if (on && leader) s_wcnt[warp * kBuckets + k] = (uint16_t)__popc(peers);
+            __syncthreads();
+            if (on) {
+                uint32_t pos = s_cur[k] + rank;
+                for (uint32_t w = 0; w < warp; ++w) pos += s_wcnt[w * kBuckets + k];
+                const int c = s_cls[i];
+                items[pos] = (uint16_t)(c >= 0 ? (kSegItem | (uint32_t)c) : i);
+            }
+            __syncthreads();
+            if (on && leader) {
+                atomicAdd(&s_cur[k], (uint32_t)__popc(peers));
+                s_wcnt[warp * kBuckets + k] = 0;
+            }
+            __syncthreads();
         }
     }
     __syncthreads();
