@@ -703,6 +703,84 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
             if (s_hist[j]) atomicAdd(&hist[j], s_hist[j]);
 }
 
+// First visit of compact flows, placed directly (pv_verify_flows).  The
+// probes of one (group, pod) pair share their source host, mask and path
+// constraint, so a pair is listed or judged as a whole: flow_groups_kernel
+// adds each listed pair's probe count to its source switch (the first hop's
+// per-switch counts) and keeps the pair's offset within that switch; after
+// the scan, walk_init_direct_kernel binds every probe and writes it straight
+// to its slot in the switch-sorted list (switch start + pair offset + rank
+// within the pair), so the first hop needs no regroup.  Probe i belongs to
+// group i / ppg and pod (i mod ppg) mod pods; the caller guarantees one path
+// constraint per group.
+template <bool kPolicy>
+__device__ __forceinline__ bool first_switch_permitted(const PolicyArgs &pa, uint32_t k, uint32_t s, uint32_t reg,
+                                                       uint32_t mask) {
+    bool ok = reg < 32 && ((mask >> reg) & 1u);
+    if (kPolicy && ok) {
+        const uint4 ph = policy_of(pa, k);
+        ok = !switch_listed(pa.sw + ph.x, ph.y, s);
+    }
+    return ok;
+}
+
+template <bool kPolicy>
+__global__ void __launch_bounds__(kGridThreads) flow_groups_kernel(uint32_t M, uint32_t H,
+                                                                   const uint16_t *__restrict__ host_switch,
+                                                                   const uint8_t *__restrict__ region, PolicyArgs pa,
+                                                                   BindArgs ba, uint32_t G, uint32_t *__restrict__ hist,
+                                                                   uint32_t *__restrict__ pair_off) {
+    for (uint32_t g = blockIdx.x * blockDim.x + threadIdx.x; g < G; g += gridDim.x * blockDim.x) {
+        const uint32_t grp = g / ba.pods, q = g - grp * ba.pods;
+        const uint32_t first = grp * ba.ppg, len = min(ba.ppg, M - first);
+        const uint32_t cnt = len > q ? (len - q + ba.pods - 1) / ba.pods : 0u;
+        const uint32_t node = ba.assign[g];
+        uint32_t off = 0;
+        if (cnt && node < H) {
+            const uint32_t s = host_switch[node];
+            if (first_switch_permitted<kPolicy>(pa, first + q, s, region[s], ba.group_mask[grp]))
+                off = atomicAdd(&hist[s], cnt);
+        }
+        pair_off[g] = off;
+    }
+}
+
+template <bool kPolicy>
+__global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
+    uint32_t M, pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
+    const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
+    uint2 *__restrict__ sorted, const uint32_t *__restrict__ seg, const uint32_t *__restrict__ pair_off,
+    PolicyArgs pa, BindArgs ba) {
+    for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < M; i += gridDim.x * blockDim.x) {
+        const uint32_t grp = i / ba.ppg, r = i - grp * ba.ppg, g = grp * ba.pods + r % ba.pods;
+        const uint32_t node = ba.assign[g];
+        const uint2 f = __ldg(ba.flows + i);
+        const bool placed = node < H;
+        const uint32_t mask = ba.group_mask[grp];
+        // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
+        reinterpret_cast<uint4 *>(probes)[i] = make_uint4(
+            placed ? ba.host_ip[node] : 0u, f.x, (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16, mask);
+        if (kPolicy) pa.hits[i] = 0;
+        pv_result res;
+        if (!placed) {
+            res.status = PV_NOSRC;
+            res.hops = 0;
+            res.last_switch = 0xFFFF;
+            out[i] = res;
+            continue;
+        }
+        const uint32_t s = host_switch[node];
+        if (first_switch_permitted<kPolicy>(pa, i, s, region[s], mask)) {
+            sorted[seg[s] + pair_off[g] + r / ba.pods] = make_uint2(i, (s << 8) | host_port[node]);
+        } else {
+            res.status = PV_VIOLATION;
+            res.hops = 1;
+            res.last_switch = (uint16_t)s;
+            out[i] = res;
+        }
+    }
+}
+
 // A live-list entry is uint2 {probe id, loc}: loc bits 0..7 in_port, 8..23
 // switch, 24..31 the hop at which a probe caught in a forwarding cycle is
 // finished (plus one; 0 = not known to cycle).
@@ -1679,7 +1757,14 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     const size_t o_desc = o_cur + align256((size_t)S * 4);
     const size_t o_ck = o_desc + 2 * align256((size_t)max_desc * 8);
     const bool cycles = ctx->opt_walk_cycles == 0 && hop_cap > kCycleCheckFrom;
-    const size_t total = o_ck + (cycles ? align256((size_t)M * 4) : 0);
+    // compact flows with one path constraint per group are placed directly
+    const bool direct = ba && (!pol || (pa->probe_pol == nullptr && (pa->per == 0 || pa->per % ba->ppg == 0)));
+    const uint64_t groups = ba ? ((uint64_t)M + ba->ppg - 1) / ba->ppg : 0;
+    const uint64_t G64 = groups * (ba ? ba->pods : 0);
+    if (direct && G64 > 0xFFFFFFFFull) return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: too many (group, pod) pairs");
+    const uint32_t G = (uint32_t)G64;
+    const size_t o_pair = o_ck + (cycles ? align256((size_t)M * 4) : 0);
+    const size_t total = o_pair + (direct ? align256((size_t)G * 4) : 0);
     uint8_t *base = (uint8_t *)pv_scratch(ctx, total);
     if (!base) return PV_ENOMEM;
     uint2 *listA = (uint2 *)(base + o_a), *listB = (uint2 *)(base + o_b), *sorted = (uint2 *)(base + o_sorted);
@@ -1699,7 +1784,25 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     pv_probe *probes_rw = const_cast<pv_probe *>(d_probes);   // written only when binding
     const PolicyArgs &pa0 = pol ? *pa : no_policy;
     const BindArgs &ba0 = ba ? *ba : no_bind;
-    if (pol && ba)
+    uint32_t *pair_off = (uint32_t *)(base + o_pair);
+    if (direct) {
+        const uint32_t gb = (uint32_t)std::min<uint64_t>((G + kGridThreads - 1) / kGridThreads, init_grid);
+        if (pol)
+            flow_groups_kernel<true><<<gb, kGridThreads, 0, st>>>(M, t.num_hosts, t.d_host_switch, t.d_region, pa0,
+                                                                 ba0, G, hist, pair_off);
+        else
+            flow_groups_kernel<false><<<gb, kGridThreads, 0, st>>>(M, t.num_hosts, t.d_host_switch, t.d_region, pa0,
+                                                                  ba0, G, hist, pair_off);
+        walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
+        if (pol)
+            walk_init_direct_kernel<true><<<init_grid, kGridThreads, 0, st>>>(
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, seg, pair_off,
+                pa0, ba0);
+        else
+            walk_init_direct_kernel<false><<<init_grid, kGridThreads, 0, st>>>(
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, seg, pair_off,
+                pa0, ba0);
+    } else if (pol && ba)
         walk_init_kernel<true, true><<<init_grid, kGridThreads, init_smem, st>>>(
             M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, pa0, S, hist,
             ba0);
@@ -1715,7 +1818,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         walk_init_kernel<false, false><<<init_grid, kGridThreads, init_smem, st>>>(
             M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, pa0, S, hist,
             ba0);
-    pv_prof_stop(ctx, st, pr, 1);
+    pv_prof_stop(ctx, st, pr, direct ? 3 : 1);
     const size_t hist_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     const size_t scat_smem = S <= kSmemHistMax ? (size_t)S * 8 : 0;
     HopArgs g;
@@ -1752,14 +1855,16 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         uint2 *nxt = (h & 1) ? listA : listB;
         uint2 *dcur = (h & 1) ? descB : descA;
         uint2 *dnxt = (h & 1) ? descA : descB;
-        pr = pv_prof_start(ctx, st, PV_K_WALK_REGROUP);
-        // hop 0's counts come from the init kernel, later hops' from the
-        // previous hop kernel when fused
-        const bool counted = h == 0 || fuse_hist;
-        if (!counted) walk_hist_kernel<<<in_slices, kGridThreads, hist_smem, st>>>(cur, dcur, S, hist);
-        walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
-        walk_scatter_kernel<<<in_slices, kGridThreads, scat_smem, st>>>(cur, dcur, S, cursor, sorted);
-        pv_prof_stop(ctx, st, pr, counted ? 2 : 3);
+        if (!(direct && h == 0)) {   // directly placed flows start switch-sorted
+            pr = pv_prof_start(ctx, st, PV_K_WALK_REGROUP);
+            // hop 0's counts come from the init kernel, later hops' from the
+            // previous hop kernel when fused
+            const bool counted = h == 0 || fuse_hist;
+            if (!counted) walk_hist_kernel<<<in_slices, kGridThreads, hist_smem, st>>>(cur, dcur, S, hist);
+            walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
+            walk_scatter_kernel<<<in_slices, kGridThreads, scat_smem, st>>>(cur, dcur, S, cursor, sorted);
+            pv_prof_stop(ctx, st, pr, counted ? 2 : 3);
+        }
         g.hist_next = (fuse_hist && h + 1 < tail_hop) ? hist : nullptr;
         g.sorted = sorted;
         g.hop = h;

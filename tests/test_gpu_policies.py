@@ -184,3 +184,53 @@ def test_constrained_pipeline_from_host(validator, chunks):
     assert (to_numpy(dev["hits"], np.uint32) == oh).all()
     assert (host["pass"].numpy() == passed).all()
     assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
+
+
+@pytest.mark.parametrize("policy_form", ["per_group", "per_probe", "per_pair_of_groups", "none"])
+def test_flow_verification_direct_and_regrouped_first_hop_agree(validator, policy_form):
+    """pv_verify_flows(_constrained) lists compact flows straight into the
+    first hop's switch order when each group has one path constraint (no
+    constraint, or probes_per_policy a multiple of the group size) and
+    regroups them otherwise (a per-probe policy array, or a stride that cuts
+    groups).  Both give the oracle's results, records and waypoint bits; a
+    ragged last group (M not a multiple of the group size) is included."""
+    e = W.end_to_end(seed=41, num_switches=64, num_intents=120, probes_per_intent=70, rules_per_switch=160)
+    v = validator
+    v.load_cluster(e.cluster)
+    v.load_network(e.network)
+    I, pods, ppg = e.intents.num_pods, e.pods_per_intent, e.probes_per_intent
+    M = I * ppg - 33                                    # ragged last group
+    pol = W.path_policies(43, e.network, 2 * I, forbid_max=1, must_max=2, hubs=6, p_noop=0.1)
+    v.load_policies(pol)
+    dev, sizes = v.alloc_end_to_end(e)
+    words = W.words_per_row(e.cluster.num_nodes)
+    B.pv_eval_selectors(v.ctx, I, dev["offs"], sizes["num_exprs"], dev["exprs"], None, dev["bits"], words,
+                        dev["flags"])
+    B.pv_place_pods(v.ctx, I, pods, dev["bits"], words, dev["draws"], dev["assign"])
+    c = e.cluster
+    bits, _ = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, e.intents.expr_offs, e.intents.exprs)
+    assign = oracle.place_pods(bits, c.num_nodes, pods, e.place_draws)
+    probes = oracle.bind_probes(e.probes.probes[:M], ppg, pods, assign, e.network.host_ip)
+    dp, out = empty_device(M * 16, v.device), empty_device(M * 4, v.device)
+    if policy_form == "none":
+        B.pv_verify_flows(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], sizes["hop_cap"], dp, out)
+        v.sync()
+        assert (to_numpy(out, W.RESULT_DTYPE) == oracle.verify_probes(e.network, probes, sizes["hop_cap"])).all()
+        assert (to_numpy(dp, W.PROBE_DTYPE) == probes).all()
+        return
+    per = {"per_group": ppg, "per_probe": 0, "per_pair_of_groups": ppg // 2}[policy_form]
+    pp = None
+    if policy_form == "per_probe":
+        pp_host = (np.arange(M) // ppg).astype(np.uint32)     # the per-group policy, given per probe
+        pp = to_device(pp_host, v.device)
+    hits = empty_device(M * 4, v.device)
+    B.pv_verify_flows_constrained(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], sizes["hop_cap"],
+                                  pp, per, 0, dp, out, hits)
+    v.sync()
+    if policy_form == "per_probe":
+        res, oh = oracle.verify_constrained(e.network, probes, sizes["hop_cap"], pol, probe_policy=pp_host)
+    else:
+        res, oh = oracle.verify_constrained(e.network, probes, sizes["hop_cap"], pol, probes_per_policy=per)
+    assert (to_numpy(out, W.RESULT_DTYPE) == res).all()
+    assert (to_numpy(hits, np.uint32) == oh).all()
+    assert (to_numpy(dp, W.PROBE_DTYPE) == probes).all()
