@@ -325,11 +325,18 @@ int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_
  *   flows: d_flows[k] = {dst_ip, dport} and the group's jurisdiction mask
  *   d_group_mask[g] give the whole probe record d_probes[k] (16-byte
  *   aligned), its source bound as above.
- * pv_verify_flows: pv_bind_flows followed by pv_verify_probes in one call:
- *   the walk's first kernel binds each flow, writes its record to d_probes
- *   (read by the later hops) and starts its walk, so the records are not
- *   read back; same results as the two calls.  pv_verify_flows_constrained
- *   is the same with the path constraints of pv_verify_probes_constrained.
+ * pv_verify_flows: pv_bind_flows followed by pv_verify_probes in one call,
+ *   with the same results: the walk's first kernel binds each flow, writes
+ *   its record to d_probes when d_probes is not NULL (NULL: the bound
+ *   records are not returned), and starts its walk.  When every group has
+ *   one path constraint (always for pv_verify_flows; for the constrained
+ *   call, no d_probe_policy and probes_per_policy 0 or a multiple of
+ *   probes_per_group), the probes of each (group, pod) pair, which share
+ *   their first switch, are counted per switch from the pairs alone and
+ *   written straight into the first hop's switch order, with a compact
+ *   walk record in the library's scratch; otherwise the first hop is
+ *   regrouped like any other.  pv_verify_flows_constrained is the same with
+ *   the path constraints of pv_verify_probes_constrained.
  * pv_aggregate_intents: d_pass[g] = 1 iff every pod of g has d_assign in
  *   row g, d_group_flags[g] has neither PV_F_UNKNOWN_VALUE nor
  *   PV_F_BAD_EXPR, and every probe of g is PV_COMPLIANT.

@@ -749,17 +749,17 @@ template <bool kPolicy>
 __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
     uint32_t M, pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
     const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
-    uint2 *__restrict__ sorted, const uint32_t *__restrict__ seg, const uint32_t *__restrict__ pair_off,
-    PolicyArgs pa, BindArgs ba) {
+    uint2 *__restrict__ sorted, uint4 *__restrict__ recs, const uint32_t *__restrict__ seg,
+    const uint32_t *__restrict__ pair_off, PolicyArgs pa, BindArgs ba) {
     for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < M; i += gridDim.x * blockDim.x) {
         const uint32_t grp = i / ba.ppg, r = i - grp * ba.ppg, g = grp * ba.pods + r % ba.pods;
         const uint32_t node = ba.assign[g];
         const uint2 f = __ldg(ba.flows + i);
         const bool placed = node < H;
         const uint32_t mask = ba.group_mask[grp];
-        // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
-        reinterpret_cast<uint4 *>(probes)[i] = make_uint4(
-            placed ? ba.host_ip[node] : 0u, f.x, (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16, mask);
+        const uint32_t z = (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16;
+        if (probes)   // the caller's copy of the bound record {src_ip, dst_ip, dport | src_host << 16, mask}
+            reinterpret_cast<uint4 *>(probes)[i] = make_uint4(placed ? ba.host_ip[node] : 0u, f.x, z, mask);
         if (kPolicy) pa.hits[i] = 0;
         pv_result res;
         if (!placed) {
@@ -771,7 +771,9 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
         }
         const uint32_t s = host_switch[node];
         if (first_switch_permitted<kPolicy>(pa, i, s, region[s], mask)) {
-            sorted[seg[s] + pair_off[g] + r / ba.pods] = make_uint2(i, (s << 8) | host_port[node]);
+            const uint32_t slot = seg[s] + pair_off[g] + r / ba.pods;
+            recs[slot] = make_uint4(i, f.x, z, mask);
+            sorted[slot] = make_uint2(slot, (s << 8) | host_port[node]);
         } else {
             res.status = PV_VIOLATION;
             res.hops = 1;
@@ -914,6 +916,7 @@ struct HopArgs {
     const int32_t *port_peer;
     const uint32_t *host_ip;
     const pv_probe *probes;
+    const uint4 *recs;   // walk records (kRec kernels)
     pv_result *out;
     uint2 *next_list;
     uint2 *next_desc;
@@ -973,6 +976,23 @@ __device__ __forceinline__ void flush_stats(unsigned long long *stats, const uin
 
 // Linear first match: 32 consecutive rules per warp step.
 // Both first-match routines return kWinFound | action, or 0 for a table miss.
+// A walk reads a probe's header through its list entry's first field: the
+// caller's probe record (pv_verify_probes; the field is the probe id) or,
+// for compact flows placed directly, the walk record the first kernel wrote
+// at the probe's first-hop slot, {probe id, dst_ip, dport | src_host << 16,
+// allowed_mask}, whose source address comes from the host table (kRec): the
+// first hop then reads its records in list order.
+template <bool kRec>
+__device__ __forceinline__ uint4 load_header(const HopArgs &g, uint32_t x, uint32_t *id) {
+    if (kRec) {
+        const uint4 r = __ldg(g.recs + x);
+        *id = r.x;
+        return make_uint4(__ldg(g.host_ip + (r.z >> 16)), r.y, r.z, r.w);
+    }
+    *id = x;
+    return __ldg(reinterpret_cast<const uint4 *>(g.probes) + x);
+}
+
 template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_linear(const uint8_t *sm, uint32_t npad, uint32_t lane, uint32_t src,
                                                        uint32_t dst, uint32_t dport, uint32_t in_port,
@@ -1158,7 +1178,7 @@ __device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t hop, uint
     }
 }
 
-template <bool kIndexed, bool kPolicy, bool kStats>
+template <bool kIndexed, bool kPolicy, bool kStats, bool kRec>
 __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
     __shared__ uint64_t s_bar;
@@ -1226,11 +1246,11 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             // lane j fetches probe j of this warp's batch; records are then
             // broadcast one at a time with shuffles
             uint2 e = make_uint2(0, 0);
-            uint4 pr = make_uint4(0, 0, 0, 0);
+            uint4 pr = make_uint4(0, 0, 0, 0);   // {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
+            uint32_t pid = 0;                     // probe id
             if (lane < cnt) {
                 e = g.sorted[wb + lane];
-                // probe record {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
-                pr = __ldg(reinterpret_cast<const uint4 *>(g.probes) + e.x);
+                pr = load_header<kRec>(g, e.x, &pid);
             }
             // a probe in a known forwarding cycle that has reached its finish hop
             const uint32_t fin = e.y >> 24;
@@ -1290,11 +1310,11 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 stc[kStMismatch] += ref != my_fm ? 1u : 0u;
             }
             if (kPolicy && lane < cnt && !fin_now) {
-                const uint4 ph = policy_of(g.pa, e.x);
+                const uint4 ph = policy_of(g.pa, pid);
                 uint32_t bits = 0;   // waypoints of the probe's policy at this switch
                 for (uint32_t i = 0; i < ph.w; ++i)
                     if (g.pa.sw[ph.z + i] == s) bits |= 1u << i;
-                if (bits) g.pa.hits[e.x] |= bits;
+                if (bits) g.pa.hits[pid] |= bits;
                 if (my_status == kAlive && switch_listed(g.pa.sw + ph.x, ph.y, my_next >> 8))
                     my_status = kViolationNext;   // the next switch is forbidden to this flow
             }
@@ -1304,7 +1324,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 r.status = (uint8_t)(at_next ? (uint32_t)PV_VIOLATION : my_status);
                 r.hops = (uint8_t)(fin_now ? g.cap : g.hop + (at_next ? 2u : 1u));
                 r.last_switch = (uint16_t)(at_next ? (my_next >> 8) : s);
-                g.out[e.x] = r;
+                g.out[pid] = r;
             }
             const bool live = lane < cnt && my_status == kAlive;
             uint32_t nloc = my_next;
@@ -1384,7 +1404,7 @@ __device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict
 // regrouping them by switch every hop would cost more in launches than the
 // table staging saves.  Results, cycle finishing, path constraints and the
 // per-hop live counts are those of walk_hop_kernel.
-template <bool kPolicy, bool kStats>
+template <bool kPolicy, bool kStats, bool kRec>
 __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *__restrict__ list,
                                                         const uint2 *__restrict__ desc, uint32_t nslices,
                                                         uint32_t first_hop) {
@@ -1397,9 +1417,10 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
             bool active = i < d.x + d.y;
             uint2 e = make_uint2(0, 0);
             uint4 pr = make_uint4(0, 0, 0, 0);
+            uint32_t pid = 0;
             if (active) {
                 e = list[i];
-                pr = __ldg(reinterpret_cast<const uint4 *>(g.probes) + e.x);
+                pr = load_header<kRec>(g, e.x, &pid);
             }
             uint32_t loc = e.y;
             for (uint32_t h = first_hop; h < g.cap; ++h) {
@@ -1408,7 +1429,7 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                 if (lane == 0) atomicAdd(&g.hop_live[h], (uint32_t)__popc(live));
                 if (!active) continue;
                 const uint32_t s = (loc >> 8) & 0xFFFFu, in_port = loc & 0xFFu, fin = loc >> 24;
-                uint32_t *out = reinterpret_cast<uint32_t *>(g.out) + e.x;   // {status, hops, last_switch}
+                uint32_t *out = reinterpret_cast<uint32_t *>(g.out) + pid;   // {status, hops, last_switch}
                 if (fin != 0 && fin - 1 == h) {   // finished at its cycle position
                     *out = (uint32_t)PV_LOOP | g.cap << 8 | s << 16;
                     active = false;
@@ -1432,11 +1453,11 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                 uint32_t status, next;
                 hop_outcome(g, h, fm, pr.y, pr.w, pbase, nports, &status, &next);
                 if (kPolicy) {
-                    const uint4 ph = policy_of(g.pa, e.x);
+                    const uint4 ph = policy_of(g.pa, pid);
                     uint32_t bits = 0;
                     for (uint32_t k = 0; k < ph.w; ++k)
                         if (g.pa.sw[ph.z + k] == s) bits |= 1u << k;
-                    if (bits) g.pa.hits[e.x] |= bits;
+                    if (bits) g.pa.hits[pid] |= bits;
                     if (status == kAlive && switch_listed(g.pa.sw + ph.x, ph.y, next >> 8)) status = kViolationNext;
                 }
                 if (status != kAlive) {
@@ -1708,13 +1729,20 @@ namespace {
 using HopKernel = void (*)(HopArgs);
 using TailKernel = void (*)(HopArgs, const uint2 *, const uint2 *, uint32_t, uint32_t);
 
-HopKernel pick_hop_kernel(bool indexed, bool pol, bool stats) {
+template <bool kRec>
+HopKernel pick_hop(bool indexed, bool pol, bool stats) {
     if (stats) {
-        if (indexed) return pol ? walk_hop_kernel<true, true, true> : walk_hop_kernel<true, false, true>;
-        return pol ? walk_hop_kernel<false, true, true> : walk_hop_kernel<false, false, true>;
+        if (indexed) return pol ? walk_hop_kernel<true, true, true, kRec> : walk_hop_kernel<true, false, true, kRec>;
+        return pol ? walk_hop_kernel<false, true, true, kRec> : walk_hop_kernel<false, false, true, kRec>;
     }
-    if (indexed) return pol ? walk_hop_kernel<true, true, false> : walk_hop_kernel<true, false, false>;
-    return pol ? walk_hop_kernel<false, true, false> : walk_hop_kernel<false, false, false>;
+    if (indexed) return pol ? walk_hop_kernel<true, true, false, kRec> : walk_hop_kernel<true, false, false, kRec>;
+    return pol ? walk_hop_kernel<false, true, false, kRec> : walk_hop_kernel<false, false, false, kRec>;
+}
+
+template <bool kRec>
+TailKernel pick_tail(bool pol, bool stats) {
+    return pol ? (stats ? walk_tail_kernel<true, true, kRec> : walk_tail_kernel<true, false, kRec>)
+               : (stats ? walk_tail_kernel<false, true, kRec> : walk_tail_kernel<false, false, kRec>);
 }
 
 int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_cap, pv_result *d_out,
@@ -1724,7 +1752,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     if (!t.loaded) return pv_fail(ctx, PV_ESTATE, "pv_verify_probes: no flow tables loaded");
     if (hop_cap == 0 || hop_cap > PV_MAX_HOP_CAP) return pv_fail(ctx, PV_EINVAL, "hop_cap must be 1..255");
     if (M == 0) return PV_OK;
-    if (!d_probes || !d_out) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: NULL device pointer");
+    if ((!d_probes && !ba) || !d_out) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: NULL device pointer");
     if (((uintptr_t)d_probes & 15) != 0) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: d_probes must be 16-byte aligned");
     const uint32_t S = t.num_switches;
     int which = ctx->opt_walk;
@@ -1740,9 +1768,11 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     const size_t hop_smem = fuse_hist ? hist_off + (size_t)S * 4 : table_smem;
     int hop_blocks_per_sm = 0;
     const bool stats = ctx->opt_walk_stats != 0;
-    const HopKernel hop_fn = pick_hop_kernel(indexed, pol, stats);
-    const TailKernel tail_fn = pol ? (stats ? walk_tail_kernel<true, true> : walk_tail_kernel<true, false>)
-                                   : (stats ? walk_tail_kernel<false, true> : walk_tail_kernel<false, false>);
+    // compact flows with one path constraint per group are placed directly
+    // (and walked through walk records)
+    const bool direct = ba && (!pol || (pa->probe_pol == nullptr && (pa->per == 0 || pa->per % ba->ppg == 0)));
+    const HopKernel hop_fn = direct ? pick_hop<true>(indexed, pol, stats) : pick_hop<false>(indexed, pol, stats);
+    const TailKernel tail_fn = direct ? pick_tail<true>(pol, stats) : pick_tail<false>(pol, stats);
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute((const void *)hop_fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           (int)hop_smem),
                 "walk_hop_kernel smem");
@@ -1757,14 +1787,15 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     const size_t o_desc = o_cur + align256((size_t)S * 4);
     const size_t o_ck = o_desc + 2 * align256((size_t)max_desc * 8);
     const bool cycles = ctx->opt_walk_cycles == 0 && hop_cap > kCycleCheckFrom;
-    // compact flows with one path constraint per group are placed directly
-    const bool direct = ba && (!pol || (pa->probe_pol == nullptr && (pa->per == 0 || pa->per % ba->ppg == 0)));
     const uint64_t groups = ba ? ((uint64_t)M + ba->ppg - 1) / ba->ppg : 0;
     const uint64_t G64 = groups * (ba ? ba->pods : 0);
     if (direct && G64 > 0xFFFFFFFFull) return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: too many (group, pod) pairs");
     const uint32_t G = (uint32_t)G64;
     const size_t o_pair = o_ck + (cycles ? align256((size_t)M * 4) : 0);
-    const size_t total = o_pair + (direct ? align256((size_t)G * 4) : 0);
+    // walk records (direct placement), or bound records the caller did not ask for
+    const bool own_recs = direct || (ba && !d_probes);
+    const size_t o_recs = o_pair + (direct ? align256((size_t)G * 4) : 0);
+    const size_t total = o_recs + (own_recs ? align256((size_t)M * 16) : 0);
     uint8_t *base = (uint8_t *)pv_scratch(ctx, total);
     if (!base) return PV_ENOMEM;
     uint2 *listA = (uint2 *)(base + o_a), *listB = (uint2 *)(base + o_b), *sorted = (uint2 *)(base + o_sorted);
@@ -1782,6 +1813,8 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     const size_t init_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
     const BindArgs no_bind = {nullptr, 1, 1, nullptr, nullptr, nullptr};
     pv_probe *probes_rw = const_cast<pv_probe *>(d_probes);   // written only when binding
+    uint4 *recs = (uint4 *)(base + o_recs);
+    if (ba && !direct && !d_probes) probes_rw = reinterpret_cast<pv_probe *>(recs);   // the walk's own copy
     const PolicyArgs &pa0 = pol ? *pa : no_policy;
     const BindArgs &ba0 = ba ? *ba : no_bind;
     uint32_t *pair_off = (uint32_t *)(base + o_pair);
@@ -1796,12 +1829,12 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
         if (pol)
             walk_init_direct_kernel<true><<<init_grid, kGridThreads, 0, st>>>(
-                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, seg, pair_off,
-                pa0, ba0);
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
+                pair_off, pa0, ba0);
         else
             walk_init_direct_kernel<false><<<init_grid, kGridThreads, 0, st>>>(
-                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, seg, pair_off,
-                pa0, ba0);
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
+                pair_off, pa0, ba0);
     } else if (pol && ba)
         walk_init_kernel<true, true><<<init_grid, kGridThreads, init_smem, st>>>(
             M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, listA, descA, pa0, S, hist,
@@ -1832,7 +1865,8 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.port_offs = t.d_port_offs;
     g.port_peer = t.d_port_peer;
     g.host_ip = t.d_host_ip;
-    g.probes = d_probes;
+    g.probes = probes_rw;
+    g.recs = recs;
     g.out = d_out;
     g.status = ctx->d_status;
     g.lane_max = (uint32_t)ctx->opt_walk_lane_max;

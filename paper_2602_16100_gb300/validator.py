@@ -146,18 +146,18 @@ class Validator:
         ppg, pods, n = e2e_sizes["probes_per_intent"], e2e_sizes["pods"], hi - lo
         words = W.words_per_row(self.num_nodes)
         P, F = W.PROBE_DTYPE.itemsize, W.FLOW_DTYPE.itemsize
-        probes, results = dev["probes"][lo * ppg * P:], dev["results"][lo * ppg * 4:]
+        results = dev["results"][lo * ppg * 4:]
         flows, masks = dev["flows"][lo * ppg * F:], dev["masks"][lo * 4:]
         bits, flags, assign = dev["bits"][lo * words * 4:], dev["flags"][lo:], dev["assign"][lo * pods * 4:]
         cap = e2e_sizes["hop_cap"]
         if "hits" in dev:
             hits = dev["hits"][lo * ppg * 4:]
             B.pv_verify_flows_constrained(self.ctx, n * ppg, flows, ppg, pods, assign, masks, cap, None, ppg, lo,
-                                          probes, results, hits, stream)
+                                          None, results, hits, stream)
             B.pv_aggregate_constrained(self.ctx, n, pods, bits, words, flags, assign, ppg, results, hits, None,
                                        dev["pass"][lo:], dev["counts"][lo * 32:], stream, first_policy=lo)
         else:
-            B.pv_verify_flows(self.ctx, n * ppg, flows, ppg, pods, assign, masks, cap, probes, results, stream)
+            B.pv_verify_flows(self.ctx, n * ppg, flows, ppg, pods, assign, masks, cap, None, results, stream)
             B.pv_aggregate_intents(self.ctx, n, pods, bits, words, flags, assign, ppg, results, dev["pass"][lo:],
                                    dev["counts"][lo * 32:], stream)
 

@@ -160,8 +160,10 @@ def _run_e2e(v, e):
     v.load_network(e.network)
     dev, sizes = v.alloc_end_to_end(e)
     v.run_end_to_end(dev, sizes)
-    v.sync()
     I, pods, ppg = sizes["intents"], sizes["pods"], sizes["probes_per_intent"]
+    # the pipeline does not return the bound records: bind them once more
+    B.pv_bind_flows(v.ctx, I * ppg, dev["flows"], ppg, pods, dev["assign"], dev["masks"], dev["probes"])
+    v.sync()
     words = W.words_per_row(e.cluster.num_nodes)
     return {
         "bits": to_numpy(dev["bits"], np.uint32, (I, words)),
