@@ -783,6 +783,108 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
     }
 }
 
+// The same placement by one block per group, with each pair's run ordered
+// by destination-port bucket of the first-match index, so the lanes of a
+// first-hop warp mostly read the same few candidate lists.  The block counts
+// its probes per (pod, bucket) in shared memory, binds and judges them in one
+// coalesced pass that drops each listed probe (destination, rank in the
+// group, port) into its pod's run in shared memory (the next slot of its
+// bucket), then writes every run out whole as walk records, so each sector
+// of the list and the records is written at once.
+// Used when the counts and the group's records fit kGroupInitSmem.
+constexpr uint32_t kGroupInitMaxPods = 16;
+constexpr uint32_t kGroupInitThreads = 512;
+constexpr size_t kGroupInitSmem = 64 * 1024;   // ppg <= 65535 also fits the rank's 16 bits
+
+template <bool kPolicy>
+__global__ void __launch_bounds__(kGroupInitThreads) walk_init_group_kernel(
+    uint32_t M, pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
+    const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
+    uint2 *__restrict__ sorted, uint4 *__restrict__ recs, const uint32_t *__restrict__ seg,
+    const uint32_t *__restrict__ pair_off, PolicyArgs pa, BindArgs ba) {
+    extern __shared__ __align__(16) uint32_t s_cur[];   // [pods][kBuckets] counts, then slots; then the runs
+    __shared__ uint32_t s_pair[kGroupInitMaxPods][3];   // per pod: {node, switch, listed}
+    const uint32_t grp = blockIdx.x, P = ba.pods, t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    uint2 *s_run = reinterpret_cast<uint2 *>(s_cur + P * kBuckets);   // {dst_ip, rank in group | dport << 16}
+    const uint32_t first = grp * ba.ppg, len = min(ba.ppg, M - first);
+    const uint32_t mask = ba.group_mask[grp];
+    for (uint32_t x = t; x < P * kBuckets; x += kGroupInitThreads) s_cur[x] = 0;
+    if (t < P) {
+        const uint32_t node = ba.assign[grp * P + t];
+        const bool placed = node < H;
+        const uint32_t sw = placed ? host_switch[node] : 0u;
+        s_pair[t][0] = node;
+        s_pair[t][1] = sw;
+        s_pair[t][2] = placed && t < len && first_switch_permitted<kPolicy>(pa, first + t, sw, region[sw], mask);
+    }
+    __syncthreads();
+    for (uint32_t r = t; r < len; r += kGroupInitThreads) {
+        const uint32_t dport = __ldg(ba.flows + first + r).y & 0xFFFFu;
+        atomicAdd(&s_cur[(r % P) * kBuckets + (dport >> kBucketShift)], 1u);
+    }
+    __syncthreads();
+    // exclusive scan of each pod's buckets, offset by the runs of the pods
+    // before it (pod q holds probes q, q + P, ...: ceil((len - q) / P) of them)
+    for (uint32_t q = warp; q < P; q += kGroupInitThreads / 32) {
+        uint32_t *c = s_cur + q * kBuckets;
+        constexpr uint32_t kPer = kBuckets / 32;
+        uint32_t v[kPer], sum = 0;
+        for (uint32_t j = 0; j < kPer; ++j) {
+            v[j] = c[lane * kPer + j];
+            sum += v[j];
+        }
+        uint32_t incl = sum;
+        for (int d = 1; d < 32; d <<= 1) {
+            const uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
+            if (lane >= (uint32_t)d) incl += y;
+        }
+        uint32_t before = 0;   // probes of pods 0 .. q - 1
+        for (uint32_t q2 = 0; q2 < q; ++q2) before += len > q2 ? (len - q2 + P - 1) / P : 0u;
+        uint32_t run = before + incl - sum;
+        for (uint32_t j = 0; j < kPer; ++j) {
+            c[lane * kPer + j] = run;
+            run += v[j];
+        }
+    }
+    __syncthreads();
+    for (uint32_t r = t; r < len; r += kGroupInitThreads) {
+        const uint32_t i = first + r, q = r % P;
+        const uint32_t node = s_pair[q][0], sw = s_pair[q][1];
+        const bool placed = node < H;
+        const uint2 f = __ldg(ba.flows + i);
+        const uint32_t z = (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16;
+        if (probes)   // the caller's copy of the bound record {src_ip, dst_ip, dport | src_host << 16, mask}
+            reinterpret_cast<uint4 *>(probes)[i] = make_uint4(placed ? ba.host_ip[node] : 0u, f.x, z, mask);
+        if (kPolicy) pa.hits[i] = 0;
+        if (s_pair[q][2]) {
+            s_run[atomicAdd(&s_cur[q * kBuckets + ((f.y & 0xFFFFu) >> kBucketShift)], 1u)] =
+                make_uint2(f.x, r | (f.y << 16));
+        } else {
+            pv_result res;
+            res.status = placed ? PV_VIOLATION : PV_NOSRC;
+            res.hops = placed ? 1 : 0;
+            res.last_switch = placed ? (uint16_t)sw : (uint16_t)0xFFFF;
+            out[i] = res;
+        }
+    }
+    __syncthreads();
+    uint32_t before = 0;
+    for (uint32_t q = 0; q < P && q < len; ++q) {
+        const uint32_t n = (len - q + P - 1) / P;
+        if (s_pair[q][2]) {
+            const uint32_t sw = s_pair[q][1];
+            const uint32_t node = s_pair[q][0];
+            const uint32_t base = seg[sw] + pair_off[grp * P + q], loc = (sw << 8) | host_port[node];
+            for (uint32_t k = t; k < n; k += kGroupInitThreads) {
+                const uint2 v = s_run[before + k];
+                recs[base + k] = make_uint4(first + (v.y & 0xFFFFu), v.x, (v.y >> 16) | node << 16, mask);
+                sorted[base + k] = make_uint2(base + k, loc);
+            }
+        }
+        before += n;
+    }
+}
+
 // A live-list entry is uint2 {probe id, loc}: loc bits 0..7 in_port, 8..23
 // switch, 24..31 the hop at which a probe caught in a forwarding cycle is
 // finished (plus one; 0 = not known to cycle).
@@ -1827,7 +1929,26 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
             flow_groups_kernel<false><<<gb, kGridThreads, 0, st>>>(M, t.num_hosts, t.d_host_switch, t.d_region, pa0,
                                                                   ba0, G, hist, pair_off);
         walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
-        if (pol)
+        const uint32_t groups32 = (uint32_t)groups;
+        const size_t gsm = (size_t)ba->pods * kBuckets * 4 + (size_t)ba->ppg * 8;
+        const bool by_group = ba->pods <= kGroupInitMaxPods && gsm <= kGroupInitSmem && groups <= 0x7FFFFFFFull;
+        if (by_group) {
+            PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_init_group_kernel<true>,
+                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGroupInitSmem),
+                        "walk_init_group_kernel smem");
+            PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_init_group_kernel<false>,
+                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGroupInitSmem),
+                        "walk_init_group_kernel smem");
+        }
+        if (by_group && pol)
+            walk_init_group_kernel<true><<<groups32, kGroupInitThreads, gsm, st>>>(
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
+                pair_off, pa0, ba0);
+        else if (by_group)
+            walk_init_group_kernel<false><<<groups32, kGroupInitThreads, gsm, st>>>(
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
+                pair_off, pa0, ba0);
+        else if (pol)
             walk_init_direct_kernel<true><<<init_grid, kGridThreads, 0, st>>>(
                 M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
                 pair_off, pa0, ba0);
