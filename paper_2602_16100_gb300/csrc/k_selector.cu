@@ -330,6 +330,75 @@ __device__ __forceinline__ uint4 expr_rows4(const pv_expr &x, uint32_t w0, bool 
     return r;
 }
 
+// A pod's expressions resolved once, one expression per lane (lists of at
+// most 32): each lane validates its expression, flags In values that no
+// node carries, and leaves the word offsets of the rows to OR (the key's
+// present row for Exists / DoesNotExist) in the warp's shared slots.  The
+// row sweep then reads only rows.  Returns bit0 = a bad expression, bit1 =
+// an unknown value (as pod_prescan).
+constexpr int kRowsWarps = kRowsThreads / 32;
+struct ResolvedExprs {
+    uint32_t meta[kRowsWarps][32];     // op | rows << 8
+    uint32_t off[kRowsWarps][32][8];   // word offset of each row in the row array
+};
+
+__device__ __forceinline__ uint32_t resolve_exprs(ResolvedExprs &rx, uint32_t warp, uint32_t lane, uint32_t lo,
+                                                  uint32_t E, const pv_expr *__restrict__ exprs, uint32_t K,
+                                                  const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
+                                                  const uint32_t *__restrict__ key_base, uint32_t num_value_rows,
+                                                  uint32_t row_words) {
+    bool bad = false, unknown = false;
+    if (lane < E) {
+        const pv_expr *xp = exprs + lo + lane;
+        const uint32_t k = xp->key, op = xp->op, nv = xp->nvals;
+        uint32_t n = 0;
+        if (k >= K) {
+            bad = true;
+        } else if (op == PV_IN || op == PV_NOTIN) {
+            bad = nv < 1 || nv > 8;
+#pragma unroll
+            for (uint32_t j = 0; j < 8; ++j) {
+                if (j >= nv || bad) continue;
+                const uint32_t v = xp->vals[j];
+                if (v == PV_ABSENT) {
+                    bad = true;
+                    continue;
+                }
+                const uint32_t w = inv[(size_t)k * kInvWords + (v >> 5)], bit = v & 31;
+                if ((w >> bit) & 1u) {
+                    const uint32_t row = key_base[k] + rank[(size_t)k * kInvWords + (v >> 5)] +
+                                         __popc(w & ((1u << bit) - 1u));
+                    rx.off[warp][lane][n++] = row * row_words;
+                } else if (op == PV_IN) {
+                    unknown = true;
+                }
+            }
+        } else if (op == PV_EXISTS || op == PV_DOESNOTEXIST) {
+            bad = nv != 0;
+            rx.off[warp][lane][n++] = (num_value_rows + k) * row_words;
+        } else {
+            bad = true;
+        }
+        rx.meta[warp][lane] = op | n << 8;
+    }
+    bad = __any_sync(PV_FULL_MASK, bad);
+    unknown = __any_sync(PV_FULL_MASK, unknown);
+    return (bad ? 1u : 0u) | (unknown ? 2u : 0u);
+}
+
+// Four words from w0 of the node set of resolved expression e.
+__device__ __forceinline__ uint4 resolved_rows4(const ResolvedExprs &rx, uint32_t warp, uint32_t e, uint32_t w0,
+                                                bool in_rows, const uint32_t *__restrict__ rows) {
+    const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = in_rows ? meta >> 8 : 0u;
+    uint4 r = make_uint4(0, 0, 0, 0);
+    for (uint32_t j = 0; j < n; ++j) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j] + w0));
+        r.x |= v.x; r.y |= v.y; r.z |= v.z; r.w |= v.w;
+    }
+    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) { r.x = ~r.x; r.y = ~r.y; r.z = ~r.z; r.w = ~r.w; }
+    return r;
+}
+
 // Clears the bits of nodes >= N in the four words from w0.
 __device__ __forceinline__ void clip_rows4(uint4 &acc, uint32_t w0, uint32_t N) {
     const uint32_t full_words = N >> 5, tail_bits = N & 31;
@@ -348,12 +417,17 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
     uint32_t W, uint8_t *__restrict__ flags, const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
     const uint32_t *__restrict__ key_base, const uint32_t *__restrict__ rows, uint32_t row_words,
     uint32_t num_value_rows) {
-    const uint32_t lane = threadIdx.x & 31;
+    __shared__ ResolvedExprs rx;
+    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t gw = (blockIdx.x * kRowsThreads + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * kRowsThreads) >> 5;
     for (uint32_t p = gw; p < P; p += nw) {
         const uint32_t lo = offs[p], hi = offs[p + 1];
-        const uint32_t pre = pod_prescan(lo, hi, num_exprs, exprs, K, inv, lane);
+        const uint32_t E = hi - lo;
+        const bool resolved = hi >= lo && hi <= num_exprs && E <= 32;
+        const uint32_t pre = resolved ? resolve_exprs(rx, warp, lane, lo, E, exprs, K, inv, rank, key_base,
+                                                      num_value_rows, row_words)
+                                      : pod_prescan(lo, hi, num_exprs, exprs, K, inv, lane);
         uint4 *out = reinterpret_cast<uint4 *>(bits + (size_t)p * W);
         if (pre & 1u) {
             for (uint32_t q = lane; q < W / 4; q += 32) out[q] = make_uint4(0, 0, 0, 0);
@@ -362,22 +436,61 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
         }
         const uint32_t a = assign ? assign[p] : PV_UNPLACED;
         bool any = false, aok = false;
-        for (uint32_t q = lane; q < W / 4; q += 32) {
+        auto finish = [&](uint4 acc, uint32_t q) {
             const uint32_t w0 = q * 4;
-            uint4 acc = make_uint4(~0u, ~0u, ~0u, ~0u);
-            const bool in_rows = w0 < row_words;
-            for (uint32_t e = lo; e < hi; ++e) {
-                const uint4 r = expr_rows4(exprs[e], w0, in_rows, inv, rank, key_base, rows, row_words,
-                                           num_value_rows);
-                acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
-            }
             clip_rows4(acc, w0, N);
-            const uint32_t *aw = &acc.x;
             out[q] = acc;
             any = any || (acc.x | acc.y | acc.z | acc.w) != 0;
+            const uint32_t *aw = &acc.x;
             if (a < N && (a >> 5) >= w0 && (a >> 5) < w0 + 4) aok = (aw[(a >> 5) - w0] >> (a & 31)) & 1u;
+        };
+        if (resolved) {
+            // a lane takes chunks q and q + 32 of each 64-chunk span, so one
+            // pass over the resolved rows (offsets, loop steps) serves both
+            for (uint32_t qb = 0; qb < W / 4; qb += 64) {
+                const uint32_t q0 = qb + lane, q1 = q0 + 32;
+                const bool h0 = q0 < W / 4, h1 = q1 < W / 4;
+                const bool l0 = h0 && q0 * 4 < row_words, l1 = h1 && q1 * 4 < row_words;
+                uint4 a0 = make_uint4(~0u, ~0u, ~0u, ~0u), a1 = a0;
+                for (uint32_t e = 0; e < E; ++e) {
+                    const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = meta >> 8;
+                    uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
+                    for (uint32_t j = 0; j < n; ++j) {
+                        const uint4 *rp = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j]);
+                        if (l0) {
+                            const uint4 x = __ldg(rp + q0);
+                            v0.x |= x.x; v0.y |= x.y; v0.z |= x.z; v0.w |= x.w;
+                        }
+                        if (l1) {
+                            const uint4 x = __ldg(rp + q1);
+                            v1.x |= x.x; v1.y |= x.y; v1.z |= x.z; v1.w |= x.w;
+                        }
+                    }
+                    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) {
+                        a0.x &= ~v0.x; a0.y &= ~v0.y; a0.z &= ~v0.z; a0.w &= ~v0.w;
+                        a1.x &= ~v1.x; a1.y &= ~v1.y; a1.z &= ~v1.z; a1.w &= ~v1.w;
+                    } else {
+                        a0.x &= v0.x; a0.y &= v0.y; a0.z &= v0.z; a0.w &= v0.w;
+                        a1.x &= v1.x; a1.y &= v1.y; a1.z &= v1.z; a1.w &= v1.w;
+                    }
+                }
+                if (h0) finish(a0, q0);
+                if (h1) finish(a1, q1);
+            }
+        } else {
+            for (uint32_t q = lane; q < W / 4; q += 32) {
+                const uint32_t w0 = q * 4;
+                uint4 acc = make_uint4(~0u, ~0u, ~0u, ~0u);
+                const bool in_rows = w0 < row_words;
+                for (uint32_t e = 0; e < E; ++e) {
+                    const uint4 r = expr_rows4(exprs[lo + e], w0, in_rows, inv, rank, key_base, rows, row_words,
+                                               num_value_rows);
+                    acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
+                }
+                finish(acc, q);
+            }
         }
-        any = __any_sync(PV_FULL_MASK, any);
+        any = __any_sync(PV_FULL_MASK, any);   // also keeps the warp's resolved rows until all lanes are done
         aok = __any_sync(PV_FULL_MASK, aok);
         if (lane == 0) flags[p] = pod_flags(any, pre & 2u, assign != nullptr, aok);
     }
@@ -394,14 +507,29 @@ __global__ void __launch_bounds__(kRowsThreads) sel_terms_kernel(
     const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits, uint32_t W, uint8_t *__restrict__ flags,
     const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank, const uint32_t *__restrict__ key_base,
     const uint32_t *__restrict__ rows, uint32_t row_words, uint32_t num_value_rows) {
-    const uint32_t lane = threadIdx.x & 31;
+    __shared__ ResolvedExprs rx;
+    const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t gw = (blockIdx.x * kRowsThreads + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * kRowsThreads) >> 5;
     for (uint32_t p = gw; p < P; p += nw) {
         const uint32_t t0 = pod_terms[p], t1 = pod_terms[p + 1];
         uint32_t pre = (t1 < t0 || t1 > num_terms) ? 1u : 0u;
-        for (uint32_t t = t0; t < t1 && !(pre & 1u); ++t)
-            pre |= pod_prescan(term_offs[t], term_offs[t + 1], num_exprs, exprs, K, inv, lane);
+        // the terms' expressions form one range; lists of at most 32 are resolved once
+        uint32_t e0 = 0, E = 0;
+        bool resolved = false;
+        if (!(pre & 1u) && t1 > t0) {
+            e0 = term_offs[t0];
+            const uint32_t e1 = term_offs[t1];
+            bool mono = e1 >= e0;
+            for (uint32_t t = t0; t < t1 && mono; ++t) mono = term_offs[t + 1] >= term_offs[t];
+            resolved = mono && e1 <= num_exprs && e1 - e0 <= 32;
+            E = resolved ? e1 - e0 : 0u;
+        }
+        if (resolved)
+            pre |= resolve_exprs(rx, warp, lane, e0, E, exprs, K, inv, rank, key_base, num_value_rows, row_words);
+        else
+            for (uint32_t t = t0; t < t1 && !(pre & 1u); ++t)
+                pre |= pod_prescan(term_offs[t], term_offs[t + 1], num_exprs, exprs, K, inv, lane);
         uint4 *out = reinterpret_cast<uint4 *>(bits + (size_t)p * W);
         if (pre & 1u) {
             for (uint32_t q = lane; q < W / 4; q += 32) out[q] = make_uint4(0, 0, 0, 0);
@@ -418,8 +546,9 @@ __global__ void __launch_bounds__(kRowsThreads) sel_terms_kernel(
                 const uint32_t lo = term_offs[t], hi = term_offs[t + 1];
                 uint4 acc = hi > lo ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
                 for (uint32_t e = lo; e < hi; ++e) {
-                    const uint4 r = expr_rows4(exprs[e], w0, in_rows, inv, rank, key_base, rows, row_words,
-                                               num_value_rows);
+                    const uint4 r = resolved ? resolved_rows4(rx, warp, e - e0, w0, in_rows, rows)
+                                             : expr_rows4(exprs[e], w0, in_rows, inv, rank, key_base, rows,
+                                                          row_words, num_value_rows);
                     acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
                 }
                 res.x |= acc.x; res.y |= acc.y; res.z |= acc.z; res.w |= acc.w;
