@@ -386,17 +386,32 @@ __device__ __forceinline__ uint32_t resolve_exprs(ResolvedExprs &rx, uint32_t wa
     return (bad ? 1u : 0u) | (unknown ? 2u : 0u);
 }
 
-// Four words from w0 of the node set of resolved expression e.
-__device__ __forceinline__ uint4 resolved_rows4(const ResolvedExprs &rx, uint32_t warp, uint32_t e, uint32_t w0,
-                                                bool in_rows, const uint32_t *__restrict__ rows) {
-    const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = in_rows ? meta >> 8 : 0u;
-    uint4 r = make_uint4(0, 0, 0, 0);
+// ANDs resolved expression e's node set into the accumulators of chunks q0
+// and q1 (loaded when l0 / l1: words past the rows read 0 before the
+// complement).
+__device__ __forceinline__ void and_resolved2(const ResolvedExprs &rx, uint32_t warp, uint32_t e,
+                                              const uint32_t *__restrict__ rows, uint32_t q0, uint32_t q1, bool l0,
+                                              bool l1, uint4 &a0, uint4 &a1) {
+    const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = meta >> 8;
+    uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
     for (uint32_t j = 0; j < n; ++j) {
-        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j] + w0));
-        r.x |= v.x; r.y |= v.y; r.z |= v.z; r.w |= v.w;
+        const uint4 *rp = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j]);
+        if (l0) {
+            const uint4 x = __ldg(rp + q0);
+            v0.x |= x.x; v0.y |= x.y; v0.z |= x.z; v0.w |= x.w;
+        }
+        if (l1) {
+            const uint4 x = __ldg(rp + q1);
+            v1.x |= x.x; v1.y |= x.y; v1.z |= x.z; v1.w |= x.w;
+        }
     }
-    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) { r.x = ~r.x; r.y = ~r.y; r.z = ~r.z; r.w = ~r.w; }
-    return r;
+    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) {
+        a0.x &= ~v0.x; a0.y &= ~v0.y; a0.z &= ~v0.z; a0.w &= ~v0.w;
+        a1.x &= ~v1.x; a1.y &= ~v1.y; a1.z &= ~v1.z; a1.w &= ~v1.w;
+    } else {
+        a0.x &= v0.x; a0.y &= v0.y; a0.z &= v0.z; a0.w &= v0.w;
+        a1.x &= v1.x; a1.y &= v1.y; a1.z &= v1.z; a1.w &= v1.w;
+    }
 }
 
 // Clears the bits of nodes >= N in the four words from w0.
@@ -452,28 +467,7 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
                 const bool h0 = q0 < W / 4, h1 = q1 < W / 4;
                 const bool l0 = h0 && q0 * 4 < row_words, l1 = h1 && q1 * 4 < row_words;
                 uint4 a0 = make_uint4(~0u, ~0u, ~0u, ~0u), a1 = a0;
-                for (uint32_t e = 0; e < E; ++e) {
-                    const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = meta >> 8;
-                    uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
-                    for (uint32_t j = 0; j < n; ++j) {
-                        const uint4 *rp = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j]);
-                        if (l0) {
-                            const uint4 x = __ldg(rp + q0);
-                            v0.x |= x.x; v0.y |= x.y; v0.z |= x.z; v0.w |= x.w;
-                        }
-                        if (l1) {
-                            const uint4 x = __ldg(rp + q1);
-                            v1.x |= x.x; v1.y |= x.y; v1.z |= x.z; v1.w |= x.w;
-                        }
-                    }
-                    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) {
-                        a0.x &= ~v0.x; a0.y &= ~v0.y; a0.z &= ~v0.z; a0.w &= ~v0.w;
-                        a1.x &= ~v1.x; a1.y &= ~v1.y; a1.z &= ~v1.z; a1.w &= ~v1.w;
-                    } else {
-                        a0.x &= v0.x; a0.y &= v0.y; a0.z &= v0.z; a0.w &= v0.w;
-                        a1.x &= v1.x; a1.y &= v1.y; a1.z &= v1.z; a1.w &= v1.w;
-                    }
-                }
+                for (uint32_t e = 0; e < E; ++e) and_resolved2(rx, warp, e, rows, q0, q1, l0, l1, a0, a1);
                 if (h0) finish(a0, q0);
                 if (h1) finish(a1, q1);
             }
@@ -538,26 +532,48 @@ __global__ void __launch_bounds__(kRowsThreads) sel_terms_kernel(
         }
         const uint32_t a = assign ? assign[p] : PV_UNPLACED;
         bool any = false, aok = false;
-        for (uint32_t q = lane; q < W / 4; q += 32) {
+        auto finish = [&](uint4 res, uint32_t q) {
             const uint32_t w0 = q * 4;
-            const bool in_rows = w0 < row_words;
-            uint4 res = t0 == t1 ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
-            for (uint32_t t = t0; t < t1; ++t) {
-                const uint32_t lo = term_offs[t], hi = term_offs[t + 1];
-                uint4 acc = hi > lo ? make_uint4(~0u, ~0u, ~0u, ~0u) : make_uint4(0, 0, 0, 0);
-                for (uint32_t e = lo; e < hi; ++e) {
-                    const uint4 r = resolved ? resolved_rows4(rx, warp, e - e0, w0, in_rows, rows)
-                                             : expr_rows4(exprs[e], w0, in_rows, inv, rank, key_base, rows,
-                                                          row_words, num_value_rows);
-                    acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
-                }
-                res.x |= acc.x; res.y |= acc.y; res.z |= acc.z; res.w |= acc.w;
-            }
             clip_rows4(res, w0, N);
-            const uint32_t *aw = &res.x;
             out[q] = res;
             any = any || (res.x | res.y | res.z | res.w) != 0;
+            const uint32_t *aw = &res.x;
             if (a < N && (a >> 5) >= w0 && (a >> 5) < w0 + 4) aok = (aw[(a >> 5) - w0] >> (a & 31)) & 1u;
+        };
+        const uint4 none = make_uint4(0, 0, 0, 0), all = make_uint4(~0u, ~0u, ~0u, ~0u);
+        if (resolved) {   // chunks q and q + 32 per lane, as in sel_rows_kernel
+            for (uint32_t qb = 0; qb < W / 4; qb += 64) {
+                const uint32_t q0 = qb + lane, q1 = q0 + 32;
+                const bool h0 = q0 < W / 4, h1 = q1 < W / 4;
+                const bool l0 = h0 && q0 * 4 < row_words, l1 = h1 && q1 * 4 < row_words;
+                uint4 r0 = t0 == t1 ? all : none, r1 = r0;
+                for (uint32_t t = t0; t < t1; ++t) {
+                    const uint32_t lo = term_offs[t] - e0, hi = term_offs[t + 1] - e0;
+                    uint4 a0 = hi > lo ? all : none, a1 = a0;
+                    for (uint32_t e = lo; e < hi; ++e) and_resolved2(rx, warp, e, rows, q0, q1, l0, l1, a0, a1);
+                    r0.x |= a0.x; r0.y |= a0.y; r0.z |= a0.z; r0.w |= a0.w;
+                    r1.x |= a1.x; r1.y |= a1.y; r1.z |= a1.z; r1.w |= a1.w;
+                }
+                if (h0) finish(r0, q0);
+                if (h1) finish(r1, q1);
+            }
+        } else {
+            for (uint32_t q = lane; q < W / 4; q += 32) {
+                const uint32_t w0 = q * 4;
+                const bool in_rows = w0 < row_words;
+                uint4 res = t0 == t1 ? all : none;
+                for (uint32_t t = t0; t < t1; ++t) {
+                    const uint32_t lo = term_offs[t], hi = term_offs[t + 1];
+                    uint4 acc = hi > lo ? all : none;
+                    for (uint32_t e = lo; e < hi; ++e) {
+                        const uint4 r = expr_rows4(exprs[e], w0, in_rows, inv, rank, key_base, rows, row_words,
+                                                   num_value_rows);
+                        acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
+                    }
+                    res.x |= acc.x; res.y |= acc.y; res.z |= acc.z; res.w |= acc.w;
+                }
+                finish(res, q);
+            }
         }
         any = __any_sync(PV_FULL_MASK, any);
         aok = __any_sync(PV_FULL_MASK, aok);
