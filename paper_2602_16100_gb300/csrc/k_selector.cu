@@ -394,7 +394,23 @@ __device__ __forceinline__ void and_resolved2(const ResolvedExprs &rx, uint32_t 
                                               bool l1, uint4 &a0, uint4 &a1) {
     const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = meta >> 8;
     uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
-    for (uint32_t j = 0; j < n; ++j) {
+    uint32_t j = 0;
+    for (; j + 1 < n; j += 2) {   // two rows per step: four loads in flight
+        const uint4 *rp = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j]);
+        const uint4 *rq = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j + 1]);
+        uint4 x0 = make_uint4(0, 0, 0, 0), y0 = x0, x1 = x0, y1 = x0;
+        if (l0) {
+            x0 = __ldg(rp + q0);
+            y0 = __ldg(rq + q0);
+        }
+        if (l1) {
+            x1 = __ldg(rp + q1);
+            y1 = __ldg(rq + q1);
+        }
+        v0.x |= x0.x | y0.x; v0.y |= x0.y | y0.y; v0.z |= x0.z | y0.z; v0.w |= x0.w | y0.w;
+        v1.x |= x1.x | y1.x; v1.y |= x1.y | y1.y; v1.z |= x1.z | y1.z; v1.w |= x1.w | y1.w;
+    }
+    if (j < n) {
         const uint4 *rp = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j]);
         if (l0) {
             const uint4 x = __ldg(rp + q0);
