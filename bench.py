@@ -238,6 +238,7 @@ class EndToEndBench:
                      "counts": torch.empty(e.intents.num_pods * 32, dtype=torch.uint8).pin_memory()}
         self.copy_stream = torch.cuda.Stream()
         self.chunks = chunks
+        self.loads_first = getattr(self, "loads_first", True)
         net = e.network
         self.h2d = (sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "masks", "flows"))
                     + e.cluster.labels.nbytes + net.rule_offs.nbytes + net.rules.nbytes + net.switch_region.nbytes
@@ -258,7 +259,8 @@ class EndToEndBench:
             if self.pol is not None:
                 v.load_policies(self.pol)
 
-        v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks, loads)
+        v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks, loads,
+                                   self.loads_first)
 
     def e2e_phases(self, v, stream, reps=3):
         """Each part of the host-buffer step alone (diagnostic, after the
@@ -774,6 +776,7 @@ def run_ours(args):
     # end-to-end through the public API from pinned host buffers
     e2e = None
     if hasattr(wl, "setup_e2e"):
+        wl.loads_first = args.e2e_loads_first
         wl.setup_e2e(v, args.e2e_chunks)
         for _ in range(max(args.warmup, 1)):
             wl.step_e2e(v, stream)
@@ -785,7 +788,8 @@ def run_ours(args):
         e_s = (time.perf_counter() - t0) / args.steps
         e_s = SH.max_over_ranks(e_s, dist, "cuda")
         e2e = {"value": units * world / e_s, "unit": wl.unit, "h2d_bytes_per_step": int(wl.h2d),
-               "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3, "upload_chunks": args.e2e_chunks}
+               "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3, "upload_chunks": args.e2e_chunks,
+               "loads": "before the uploads" if args.e2e_loads_first else "after the uploads are queued"}
         if hasattr(wl, "e2e_phases"):
             e2e["phases"] = wl.e2e_phases(v, stream)
 
@@ -822,8 +826,10 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", choices=tuple(WORKLOADS), default="e2e")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--e2e-chunks", type=int, default=2,
+    ap.add_argument("--e2e-chunks", type=int, default=1,
                     help="intent ranges whose probe upload overlaps verification in the host-buffer step")
+    ap.add_argument("--e2e-loads-first", action="store_true",
+                    help="host-buffer step: run the table loads before queueing the input uploads (default: after)")
     ap.add_argument("--intents", type=int, default=None,
                     help="end-to-end only: fewer intents (a smaller case for profiling, not a bench line)")
     args = ap.parse_args()

@@ -164,7 +164,7 @@ class Validator:
     _INPUTS = ("offs", "exprs", "draws", "masks", "flows")
 
     def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
-                                 chunks: int = 2, loads=None) -> dict:
+                                 chunks: int = 2, loads=None, loads_first: bool = True) -> dict:
         """The end-to-end pipeline on inputs in pinned HOST memory.
         ``loads()``, if given, runs first (the table loads: their copies go
         out ahead of the inputs, and their device work, which the evaluation
@@ -193,7 +193,7 @@ class Validator:
         P = W.PROBE_DTYPE.itemsize
         F = W.FLOW_DTYPE.itemsize
         ranges = [(lo, hi) for lo, hi in zip(edges[:-1], edges[1:]) if hi > lo]
-        if loads is not None:
+        if loads is not None and loads_first:
             loads()
         if "_inputs" not in dev:   # the second input set, and each set's last reader
             dev["_inputs"] = [{k: dev[k] for k in self._INPUTS},
@@ -218,6 +218,8 @@ class Validator:
                 ev = torch.cuda.Event()
                 ev.record(copy_stream)
                 ready.append(ev)
+        if loads is not None and not loads_first:   # after the uploads are queued
+            loads()
         for (lo, hi), ev in zip(ranges, ready):
             n = hi - lo
             stream.wait_event(ev)
