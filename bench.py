@@ -226,7 +226,7 @@ class EndToEndBench:
         return self.hop_entries if group in ("walk_hop", "walk_regroup") else None
 
     # host-buffer end-to-end step through the public API
-    def setup_e2e(self, v, chunks=2):
+    def setup_e2e(self, v, chunks=1):
         import torch
         e = self.e
         pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1).copy()).pin_memory()
@@ -239,6 +239,7 @@ class EndToEndBench:
         self.copy_stream = torch.cuda.Stream()
         self.chunks = chunks
         self.loads_first = getattr(self, "loads_first", True)
+        self.load_split = getattr(self, "load_split", 0.5)
         net = e.network
         self.h2d = (sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "masks", "flows"))
                     + e.cluster.labels.nbytes + net.rule_offs.nbytes + net.rules.nbytes + net.switch_region.nbytes
@@ -260,7 +261,7 @@ class EndToEndBench:
                 v.load_policies(self.pol)
 
         v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks, loads,
-                                   self.loads_first)
+                                   self.loads_first, self.load_split)
 
     def e2e_phases(self, v, stream, reps=3):
         """Each part of the host-buffer step alone (diagnostic, after the
@@ -777,6 +778,7 @@ def run_ours(args):
     e2e = None
     if hasattr(wl, "setup_e2e"):
         wl.loads_first = args.e2e_loads_first
+        wl.load_split = args.e2e_load_split
         wl.setup_e2e(v, args.e2e_chunks)
         for _ in range(max(args.warmup, 1)):
             wl.step_e2e(v, stream)
@@ -830,6 +832,8 @@ def main():
                     help="intent ranges whose probe upload overlaps verification in the host-buffer step")
     ap.add_argument("--e2e-loads-first", action="store_true",
                     help="host-buffer step: run the table loads before queueing the input uploads (default: after)")
+    ap.add_argument("--e2e-load-split", type=float, default=0.5,
+                    help="host-buffer step: fraction of the flow upload queued before the table loads")
     ap.add_argument("--intents", type=int, default=None,
                     help="end-to-end only: fewer intents (a smaller case for profiling, not a bench line)")
     args = ap.parse_args()

@@ -164,14 +164,17 @@ class Validator:
     _INPUTS = ("offs", "exprs", "draws", "masks", "flows")
 
     def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
-                                 chunks: int = 2, loads=None, loads_first: bool = True) -> dict:
-        """The end-to-end pipeline on inputs in pinned HOST memory.
-        ``loads()``, if given, runs first (the table loads: their copies go
-        out ahead of the inputs, and their device work, which the evaluation
-        calls wait for on the device, overlaps the upload); every input
-        upload is then enqueued on `copy_stream`, the flows cut into `chunks`
-        intent ranges (independent units), and range c is verified on
-        `stream` as soon as its flows have arrived.  The per-intent verdicts and
+                                 chunks: int = 1, loads=None, loads_first: bool = False,
+                                 load_split: float = 0.5) -> dict:
+        """The end-to-end pipeline on inputs in pinned HOST memory.  Every
+        input upload is enqueued on `copy_stream`, the flows cut into
+        `chunks` intent ranges (independent units), and range c is verified
+        on `stream` as soon as its flows have arrived.  ``loads()``, if given
+        (the cluster and table loads), runs between the first `load_split`
+        of the flow upload and the rest, so its copies wait only for that
+        part and its device work (which the evaluation calls wait for on the
+        device) runs while the rest arrives; with `loads_first` it runs
+        before any upload is queued.  The per-intent verdicts and
         counters come back into ``host["pass"]`` and ``host["counts"]`` on
         `stream` (not synchronised).
 
@@ -208,18 +211,30 @@ class Validator:
         if read[k_slot] is not None:
             copy_stream.wait_event(read[k_slot])
         ready = []
+
+        def upload(lo, hi):   # flows of intents [lo, hi)
+            with torch.cuda.stream(copy_stream):
+                dev["flows"][lo * ppg * F:hi * ppg * F].copy_(host["flows"][lo * ppg * F:hi * ppg * F],
+                                                               non_blocking=True)
+
         with torch.cuda.stream(copy_stream):
             for k in ("offs", "exprs", "draws", "masks"):
                 n = host[k].numel()
                 dev[k][:n].copy_(host[k], non_blocking=True)
-            for lo, hi in ranges:
-                dev["flows"][lo * ppg * F:hi * ppg * F].copy_(host["flows"][lo * ppg * F:hi * ppg * F],
-                                                               non_blocking=True)
-                ev = torch.cuda.Event()
-                ev.record(copy_stream)
-                ready.append(ev)
-        if loads is not None and not loads_first:   # after the uploads are queued
-            loads()
+        # with loads after the uploads, the loads go between the first
+        # load_split of the flows and the rest: their copies wait for the
+        # first part only, and their kernels run while the rest arrives
+        cut = ranges[0][0] + int((ranges[0][1] - ranges[0][0]) * load_split) if (loads and not loads_first) else None
+        for c, (lo, hi) in enumerate(ranges):
+            if c == 0 and cut is not None:
+                upload(lo, cut)
+                loads()
+                upload(cut, hi)
+            else:
+                upload(lo, hi)
+            ev = torch.cuda.Event()
+            ev.record(copy_stream)
+            ready.append(ev)
         for (lo, hi), ev in zip(ranges, ready):
             n = hi - lo
             stream.wait_event(ev)

@@ -261,7 +261,8 @@ def test_end_to_end_pipelined_from_host(validator, chunks):
     assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
 
 
-def test_back_to_back_host_steps_each_with_its_own_tables(validator):
+@pytest.mark.parametrize("loads_first", [False, True])
+def test_back_to_back_host_steps_each_with_its_own_tables(validator, loads_first):
     """Three host-buffer steps enqueued back to back with no synchronisation,
     each loading its own cluster and flow tables and verifying its own batch
     (batches A, B, A): the alternating input buffers and the loads that
@@ -289,8 +290,9 @@ def test_back_to_back_host_steps_each_with_its_own_tables(validator):
     stream, cs = torch.cuda.current_stream(), torch.cuda.Stream()
     steps = [(ea, host(ea)), (eb, host(eb)), (ea, host(ea))]
     for e, h in steps:
-        v.run_end_to_end_from_host(h, dev, sizes(e), stream, cs, 2,
-                                   lambda e=e: (v.load_cluster(e.cluster), v.load_network(e.network)))
+        v.run_end_to_end_from_host(h, dev, sizes(e), stream, cs, 2 if loads_first else 1,
+                                   lambda e=e: (v.load_cluster(e.cluster), v.load_network(e.network)),
+                                   loads_first=loads_first)
     stream.synchronize()
     v.sync()
     for e, h in steps:
