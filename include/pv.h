@@ -466,9 +466,11 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  *   gives (checkpoints at hops 4, 8, 16, ...); 1 = walk every hop to the cap.
  *   Both give the same results; PV_STAT_WALK_LIVE_TOTAL differs.
  * PV_OPT_WALK_TAIL_HOP: with the indexed kernel, the walk's hops from this
- *   one on (default 8; 0 = none) run in a single launch, one thread per
- *   probe still walking, tables read from L2 instead of staged per switch.
- *   Same results.
+ *   one on (0 = none) run in a single launch, one thread per probe still
+ *   walking, tables read from L2 instead of staged per switch.  Same
+ *   results.  Default (-1): chosen by pv_load_flow_tables from the loaded
+ *   index, hop 5 when its candidate lists hold at most 12 items per
+ *   destination-port bucket on average, else hop 8.
  * PV_OPT_REACH_KERNEL: 0 = automatic (on a symmetric graph, rows are the
  *   connected components of the permitted subgraph; otherwise multi-source
  *   pull sweeps), 1 = sweeps always.  Both give the same rows.

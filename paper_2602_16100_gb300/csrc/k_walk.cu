@@ -187,6 +187,7 @@ __global__ void __launch_bounds__(1024) compile_tables_kernel(const uint32_t *__
 constexpr uint32_t kBuckets = 256;          // dport >> kBucketShift
 constexpr uint32_t kBucketShift = 8;
 constexpr uint32_t kMinSegment = 4;         // shorter destination-only runs stay plain items
+constexpr uint32_t kTailEarlyItems = 12;    // candidate items per bucket below which the tail starts at hop 5
 constexpr uint32_t kMaxSegment = 4096;      // longer runs are split (in order: still exact)
 constexpr uint32_t kSegItem = 0x8000u;
 constexpr uint32_t kWinFound = 0x80000000u;
@@ -1767,9 +1768,11 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
                        r.dport_lo, r.dport_hi);
     }
     uint32_t max_blob = 0, max_linear = 0;
+    uint64_t all_items = 0;
     if (e == cudaSuccess) {
         for (uint32_t s = 0; s < S; ++s) {
             const uint32_t npad = tab[s + 1] - tab[s];
+            all_items += sizes[3 * s];
             const BlobLayout L(npad, sizes[3 * s], sizes[3 * s + 1], sizes[3 * s + 2]);
             boffs[s + 1] = boffs[s] + L.total;
             max_blob = std::max(max_blob, L.total);
@@ -1795,6 +1798,10 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     }
     t.num_switches = S;
     t.num_hosts = H;
+    // The tail launch walks each probe's candidate lists from L2, one thread
+    // per probe: with short lists (at most kTailEarlyItems items per bucket
+    // on average) it pays from hop 5 on, with long ones only from hop 8.
+    t.tail_hop = all_items <= (uint64_t)kTailEarlyItems * kBuckets * S ? 5u : 8u;
     t.max_rules_padded = max_pad;
     t.max_blob_bytes = max_blob;
     t.max_linear_bytes = max_linear;
@@ -2003,7 +2010,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
     uint32_t in_slices = init_grid;
     // hops from tail_hop on run in one walk_tail_kernel launch (indexed tables only)
-    const uint32_t opt_tail = (uint32_t)ctx->opt_walk_tail_hop;
+    const uint32_t opt_tail = ctx->opt_walk_tail_hop < 0 ? t.tail_hop : (uint32_t)ctx->opt_walk_tail_hop;
     const uint32_t tail_hop = (indexed && opt_tail > 0 && opt_tail < hop_cap) ? opt_tail : hop_cap;
     for (uint32_t h = 0; h < tail_hop; ++h) {
         uint2 *cur = (h & 1) ? listB : listA;

@@ -333,7 +333,7 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         ctx->opt_walk_cycles = (int)value;
         return PV_OK;
     case PV_OPT_WALK_TAIL_HOP:
-        if (value < 0 || value > PV_MAX_HOP_CAP) return pv_fail(ctx, PV_EINVAL, "tail hop must be 0..255");
+        if (value < -1 || value > PV_MAX_HOP_CAP) return pv_fail(ctx, PV_EINVAL, "tail hop must be -1..255");
         ctx->opt_walk_tail_hop = (int)value;
         return PV_OK;
     case PV_OPT_REACH_KERNEL:

@@ -38,6 +38,7 @@ struct pv_table_state {
     uint8_t *d_blob = nullptr;
     uint64_t *d_blob_offs = nullptr;  // [S + 1] byte offsets
     uint32_t max_blob_bytes = 0;      // largest blob (indexed kernel stages it whole)
+    uint32_t tail_hop = 8;            // default first tail hop for these tables (see walk_probes)
     uint32_t max_linear_bytes = 0;    // largest header + rules prefix (linear-scan kernel)
     bool index_fits = false;          // every blob fits shared memory
     uint8_t *d_region = nullptr;      // [S]
@@ -106,7 +107,7 @@ struct pv_ctx {
     int opt_selector = 0, opt_walk = 0;
     int opt_walk_lane_max = 96;
     int opt_walk_cycles = 0;
-    int opt_walk_tail_hop = 8;        // hops from here on run in one tail launch (0: never)
+    int opt_walk_tail_hop = -1;       // hops from here on run in one tail launch (0: never, -1: by the tables)
     int opt_walk_stats = 0;           // 1: walks run the statistics kernels
     unsigned long long *d_walk_stats = nullptr;   // [PV_WALK_STATS] counters of the last statistics walk
     int opt_test_stall_staging = 0;   // failure test: staging waits expect bytes that never come

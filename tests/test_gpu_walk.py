@@ -234,7 +234,7 @@ def test_index_stress_tables(validator, seed):
     assert len(np.unique(o["status"])) >= 3
 
 
-@pytest.mark.parametrize("tail", [0, 1, 5, 8])
+@pytest.mark.parametrize("tail", [0, 1, 5, 8, -1])
 def test_tail_launch_agrees(validator, tail):
     """The last hops in one launch (one thread per probe, tables from L2)
     give the results of the hop-by-hop walk, from any switch-over hop, with
@@ -265,7 +265,7 @@ def test_tail_launch_agrees(validator, tail):
         oc, oh = oracle.verify_constrained(net, pr, 32, pol, probes_per_policy=400)
         assert (to_numpy(out, W.RESULT_DTYPE) == oc).all() and (to_numpy(hits, np.uint32) == oh).all()
     finally:
-        validator.set_option(B.PV_OPT_WALK_TAIL_HOP, 8)
+        validator.set_option(B.PV_OPT_WALK_TAIL_HOP, -1)
         validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
 
 
@@ -441,7 +441,7 @@ def test_walk_statistics_count_first_matches_and_scan_depth(validator, kernel, t
         depth, bad = stat(B.PV_STAT_WALK_SCAN_DEPTH), stat(B.PV_STAT_WALK_INDEX_MISMATCHES)
     finally:
         v.set_option(B.PV_OPT_WALK_STATS, 0)
-        v.set_option(B.PV_OPT_WALK_TAIL_HOP, 8)
+        v.set_option(B.PV_OPT_WALK_TAIL_HOP, -1)
         v.set_option(B.PV_OPT_WALK_CYCLES, 0)
     assert _same(g, o)
     assert (fm, depth, bad) == (want_fm, want_depth, 0)
