@@ -382,6 +382,43 @@ class PlacementBench:
         return self.s.num_pods
 
 
+class ReplicasBench(PlacementBench):
+    """Placement scale with repeated selectors (100,000 pods drawing their
+    expression lists from 10,000 by Zipf popularity, as replicas of
+    deployments do), evaluated with PV_OPT_SELECTOR_DEDUPE; the same step
+    without it is reported beside."""
+    name = "placement-scale, repeated selectors"
+
+    def __init__(self, seed):
+        d = W.selector_replicas(seed=20260226 + seed)
+        self.c, self.s = d["cluster"], d["selectors"]
+        self.distinct = int(len(np.unique(d["pick"])))
+
+    def config(self):
+        return {**super().config(), "distinct_lists": self.distinct, "dedupe": True}
+
+    def setup(self, v):
+        from paper_2602_16100_gb300 import binding as B
+        super().setup(v)
+        B.pv_set_option(v.ctx, B.PV_OPT_SELECTOR_DEDUPE, 1)
+
+    def extra(self, secs_per_step):
+        import torch
+        from paper_2602_16100_gb300 import binding as B
+        B.pv_set_option(self.v.ctx, B.PV_OPT_SELECTOR_DEDUPE, 0)
+        stream = torch.cuda.current_stream()
+        for _ in range(3):
+            self.step(stream)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(10):
+            self.step(stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        B.pv_set_option(self.v.ctx, B.PV_OPT_SELECTOR_DEDUPE, 1)
+        return {"ms_per_step_without_dedupe": a.elapsed_time(b) / 10}
+
+
 class PlacementTermsBench:
     name = "placement-scale, multi-term node affinity"
     unit = "pod×node selector evals/s"
@@ -633,7 +670,8 @@ class WanBench:
 
 
 WORKLOADS = {"e2e": EndToEndBench, "placement_terms": PlacementTermsBench, "schedule": ScheduleBench,
-             "e2e_policies": lambda seed, **kw: EndToEndBench(seed, policies=True, **kw), "placement": PlacementBench, "flow": FlowBench, "wan": WanBench}
+             "e2e_policies": lambda seed, **kw: EndToEndBench(seed, policies=True, **kw), "placement": PlacementBench, "flow": FlowBench, "wan": WanBench,
+             "placement_replicas": ReplicasBench}
 SOURCES = {"schedule": ("k_sched.cu",), "walk_hop": ("k_walk.cu",), "walk_regroup": ("k_walk.cu",), "selector": ("k_selector.cu",),
            "reach": ("k_reach.cu",)}
 

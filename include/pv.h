@@ -452,6 +452,14 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  * PV_OPT_SELECTOR_KERNEL: 0 = automatic, 1 = per-node label comparison over
  *   shared-memory label tiles, 2 = per-(key, value) node-bitset rows
  *   (needs the rows to have been built by pv_load_cluster).
+ * PV_OPT_SELECTOR_DEDUPE: 0 (default) or 1 = pv_eval_selectors evaluates
+ *   each distinct expression list once: pods whose lists are equal (the
+ *   same expressions in the same order, unused value slots ignored), such as
+ *   the replicas of one deployment or intents sharing a selector, get their
+ *   representative's row (the smallest such pod) and flags, with their own
+ *   placement check.  Same results; pays off when lists repeat.  2 = the
+ *   same with deliberately weak hashes (tests: every collision is resolved
+ *   by comparing the lists).  Not used by pv_eval_selector_terms.
  * PV_OPT_WALK_KERNEL: 0 = automatic, 1 = linear first-match scan of the
  *   staged table, 2 = indexed first match (per-dport-bucket candidate lists
  *   and destination-interval maps built by pv_load_flow_tables; needs every
@@ -502,7 +510,8 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  * ------------------------------------------------------------------------- */
 enum {
     PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4,
-    PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6, PV_OPT_WALK_TAIL_HOP = 7, PV_OPT_WALK_STATS = 8
+    PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6, PV_OPT_WALK_TAIL_HOP = 7, PV_OPT_WALK_STATS = 8,
+    PV_OPT_SELECTOR_DEDUPE = 9
 };
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,

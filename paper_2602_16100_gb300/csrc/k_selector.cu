@@ -207,7 +207,7 @@ __global__ void __launch_bounds__(kCmpThreads) sel_cmp_kernel(
     uint32_t N, uint32_t K, const uint16_t *__restrict__ labels, uint32_t tile, uint32_t P,
     const uint32_t *__restrict__ offs, uint32_t num_exprs, const pv_expr *__restrict__ exprs,
     const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits, uint32_t W, uint8_t *__restrict__ flags,
-    const uint32_t *__restrict__ inv) {
+    const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rep_of) {
     extern __shared__ uint16_t s_lab[];   // [K][tile]
     __shared__ uint8_t s_state[kCmpPods]; // bit0 nonempty, bit1 assign ok, bit2 bad, bit3 unknown
     __shared__ pv_expr s_ex[kCmpWarps][kCmpCache];
@@ -220,6 +220,7 @@ __global__ void __launch_bounds__(kCmpThreads) sel_cmp_kernel(
     // per-pod validation / unknown scan (warp per pod)
     for (uint32_t pl = warp; pl < np; pl += kCmpWarps) {
         uint32_t p = p0 + pl;
+        if (rep_of && rep_of[p] != p) continue;   // a duplicate: sel_copy_kernel writes it
         uint32_t r = pod_prescan(offs[p], offs[p + 1], num_exprs, exprs, K, inv, lane);
         if (lane == 0) s_state[pl] = (uint8_t)(((r & 1u) ? 4u : 0u) | ((r & 2u) ? 8u : 0u));
     }
@@ -235,6 +236,7 @@ __global__ void __launch_bounds__(kCmpThreads) sel_cmp_kernel(
         const uint32_t groups = (tn + 31) / 32;
         for (uint32_t pl = warp; pl < np; pl += kCmpWarps) {
             const uint32_t p = p0 + pl;
+            if (rep_of && rep_of[p] != p) continue;
             const uint8_t st = s_state[pl];
             uint32_t *row = bits + (size_t)p * W + (n0 >> 5);
             if (st & 4u) {
@@ -287,6 +289,7 @@ __global__ void __launch_bounds__(kCmpThreads) sel_cmp_kernel(
     // padding words and flags
     for (uint32_t pl = warp; pl < np; pl += kCmpWarps) {
         const uint32_t p = p0 + pl;
+        if (rep_of && rep_of[p] != p) continue;
         for (uint32_t w = nvalid_words + lane; w < W; w += 32) bits[(size_t)p * W + w] = 0;
         if (lane == 0) {
             const uint8_t st = s_state[pl];
@@ -447,12 +450,14 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
     const pv_expr *__restrict__ exprs, const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits,
     uint32_t W, uint8_t *__restrict__ flags, const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
     const uint32_t *__restrict__ key_base, const uint32_t *__restrict__ rows, uint32_t row_words,
-    uint32_t num_value_rows) {
+    uint32_t num_value_rows, const uint32_t *__restrict__ pod_list, const uint32_t *__restrict__ list_len) {
     __shared__ ResolvedExprs rx;
     const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const uint32_t gw = (blockIdx.x * kRowsThreads + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * kRowsThreads) >> 5;
-    for (uint32_t p = gw; p < P; p += nw) {
+    const uint32_t n = pod_list ? *list_len : P;   // with a list: only the pods it names
+    for (uint32_t i = gw; i < n; i += nw) {
+        const uint32_t p = pod_list ? pod_list[i] : i;
         const uint32_t lo = offs[p], hi = offs[p + 1];
         const uint32_t E = hi - lo;
         const bool resolved = hi >= lo && hi <= num_exprs && E <= 32;
@@ -597,6 +602,153 @@ __global__ void __launch_bounds__(kRowsThreads) sel_terms_kernel(
     }
 }
 
+// ---------------------------------------------------------------------------
+// identical selectors evaluated once (pods sharing an expression list, such
+// as the replicas of one deployment, or intents with the same selector)
+// ---------------------------------------------------------------------------
+// A list's canonical form: per expression its key / operator / count word
+// and its value words with the unused value slots zeroed (evaluation never
+// reads them), so equal canonical lists give equal rows and flags.  Each
+// pod's list is hashed (splitmix64's finalizer over the words, mixed with
+// the expression's position) into an open-addressing table whose entries
+// keep the smallest pod with that hash; every other pod with the hash is
+// compared word by word with it, so a hash collision costs only an extra
+// evaluation, never a wrong row.  Representatives are evaluated as usual;
+// each duplicate then copies its representative's row and flags and redoes
+// its own placement check.
+__device__ __forceinline__ uint64_t mix64(uint64_t z) {
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ void canon_expr(const pv_expr *x, uint32_t w[5]) {
+    const uint32_t *raw = reinterpret_cast<const uint32_t *>(x);   // 20-byte records, 4-byte aligned
+    w[0] = raw[0];
+    const bool listed = (x->op == PV_IN || x->op == PV_NOTIN) && x->nvals <= 8;
+    const uint32_t nv = listed ? x->nvals : 0u;
+#pragma unroll
+    for (uint32_t i = 0; i < 4; ++i) {
+        const uint32_t v = raw[1 + i];
+        w[1 + i] = (2 * i < nv ? (v & 0xFFFFu) : 0u) | (2 * i + 1 < nv ? (v & 0xFFFF0000u) : 0u);
+    }
+}
+
+__device__ __forceinline__ uint64_t warp_sum64(uint64_t v) {
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(PV_FULL_MASK, v, o);
+    return v;
+}
+
+// Warp per pod: hashes[p] (0 for a malformed range, which is never shared)
+// and the pod's entry in the table (keys: hash, 0 = free; reps: smallest pod).
+__global__ void __launch_bounds__(256) sel_hash_kernel(uint32_t P, const uint32_t *__restrict__ offs,
+                                                       uint32_t num_exprs, const pv_expr *__restrict__ exprs,
+                                                       unsigned long long *__restrict__ keys,
+                                                       uint32_t *__restrict__ reps, uint32_t cap_mask,
+                                                       uint32_t weak, unsigned long long *__restrict__ hashes) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, nw = (gridDim.x * blockDim.x) >> 5;
+    for (uint32_t p = gw; p < P; p += nw) {
+        const uint32_t lo = offs[p], hi = offs[p + 1];
+        if (hi < lo || hi > num_exprs) {
+            if (lane == 0) hashes[p] = 0;
+            continue;
+        }
+        const uint32_t E = hi - lo;
+        uint64_t acc = 0;
+        for (uint32_t e = lane; e < E; e += 32) {
+            uint32_t w[5];
+            canon_expr(exprs + lo + e, w);
+            uint64_t h = mix64(((uint64_t)e << 32) ^ w[0]);
+#pragma unroll
+            for (uint32_t i = 1; i < 5; ++i) h = mix64(h ^ ((uint64_t)i << 40) ^ w[i]);
+            acc += h;
+        }
+        acc = warp_sum64(acc);
+        uint64_t h = mix64(acc ^ ((uint64_t)E * 0x9E3779B97F4A7C15ull)) | 1ull;
+        if (weak) h = (h & 7ull) + 1ull;   // test mode: eight hash values, so most lists collide
+        if (lane == 0) {
+            hashes[p] = h;
+            // popular lists share a slot: read first, and take an atomic only
+            // to claim a free slot or to lower the slot's pod
+            uint32_t slot = (uint32_t)(h * 0x9E3779B97F4A7C15ull >> 32) & cap_mask;
+            for (uint32_t probe = 0; probe <= cap_mask; ++probe) {   // the table has room for every pod
+                unsigned long long k = *(volatile unsigned long long *)(keys + slot);
+                if (k == 0ull) k = atomicCAS(keys + slot, 0ull, (unsigned long long)h);
+                if (k == 0ull || k == h) {
+                    if (*(volatile uint32_t *)(reps + slot) > p) atomicMin(reps + slot, p);
+                    break;
+                }
+                slot = (slot + 1) & cap_mask;
+            }
+        }
+    }
+}
+
+// Warp per pod: rep_of[p] = the table's pod for p's hash when its canonical
+// list equals p's, else p.
+__global__ void __launch_bounds__(256) sel_rep_kernel(uint32_t P, const uint32_t *__restrict__ offs,
+                                                      const pv_expr *__restrict__ exprs,
+                                                      const unsigned long long *__restrict__ keys,
+                                                      const uint32_t *__restrict__ reps, uint32_t cap_mask,
+                                                      const unsigned long long *__restrict__ hashes,
+                                                      uint32_t *__restrict__ rep_of, uint32_t *__restrict__ rep_list,
+                                                      uint32_t *__restrict__ rep_count) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, nw = (gridDim.x * blockDim.x) >> 5;
+    for (uint32_t p = gw; p < P; p += nw) {
+        const uint64_t h = hashes[p];
+        uint32_t r = p;
+        if (h != 0) {
+            uint32_t slot = (uint32_t)(h * 0x9E3779B97F4A7C15ull >> 32) & cap_mask;
+            for (uint32_t probe = 0; probe <= cap_mask && keys[slot] != h; ++probe) slot = (slot + 1) & cap_mask;
+            r = keys[slot] == h ? reps[slot] : p;
+        }
+        if (r != p) {
+            const uint32_t lo = offs[p], E = offs[p + 1] - lo, lr = offs[r], Er = offs[r + 1] - lr;
+            bool same = E == Er;
+            for (uint32_t e = lane; same && e < E; e += 32) {
+                uint32_t a[5], b[5];
+                canon_expr(exprs + lo + e, a);
+                canon_expr(exprs + lr + e, b);
+#pragma unroll
+                for (int i = 0; i < 5; ++i) same = same && a[i] == b[i];
+            }
+            if (!__all_sync(PV_FULL_MASK, same)) r = p;
+        }
+        if (lane == 0) {
+            rep_of[p] = r;
+            if (r == p) rep_list[atomicAdd(rep_count, 1u)] = p;
+        }
+    }
+}
+
+// Warp per duplicate pod: its representative's row, flags without the
+// placement bits, and its own placement check.
+__global__ void __launch_bounds__(256) sel_copy_kernel(uint32_t P, uint32_t N, uint32_t W,
+                                                       const uint32_t *__restrict__ rep_of,
+                                                       const uint32_t *__restrict__ assign, uint32_t *__restrict__ bits,
+                                                       uint8_t *__restrict__ flags) {
+    const uint32_t lane = threadIdx.x & 31;
+    const uint32_t gw = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, nw = (gridDim.x * blockDim.x) >> 5;
+    for (uint32_t p = gw; p < P; p += nw) {
+        const uint32_t r = rep_of[p];
+        if (r == p) continue;
+        const uint4 *src = reinterpret_cast<const uint4 *>(bits + (size_t)r * W);
+        uint4 *dst = reinterpret_cast<uint4 *>(bits + (size_t)p * W);
+        for (uint32_t q = lane; q < W / 4; q += 32) dst[q] = src[q];
+        if (lane == 0) {
+            uint8_t f = flags[r] & (uint8_t)(PV_F_EMPTY | PV_F_UNKNOWN_VALUE | PV_F_BAD_EXPR);
+            const uint32_t a = assign ? assign[p] : PV_UNPLACED;
+            if (a < N && ((bits[(size_t)r * W + (a >> 5)] >> (a & 31)) & 1u)) {
+                f |= PV_F_ASSIGN_OK;
+                if (!(f & PV_F_UNKNOWN_VALUE)) f |= PV_F_PASS;
+            }
+            flags[p] = f;
+        }
+    }
+}
+
 }  // namespace
 
 // -----------------------------------------------------------------------------
@@ -677,35 +829,60 @@ extern "C" int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t 
     if (which == 2 && !c.rows_built)
         return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: value rows were not built for this cluster");
     cudaStream_t st = (cudaStream_t)stream;
-    if (which == 2) {
-        uint32_t blocks = std::min<uint32_t>((num_pods + 7) / 8, (uint32_t)ctx->num_sms * 16);
-        pv_use_begin(ctx, st);
-        const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
-        sel_rows_kernel<<<blocks, kRowsThreads, 0, st>>>(c.num_nodes, c.num_keys, num_pods, d_expr_offs, num_exprs,
-                                                         d_exprs, d_assign, d_bits, words_per_row, d_flags, c.d_inv,
-                                                         c.d_inv_rank, c.d_key_base, c.d_rows, c.row_words,
-                                                         c.num_value_rows);
-        pv_prof_stop(ctx, st, pr, 1);
-        pv_mark_use(ctx, st);
-        return pv_check_launch(ctx, "sel_rows_kernel");
-    }
-    // tile: as many nodes (multiple of 32) as fit 96 KB of label columns
-    const size_t budget = 96 * 1024;
-    uint32_t tile = (uint32_t)(budget / (2ull * c.num_keys)) / 32 * 32;
-    if (tile < 32) return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: too many keys for the comparison kernel");
+    const uint32_t wblocks = std::min<uint32_t>((num_pods + 7) / 8, (uint32_t)ctx->num_sms * 16);   // warp per pod
+    // comparison kernel: node tiles of as many nodes (multiple of 32) as fit 96 KB of label columns
+    uint32_t tile = (uint32_t)((96 * 1024) / (2ull * c.num_keys)) / 32 * 32;
+    if (which == 1 && tile < 32)
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: too many keys for the comparison kernel");
     tile = min(tile, ((c.num_nodes + 31) / 32) * 32);
-    const size_t smem = (size_t)tile * c.num_keys * 2;
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(sel_cmp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
-                "sel_cmp_kernel smem");
-    const uint32_t blocks = (num_pods + kCmpPods - 1) / kCmpPods;
+    uint32_t *rep_of = nullptr, *rep_list = nullptr, *rep_count = nullptr;
     pv_use_begin(ctx, st);
     const int pr = pv_prof_start(ctx, st, PV_K_SELECTOR);
-    sel_cmp_kernel<<<blocks, kCmpThreads, smem, st>>>(c.num_nodes, c.num_keys, c.d_labels, tile, num_pods,
-                                                      d_expr_offs, num_exprs, d_exprs, d_assign, d_bits,
-                                                      words_per_row, d_flags, c.d_inv);
-    pv_prof_stop(ctx, st, pr, 1);
+    if (ctx->opt_selector_dedupe && num_pods <= (1u << 30)) {
+        uint32_t cap = 1;
+        while ((uint64_t)cap < 2ull * num_pods) cap <<= 1;
+        const size_t o_reps = (size_t)cap * 8, o_hash = o_reps + (((size_t)cap * 4 + 255) & ~(size_t)255);
+        const size_t o_rep = o_hash + (size_t)num_pods * 8, o_list = o_rep + (((size_t)num_pods * 4 + 255) & ~(size_t)255);
+        const size_t total = o_list + (size_t)num_pods * 4 + 256;
+        uint8_t *base = (uint8_t *)pv_scratch(ctx, total);
+        if (!base) {
+            pv_prof_stop(ctx, st, pr, 0);
+            return PV_ENOMEM;
+        }
+        auto *keys = reinterpret_cast<unsigned long long *>(base);
+        auto *reps = reinterpret_cast<uint32_t *>(base + o_reps);
+        auto *hashes = reinterpret_cast<unsigned long long *>(base + o_hash);
+        rep_of = reinterpret_cast<uint32_t *>(base + o_rep);
+        rep_list = reinterpret_cast<uint32_t *>(base + o_list);
+        rep_count = rep_list + num_pods;
+        PV_TRY_CUDA(ctx, cudaMemsetAsync(rep_count, 0, 4, st), "selector list clear");
+        PV_TRY_CUDA(ctx, cudaMemsetAsync(keys, 0, (size_t)cap * 8, st), "selector table clear");
+        PV_TRY_CUDA(ctx, cudaMemsetAsync(reps, 0xFF, (size_t)cap * 4, st), "selector table clear");
+        sel_hash_kernel<<<wblocks, 256, 0, st>>>(num_pods, d_expr_offs, num_exprs, d_exprs, keys, reps, cap - 1,
+                                                  ctx->opt_selector_dedupe == 2 ? 1u : 0u, hashes);
+        sel_rep_kernel<<<wblocks, 256, 0, st>>>(num_pods, d_expr_offs, d_exprs, keys, reps, cap - 1, hashes, rep_of,
+                                                 rep_list, rep_count);
+    }
+    if (which == 2) {
+        sel_rows_kernel<<<wblocks, kRowsThreads, 0, st>>>(c.num_nodes, c.num_keys, num_pods, d_expr_offs, num_exprs,
+                                                          d_exprs, d_assign, d_bits, words_per_row, d_flags, c.d_inv,
+                                                          c.d_inv_rank, c.d_key_base, c.d_rows, c.row_words,
+                                                          c.num_value_rows, rep_list, rep_count);
+    } else {
+        const size_t smem = (size_t)tile * c.num_keys * 2;
+        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(sel_cmp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
+                    "sel_cmp_kernel smem");
+        const uint32_t blocks = (num_pods + kCmpPods - 1) / kCmpPods;
+        sel_cmp_kernel<<<blocks, kCmpThreads, smem, st>>>(c.num_nodes, c.num_keys, c.d_labels, tile, num_pods,
+                                                          d_expr_offs, num_exprs, d_exprs, d_assign, d_bits,
+                                                          words_per_row, d_flags, c.d_inv, rep_of);
+    }
+    if (rep_of)
+        sel_copy_kernel<<<wblocks, 256, 0, st>>>(num_pods, c.num_nodes, words_per_row, rep_of, d_assign, d_bits,
+                                                 d_flags);
+    pv_prof_stop(ctx, st, pr, rep_of ? 4 : 1);
     pv_mark_use(ctx, st);
-    return pv_check_launch(ctx, "sel_cmp_kernel");
+    return pv_check_launch(ctx, "selector kernels");
 }
 
 extern "C" int pv_eval_selector_terms(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_pod_terms, uint32_t num_terms,

@@ -538,6 +538,28 @@ def selector_workload(seed: int = 20260217, num_nodes: int = 5000, num_keys: int
     return dict(cluster=cluster, selectors=Selectors(P, offs, exprs, assign))
 
 
+def selector_replicas(seed: int = 20260226, num_distinct: int = 10_000, num_pods: int = 100_000,
+                      zipf_s: float = 1.1, **kw):
+    """Pods whose selectors repeat, as the replicas of a deployment (or
+    intents sharing a selector) do: ``num_distinct`` expression lists drawn
+    as in selector_workload, each pod taking one of them by Zipf(s)
+    popularity (list 0 the most common), written out in full per pod; one
+    uniform assignment per pod."""
+    d = selector_workload(seed=seed, num_pods=num_distinct, **kw)
+    base = d["selectors"]
+    st = Stream(seed, "replicas")
+    pick = st.zipf(zipf_s, num_distinct, num_pods).astype(np.int64)   # ids 0 .. num_distinct - 1
+    bo = base.expr_offs.astype(np.int64)
+    n = np.diff(bo)[pick]
+    offs = np.zeros(num_pods + 1, np.uint32)
+    offs[1:] = np.cumsum(n)
+    # expression k of pod p is expression k of its list
+    src = bo[np.repeat(pick, n)] + (np.arange(int(n.sum())) - np.repeat(offs[:-1].astype(np.int64), n))
+    exprs = base.exprs[src].copy()
+    assign = st.ints(0, d["cluster"].num_nodes - 1, num_pods).astype(np.uint32)
+    return dict(cluster=d["cluster"], selectors=Selectors(num_pods, offs, exprs, assign), pick=pick)
+
+
 def selector_terms(seed: int = 20260222, num_nodes: int = 5000, num_keys: int = 64, num_values: int = 256,
                    num_pods: int = 100_000, max_terms: int = 3, max_exprs: int = 4, p_empty_term: float = 0.0,
                    **kw):

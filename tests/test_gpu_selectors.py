@@ -137,3 +137,55 @@ def test_placement_scale_sampled(validator):
     validator.set_option(B.PV_OPT_SELECTOR_KERNEL, 0)
     assert (to_numpy(bits1, np.uint32, (len(idx), words)) == ob).all()
     assert (to_numpy(flags1, np.uint8) == of).all()
+
+
+@pytest.mark.parametrize("kernel", [1, 2])
+@pytest.mark.parametrize("mode", [1, 2])
+def test_identical_selectors_evaluated_once(validator, kernel, mode):
+    """PV_OPT_SELECTOR_DEDUPE: pods sharing an expression list (Zipf
+    popularity over a few hundred lists, with absent labels, unknown values,
+    DoesNotExist, malformed expressions, lists that differ only in unused
+    value slots, and pods whose offsets are out of range) give the oracle's
+    rows and flags, each with its own placement check; with weak hashes
+    (mode 2) every list collides with others and is resolved by comparison."""
+    d = W.selector_replicas(seed=61, num_distinct=300, num_pods=5000, num_nodes=1500, num_keys=20, num_values=30,
+                            p_absent=0.05, p_unknown=0.03, with_doesnotexist=True)
+    c, s = d["cluster"], d["selectors"]
+    ex = s.exprs.copy()
+    st = W.Stream(62, "dedupe-edits")
+    bad = st.ints(0, len(ex) - 1, 40)
+    ex["nvals"][bad[:20]] = 9                      # malformed counts
+    ex["op"][bad[20:]] = 7                         # unknown operators
+    slack = np.nonzero((ex["op"] == W.OP_IN) & (ex["nvals"] < 8))[0][:50]
+    ex["vals"][slack, 7] = 29                      # unused slots differ: still the same list
+    offs = s.expr_offs.copy()
+    sel = W.Selectors(s.num_pods, offs, ex, s.assign)
+    ob, of = _oracle_eval(c, sel)
+    v = validator
+    v.set_option(B.PV_OPT_SELECTOR_DEDUPE, mode)
+    try:
+        gb, gf = _gpu_eval(v, c, sel, kernel)
+    finally:
+        v.set_option(B.PV_OPT_SELECTOR_DEDUPE, 0)
+    assert (gf == of).all()
+    assert (gb == ob).all()
+    assert len(np.unique(d["pick"])) < 300 and s.num_pods == 5000   # lists really repeat
+
+
+def test_identical_selectors_with_out_of_range_offsets(validator):
+    """A pod whose expression range is malformed is its own representative
+    (row empty, PV_F_BAD_EXPR), also with dedupe on."""
+    d = W.selector_replicas(seed=63, num_distinct=40, num_pods=400, num_nodes=300, num_keys=8, num_values=12)
+    c, s = d["cluster"], d["selectors"]
+    offs = s.expr_offs.copy()
+    offs[100] = offs[101] + 3                      # pod 100's range is reversed (pod 99's overlaps pod 100's list)
+    sel = W.Selectors(s.num_pods, offs, s.exprs, s.assign)
+    ob, of = _oracle_eval(c, sel)
+    v = validator
+    v.set_option(B.PV_OPT_SELECTOR_DEDUPE, 1)
+    try:
+        gb, gf = _gpu_eval(v, c, sel, 2)
+    finally:
+        v.set_option(B.PV_OPT_SELECTOR_DEDUPE, 0)
+    assert (gf == of).all() and (gb == ob).all()
+    assert of[100] == W.F_BAD_EXPR
