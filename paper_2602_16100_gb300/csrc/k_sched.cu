@@ -47,6 +47,10 @@ __device__ __forceinline__ uint32_t link_weight(const SchedArgs &a, uint32_t u, 
     return w ? w : 1u;   // a weight of 0 counts as 1
 }
 
+// With kStaged the block first copies the links into each switch, with their
+// weights resolved, to shared memory, where every sweep and the predecessor
+// pass read them.
+template <bool kStaged>
 __global__ void __launch_bounds__(kSchedThreads) sched_paths_kernel(SchedArgs a) {
     extern __shared__ uint32_t s_mem[];
     const uint32_t S = a.S, okw = (S + 31) / 32;
@@ -54,9 +58,30 @@ __global__ void __launch_bounds__(kSchedThreads) sched_paths_kernel(SchedArgs a)
     uint32_t *ok = s_mem + S;                        // [okw] permitted switches
     uint32_t *vis = ok + okw;                        // [max_len] visits
     uint32_t *back = vis + a.max_len;                // [max_len] links of a segment, last first
+    uint32_t *pred = back + a.max_len;               // [S] canonical predecessor link (kStaged)
+    uint32_t *g_offs = pred + (kStaged ? S : 0u);    // [S + 1]
+    const uint32_t L = a.in_offs[S];
+    uint32_t *g_links = g_offs + (kStaged ? S + 1 : 0u);   // [L]
+    uint16_t *g_w = reinterpret_cast<uint16_t *>(g_links + (kStaged ? L : 0u));   // [L] link weights
     __shared__ uint32_t s_st, s_n;
     const uint32_t t = threadIdx.x, nt = blockDim.x;
     auto allowed = [&](uint32_t s) { return (ok[s >> 5] >> (s & 31)) & 1u; };
+    const uint32_t *in_offs = a.in_offs, *in_links = a.in_links;
+    if (kStaged) {
+        for (uint32_t v = t; v <= S; v += nt) g_offs[v] = a.in_offs[v];
+        for (uint32_t l = t; l < L; l += nt) {
+            const uint32_t x = a.in_links[l];
+            g_links[l] = x;
+            g_w[l] = (uint16_t)link_weight(a, x >> 16, (x >> 8) & 0xFFu);
+        }
+        __syncthreads();
+        in_offs = g_offs;
+        in_links = g_links;
+    }
+    // weight of in-link l = (u, p) of switch v
+    auto lw = [&](uint32_t l, uint32_t x) -> uint32_t {
+        return kStaged ? (uint32_t)g_w[l] : link_weight(a, x >> 16, (x >> 8) & 0xFFu);
+    };
     for (uint32_t r = blockIdx.x; r < a.R; r += gridDim.x) {
         const pv_path_req q = a.req[r];
         if (q.src_host >= a.H || q.dst_host >= a.H) {
@@ -98,12 +123,12 @@ __global__ void __launch_bounds__(kSchedThreads) sched_paths_kernel(SchedArgs a)
                 for (uint32_t v = t; v < S; v += nt) {
                     if (v == cur || !allowed(v)) continue;
                     uint32_t best = dist[v];
-                    for (uint32_t l = a.in_offs[v]; l < a.in_offs[v + 1]; ++l) {
-                        const uint32_t L = a.in_links[l], u = L >> 16;
+                    for (uint32_t l = in_offs[v]; l < in_offs[v + 1]; ++l) {
+                        const uint32_t x = in_links[l], u = x >> 16;
                         if (!allowed(u)) continue;
                         const uint32_t du = dist[u];
                         if (du == kInf) continue;
-                        const uint32_t c = du + link_weight(a, u, (L >> 8) & 0xFFu);
+                        const uint32_t c = du + lw(l, x);
                         if (c < best) best = c;
                     }
                     if (best < dist[v]) {
@@ -117,16 +142,34 @@ __global__ void __launch_bounds__(kSchedThreads) sched_paths_kernel(SchedArgs a)
                 st = PV_PATH_BLOCKED;
                 break;
             }
+            if (kStaged) {
+                // every switch's canonical predecessor at once: the first link
+                // (smallest (u, p)) on a shortest path into it
+                for (uint32_t v = t; v < S; v += nt) {
+                    uint32_t pick = kInf;
+                    if (v != cur && dist[v] != kInf)
+                        for (uint32_t l = in_offs[v]; l < in_offs[v + 1] && pick == kInf; ++l) {
+                            const uint32_t x = in_links[l], u = x >> 16;
+                            if (allowed(u) && dist[u] != kInf && dist[u] + lw(l, x) == dist[v]) pick = x;
+                        }
+                    pred[v] = pick;
+                }
+                __syncthreads();
+            }
             if (t == 0) {
                 // canonical walk back from tgt: smallest (u, p) on a shortest path
                 const uint32_t room = a.max_len - n;
                 uint32_t k = 0, v = tgt, s_status = PV_PATH_OK;
                 while (v != cur) {
                     uint32_t pick = kInf;
-                    for (uint32_t l = a.in_offs[v]; l < a.in_offs[v + 1] && pick == kInf; ++l) {
-                        const uint32_t L = a.in_links[l], u = L >> 16;
-                        if (!allowed(u) || dist[u] == kInf) continue;
-                        if (dist[u] + link_weight(a, u, (L >> 8) & 0xFFu) == dist[v]) pick = L;
+                    if (kStaged) {
+                        pick = pred[v];
+                    } else {
+                        for (uint32_t l = in_offs[v]; l < in_offs[v + 1] && pick == kInf; ++l) {
+                            const uint32_t x = in_links[l], u = x >> 16;
+                            if (!allowed(u) || dist[u] == kInf) continue;
+                            if (dist[u] + lw(l, x) == dist[v]) pick = x;
+                        }
                     }
                     if (pick == kInf) {   // cannot happen once the distances are exact
                         s_status = PV_PATH_BLOCKED;
@@ -245,15 +288,23 @@ extern "C" int pv_schedule_paths(pv_ctx *ctx, uint32_t num_requests, const pv_pa
     a.visits = d_visits;
     a.len = d_len;
     a.status = d_status;
-    const size_t smem = ((size_t)a.S + (a.S + 31) / 32 + 2 * (size_t)max_len) * 4;
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(sched_paths_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
-                "sched smem");
+    const size_t base_smem = ((size_t)a.S + (a.S + 31) / 32 + 2 * (size_t)max_len) * 4;
+    // the links (with weights) and the predecessors staged when they fit
+    const uint32_t L = t.num_links;
+    const size_t staged_smem = base_smem + ((size_t)a.S + (size_t)a.S + 1 + L) * 4 + ((size_t)L * 2 + 15) / 16 * 16;
+    const bool staged = staged_smem <= std::min<size_t>(96 * 1024, ctx->max_smem_optin - 1024);
+    const size_t smem = staged ? staged_smem : base_smem;
+    const void *fn = staged ? (const void *)sched_paths_kernel<true> : (const void *)sched_paths_kernel<false>;
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem), "sched smem");
     int per_sm = 1;
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, sched_paths_kernel, kSchedThreads, smem);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kSchedThreads, smem);
     const uint32_t grid = std::min<uint32_t>(num_requests, (uint32_t)std::max(per_sm, 1) * ctx->num_sms);
     pv_use_begin(ctx, (cudaStream_t)stream);
     const int pr = pv_prof_start(ctx, (cudaStream_t)stream, PV_K_SCHEDULE);
-    sched_paths_kernel<<<grid, kSchedThreads, smem, (cudaStream_t)stream>>>(a);
+    if (staged)
+        sched_paths_kernel<true><<<grid, kSchedThreads, smem, (cudaStream_t)stream>>>(a);
+    else
+        sched_paths_kernel<false><<<grid, kSchedThreads, smem, (cudaStream_t)stream>>>(a);
     pv_prof_stop(ctx, (cudaStream_t)stream, pr, 1);
     pv_mark_use(ctx, (cudaStream_t)stream);
     return pv_check_launch(ctx, "sched_paths_kernel");

@@ -1711,6 +1711,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         int rc2;
         if ((rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_offs, (S + 1) * 4, "in-link offsets")) ||
             (rc2 = pv_pool_alloc(ctx, (void **)&t.d_in_links, links.size() * 4, "in-links"))) {
+            t.num_links = 0;
             free_temps();
             pv_free_tables(ctx, t);
             return rc2;
@@ -1718,6 +1719,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         cudaError_t e2 = cudaMemcpyAsync(t.d_in_offs, in_offs.data(), (S + 1) * 4, cudaMemcpyHostToDevice, ls);
         if (e2 == cudaSuccess)
             e2 = cudaMemcpyAsync(t.d_in_links, links.data(), links.size() * 4, cudaMemcpyHostToDevice, ls);
+        t.num_links = in_offs[S];
 
         if (e2 != cudaSuccess) {
             free_temps();

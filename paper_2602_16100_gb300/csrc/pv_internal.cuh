@@ -50,6 +50,7 @@ struct pv_table_state {
     // source port): u << 16 | p << 8 | q for port p of u cabled to port q
     uint32_t *d_in_offs = nullptr;    // [S + 1]
     uint32_t *d_in_links = nullptr;   // [links]
+    uint32_t num_links = 0;           // switch-to-switch links
     pv_rule *d_raw = nullptr;         // [rules] as loaded (for rule installation)
 };
 
