@@ -460,6 +460,11 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  *   placement check.  Same results; pays off when lists repeat.  2 = the
  *   same with deliberately weak hashes (tests: every collision is resolved
  *   by comparing the lists).  Not used by pv_eval_selector_terms.
+ * PV_OPT_SCHED_KERNEL: pv_schedule_paths' kernel (one block per request):
+ *   0 = automatic (the links into each switch, with their weights, staged
+ *   in shared memory when they fit, else read from global memory); 1 =
+ *   links from global memory; 2 = staged (PV_EINVAL if they do not fit).
+ *   Both give the same paths.
  * PV_OPT_WALK_KERNEL: 0 = automatic, 1 = linear first-match scan of the
  *   staged table, 2 = indexed first match (per-dport-bucket candidate lists
  *   and destination-interval maps built by pv_load_flow_tables; needs every
@@ -511,7 +516,7 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
 enum {
     PV_OPT_SELECTOR_KERNEL = 1, PV_OPT_WALK_KERNEL = 2, PV_OPT_WALK_LANE_MAX = 3, PV_OPT_TEST_STALL_STAGING = 4,
     PV_OPT_REACH_KERNEL = 5, PV_OPT_WALK_CYCLES = 6, PV_OPT_WALK_TAIL_HOP = 7, PV_OPT_WALK_STATS = 8,
-    PV_OPT_SELECTOR_DEDUPE = 9
+    PV_OPT_SELECTOR_DEDUPE = 9, PV_OPT_SCHED_KERNEL = 10
 };
 enum {
     PV_STAT_SELECTOR_ROWS_BUILT = 1, PV_STAT_SCRATCH_BYTES = 2, PV_STAT_WALK_INDEX_FITS = 3,

@@ -24,7 +24,7 @@ PV_OPT_SELECTOR_KERNEL, PV_OPT_WALK_KERNEL, PV_OPT_WALK_LANE_MAX, PV_OPT_TEST_ST
 PV_STAT_SELECTOR_ROWS_BUILT, PV_STAT_SCRATCH_BYTES, PV_STAT_WALK_INDEX_FITS, PV_STAT_WALK_INDEX_BYTES = 1, 2, 3, 4
 PV_STAT_WALK_LIVE_TOTAL, PV_STAT_REACH_COMPONENTS = 5, 6
 PV_OPT_REACH_KERNEL, PV_OPT_WALK_CYCLES, PV_OPT_WALK_TAIL_HOP = 5, 6, 7
-PV_OPT_WALK_STATS, PV_OPT_SELECTOR_DEDUPE = 8, 9
+PV_OPT_WALK_STATS, PV_OPT_SELECTOR_DEDUPE, PV_OPT_SCHED_KERNEL = 8, 9, 10
 (PV_STAT_WALK_FIRST_MATCHES, PV_STAT_WALK_RULE_TESTS, PV_STAT_WALK_INTERVAL_LOOKUPS, PV_STAT_WALK_SCAN_DEPTH,
  PV_STAT_WALK_INDEX_MISMATCHES) = 7, 8, 9, 10, 11
 

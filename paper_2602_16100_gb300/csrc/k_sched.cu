@@ -292,7 +292,11 @@ extern "C" int pv_schedule_paths(pv_ctx *ctx, uint32_t num_requests, const pv_pa
     // the links (with weights) and the predecessors staged when they fit
     const uint32_t L = t.num_links;
     const size_t staged_smem = base_smem + ((size_t)a.S + (size_t)a.S + 1 + L) * 4 + ((size_t)L * 2 + 15) / 16 * 16;
-    const bool staged = staged_smem <= std::min<size_t>(96 * 1024, ctx->max_smem_optin - 1024);
+    const int force = ctx->opt_sched_kernel;   // 0 automatic, 1 links from global memory, 2 staged
+    const bool staged_fits = staged_smem <= std::min<size_t>(96 * 1024, ctx->max_smem_optin - 1024);
+    if (force == 2 && !staged_fits)
+        return pv_fail(ctx, PV_EINVAL, "pv_schedule_paths: the staged links do not fit shared memory");
+    const bool staged = force == 2 || (force == 0 && staged_fits);
     const size_t smem = staged ? staged_smem : base_smem;
     const void *fn = staged ? (const void *)sched_paths_kernel<true> : (const void *)sched_paths_kernel<false>;
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem), "sched smem");

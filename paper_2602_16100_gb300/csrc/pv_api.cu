@@ -340,6 +340,10 @@ extern "C" int pv_set_option(pv_ctx *ctx, int option, int64_t value) {
         if (value < 0 || value > 1) return pv_fail(ctx, PV_EINVAL, "reach kernel must be 0 or 1");
         ctx->opt_reach = (int)value;
         return PV_OK;
+    case PV_OPT_SCHED_KERNEL:
+        if (value < 0 || value > 2) return pv_fail(ctx, PV_EINVAL, "scheduler kernel must be 0..2");
+        ctx->opt_sched_kernel = (int)value;
+        return PV_OK;
     case PV_OPT_SELECTOR_DEDUPE:
         if (value < 0 || value > 2) return pv_fail(ctx, PV_EINVAL, "selector dedupe switch must be 0, 1 or 2");
         ctx->opt_selector_dedupe = (int)value;

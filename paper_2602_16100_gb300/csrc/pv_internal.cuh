@@ -106,7 +106,8 @@ struct pv_ctx {
     std::string err;
     int32_t *d_status = nullptr;      // first device-detected error (0 = none)
     int opt_selector = 0, opt_walk = 0;
-    int opt_selector_dedupe = 0;      // 1: identical selectors evaluated once (2: with weak hashes, for tests)
+    int opt_selector_dedupe = 0;
+    int opt_sched_kernel = 0;         // path scheduler kernel: 0 automatic, 1-2 forced (tests)      // 1: identical selectors evaluated once (2: with weak hashes, for tests)
     int opt_walk_lane_max = 96;
     int opt_walk_cycles = 0;
     int opt_walk_tail_hop = -1;       // hops from here on run in one tail launch (0: never, -1: by the tables)

@@ -80,9 +80,10 @@ def _closed_loop(v, net, req, pol, rules, rsw, o_ln, o_st):
     assert (h == ((1 << nm) - 1)).all()
 
 
+@pytest.mark.parametrize("kernel", [0, 1, 2])   # automatic; links from global memory; staged
 @pytest.mark.parametrize("seed,weighted,with_pol,max_len", [(0, False, False, 64), (1, True, True, 64),
                                                               (2, True, True, 10), (3, False, True, 255)])
-def test_random_schedules_and_closed_loop(validator, seed, weighted, with_pol, max_len):
+def test_random_schedules_and_closed_loop(validator, seed, weighted, with_pol, max_len, kernel):
     e = W.end_to_end(seed=80 + seed, num_switches=90, num_intents=4, probes_per_intent=4, rules_per_switch=120)
     net = e.network
     pol = W.path_policies(seed, net, 60, forbid_max=3, must_max=3, hubs=12) if with_pol else None
@@ -90,7 +91,11 @@ def test_random_schedules_and_closed_loop(validator, seed, weighted, with_pol, m
     weights = None
     if weighted:
         weights = W.Stream(seed, "gpu-weights").ints(0, 30, int(net.port_offs[-1])).astype(np.uint16)
-    d_req, rules, rsw, o_ln, o_st = _run(validator, net, req, pol, weights, max_len)
+    validator.set_option(B.PV_OPT_SCHED_KERNEL, kernel)
+    try:
+        d_req, rules, rsw, o_ln, o_st = _run(validator, net, req, pol, weights, max_len)
+    finally:
+        validator.set_option(B.PV_OPT_SCHED_KERNEL, 0)
     assert (o_st == W.PATH_OK).sum() > 50
     _closed_loop(validator, net, req, pol, rules, rsw, o_ln, o_st)
 
