@@ -279,7 +279,7 @@ __device__ uint32_t block_exclusive_scan(uint32_t *v, uint32_t n, uint32_t *s_wa
 }
 
 // Pass 1 (kFill = false) writes sizes[s] = {n_items, n_segs, n_bnd}; pass 2
-// writes the blob at blob_offs[s].  One 1024-thread block per switch.
+// writes the blob at blob_offs[s].  One kIndexThreads-thread block per switch.
 template <bool kFill>
 __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32_t *__restrict__ rule_offs,
                                                            const uint32_t *__restrict__ tab_offs,
@@ -709,11 +709,14 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
 // constraint, so a pair is listed or judged as a whole: flow_groups_kernel
 // adds each listed pair's probe count to its source switch (the first hop's
 // per-switch counts) and keeps the pair's offset within that switch; after
-// the scan, walk_init_direct_kernel binds every probe and writes it straight
-// to its slot in the switch-sorted list (switch start + pair offset + rank
-// within the pair), so the first hop needs no regroup.  Probe i belongs to
-// group i / ppg and pod (i mod ppg) mod pods; the caller guarantees one path
-// constraint per group.
+// the scan, the walk's first kernel binds every probe and writes its walk
+// record and list entry straight to its slot in the switch-sorted list
+// (switch start + pair offset + rank within the pair), so the first hop
+// needs no regroup.  walk_init_group_kernel (below) does so one group per
+// block with each pair's run in bucket order; walk_init_direct_kernel is the
+// grid-stride form for groups too large for its shared memory.  Probe i
+// belongs to group i / ppg and pod (i mod ppg) mod pods; the caller
+// guarantees one path constraint per group.
 template <bool kPolicy>
 __device__ __forceinline__ bool first_switch_permitted(const PolicyArgs &pa, uint32_t k, uint32_t s, uint32_t reg,
                                                        uint32_t mask) {
