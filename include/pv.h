@@ -506,7 +506,8 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  *   and the context stays usable.  Never set it outside a test.
  * pv_get_stat: PV_STAT_SELECTOR_ROWS_BUILT (1 if value rows exist),
  *   PV_STAT_SCRATCH_BYTES, PV_STAT_WALK_INDEX_FITS (1 if kernel 2 is
- *   usable), PV_STAT_WALK_INDEX_BYTES (largest per-switch table + index),
+ *   usable), PV_STAT_WALK_INDEX_BYTES (largest shared-memory
+ *   stage of an indexed table: header, plain rules and index),
  *   PV_STAT_WALK_LIVE_TOTAL (probe-hop entries the last pv_verify_probes
  *   processed: the sum over its hops of the probes still walking; reading it
  *   synchronises with the device), PV_STAT_REACH_COMPONENTS (1 if the last

@@ -167,15 +167,21 @@ __global__ void __launch_bounds__(1024) compile_tables_kernel(const uint32_t *__
 // load: first-match index
 // ---------------------------------------------------------------------------
 // A switch's blob (sections 16-byte aligned):
-//   header   uint4 {npad, n_items, n_segs, n_bnd}
-//   A[npad] uint4, B[npad] uint2     rules in first-match order (as above)
+//   header   uint4 {npad | n_plain << 16, n_items, n_segs, n_bnd}
+//   A[n_plain] uint4, B[n_plain] uint2   the plain rules (those not in a
+//                                    segment, the only ones items name), in
+//                                    first-match order (records as above)
 //   boff[kBuckets + 1] u32           item range of each destination-port bucket
-//   items[n_items] u16               per bucket, in first-match order: a rule
-//                                    position, or kSegItem | segment id
+//   items[n_items] u16               per bucket, in first-match order: a plain
+//                                    rule's position, or kSegItem | segment id
 //   segs[n_segs] uint2               {first boundary, number of boundaries}
 //   bnd[n_bnd] u32, win[n_bnd] u32   per segment: ascending elementary-interval
 //                                    starts (the first is 0) and the interval's
 //                                    winner (kWinFound | action, or 0 = none)
+//   A[npad] uint4, B[npad] uint2     all rules in first-match order, padded to a
+//                                    multiple of 32 (linear scan, statistics)
+// The indexed kernel stages everything before the full rule list; the
+// linear kernel stages the header and the full rule list.
 // Exactness.  A header whose dport lies in bucket k can only match rules whose
 // port range meets bucket k; bucket k's list keeps the first-match order, so
 // its first hit is the first match of the whole table.  A segment is a run of
@@ -200,6 +206,8 @@ static_assert(kIndexThreads / 32 == 16, "bucket fill counts are laid out for 16 
 // rule classes, segment bounds, one segment's prefixes and actions, and the
 // bucket fill's per-warp counts and cursors.
 constexpr uint32_t kIndexWarps = 512 / 32;
+static_assert(PV_MAX_RULES * 4 <= kMaxSegment * 10, "plain-rule ranks overlay one segment's staging area");
+static_assert(PV_MAX_RULES < kSegItem, "plain-rule positions fit an item below the segment flag");
 struct IndexSmem {
     uint32_t sort_cap, key_cap, rules_cap, segs_cap, seg_cap;
     size_t bytes;
@@ -224,18 +232,27 @@ struct IndexSmem {
 __host__ __device__ inline uint32_t up16(uint32_t b) { return (b + 15u) & ~15u; }
 
 struct BlobLayout {
-    uint32_t a, b, boff, items, segs, bnd, win, total;
-    __host__ __device__ BlobLayout(uint32_t npad, uint32_t n_items, uint32_t n_segs, uint32_t n_bnd) {
+    uint32_t a, b, boff, items, segs, bnd, win, fa, fb, total;
+    __host__ __device__ BlobLayout(uint32_t npad, uint32_t n_plain, uint32_t n_items, uint32_t n_segs,
+                                   uint32_t n_bnd) {
         a = 16;
-        b = a + npad * 16;
-        boff = b + npad * 8;
+        b = a + up16(n_plain * 16);
+        boff = b + up16(n_plain * 8);
         items = boff + up16((kBuckets + 1) * 4);
         segs = items + up16(n_items * 2);
         bnd = segs + up16(n_segs * 8);
         win = bnd + up16(n_bnd * 4);
-        total = win + up16(n_bnd * 4);
+        fa = win + up16(n_bnd * 4);
+        fb = fa + npad * 16;
+        total = fb + npad * 8;
     }
+    __host__ __device__ explicit BlobLayout(uint4 hdr)
+        : BlobLayout(hdr.x & 0xFFFFu, hdr.x >> 16, hdr.y, hdr.z, hdr.w) {}
 };
+
+// Rules as the linear kernel stages them: the header, then all rules' A and B
+// records from the blob's end.
+__host__ __device__ inline uint32_t linear_bytes(uint32_t npad) { return 16 + npad * 24; }
 
 __device__ __forceinline__ bool rule_dst_only(uint4 a, uint2 b) {
     return a.y == 0 && b.x == 0xFFFF0000u && ((b.y >> 8) & 0xFFu) == 0;
@@ -278,8 +295,8 @@ __device__ uint32_t block_exclusive_scan(uint32_t *v, uint32_t n, uint32_t *s_wa
     return total;
 }
 
-// Pass 1 (kFill = false) writes sizes[s] = {n_items, n_segs, n_bnd}; pass 2
-// writes the blob at blob_offs[s].  One kIndexThreads-thread block per switch.
+// Pass 1 (kFill = false) writes sizes[4s..4s+3] = {n_items, n_segs, n_bnd,
+// n_plain}; pass 2 writes the blob at blob_offs[s].  One kIndexThreads-thread block per switch.
 template <bool kFill>
 __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32_t *__restrict__ rule_offs,
                                                            const uint32_t *__restrict__ tab_offs,
@@ -360,11 +377,25 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
         s_cls[i] = r1 - r0 < kMinSegment ? (int16_t)-1 : (int16_t)(s_pos[lo] + (i - r0) / kMaxSegment);
     }
     __syncthreads();
+    // plain rules (not in a segment) and their positions among themselves;
+    // the ranks sit in the segment staging area (s_rules and s_act, free
+    // until step 3: seg_cap * 10 bytes hold n words for n <= PV_MAX_RULES)
+    uint32_t *s_plain = reinterpret_cast<uint32_t *>(s_rules);   // [n]
+    for (uint32_t i = t; i < n; i += nt) s_plain[i] = s_cls[i] < 0 ? 1u : 0u;
+    __syncthreads();
+    const uint32_t n_plain = block_exclusive_scan(s_plain, n, s_warp);
     uint8_t *out = nullptr;
-    BlobLayout L(npad, 0, 0, 0);
+    BlobLayout L(npad, n_plain, 0, 0, 0);
     if (kFill) {
         out = blob + blob_offs[s];
-        L = BlobLayout(npad, sizes[3 * s], sizes[3 * s + 1], sizes[3 * s + 2]);
+        L = BlobLayout(npad, n_plain, sizes[4 * s], sizes[4 * s + 1], sizes[4 * s + 2]);
+        uint4 *ca = reinterpret_cast<uint4 *>(out + L.a);
+        uint2 *cb = reinterpret_cast<uint2 *>(out + L.b);
+        for (uint32_t i = t; i < n; i += nt)
+            if (s_cls[i] < 0) {
+                ca[s_plain[i]] = a[i];
+                cb[s_plain[i]] = b[i];
+            }
     }
 
     // 2. bucket lists.  Rule i puts one item into each bucket its port range
@@ -432,7 +463,7 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
                 uint32_t pos = s_cur[k] + rank;
                 for (uint32_t w = 0; w < warp; ++w) pos += s_wcnt[w * kBuckets + k];
                 const int c = s_cls[i];
-                items[pos] = (uint16_t)(c >= 0 ? (kSegItem | (uint32_t)c) : i);
+                items[pos] = (uint16_t)(c >= 0 ? (kSegItem | (uint32_t)c) : s_plain[i]);
             }
             __syncthreads();
             if (on && leader) {
@@ -556,19 +587,20 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
         __syncthreads();
     }
 
-    // 4. header and rules
+    // 4. header and the full rule list
     if (kFill) {
-        if (t == 0) *reinterpret_cast<uint4 *>(out) = make_uint4(npad, n_items, nsegs, n_bnd);
-        uint4 *oa = reinterpret_cast<uint4 *>(out + L.a);
-        uint2 *ob = reinterpret_cast<uint2 *>(out + L.b);
+        if (t == 0) *reinterpret_cast<uint4 *>(out) = make_uint4(npad | n_plain << 16, n_items, nsegs, n_bnd);
+        uint4 *oa = reinterpret_cast<uint4 *>(out + L.fa);
+        uint2 *ob = reinterpret_cast<uint2 *>(out + L.fb);
         for (uint32_t i = t; i < npad; i += nt) {
             oa[i] = a[i];
             ob[i] = b[i];
         }
     } else if (t == 0) {
-        sizes[3 * s] = n_items;
-        sizes[3 * s + 1] = nsegs;
-        sizes[3 * s + 2] = n_bnd;
+        sizes[4 * s] = n_items;
+        sizes[4 * s + 1] = nsegs;
+        sizes[4 * s + 2] = n_bnd;
+        sizes[4 * s + 3] = n_plain;
     }
 }
 
@@ -1103,9 +1135,8 @@ template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_linear(const uint8_t *sm, uint32_t npad, uint32_t lane, uint32_t src,
                                                        uint32_t dst, uint32_t dport, uint32_t in_port,
                                                        uint32_t &tests) {
-    const BlobLayout L(npad, 0, 0, 0);
-    const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
-    const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
+    const uint4 *sA = reinterpret_cast<const uint4 *>(sm + 16);               // staged by the linear kernel
+    const uint2 *sB = reinterpret_cast<const uint2 *>(sm + 16 + npad * 16);
     for (uint32_t base = 0; base < npad; base += 32) {
         const uint4 a = sA[base + lane];
         const uint2 b = sB[base + lane];
@@ -1141,7 +1172,7 @@ template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_indexed(const uint8_t *sm, const uint4 hdr, uint32_t lane,
                                                         uint32_t src, uint32_t dst, uint32_t dport, uint32_t in_port,
                                                         uint32_t &tests, uint32_t &lookups) {
-    const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
+    const BlobLayout L(hdr);
     const uint4 *sA = reinterpret_cast<const uint4 *>(sm + L.a);
     const uint2 *sB = reinterpret_cast<const uint2 *>(sm + L.b);
     const uint32_t *boff = reinterpret_cast<const uint32_t *>(sm + L.boff);
@@ -1326,13 +1357,19 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
         const uint32_t seg_end = min(r1, g.seg[s + 1]);
         const uint8_t *src_blob = g.blob + g.blob_offs[s];
         const uint4 hdr = __ldg(reinterpret_cast<const uint4 *>(src_blob));
-        const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
-        const uint32_t bytes = kIndexed ? L.total : L.boff;   // header + rules (+ index)
+        const BlobLayout L(hdr);
+        const uint32_t npad = hdr.x & 0xFFFFu;
         __syncthreads();   // everyone is done with the previous table
         if (threadIdx.x == 0) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            mbar_arrive_expect_tx(&s_bar, bytes + g.wait_extra);
-            bulk_g2s_keep(s_raw, src_blob, bytes, &s_bar);
+            if (kIndexed) {   // header, plain rules, index
+                mbar_arrive_expect_tx(&s_bar, L.fa + g.wait_extra);
+                bulk_g2s_keep(s_raw, src_blob, L.fa, &s_bar);
+            } else {          // header and the full rule list
+                mbar_arrive_expect_tx(&s_bar, linear_bytes(npad) + g.wait_extra);
+                bulk_g2s_keep(s_raw, src_blob, 16, &s_bar);
+                if (npad) bulk_g2s_keep(s_raw + 16, src_blob + L.fa, npad * 24, &s_bar);
+            }
         }
         const bool ok = mbar_wait_bounded(&s_bar, parity, g.wait_ns);
         if (__syncthreads_or(!ok)) {
@@ -1392,7 +1429,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                     uint32_t tests = 0, lookups = 0;
                     const uint32_t fm =
                         kIndexed ? first_match_indexed<kStats>(s_raw, hdr, lane, src, dst, dport, in_port, tests, lookups)
-                                 : first_match_linear<kStats>(s_raw, hdr.x, lane, src, dst, dport, in_port, tests);
+                                 : first_match_linear<kStats>(s_raw, npad, lane, src, dst, dport, in_port, tests);
                     uint32_t status, next;
                     hop_outcome(g, g.hop, fm, dst, mask, pbase, nports, &status, &next);
                     if (lane == j) {
@@ -1408,9 +1445,11 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             }
             if (kStats && lane < cnt && !fin_now) {
                 uint32_t depth = 0;
-                const uint32_t ref = scan_first_match(reinterpret_cast<const uint4 *>(s_raw + L.a),
-                                                      reinterpret_cast<const uint2 *>(s_raw + L.b), hdr.x, pr.x,
-                                                      pr.y, pr.z & 0xFFFFu, e.y & 0xFFu, &depth);
+                // the full rule list: staged by the linear kernel, read from
+                // the blob by the indexed one
+                const uint4 *fa = reinterpret_cast<const uint4 *>(kIndexed ? src_blob + L.fa : s_raw + 16);
+                const uint2 *fb = reinterpret_cast<const uint2 *>(kIndexed ? src_blob + L.fb : s_raw + 16 + npad * 16);
+                const uint32_t ref = scan_first_match(fa, fb, npad, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu, &depth);
                 ++stc[kStFirstMatches];
                 stc[kStLinearDepth] += depth;
                 stc[kStMismatch] += ref != my_fm ? 1u : 0u;
@@ -1543,14 +1582,14 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                 }
                 const uint8_t *blob = g.blob + g.blob_offs[s];
                 const uint4 hdr = __ldg(reinterpret_cast<const uint4 *>(blob));
-                const BlobLayout L(hdr.x, hdr.y, hdr.z, hdr.w);
+                const BlobLayout L(hdr);
                 const uint32_t fm = first_match_thread<kStats>(blob, L, pr.x, pr.y, pr.z & 0xFFFFu, in_port,
                                                                stc[kStRuleTests], stc[kStLookups]);
                 if (kStats) {
                     uint32_t depth = 0;
-                    const uint32_t ref = scan_first_match(reinterpret_cast<const uint4 *>(blob + L.a),
-                                                          reinterpret_cast<const uint2 *>(blob + L.b), hdr.x, pr.x,
-                                                          pr.y, pr.z & 0xFFFFu, in_port, &depth);
+                    const uint32_t ref = scan_first_match(reinterpret_cast<const uint4 *>(blob + L.fa),
+                                                          reinterpret_cast<const uint2 *>(blob + L.fb),
+                                                          hdr.x & 0xFFFFu, pr.x, pr.y, pr.z & 0xFFFFu, in_port, &depth);
                     ++stc[kStFirstMatches];
                     stc[kStLinearDepth] += depth;
                     stc[kStMismatch] += ref != fm ? 1u : 0u;
@@ -1660,7 +1699,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     if ((rc = pv_pool_alloc(ctx, (void **)&d_tab_offs, (S + 1) * 4, "table offsets")) ||
         (rc = pv_pool_alloc(ctx, (void **)&d_rule_a, (size_t)T * 16, "rules A")) ||
         (rc = pv_pool_alloc(ctx, (void **)&d_rule_b, (size_t)T * 8, "rules B")) ||
-        (rc = pv_pool_alloc(ctx, (void **)&d_sizes, (size_t)S * 12 + 4, "index sizes")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&d_sizes, (size_t)S * 16 + 4, "index sizes")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_blob_offs, ((size_t)S + 1) * 8, "blob offsets")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_region, S, "regions")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_port_offs, (S + 1) * 4, "port offsets")) ||
@@ -1736,7 +1775,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     if (e == cudaSuccess) {
         uint32_t npow = 1;
         while (npow < maxn) npow <<= 1;
-        uint32_t *d_bad = d_sizes + (size_t)S * 3;   // lowest invalid rule index
+        uint32_t *d_bad = d_sizes + (size_t)S * 4;   // lowest invalid rule index
         e = cudaMemsetAsync(d_bad, 0xFF, 4, ls);
         if (e == cudaSuccess) {
             compile_tables_kernel<<<S, 1024, npow * 4, ls>>>(d_rule_offs, t.d_raw, t.d_port_offs, d_tab_offs,
@@ -1756,12 +1795,12 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
         }
     }
     // blob layout from the index sizes (and the device-side rule validation)
-    std::vector<uint32_t> sizes((size_t)S * 3 + 1);
+    std::vector<uint32_t> sizes((size_t)S * 4 + 1);
     std::vector<uint64_t> boffs(S + 1, 0);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(sizes.data(), d_sizes, (size_t)S * 12 + 4, cudaMemcpyDeviceToHost, ls);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(sizes.data(), d_sizes, (size_t)S * 16 + 4, cudaMemcpyDeviceToHost, ls);
     if (e == cudaSuccess) e = cudaStreamSynchronize(ls);
-    if (e == cudaSuccess && sizes[(size_t)S * 3] != 0xFFFFFFFFu) {
-        const uint32_t i = sizes[(size_t)S * 3];
+    if (e == cudaSuccess && sizes[(size_t)S * 4] != 0xFFFFFFFFu) {
+        const uint32_t i = sizes[(size_t)S * 4];
         const uint32_t s = (uint32_t)(std::upper_bound(rule_offs, rule_offs + S + 1, i) - rule_offs) - 1;
         const pv_rule &r = rules[i];
         free_temps();
@@ -1777,11 +1816,11 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     if (e == cudaSuccess) {
         for (uint32_t s = 0; s < S; ++s) {
             const uint32_t npad = tab[s + 1] - tab[s];
-            all_items += sizes[3 * s];
-            const BlobLayout L(npad, sizes[3 * s], sizes[3 * s + 1], sizes[3 * s + 2]);
+            all_items += sizes[4 * s];
+            const BlobLayout L(npad, sizes[4 * s + 3], sizes[4 * s], sizes[4 * s + 1], sizes[4 * s + 2]);
             boffs[s + 1] = boffs[s] + L.total;
-            max_blob = std::max(max_blob, L.total);
-            max_linear = std::max(max_linear, L.boff);
+            max_blob = std::max(max_blob, L.fa);             // staged by the indexed kernel
+            max_linear = std::max(max_linear, linear_bytes(npad));
         }
         e = cudaMemcpyAsync(t.d_blob_offs, boffs.data(), ((size_t)S + 1) * 8, cudaMemcpyHostToDevice, ls);
     }

@@ -33,13 +33,13 @@ struct pv_table_state {
     bool loaded = false;
     uint32_t num_switches = 0, num_hosts = 0;
     uint32_t max_rules_padded = 0;    // largest per-switch table, in rules (multiple of 32)
-    // One blob per switch (16-byte aligned): header, compiled rules in first-
-    // match order, then the first-match index (see k_walk.cu).
+    // One blob per switch (16-byte aligned): header, the plain rules, the
+    // first-match index, then every rule in first-match order (see k_walk.cu).
     uint8_t *d_blob = nullptr;
     uint64_t *d_blob_offs = nullptr;  // [S + 1] byte offsets
-    uint32_t max_blob_bytes = 0;      // largest blob (indexed kernel stages it whole)
+    uint32_t max_blob_bytes = 0;      // largest stage of the indexed kernel (all but the full rule list)
     uint32_t tail_hop = 8;            // default first tail hop for these tables (see walk_probes)
-    uint32_t max_linear_bytes = 0;    // largest header + rules prefix (linear-scan kernel)
+    uint32_t max_linear_bytes = 0;    // largest header + full rule list (linear-scan kernel)
     bool index_fits = false;          // every blob fits shared memory
     uint8_t *d_region = nullptr;      // [S]
     uint32_t *d_port_offs = nullptr;  // [S + 1]
