@@ -239,7 +239,6 @@ class EndToEndBench:
         self.copy_stream = torch.cuda.Stream()
         self.chunks = chunks
         self.loads_first = getattr(self, "loads_first", True)
-        self.load_split = getattr(self, "load_split", 0.5)
         net = e.network
         self.h2d = (sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "masks", "flows"))
                     + e.cluster.labels.nbytes + net.rule_offs.nbytes + net.rules.nbytes + net.switch_region.nbytes
@@ -250,18 +249,20 @@ class EndToEndBench:
     def step_e2e(self, v, stream):
         """Every input from host memory: intents (selectors, placement draws,
         masks) and their flows copied (8 B per flow), the cluster labels and
-        flow tables loaded meanwhile, verification of `chunks` intent ranges
-        as their flows arrive, verdicts and counters copied back."""
+        flow tables loaded meanwhile (the table load in two halves around
+        the queued uploads), verification of `chunks` intent ranges as their
+        flows arrive, verdicts and counters copied back."""
         e = self.e
 
         def loads():
             v.load_cluster(e.cluster)
-            v.load_network(e.network)
-            if self.pol is not None:
+            if self.pol is not None:   # checked against the installed tables: the same network every step
                 v.load_policies(self.pol)
+            v.begin_network(e.network)
+            return v.finish_network
 
         v.run_end_to_end_from_host(self.host, self.dev, self.sizes, stream, self.copy_stream, self.chunks, loads,
-                                   self.loads_first, self.load_split)
+                                   self.loads_first)
 
     def e2e_phases(self, v, stream, reps=3):
         """Each part of the host-buffer step alone (diagnostic, after the
@@ -816,7 +817,6 @@ def run_ours(args):
     e2e = None
     if hasattr(wl, "setup_e2e"):
         wl.loads_first = args.e2e_loads_first
-        wl.load_split = args.e2e_load_split
         wl.setup_e2e(v, args.e2e_chunks)
         for _ in range(max(args.warmup, 1)):
             wl.step_e2e(v, stream)
@@ -829,7 +829,8 @@ def run_ours(args):
         e_s = SH.max_over_ranks(e_s, dist, "cuda")
         e2e = {"value": units * world / e_s, "unit": wl.unit, "h2d_bytes_per_step": int(wl.h2d),
                "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3, "upload_chunks": args.e2e_chunks,
-               "loads": "before the uploads" if args.e2e_loads_first else "after the uploads are queued"}
+               "loads": ("before the uploads" if args.e2e_loads_first
+                         else "uploads of the tables queued first, the rest of the load while the inputs arrive")}
         if hasattr(wl, "e2e_phases"):
             e2e["phases"] = wl.e2e_phases(v, stream)
 
@@ -869,9 +870,8 @@ def main():
     ap.add_argument("--e2e-chunks", type=int, default=1,
                     help="intent ranges whose probe upload overlaps verification in the host-buffer step")
     ap.add_argument("--e2e-loads-first", action="store_true",
-                    help="host-buffer step: run the table loads before queueing the input uploads (default: after)")
-    ap.add_argument("--e2e-load-split", type=float, default=0.5,
-                    help="host-buffer step: fraction of the flow upload queued before the table loads")
+                    help="host-buffer step: finish the table loads before queueing the input uploads "
+                         "(default: the second half of the table load runs while the inputs arrive)")
     ap.add_argument("--intents", type=int, default=None,
                     help="end-to-end only: fewer intents (a smaller case for profiling, not a bench line)")
     args = ap.parse_args()

@@ -236,6 +236,31 @@ int pv_load_flow_tables(pv_ctx *ctx, uint32_t num_switches, const uint32_t *rule
                         const uint32_t *host_ip);
 
 /* ---------------------------------------------------------------------------
+ * pv_load_flow_tables_begin / pv_load_flow_tables_end -- pv_load_flow_tables
+ * in two halves, so that a caller can queue its own transfers between them.
+ * begin takes the same arguments and does the host checks (the same errors),
+ * queues every upload of the tables and the first device passes on the
+ * context's load stream, and returns without waiting for the device.  end
+ * waits for those passes, reports the device-side rule errors (PV_EINVAL,
+ * as pv_load_flow_tables), builds the index and installs the tables.
+ * Between the two:
+ *   - every host array given to begin stays allocated and unchanged (end
+ *     reads them again);
+ *   - evaluation calls keep using the tables installed before begin, and
+ *     the other loads work as usual;
+ *   - a second begin, pv_load_flow_tables or pv_install_path_rules (which
+ *     loads tables) fails with PV_ESTATE.
+ * end without a begin fails with PV_ESTATE.  If begin fails nothing is in
+ * progress; if end fails the previous tables stay installed.  pv_destroy
+ * frees a load that was begun and not ended.
+ * ------------------------------------------------------------------------- */
+int pv_load_flow_tables_begin(pv_ctx *ctx, uint32_t num_switches, const uint32_t *rule_offs, const pv_rule *rules,
+                              const uint8_t *switch_region, const uint32_t *port_offs, const int32_t *port_peer,
+                              uint32_t num_hosts, const uint16_t *host_switch, const uint16_t *host_port,
+                              const uint32_t *host_ip);
+int pv_load_flow_tables_end(pv_ctx *ctx);
+
+/* ---------------------------------------------------------------------------
  * pv_verify_probes -- routing constraints Phi_N on the realised paths
  * (Sec. 3.3 satisfaction (ii): "for all v on the path"; Sec. 5.5 network
  * check; Sec. 6.3 item 4: transit switches are checked hop by hop).

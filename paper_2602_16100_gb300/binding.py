@@ -35,7 +35,8 @@ SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", 
            "pv_profile_enable", "pv_profile_collect", "pv_profile_read", "pv_compliant_reach_noalloc",
            "pv_load_path_policies", "pv_verify_probes_constrained", "pv_aggregate_constrained",
            "pv_eval_selector_terms", "pv_schedule_paths", "pv_compile_path_rules", "pv_install_path_rules",
-           "pv_bind_flows", "pv_verify_flows", "pv_verify_flows_constrained")
+           "pv_bind_flows", "pv_verify_flows", "pv_verify_flows_constrained", "pv_load_flow_tables_begin",
+           "pv_load_flow_tables_end")
 
 #: kernel groups timed by the library profiler (PV_K_* in include/pv.h)
 PV_K_NAMES = ("selector", "place", "bind", "walk_init", "walk_regroup", "walk_hop", "aggregate", "reach", "schedule")
@@ -72,6 +73,8 @@ def load_library(path: Optional[str] = None):
         "pv_load_cluster": (ctypes.c_int, [vp, u32, u32, vp]),
         "pv_eval_selectors": (ctypes.c_int, [vp, u32, vp, u32, vp, vp, vp, u32, vp, vp]),
         "pv_load_flow_tables": (ctypes.c_int, [vp, u32, vp, vp, vp, vp, vp, u32, vp, vp, vp]),
+        "pv_load_flow_tables_begin": (ctypes.c_int, [vp, u32, vp, vp, vp, vp, vp, u32, vp, vp, vp]),
+        "pv_load_flow_tables_end": (ctypes.c_int, [vp]),
         "pv_verify_probes": (ctypes.c_int, [vp, u32, vp, u32, vp, vp]),
         "pv_compliant_reach": (ctypes.c_int, [vp, u32, vp, u32, vp, vp, u32, vp, u32, vp, vp, u32, vp]),
         "pv_place_pods": (ctypes.c_int, [vp, u32, u32, vp, u32, vp, vp, vp]),
@@ -163,6 +166,7 @@ def pv_create(cuda_device: int = 0):
 
 def pv_destroy(ctx) -> None:
     load_library().pv_destroy(ctx)
+    _TABLE_LOADS.pop(ctx.value, None)
 
 
 def pv_last_error(ctx) -> str:
@@ -211,15 +215,40 @@ def pv_eval_selectors(ctx, num_pods, d_expr_offs, num_exprs, d_exprs, d_assign, 
                                                         _stream(stream)))
 
 
+def _table_arrays(rule_offs, rules, switch_region, port_offs, port_peer, host_switch, host_port, host_ip):
+    return [np.ascontiguousarray(rule_offs, np.uint32), np.ascontiguousarray(rules),
+            np.ascontiguousarray(switch_region, np.uint8), np.ascontiguousarray(port_offs, np.uint32),
+            np.ascontiguousarray(port_peer, np.int32), np.ascontiguousarray(host_switch, np.uint16),
+            np.ascontiguousarray(host_port, np.uint16), np.ascontiguousarray(host_ip, np.uint32)]
+
+
 def pv_load_flow_tables(ctx, num_switches, rule_offs, rules, switch_region, port_offs, port_peer, num_hosts,
                         host_switch, host_port, host_ip) -> int:
-    a = [np.ascontiguousarray(rule_offs, np.uint32), np.ascontiguousarray(rules),
-         np.ascontiguousarray(switch_region, np.uint8), np.ascontiguousarray(port_offs, np.uint32),
-         np.ascontiguousarray(port_peer, np.int32), np.ascontiguousarray(host_switch, np.uint16),
-         np.ascontiguousarray(host_port, np.uint16), np.ascontiguousarray(host_ip, np.uint32)]
+    a = _table_arrays(rule_offs, rules, switch_region, port_offs, port_peer, host_switch, host_port, host_ip)
     return _check(ctx, load_library().pv_load_flow_tables(ctx, num_switches, _host(a[0]), _host(a[1]), _host(a[2]),
                                                           _host(a[3]), _host(a[4]), num_hosts, _host(a[5]),
                                                           _host(a[6]), _host(a[7])))
+
+
+#: host arrays of a two-part table load, kept alive until its end (by context)
+_TABLE_LOADS = {}
+
+
+def pv_load_flow_tables_begin(ctx, num_switches, rule_offs, rules, switch_region, port_offs, port_peer, num_hosts,
+                              host_switch, host_port, host_ip) -> int:
+    a = _table_arrays(rule_offs, rules, switch_region, port_offs, port_peer, host_switch, host_port, host_ip)
+    rc = _check(ctx, load_library().pv_load_flow_tables_begin(ctx, num_switches, _host(a[0]), _host(a[1]),
+                                                              _host(a[2]), _host(a[3]), _host(a[4]), num_hosts,
+                                                              _host(a[5]), _host(a[6]), _host(a[7])))
+    _TABLE_LOADS[ctx.value] = a
+    return rc
+
+
+def pv_load_flow_tables_end(ctx) -> int:
+    try:
+        return _check(ctx, load_library().pv_load_flow_tables_end(ctx))
+    finally:
+        _TABLE_LOADS.pop(ctx.value, None)
 
 
 def pv_verify_probes(ctx, num_probes, d_probes, hop_cap, d_out, stream=None) -> int:

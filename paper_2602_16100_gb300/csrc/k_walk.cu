@@ -54,15 +54,9 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
                  : "memory");
 }
-__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-            smem_u32(dst)),
-        "l"(src), "r"(bytes), "r"(smem_u32(bar))
-        : "memory");
-}
-// Same copy, asking L2 to keep the source lines (evict_last): the flow-table
-// blobs are re-read every hop while the probe lists stream through L2.
+// Bulk copy global -> shared completed on an mbarrier, asking L2 to keep the
+// source lines (evict_last): the flow-table blobs are re-read every hop while
+// the probe lists stream through L2.
 __device__ __forceinline__ void bulk_g2s_keep(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
     asm volatile(
         "{\n\t.reg .b64 pol;\n\t"
@@ -1633,21 +1627,59 @@ inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
 }  // namespace
 
-// -----------------------------------------------------------------------------
-// C ABI
-// -----------------------------------------------------------------------------
-extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule_offs, const pv_rule *rules,
-                                   const uint8_t *switch_region, const uint32_t *port_offs,
-                                   const int32_t *port_peer, uint32_t H, const uint16_t *host_switch,
-                                   const uint16_t *host_port, const uint32_t *host_ip) {
+// A flow-table load between its two halves: the first has validated the
+// structure on the host and queued the uploads and the index-size pass; the
+// second reads the sizes back, builds the blobs and installs the tables.
+struct pv_table_load {
+    uint32_t S = 0, H = 0, P = 0, max_pad = 0, max_rules = 0;
+    const uint32_t *rule_offs = nullptr, *port_offs = nullptr, *host_ip = nullptr;
+    const pv_rule *rules = nullptr;
+    const uint8_t *switch_region = nullptr;
+    const int32_t *port_peer = nullptr;
+    const uint16_t *host_switch = nullptr, *host_port = nullptr;
+    std::vector<uint32_t> tab;   // first compiled rule of each switch (tables padded to 32 rules)
+    pv_table_state t;            // the new tables (the loaded ones stay in use until these are complete)
+    uint32_t *d_rule_offs = nullptr, *d_tab_offs = nullptr, *d_sizes = nullptr;
+    uint4 *d_rule_a = nullptr;
+    uint2 *d_rule_b = nullptr;
+    void free_temps(pv_ctx *ctx) {
+        pv_pool_free(ctx, d_rule_offs);
+        pv_pool_free(ctx, d_tab_offs);
+        pv_pool_free(ctx, d_rule_a);
+        pv_pool_free(ctx, d_rule_b);
+        pv_pool_free(ctx, d_sizes);
+        d_rule_offs = d_tab_offs = d_sizes = nullptr;
+        d_rule_a = nullptr;
+        d_rule_b = nullptr;
+    }
+};
+
+void pv_discard_table_load(pv_ctx *ctx) {
+    if (!ctx->table_load) return;
+    ctx->table_load->free_temps(ctx);
+    pv_free_tables(ctx, ctx->table_load->t);
+    delete ctx->table_load;
+    ctx->table_load = nullptr;
+}
+
+namespace {
+
+// First half: host validation of the structure, every upload, rule
+// compilation and the index-size pass, all queued on the load stream; the
+// host does not wait for the device.
+int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule_offs, const pv_rule *rules,
+                 const uint8_t *switch_region, const uint32_t *port_offs, const int32_t *port_peer,
+                 uint32_t H, const uint16_t *host_switch, const uint16_t *host_port, const uint32_t *host_ip) {
     if (!ctx) return PV_EINVAL;
     if (S == 0 || S > PV_MAX_SWITCHES) return pv_fail(ctx, PV_EINVAL, "num_switches must be 1..%d", PV_MAX_SWITCHES);
     if (H > PV_MAX_HOSTS) return pv_fail(ctx, PV_EINVAL, "num_hosts must be <= %d", PV_MAX_HOSTS);
     if (!rule_offs || !switch_region || !port_offs || (H && (!host_switch || !host_port || !host_ip)))
         return pv_fail(ctx, PV_EINVAL, "pv_load_flow_tables: NULL host pointer");
     if (rule_offs[0] != 0 || port_offs[0] != 0) return pv_fail(ctx, PV_EINVAL, "offsets must start at 0");
-    std::vector<uint32_t> tab(S + 1, 0);
-    uint32_t max_pad = 0;
+    std::vector<uint32_t> &tab = L.tab;
+    tab.assign(S + 1, 0);
+    uint32_t &max_pad = L.max_pad;
+    max_pad = 0;
     for (uint32_t s = 0; s < S; ++s) {
         if (rule_offs[s + 1] < rule_offs[s] || port_offs[s + 1] < port_offs[s])
             return pv_fail(ctx, PV_EINVAL, "offsets not monotone at switch %u", s);
@@ -1683,18 +1715,12 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
 
     if (int rc0 = pv_load_begin(ctx)) return rc0;
     cudaStream_t ls = ctx->load_stream;
-    pv_table_state t;   // the new tables (the loaded ones stay in use until these are complete)
+    pv_table_state &t = L.t;
     const uint32_t T = tab[S];
-    uint32_t *d_rule_offs = nullptr, *d_tab_offs = nullptr, *d_sizes = nullptr;
-    uint4 *d_rule_a = nullptr;
-    uint2 *d_rule_b = nullptr;
-    auto free_temps = [&]() {
-        pv_pool_free(ctx, d_rule_offs);
-        pv_pool_free(ctx, d_tab_offs);
-        pv_pool_free(ctx, d_rule_a);
-        pv_pool_free(ctx, d_rule_b);
-        pv_pool_free(ctx, d_sizes);
-    };
+    uint32_t *&d_rule_offs = L.d_rule_offs, *&d_tab_offs = L.d_tab_offs, *&d_sizes = L.d_sizes;
+    uint4 *&d_rule_a = L.d_rule_a;
+    uint2 *&d_rule_b = L.d_rule_b;
+    auto free_temps = [&]() { L.free_temps(ctx); };
     int rc;
     if ((rc = pv_pool_alloc(ctx, (void **)&d_tab_offs, (S + 1) * 4, "table offsets")) ||
         (rc = pv_pool_alloc(ctx, (void **)&d_rule_a, (size_t)T * 16, "rules A")) ||
@@ -1771,6 +1797,7 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     }
     uint32_t maxn = 0;
     for (uint32_t s = 0; s < S; ++s) maxn = std::max(maxn, rule_offs[s + 1] - rule_offs[s]);
+    L.max_rules = maxn;
     const IndexSmem ism(maxn);
     if (e == cudaSuccess) {
         uint32_t npow = 1;
@@ -1794,6 +1821,49 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
             e = cudaGetLastError();
         }
     }
+    if (e != cudaSuccess) {
+        free_temps();
+        pv_free_tables(ctx, t);
+        return pv_cuda_fail(ctx, e, "pv_load_flow_tables");
+    }
+    L.S = S;
+    L.H = H;
+    L.P = P;
+    L.rule_offs = rule_offs;
+    L.rules = rules;
+    L.switch_region = switch_region;
+    L.port_offs = port_offs;
+    L.port_peer = port_peer;
+    L.host_switch = host_switch;
+    L.host_port = host_port;
+    L.host_ip = host_ip;
+    return PV_OK;
+}
+
+// Second half: waits for the index sizes (and the device-side rule
+// validation), lays out and fills the blobs, installs the tables.
+int tables_end(pv_ctx *ctx, pv_table_load &L) {
+    const uint32_t S = L.S, H = L.H, P = L.P, max_pad = L.max_pad;
+    const uint32_t *rule_offs = L.rule_offs, *port_offs = L.port_offs, *host_ip = L.host_ip;
+    const pv_rule *rules = L.rules;
+    const uint8_t *switch_region = L.switch_region;
+    const int32_t *port_peer = L.port_peer;
+    const uint16_t *host_switch = L.host_switch, *host_port = L.host_port;
+    const std::vector<uint32_t> &tab = L.tab;
+    const IndexSmem ism(L.max_rules);
+    pv_table_state &t = L.t;
+    uint32_t *d_rule_offs = L.d_rule_offs, *d_tab_offs = L.d_tab_offs, *d_sizes = L.d_sizes;
+    uint4 *d_rule_a = L.d_rule_a;
+    uint2 *d_rule_b = L.d_rule_b;
+    auto free_temps = [&]() { L.free_temps(ctx); };
+    if (int rc0 = pv_load_begin(ctx)) {
+        free_temps();
+        pv_free_tables(ctx, t);
+        return rc0;
+    }
+    cudaStream_t ls = ctx->load_stream;
+    cudaError_t e = cudaSuccess;
+    int rc = PV_OK;
     // blob layout from the index sizes (and the device-side rule validation)
     std::vector<uint32_t> sizes((size_t)S * 4 + 1);
     std::vector<uint64_t> boffs(S + 1, 0);
@@ -1873,6 +1943,50 @@ extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule
     pv_retire_end(ctx);
     ctx->tb = t;
     return pv_load_end(ctx);
+}
+
+}  // namespace
+
+// -----------------------------------------------------------------------------
+// C ABI
+// -----------------------------------------------------------------------------
+extern "C" int pv_load_flow_tables(pv_ctx *ctx, uint32_t S, const uint32_t *rule_offs, const pv_rule *rules,
+                                   const uint8_t *switch_region, const uint32_t *port_offs,
+                                   const int32_t *port_peer, uint32_t H, const uint16_t *host_switch,
+                                   const uint16_t *host_port, const uint32_t *host_ip) {
+    if (!ctx) return PV_EINVAL;
+    if (ctx->table_load) return pv_fail(ctx, PV_ESTATE, "pv_load_flow_tables: a two-part table load is in progress");
+    pv_table_load L;
+    if (int rc = tables_begin(ctx, L, S, rule_offs, rules, switch_region, port_offs, port_peer, H, host_switch,
+                              host_port, host_ip))
+        return rc;
+    return tables_end(ctx, L);
+}
+
+extern "C" int pv_load_flow_tables_begin(pv_ctx *ctx, uint32_t S, const uint32_t *rule_offs, const pv_rule *rules,
+                                         const uint8_t *switch_region, const uint32_t *port_offs,
+                                         const int32_t *port_peer, uint32_t H, const uint16_t *host_switch,
+                                         const uint16_t *host_port, const uint32_t *host_ip) {
+    if (!ctx) return PV_EINVAL;
+    if (ctx->table_load) return pv_fail(ctx, PV_ESTATE, "pv_load_flow_tables_begin: a table load is in progress");
+    pv_table_load *L = new pv_table_load;
+    if (int rc = tables_begin(ctx, *L, S, rule_offs, rules, switch_region, port_offs, port_peer, H, host_switch,
+                              host_port, host_ip)) {
+        delete L;
+        return rc;
+    }
+    ctx->table_load = L;
+    return PV_OK;
+}
+
+extern "C" int pv_load_flow_tables_end(pv_ctx *ctx) {
+    if (!ctx) return PV_EINVAL;
+    pv_table_load *L = ctx->table_load;
+    if (!L) return pv_fail(ctx, PV_ESTATE, "pv_load_flow_tables_end: no table load in progress");
+    ctx->table_load = nullptr;
+    const int rc = tables_end(ctx, *L);
+    delete L;
+    return rc;
 }
 
 namespace {

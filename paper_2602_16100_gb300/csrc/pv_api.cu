@@ -271,6 +271,7 @@ extern "C" int pv_create(pv_ctx **out, int cuda_device) {
 extern "C" void pv_destroy(pv_ctx *ctx) {
     if (!ctx) return;
     cudaDeviceSynchronize();
+    pv_discard_table_load(ctx);
     pv_free_cluster(ctx, ctx->cl);
     pv_free_tables(ctx, ctx->tb);
     pv_free_policies(ctx, ctx->pol);

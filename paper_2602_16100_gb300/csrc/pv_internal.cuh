@@ -84,6 +84,8 @@ struct pv_prof_state {
     uint64_t launches[PV_K_COUNT] = {};
 };
 
+struct pv_table_load;   // a two-part flow-table load in progress (k_walk.cu)
+
 struct pv_ctx {
     int device = 0;
     // Loads run on their own stream with memory from the context's pool, so
@@ -106,8 +108,8 @@ struct pv_ctx {
     std::string err;
     int32_t *d_status = nullptr;      // first device-detected error (0 = none)
     int opt_selector = 0, opt_walk = 0;
-    int opt_selector_dedupe = 0;
-    int opt_sched_kernel = 0;         // path scheduler kernel: 0 automatic, 1-2 forced (tests)      // 1: identical selectors evaluated once (2: with weak hashes, for tests)
+    int opt_selector_dedupe = 0;      // 1: identical selectors evaluated once (2: with weak hashes, for tests)
+    int opt_sched_kernel = 0;         // path scheduler kernel: 0 automatic, 1-2 forced (tests)
     int opt_walk_lane_max = 96;
     int opt_walk_cycles = 0;
     int opt_walk_tail_hop = -1;       // hops from here on run in one tail launch (0: never, -1: by the tables)
@@ -124,6 +126,7 @@ struct pv_ctx {
     pv_cluster_state cl;
     pv_table_state tb;
     pv_table_host tbh;
+    pv_table_load *table_load = nullptr;   // between pv_load_flow_tables_begin and _end
     pv_policy_state pol;
 };
 
@@ -193,4 +196,6 @@ inline void pv_free_ptr(pv_ctx *ctx, T *&p) {
 
 void pv_free_cluster(pv_ctx *ctx, pv_cluster_state &c);
 void pv_free_tables(pv_ctx *ctx, pv_table_state &t);
+// Frees a two-part table load that was begun and not ended (pv_destroy).
+void pv_discard_table_load(pv_ctx *ctx);
 void pv_free_policies(pv_ctx *ctx, pv_policy_state &p);

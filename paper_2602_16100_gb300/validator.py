@@ -79,6 +79,20 @@ class Validator:
                               net.host_ip)
         self.num_hosts = net.num_hosts
 
+    def begin_network(self, net: W.Network):
+        """First half of a table load: host checks, the uploads and the first
+        device passes queued; evaluation keeps the installed tables until
+        finish_network installs these."""
+        B.pv_load_flow_tables_begin(self.ctx, net.num_switches, net.rule_offs, net.rules, net.switch_region,
+                                    net.port_offs, net.port_peer, net.num_hosts, net.host_switch, net.host_port,
+                                    net.host_ip)
+        self._pending_hosts = net.num_hosts
+
+    def finish_network(self):
+        """Second half of a table load begun by begin_network."""
+        B.pv_load_flow_tables_end(self.ctx)
+        self.num_hosts = self._pending_hosts
+
     # -- evaluation (device tensors) -----------------------------------------
     def eval_selectors(self, d_offs, num_exprs, d_exprs, d_assign, num_pods, words=None, d_bits=None,
                        d_flags=None, stream=None):
@@ -164,19 +178,20 @@ class Validator:
     _INPUTS = ("offs", "exprs", "draws", "masks", "flows")
 
     def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
-                                 chunks: int = 1, loads=None, loads_first: bool = False,
-                                 load_split: float = 0.5) -> dict:
+                                 chunks: int = 1, loads=None, loads_first: bool = False) -> dict:
         """The end-to-end pipeline on inputs in pinned HOST memory.  Every
         input upload is enqueued on `copy_stream`, the flows cut into
         `chunks` intent ranges (independent units), and range c is verified
         on `stream` as soon as its flows have arrived.  ``loads()``, if given
-        (the cluster and table loads), runs between the first `load_split`
-        of the flow upload and the rest, so its copies wait only for that
-        part and its device work (which the evaluation calls wait for on the
-        device) runs while the rest arrives; with `loads_first` it runs
-        before any upload is queued.  The per-intent verdicts and
-        counters come back into ``host["pass"]`` and ``host["counts"]`` on
-        `stream` (not synchronised).
+        (the cluster and table loads), runs before any upload is queued, so
+        its copies go first on the host-to-device link; if it returns a
+        callable (the second half of a two-part table load, which waits on
+        the host for the load's first device passes), that runs once every
+        upload is queued, while the inputs arrive, or at once with
+        `loads_first`.  The evaluation calls wait for the loads' device work
+        on the device.  The per-intent verdicts and counters come back into
+        ``host["pass"]`` and ``host["counts"]`` on `stream` (not
+        synchronised).
 
         ``host`` holds pinned byte tensors "offs", "exprs", "draws", "masks",
         "flows" (inputs, as alloc_end_to_end lays them out: 8-byte flows, the
@@ -196,8 +211,10 @@ class Validator:
         P = W.PROBE_DTYPE.itemsize
         F = W.FLOW_DTYPE.itemsize
         ranges = [(lo, hi) for lo, hi in zip(edges[:-1], edges[1:]) if hi > lo]
-        if loads is not None and loads_first:
-            loads()
+        finish = loads() if loads is not None else None
+        if callable(finish) and loads_first:
+            finish()
+            finish = None
         if "_inputs" not in dev:   # the second input set, and each set's last reader
             dev["_inputs"] = [{k: dev[k] for k in self._INPUTS},
                               {k: torch.empty_like(dev[k]) for k in self._INPUTS}]
@@ -208,33 +225,21 @@ class Validator:
         read = dev["_read"]
         dev = {**dev, **dev["_inputs"][k_slot]}
         # the kernels that last read this input set must be done with it
-        if read[k_slot] is not None:
-            copy_stream.wait_event(read[k_slot])
         ready = []
-
-        def upload(lo, hi):   # flows of intents [lo, hi)
-            with torch.cuda.stream(copy_stream):
-                dev["flows"][lo * ppg * F:hi * ppg * F].copy_(host["flows"][lo * ppg * F:hi * ppg * F],
-                                                               non_blocking=True)
-
         with torch.cuda.stream(copy_stream):
+            if read[k_slot] is not None:
+                copy_stream.wait_event(read[k_slot])
             for k in ("offs", "exprs", "draws", "masks"):
                 n = host[k].numel()
                 dev[k][:n].copy_(host[k], non_blocking=True)
-        # with loads after the uploads, the loads go between the first
-        # load_split of the flows and the rest: their copies wait for the
-        # first part only, and their kernels run while the rest arrives
-        cut = ranges[0][0] + int((ranges[0][1] - ranges[0][0]) * load_split) if (loads and not loads_first) else None
-        for c, (lo, hi) in enumerate(ranges):
-            if c == 0 and cut is not None:
-                upload(lo, cut)
-                loads()
-                upload(cut, hi)
-            else:
-                upload(lo, hi)
-            ev = torch.cuda.Event()
-            ev.record(copy_stream)
-            ready.append(ev)
+            for lo, hi in ranges:   # flows of intents [lo, hi)
+                dev["flows"][lo * ppg * F:hi * ppg * F].copy_(host["flows"][lo * ppg * F:hi * ppg * F],
+                                                               non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(copy_stream)
+                ready.append(ev)
+        if callable(finish):
+            finish()
         for (lo, hi), ev in zip(ranges, ready):
             n = hi - lo
             stream.wait_event(ev)

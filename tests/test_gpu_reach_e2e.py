@@ -261,13 +261,14 @@ def test_end_to_end_pipelined_from_host(validator, chunks):
     assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
 
 
-@pytest.mark.parametrize("loads_first", [False, True])
-def test_back_to_back_host_steps_each_with_its_own_tables(validator, loads_first):
+@pytest.mark.parametrize("loads_first,two_part", [(False, False), (False, True), (True, False), (True, True)])
+def test_back_to_back_host_steps_each_with_its_own_tables(validator, loads_first, two_part):
     """Three host-buffer steps enqueued back to back with no synchronisation,
-    each loading its own cluster and flow tables and verifying its own batch
-    (batches A, B, A): the alternating input buffers and the loads that
-    retire the replaced state only after its last use give every step the
-    oracle's verdicts for its batch."""
+    each loading its own cluster and flow tables (in one call, or in two
+    halves around the queued uploads) and verifying its own batch (batches
+    A, B, A): the alternating input buffers and the loads that retire the
+    replaced state only after its last use give every step the oracle's
+    verdicts for its batch."""
     import torch
     kw = dict(num_switches=48, num_intents=160, probes_per_intent=90, rules_per_switch=150)
     ea, eb = W.end_to_end(seed=31, **kw), W.end_to_end(seed=32, **kw)
@@ -287,11 +288,18 @@ def test_back_to_back_host_steps_each_with_its_own_tables(validator, loads_first
                 "flows": _pinned(flows_of(e)), "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
                 "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
 
+    def loads(e):
+        v.load_cluster(e.cluster)
+        if not two_part:
+            v.load_network(e.network)
+            return None
+        v.begin_network(e.network)
+        return v.finish_network
+
     stream, cs = torch.cuda.current_stream(), torch.cuda.Stream()
     steps = [(ea, host(ea)), (eb, host(eb)), (ea, host(ea))]
     for e, h in steps:
-        v.run_end_to_end_from_host(h, dev, sizes(e), stream, cs, 2 if loads_first else 1,
-                                   lambda e=e: (v.load_cluster(e.cluster), v.load_network(e.network)),
+        v.run_end_to_end_from_host(h, dev, sizes(e), stream, cs, 2 if loads_first else 1, lambda e=e: loads(e),
                                    loads_first=loads_first)
     stream.synchronize()
     v.sync()
@@ -325,6 +333,55 @@ def test_failed_table_load_keeps_the_loaded_tables(validator):
     v.sync()
     assert (again == first).all()
     assert (first == oracle.verify_probes(net, pr, 16)).all()
+
+
+def test_two_part_table_load(validator):
+    """Between pv_load_flow_tables_begin and _end, walks use the tables
+    installed before the begin; after the end, the new ones.  A second begin,
+    a one-part load in between, or an end with nothing begun are refused."""
+    a, b = W.tiny(seed=41)["network"], W.tiny(seed=42)["network"]
+    pr = W.tiny(seed=41)["probes"].probes
+    v = validator
+    v.load_network(a)
+    d_pr = to_device(pr, v.device)
+    want_a, want_b = oracle.verify_probes(a, pr, 16), oracle.verify_probes(b, pr, 16)
+    assert not (want_a == want_b).all()
+    v.begin_network(b)
+    try:
+        mid = to_numpy(v.verify_probes(d_pr, len(pr), 16), W.RESULT_DTYPE)
+        for call in (lambda: v.begin_network(b), lambda: v.load_network(b)):
+            with pytest.raises(B.PVError) as e:
+                call()
+            assert e.value.code == B.PV_ESTATE
+    finally:
+        v.finish_network()
+    after = to_numpy(v.verify_probes(d_pr, len(pr), 16), W.RESULT_DTYPE)
+    v.sync()
+    assert (mid == want_a).all()
+    assert (after == want_b).all()
+    with pytest.raises(B.PVError) as e:
+        v.finish_network()
+    assert e.value.code == B.PV_ESTATE
+
+
+def test_two_part_load_with_a_bad_rule_keeps_the_tables(validator):
+    """A rule field out of range is found by the device pass; the begin
+    succeeds, the end reports PV_EINVAL and the installed tables stay."""
+    d = W.tiny()
+    net, pr = d["network"], d["probes"].probes
+    v = validator
+    v.load_network(net)
+    bad = net.rules.copy()
+    bad[5]["dst_len"] = 40
+    B.pv_load_flow_tables_begin(v.ctx, net.num_switches, net.rule_offs, bad, net.switch_region, net.port_offs,
+                                net.port_peer, net.num_hosts, net.host_switch, net.host_port, net.host_ip)
+    with pytest.raises(B.PVError) as e:
+        B.pv_load_flow_tables_end(v.ctx)
+    assert e.value.code == B.PV_EINVAL
+    got = to_numpy(v.verify_probes(to_device(pr, v.device), len(pr), 16), W.RESULT_DTYPE)
+    v.sync()
+    assert (got == oracle.verify_probes(net, pr, 16)).all()
+    v.load_network(net)   # nothing left in progress
 
 
 def test_flow_binding_and_fused_walk(validator):
