@@ -126,3 +126,52 @@ int main(void) {
                                                   f["policy"][1], f["reserved"][1]]
     assert [int(x) for x in lines[1].split()] == [W.PATH_OK, W.PATH_NOSRC, W.PATH_BLOCKED, W.PATH_TOO_LONG,
                                                   W.PATH_REPEAT]
+
+
+def test_two_part_table_load_keeps_its_host_arrays_until_the_end(monkeypatch):
+    """The binding keeps the arrays it hands to pv_load_flow_tables_begin
+    (converted copies included) alive until pv_load_flow_tables_end or
+    pv_destroy, and drops them afterwards, whether the end succeeds or not
+    (a fake library stands in for libpv: no GPU is needed)."""
+    seen = {}
+
+    class Fake:
+        def __init__(self):
+            self.end_rc = B.PV_OK
+
+        def pv_load_flow_tables_begin(self, ctx, S, *ptrs):
+            seen["ptrs"] = ptrs
+            return B.PV_OK
+
+        def pv_load_flow_tables_end(self, ctx):
+            return self.end_rc
+
+        def pv_destroy(self, ctx):
+            pass
+
+        def pv_last_error(self, ctx):
+            return b"fake failure"
+
+    fake = Fake()
+    monkeypatch.setattr(B, "load_library", lambda path=None: fake)
+    ctx = ctypes.c_void_p(0x1234)
+    net = W.tiny()["network"]
+    offs = net.rule_offs.astype(np.int64)   # converted to u32 by the binding: a temporary it must keep
+    args = (net.num_switches, offs, net.rules, net.switch_region, net.port_offs, net.port_peer, net.num_hosts,
+            net.host_switch, net.host_port, net.host_ip)
+    B.pv_load_flow_tables_begin(ctx, *args)
+    kept = B._TABLE_LOADS[ctx.value]
+    assert kept[0].dtype == np.uint32 and kept[0].ctypes.data == seen["ptrs"][0]
+    assert (kept[0] == net.rule_offs).all()
+    B.pv_load_flow_tables_end(ctx)
+    assert ctx.value not in B._TABLE_LOADS
+
+    fake.end_rc = B.PV_EINVAL
+    B.pv_load_flow_tables_begin(ctx, *args)
+    with pytest.raises(B.PVError) as e:
+        B.pv_load_flow_tables_end(ctx)
+    assert e.value.code == B.PV_EINVAL and ctx.value not in B._TABLE_LOADS
+
+    B.pv_load_flow_tables_begin(ctx, *args)
+    B.pv_destroy(ctx)
+    assert ctx.value not in B._TABLE_LOADS
