@@ -290,10 +290,12 @@ int pv_verify_probes(pv_ctx *ctx, uint32_t num_probes, const pv_probe *d_probes,
  * u -> v: the out-neighbours of u are d_cols[d_offs[u] .. d_offs[u+1])),
  * d_region[V] (< 32), d_src[num_src] (vertex ids), d_masks[num_masks].
  * Device output: d_reach[num_masks][num_src][words_per_row] bitsets over V.
- * Malformed CSR entries (decreasing offsets, offsets > num_edges, cols >= V,
- * region >= 32) are
- * skipped and reported as PV_EINVAL by the next pv_sync(); out-of-range
- * sources give empty rows.  When every remaining edge has its reverse (and
+ * Malformed inputs are reported as PV_EINVAL by the next pv_sync() and never
+ * cause an access outside the arrays above: malformed offsets (some row
+ * with d_offs[u+1] < d_offs[u] or d_offs[u+1] > num_edges) make the graph
+ * count as having no edges at all (so R(s, m) = {s} for a permitted s); an
+ * edge with cols >= V is skipped; a vertex with region >= 32 is in no
+ * permitted set.  Out-of-range sources give empty rows.  When every remaining edge has its reverse (and
  * no vertex has more than 64 out-edges) the rows are taken from the
  * connected components of the permitted subgraph, which on such a graph is
  * the same set (PV_OPT_REACH_KERNEL).
@@ -322,8 +324,11 @@ int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_offs, uint32_t
  * allocation); make that first call before any stream capture.
  * All calls share the one array and each call overwrites it, so calls whose
  * work overlaps on the GPU (different streams, or host threads without
- * ordering) race; order them on one stream.  Malformed CSR entries are
- * skipped as in pv_compliant_reach, but no error is reported for them here.
+ * ordering) race; order them on one stream.  The address looked up on a
+ * device's first call is kept for the life of the process, so the library
+ * must not be used on a device after cudaDeviceReset.  Malformed inputs get
+ * the rows pv_compliant_reach gives them (malformed offsets: no edges;
+ * columns >= V skipped), but no error is reported for them here.
  * Returns PV_OK, PV_EINVAL (limits, NULL or misaligned pointers) or
  * PV_ECUDA.
  * ------------------------------------------------------------------------- */

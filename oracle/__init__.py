@@ -144,7 +144,8 @@ def compliant_reach(graph, sources, masks, pairs=None, words=None):
         pr = np.ascontiguousarray(pairs, np.uint32).reshape(-1, 2)
         npairs = len(pr)
         out = np.zeros((npairs, W), np.uint32)
-    rc = lib.oracle_compliant_reach(ctypes.c_uint32(V), _p(offs), _p(cols), _p(region), ctypes.c_uint32(len(src)),
+    rc = lib.oracle_compliant_reach(ctypes.c_uint32(V), _p(offs), ctypes.c_uint32(len(cols)), _p(cols), _p(region),
+                                    ctypes.c_uint32(len(src)),
                                     _p(src), ctypes.c_uint32(len(msk)), _p(msk), _p(pr), ctypes.c_uint32(npairs),
                                     _p(out), ctypes.c_uint32(W))
     if rc != 0:

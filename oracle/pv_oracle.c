@@ -352,15 +352,17 @@ int oracle_eval_selector_terms(uint32_t num_nodes, uint32_t num_keys, const uint
  * breadth-first search from s over CSR edges u -> v that enters v only if
  * region(v) is permitted.  Row layout as the selector bitsets.  Out-of-range
  * neighbours and regions >= 32 are never entered; an out-of-range source
- * yields an empty row.  pairs (optional) lists (mask index, source index)
- * to compute; rows are written in pair order.  Without pairs, all
- * num_masks x num_src rows are written mask-major.
+ * yields an empty row.  A CSR whose offsets are malformed (some row with
+ * offs[u+1] < offs[u] or offs[u+1] > num_edges) has no usable edge list, so
+ * it is read as a graph with no edges.  pairs (optional) lists (mask index,
+ * source index) to compute; rows are written in pair order.  Without pairs,
+ * all num_masks x num_src rows are written mask-major.
  * ---------------------------------------------------------------------- */
 static int vertex_allowed(const uint8_t *region, uint32_t v, uint32_t mask) {
     return region[v] < 32 && ((mask >> region[v]) & 1u);
 }
 
-static void bfs_row(uint32_t V, const uint32_t *offs, const uint32_t *cols, const uint8_t *region,
+static void bfs_row(uint32_t V, const uint32_t *offs, const uint32_t *cols, int has_edges, const uint8_t *region,
                     uint32_t s, uint32_t mask, uint32_t *row, uint32_t words_per_row,
                     uint32_t *queue, uint8_t *seen) {
     memset(row, 0, (size_t)words_per_row * 4);
@@ -372,6 +374,7 @@ static void bfs_row(uint32_t V, const uint32_t *offs, const uint32_t *cols, cons
     while (head < tail) {
         uint32_t u = queue[head++];
         row[u >> 5] |= 1u << (u & 31);
+        if (!has_edges) continue;
         for (uint32_t e = offs[u]; e < offs[u + 1]; ++e) {
             uint32_t v = cols[e];
             if (v >= V || seen[v] || !vertex_allowed(region, v, mask)) continue;
@@ -381,22 +384,26 @@ static void bfs_row(uint32_t V, const uint32_t *offs, const uint32_t *cols, cons
     }
 }
 
-int oracle_compliant_reach(uint32_t V, const uint32_t *offs, const uint32_t *cols, const uint8_t *region,
-                           uint32_t num_src, const uint32_t *src, uint32_t num_masks, const uint32_t *masks,
-                           const uint32_t *pairs, uint32_t num_pairs, uint32_t *reach, uint32_t words_per_row) {
+int oracle_compliant_reach(uint32_t V, const uint32_t *offs, uint32_t num_edges, const uint32_t *cols,
+                           const uint8_t *region, uint32_t num_src, const uint32_t *src, uint32_t num_masks,
+                           const uint32_t *masks, const uint32_t *pairs, uint32_t num_pairs, uint32_t *reach,
+                           uint32_t words_per_row) {
     uint32_t *queue = (uint32_t *)malloc((size_t)(V + 1) * 4);
     uint8_t *seen = (uint8_t *)malloc((size_t)V + 1);
     if (!queue || !seen) { free(queue); free(seen); return -1; }
+    int has_edges = 1;
+    for (uint32_t u = 0; u < V; ++u)
+        if (offs[u + 1] < offs[u] || offs[u + 1] > num_edges) has_edges = 0;
     if (pairs) {
         for (uint32_t i = 0; i < num_pairs; ++i) {
             uint32_t m = pairs[2 * i], j = pairs[2 * i + 1];
-            bfs_row(V, offs, cols, region, src[j], masks[m], reach + (size_t)i * words_per_row,
+            bfs_row(V, offs, cols, has_edges, region, src[j], masks[m], reach + (size_t)i * words_per_row,
                     words_per_row, queue, seen);
         }
     } else {
         for (uint32_t m = 0; m < num_masks; ++m)
             for (uint32_t j = 0; j < num_src; ++j)
-                bfs_row(V, offs, cols, region, src[j], masks[m],
+                bfs_row(V, offs, cols, has_edges, region, src[j], masks[m],
                         reach + ((size_t)m * num_src + j) * words_per_row, words_per_row, queue, seen);
     }
     free(queue);

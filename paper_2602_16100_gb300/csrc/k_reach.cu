@@ -38,7 +38,19 @@ constexpr int kGridThreads = 256;
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-// In-degree count with validation of the caller's CSR.
+// A CSR whose offsets are malformed (some row with offs[u + 1] < offs[u] or
+// offs[u + 1] > E) counts as having no edges at all: its well-formed rows
+// could overlap, so their lengths could add up past E, the size of every
+// edge-indexed scratch array.  indeg[V] (cleared with the counts, never
+// counted into) is that per-call flag; every later kernel of the call reads
+// it before it touches an edge.
+__device__ __forceinline__ bool csr_offsets_bad(const uint32_t *bad) {
+    return *(volatile const uint32_t *)bad != 0;
+}
+
+// In-degree count with validation of the caller's CSR.  An out-of-range
+// column skips that edge; malformed offsets set the flag at indeg[V] (the
+// counts of this pass are then unused).
 __global__ void reach_indeg_kernel(uint32_t V, uint32_t E, const uint32_t *__restrict__ offs,
                                    const uint32_t *__restrict__ cols, const uint8_t *__restrict__ region,
                                    uint32_t *__restrict__ indeg, int32_t *status) {
@@ -47,6 +59,7 @@ __global__ void reach_indeg_kernel(uint32_t V, uint32_t E, const uint32_t *__res
         const uint32_t a = offs[u], b = offs[u + 1];
         if (b < a || b > E) {
             pv_device_error(status, PV_EINVAL);
+            atomicOr(&indeg[V], 1u);
             continue;
         }
         for (uint32_t e = a; e < b; ++e) {
@@ -61,18 +74,20 @@ __global__ void reach_indeg_kernel(uint32_t V, uint32_t E, const uint32_t *__res
 }
 
 // Single block: in_offs = exclusive scan of indeg (V+1 entries); cursor copy.
+// With malformed offsets every in-edge list is empty.
 __global__ void __launch_bounds__(1024) reach_scan_kernel(uint32_t V, const uint32_t *__restrict__ indeg,
                                                           uint32_t *__restrict__ in_offs,
                                                           uint32_t *__restrict__ cursor, const uint32_t *asym) {
     if (asym && *(volatile const uint32_t *)asym == 0) return;   // symmetric: in-edges unused
     __shared__ uint32_t s_warp[32];
     __shared__ uint32_t s_carry;
+    const bool bad = csr_offsets_bad(indeg + V);
     const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5;
     if (t == 0) s_carry = 0;
     __syncthreads();
     for (uint32_t c0 = 0; c0 < V; c0 += 1024) {
         const uint32_t i = c0 + t;
-        const uint32_t x = i < V ? indeg[i] : 0;
+        const uint32_t x = i < V && !bad ? indeg[i] : 0;
         uint32_t incl = x;
         for (int d = 1; d < 32; d <<= 1) {
             uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
@@ -103,8 +118,9 @@ __global__ void __launch_bounds__(1024) reach_scan_kernel(uint32_t V, const uint
 
 __global__ void reach_fill_kernel(uint32_t V, uint32_t E, const uint32_t *__restrict__ offs,
                                   const uint32_t *__restrict__ cols, uint32_t *__restrict__ cursor,
-                                  uint32_t *__restrict__ in_cols, const uint32_t *asym) {
+                                  uint32_t *__restrict__ in_cols, const uint32_t *asym, const uint32_t *bad) {
     if (asym && *(volatile const uint32_t *)asym == 0) return;   // symmetric: in-edges unused
+    if (csr_offsets_bad(bad)) return;                            // no edges
     for (uint32_t u = blockIdx.x * blockDim.x + threadIdx.x; u < V; u += gridDim.x * blockDim.x) {
         const uint32_t a = offs[u], b = offs[u + 1];
         if (b < a || b > E) continue;
@@ -119,13 +135,16 @@ __global__ void reach_fill_kernel(uint32_t V, uint32_t E, const uint32_t *__rest
 // *asym != 0 unless every edge u -> v (v < V, both lists well formed) has
 // its reverse v -> u.  Vertices whose list is longer than kSymScanMax make
 // the graph count as asymmetric (the sweep path then runs; still exact).
+// With malformed offsets (flag set by the in-degree pass) the graph has no
+// edges, which is symmetric: nothing is listed.
 // The same pass lists each undirected edge once, as pairs[] = u << 16 | v
 // with v < u (*npairs of them, in no particular order).
 constexpr uint32_t kSymScanMax = 64;
 
 __global__ void reach_symcheck_kernel(uint32_t V, uint32_t E, const uint32_t *__restrict__ offs,
                                       const uint32_t *__restrict__ cols, uint32_t *asym, uint32_t *pairs,
-                                      uint32_t *npairs) {
+                                      uint32_t *npairs, const uint32_t *bad) {
+    if (csr_offsets_bad(bad)) return;   // no edges: symmetric, no pairs
     const uint32_t lane = threadIdx.x & 31;
     const uint32_t nwarps = gridDim.x * (blockDim.x / 32);
     for (uint32_t u = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32; u < V; u += nwarps) {
@@ -180,7 +199,8 @@ __device__ __forceinline__ uint32_t uf_find(volatile uint32_t *parent, uint32_t 
     }
 }
 
-__device__ __forceinline__ void uf_union(volatile uint32_t *parent, uint32_t a, uint32_t b, uint32_t limit) {
+__device__ __forceinline__ void uf_union(volatile uint32_t *parent, uint32_t a, uint32_t b, uint32_t limit,
+                                         int32_t *status) {
     for (uint32_t it = 0; it < limit; ++it) {
         a = uf_find(parent, a);
         b = uf_find(parent, b);
@@ -192,6 +212,9 @@ __device__ __forceinline__ void uf_union(volatile uint32_t *parent, uint32_t a, 
         }
         if (atomicCAS(const_cast<uint32_t *>(parent + a), a, b) == a) return;
     }
+    // not reachable by the argument above; should it happen all the same,
+    // the row would be wrong, so the call reports it rather than pass
+    pv_device_error(status, PV_ETIMEOUT);
 }
 
 constexpr int kCompThreads = 512;
@@ -211,7 +234,7 @@ constexpr int kLabelThreads = 1024;
 __global__ void __launch_bounds__(kLabelThreads) reach_labels_kernel(
     uint32_t V, const uint32_t *__restrict__ pairs, const uint32_t *__restrict__ npairs,
     const uint8_t *__restrict__ region, const uint32_t *__restrict__ masks, uint16_t *__restrict__ lab,
-    const uint32_t *asym) {
+    const uint32_t *asym, int32_t *status) {
     if (*(volatile const uint32_t *)asym) return;       // not symmetric: the sweep kernel runs
     extern __shared__ __align__(16) uint8_t s_dyn[];
     volatile uint32_t *parent = reinterpret_cast<uint32_t *>(s_dyn);              // [V]
@@ -252,7 +275,7 @@ __global__ void __launch_bounds__(kLabelThreads) reach_labels_kernel(
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const uint32_t u = pq[k] >> 16, v = pq[k] & 0xFFFFu;
-            if (i + k < np && allowed(u) && allowed(v)) uf_union(parent, u, v, 2 * V + 2);
+            if (i + k < np && allowed(u) && allowed(v)) uf_union(parent, u, v, 2 * V + 2, status);
         }
     }
     __syncthreads();
@@ -446,6 +469,37 @@ __global__ void __launch_bounds__(kReachThreads) reach_msbfs_kernel(
     }
 }
 
+// The dynamic shared-memory limits of the three block-wide kernels are
+// process-wide settings per device.  They are raised once per device to the
+// largest size any call can ask for (under a mutex), so that no call lowers
+// the limit between another thread's setting and launch.
+constexpr int kSmemAttrMaxDevices = 64;
+std::mutex g_smem_attr_mutex;
+bool g_smem_attr_set[kSmemAttrMaxDevices] = {};
+
+cudaError_t reach_smem_limits() {
+    int dev = 0, optin = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kSmemAttrMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_smem_attr_mutex);
+    if (g_smem_attr_set[dev]) return cudaSuccess;
+    e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e != cudaSuccess) return e;
+    const int rows_max = optin - 1024;
+    const int lab_max = (int)(up16u(kReachMaxV * 4) + up16u(kReachMaxV / 32 * 4));
+    const int bfs_max = (int)(kReachMaxV * 8);
+    if ((e = cudaFuncSetAttribute(reach_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, rows_max)) !=
+            cudaSuccess ||
+        (e = cudaFuncSetAttribute(reach_labels_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  std::min(lab_max, rows_max))) != cudaSuccess ||
+        (e = cudaFuncSetAttribute(reach_msbfs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  std::min(bfs_max, rows_max))) != cudaSuccess)
+        return e;
+    g_smem_attr_set[dev] = true;
+    return cudaSuccess;
+}
+
 }  // namespace
 
 extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_offs, uint32_t num_edges,
@@ -495,6 +549,7 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
         if (rows_smem > limit) return pv_fail(ctx, PV_EINVAL, "pv_compliant_reach: words_per_row too large");
     }
     uint16_t *lab = (uint16_t *)(base + o_lab);   // [num_masks][V] (component path only)
+    PV_TRY_CUDA(ctx, reach_smem_limits(), "reach shared-memory limits");
     PV_TRY_CUDA(ctx, cudaMemsetAsync(indeg, 0, (size_t)(V + 1) * 4, st), "indeg clear");
     if (comp) {
         PV_TRY_CUDA(ctx, cudaMemsetAsync(ctx->d_reach_asym, 0, 4, st), "symmetry flag clear");
@@ -510,20 +565,15 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
         const uint32_t wgrid = std::min<uint32_t>((V + kGridThreads / 32 - 1) / (kGridThreads / 32),
                                                   (uint32_t)ctx->num_sms * 8);
         reach_symcheck_kernel<<<wgrid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, ctx->d_reach_asym, pairs,
-                                                              npairs);
+                                                              npairs, indeg + V);
         launches += 3;
     }
     reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor, sym_flag);
-    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, sym_flag);
+    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, sym_flag,
+                                                     indeg + V);
     if (comp) {
-        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(reach_labels_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              (int)lab_smem),
-                    "labels smem");
         reach_labels_kernel<<<num_masks, kLabelThreads, lab_smem, st>>>(V, pairs, npairs, d_region, d_masks, lab,
-                                                                         ctx->d_reach_asym);
-        PV_TRY_CUDA(ctx, cudaFuncSetAttribute(reach_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                              (int)rows_smem),
-                    "rows smem");
+                                                                         ctx->d_reach_asym, ctx->d_status);
         int per_sm = 1;
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, reach_rows_kernel, kCompThreads, rows_smem);
         // one wave of resident blocks over masks x source slices
@@ -535,8 +585,6 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
                                                                cap, ctx->d_reach_asym);
     }
     const size_t smem = (size_t)V * 8;
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(reach_msbfs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem),
-                "reach smem");
     int bfs_per_sm = 1;
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bfs_per_sm, reach_msbfs_kernel, kReachThreads, smem);
     const uint64_t items = (uint64_t)((num_src + 63) / 64) * num_masks;
@@ -576,7 +624,10 @@ std::mutex g_noalloc_mutex;
 uint8_t *g_noalloc_base[kNoAllocMaxDevices] = {};
 
 // Device address of the static array on the current device, looked up once
-// per device (in host code the array's name is not a device address).
+// per device (in host code the array's name is not a device address) and
+// kept for the life of the process: after a cudaDeviceReset the module is
+// loaded again and the kept address would be stale, so the library is not
+// to be used on a device after a reset.
 int noalloc_scratch(uint8_t **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return PV_ECUDA;
@@ -621,11 +672,10 @@ extern "C" int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, ui
     const uint32_t grid = std::min<uint32_t>((V + kGridThreads - 1) / kGridThreads, (uint32_t)sms * 8);
     reach_indeg_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, d_region, indeg, status);
     reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor, nullptr);
-    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, nullptr);
+    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, nullptr,
+                                                     indeg + V);
     const size_t smem = (size_t)V * 8;
-    if (cudaFuncSetAttribute(reach_msbfs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-        cudaSuccess)
-        return PV_ECUDA;
+    if (reach_smem_limits() != cudaSuccess) return PV_ECUDA;
     const uint64_t items = (uint64_t)((num_src + 63) / 64) * num_masks;
     const uint32_t g2 = (uint32_t)std::min<uint64_t>(items, (uint64_t)sms * 4);
     reach_msbfs_kernel<<<g2, kReachThreads, smem, st>>>(V, in_offs, in_cols, d_region, num_src, d_src, num_masks,

@@ -145,6 +145,36 @@ def test_malformed_csr_is_reported(validator):
         B.pv_compliant_reach(validator.ctx, 0, 0, 0, 0, 0, 1, 0, 1, 0, 0, 4)
 
 
+@pytest.mark.parametrize("kernel", [0, 1])
+def test_overlapping_offsets_read_as_no_edges(validator, kernel):
+    """Offsets that go back down let well-formed rows overlap (rows 0, 2, 4,
+    ... all cover every edge), so their lengths add up to many times the
+    edge count.  The call reports PV_EINVAL, writes nothing past the edge
+    arrays, and gives the oracle's rows for a graph without edges, on the
+    component path (kernel 0) and on the sweeps (kernel 1)."""
+    V, E = 64, 300
+    g0 = W.random_digraph(35, V, E)
+    offs = np.where(np.arange(V + 1) % 2 == 0, 0, E).astype(np.uint32)
+    bad = W.Graph(V, offs, g0.cols, g0.region)
+    src = np.arange(V, dtype=np.uint32)
+    masks = np.array([0xFFFFFFFF, 0b1011, 0], np.uint32)
+    want = oracle.compliant_reach(bad, src, masks)
+    assert (want.sum(axis=(0, 1)) != 0).any()
+    dev = validator.device
+    validator.set_option(B.PV_OPT_REACH_KERNEL, kernel)
+    try:
+        out = validator.compliant_reach(validator.upload_graph(bad), V, to_device(src, dev), len(masks),
+                                        to_device(masks, dev))
+        with pytest.raises(B.PVError) as e:
+            validator.sync()
+        assert e.value.code == B.PV_EINVAL
+        validator.sync()
+    finally:
+        validator.set_option(B.PV_OPT_REACH_KERNEL, 0)
+    got = to_numpy(out, np.uint32, want.shape)
+    assert (got == want).all()
+
+
 def test_continuum_wan_full_size_sampled(validator):
     q = W.continuum_wan()
     gr = _gpu_reach(validator, q.graph, q.sources, q.masks)

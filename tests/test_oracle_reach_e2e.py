@@ -116,6 +116,26 @@ def test_reach_pairs_and_out_of_range_inputs():
     assert _members(R3[0, 0], 3) == {0} and not R3[0, 1].any()
 
 
+@pytest.mark.parametrize("offs", [[0, 6, 2, 6], [0, 2, 4, 7], [1, 3, 2, 3]])
+def test_reach_malformed_offsets_read_as_no_edges(offs):
+    """Offsets that decrease or pass the edge count leave no usable edge
+    list: every row is {s} for a permitted source (the closed form of a
+    graph without edges), whatever well-formed rows the array also has."""
+    cols = np.array([1, 2, 0, 2, 0, 1], np.uint32)
+    region = np.array([0, 1, 0], np.uint8)
+    g = W.Graph(3, np.array(offs, np.uint32), cols, region)
+    masks = np.array([0xFFFFFFFF, 0b01], np.uint32)
+    R = oracle.compliant_reach(g, np.arange(3, dtype=np.uint32), masks)
+    for m, mask in enumerate(masks):
+        for s in range(3):
+            want = {s} if (int(mask) >> int(region[s])) & 1 else set()
+            assert _members(R[m, s], 3) == want
+    # the same arrays with well-formed offsets do have edges
+    ok = oracle.compliant_reach(W.Graph(3, np.array([0, 2, 4, 6], np.uint32), cols, region),
+                                np.arange(3, dtype=np.uint32), masks)
+    assert _members(ok[0, 0], 3) == {0, 1, 2}
+
+
 def test_placement_binding_and_verdict():
     st = W.Stream(5, "e2e-pins")
     G, N, pods = 50, 70, 4

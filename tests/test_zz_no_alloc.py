@@ -7,12 +7,15 @@ them the library offers pv_compliant_reach_noalloc, which needs no context and
 works in one static device array.  This test calls it through the C ABI twice
 in a row (on different inputs, so the second call must not see leftovers of
 the first) and compares each result with the regular pv_compliant_reach
-bit for bit, and checks that oversized inputs are refused.  The file is named
-to be collected last.
+bit for bit and with the CPU oracle, gives the oracle's rows for a CSR with
+overlapping rows (malformed offsets: no edges) without writing past its
+array, and checks that oversized inputs are refused.  The file is named to
+be collected last.
 """
 import numpy as np
 import pytest
 
+import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
 from paper_2602_16100_gb300.validator import empty_device, to_device, to_numpy
@@ -57,6 +60,21 @@ def test_noalloc_reach_matches_regular_call_twice(validator):
         got = _noalloc(validator, x)
         assert (got == want).all()
         assert want.any()
+        assert (got == oracle.compliant_reach(g, src, masks).reshape(-1)).all()
+
+
+def test_noalloc_reach_overlapping_offsets_read_as_no_edges(validator):
+    V, E = 64, 300
+    g0 = W.random_digraph(36, V, E)
+    offs = np.where(np.arange(V + 1) % 2 == 0, 0, E).astype(np.uint32)   # rows overlap; total >> E
+    bad = W.Graph(V, offs, g0.cols, g0.region)
+    src = np.arange(V, dtype=np.uint32)
+    masks = np.array([0xFFFFFFFF, 0b1011], np.uint32)
+    got = _noalloc(validator, _inputs(validator, bad, src, masks))
+    assert (got == oracle.compliant_reach(bad, src, masks).reshape(-1)).all()
+    # the next call on a well-formed graph is not affected
+    x = _inputs(validator, g0, src, masks)
+    assert (_noalloc(validator, x) == oracle.compliant_reach(g0, src, masks).reshape(-1)).all()
 
 
 def test_noalloc_reach_rejects_oversized_inputs(validator):
