@@ -9,7 +9,8 @@ probes, hop cap 32).  One step = selector rows -> placement -> probe binding
 -> hop-synchronous walks -> per-intent verdicts, all in libpv's kernels.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--workload e2e|placement|flow|wan]
+                  [--workload e2e|e2e_policies|placement|placement_terms|placement_replicas|flow|wan|schedule]
+                  [--no-extra-configs] [--no-cpu-baseline]
 
 Prints one JSON line (rank 0).  `value` is device-timed throughput with the
 inputs resident in HBM (CUDA events on the launching stream, K steps after W
@@ -17,10 +18,15 @@ warm-ups, max over ranks); `e2e` is the same metric through the public API
 from pinned host buffers (loads, host->device copies, the step and the
 device->host read of the verdicts inside the timed region).  `kernels` and
 `roofline` come from a second pass of the same K steps under the library's
-CUDA-event profiler, so its events stay out of the timed region.  Under torchrun
-each rank processes its own shard (seed offset by rank): weak scaling, no
-collective on the data path.  `--impl reference` times the CPU oracle on a
-bounded sample of the same workload.
+CUDA-event profiler, so its events stay out of the timed region.  With the
+default workload, `configs` holds the other configurations of the metric
+(placement-scale, flow-verification, continuum WAN), each measured the same
+way on its own device-resident batch with its own roofline and CPU baseline
+(`--no-extra-configs` leaves them out).  Under torchrun each rank processes
+its own shard (seed offset by rank): weak scaling, no collective on the data
+path; after the timed regions the per-status counters and verdict counts are
+summed over ranks (`summed_over_ranks`).  `--impl reference` times the CPU
+oracle on a bounded sample of the same workload.
 """
 from __future__ import annotations
 
@@ -203,6 +209,16 @@ class EndToEndBench:
                 "probe_hops_per_step": self.probe_hops, "hop_kernel_entries_per_step": self.hop_entries,
                 "status_histogram": dict(zip(W.STATUS_NAMES, self.status_hist)),
                 "intents_passed": self.pass_count}
+
+    def counters(self):
+        return (list(W.STATUS_NAMES) + ["probe_hops", "intents_passed"],
+                list(self.status_hist) + [self.probe_hops, self.pass_count])
+
+    def release(self):
+        """Drop the batch's device and pinned host buffers."""
+        for k in ("dev", "host"):
+            if hasattr(self, k):
+                delattr(self, k)
 
     def algorithmic_bytes(self, group):
         e = self.e
@@ -594,6 +610,14 @@ class FlowBench:
         return {"probe_hops_per_step": self.probe_hops, "hop_kernel_entries_per_step": self.hop_entries,
                 "status_histogram": dict(zip(W.STATUS_NAMES, self.hist))}
 
+    def counters(self):
+        return list(W.STATUS_NAMES) + ["probe_hops"], list(self.hist) + [self.probe_hops]
+
+    def release(self):
+        for k in ("d_probes", "d_out"):
+            if hasattr(self, k):
+                delattr(self, k)
+
     def algorithmic_bytes(self, group):
         return {"walk_hop": 20, "walk_regroup": 16}.get(group, 0) * self.hop_entries + \
             (len(self.p.probes) * 16 if group == "walk_init" else 0)
@@ -687,6 +711,33 @@ def timed_oracle(wl, target_s=12.0, cap_s=40.0):
         n = min(wl.oracle_max(), int(n * max(1.5, min(8.0, target_s / max(dt, 1e-3)))))
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (x86: /proc/cpuinfo; Arm: lscpu)."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def cpu_baseline(wl, target_s):
+    """The oracle, single-threaded as written, on a bounded sample."""
+    u, dt, desc, _ = timed_oracle(wl, target_s=target_s, cap_s=max(40.0, 3 * target_s))
+    return {"value": u / dt, "unit": wl.unit, "cores": 1, "host_cores": os.cpu_count(), "cpu_model": cpu_model(),
+            "kind": "oracle", "sample": desc, "seconds": dt}
+
+
 # ----------------------------------------------------------------------------
 # arms
 # ----------------------------------------------------------------------------
@@ -710,49 +761,27 @@ def run_reference(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u32",
             "data": "synthetic", "config": wl.config(),
-            "cpu_baseline": {"value": value, "unit": wl.unit, "cores": 1, "kind": "oracle", "sample": desc},
+            "cpu_baseline": {"value": value, "unit": wl.unit, "cores": 1, "host_cores": os.cpu_count(),
+                             "cpu_model": cpu_model(), "kind": "oracle", "sample": desc},
             "e2e": {"value": value, "unit": wl.unit, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
 
 
-def run_ours(args):
+def measure(wl, v, args, stream, barrier, dist, gpu_index):
+    """One workload on the device: W warm-up steps, K steps timed with CUDA
+    events on the launching stream (clocks sampled meanwhile), the same K
+    steps once more under the library's CUDA-event profiler (per kernel
+    group), and for walks one diagnostic step with the counting kernels.
+    Returns the timing, the kernel groups and the dominant group's roofline."""
     import torch
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl")
-    torch.cuda.set_device(local)
     from paper_2602_16100_gb300 import binding as B
-    from paper_2602_16100_gb300 import build
     from paper_2602_16100_gb300 import sharding as SH
-    from paper_2602_16100_gb300.validator import Validator
-    if rank == 0 or world == 1:
-        build.build_library()
-    if dist:
-        dist.barrier()
-    # weak scaling: every rank verifies its own batch of the same shape (the
-    # units are independent; no collective on the data path)
-    wl = WORKLOADS[args.workload](SH.shard_seed(0, rank), **({"intents": args.intents} if args.intents else {}))
-    v = Validator(local)
     wl.setup(v)
-    stream = torch.cuda.current_stream()
     for _ in range(max(args.warmup, 1)):
         wl.step(stream)
     v.sync(stream)
     units = wl.measure_units()
-
-    def barrier():
-        torch.cuda.synchronize()
-        if dist:
-            dist.barrier()
-        torch.cuda.synchronize()
-
-    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
-    gpu_index = vis.split(",")[local] if vis else local
     barrier()
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(gpu_index) as clk:
@@ -787,9 +816,6 @@ def run_ours(args):
         walk_stats = walk_statistics(v)
     ms = SH.max_over_ranks(ms, dist, "cuda")
     secs_per_step = ms / 1e3 / args.steps
-    value = units * world / secs_per_step
-
-    # per-kernel-group device time of the profiled pass (same steps, same launches)
     kernels, launches = {}, 0
     for gi, name in enumerate(B.PV_K_NAMES):
         kms, n = B.pv_profile_read(v.ctx, gi)
@@ -812,6 +838,65 @@ def run_ours(args):
         roofline = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                     "frac": achieved / peak, "peak_source": peak_kind, "traffic": traffic,
                     "algorithmic_bytes_per_launch": bytes_per_launch, "avg_launch_ms": avg_launch_s * 1e3}
+    if walk_stats:
+        walk_stats = dict(walk_stats)
+        walk_stats["rule_tests_per_s"] = (walk_stats["index_rule_tests"] + walk_stats["interval_lookups"]) / \
+            secs_per_step
+        walk_stats["scan_equivalent_rules_per_s"] = walk_stats["scan_depth"] / secs_per_step
+    return {"units": units, "ms": ms, "secs_per_step": secs_per_step, "kernels": kernels, "launches": launches,
+            "roofline": roofline, "clocks": clk.result, "walk_statistics": walk_stats}
+
+
+def sum_counters(wl, dist):
+    """The per-status histogram, probe-hop count and verdict count of a
+    rank's batch summed over all ranks (host bookkeeping after the timed
+    regions; one all-reduce of a few integers)."""
+    from paper_2602_16100_gb300 import sharding as SH
+    if not hasattr(wl, "counters"):
+        return {}
+    names, vals = wl.counters()
+    tot = SH.sum_vector_over_ranks(vals, dist, "cuda")
+    return {"summed_over_ranks": dict(zip(names, (int(x) for x in tot)))}
+
+
+EXTRA_CONFIGS = ("placement", "flow", "wan")   # measured beside the end-to-end headline
+
+
+def run_ours(args):
+    import torch
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    from paper_2602_16100_gb300 import build
+    from paper_2602_16100_gb300 import sharding as SH
+    from paper_2602_16100_gb300.validator import Validator
+    if rank == 0 or world == 1:
+        build.build_library()
+    if dist:
+        dist.barrier()
+    # weak scaling: every rank verifies its own batch of the same shape (the
+    # units are independent; no collective on the data path)
+    wl = WORKLOADS[args.workload](SH.shard_seed(0, rank), **({"intents": args.intents} if args.intents else {}))
+    v = Validator(local)
+    stream = torch.cuda.current_stream()
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    gpu_index = vis.split(",")[local] if vis else local
+    m = measure(wl, v, args, stream, barrier, dist, gpu_index)
+    secs_per_step = m["secs_per_step"]
+    value = m["units"] * world / secs_per_step
+    sums = sum_counters(wl, dist)
 
     # end-to-end through the public API from pinned host buffers
     e2e = None
@@ -827,31 +912,48 @@ def run_ours(args):
         barrier()
         e_s = (time.perf_counter() - t0) / args.steps
         e_s = SH.max_over_ranks(e_s, dist, "cuda")
-        e2e = {"value": units * world / e_s, "unit": wl.unit, "h2d_bytes_per_step": int(wl.h2d),
+        e2e = {"value": m["units"] * world / e_s, "unit": wl.unit, "h2d_bytes_per_step": int(wl.h2d),
                "d2h_bytes_per_step": int(wl.d2h), "ms_per_step": e_s * 1e3, "upload_chunks": args.e2e_chunks,
                "loads": ("before the uploads" if args.e2e_loads_first
                          else "uploads of the tables queued first, the rest of the load while the inputs arrive")}
         if hasattr(wl, "e2e_phases"):
             e2e["phases"] = wl.e2e_phases(v, stream)
+        wl.release()
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        u, dt, desc, _ = timed_oracle(wl)
-        cpu = {"value": u / dt, "unit": wl.unit, "cores": 1, "kind": "oracle", "sample": desc,
-               "seconds": dt}
+    baseline_s = 12.0
+    cpu = cpu_baseline(wl, baseline_s) if rank == 0 and world == 1 and not args.no_cpu_baseline else None
+
+    # the other configurations of the metric, each timed the same way on its
+    # own batch (one device-resident step each; the headline stays the
+    # end-to-end line)
+    configs = {}
+    if args.workload == "e2e" and not args.no_extra_configs:
+        for name in EXTRA_CONFIGS:
+            xw = WORKLOADS[name](SH.shard_seed(0, rank))
+            xm = measure(xw, v, args, stream, barrier, dist, gpu_index)
+            entry = {"value": xm["units"] * world / xm["secs_per_step"], "unit": xw.unit,
+                     "ms_per_step": xm["ms"] / args.steps, "config": xw.config(), "roofline": xm["roofline"],
+                     "kernels": xm["kernels"], "gpu_launches": xm["launches"], "clocks": xm["clocks"],
+                     **xw.extra(xm["secs_per_step"]), **sum_counters(xw, dist)}
+            if xm["walk_statistics"]:
+                entry["walk_statistics"] = xm["walk_statistics"]
+            if rank == 0 and world == 1 and not args.no_cpu_baseline:
+                entry["cpu_baseline"] = cpu_baseline(xw, 6.0)
+            configs[xw.name] = entry
+            if hasattr(xw, "release"):
+                xw.release()
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": wl.unit, "n_gpus": world, "steps": args.steps,
-                "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+                "warmup": args.warmup, "ms_per_step": m["ms"] / args.steps, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "u32", "data": "synthetic",
                 "config": {**wl.config(), "parallelism": f"independent shards x{world}"},
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
-                "clocks": clk.result, "kernels": kernels, **wl.extra(secs_per_step)}
-        if walk_stats:
-            ws = dict(walk_stats)
-            ws["rule_tests_per_s"] = (ws["index_rule_tests"] + ws["interval_lookups"]) / secs_per_step
-            ws["scan_equivalent_rules_per_s"] = ws["scan_depth"] / secs_per_step
-            line["walk_statistics"] = ws
+                "roofline": m["roofline"], "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": m["launches"],
+                "clocks": m["clocks"], "kernels": m["kernels"], **wl.extra(secs_per_step), **sums}
+        if m["walk_statistics"]:
+            line["walk_statistics"] = m["walk_statistics"]
+        if configs:
+            line["configs"] = configs
         print(json.dumps(line), flush=True)
     v.close()
     if dist:
@@ -867,6 +969,8 @@ def main():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", choices=tuple(WORKLOADS), default="e2e")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra-configs", action="store_true",
+                    help="end-to-end only: leave out the placement, flow-verification and WAN entries of `configs`")
     ap.add_argument("--e2e-chunks", type=int, default=1,
                     help="intent ranges whose probe upload overlaps verification in the host-buffer step")
     ap.add_argument("--e2e-loads-first", action="store_true",

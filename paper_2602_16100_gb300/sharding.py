@@ -6,8 +6,10 @@ intent's inputs plus the shared cluster labels and flow tables (Sec. 4.2, the
 per-intent cross-layer check; Sec. 5.5, one verdict per intent).  A batch
 therefore splits into contiguous intent ranges with no exchange between
 ranks: each rank loads the shared cluster and network, runs its own range on
-its own GPU, and the only collectives are host-side bookkeeping (a barrier
-and the max over ranks of the timed region, outside the data path).
+its own GPU, and the only collectives are host-side bookkeeping outside the
+data path: a barrier, the max over ranks of the timed region, and the sum
+over ranks of the per-status counters and verdict counts once the batch is
+done.
 
 This module holds the host-side range arithmetic, the slicing of an
 end-to-end batch and the rank bookkeeping.  It does no compliance arithmetic.
@@ -79,3 +81,15 @@ def sum_over_ranks(x: int, dist=None, device: Optional[str] = None) -> int:
     t = torch.tensor([int(x)], dtype=torch.int64, device=device or "cpu")
     dist.all_reduce(t, op=dist.ReduceOp.SUM)
     return int(t.item())
+
+
+def sum_vector_over_ranks(v, dist=None, device: Optional[str] = None) -> np.ndarray:
+    """Elementwise sum of an integer vector (per-status counters, verdict
+    counts) over all ranks; a copy of `v` without a process group."""
+    a = np.asarray(v, dtype=np.int64).copy()
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return a
+    import torch
+    t = torch.from_numpy(a).to(device or "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return t.cpu().numpy()

@@ -68,6 +68,7 @@ STATUS_NAMES = ("compliant", "violation", "drop", "loop", "misdelivered", "nosrc
 F_ASSIGN_OK, F_EMPTY, F_UNKNOWN_VALUE, F_PASS, F_BAD_EXPR = 1, 2, 4, 8, 16
 
 ROUTING_PRIORITY = 100
+PASS_DPORT_LO = 49152    # end-to-end variant with passing intents: ports no ACL rule covers
 
 _GAMMA = 0x9E3779B97F4A7C15
 _M1 = 0xBF58476D1CE4E5B9
@@ -290,11 +291,12 @@ def _random_host_prefix(st: Stream, host_ip: np.ndarray, lens: np.ndarray) -> np
 
 
 def _acl_fill(st: Stream, n: int, nports: int, host_ip: np.ndarray, *, src_len_range, dst_len_range,
-              dport_width_max, p_any_in, p_drop, p_shadow):
+              dport_width_max, p_any_in, p_drop, p_shadow, dport_max: int = 65535):
     """n ACL rules above routing priority; a fraction are shadowed copies of
-    an earlier rule (narrower match, strictly lower priority).  Returns the
-    rule records and, per rule, the local index of the rule that shadows it
-    (or -1)."""
+    an earlier rule (narrower match, strictly lower priority).  Port ranges
+    lie in [0, dport_max] (the draws are scaled into it when dport_max is
+    below 65535, so the stream is consumed alike).  Returns the rule records
+    and, per rule, the local index of the rule that shadows it (or -1)."""
     r = np.zeros(n, RULE_DTYPE)
     shadow_of = np.full(n, -1, np.int64)
     if n == 0:
@@ -315,8 +317,10 @@ def _acl_fill(st: Stream, n: int, nports: int, host_ip: np.ndarray, *, src_len_r
     else:
         lo = st.ints(0, 65535, n)
         w = st.ints(0, dport_width_max, n)
+        if dport_max < 65535:
+            lo = lo * (dport_max + 1) // 65536
         r["dport_lo"] = lo
-        r["dport_hi"] = np.minimum(lo + w, 65535)
+        r["dport_hi"] = np.minimum(lo + w, dport_max)
     anyp = st.floats(n) < p_any_in
     r["in_port"] = np.where(anyp, ANY_PORT, st.ints(0, nports - 1, n))
     drop = st.floats(n) < p_drop
@@ -764,7 +768,7 @@ def random_digraph(seed: int, num_vertices: int, num_edges: int, num_regions: in
 def end_to_end(seed: int = 20260220, num_switches: int = 512, avg_degree: float = 5.0,
                num_regions: int = 16, hosts_per_switch: int = 2, num_keys: int = 32,
                rules_per_switch: int = 1000, num_intents: int = 10_000, pods_per_intent: int = 4,
-               probes_per_intent: int = 5000, hop_cap: int = 32, mask_pop=(2, 8)):
+               probes_per_intent: int = 5000, hop_cap: int = 32, mask_pop=(2, 8), pass_share: float = 0.0):
     """Random switch graph (random spanning tree + uniform extra edges to the
     average degree), regions uniform, 2 hosts per switch (host n = cluster
     node n) at 10.(s>>8).(s&255).(h+1); /24 BFS routing to every other switch
@@ -772,7 +776,15 @@ def end_to_end(seed: int = 20260220, num_switches: int = 512, avg_degree: float 
     region mask (U[lo,hi] regions), a selector whose first term is
     region In (the mask's regions) plus 0-3 equality/In terms on other keys
     (Zipf(1.1, 64) values), 4 pods placed by seeded choice among feasible
-    nodes, and probes from the pods' hosts (round-robin) to uniform hosts."""
+    nodes, and probes from the pods' hosts (round-robin) to uniform hosts.
+
+    pass_share > 0 gives the variant in which intents can pass: the ACL
+    rules' port ranges lie in [0, 49151], and a pass_share fraction of the
+    intents (drawn from a stream of their own, so every other draw is that
+    of the plain workload) permit every region (selector term region
+    Exists) and send their flows to ports in [49152, 65535].  No ACL rule
+    matches those flows, so the routing rules deliver each one along BFS
+    next hops; such an intent passes when all its pods are placed."""
     st = Stream(seed, "e2e")
     S = num_switches
     perm = st.permutation(S)
@@ -805,7 +817,8 @@ def end_to_end(seed: int = 20260220, num_switches: int = 512, avg_degree: float 
         rt = np.concatenate(rt)
         acl, sh = _acl_fill(st, max(0, rules_per_switch - len(rt)), nports, host_ip,
                             src_len_range=(8, 32), dst_len_range=(8, 32), dport_width_max=1023,
-                            p_any_in=0.75, p_drop=0.2, p_shadow=0.05)
+                            p_any_in=0.75, p_drop=0.2, p_shadow=0.05,
+                            dport_max=PASS_DPORT_LO - 1 if pass_share > 0 else 65535)
         rules.append(np.concatenate([rt, acl]))
         shadows.append(np.concatenate([np.full(len(rt), -1), np.where(sh >= 0, sh + len(rt), -1)]))
     rule_offs, all_rules, shadowed_by = _assemble_tables(st, rules, shadows)
@@ -862,6 +875,16 @@ def end_to_end(seed: int = 20260220, num_switches: int = 512, avg_degree: float 
     pr["src_host"] = NO_HOST
     pr["dst_ip"] = host_ip[st.ints(0, H - 1, M)]
     pr["dport"] = st.ints(0, 65535, M)
+    if pass_share > 0:
+        sp = Stream(seed, "e2e-pass")
+        chosen = np.nonzero(sp.floats(I) < pass_share)[0]
+        masks[chosen] = (1 << num_regions) - 1 if num_regions < 32 else 0xFFFFFFFF
+        first = offs[chosen].astype(np.int64)
+        exprs["op"][first] = OP_EXISTS
+        exprs["nvals"][first] = 0
+        exprs["vals"][first] = 0
+        k = (chosen[:, None] * probes_per_intent + np.arange(probes_per_intent)[None, :]).reshape(-1)
+        pr["dport"][k] = sp.ints(PASS_DPORT_LO, 65535, len(k))
     pr["allowed_mask"] = np.repeat(masks, probes_per_intent)
     return EndToEnd(cluster, intents, masks, pods_per_intent, draws, net, Probes(pr, hop_cap),
                     probes_per_intent)

@@ -23,3 +23,12 @@ def sample(n: int, k: int, seed: int = 0) -> np.ndarray:
         return np.arange(n)
     s = np.unique(np.concatenate([[0, n - 1], (st.u64(k) % np.uint64(n)).astype(np.int64)]))
     return s
+
+
+# Small end-to-end batches of the GPU parity tests, shared with the CPU test
+# that shows their expected verdicts tell planted faults apart.
+E2E_PASS_SMALL = dict(seed=21, num_switches=64, num_intents=300, probes_per_intent=200, rules_per_switch=200,
+                      pass_share=0.3)
+E2E_CONSTRAINED = dict(seed=25, num_switches=64, num_intents=300, probes_per_intent=100, rules_per_switch=200,
+                       pass_share=0.3)
+POLICIES_CONSTRAINED = dict(seed=7, forbid_max=1, must_max=2, hubs=6, p_noop=0.3)

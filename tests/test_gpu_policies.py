@@ -2,8 +2,10 @@
 status, hops, last switch and waypoint bits): the backup-switch waypoint
 case, random networks and policies under both first-match kernels, hop caps
 that do and do not reach the forwarding-cycle shortcut, per-probe and
-strided policy indices, the constrained end-to-end verdict, invalid calls,
-and the full end-to-end workload with a policy per intent on sampled probes."""
+strided policy indices, the constrained end-to-end verdict (with intents
+that pass, fail on a missed waypoint or a forbidden switch, or fail for want
+of a concrete flow), invalid calls, and the full end-to-end workload with a
+policy per intent on every output."""
 import numpy as np
 import pytest
 
@@ -11,7 +13,7 @@ import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
 from paper_2602_16100_gb300.validator import flows_of, empty_device, to_device, to_numpy
-from gpu_util import sample
+from gpu_util import E2E_CONSTRAINED, POLICIES_CONSTRAINED
 from test_oracle_policies import _backup_switch_net, _policies
 from netbuild import probe
 
@@ -72,8 +74,9 @@ def test_random_policies(validator, seed, cap, kernel):
 
 
 def test_constrained_end_to_end(validator):
-    e = W.end_to_end(seed=25, num_switches=64, num_intents=300, probes_per_intent=100, rules_per_switch=200)
-    pol = W.path_policies(7, e.network, 300, forbid_max=1, must_max=2, hubs=6, p_noop=0.1)
+    e = W.end_to_end(**E2E_CONSTRAINED)
+    kw = dict(POLICIES_CONSTRAINED)
+    pol = W.path_policies(kw.pop("seed"), e.network, e.intents.num_pods, **kw)
     v = validator
     v.load_cluster(e.cluster)
     v.load_network(e.network)
@@ -100,7 +103,7 @@ def test_constrained_end_to_end(validator):
     assert (to_numpy(hits, np.uint32) == oh).all()
     assert (to_numpy(dev["pass"], np.uint8)[:I] == passed).all()
     assert (to_numpy(dev["counts"], np.uint32, (I, 8)) == counts).all()
-    assert counts[:, 7].any()
+    assert counts[:, 7].any() and passed.any()
 
 
 def test_invalid_policy_calls(validator):
@@ -133,23 +136,31 @@ def test_invalid_policy_calls(validator):
         B.pv_verify_probes_constrained(validator.ctx, 10, pr, 16, None, 10, out, None)
 
 
-def test_full_size_end_to_end_policies_sampled(validator):
+@pytest.mark.parametrize("variant", ["plain", "pass"])
+def test_full_size_end_to_end_policies(validator, variant):
     """The full end-to-end workload (10,000 intents, 50M probes) with one
-    policy per intent; the oracle walks a sample of probes."""
-    e = W.end_to_end()
-    pol = W.path_policies(11, e.network, e.intents.num_pods)
+    policy per intent, in the benchmark's launch configuration (plain), and
+    its variant in which intents can pass (pass); every result, waypoint
+    word, verdict and count is compared with the oracle's."""
+    from test_gpu_reach_e2e import _check_e2e_full
+    e = W.end_to_end(**({"pass_share": 0.3} if variant == "pass" else {}))
+    pol = W.path_policies(20260221, e.network, e.intents.num_pods)
     v = validator
+    v.load_cluster(e.cluster)
     v.load_network(e.network)
     v.load_policies(pol)
-    pr = e.probes.probes.copy()
-    st = W.Stream(12, "full-policy-probes")
-    pr["src_host"] = st.ints(0, e.network.num_hosts - 1, len(pr))
-    pr["src_ip"] = e.network.host_ip[pr["src_host"]]
-    g, gh = _walk(v, e.network, pol, pr, e.probes.hop_cap, per=e.probes_per_intent)
-    idx = sample(len(pr), 20000, seed=5)
-    o, oh = oracle.verify_constrained(e.network, pr, e.probes.hop_cap, pol, probes_per_policy=e.probes_per_intent,
-                                      idx=idx)
-    assert (g[idx] == o).all() and (gh[idx] == oh).all()
+    dev, sizes = v.alloc_end_to_end(e, with_policies=True)
+    v.run_end_to_end(dev, sizes)
+    v.sync()
+    I, words = sizes["intents"], W.words_per_row(e.cluster.num_nodes)
+    g = {"bits": to_numpy(dev["bits"], np.uint32, (I, words)), "flags": to_numpy(dev["flags"], np.uint8),
+         "assign": to_numpy(dev["assign"], np.uint32), "results": to_numpy(dev["results"], W.RESULT_DTYPE),
+         "hits": to_numpy(dev["hits"], np.uint32), "pass": to_numpy(dev["pass"], np.uint8),
+         "counts": to_numpy(dev["counts"], np.uint32, (I, 8))}
+    want = _check_e2e_full(g, e, f"end-to-end-policies/{variant}", pol)
+    assert want["hits"].any()
+    if variant == "pass":
+        assert want["passed"].any()
 
 
 @pytest.mark.parametrize("chunks", [1, 3])
@@ -158,7 +169,8 @@ def test_constrained_pipeline_from_host(validator, chunks):
     (each chunk keeps its intents' policies through first_policy)."""
     import torch
     from test_gpu_reach_e2e import _pinned
-    e = W.end_to_end(seed=26, num_switches=64, num_intents=203, probes_per_intent=80, rules_per_switch=200)
+    e = W.end_to_end(seed=26, num_switches=64, num_intents=203, probes_per_intent=80, rules_per_switch=200,
+                     pass_share=0.3)
     pol = W.path_policies(8, e.network, 203, forbid_max=1, must_max=2, hubs=6, p_noop=0.1)
     v = validator
     v.load_cluster(e.cluster)
@@ -184,6 +196,7 @@ def test_constrained_pipeline_from_host(validator, chunks):
     assert (to_numpy(dev["hits"], np.uint32) == oh).all()
     assert (host["pass"].numpy() == passed).all()
     assert (host["counts"].numpy().view(np.uint32).reshape(I, 8) == counts).all()
+    assert passed.any()
 
 
 @pytest.mark.parametrize("policy_form", ["per_group", "per_probe", "per_pair_of_groups", "none"])

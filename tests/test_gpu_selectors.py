@@ -2,7 +2,7 @@
 both kernels (label-tile comparison and per-value bitset rows), ragged node
 counts spanning several tiles, absent labels, hallucinated values,
 DoesNotExist, malformed expressions, empty inputs, and the placement-scale
-workload (100,000 pods x 5,000 nodes) on sampled pods."""
+workload (100,000 pods x 5,000 nodes) on every row and flag."""
 import numpy as np
 import pytest
 import torch
@@ -11,7 +11,7 @@ import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
 from paper_2602_16100_gb300.validator import empty_device, to_device, to_numpy
-from gpu_util import sample, sub_selectors
+import full_oracle as F
 
 pytestmark = pytest.mark.gpu
 
@@ -110,33 +110,22 @@ def test_empty_and_invalid_calls(validator):
     assert e.value.code == B.PV_EINVAL
 
 
-def test_placement_scale_sampled(validator):
-    """Full placement-scale workload in the benchmark's launch configuration;
-    the oracle recomputes a sample of pods (both ends included)."""
+@pytest.mark.parametrize("kernel", [0, 1])
+def test_placement_scale_full(validator, kernel):
+    """Full placement-scale workload (100,000 pods x 5,000 nodes) in the
+    benchmark's launch configuration (kernel 0: the library's choice, the
+    value-row kernel) and with the comparison kernel (1); every row and
+    flag is compared with the oracle's."""
     d = W.selector_workload()
     c, sel = d["cluster"], d["selectors"]
     validator.load_cluster(c)
     assert B.pv_get_stat(validator.ctx, B.PV_STAT_SELECTOR_ROWS_BUILT) == 1
-    dev = validator.device
     words = W.words_per_row(c.num_nodes)
-    bits, flags = validator.eval_selectors(to_device(sel.expr_offs.astype(np.uint32), dev), len(sel.exprs),
-                                           to_device(sel.exprs, dev), to_device(sel.assign.astype(np.uint32), dev),
-                                           sel.num_pods, words=words)
-    validator.sync()
-    gb = to_numpy(bits, np.uint32, (sel.num_pods, words))
-    gf = to_numpy(flags, np.uint8)
-    idx = sample(sel.num_pods, 3000, seed=1)
-    offs, ex, asg = sub_selectors(sel, idx)
-    ob, of = oracle.eval_selectors(c.num_nodes, c.num_keys, c.labels, offs, ex, asg, words=words)
-    assert (gb[idx] == ob).all() and (gf[idx] == of).all()
-    # the comparison kernel agrees on the same sample
-    validator.set_option(B.PV_OPT_SELECTOR_KERNEL, 1)
-    bits1, flags1 = validator.eval_selectors(to_device(offs, dev), len(ex), to_device(ex, dev),
-                                             to_device(asg, dev), len(idx), words=words)
-    validator.sync()
-    validator.set_option(B.PV_OPT_SELECTOR_KERNEL, 0)
-    assert (to_numpy(bits1, np.uint32, (len(idx), words)) == ob).all()
-    assert (to_numpy(flags1, np.uint8) == of).all()
+    gb, gf = _gpu_eval(validator, c, sel, kernel, words)
+    want = F.cached("placement-scale/default", lambda: dict(zip(("bits", "flags"), F.eval_selectors(c, sel, words))))
+    assert (gf == want["flags"]).all()
+    assert (gb == want["bits"]).all()
+    assert gf.any() and (gf & W.F_PASS).any()
 
 
 @pytest.mark.parametrize("kernel", [1, 2])

@@ -1,7 +1,9 @@
-"""The multi-rank path on CPU: intent-range sharding is exact (two gloo ranks
+"""The multi-rank path on CPU: intent-range sharding is exact (gloo ranks
 each run the oracle pipeline on their own range; the concatenation equals
 the unsharded run), the ranges partition the batch, and the host-side
-max / sum over ranks used by the benchmark's timing behave."""
+reductions the benchmark uses behave: the max over ranks of the timed
+region, and the sums over ranks of the per-status counters and verdict
+counts, which equal the unsharded run's (a batch in which intents pass)."""
 import os
 import socket
 
@@ -16,7 +18,7 @@ from paper_2602_16100_gb300 import workloads as W
 
 def _batch():
     return W.end_to_end(seed=31, num_switches=48, num_intents=37, probes_per_intent=40, rules_per_switch=120,
-                        hop_cap=16)
+                        hop_cap=16, pass_share=0.3)
 
 
 def _pipeline(e):
@@ -49,6 +51,11 @@ def _rank_main(rank, world, port, outdir):
         m = SH.max_over_ranks(10.0 + r, dist)
         s = SH.sum_over_ranks(int(part["pass"].sum()), dist)
         np.save(os.path.join(outdir, f"agg{r}.npy"), np.array([m, s], np.float64))
+        # per-status histogram of the rank's probes, the per-intent counter
+        # columns and the verdict count, summed over ranks
+        local = np.concatenate([np.bincount(part["results"]["status"], minlength=6),
+                                part["counts"].astype(np.int64).sum(axis=0), [int(part["pass"].sum())]])
+        np.save(os.path.join(outdir, f"sums{r}.npy"), SH.sum_vector_over_ranks(local, dist))
         dist.barrier()
     finally:
         dist.destroy_process_group()
@@ -63,9 +70,13 @@ def test_sharded_pipeline_equals_unsharded(tmp_path, world):
     for k in ("bits", "flags", "assign", "probes", "results", "pass", "counts"):
         got = np.concatenate([p[k] for p in parts])
         assert (got == whole[k]).all(), k
+    want = np.concatenate([np.bincount(whole["results"]["status"], minlength=6),
+                           whole["counts"].astype(np.int64).sum(axis=0), [int(whole["pass"].sum())]])
+    assert whole["pass"].sum() > 0
     for r in range(world):
         m, s = np.load(tmp_path / f"agg{r}.npy")
         assert m == 10.0 + world - 1 and s == int(whole["pass"].sum())
+        assert (np.load(tmp_path / f"sums{r}.npy") == want).all()
 
 
 def test_shard_ranges_partition():
@@ -86,3 +97,4 @@ def test_shard_ranges_partition():
 
 def test_single_process_reductions_are_identity():
     assert SH.max_over_ranks(3.5) == 3.5 and SH.sum_over_ranks(4) == 4
+    assert (SH.sum_vector_over_ranks([1, 2, 3]) == [1, 2, 3]).all()
