@@ -1368,7 +1368,11 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
         const bool ok = mbar_wait_bounded(&s_bar, parity, g.wait_ns);
         if (__syncthreads_or(!ok)) {
             // give up: record the timeout, leave an empty slice for the next
-            // hop, let the copy in flight land (bounded again), return
+            // hop, let the copy in flight land (bounded again), return.
+            // Accepted edge case: a copy still in flight after both bounds
+            // (4 s for a copy of at most a few hundred KB) may land after
+            // the block has exited; the call then reports PV_ETIMEOUT and
+            // its results are not to be used.
             if (threadIdx.x == 0) {
                 pv_device_error(g.status, PV_ETIMEOUT);
                 g.next_desc[blockIdx.x] = make_uint2(r0, 0);
