@@ -244,6 +244,9 @@ struct BlobLayout {
         : BlobLayout(hdr.x & 0xFFFFu, hdr.x >> 16, hdr.y, hdr.z, hdr.w) {}
 };
 
+// Bytes of the hop kernel's staged port table ({peer, aux} per port).
+inline size_t port_stage_bytes(uint32_t max_ports) { return ((size_t)max_ports * 8 + 15) & ~(size_t)15; }
+
 // Rules as the linear kernel stages them: the header, then all rules' A and B
 // records from the blob's end.
 __host__ __device__ inline uint32_t linear_bytes(uint32_t npad) { return 16 + npad * 24; }
@@ -1062,6 +1065,7 @@ struct HopArgs {
     PolicyArgs pa;       // path constraints (used by the kPolicy kernels)
     uint32_t *hist_next; // per-switch counts of the next hop's list (null: a separate pass counts)
     uint32_t hist_off;   // byte offset of the block's count array in dynamic shared memory
+    uint32_t port_off;   // byte offset of the staged port table in dynamic shared memory
     unsigned long long *stats;   // [PV_WALK_STATS] counters of the statistics kernels (kStats)
 };
 
@@ -1309,6 +1313,50 @@ __device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t hop, uint
     }
 }
 
+// The hop kernel stages the current switch's ports once per table: port p
+// as {peer, aux}, aux = the region of the peer switch, or the address of
+// the attached host (0 for a host index out of range, which the outcome
+// rejects by its index), so a hop's outcome reads shared memory only.
+__device__ __forceinline__ uint2 port_entry(const HopArgs &g, uint32_t pbase, uint32_t p) {
+    const int32_t peer = g.port_peer[pbase + p];
+    uint32_t aux = 0;
+    if (peer >= 0) {
+        if (peer & PV_PEER_HOST) {
+            const uint32_t q = (uint32_t)(peer & ~PV_PEER_HOST);
+            aux = q < g.H ? g.host_ip[q] : 0u;
+        } else {
+            aux = g.region[(uint32_t)peer >> 8];
+        }
+    }
+    return make_uint2((uint32_t)peer, aux);
+}
+
+// hop_outcome with the port table staged in shared memory (same outcomes).
+__device__ __forceinline__ void hop_outcome_staged(const HopArgs &g, const uint2 *s_port, uint32_t hop, uint32_t fm,
+                                                   uint32_t dst, uint32_t mask, uint32_t nports, uint32_t *status,
+                                                   uint32_t *next) {
+    *next = 0;
+    const uint32_t act = fm & 0xFFFFu;
+    if (!(fm & kWinFound) || act == PV_DROP || act >= nports) {
+        *status = PV_DROPPED;
+        return;
+    }
+    const uint2 pe = s_port[act];
+    const int32_t peer = (int32_t)pe.x;
+    if (peer < 0) {
+        *status = PV_DROPPED;
+    } else if (peer & PV_PEER_HOST) {
+        const uint32_t q = (uint32_t)(peer & ~PV_PEER_HOST);
+        *status = (q < g.H && pe.y == dst) ? PV_COMPLIANT : PV_MISDELIVERED;
+    } else if (hop + 1 >= g.cap) {
+        *status = PV_LOOP;
+    } else {
+        const uint32_t r2 = pe.y;
+        *status = (r2 < 32 && ((mask >> r2) & 1u)) ? kAlive : kViolationNext;
+        *next = (uint32_t)peer;
+    }
+}
+
 template <bool kIndexed, bool kPolicy, bool kStats, bool kRec>
 __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
@@ -1333,6 +1381,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
         s_count = 0;
     }
     uint32_t *s_hist = reinterpret_cast<uint32_t *>(s_raw + g.hist_off);   // [S] when g.hist_next
+    uint2 *s_port = reinterpret_cast<uint2 *>(s_raw + g.port_off);        // [ports of the current switch]
     if (g.hist_next)
         for (uint32_t j = threadIdx.x; j < g.S; j += kHopThreads) s_hist[j] = 0;
     __syncthreads();
@@ -1353,7 +1402,8 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
         const uint4 hdr = __ldg(reinterpret_cast<const uint4 *>(src_blob));
         const BlobLayout L(hdr);
         const uint32_t npad = hdr.x & 0xFFFFu;
-        __syncthreads();   // everyone is done with the previous table
+        const uint32_t pbase = g.port_offs[s], nports = g.port_offs[s + 1] - pbase;
+        __syncthreads();   // everyone is done with the previous table and ports
         if (threadIdx.x == 0) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             if (kIndexed) {   // header, plain rules, index
@@ -1365,6 +1415,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 if (npad) bulk_g2s_keep(s_raw + 16, src_blob + L.fa, npad * 24, &s_bar);
             }
         }
+        for (uint32_t p = threadIdx.x; p < nports; p += kHopThreads) s_port[p] = port_entry(g, pbase, p);
         const bool ok = mbar_wait_bounded(&s_bar, parity, g.wait_ns);
         if (__syncthreads_or(!ok)) {
             // give up: record the timeout, leave an empty slice for the next
@@ -1380,8 +1431,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             mbar_wait_bounded(&s_bar, parity, g.wait_ns);
             return;
         }
-        parity ^= 1u;
-        const uint32_t pbase = g.port_offs[s], nports = g.port_offs[s + 1] - pbase;
+        parity ^= 1u;   // the barrier above also published s_port
         for (uint32_t wb = pos + warp * 32; wb < seg_end; wb += 32 * kHopWarps) {
             const uint32_t cnt = min(32u, seg_end - wb);
             // lane j fetches probe j of this warp's batch; records are then
@@ -1415,7 +1465,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                 const uint32_t fm = first_match_lane<kStats>(s_raw, L, act, pr.x, pr.y, pr.z & 0xFFFFu, e.y & 0xFFu,
                                                              stc[kStRuleTests], stc[kStLookups]);
                 my_fm = fm;
-                if (act) hop_outcome(g, g.hop, fm, pr.y, pr.w, pbase, nports, &my_status, &my_next);
+                if (act) hop_outcome_staged(g, s_port, g.hop, fm, pr.y, pr.w, nports, &my_status, &my_next);
             } else {
                 for (uint32_t j = 0; j < cnt; ++j) {
                     if ((fin_lanes >> j) & 1u) continue;
@@ -1429,7 +1479,7 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
                         kIndexed ? first_match_indexed<kStats>(s_raw, hdr, lane, src, dst, dport, in_port, tests, lookups)
                                  : first_match_linear<kStats>(s_raw, npad, lane, src, dst, dport, in_port, tests);
                     uint32_t status, next;
-                    hop_outcome(g, g.hop, fm, dst, mask, pbase, nports, &status, &next);
+                    hop_outcome_staged(g, s_port, g.hop, fm, dst, mask, nports, &status, &next);
                     if (lane == j) {
                         my_status = status;
                         my_next = next;
@@ -1635,7 +1685,7 @@ inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 // structure on the host and queued the uploads and the index-size pass; the
 // second reads the sizes back, builds the blobs and installs the tables.
 struct pv_table_load {
-    uint32_t S = 0, H = 0, P = 0, max_pad = 0, max_rules = 0;
+    uint32_t S = 0, H = 0, P = 0, max_pad = 0, max_rules = 0, max_ports = 0;
     const uint32_t *rule_offs = nullptr, *port_offs = nullptr, *host_ip = nullptr;
     const pv_rule *rules = nullptr;
     const uint8_t *switch_region = nullptr;
@@ -1684,6 +1734,7 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
     tab.assign(S + 1, 0);
     uint32_t &max_pad = L.max_pad;
     max_pad = 0;
+    L.max_ports = 0;
     for (uint32_t s = 0; s < S; ++s) {
         if (rule_offs[s + 1] < rule_offs[s] || port_offs[s + 1] < port_offs[s])
             return pv_fail(ctx, PV_EINVAL, "offsets not monotone at switch %u", s);
@@ -1694,6 +1745,7 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
         const uint32_t pad = (nr + 31) / 32 * 32;
         tab[s + 1] = tab[s] + pad;
         max_pad = std::max(max_pad, pad);
+        L.max_ports = std::max(L.max_ports, np);
     }
     const uint32_t R = rule_offs[S], P = port_offs[S];
     if (R && !rules) return pv_fail(ctx, PV_EINVAL, "NULL rules");
@@ -1921,9 +1973,11 @@ int tables_end(pv_ctx *ctx, pv_table_load &L) {
     // on average) it pays from hop 5 on, with long ones only from hop 8.
     t.tail_hop = all_items <= (uint64_t)kTailEarlyItems * kBuckets * S ? 5u : 8u;
     t.max_rules_padded = max_pad;
+    t.max_ports = L.max_ports;
     t.max_blob_bytes = max_blob;
     t.max_linear_bytes = max_linear;
-    const size_t smem_cap = ctx->max_smem_optin - 1024;
+    // the hop kernel stages the port table after the table (16-byte aligned)
+    const size_t smem_cap = ctx->max_smem_optin - 1024 - 16 - port_stage_bytes(t.max_ports);
     t.index_fits = max_blob <= smem_cap;
     if (max_linear > smem_cap) {
         pv_free_tables(ctx, t);
@@ -2034,9 +2088,13 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     const size_t table_smem = indexed ? t.max_blob_bytes : t.max_linear_bytes;
     // the next hop's per-switch counts ride in the hop kernel's shared memory
     // after the staged table, when they fit
+    // (and the current switch's port table after both)
     const size_t hist_off = (table_smem + 15) & ~(size_t)15;
-    const bool fuse_hist = S <= kSmemHistMax && hist_off + (size_t)S * 4 <= ctx->max_smem_optin - 1024;
-    const size_t hop_smem = fuse_hist ? hist_off + (size_t)S * 4 : table_smem;
+    const size_t port_bytes = port_stage_bytes(t.max_ports);
+    const bool fuse_hist =
+        S <= kSmemHistMax && hist_off + (size_t)S * 4 + 16 + port_bytes <= ctx->max_smem_optin - 1024;
+    const size_t port_off = fuse_hist ? ((hist_off + (size_t)S * 4 + 15) & ~(size_t)15) : hist_off;
+    const size_t hop_smem = port_off + port_bytes;
     int hop_blocks_per_sm = 0;
     const bool stats = ctx->opt_walk_stats != 0;
     // compact flows with one path constraint per group are placed directly
@@ -2166,6 +2224,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.pa = pol ? *pa : no_policy;
     g.hist_next = nullptr;
     g.hist_off = (uint32_t)hist_off;
+    g.port_off = (uint32_t)port_off;
     g.stats = ctx->d_walk_stats;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;

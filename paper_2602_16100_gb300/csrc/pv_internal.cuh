@@ -40,6 +40,7 @@ struct pv_table_state {
     uint32_t max_blob_bytes = 0;      // largest stage of the indexed kernel (all but the full rule list)
     uint32_t tail_hop = 8;            // default first tail hop for these tables (see walk_probes)
     uint32_t max_linear_bytes = 0;    // largest header + full rule list (linear-scan kernel)
+    uint32_t max_ports = 0;           // most ports on one switch
     bool index_fits = false;          // every blob fits shared memory
     uint8_t *d_region = nullptr;      // [S]
     uint32_t *d_port_offs = nullptr;  // [S + 1]
