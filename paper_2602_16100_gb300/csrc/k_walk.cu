@@ -1066,6 +1066,7 @@ struct HopArgs {
     uint32_t *hist_next; // per-switch counts of the next hop's list (null: a separate pass counts)
     uint32_t hist_off;   // byte offset of the block's count array in dynamic shared memory
     uint32_t port_off;   // byte offset of the staged port table in dynamic shared memory
+    uint32_t recs_at_position;   // 1: entry i's record index is i (first hop of directly placed flows)
     unsigned long long *stats;   // [PV_WALK_STATS] counters of the statistics kernels (kStats)
 };
 
@@ -1127,6 +1128,23 @@ __device__ __forceinline__ uint4 load_header(const HopArgs &g, uint32_t x, uint3
     }
     *id = x;
     return __ldg(reinterpret_cast<const uint4 *>(g.probes) + x);
+}
+
+// The same in two steps, so the record's load can run ahead of its use:
+// the record (or probe) at index x, then the header and probe id from it.
+template <bool kRec>
+__device__ __forceinline__ uint4 load_raw(const HopArgs &g, uint32_t x) {
+    return kRec ? __ldg(g.recs + x) : __ldg(reinterpret_cast<const uint4 *>(g.probes) + x);
+}
+
+template <bool kRec>
+__device__ __forceinline__ uint4 header_of(const HopArgs &g, uint4 raw, uint32_t x, uint32_t *id) {
+    if (kRec) {
+        *id = raw.x;
+        return make_uint4(__ldg(g.host_ip + (raw.z >> 16)), raw.y, raw.z, raw.w);
+    }
+    *id = x;
+    return raw;
 }
 
 template <bool kStats>
@@ -1358,7 +1376,7 @@ __device__ __forceinline__ void hop_outcome_staged(const HopArgs &g, const uint2
 }
 
 template <bool kIndexed, bool kPolicy, bool kStats, bool kRec>
-__global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
+__global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
     __shared__ uint64_t s_bar;
     __shared__ uint32_t s_count;
@@ -1432,17 +1450,30 @@ __global__ void __launch_bounds__(kHopThreads, 5) walk_hop_kernel(HopArgs g) {
             return;
         }
         parity ^= 1u;   // the barrier above also published s_port
-        for (uint32_t wb = pos + warp * 32; wb < seg_end; wb += 32 * kHopWarps) {
+        // Lane j handles probe j of each batch of 32.  Loads run ahead of the
+        // batch in hand: the list entry two batches ahead and the record one
+        // batch ahead (its index comes from the entry fetched a batch
+        // earlier), so neither waits on the other or on the batch's work.
+        constexpr uint32_t kStride = 32 * kHopWarps;
+        const uint32_t wb0 = pos + warp * 32;
+        uint2 e1 = make_uint2(0, 0), e2 = make_uint2(0, 0);   // entries of batches wb, wb + kStride
+        uint4 raw1 = make_uint4(0, 0, 0, 0);                  // record of batch wb
+        if (wb0 + lane < seg_end) {
+            e1 = g.sorted[wb0 + lane];
+            raw1 = load_raw<kRec>(g, g.recs_at_position ? wb0 + lane : e1.x);
+        }
+        if (wb0 + kStride + lane < seg_end) e2 = g.sorted[wb0 + kStride + lane];
+        for (uint32_t wb = wb0; wb < seg_end; wb += kStride) {
             const uint32_t cnt = min(32u, seg_end - wb);
-            // lane j fetches probe j of this warp's batch; records are then
-            // broadcast one at a time with shuffles
-            uint2 e = make_uint2(0, 0);
+            const uint2 e = e1;
+            const uint4 raw = raw1;
+            if (wb + kStride + lane < seg_end)
+                raw1 = load_raw<kRec>(g, g.recs_at_position ? wb + kStride + lane : e2.x);
+            e1 = e2;
+            if (wb + 2 * kStride + lane < seg_end) e2 = g.sorted[wb + 2 * kStride + lane];
             uint4 pr = make_uint4(0, 0, 0, 0);   // {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
             uint32_t pid = 0;                     // probe id
-            if (lane < cnt) {
-                e = g.sorted[wb + lane];
-                pr = load_header<kRec>(g, e.x, &pid);
-            }
+            if (lane < cnt) pr = header_of<kRec>(g, raw, e.x, &pid);
             // a probe in a known forwarding cycle that has reached its finish hop
             const uint32_t fin = e.y >> 24;
             const bool fin_now = lane < cnt && fin != 0 && fin - 1 == g.hop;
@@ -2225,6 +2256,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.hist_next = nullptr;
     g.hist_off = (uint32_t)hist_off;
     g.port_off = (uint32_t)port_off;
+    g.recs_at_position = 0;
     g.stats = ctx->d_walk_stats;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
@@ -2251,6 +2283,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         g.hist_next = (fuse_hist && h + 1 < tail_hop) ? hist : nullptr;
         g.sorted = sorted;
         g.hop = h;
+        g.recs_at_position = (direct && h == 0) ? 1u : 0u;
         g.next_list = nxt;
         g.next_desc = dnxt;
         pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
