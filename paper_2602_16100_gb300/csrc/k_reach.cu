@@ -226,10 +226,28 @@ __host__ __device__ inline uint32_t up16u(uint32_t x) { return (x + 15u) & ~15u;
 
 // Component labels of one mask per block: lab[m][v] = the smallest vertex
 // of v's component in the permitted subgraph, kNoLabel for a vertex whose
-// region the mask does not permit.  Before the union pass every permitted
-// vertex points at its smallest permitted neighbour below it (a valid
-// forest of the same components, so most unions then find one root).
+// region the mask does not permit.  One pass over the pair list (from L2)
+// points every permitted vertex at its smallest permitted neighbour below
+// it (a valid forest of the same components, so most unions then find one
+// root) and copies the pairs inside the permitted subgraph, usually a small
+// share of them, to shared memory; the union pass then runs over that
+// compact list (over the whole list again when it did not fit).
 constexpr int kLabelThreads = 1024;
+constexpr size_t kLabelSmemTarget = 100 * 1024;   // two label blocks per SM
+
+// Layout of the labels kernel's dynamic shared memory for V vertices:
+// parent[V], the permitted-vertex bitmap, then the compact pair list.
+struct LabelSmem {
+    uint32_t allow, pairs, cap;
+    size_t total;
+    __host__ __device__ explicit LabelSmem(uint32_t V) {
+        allow = up16u(V * 4);
+        pairs = allow + up16u(((V + 31) / 32) * 4);
+        const size_t left = kLabelSmemTarget > pairs ? kLabelSmemTarget - pairs : 0;
+        cap = (uint32_t)(left / 4) & ~3u;
+        total = (size_t)pairs + (size_t)cap * 4;
+    }
+};
 
 __global__ void __launch_bounds__(kLabelThreads) reach_labels_kernel(
     uint32_t V, const uint32_t *__restrict__ pairs, const uint32_t *__restrict__ npairs,
@@ -237,8 +255,11 @@ __global__ void __launch_bounds__(kLabelThreads) reach_labels_kernel(
     const uint32_t *asym, int32_t *status) {
     if (*(volatile const uint32_t *)asym) return;       // not symmetric: the sweep kernel runs
     extern __shared__ __align__(16) uint8_t s_dyn[];
+    __shared__ uint32_t s_np;                                                      // compact pairs
+    const LabelSmem L(V);
     volatile uint32_t *parent = reinterpret_cast<uint32_t *>(s_dyn);              // [V]
-    uint32_t *s_allow = reinterpret_cast<uint32_t *>(s_dyn + up16u(V * 4));        // [ceil(V / 32)]
+    uint32_t *s_allow = reinterpret_cast<uint32_t *>(s_dyn + L.allow);            // [ceil(V / 32)]
+    uint32_t *s_pairs = reinterpret_cast<uint32_t *>(s_dyn + L.pairs);            // [L.cap]
     const uint32_t t = threadIdx.x, lane = t & 31, warp = t >> 5, nt = blockDim.x;
     const uint32_t m = blockIdx.x, mask = masks[m];
     auto allowed = [&](uint32_t v) { return (s_allow[v >> 5] >> (v & 31)) & 1u; };
@@ -254,28 +275,52 @@ __global__ void __launch_bounds__(kLabelThreads) reach_labels_kernel(
         const uint32_t bal = __ballot_sync(PV_FULL_MASK, ok);
         if (lane == 0 && v0 + warp * 32 < V) s_allow[(v0 >> 5) + warp] = bal;
     }
+    if (t == 0) s_np = 0;
     __syncthreads();
-    // each permitted vertex under its smallest permitted neighbour
+    // each permitted vertex under its smallest permitted neighbour; the
+    // pairs inside the permitted subgraph copied to the compact list
     const uint32_t np = *npairs;
-    for (uint32_t i = 4 * t; i < np; i += 4 * nt) {
-        const uint4 q = *reinterpret_cast<const uint4 *>(pairs + i);
-        const uint32_t pq[4] = {q.x, q.y, q.z, q.w};
+    for (uint32_t i0 = 0; i0 < np; i0 += 4 * nt) {
+        const uint32_t i = i0 + 4 * t;
+        uint32_t pq[4] = {0, 0, 0, 0};
+        if (i < np) {
+            const uint4 q = *reinterpret_cast<const uint4 *>(pairs + i);
+            pq[0] = q.x;
+            pq[1] = q.y;
+            pq[2] = q.z;
+            pq[3] = q.w;
+        }
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const uint32_t u = pq[k] >> 16, v = pq[k] & 0xFFFFu;   // v < u
-            if (i + k < np && allowed(u) && allowed(v)) atomicMin(const_cast<uint32_t *>(parent + u), v);
+            const bool in = i + k < np && allowed(u) && allowed(v);
+            if (in) atomicMin(const_cast<uint32_t *>(parent + u), v);
+            const uint32_t bal = __ballot_sync(PV_FULL_MASK, in);
+            uint32_t base = 0;
+            if (lane == 0 && bal) base = atomicAdd(&s_np, (uint32_t)__popc(bal));
+            base = __shfl_sync(PV_FULL_MASK, base, 0) + __popc(bal & ((1u << lane) - 1u));
+            if (in && base < L.cap) s_pairs[base] = pq[k];
         }
     }
     __syncthreads();
     // union the endpoints of every undirected edge inside the permitted
-    // vertices (the pair list holds each once; four pairs per load)
-    for (uint32_t i = 4 * t; i < np; i += 4 * nt) {
-        const uint4 q = *reinterpret_cast<const uint4 *>(pairs + i);
-        const uint32_t pq[4] = {q.x, q.y, q.z, q.w};
+    // vertices (each pair once): from the compact list, or from the whole
+    // list again when the compact one overflowed
+    const uint32_t nc = s_np;
+    if (nc <= L.cap) {
+        for (uint32_t i = t; i < nc; i += nt) {
+            const uint32_t p = s_pairs[i];
+            uf_union(parent, p >> 16, p & 0xFFFFu, 2 * V + 2, status);
+        }
+    } else {
+        for (uint32_t i = 4 * t; i < np; i += 4 * nt) {
+            const uint4 q = *reinterpret_cast<const uint4 *>(pairs + i);
+            const uint32_t pq[4] = {q.x, q.y, q.z, q.w};
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const uint32_t u = pq[k] >> 16, v = pq[k] & 0xFFFFu;
-            if (i + k < np && allowed(u) && allowed(v)) uf_union(parent, u, v, 2 * V + 2, status);
+            for (int k = 0; k < 4; ++k) {
+                const uint32_t u = pq[k] >> 16, v = pq[k] & 0xFFFFu;
+                if (i + k < np && allowed(u) && allowed(v)) uf_union(parent, u, v, 2 * V + 2, status);
+            }
         }
     }
     __syncthreads();
@@ -487,7 +532,7 @@ cudaError_t reach_smem_limits() {
     e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     if (e != cudaSuccess) return e;
     const int rows_max = optin - 1024;
-    const int lab_max = (int)(up16u(kReachMaxV * 4) + up16u(kReachMaxV / 32 * 4));
+    const int lab_max = (int)LabelSmem(kReachMaxV).total;
     const int bfs_max = (int)(kReachMaxV * 8);
     if ((e = cudaFuncSetAttribute(reach_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, rows_max)) !=
             cudaSuccess ||
@@ -534,7 +579,7 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
     // does not fit (rows then come straight from the ballots)
     uint32_t cap = 0;
     size_t rows_smem = 0;
-    const size_t lab_smem = up16u(V * 4) + up16u(((V + 31) / 32) * 4);
+    const size_t lab_smem = LabelSmem(V).total;
     const size_t limit = ctx->max_smem_optin - 1024;
     if (comp) {
         const size_t fixed = RowSmem(V, words_per_row, 0).total;
