@@ -161,6 +161,9 @@ def _walk_entries(v):
 # ----------------------------------------------------------------------------
 # workloads
 # ----------------------------------------------------------------------------
+INPUT_KEYS = ("offs", "exprs", "draws", "masks", "dst", "dport")   # host-buffer step inputs
+
+
 class EndToEndBench:
     name = "end-to-end cross-layer"
     unit = "probe-hop verifications/s"
@@ -179,7 +182,7 @@ class EndToEndBench:
                 "label_keys": e.cluster.num_keys, "switches": e.network.num_switches,
                 "rules_per_switch": int(np.diff(e.network.rule_offs).max()), "pods_per_intent": e.pods_per_intent,
                 "probes": len(e.probes.probes), "hop_cap": e.probes.hop_cap,
-                "l2": "inputs larger than L2 (400 MB of flows in, 800 MB of probe records built and 200 MB of results per step)",
+                "l2": "inputs larger than L2 (300 MB of flow columns in, a 16-byte walk record built per listed flow, 200 MB of results per step)",
                 **({"path_policies": self.pol.num_policies, "forbidden_switches": len(self.pol.forbid),
                     "waypoints": len(self.pol.must)} if self.pol is not None else {})}
 
@@ -246,17 +249,18 @@ class EndToEndBench:
         import torch
         e = self.e
         pin = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.uint8).reshape(-1).copy()).pin_memory()
-        from paper_2602_16100_gb300.validator import flows_of
+        from paper_2602_16100_gb300.validator import flow_columns_of
+        dst, dport = flow_columns_of(e)
         self.host = {"offs": pin(e.intents.expr_offs.astype(np.uint32)), "exprs": pin(e.intents.exprs),
                      "draws": pin(e.place_draws.astype(np.uint64)), "masks": pin(e.intent_mask.astype(np.uint32)),
-                     "flows": pin(flows_of(e)),
+                     "dst": pin(dst), "dport": pin(dport),
                      "pass": torch.empty(e.intents.num_pods, dtype=torch.uint8).pin_memory(),
                      "counts": torch.empty(e.intents.num_pods * 32, dtype=torch.uint8).pin_memory()}
         self.copy_stream = torch.cuda.Stream()
         self.chunks = chunks
         self.loads_first = getattr(self, "loads_first", True)
         net = e.network
-        self.h2d = (sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "masks", "flows"))
+        self.h2d = (sum(self.host[k].numel() for k in INPUT_KEYS)
                     + e.cluster.labels.nbytes + net.rule_offs.nbytes + net.rules.nbytes + net.switch_region.nbytes
                     + net.port_offs.nbytes + net.port_peer.nbytes + net.host_switch.nbytes + net.host_port.nbytes
                     + net.host_ip.nbytes)
@@ -298,7 +302,7 @@ class EndToEndBench:
         t0 = time.perf_counter()
         for _ in range(reps):
             with torch.cuda.stream(self.copy_stream):
-                for k in ("offs", "exprs", "draws", "masks", "flows"):
+                for k in INPUT_KEYS:
                     self.dev[k][: self.host[k].numel()].copy_(self.host[k], non_blocking=True)
         torch.cuda.synchronize()
         upload = (time.perf_counter() - t0) / reps
@@ -307,7 +311,7 @@ class EndToEndBench:
             self.v.run_end_to_end(self.dev, self.sizes, stream)
         torch.cuda.synchronize()
         dev = (time.perf_counter() - t0) / reps
-        up_bytes = sum(self.host[k].numel() for k in ("offs", "exprs", "draws", "masks", "flows"))
+        up_bytes = sum(self.host[k].numel() for k in INPUT_KEYS)
         return {"load_tables_ms": load * 1e3, "upload_inputs_ms": upload * 1e3,
                 "upload_gbs": up_bytes / upload / 1e9, "device_pipeline_ms": dev * 1e3}
 

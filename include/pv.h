@@ -367,6 +367,10 @@ int pv_compliant_reach_noalloc(uint32_t V, const uint32_t *d_offs, uint32_t num_
  *   walk record in the library's scratch; otherwise the first hop is
  *   regrouped like any other.  pv_verify_flows_constrained is the same with
  *   the path constraints of pv_verify_probes_constrained.
+ * pv_verify_flow_columns(_constrained): the same calls with the flows as two
+ *   columns, d_dst_ip[k] (4-byte aligned) and d_dport[k] (2-byte aligned):
+ *   6 bytes per flow instead of the 8 of a pv_flow record, which is what a
+ *   caller uploading its flows from host memory pays for.  Same results.
  * pv_aggregate_intents: d_pass[g] = 1 iff every pod of g has d_assign in
  *   row g, d_group_flags[g] has neither PV_F_UNKNOWN_VALUE nor
  *   PV_F_BAD_EXPR, and every probe of g is PV_COMPLIANT.
@@ -385,6 +389,16 @@ int pv_verify_flows_constrained(pv_ctx *ctx, uint32_t num_probes, const pv_flow 
                                 uint32_t hop_cap, const uint32_t *d_probe_policy, uint32_t probes_per_policy,
                                 uint32_t first_policy, pv_probe *d_probes, pv_result *d_out, uint32_t *d_waypoints,
                                 pv_stream stream);
+int pv_verify_flow_columns(pv_ctx *ctx, uint32_t num_probes, const uint32_t *d_dst_ip, const uint16_t *d_dport,
+                           uint32_t probes_per_group, uint32_t pods_per_group, const uint32_t *d_assign,
+                           const uint32_t *d_group_mask, uint32_t hop_cap, pv_probe *d_probes, pv_result *d_out,
+                           pv_stream stream);
+int pv_verify_flow_columns_constrained(pv_ctx *ctx, uint32_t num_probes, const uint32_t *d_dst_ip,
+                                       const uint16_t *d_dport, uint32_t probes_per_group, uint32_t pods_per_group,
+                                       const uint32_t *d_assign, const uint32_t *d_group_mask, uint32_t hop_cap,
+                                       const uint32_t *d_probe_policy, uint32_t probes_per_policy,
+                                       uint32_t first_policy, pv_probe *d_probes, pv_result *d_out,
+                                       uint32_t *d_waypoints, pv_stream stream);
 int pv_place_pods(pv_ctx *ctx, uint32_t num_groups, uint32_t pods_per_group, const uint32_t *d_bits,
                   uint32_t words_per_row, const uint64_t *d_draws, uint32_t *d_assign, pv_stream stream);
 int pv_bind_probes(pv_ctx *ctx, uint32_t num_probes, pv_probe *d_probes, uint32_t probes_per_group,

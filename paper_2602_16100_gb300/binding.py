@@ -35,7 +35,8 @@ SYMBOLS = ("pv_create", "pv_destroy", "pv_last_error", "pv_sync", "pv_version", 
            "pv_profile_enable", "pv_profile_collect", "pv_profile_read", "pv_compliant_reach_noalloc",
            "pv_load_path_policies", "pv_verify_probes_constrained", "pv_aggregate_constrained",
            "pv_eval_selector_terms", "pv_schedule_paths", "pv_compile_path_rules", "pv_install_path_rules",
-           "pv_bind_flows", "pv_verify_flows", "pv_verify_flows_constrained", "pv_load_flow_tables_begin",
+           "pv_bind_flows", "pv_verify_flows", "pv_verify_flows_constrained", "pv_verify_flow_columns",
+           "pv_verify_flow_columns_constrained", "pv_load_flow_tables_begin",
            "pv_load_flow_tables_end")
 
 #: kernel groups timed by the library profiler (PV_K_* in include/pv.h)
@@ -83,6 +84,9 @@ def load_library(path: Optional[str] = None):
         "pv_verify_flows": (ctypes.c_int, [vp, u32, vp, u32, u32, vp, vp, u32, vp, vp, vp]),
         "pv_verify_flows_constrained": (ctypes.c_int, [vp, u32, vp, u32, u32, vp, vp, u32, vp, u32, u32, vp, vp, vp,
                                                        vp]),
+        "pv_verify_flow_columns": (ctypes.c_int, [vp, u32, vp, vp, u32, u32, vp, vp, u32, vp, vp, vp]),
+        "pv_verify_flow_columns_constrained": (ctypes.c_int, [vp, u32, vp, vp, u32, u32, vp, vp, u32, vp, u32, u32,
+                                                              vp, vp, vp, vp]),
         "pv_aggregate_intents": (ctypes.c_int, [vp, u32, u32, vp, u32, vp, vp, u32, vp, vp, vp, vp]),
         "pv_set_option": (ctypes.c_int, [vp, ctypes.c_int, i64]),
         "pv_get_stat": (ctypes.c_int, [vp, ctypes.c_int, ctypes.POINTER(i64)]),
@@ -347,6 +351,22 @@ def pv_verify_flows_constrained(ctx, num_probes, d_flows, probes_per_group, pods
         ctx, num_probes, _dev(d_flows), probes_per_group, pods_per_group, _dev(d_assign), _dev(d_group_mask),
         hop_cap, _dev(d_probe_policy), probes_per_policy, first_policy, _dev(d_probes), _dev(d_out),
         _dev(d_waypoints), _stream(stream)))
+
+
+def pv_verify_flow_columns(ctx, num_probes, d_dst_ip, d_dport, probes_per_group, pods_per_group, d_assign,
+                           d_group_mask, hop_cap, d_probes, d_out, stream=None) -> int:
+    return _check(ctx, load_library().pv_verify_flow_columns(
+        ctx, num_probes, _dev(d_dst_ip), _dev(d_dport), probes_per_group, pods_per_group, _dev(d_assign),
+        _dev(d_group_mask), hop_cap, _dev(d_probes), _dev(d_out), _stream(stream)))
+
+
+def pv_verify_flow_columns_constrained(ctx, num_probes, d_dst_ip, d_dport, probes_per_group, pods_per_group,
+                                       d_assign, d_group_mask, hop_cap, d_probe_policy, probes_per_policy,
+                                       first_policy, d_probes, d_out, d_waypoints, stream=None) -> int:
+    return _check(ctx, load_library().pv_verify_flow_columns_constrained(
+        ctx, num_probes, _dev(d_dst_ip), _dev(d_dport), probes_per_group, pods_per_group, _dev(d_assign),
+        _dev(d_group_mask), hop_cap, _dev(d_probe_policy), probes_per_policy, first_policy, _dev(d_probes),
+        _dev(d_out), _dev(d_waypoints), _stream(stream)))
 
 
 def pv_aggregate_intents(ctx, num_groups, pods_per_group, d_bits, words_per_row, d_group_flags, d_assign,

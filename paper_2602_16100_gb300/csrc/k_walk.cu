@@ -653,12 +653,25 @@ __device__ __forceinline__ bool switch_listed(const uint16_t *list, uint32_t n, 
 // kBind, the probe records are first built from compact flows and the
 // placement (the binding of pv_bind_flows) and written for the later hops.
 struct BindArgs {
-    const uint2 *flows;          // [M] {dst_ip, dport}
+    // flow i: destination address dst[i * dst_stride], port dport[i * dport_stride]
+    // (records {dst_ip, dport, 0}: strides 2 and 4; columns: 1 and 1)
+    const uint32_t *dst;
+    const uint16_t *dport;
+    uint32_t dst_stride, dport_stride;
     uint32_t ppg, pods;          // probes and pods per group
     const uint32_t *assign;      // [groups * pods]
     const uint32_t *group_mask;  // [groups]
     const uint32_t *host_ip;     // [H]
 };
+
+// Flow i as {dst_ip, dport}.
+__device__ __forceinline__ uint2 flow_at(const BindArgs &ba, uint32_t i) {
+    return make_uint2(__ldg(ba.dst + (size_t)i * ba.dst_stride), __ldg(ba.dport + (size_t)i * ba.dport_stride));
+}
+
+__device__ __forceinline__ uint32_t flow_dport(const BindArgs &ba, uint32_t i) {
+    return __ldg(ba.dport + (size_t)i * ba.dport_stride);
+}
 
 template <bool kPolicy, bool kBind>
 __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
@@ -685,7 +698,7 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
             if (kBind) {
                 const uint32_t grp = i / ba.ppg;
                 const uint32_t node = ba.assign[grp * ba.pods + (i - grp * ba.ppg) % ba.pods];
-                const uint2 f = __ldg(ba.flows + i);
+                const uint2 f = flow_at(ba, i);
                 const bool placed = node < H;
                 pr = make_uint4(placed ? ba.host_ip[node] : 0u, f.x,
                                 (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16, ba.group_mask[grp]);
@@ -739,9 +752,10 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
 // adds each listed pair's probe count to its source switch (the first hop's
 // per-switch counts) and keeps the pair's offset within that switch; after
 // the scan, the walk's first kernel binds every probe and writes its walk
-// record and list entry straight to its slot in the switch-sorted list
-// (switch start + pair offset + rank within the pair), so the first hop
-// needs no regroup.  walk_init_group_kernel (below) does so one group per
+// record straight to its slot in the first hop's switch order (switch start
+// + pair offset + rank within the pair), so the first hop needs neither a
+// regroup nor a list: it reads records by position and takes each in_port
+// from the record's source host.  walk_init_group_kernel (below) does so one group per
 // block with each pair's run in bucket order; walk_init_direct_kernel is the
 // grid-stride form for groups too large for its shared memory.  Probe i
 // belongs to group i / ppg and pod (i mod ppg) mod pods; the caller
@@ -781,13 +795,13 @@ __global__ void __launch_bounds__(kGridThreads) flow_groups_kernel(uint32_t M, u
 template <bool kPolicy>
 __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
     uint32_t M, pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
-    const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
-    uint2 *__restrict__ sorted, uint4 *__restrict__ recs, const uint32_t *__restrict__ seg,
+    const uint8_t *__restrict__ region, pv_result *__restrict__ out, uint4 *__restrict__ recs,
+    const uint32_t *__restrict__ seg,
     const uint32_t *__restrict__ pair_off, PolicyArgs pa, BindArgs ba) {
     for (uint32_t i = blockIdx.x * blockDim.x + threadIdx.x; i < M; i += gridDim.x * blockDim.x) {
         const uint32_t grp = i / ba.ppg, r = i - grp * ba.ppg, g = grp * ba.pods + r % ba.pods;
         const uint32_t node = ba.assign[g];
-        const uint2 f = __ldg(ba.flows + i);
+        const uint2 f = flow_at(ba, i);
         const bool placed = node < H;
         const uint32_t mask = ba.group_mask[grp];
         const uint32_t z = (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16;
@@ -806,7 +820,6 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
         if (first_switch_permitted<kPolicy>(pa, i, s, region[s], mask)) {
             const uint32_t slot = seg[s] + pair_off[g] + r / ba.pods;
             recs[slot] = make_uint4(i, f.x, z, mask);
-            sorted[slot] = make_uint2(slot, (s << 8) | host_port[node]);
         } else {
             res.status = PV_VIOLATION;
             res.hops = 1;
@@ -818,28 +831,111 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
 
 // The same placement by one block per group, with each pair's run ordered
 // by destination-port bucket of the first-match index, so the lanes of a
-// first-hop warp mostly read the same few candidate lists.  The block counts
-// its probes per (pod, bucket) in shared memory, binds and judges them in one
-// coalesced pass that drops each listed probe (destination, rank in the
-// group, port) into its pod's run in shared memory (the next slot of its
-// bucket), then writes every run out whole as walk records, so each sector
-// of the list and the records is written at once.
-// Used when the counts and the group's records fit kGroupInitSmem.
+// first-hop warp mostly read the same few candidate lists.  The block brings
+// its group's slice of the flows into shared memory with bulk copies (one
+// per column, or one for records; the few elements outside the copies'
+// 16-byte-aligned middles by plain loads), counts its probes per (pod,
+// bucket), binds and judges them in one pass that drops each listed probe's
+// rank into its pod's run (the next slot of its bucket), then writes every
+// run out whole as walk records, so each sector of the records is written
+// at once.  Used when the counts, ranks and flow slices fit
+// kGroupInitSmem.
 constexpr uint32_t kGroupInitMaxPods = 16;
 constexpr uint32_t kGroupInitThreads = 512;
 constexpr size_t kGroupInitSmem = 64 * 1024;   // ppg <= 65535 also fits the rank's 16 bits
 
+// Shared-memory layout of walk_init_group_kernel: bucket counts / run
+// slots [pods][kBuckets], ranks [ppg], then the destination slice and the
+// port slice (the same slice for records), each with 16 bytes of slack so
+// that its elements keep their global address modulo 16.
+struct GroupInitSmem {
+    uint32_t rank, dst, dport, total;
+    __host__ __device__ GroupInitSmem(uint32_t pods, uint32_t ppg, bool records) {
+        rank = pods * kBuckets * 4;
+        dst = rank + ((ppg * 2 + 15) & ~15u);
+        dport = dst + (records ? 0u : ((ppg * 4 + 16 + 15) & ~15u));
+        total = dport + (records ? ppg * 8 + 16 : ((ppg * 2 + 16 + 15) & ~15u));
+    }
+};
+
+// A slice of n elements of es bytes at global address src, staged in
+// shared memory from s_base + (src mod 16), so that its 16-byte-aligned
+// middle [b0, b1) can come by one bulk copy; the elements outside it
+// (at most 15 bytes at each end, or all of them when there is no middle)
+// come by plain loads.
+struct Slice {
+    uintptr_t a0, b0, b1;
+    uint32_t n, es;
+    __device__ Slice(const void *src, uint32_t n_, uint32_t es_) : n(n_), es(es_) {
+        a0 = reinterpret_cast<uintptr_t>(src);
+        b0 = (a0 + 15) & ~(uintptr_t)15;
+        b1 = (a0 + (uintptr_t)n * es) & ~(uintptr_t)15;
+        if (b1 < b0) b1 = b0;
+    }
+    __device__ uint32_t bulk_bytes() const { return (uint32_t)(b1 - b0); }
+    __device__ uint8_t *staged(uint8_t *s_base) const { return s_base + (a0 & 15); }
+};
+
+// Thread 0 (after the barrier's expect-tx): the slice's bulk copy on bar.
+__device__ __forceinline__ void slice_copy(const Slice &sl, uint8_t *s_base, uint64_t *bar) {
+    if (sl.b1 > sl.b0)
+        bulk_g2s_keep(sl.staged(s_base) + (sl.b0 - sl.a0), reinterpret_cast<const void *>(sl.b0), sl.bulk_bytes(),
+                      bar);
+}
+
+// All threads: the slice's elements outside the bulk copy.
+__device__ __forceinline__ void slice_edges(const Slice &sl, uint8_t *s_base) {
+    const uint32_t n = sl.n, es = sl.es;
+    const bool body = sl.b1 > sl.b0;
+    const uint32_t lo = body ? (uint32_t)((sl.b0 - sl.a0) / es) : n;
+    const uint32_t hi = body ? (uint32_t)((sl.b1 - sl.a0) / es) : n;
+    uint8_t *dst = sl.staged(s_base);
+    const void *src = reinterpret_cast<const void *>(sl.a0);
+    for (uint32_t k = threadIdx.x; k < lo; k += blockDim.x) {
+        if (es == 2) reinterpret_cast<uint16_t *>(dst)[k] = __ldg(reinterpret_cast<const uint16_t *>(src) + k);
+        else reinterpret_cast<uint32_t *>(dst)[k * (es / 4)] = __ldg(reinterpret_cast<const uint32_t *>(src) + k * (es / 4));
+        if (es == 8)
+            reinterpret_cast<uint32_t *>(dst)[2 * k + 1] = __ldg(reinterpret_cast<const uint32_t *>(src) + 2 * k + 1);
+    }
+    for (uint32_t k = hi + threadIdx.x; k < n; k += blockDim.x) {
+        if (es == 2) reinterpret_cast<uint16_t *>(dst)[k] = __ldg(reinterpret_cast<const uint16_t *>(src) + k);
+        else reinterpret_cast<uint32_t *>(dst)[k * (es / 4)] = __ldg(reinterpret_cast<const uint32_t *>(src) + k * (es / 4));
+        if (es == 8)
+            reinterpret_cast<uint32_t *>(dst)[2 * k + 1] = __ldg(reinterpret_cast<const uint32_t *>(src) + 2 * k + 1);
+    }
+}
+
 template <bool kPolicy>
 __global__ void __launch_bounds__(kGroupInitThreads) walk_init_group_kernel(
     uint32_t M, pv_probe *__restrict__ probes, uint32_t H, const uint16_t *__restrict__ host_switch,
-    const uint16_t *__restrict__ host_port, const uint8_t *__restrict__ region, pv_result *__restrict__ out,
-    uint2 *__restrict__ sorted, uint4 *__restrict__ recs, const uint32_t *__restrict__ seg,
-    const uint32_t *__restrict__ pair_off, PolicyArgs pa, BindArgs ba) {
-    extern __shared__ __align__(16) uint32_t s_cur[];   // [pods][kBuckets] counts, then slots; then the runs
+    const uint8_t *__restrict__ region, pv_result *__restrict__ out, uint4 *__restrict__ recs,
+    const uint32_t *__restrict__ seg,
+    const uint32_t *__restrict__ pair_off, PolicyArgs pa, BindArgs ba, uint64_t wait_ns, int32_t *status) {
+    extern __shared__ __align__(16) uint8_t s_raw[];
     __shared__ uint32_t s_pair[kGroupInitMaxPods][3];   // per pod: {node, switch, listed}
+    __shared__ uint64_t s_bar;
     const uint32_t grp = blockIdx.x, P = ba.pods, t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    uint2 *s_run = reinterpret_cast<uint2 *>(s_cur + P * kBuckets);   // {dst_ip, rank in group | dport << 16}
+    const bool records = ba.dst_stride == 2;
+    const GroupInitSmem L(P, ba.ppg, records);
+    uint32_t *s_cur = reinterpret_cast<uint32_t *>(s_raw);                  // [pods][kBuckets] counts, then slots
+    uint16_t *s_rank = reinterpret_cast<uint16_t *>(s_raw + L.rank);        // pod runs: ranks in the group
     const uint32_t first = grp * ba.ppg, len = min(ba.ppg, M - first);
+    // the group's flows: destination and port slices (one slice for records)
+    const Slice sa = records ? Slice(ba.dst + (size_t)first * 2, len, 8) : Slice(ba.dst + first, len, 4);
+    const Slice sb = records ? Slice(ba.dst, 0, 8) : Slice(ba.dport + first, len, 2);
+    if (t == 0) {
+        mbar_init(&s_bar, 1);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        mbar_arrive_expect_tx(&s_bar, sa.bulk_bytes() + sb.bulk_bytes());
+        slice_copy(sa, s_raw + L.dst, &s_bar);
+        slice_copy(sb, s_raw + L.dport, &s_bar);
+    }
+    slice_edges(sa, s_raw + L.dst);
+    slice_edges(sb, s_raw + L.dport);
+    const uint32_t *s_dst = reinterpret_cast<const uint32_t *>(sa.staged(s_raw + L.dst));
+    const uint16_t *s_dport = records ? reinterpret_cast<const uint16_t *>(s_dst) + 2
+                                      : reinterpret_cast<const uint16_t *>(sb.staged(s_raw + L.dport));
+    const uint32_t ds = records ? 2u : 1u, ps = records ? 4u : 1u;
     const uint32_t mask = ba.group_mask[grp];
     for (uint32_t x = t; x < P * kBuckets; x += kGroupInitThreads) s_cur[x] = 0;
     if (t < P) {
@@ -850,11 +946,19 @@ __global__ void __launch_bounds__(kGroupInitThreads) walk_init_group_kernel(
         s_pair[t][1] = sw;
         s_pair[t][2] = placed && t < len && first_switch_permitted<kPolicy>(pa, first + t, sw, region[sw], mask);
     }
-    __syncthreads();
-    for (uint32_t r = t; r < len; r += kGroupInitThreads) {
-        const uint32_t dport = __ldg(ba.flows + first + r).y & 0xFFFFu;
-        atomicAdd(&s_cur[(r % P) * kBuckets + (dport >> kBucketShift)], 1u);
+    __syncthreads();   // barrier initialised before anyone waits on it
+    const bool ok = mbar_wait_bounded(&s_bar, 0, wait_ns);
+    if (__syncthreads_or(!ok)) {
+        // the flows did not arrive in time: report it (the call's results are
+        // not to be used), wait for the copies once more (bounded), and bind
+        // from global memory, so the later hops still read valid records
+        if (t == 0) pv_device_error(status, PV_ETIMEOUT);
+        mbar_wait_bounded(&s_bar, 0, wait_ns);
+        s_dst = records ? ba.dst + (size_t)first * 2 : ba.dst + first;
+        s_dport = records ? ba.dport + (size_t)first * 4 : ba.dport + first;
     }
+    for (uint32_t r = t; r < len; r += kGroupInitThreads)
+        atomicAdd(&s_cur[(r % P) * kBuckets + (s_dport[r * ps] >> kBucketShift)], 1u);
     __syncthreads();
     // exclusive scan of each pod's buckets, offset by the runs of the pods
     // before it (pod q holds probes q, q + P, ...: ceil((len - q) / P) of them)
@@ -884,14 +988,14 @@ __global__ void __launch_bounds__(kGroupInitThreads) walk_init_group_kernel(
         const uint32_t i = first + r, q = r % P;
         const uint32_t node = s_pair[q][0], sw = s_pair[q][1];
         const bool placed = node < H;
-        const uint2 f = __ldg(ba.flows + i);
-        const uint32_t z = (f.y & 0xFFFFu) | (placed ? node : (uint32_t)PV_NO_HOST) << 16;
+        const uint32_t dport = s_dport[r * ps];
         if (probes)   // the caller's copy of the bound record {src_ip, dst_ip, dport | src_host << 16, mask}
-            reinterpret_cast<uint4 *>(probes)[i] = make_uint4(placed ? ba.host_ip[node] : 0u, f.x, z, mask);
+            reinterpret_cast<uint4 *>(probes)[i] = make_uint4(placed ? ba.host_ip[node] : 0u, s_dst[r * ds],
+                                                              dport | (placed ? node : (uint32_t)PV_NO_HOST) << 16,
+                                                              mask);
         if (kPolicy) pa.hits[i] = 0;
         if (s_pair[q][2]) {
-            s_run[atomicAdd(&s_cur[q * kBuckets + ((f.y & 0xFFFFu) >> kBucketShift)], 1u)] =
-                make_uint2(f.x, r | (f.y << 16));
+            s_rank[atomicAdd(&s_cur[q * kBuckets + (dport >> kBucketShift)], 1u)] = (uint16_t)r;
         } else {
             pv_result res;
             res.status = placed ? PV_VIOLATION : PV_NOSRC;
@@ -907,11 +1011,10 @@ __global__ void __launch_bounds__(kGroupInitThreads) walk_init_group_kernel(
         if (s_pair[q][2]) {
             const uint32_t sw = s_pair[q][1];
             const uint32_t node = s_pair[q][0];
-            const uint32_t base = seg[sw] + pair_off[grp * P + q], loc = (sw << 8) | host_port[node];
+            const uint32_t base = seg[sw] + pair_off[grp * P + q];
             for (uint32_t k = t; k < n; k += kGroupInitThreads) {
-                const uint2 v = s_run[before + k];
-                recs[base + k] = make_uint4(first + (v.y & 0xFFFFu), v.x, (v.y >> 16) | node << 16, mask);
-                sorted[base + k] = make_uint2(base + k, loc);
+                const uint32_t r = s_rank[before + k];
+                recs[base + k] = make_uint4(first + r, s_dst[r * ds], s_dport[r * ps] | node << 16, mask);
             }
         }
         before += n;
@@ -1066,7 +1169,8 @@ struct HopArgs {
     uint32_t *hist_next; // per-switch counts of the next hop's list (null: a separate pass counts)
     uint32_t hist_off;   // byte offset of the block's count array in dynamic shared memory
     uint32_t port_off;   // byte offset of the staged port table in dynamic shared memory
-    uint32_t recs_at_position;   // 1: entry i's record index is i (first hop of directly placed flows)
+    uint32_t recs_at_position;   // 1: no list, entry i is record i (first hop of directly placed flows)
+    const uint2 *host_addr;      // [H] {address, attachment port} of each host
     unsigned long long *stats;   // [PV_WALK_STATS] counters of the statistics kernels (kStats)
 };
 
@@ -1138,10 +1242,13 @@ __device__ __forceinline__ uint4 load_raw(const HopArgs &g, uint32_t x) {
 }
 
 template <bool kRec>
-__device__ __forceinline__ uint4 header_of(const HopArgs &g, uint4 raw, uint32_t x, uint32_t *id) {
+__device__ __forceinline__ uint4 header_of(const HopArgs &g, uint4 raw, uint32_t x, uint32_t *id,
+                                           uint32_t *src_port) {
     if (kRec) {
         *id = raw.x;
-        return make_uint4(__ldg(g.host_ip + (raw.z >> 16)), raw.y, raw.z, raw.w);
+        const uint2 ha = __ldg(g.host_addr + (raw.z >> 16));   // the source host's address and port
+        *src_port = ha.y;
+        return make_uint4(ha.x, raw.y, raw.z, raw.w);
     }
     *id = x;
     return raw;
@@ -1456,24 +1563,32 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
         // earlier), so neither waits on the other or on the batch's work.
         constexpr uint32_t kStride = 32 * kHopWarps;
         const uint32_t wb0 = pos + warp * 32;
+        // At the first hop of directly placed flows there is no list: entry
+        // i is record i, and its in_port is its source host's port.
+        const bool at_pos = kRec && g.recs_at_position != 0;
         uint2 e1 = make_uint2(0, 0), e2 = make_uint2(0, 0);   // entries of batches wb, wb + kStride
         uint4 raw1 = make_uint4(0, 0, 0, 0);                  // record of batch wb
         if (wb0 + lane < seg_end) {
-            e1 = g.sorted[wb0 + lane];
-            raw1 = load_raw<kRec>(g, g.recs_at_position ? wb0 + lane : e1.x);
+            e1 = at_pos ? make_uint2(wb0 + lane, 0) : g.sorted[wb0 + lane];
+            raw1 = load_raw<kRec>(g, e1.x);
         }
-        if (wb0 + kStride + lane < seg_end) e2 = g.sorted[wb0 + kStride + lane];
+        if (wb0 + kStride + lane < seg_end)
+            e2 = at_pos ? make_uint2(wb0 + kStride + lane, 0) : g.sorted[wb0 + kStride + lane];
         for (uint32_t wb = wb0; wb < seg_end; wb += kStride) {
             const uint32_t cnt = min(32u, seg_end - wb);
-            const uint2 e = e1;
+            uint2 e = e1;
             const uint4 raw = raw1;
-            if (wb + kStride + lane < seg_end)
-                raw1 = load_raw<kRec>(g, g.recs_at_position ? wb + kStride + lane : e2.x);
+            if (wb + kStride + lane < seg_end) raw1 = load_raw<kRec>(g, e2.x);
             e1 = e2;
-            if (wb + 2 * kStride + lane < seg_end) e2 = g.sorted[wb + 2 * kStride + lane];
+            if (wb + 2 * kStride + lane < seg_end)
+                e2 = at_pos ? make_uint2(wb + 2 * kStride + lane, 0) : g.sorted[wb + 2 * kStride + lane];
             uint4 pr = make_uint4(0, 0, 0, 0);   // {src_ip, dst_ip, dport | src_host << 16, allowed_mask}
             uint32_t pid = 0;                     // probe id
-            if (lane < cnt) pr = header_of<kRec>(g, raw, e.x, &pid);
+            if (lane < cnt) {
+                uint32_t src_port = 0;
+                pr = header_of<kRec>(g, raw, e.x, &pid, &src_port);
+                if (at_pos) e.y = src_port;
+            }
             // a probe in a known forwarding cycle that has reached its finish hop
             const uint32_t fin = e.y >> 24;
             const bool fin_now = lane < cnt && fin != 0 && fin - 1 == g.hop;
@@ -1710,6 +1825,13 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+// addr[h] = {host_ip[h], host_port[h]}.
+__global__ void host_addr_kernel(uint32_t H, const uint32_t *__restrict__ ip, const uint16_t *__restrict__ port,
+                                 uint2 *__restrict__ addr) {
+    const uint32_t h = blockIdx.x * blockDim.x + threadIdx.x;
+    if (h < H) addr[h] = make_uint2(ip[h], port[h]);
+}
+
 }  // namespace
 
 // A flow-table load between its two halves: the first has validated the
@@ -1820,6 +1942,7 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
         (rc = pv_pool_alloc(ctx, (void **)&t.d_host_switch, (size_t)H * 2, "host switch")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_host_port, (size_t)H * 2, "host port")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_host_ip, (size_t)H * 4, "host ip")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_host_addr, (size_t)H * 8, "host addresses")) ||
         (rc = pv_pool_alloc(ctx, (void **)&d_rule_offs, (S + 1) * 4, "rule offsets")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_raw, (size_t)R * sizeof(pv_rule), "raw rules"))) {
         free_temps();
@@ -1835,6 +1958,9 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
         e = e ? e : cudaMemcpyAsync(t.d_host_switch, host_switch, (size_t)H * 2, cudaMemcpyHostToDevice, ls);
         e = e ? e : cudaMemcpyAsync(t.d_host_port, host_port, (size_t)H * 2, cudaMemcpyHostToDevice, ls);
         e = e ? e : cudaMemcpyAsync(t.d_host_ip, host_ip, (size_t)H * 4, cudaMemcpyHostToDevice, ls);
+        if (e == cudaSuccess)
+            host_addr_kernel<<<(H + 255) / 256, 256, 0, ls>>>(H, t.d_host_ip, t.d_host_port, t.d_host_addr);
+        e = e ? e : cudaGetLastError();
     }
     e = e ? e : cudaMemcpyAsync(d_rule_offs, rule_offs, (S + 1) * 4, cudaMemcpyHostToDevice, ls);
     if (R) e = e ? e : cudaMemcpyAsync(t.d_raw, rules, (size_t)R * sizeof(pv_rule), cudaMemcpyHostToDevice, ls);
@@ -2171,7 +2297,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     int pr = pv_prof_start(ctx, st, PV_K_WALK_INIT);
     const PolicyArgs no_policy = {nullptr, nullptr, 0, nullptr, 0, 0, nullptr};
     const size_t init_smem = S <= kSmemHistMax ? (size_t)S * 4 : 0;
-    const BindArgs no_bind = {nullptr, 1, 1, nullptr, nullptr, nullptr};
+    const BindArgs no_bind = {nullptr, nullptr, 0, 0, 1, 1, nullptr, nullptr, nullptr};
     pv_probe *probes_rw = const_cast<pv_probe *>(d_probes);   // written only when binding
     uint4 *recs = (uint4 *)(base + o_recs);
     if (ba && !direct && !d_probes) probes_rw = reinterpret_cast<pv_probe *>(recs);   // the walk's own copy
@@ -2188,8 +2314,9 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
                                                                   ba0, G, hist, pair_off);
         walk_scan_kernel<<<1, 1024, 0, st>>>(S, hist, seg, cursor);
         const uint32_t groups32 = (uint32_t)groups;
-        const size_t gsm = (size_t)ba->pods * kBuckets * 4 + (size_t)ba->ppg * 8;
+        const size_t gsm = ba->ppg <= 0xFFFFu ? GroupInitSmem(ba->pods, ba->ppg, ba->dst_stride == 2).total : ~(size_t)0;
         const bool by_group = ba->pods <= kGroupInitMaxPods && gsm <= kGroupInitSmem && groups <= 0x7FFFFFFFull;
+        const uint64_t wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
         if (by_group) {
             PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_init_group_kernel<true>,
                                                   cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGroupInitSmem),
@@ -2200,19 +2327,19 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         }
         if (by_group && pol)
             walk_init_group_kernel<true><<<groups32, kGroupInitThreads, gsm, st>>>(
-                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
-                pair_off, pa0, ba0);
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_region, d_out, recs, seg,
+                pair_off, pa0, ba0, wait_ns, ctx->d_status);
         else if (by_group)
             walk_init_group_kernel<false><<<groups32, kGroupInitThreads, gsm, st>>>(
-                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
-                pair_off, pa0, ba0);
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_region, d_out, recs, seg,
+                pair_off, pa0, ba0, wait_ns, ctx->d_status);
         else if (pol)
             walk_init_direct_kernel<true><<<init_grid, kGridThreads, 0, st>>>(
-                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_region, d_out, recs, seg,
                 pair_off, pa0, ba0);
         else
             walk_init_direct_kernel<false><<<init_grid, kGridThreads, 0, st>>>(
-                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_host_port, t.d_region, d_out, sorted, recs, seg,
+                M, probes_rw, t.num_hosts, t.d_host_switch, t.d_region, d_out, recs, seg,
                 pair_off, pa0, ba0);
     } else if (pol && ba)
         walk_init_kernel<true, true><<<init_grid, kGridThreads, init_smem, st>>>(
@@ -2257,6 +2384,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.hist_off = (uint32_t)hist_off;
     g.port_off = (uint32_t)port_off;
     g.recs_at_position = 0;
+    g.host_addr = t.d_host_addr;
     g.stats = ctx->d_walk_stats;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;
@@ -2326,15 +2454,48 @@ extern "C" int pv_verify_probes_constrained(pv_ctx *ctx, uint32_t M, const pv_pr
     return walk_probes(ctx, M, d_probes, hop_cap, d_out, &pa, stream);
 }
 
+namespace {
+
+// Checks shared by the compact-flow walks (records or columns).
+int check_flow_call(pv_ctx *ctx, const char *fn, uint32_t M, const void *d_dst, const void *d_dport, uint32_t ppg,
+                    uint32_t pods, const uint32_t *d_assign, const uint32_t *d_group_mask) {
+    if (M && (!d_dst || !d_dport || !d_assign || !d_group_mask))
+        return pv_fail(ctx, PV_EINVAL, "%s: NULL device pointer", fn);
+    if (M && (ppg == 0 || pods == 0)) return pv_fail(ctx, PV_EINVAL, "%s: group sizes must be > 0", fn);
+    return PV_OK;
+}
+
+BindArgs flow_records(const pv_ctx *ctx, const pv_flow *f, uint32_t ppg, uint32_t pods, const uint32_t *assign,
+                      const uint32_t *group_mask) {
+    return {reinterpret_cast<const uint32_t *>(f), reinterpret_cast<const uint16_t *>(f) + 2, 2, 4, ppg, pods,
+            assign, group_mask, ctx->tb.d_host_ip};
+}
+
+BindArgs flow_columns(const pv_ctx *ctx, const uint32_t *dst, const uint16_t *dport, uint32_t ppg, uint32_t pods,
+                      const uint32_t *assign, const uint32_t *group_mask) {
+    return {dst, dport, 1, 1, ppg, pods, assign, group_mask, ctx->tb.d_host_ip};
+}
+
+int verify_flows_policies(pv_ctx *ctx, const char *fn, uint32_t M, const BindArgs &ba, uint32_t hop_cap,
+                          const uint32_t *d_probe_policy, uint32_t probes_per_policy, uint32_t first_policy,
+                          pv_probe *d_probes, pv_result *d_out, uint32_t *d_waypoints, pv_stream stream) {
+    if (!ctx->pol.loaded) return pv_fail(ctx, PV_ESTATE, "%s: no path policies loaded", fn);
+    if (M && !d_waypoints) return pv_fail(ctx, PV_EINVAL, "%s: NULL device pointer", fn);
+    const PolicyArgs pa = {ctx->pol.d_hdr, ctx->pol.d_sw, ctx->pol.num, d_probe_policy, probes_per_policy,
+                           first_policy, d_waypoints};
+    return walk_probes(ctx, M, d_probes, hop_cap, d_out, &pa, stream, &ba);
+}
+
+}  // namespace
+
 extern "C" int pv_verify_flows(pv_ctx *ctx, uint32_t M, const pv_flow *d_flows, uint32_t ppg, uint32_t pods,
                                const uint32_t *d_assign, const uint32_t *d_group_mask, uint32_t hop_cap,
                                pv_probe *d_probes, pv_result *d_out, pv_stream stream) {
     if (!ctx) return PV_EINVAL;
-    if (M && (!d_flows || !d_assign || !d_group_mask))
-        return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: NULL device pointer");
-    if (M && (ppg == 0 || pods == 0)) return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: group sizes must be > 0");
+    if (int rc = check_flow_call(ctx, "pv_verify_flows", M, d_flows, d_flows, ppg, pods, d_assign, d_group_mask))
+        return rc;
     if (((uintptr_t)d_flows & 7) != 0) return pv_fail(ctx, PV_EINVAL, "pv_verify_flows: d_flows must be 8-byte aligned");
-    const BindArgs ba = {reinterpret_cast<const uint2 *>(d_flows), ppg, pods, d_assign, d_group_mask, ctx->tb.d_host_ip};
+    const BindArgs ba = flow_records(ctx, d_flows, ppg, pods, d_assign, d_group_mask);
     return walk_probes(ctx, M, d_probes, hop_cap, d_out, nullptr, stream, &ba);
 }
 
@@ -2344,17 +2505,47 @@ extern "C" int pv_verify_flows_constrained(pv_ctx *ctx, uint32_t M, const pv_flo
                                            uint32_t probes_per_policy, uint32_t first_policy, pv_probe *d_probes,
                                            pv_result *d_out, uint32_t *d_waypoints, pv_stream stream) {
     if (!ctx) return PV_EINVAL;
-    if (!ctx->pol.loaded) return pv_fail(ctx, PV_ESTATE, "pv_verify_flows_constrained: no path policies loaded");
-    if (M && (!d_flows || !d_assign || !d_group_mask || !d_waypoints))
-        return pv_fail(ctx, PV_EINVAL, "pv_verify_flows_constrained: NULL device pointer");
-    if (M && (ppg == 0 || pods == 0))
-        return pv_fail(ctx, PV_EINVAL, "pv_verify_flows_constrained: group sizes must be > 0");
+    if (int rc = check_flow_call(ctx, "pv_verify_flows_constrained", M, d_flows, d_flows, ppg, pods, d_assign,
+                                 d_group_mask))
+        return rc;
     if (((uintptr_t)d_flows & 7) != 0)
         return pv_fail(ctx, PV_EINVAL, "pv_verify_flows_constrained: d_flows must be 8-byte aligned");
-    const BindArgs ba = {reinterpret_cast<const uint2 *>(d_flows), ppg, pods, d_assign, d_group_mask, ctx->tb.d_host_ip};
-    const PolicyArgs pa = {ctx->pol.d_hdr, ctx->pol.d_sw, ctx->pol.num, d_probe_policy, probes_per_policy,
-                           first_policy, d_waypoints};
-    return walk_probes(ctx, M, d_probes, hop_cap, d_out, &pa, stream, &ba);
+    const BindArgs ba = flow_records(ctx, d_flows, ppg, pods, d_assign, d_group_mask);
+    return verify_flows_policies(ctx, "pv_verify_flows_constrained", M, ba, hop_cap, d_probe_policy,
+                                 probes_per_policy, first_policy, d_probes, d_out, d_waypoints, stream);
+}
+
+extern "C" int pv_verify_flow_columns(pv_ctx *ctx, uint32_t M, const uint32_t *d_dst_ip, const uint16_t *d_dport,
+                                      uint32_t ppg, uint32_t pods, const uint32_t *d_assign,
+                                      const uint32_t *d_group_mask, uint32_t hop_cap, pv_probe *d_probes,
+                                      pv_result *d_out, pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (int rc = check_flow_call(ctx, "pv_verify_flow_columns", M, d_dst_ip, d_dport, ppg, pods, d_assign,
+                                 d_group_mask))
+        return rc;
+    if (((uintptr_t)d_dst_ip & 3) != 0 || ((uintptr_t)d_dport & 1) != 0)
+        return pv_fail(ctx, PV_EINVAL, "pv_verify_flow_columns: d_dst_ip must be 4-byte and d_dport 2-byte aligned");
+    const BindArgs ba = flow_columns(ctx, d_dst_ip, d_dport, ppg, pods, d_assign, d_group_mask);
+    return walk_probes(ctx, M, d_probes, hop_cap, d_out, nullptr, stream, &ba);
+}
+
+extern "C" int pv_verify_flow_columns_constrained(pv_ctx *ctx, uint32_t M, const uint32_t *d_dst_ip,
+                                                  const uint16_t *d_dport, uint32_t ppg, uint32_t pods,
+                                                  const uint32_t *d_assign, const uint32_t *d_group_mask,
+                                                  uint32_t hop_cap, const uint32_t *d_probe_policy,
+                                                  uint32_t probes_per_policy, uint32_t first_policy,
+                                                  pv_probe *d_probes, pv_result *d_out, uint32_t *d_waypoints,
+                                                  pv_stream stream) {
+    if (!ctx) return PV_EINVAL;
+    if (int rc = check_flow_call(ctx, "pv_verify_flow_columns_constrained", M, d_dst_ip, d_dport, ppg, pods,
+                                 d_assign, d_group_mask))
+        return rc;
+    if (((uintptr_t)d_dst_ip & 3) != 0 || ((uintptr_t)d_dport & 1) != 0)
+        return pv_fail(ctx, PV_EINVAL,
+                       "pv_verify_flow_columns_constrained: d_dst_ip must be 4-byte and d_dport 2-byte aligned");
+    const BindArgs ba = flow_columns(ctx, d_dst_ip, d_dport, ppg, pods, d_assign, d_group_mask);
+    return verify_flows_policies(ctx, "pv_verify_flow_columns_constrained", M, ba, hop_cap, d_probe_policy,
+                                 probes_per_policy, first_policy, d_probes, d_out, d_waypoints, stream);
 }
 
 extern "C" int pv_load_path_policies(pv_ctx *ctx, uint32_t num_policies, const uint32_t *forbid_offs,

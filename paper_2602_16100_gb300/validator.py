@@ -40,6 +40,13 @@ def flows_of(e: W.EndToEnd) -> np.ndarray:
     return f
 
 
+def flow_columns_of(e: W.EndToEnd) -> tuple:
+    """The same flows as two columns: destination addresses (uint32) and
+    destination ports (uint16), 6 bytes per flow."""
+    pr = e.probes.probes
+    return np.ascontiguousarray(pr["dst_ip"], np.uint32), np.ascontiguousarray(pr["dport"], np.uint16)
+
+
 class Validator:
     """One GPU validator context (not thread-safe)."""
 
@@ -159,23 +166,23 @@ class Validator:
         (policy i for intent i) when ``dev`` holds a "hits" buffer."""
         ppg, pods, n = e2e_sizes["probes_per_intent"], e2e_sizes["pods"], hi - lo
         words = W.words_per_row(self.num_nodes)
-        P, F = W.PROBE_DTYPE.itemsize, W.FLOW_DTYPE.itemsize
         results = dev["results"][lo * ppg * 4:]
-        flows, masks = dev["flows"][lo * ppg * F:], dev["masks"][lo * 4:]
+        dst, dport, masks = dev["dst"][lo * ppg * 4:], dev["dport"][lo * ppg * 2:], dev["masks"][lo * 4:]
         bits, flags, assign = dev["bits"][lo * words * 4:], dev["flags"][lo:], dev["assign"][lo * pods * 4:]
         cap = e2e_sizes["hop_cap"]
         if "hits" in dev:
             hits = dev["hits"][lo * ppg * 4:]
-            B.pv_verify_flows_constrained(self.ctx, n * ppg, flows, ppg, pods, assign, masks, cap, None, ppg, lo,
-                                          None, results, hits, stream)
+            B.pv_verify_flow_columns_constrained(self.ctx, n * ppg, dst, dport, ppg, pods, assign, masks, cap, None,
+                                                 ppg, lo, None, results, hits, stream)
             B.pv_aggregate_constrained(self.ctx, n, pods, bits, words, flags, assign, ppg, results, hits, None,
                                        dev["pass"][lo:], dev["counts"][lo * 32:], stream, first_policy=lo)
         else:
-            B.pv_verify_flows(self.ctx, n * ppg, flows, ppg, pods, assign, masks, cap, None, results, stream)
+            B.pv_verify_flow_columns(self.ctx, n * ppg, dst, dport, ppg, pods, assign, masks, cap, None, results,
+                                     stream)
             B.pv_aggregate_intents(self.ctx, n, pods, bits, words, flags, assign, ppg, results, dev["pass"][lo:],
                                    dev["counts"][lo * 32:], stream)
 
-    _INPUTS = ("offs", "exprs", "draws", "masks", "flows")
+    _INPUTS = ("offs", "exprs", "draws", "masks", "dst", "dport")
 
     def run_end_to_end_from_host(self, host: dict, dev: dict, e2e_sizes: dict, stream, copy_stream,
                                  chunks: int = 1, loads=None, loads_first: bool = False) -> dict:
@@ -194,8 +201,9 @@ class Validator:
         synchronised).
 
         ``host`` holds pinned byte tensors "offs", "exprs", "draws", "masks",
-        "flows" (inputs, as alloc_end_to_end lays them out: 8-byte flows, the
-        probe records are built on the device) and "pass", "counts" (outputs);
+        "dst", "dport" (inputs, as alloc_end_to_end lays them out: the flows
+        as two columns, 6 bytes each, the probe records are built on the
+        device) and "pass", "counts" (outputs);
         ``dev`` the device buffers of alloc_end_to_end.
 
         Consecutive calls alternate between two sets of device input buffers,
@@ -208,8 +216,6 @@ class Validator:
         chunks = max(1, min(int(chunks), max(1, I // 4)))
         # range edges on multiples of 4 intents (keeps every slice 16-byte aligned)
         edges = [0] + [((I * c) // chunks) & ~3 for c in range(1, chunks)] + [I]
-        P = W.PROBE_DTYPE.itemsize
-        F = W.FLOW_DTYPE.itemsize
         ranges = [(lo, hi) for lo, hi in zip(edges[:-1], edges[1:]) if hi > lo]
         finish = loads() if loads is not None else None
         if callable(finish) and loads_first:
@@ -233,8 +239,8 @@ class Validator:
                 n = host[k].numel()
                 dev[k][:n].copy_(host[k], non_blocking=True)
             for lo, hi in ranges:   # flows of intents [lo, hi)
-                dev["flows"][lo * ppg * F:hi * ppg * F].copy_(host["flows"][lo * ppg * F:hi * ppg * F],
-                                                               non_blocking=True)
+                for k, b in (("dst", 4), ("dport", 2)):
+                    dev[k][lo * ppg * b:hi * ppg * b].copy_(host[k][lo * ppg * b:hi * ppg * b], non_blocking=True)
                 ev = torch.cuda.Event()
                 ev.record(copy_stream)
                 ready.append(ev)
@@ -272,6 +278,8 @@ class Validator:
             "draws": to_device(e.place_draws.astype(np.uint64), d),
             "probes": to_device(e.probes.probes, d),
             "flows": to_device(flows_of(e), d),
+            "dst": to_device(flow_columns_of(e)[0], d),
+            "dport": to_device(flow_columns_of(e)[1], d),
             "masks": to_device(e.intent_mask.astype(np.uint32), d),
             "bits": empty_device(I * words * 4, d),
             "flags": empty_device(I, d),

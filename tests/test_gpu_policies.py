@@ -12,7 +12,7 @@ import pytest
 import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
-from paper_2602_16100_gb300.validator import flows_of, empty_device, to_device, to_numpy
+from paper_2602_16100_gb300.validator import flow_columns_of, empty_device, to_device, to_numpy
 from gpu_util import E2E_CONSTRAINED, POLICIES_CONSTRAINED
 from test_oracle_policies import _backup_switch_net, _policies
 from netbuild import probe
@@ -180,7 +180,7 @@ def test_constrained_pipeline_from_host(validator, chunks):
     I, pods, ppg = sizes["intents"], sizes["pods"], sizes["probes_per_intent"]
     host = {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
             "draws": _pinned(e.place_draws.astype(np.uint64)), "masks": _pinned(e.intent_mask.astype(np.uint32)),
-            "flows": _pinned(flows_of(e)),
+            "dst": _pinned(flow_columns_of(e)[0]), "dport": _pinned(flow_columns_of(e)[1]),
             "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
             "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
     stream = torch.cuda.current_stream()
@@ -199,14 +199,17 @@ def test_constrained_pipeline_from_host(validator, chunks):
     assert passed.any()
 
 
+@pytest.mark.parametrize("form", ["records", "columns"])
 @pytest.mark.parametrize("policy_form", ["per_group", "per_probe", "per_pair_of_groups", "none"])
-def test_flow_verification_direct_and_regrouped_first_hop_agree(validator, policy_form):
+def test_flow_verification_direct_and_regrouped_first_hop_agree(validator, policy_form, form):
     """pv_verify_flows(_constrained) lists compact flows straight into the
     first hop's switch order when each group has one path constraint (no
     constraint, or probes_per_policy a multiple of the group size) and
     regroups them otherwise (a per-probe policy array, or a stride that cuts
     groups).  Both give the oracle's results, records and waypoint bits; a
-    ragged last group (M not a multiple of the group size) is included."""
+    ragged last group (M not a multiple of the group size) is included.  The
+    flows are given as 8-byte records or as the two columns of
+    pv_verify_flow_columns(_constrained), read from a 2-byte offset."""
     e = W.end_to_end(seed=41, num_switches=64, num_intents=120, probes_per_intent=70, rules_per_switch=160)
     v = validator
     v.load_cluster(e.cluster)
@@ -225,8 +228,16 @@ def test_flow_verification_direct_and_regrouped_first_hop_agree(validator, polic
     assign = oracle.place_pods(bits, c.num_nodes, pods, e.place_draws)
     probes = oracle.bind_probes(e.probes.probes[:M], ppg, pods, assign, e.network.host_ip)
     dp, out = empty_device(M * 16, v.device), empty_device(M * 4, v.device)
+    dst = dev["dst"]
+    dport = empty_device(M * 2 + 2, v.device)[2:]       # columns need only their element alignment
+    dport.copy_(dev["dport"][: M * 2])
     if policy_form == "none":
-        B.pv_verify_flows(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], sizes["hop_cap"], dp, out)
+        if form == "records":
+            B.pv_verify_flows(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], sizes["hop_cap"], dp,
+                              out)
+        else:
+            B.pv_verify_flow_columns(v.ctx, M, dst, dport, ppg, pods, dev["assign"], dev["masks"], sizes["hop_cap"],
+                                     dp, out)
         v.sync()
         assert (to_numpy(out, W.RESULT_DTYPE) == oracle.verify_probes(e.network, probes, sizes["hop_cap"])).all()
         assert (to_numpy(dp, W.PROBE_DTYPE) == probes).all()
@@ -237,8 +248,12 @@ def test_flow_verification_direct_and_regrouped_first_hop_agree(validator, polic
         pp_host = (np.arange(M) // ppg).astype(np.uint32)     # the per-group policy, given per probe
         pp = to_device(pp_host, v.device)
     hits = empty_device(M * 4, v.device)
-    B.pv_verify_flows_constrained(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"], sizes["hop_cap"],
-                                  pp, per, 0, dp, out, hits)
+    if form == "records":
+        B.pv_verify_flows_constrained(v.ctx, M, dev["flows"], ppg, pods, dev["assign"], dev["masks"],
+                                      sizes["hop_cap"], pp, per, 0, dp, out, hits)
+    else:
+        B.pv_verify_flow_columns_constrained(v.ctx, M, dst, dport, ppg, pods, dev["assign"], dev["masks"],
+                                             sizes["hop_cap"], pp, per, 0, dp, out, hits)
     v.sync()
     if policy_form == "per_probe":
         res, oh = oracle.verify_constrained(e.network, probes, sizes["hop_cap"], pol, probe_policy=pp_host)

@@ -11,7 +11,7 @@ import pytest
 import oracle
 from paper_2602_16100_gb300 import binding as B
 from paper_2602_16100_gb300 import workloads as W
-from paper_2602_16100_gb300.validator import empty_device, flows_of, to_device, to_numpy
+from paper_2602_16100_gb300.validator import empty_device, flow_columns_of, to_device, to_numpy
 import full_oracle as F
 from gpu_util import E2E_PASS_SMALL
 
@@ -291,12 +291,12 @@ def test_end_to_end_pipelined_from_host(validator, chunks):
     validator.load_cluster(e.cluster)
     validator.load_network(e.network)
     dev, sizes = validator.alloc_end_to_end(e)
-    for k in ("offs", "exprs", "draws", "masks", "flows", "probes"):
+    for k in ("offs", "exprs", "draws", "masks", "dst", "dport", "flows", "probes"):
         dev[k].zero_()
     I = e.intents.num_pods
     host = {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
             "draws": _pinned(e.place_draws.astype(np.uint64)), "masks": _pinned(e.intent_mask.astype(np.uint32)),
-            "flows": _pinned(flows_of(e)),
+            "dst": _pinned(flow_columns_of(e)[0]), "dport": _pinned(flow_columns_of(e)[1]),
             "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
             "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
     stream = torch.cuda.current_stream()
@@ -341,7 +341,7 @@ def test_back_to_back_host_steps_each_with_its_own_tables(validator, loads_first
         I = e.intents.num_pods
         return {"offs": _pinned(e.intents.expr_offs.astype(np.uint32)), "exprs": _pinned(e.intents.exprs),
                 "draws": _pinned(e.place_draws.astype(np.uint64)), "masks": _pinned(e.intent_mask.astype(np.uint32)),
-                "flows": _pinned(flows_of(e)), "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
+                "dst": _pinned(flow_columns_of(e)[0]), "dport": _pinned(flow_columns_of(e)[1]), "pass": torch.zeros(I, dtype=torch.uint8).pin_memory(),
                 "counts": torch.zeros(I * 32, dtype=torch.uint8).pin_memory()}
 
     def loads(e):
