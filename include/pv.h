@@ -273,9 +273,11 @@ int pv_load_flow_tables_end(pv_ctx *ctx);
  * next hop.  Not terminated within hop_cap visits -> PV_LOOP.
  *
  * Device input d_probes[num_probes] (16-byte aligned); device output
- * d_out[num_probes].
- * Errors: PV_ESTATE (no tables), PV_EINVAL (hop_cap 0 or > 255, NULL
- * pointers with num_probes > 0).  Out-of-range src_host gives PV_NOSRC.
+ * d_out[num_probes] (4-byte aligned; every walk call writes each result as
+ * one 32-bit word).
+ * Errors: PV_ESTATE (no tables), PV_EINVAL (hop_cap 0 or > 255, NULL or
+ * misaligned pointers with num_probes > 0).  Out-of-range src_host gives
+ * PV_NOSRC.
  * ------------------------------------------------------------------------- */
 int pv_verify_probes(pv_ctx *ctx, uint32_t num_probes, const pv_probe *d_probes, uint32_t hop_cap,
                      pv_result *d_out, pv_stream stream);

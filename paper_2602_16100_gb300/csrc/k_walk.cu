@@ -609,6 +609,15 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
 // per block.  Warps reserve slots of their block's slice with shared-memory
 // atomics, so producing a list needs neither a global counter nor barriers.
 // Entry: x = probe id, y = location (switch << 8 | in_port).
+// Walk result i as one 32-bit store {status, hops, last_switch} (the
+// struct's own alignment is 2, so a member-wise store would be two or three
+// narrow writes, each a separate sector write at L2; walks require a 4-byte
+// aligned result array).
+__device__ __forceinline__ void put_result(pv_result *out, uint32_t i, uint32_t status, uint32_t hops,
+                                           uint32_t last) {
+    reinterpret_cast<uint32_t *>(out)[i] = status | hops << 8 | last << 16;
+}
+
 __device__ __forceinline__ uint32_t warp_reserve(bool want, uint32_t *s_count) {
     const uint32_t lane = threadIdx.x & 31;
     const uint32_t m = __ballot_sync(PV_FULL_MASK, want);
@@ -707,7 +716,6 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
                 pr = __ldg(reinterpret_cast<const uint4 *>(probes) + i);
             }
             const uint32_t h = pr.z >> 16;
-            pv_result r;
             if (kPolicy) pa.hits[i] = 0;
             if (h < H) {
                 const uint32_t s = host_switch[h];
@@ -721,16 +729,10 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_kernel(
                     live = true;
                     loc = (s << 8) | host_port[h];
                 } else {
-                    r.status = PV_VIOLATION;
-                    r.hops = 1;
-                    r.last_switch = (uint16_t)s;
-                    out[i] = r;
+                    put_result(out, i, PV_VIOLATION, 1, s);
                 }
             } else {
-                r.status = PV_NOSRC;
-                r.hops = 0;
-                r.last_switch = 0xFFFF;
-                out[i] = r;
+                put_result(out, i, PV_NOSRC, 0, 0xFFFF);
             }
         }
         const uint32_t slot = warp_reserve(live, &s_count);
@@ -808,12 +810,8 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
         if (probes)   // the caller's copy of the bound record {src_ip, dst_ip, dport | src_host << 16, mask}
             reinterpret_cast<uint4 *>(probes)[i] = make_uint4(placed ? ba.host_ip[node] : 0u, f.x, z, mask);
         if (kPolicy) pa.hits[i] = 0;
-        pv_result res;
         if (!placed) {
-            res.status = PV_NOSRC;
-            res.hops = 0;
-            res.last_switch = 0xFFFF;
-            out[i] = res;
+            put_result(out, i, PV_NOSRC, 0, 0xFFFF);
             continue;
         }
         const uint32_t s = host_switch[node];
@@ -821,10 +819,7 @@ __global__ void __launch_bounds__(kGridThreads) walk_init_direct_kernel(
             const uint32_t slot = seg[s] + pair_off[g] + r / ba.pods;
             recs[slot] = make_uint4(i, f.x, z, mask);
         } else {
-            res.status = PV_VIOLATION;
-            res.hops = 1;
-            res.last_switch = (uint16_t)s;
-            out[i] = res;
+            put_result(out, i, PV_VIOLATION, 1, s);
         }
     }
 }
@@ -997,11 +992,7 @@ __global__ void __launch_bounds__(kGroupInitThreads) walk_init_group_kernel(
         if (s_pair[q][2]) {
             s_rank[atomicAdd(&s_cur[q * kBuckets + (dport >> kBucketShift)], 1u)] = (uint16_t)r;
         } else {
-            pv_result res;
-            res.status = placed ? PV_VIOLATION : PV_NOSRC;
-            res.hops = placed ? 1 : 0;
-            res.last_switch = placed ? (uint16_t)sw : (uint16_t)0xFFFF;
-            out[i] = res;
+            put_result(out, i, placed ? PV_VIOLATION : PV_NOSRC, placed ? 1u : 0u, placed ? sw : 0xFFFFu);
         }
     }
     __syncthreads();
@@ -1659,11 +1650,8 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
             }
             if (lane < cnt && my_status != kAlive) {
                 const bool at_next = my_status == kViolationNext;
-                pv_result r;
-                r.status = (uint8_t)(at_next ? (uint32_t)PV_VIOLATION : my_status);
-                r.hops = (uint8_t)(fin_now ? g.cap : g.hop + (at_next ? 2u : 1u));
-                r.last_switch = (uint16_t)(at_next ? (my_next >> 8) : s);
-                g.out[pid] = r;
+                put_result(g.out, pid, at_next ? (uint32_t)PV_VIOLATION : my_status,
+                           fin_now ? g.cap : g.hop + (at_next ? 2u : 1u), at_next ? (my_next >> 8) : s);
             }
             const bool live = lane < cnt && my_status == kAlive;
             uint32_t nloc = my_next;
@@ -2236,6 +2224,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     if (M == 0) return PV_OK;
     if ((!d_probes && !ba) || !d_out) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: NULL device pointer");
     if (((uintptr_t)d_probes & 15) != 0) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: d_probes must be 16-byte aligned");
+    if (((uintptr_t)d_out & 3) != 0) return pv_fail(ctx, PV_EINVAL, "pv_verify_probes: d_out must be 4-byte aligned");
     const uint32_t S = t.num_switches;
     int which = ctx->opt_walk;
     if (which == 0) which = t.index_fits ? 2 : 1;
