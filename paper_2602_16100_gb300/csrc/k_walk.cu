@@ -172,6 +172,14 @@ __global__ void __launch_bounds__(1024) compile_tables_kernel(const uint32_t *__
 //   bnd[n_bnd] u32, win[n_bnd] u32   per segment: ascending elementary-interval
 //                                    starts (the first is 0) and the interval's
 //                                    winner (kWinFound | action, or 0 = none)
+//   jmp[n_segs]                      per segment, kJumpBytes: {base, shift,
+//                                    J[kJumpSlots + 1] u16}: base = the
+//                                    segment's second boundary (its first
+//                                    non-zero one), and J[j] = the last
+//                                    boundary index <= base + (j << shift)
+//                                    (J[kJumpSlots] = the last index), so an
+//                                    address's interval is searched among
+//                                    J[j] .. J[j + 1] only
 //   A[npad] uint4, B[npad] uint2     all rules in first-match order, padded to a
 //                                    multiple of 32 (linear scan, statistics)
 // The indexed kernel stages everything before the full rule list; the
@@ -191,6 +199,9 @@ constexpr uint32_t kTailEarlyItems = 12;    // candidate items per bucket below 
 constexpr uint32_t kMaxSegment = 4096;      // longer runs are split (in order: still exact)
 constexpr uint32_t kSegItem = 0x8000u;
 constexpr uint32_t kWinFound = 0x80000000u;
+constexpr uint32_t kJumpSlots = 256;
+constexpr uint32_t kJumpBytes = (8 + (kJumpSlots + 1) * 2 + 15) / 16 * 16;   // 528
+static_assert(kJumpBytes % 16 == 0, "jump blocks keep the blob's later sections 16-byte aligned");
 constexpr int kIndexThreads = 512;
 static_assert(kIndexThreads / 32 == 16, "bucket fill counts are laid out for 16 warps");
 
@@ -226,7 +237,7 @@ struct IndexSmem {
 __host__ __device__ inline uint32_t up16(uint32_t b) { return (b + 15u) & ~15u; }
 
 struct BlobLayout {
-    uint32_t a, b, boff, items, segs, bnd, win, fa, fb, total;
+    uint32_t a, b, boff, items, segs, bnd, win, jmp, fa, fb, total;
     __host__ __device__ BlobLayout(uint32_t npad, uint32_t n_plain, uint32_t n_items, uint32_t n_segs,
                                    uint32_t n_bnd) {
         a = 16;
@@ -236,7 +247,8 @@ struct BlobLayout {
         segs = items + up16(n_items * 2);
         bnd = segs + up16(n_segs * 8);
         win = bnd + up16(n_bnd * 4);
-        fa = win + up16(n_bnd * 4);
+        jmp = win + up16(n_bnd * 4);
+        fa = jmp + n_segs * kJumpBytes;
         fb = fa + npad * 16;
         total = fb + npad * 8;
     }
@@ -579,6 +591,31 @@ __global__ void __launch_bounds__(kIndexThreads) index_build_kernel(const uint32
                     bnd[n_bnd + s_pos[x]] = s_keys[x];
                     win[n_bnd + s_pos[x]] = s_win[x];
                 }
+            __syncthreads();   // the segment's boundaries are in the blob
+            uint8_t *jb = out + L.jmp + j * kJumpBytes;
+            const uint32_t *bb = bnd + n_bnd;
+            const uint32_t base = K2 > 1 ? bb[1] : 0xFFFFFFFFu, top = bb[K2 - 1];
+            uint32_t shift = 0;
+            while (shift < 32 && ((uint64_t)(top - (K2 > 1 ? base : top)) >> shift) >= kJumpSlots) ++shift;
+            if (t == 0) {
+                reinterpret_cast<uint32_t *>(jb)[0] = base;
+                reinterpret_cast<uint32_t *>(jb)[1] = shift;
+            }
+            uint16_t *J = reinterpret_cast<uint16_t *>(jb + 8);
+            for (uint32_t x = t; x <= kJumpSlots; x += nt) {
+                const uint64_t start = (uint64_t)base + ((uint64_t)x << shift);
+                uint32_t v = K2 - 1;   // last index with bb[v] <= start
+                if (x < kJumpSlots && start < 0xFFFFFFFFull) {
+                    uint32_t lo = 0, hi = K2;   // bb[lo] <= start < bb[hi]
+                    while (hi - lo > 1) {
+                        const uint32_t mid = (lo + hi) >> 1;
+                        if (bb[mid] <= (uint32_t)start) lo = mid;
+                        else hi = mid;
+                    }
+                    v = lo;
+                }
+                J[x] = (uint16_t)v;
+            }
         }
         n_bnd += K2;
         __syncthreads();
@@ -1263,6 +1300,23 @@ __device__ __forceinline__ uint32_t first_match_linear(const uint8_t *sm, uint32
     return 0u;
 }
 
+// The boundary range of a segment that holds dst's interval, from the
+// segment's jump block jb (shared or global memory): the answer (the last
+// boundary <= dst) is in [*lo, *lo + *len).
+__device__ __forceinline__ void jump_range(const uint8_t *jb, uint32_t dst, uint32_t *lo, uint32_t *len) {
+    const uint2 bs = *reinterpret_cast<const uint2 *>(jb);   // {base, shift}
+    if (dst < bs.x) {
+        *lo = 0;
+        *len = 1;
+        return;
+    }
+    const uint32_t j = min((dst - bs.x) >> bs.y, kJumpSlots - 1);
+    const uint16_t *J = reinterpret_cast<const uint16_t *>(jb + 8);
+    const uint32_t a = J[j], b = J[j + 1];
+    *lo = a;
+    *len = b - a + 1;
+}
+
 // Winner of the elementary interval holding dst: the warp narrows the range
 // 32-ways per step (bnd ascending, bnd[0] = 0 <= dst).
 __device__ __forceinline__ uint32_t segment_lookup(const uint32_t *bnd, const uint32_t *win, uint32_t cnt,
@@ -1378,7 +1432,8 @@ __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const Bl
         if (seg != 0xFFFFFFFFu) {
             const uint2 sd = segs[seg];
             const uint32_t *b = bnd + sd.x;
-            uint32_t lo = 0, len = sd.y;   // b[0] = 0 <= dst; answer in [lo, lo + len)
+            uint32_t lo, len;   // b[lo] <= dst; answer in [lo, lo + len)
+            jump_range(sm + L.jmp + seg * kJumpBytes, dst, &lo, &len);
             while (len > 1) {
                 const uint32_t half = len >> 1;
                 lo = b[lo + half] <= dst ? lo + half : lo;
@@ -1704,6 +1759,9 @@ __device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict
         const uint32_t it = __ldg(items + i);
         if (it & kSegItem) {
             const uint2 sd = __ldg(segs + (it & 0x7FFFu));
+            // a plain binary search: measured faster here than starting from
+            // the jump block, whose loads lengthen each lookup's chain of L2
+            // round trips more than they shorten the search
             uint32_t lo = 0, len = sd.y;   // bnd[sd.x] = 0 <= dst
             while (len > 1) {
                 const uint32_t half = len >> 1;
