@@ -169,14 +169,15 @@ int pv_load_cluster(pv_ctx *ctx, uint32_t num_nodes, uint32_t num_keys, const ui
  * empty expression list admits every node.
  *
  * Device inputs: d_expr_offs[num_pods + 1] (CSR offsets into d_exprs,
- * num_exprs entries), d_assign[num_pods] or NULL (the placement sigma).
- * Device outputs: d_bits[num_pods][words_per_row] feasible-node bitsets;
- * d_flags[num_pods] PV_F_* bits (ASSIGN_OK and PASS need d_assign).
+ * num_exprs entries, 4-byte aligned), d_assign[num_pods] or NULL (the
+ * placement sigma).  Device outputs: d_bits[num_pods][words_per_row]
+ * (16-byte aligned) feasible-node bitsets; d_flags[num_pods] PV_F_* bits
+ * (ASSIGN_OK and PASS need d_assign).
  * Malformed expression lists (offsets decreasing or beyond num_exprs, key
  * >= num_keys, unknown op, bad nvals, PV_ABSENT as a value) give an empty
  * row and PV_F_BAD_EXPR for that pod; they are not call errors.
  * Errors: PV_ESTATE (no cluster), PV_EINVAL (words_per_row too small or
- * not a multiple of 4, NULL pointers with num_pods > 0).
+ * not a multiple of 4, NULL or misaligned pointers with num_pods > 0).
  * ------------------------------------------------------------------------- */
 int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t *d_expr_offs, uint32_t num_exprs,
                       const pv_expr *d_exprs, const uint32_t *d_assign, uint32_t *d_bits,

@@ -343,8 +343,10 @@ constexpr int kRowsWarps = kRowsThreads / 32;
 struct ResolvedExprs {
     uint32_t meta[kRowsWarps][32];     // op | rows << 8
     uint32_t off[kRowsWarps][32][8];   // word offset of each row in the row array
+    uint8_t order[kRowsWarps][32];     // evaluation order of the expressions (sel_rows_kernel)
 };
 
+template <bool kOrder>
 __device__ __forceinline__ uint32_t resolve_exprs(ResolvedExprs &rx, uint32_t warp, uint32_t lane, uint32_t lo,
                                                   uint32_t E, const pv_expr *__restrict__ exprs, uint32_t K,
                                                   const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
@@ -384,6 +386,108 @@ __device__ __forceinline__ uint32_t resolve_exprs(ResolvedExprs &rx, uint32_t wa
         }
         rx.meta[warp][lane] = op | n << 8;
     }
+    // Evaluation order (the AND of the expressions' sets does not depend on
+    // it): In expressions with the fewest carried values first, then
+    // DoesNotExist, Exists and NotIn, the sparsest sets first, so that a pod
+    // whose row empties early stops reading rows.  Ties keep list order.
+    uint32_t key = 0xFFFFFFFFu;
+    if (kOrder && lane < E) {
+        const uint32_t op = rx.meta[warp][lane] & 0xFFu, n = rx.meta[warp][lane] >> 8;
+        const uint32_t cls = op == PV_IN ? 0u : op == PV_DOESNOTEXIST ? 1u : op == PV_EXISTS ? 2u : 3u;
+        key = cls << 8 | n;
+    }
+    uint32_t place = 0;
+    for (uint32_t j = 0; kOrder && j < E; ++j) {
+        const uint32_t kj = __shfl_sync(PV_FULL_MASK, key, j);
+        place += (kj < key || (kj == key && j < lane)) ? 1u : 0u;
+    }
+    if (kOrder && lane < E) rx.order[warp][place] = (uint8_t)lane;
+    __syncwarp();
+    bad = __any_sync(PV_FULL_MASK, bad);
+    unknown = __any_sync(PV_FULL_MASK, unknown);
+    return (bad ? 1u : 0u) | (unknown ? 2u : 0u);
+}
+
+// The same resolution with one lane per (expression, value) slot: lanes
+// 0 .. E - 1 read their expression's header word, a warp scan lays the
+// slots out (an In or NotIn expression takes one slot per listed value,
+// any other one slot), and every slot's lane resolves its value's row in
+// one step.  For lists of at most 32 slots (returns bit2 and resolves
+// nothing when there are more).  Same results, flags and order as
+// resolve_exprs<true>.
+__device__ __forceinline__ uint32_t resolve_slots(ResolvedExprs &rx, uint32_t warp, uint32_t lane, uint32_t lo,
+                                                  uint32_t E, const pv_expr *__restrict__ exprs, uint32_t K,
+                                                  const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
+                                                  const uint32_t *__restrict__ key_base, uint32_t num_value_rows,
+                                                  uint32_t row_words) {
+    // header word: key (bits 0..15), op (16..23), nvals (24..31)
+    uint32_t hdr = 0, m = 0;
+    bool bad = false;
+    if (lane < E) {
+        hdr = __ldg(reinterpret_cast<const uint32_t *>(exprs + lo + lane));
+        const uint32_t k = hdr & 0xFFFFu, op = (hdr >> 16) & 0xFFu, nv = hdr >> 24;
+        const bool listed = op == PV_IN || op == PV_NOTIN;
+        bad = k >= K || (listed ? (nv < 1 || nv > 8) : (op == PV_EXISTS || op == PV_DOESNOTEXIST) ? nv != 0 : true);
+        m = (listed && !bad) ? nv : 1u;
+    }
+    uint32_t incl = m;   // slots of expressions 0 .. lane
+    for (int d = 1; d < 32; d <<= 1) {
+        const uint32_t y = __shfl_up_sync(PV_FULL_MASK, incl, d);
+        if (lane >= (uint32_t)d) incl += y;
+    }
+    const uint32_t T = __shfl_sync(PV_FULL_MASK, incl, 31);
+    if (T > 32) return 4u;
+    const uint32_t pre = incl - m;
+    const uint32_t starts = __reduce_or_sync(PV_FULL_MASK, lane < E ? 1u << pre : 0u);
+    // slot lane: expression e, value j
+    const uint32_t upto = lane == 31 ? ~0u : (2u << lane) - 1u;
+    const uint32_t e = lane < T ? (uint32_t)__popc(starts & upto) - 1u : 0u;
+    const uint32_t pre_e = __shfl_sync(PV_FULL_MASK, pre, e);
+    const uint32_t hdr_e = __shfl_sync(PV_FULL_MASK, hdr, e);
+    const uint32_t m_e = __shfl_sync(PV_FULL_MASK, m, e);
+    const bool bad_e = __shfl_sync(PV_FULL_MASK, bad ? 1u : 0u, e) != 0;
+    const uint32_t k = hdr_e & 0xFFFFu, op = (hdr_e >> 16) & 0xFFu;
+    bool carried = false, unknown = false;
+    uint32_t off = 0;
+    if (lane < T && !bad_e) {
+        if (op == PV_IN || op == PV_NOTIN) {
+            const uint32_t v = __ldg(&exprs[lo + e].vals[lane - pre_e]);
+            if (v == PV_ABSENT) {
+                bad = true;
+            } else {
+                const uint32_t w = __ldg(inv + (size_t)k * kInvWords + (v >> 5)), bit = v & 31;
+                carried = (w >> bit) & 1u;
+                if (carried)
+                    off = (__ldg(key_base + k) + __ldg(rank + (size_t)k * kInvWords + (v >> 5)) +
+                           __popc(w & ((1u << bit) - 1u))) * row_words;
+                else if (op == PV_IN)
+                    unknown = true;
+            }
+        } else {
+            carried = true;
+            off = (num_value_rows + k) * row_words;
+        }
+    }
+    // carried rows of each expression, packed in slot order
+    const uint32_t C = __ballot_sync(PV_FULL_MASK, carried);
+    const uint32_t below = (1u << lane) - 1u;
+    if (carried) rx.off[warp][e][__popc(C & below & ~((1u << pre_e) - 1u))] = off;
+    uint32_t key = 0xFFFFFFFFu;
+    if (lane < E) {
+        const uint32_t span = (m >= 32 ? ~0u : (1u << m) - 1u) << pre;
+        const uint32_t n = __popc(C & span), opl = (hdr >> 16) & 0xFFu;
+        rx.meta[warp][lane] = opl | n << 8;
+        const uint32_t cls = opl == PV_IN ? 0u : opl == PV_DOESNOTEXIST ? 1u : opl == PV_EXISTS ? 2u : 3u;
+        key = cls << 8 | n;
+    }
+    (void)m_e;
+    uint32_t place = 0;
+    for (uint32_t j = 0; j < E; ++j) {
+        const uint32_t kj = __shfl_sync(PV_FULL_MASK, key, j);
+        place += (kj < key || (kj == key && j < lane)) ? 1u : 0u;
+    }
+    if (lane < E) rx.order[warp][place] = (uint8_t)lane;
+    __syncwarp();
     bad = __any_sync(PV_FULL_MASK, bad);
     unknown = __any_sync(PV_FULL_MASK, unknown);
     return (bad ? 1u : 0u) | (unknown ? 2u : 0u);
@@ -461,9 +565,12 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
         const uint32_t lo = offs[p], hi = offs[p + 1];
         const uint32_t E = hi - lo;
         const bool resolved = hi >= lo && hi <= num_exprs && E <= 32;
-        const uint32_t pre = resolved ? resolve_exprs(rx, warp, lane, lo, E, exprs, K, inv, rank, key_base,
-                                                      num_value_rows, row_words)
-                                      : pod_prescan(lo, hi, num_exprs, exprs, K, inv, lane);
+        uint32_t pre = resolved ? resolve_slots(rx, warp, lane, lo, E, exprs, K, inv, rank, key_base, num_value_rows,
+                                                row_words)
+                                : pod_prescan(lo, hi, num_exprs, exprs, K, inv, lane);
+        if (resolved && (pre & 4u))   // more than 32 slots: one lane per expression
+            pre = resolve_exprs<true>(rx, warp, lane, lo, E, exprs, K, inv, rank, key_base, num_value_rows,
+                                      row_words);
         uint4 *out = reinterpret_cast<uint4 *>(bits + (size_t)p * W);
         if (pre & 1u) {
             for (uint32_t q = lane; q < W / 4; q += 32) out[q] = make_uint4(0, 0, 0, 0);
@@ -488,7 +595,17 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
                 const bool h0 = q0 < W / 4, h1 = q1 < W / 4;
                 const bool l0 = h0 && q0 * 4 < row_words, l1 = h1 && q1 * 4 < row_words;
                 uint4 a0 = make_uint4(~0u, ~0u, ~0u, ~0u), a1 = a0;
-                for (uint32_t e = 0; e < E; ++e) and_resolved2(rx, warp, e, rows, q0, q1, l0, l1, a0, a1);
+                for (uint32_t i = 0; i < E; ++i) {
+                    and_resolved2(rx, warp, rx.order[warp][i], rows, q0, q1, l0, l1, a0, a1);
+                    // every node of the span rejected: the remaining sets
+                    // cannot add any back (chunks past the rows hold no nodes)
+                    const bool nz = (l0 && (a0.x | a0.y | a0.z | a0.w)) || (l1 && (a1.x | a1.y | a1.z | a1.w));
+                    if (!__any_sync(PV_FULL_MASK, nz)) {
+                        a0 = make_uint4(0, 0, 0, 0);
+                        a1 = a0;
+                        break;
+                    }
+                }
                 if (h0) finish(a0, q0);
                 if (h1) finish(a1, q1);
             }
@@ -541,7 +658,7 @@ __global__ void __launch_bounds__(kRowsThreads) sel_terms_kernel(
             E = resolved ? e1 - e0 : 0u;
         }
         if (resolved)
-            pre |= resolve_exprs(rx, warp, lane, e0, E, exprs, K, inv, rank, key_base, num_value_rows, row_words);
+            pre |= resolve_exprs<false>(rx, warp, lane, e0, E, exprs, K, inv, rank, key_base, num_value_rows, row_words);
         else
             for (uint32_t t = t0; t < t1 && !(pre & 1u); ++t)
                 pre |= pod_prescan(term_offs[t], term_offs[t + 1], num_exprs, exprs, K, inv, lane);
@@ -824,6 +941,8 @@ extern "C" int pv_eval_selectors(pv_ctx *ctx, uint32_t num_pods, const uint32_t 
     if (words_per_row % 4 != 0 || words_per_row < (c.num_nodes + 31) / 32)
         return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: words_per_row must be >= ceil(N/32) and a multiple of 4");
     if (((uintptr_t)d_bits & 15) != 0) return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: d_bits must be 16-byte aligned");
+    if (((uintptr_t)d_exprs & 3) != 0)   // expressions are read a 32-bit word at a time
+        return pv_fail(ctx, PV_EINVAL, "pv_eval_selectors: d_exprs must be 4-byte aligned");
     int which = ctx->opt_selector;
     if (which == 0) which = c.rows_built ? 2 : 1;
     if (which == 2 && !c.rows_built)

@@ -105,6 +105,10 @@ def test_empty_and_invalid_calls(validator):
     assert e.value.code == B.PV_EINVAL
     with pytest.raises(B.PVError):
         B.pv_eval_selectors(validator.ctx, 4, offs, len(d["selectors"].exprs), ex, None, bits, 6, flags)
+    odd = empty_device(d["selectors"].exprs.nbytes + 2, dev)[2:]   # expressions off a 4-byte boundary
+    with pytest.raises(B.PVError) as e:
+        B.pv_eval_selectors(validator.ctx, 4, offs, len(d["selectors"].exprs), odd, None, bits, 4, flags)
+    assert e.value.code == B.PV_EINVAL
     with pytest.raises(B.PVError) as e:
         B.pv_load_cluster(validator.ctx, 0, 4, np.zeros(0, np.uint16))
     assert e.value.code == B.PV_EINVAL
