@@ -1741,7 +1741,12 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
 
 // First match of one probe by one thread, reading the switch's blob from
 // global memory (L2-resident tables): the per-lane walk of first_match_lane
-// without its warp phases.
+// without its warp phases.  The candidate list is read four items at a time
+// and the four candidates' rules are loaded together before any is tested,
+// so a probe's chain of dependent L2 round trips per hop shrinks about as
+// many times (a tail walk is as long as its slowest probe's chain).
+constexpr uint32_t kTailBatch = 4;
+
 template <bool kStats>
 __device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict__ blob, const BlobLayout &L,
                                                        uint32_t src, uint32_t dst, uint32_t dport,
@@ -1755,29 +1760,40 @@ __device__ __forceinline__ uint32_t first_match_thread(const uint8_t *__restrict
     const uint32_t *win = reinterpret_cast<const uint32_t *>(blob + L.win);
     const uint32_t k = dport >> kBucketShift;
     const uint32_t i1 = __ldg(boff + k + 1);
-    for (uint32_t i = __ldg(boff + k); i < i1; ++i) {
-        const uint32_t it = __ldg(items + i);
-        if (it & kSegItem) {
-            const uint2 sd = __ldg(segs + (it & 0x7FFFu));
-            // a plain binary search: measured faster here than starting from
-            // the jump block, whose loads lengthen each lookup's chain of L2
-            // round trips more than they shorten the search
-            uint32_t lo = 0, len = sd.y;   // bnd[sd.x] = 0 <= dst
-            while (len > 1) {
-                const uint32_t half = len >> 1;
-                lo = __ldg(bnd + sd.x + lo + half) <= dst ? lo + half : lo;
-                len -= half;
-            }
-            const uint32_t w = __ldg(win + sd.x + lo);
-            if (kStats) ++lookups;
-            if (w & kWinFound) return w;
-            continue;
+    for (uint32_t i = __ldg(boff + k); i < i1; i += kTailBatch) {
+        uint32_t it[kTailBatch];
+        uint4 a[kTailBatch];
+        uint2 bb[kTailBatch];
+#pragma unroll
+        for (uint32_t j = 0; j < kTailBatch; ++j) it[j] = i + j < i1 ? __ldg(items + i + j) : 0xFFFFu;
+#pragma unroll
+        for (uint32_t j = 0; j < kTailBatch; ++j) {
+            const bool rule = it[j] != 0xFFFFu && !(it[j] & kSegItem);
+            a[j] = rule ? __ldg(A + it[j]) : make_uint4(0, 0, 0, 0);
+            bb[j] = rule ? __ldg(Bv + it[j]) : make_uint2(1u, 0u);   // lo 1 > hi 0: never matches
         }
-        if (kStats) ++tests;
-        const uint4 a = __ldg(A + it);
-        const uint2 bb = __ldg(Bv + it);
-        const uint32_t diff = ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
-        if (diff == 0 && dport >= (bb.x & 0xFFFFu) && dport <= (bb.x >> 16)) return kWinFound | (bb.y >> 16);
+#pragma unroll
+        for (uint32_t j = 0; j < kTailBatch; ++j) {
+            if (it[j] == 0xFFFFu) return 0u;   // past the list's end: table miss
+            if (it[j] & kSegItem) {
+                const uint2 sd = __ldg(segs + (it[j] & 0x7FFFu));
+                uint32_t lo = 0, len = sd.y;   // bnd[sd.x] = 0 <= dst
+                while (len > 1) {
+                    const uint32_t half = len >> 1;
+                    lo = __ldg(bnd + sd.x + lo + half) <= dst ? lo + half : lo;
+                    len -= half;
+                }
+                const uint32_t w = __ldg(win + sd.x + lo);
+                if (kStats) ++lookups;
+                if (w & kWinFound) return w;
+                continue;
+            }
+            if (kStats) ++tests;
+            const uint32_t diff = ((src ^ a[j].x) & a[j].y) | ((dst ^ a[j].z) & a[j].w) |
+                                  ((in_port ^ bb[j].y) & ((bb[j].y >> 8) & 0xFFu));
+            if (diff == 0 && dport >= (bb[j].x & 0xFFFFu) && dport <= (bb[j].x >> 16))
+                return kWinFound | (bb[j].y >> 16);
+        }
     }
     return 0u;
 }
