@@ -104,10 +104,49 @@ __global__ void __launch_bounds__(kThreads) aggregate_kernel(uint32_t G, uint32_
         }
         uint32_t c[6] = {0, 0, 0, 0, 0, 0};
         const uint32_t *res = reinterpret_cast<const uint32_t *>(results + (size_t)g * ppg);
-        for (uint32_t k = lane; k < ppg; k += 32) {
-            const uint32_t st = __ldg(res + k) & 0xFFu;
+        if ((((uintptr_t)res) & 15) == 0) {
+            // 16-byte loads, statuses counted in a packed histogram (8 bits per
+            // status; flushed before any field could reach 256)
+            const uint4 *res4 = reinterpret_cast<const uint4 *>(res);
+            const uint32_t n4 = ppg / 4;
+            uint64_t acc = 0;
+            uint32_t since = 0;
+            auto bump = [](uint32_t r) {   // statuses past PV_NOSRC are not counted
+                const uint32_t st = r & 0xFFu;
+                return st < 6u ? 1ull << (st * 8u) : 0ull;
+            };
+            auto flush = [&]() {
 #pragma unroll
-            for (int s = 0; s < 6; ++s) c[s] += st == (uint32_t)s;
+                for (int s = 0; s < 6; ++s) c[s] += (uint32_t)(acc >> (8 * s)) & 0xFFu;
+                acc = 0;
+                since = 0;
+            };
+            uint32_t k = lane;
+            for (; k + 96 < n4; k += 128) {   // four loads in flight per lane
+                const uint4 v0 = __ldg(res4 + k), v1 = __ldg(res4 + k + 32);
+                const uint4 v2 = __ldg(res4 + k + 64), v3 = __ldg(res4 + k + 96);
+                acc += bump(v0.x) + bump(v0.y) + bump(v0.z) + bump(v0.w) + bump(v1.x) + bump(v1.y) + bump(v1.z) +
+                       bump(v1.w) + bump(v2.x) + bump(v2.y) + bump(v2.z) + bump(v2.w) + bump(v3.x) + bump(v3.y) +
+                       bump(v3.z) + bump(v3.w);
+                if (++since == 15) flush();   // at most 16 per field each step
+            }
+            flush();
+            for (; k < n4; k += 32) {
+                const uint4 v = __ldg(res4 + k);
+                acc += bump(v.x) + bump(v.y) + bump(v.z) + bump(v.w);
+            }
+            flush();
+            for (uint32_t k = 4 * n4 + lane; k < ppg; k += 32) {
+                const uint32_t st = __ldg(res + k) & 0xFFu;
+#pragma unroll
+                for (int s = 0; s < 6; ++s) c[s] += st == (uint32_t)s;
+            }
+        } else {
+            for (uint32_t k = lane; k < ppg; k += 32) {
+                const uint32_t st = __ldg(res + k) & 0xFFu;
+#pragma unroll
+                for (int s = 0; s < 6; ++s) c[s] += st == (uint32_t)s;
+            }
         }
         // path constraints: every probe must have entered all waypoints of the
         // group's policy, and the policy must name a concrete flow

@@ -1155,7 +1155,16 @@ __global__ void __launch_bounds__(kGridThreads) walk_scatter_kernel(const uint2 
     uint32_t *s_base = s_cnt + S;
     for (uint32_t j = threadIdx.x; j < S; j += kGridThreads) s_cnt[j] = 0;
     __syncthreads();
-    for (uint32_t i = b0 + threadIdx.x; i < b1; i += kGridThreads) atomicAdd(&s_cnt[entry_switch(list[i].y)], 1u);
+    // both passes keep four independent list loads in flight per thread
+    constexpr uint32_t kU = 4, kStep = kU * kGridThreads;
+    for (uint32_t i0 = b0 + threadIdx.x; i0 < b1; i0 += kStep) {
+        uint32_t loc[kU];
+#pragma unroll
+        for (uint32_t j = 0; j < kU; ++j) loc[j] = i0 + j * kGridThreads < b1 ? list[i0 + j * kGridThreads].y : 0u;
+#pragma unroll
+        for (uint32_t j = 0; j < kU; ++j)
+            if (i0 + j * kGridThreads < b1) atomicAdd(&s_cnt[entry_switch(loc[j])], 1u);
+    }
     __syncthreads();
     for (uint32_t j = threadIdx.x; j < S; j += kGridThreads) {
         const uint32_t c = s_cnt[j];
@@ -1163,10 +1172,16 @@ __global__ void __launch_bounds__(kGridThreads) walk_scatter_kernel(const uint2 
         s_cnt[j] = 0;
     }
     __syncthreads();
-    for (uint32_t i = b0 + threadIdx.x; i < b1; i += kGridThreads) {
-        const uint2 e = list[i];
-        const uint32_t s = entry_switch(e.y);
-        sorted[s_base[s] + atomicAdd(&s_cnt[s], 1u)] = e;
+    for (uint32_t i0 = b0 + threadIdx.x; i0 < b1; i0 += kStep) {
+        uint2 e[kU];
+#pragma unroll
+        for (uint32_t j = 0; j < kU; ++j) e[j] = i0 + j * kGridThreads < b1 ? list[i0 + j * kGridThreads] : make_uint2(0, 0);
+#pragma unroll
+        for (uint32_t j = 0; j < kU; ++j)
+            if (i0 + j * kGridThreads < b1) {
+                const uint32_t s = entry_switch(e[j].y);
+                sorted[s_base[s] + atomicAdd(&s_cnt[s], 1u)] = e[j];
+            }
     }
 }
 
