@@ -1214,6 +1214,7 @@ struct HopArgs {
     uint32_t port_off;   // byte offset of the staged port table in dynamic shared memory
     uint32_t recs_at_position;   // 1: no list, entry i is record i (first hop of directly placed flows)
     const uint2 *host_addr;      // [H] {address, attachment port} of each host
+    const uint2 *port_stage;     // [ports] {peer, aux} as the hop kernel stages them
     unsigned long long *stats;   // [PV_WALK_STATS] counters of the statistics kernels (kStats)
 };
 
@@ -1499,24 +1500,10 @@ __device__ __forceinline__ void hop_outcome(const HopArgs &g, uint32_t hop, uint
     }
 }
 
-// The hop kernel stages the current switch's ports once per table: port p
-// as {peer, aux}, aux = the region of the peer switch, or the address of
-// the attached host (0 for a host index out of range, which the outcome
-// rejects by its index), so a hop's outcome reads shared memory only.
-__device__ __forceinline__ uint2 port_entry(const HopArgs &g, uint32_t pbase, uint32_t p) {
-    const int32_t peer = g.port_peer[pbase + p];
-    uint32_t aux = 0;
-    if (peer >= 0) {
-        if (peer & PV_PEER_HOST) {
-            const uint32_t q = (uint32_t)(peer & ~PV_PEER_HOST);
-            aux = q < g.H ? g.host_ip[q] : 0u;
-        } else {
-            aux = g.region[(uint32_t)peer >> 8];
-        }
-    }
-    return make_uint2((uint32_t)peer, aux);
-}
-
+// The hop kernel stages the current switch's ports once per table from the
+// port stage the table loader builds (port_stage_kernel): port p as {peer,
+// aux}, aux = the region of the peer switch, or the address of the attached
+// host, so a hop's outcome reads shared memory only.
 // hop_outcome with the port table staged in shared memory (same outcomes).
 __device__ __forceinline__ void hop_outcome_staged(const HopArgs &g, const uint2 *s_port, uint32_t hop, uint32_t fm,
                                                    uint32_t dst, uint32_t mask, uint32_t nports, uint32_t *status,
@@ -1575,12 +1562,16 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
     uint32_t pos = r0;
     uint32_t stc[kStCount] = {};
     while (pos < r1) {
-        // switch owning position pos: last s with seg[s] <= pos
-        uint32_t lo = 0, hi = g.S;   // seg[lo] <= pos < seg[hi]
-        while (hi - lo > 1) {
-            const uint32_t mid = (lo + hi) >> 1;
-            if (g.seg[mid] <= pos) lo = mid;
-            else hi = mid;
+        // switch owning position pos: the last s with seg[s] <= pos (empty
+        // switches repeat their successor's start), found by each warp with
+        // a 32-way search (two rounds of loads for 512 switches)
+        uint32_t lo = 0, len = g.S;   // seg[lo] <= pos; answer in [lo, lo + len)
+        while (len > 1) {
+            const uint32_t stride = (len + 31) >> 5;
+            const bool le = lane * stride < len && __ldg(g.seg + lo + lane * stride) <= pos;
+            const uint32_t c = __popc(__ballot_sync(PV_FULL_MASK, le));   // lane 0 always
+            lo += (c - 1) * stride;
+            len = min(stride, len - (c - 1) * stride);
         }
         const uint32_t s = lo;
         const uint32_t seg_end = min(r1, g.seg[s + 1]);
@@ -1601,7 +1592,7 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
                 if (npad) bulk_g2s_keep(s_raw + 16, src_blob + L.fa, npad * 24, &s_bar);
             }
         }
-        for (uint32_t p = threadIdx.x; p < nports; p += kHopThreads) s_port[p] = port_entry(g, pbase, p);
+        for (uint32_t p = threadIdx.x; p < nports; p += kHopThreads) s_port[p] = __ldg(g.port_stage + pbase + p);
         const bool ok = mbar_wait_bounded(&s_bar, parity, g.wait_ns);
         if (__syncthreads_or(!ok)) {
             // give up: record the timeout, leave an empty slice for the next
@@ -1902,6 +1893,26 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
 
 inline size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
+// stage[p] = port p's {peer, aux} as walk_hop_kernel stages it: aux = the
+// peer switch's region, or the attached host's address (0 for a host index
+// out of range, which the outcome rejects by its index).
+__global__ void port_stage_kernel(uint32_t P, const int32_t *__restrict__ peer, const uint8_t *__restrict__ region,
+                                  uint32_t H, const uint32_t *__restrict__ host_ip, uint2 *__restrict__ stage) {
+    const uint32_t p = blockIdx.x * blockDim.x + threadIdx.x;
+    if (p >= P) return;
+    const int32_t x = peer[p];
+    uint32_t aux = 0;
+    if (x >= 0) {
+        if (x & PV_PEER_HOST) {
+            const uint32_t q = (uint32_t)(x & ~PV_PEER_HOST);
+            aux = q < H ? host_ip[q] : 0u;
+        } else {
+            aux = region[(uint32_t)x >> 8];
+        }
+    }
+    stage[p] = make_uint2((uint32_t)x, aux);
+}
+
 // addr[h] = {host_ip[h], host_port[h]}.
 __global__ void host_addr_kernel(uint32_t H, const uint32_t *__restrict__ ip, const uint16_t *__restrict__ port,
                                  uint2 *__restrict__ addr) {
@@ -2020,6 +2031,7 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
         (rc = pv_pool_alloc(ctx, (void **)&t.d_host_port, (size_t)H * 2, "host port")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_host_ip, (size_t)H * 4, "host ip")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_host_addr, (size_t)H * 8, "host addresses")) ||
+        (rc = pv_pool_alloc(ctx, (void **)&t.d_port_stage, std::max<size_t>((size_t)P, 1) * 8, "port stage")) ||
         (rc = pv_pool_alloc(ctx, (void **)&d_rule_offs, (S + 1) * 4, "rule offsets")) ||
         (rc = pv_pool_alloc(ctx, (void **)&t.d_raw, (size_t)R * sizeof(pv_rule), "raw rules"))) {
         free_temps();
@@ -2038,6 +2050,11 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
         if (e == cudaSuccess)
             host_addr_kernel<<<(H + 255) / 256, 256, 0, ls>>>(H, t.d_host_ip, t.d_host_port, t.d_host_addr);
         e = e ? e : cudaGetLastError();
+    }
+    if (P && e == cudaSuccess) {
+        port_stage_kernel<<<(P + 255) / 256, 256, 0, ls>>>(P, t.d_port_peer, t.d_region, H, t.d_host_ip,
+                                                            t.d_port_stage);
+        e = cudaGetLastError();
     }
     e = e ? e : cudaMemcpyAsync(d_rule_offs, rule_offs, (S + 1) * 4, cudaMemcpyHostToDevice, ls);
     if (R) e = e ? e : cudaMemcpyAsync(t.d_raw, rules, (size_t)R * sizeof(pv_rule), cudaMemcpyHostToDevice, ls);
@@ -2463,6 +2480,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.port_off = (uint32_t)port_off;
     g.recs_at_position = 0;
     g.host_addr = t.d_host_addr;
+    g.port_stage = t.d_port_stage;
     g.stats = ctx->d_walk_stats;
     ctx->last_walk_cap = hop_cap;
     g.wait_extra = ctx->opt_test_stall_staging ? 16u : 0u;

@@ -129,6 +129,7 @@ void pv_free_tables(pv_ctx *ctx, pv_table_state &t) {
     pv_free_ptr(ctx, t.d_host_port);
     pv_free_ptr(ctx, t.d_host_ip);
     pv_free_ptr(ctx, t.d_host_addr);
+    pv_free_ptr(ctx, t.d_port_stage);
     pv_free_ptr(ctx, t.d_in_offs);
     pv_free_ptr(ctx, t.d_in_links);
     pv_free_ptr(ctx, t.d_raw);

@@ -48,6 +48,7 @@ struct pv_table_state {
     uint16_t *d_host_switch = nullptr, *d_host_port = nullptr;
     uint32_t *d_host_ip = nullptr;
     uint2 *d_host_addr = nullptr;     // [H] {address, attachment port}: one load for a walk's source host
+    uint2 *d_port_stage = nullptr;    // [ports] {peer, peer's region or host address}: the hop kernel's port stage
     // switch-to-switch links into each switch, sorted by (source switch,
     // source port): u << 16 | p << 8 | q for port p of u cabled to port q
     uint32_t *d_in_offs = nullptr;    // [S + 1]
