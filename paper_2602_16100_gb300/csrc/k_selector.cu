@@ -415,16 +415,21 @@ __device__ __forceinline__ uint32_t resolve_exprs(ResolvedExprs &rx, uint32_t wa
 // one step.  For lists of at most 32 slots (returns bit2 and resolves
 // nothing when there are more).  Same results, flags and order as
 // resolve_exprs<true>.
+__device__ __forceinline__ uint32_t expr_header(const pv_expr *__restrict__ exprs, uint32_t lo, uint32_t lane) {
+    return __ldg(reinterpret_cast<const uint32_t *>(exprs + lo + lane));
+}
+
 __device__ __forceinline__ uint32_t resolve_slots(ResolvedExprs &rx, uint32_t warp, uint32_t lane, uint32_t lo,
                                                   uint32_t E, const pv_expr *__restrict__ exprs, uint32_t K,
                                                   const uint32_t *__restrict__ inv, const uint32_t *__restrict__ rank,
                                                   const uint32_t *__restrict__ key_base, uint32_t num_value_rows,
-                                                  uint32_t row_words) {
-    // header word: key (bits 0..15), op (16..23), nvals (24..31)
+                                                  uint32_t row_words, uint32_t lane_hdr) {
+    // header word (expr_header, fetched by the caller): key (bits 0..15),
+    // op (16..23), nvals (24..31)
     uint32_t hdr = 0, m = 0;
     bool bad = false;
     if (lane < E) {
-        hdr = __ldg(reinterpret_cast<const uint32_t *>(exprs + lo + lane));
+        hdr = lane_hdr;
         const uint32_t k = hdr & 0xFFFFu, op = (hdr >> 16) & 0xFFu, nv = hdr >> 24;
         const bool listed = op == PV_IN || op == PV_NOTIN;
         bad = k >= K || (listed ? (nv < 1 || nv > 8) : (op == PV_EXISTS || op == PV_DOESNOTEXIST) ? nv != 0 : true);
@@ -560,24 +565,46 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
     const uint32_t gw = (blockIdx.x * kRowsThreads + threadIdx.x) >> 5;
     const uint32_t nw = (gridDim.x * kRowsThreads) >> 5;
     const uint32_t n = pod_list ? *list_len : P;   // with a list: only the pods it names
+    // The next pod's offsets are loaded while this pod is resolved, and its
+    // expression headers while this pod's rows are swept, so a pod's chain
+    // of dependent loads starts at its values.
+    auto pod_at = [&](uint32_t i) { return pod_list ? pod_list[i] : i; };
+    auto headed = [&](uint32_t lo, uint32_t hi) { return hi >= lo && hi <= num_exprs && hi - lo <= 32; };
+    uint32_t p = 0, lo = 0, hi = 0, hdr = 0;
+    if (gw < n) {
+        p = pod_at(gw);
+        lo = offs[p];
+        hi = offs[p + 1];
+        hdr = headed(lo, hi) && lane < hi - lo ? expr_header(exprs, lo, lane) : 0u;
+    }
     for (uint32_t i = gw; i < n; i += nw) {
-        const uint32_t p = pod_list ? pod_list[i] : i;
-        const uint32_t lo = offs[p], hi = offs[p + 1];
+        uint32_t np = 0, nlo = 0, nhi = 0;
+        if (i + nw < n) {
+            np = pod_at(i + nw);
+            nlo = offs[np];
+            nhi = offs[np + 1];
+        }
+        const uint32_t a = assign ? assign[p] : PV_UNPLACED;
         const uint32_t E = hi - lo;
-        const bool resolved = hi >= lo && hi <= num_exprs && E <= 32;
+        const bool resolved = headed(lo, hi);
         uint32_t pre = resolved ? resolve_slots(rx, warp, lane, lo, E, exprs, K, inv, rank, key_base, num_value_rows,
-                                                row_words)
+                                                row_words, hdr)
                                 : pod_prescan(lo, hi, num_exprs, exprs, K, inv, lane);
         if (resolved && (pre & 4u))   // more than 32 slots: one lane per expression
             pre = resolve_exprs<true>(rx, warp, lane, lo, E, exprs, K, inv, rank, key_base, num_value_rows,
                                       row_words);
+        const uint32_t nhdr = i + nw < n && headed(nlo, nhi) && lane < nhi - nlo ? expr_header(exprs, nlo, lane) : 0u;
         uint4 *out = reinterpret_cast<uint4 *>(bits + (size_t)p * W);
+        const uint32_t pc = p, lc = lo;   // this pod (the names below move on to the next one)
+        p = np;
+        lo = nlo;
+        hi = nhi;
+        hdr = nhdr;
         if (pre & 1u) {
             for (uint32_t q = lane; q < W / 4; q += 32) out[q] = make_uint4(0, 0, 0, 0);
-            if (lane == 0) flags[p] = PV_F_BAD_EXPR;
+            if (lane == 0) flags[pc] = PV_F_BAD_EXPR;
             continue;
         }
-        const uint32_t a = assign ? assign[p] : PV_UNPLACED;
         bool any = false, aok = false;
         auto finish = [&](uint4 acc, uint32_t q) {
             const uint32_t w0 = q * 4;
@@ -615,7 +642,7 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
                 uint4 acc = make_uint4(~0u, ~0u, ~0u, ~0u);
                 const bool in_rows = w0 < row_words;
                 for (uint32_t e = 0; e < E; ++e) {
-                    const uint4 r = expr_rows4(exprs[lo + e], w0, in_rows, inv, rank, key_base, rows, row_words,
+                    const uint4 r = expr_rows4(exprs[lc + e], w0, in_rows, inv, rank, key_base, rows, row_words,
                                                num_value_rows);
                     acc.x &= r.x; acc.y &= r.y; acc.z &= r.z; acc.w &= r.w;
                 }
@@ -624,7 +651,7 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
         }
         any = __any_sync(PV_FULL_MASK, any);   // also keeps the warp's resolved rows until all lanes are done
         aok = __any_sync(PV_FULL_MASK, aok);
-        if (lane == 0) flags[p] = pod_flags(any, pre & 2u, assign != nullptr, aok);
+        if (lane == 0) flags[pc] = pod_flags(any, pre & 2u, assign != nullptr, aok);
     }
 }
 
