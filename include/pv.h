@@ -301,7 +301,10 @@ int pv_verify_probes(pv_ctx *ctx, uint32_t num_probes, const pv_probe *d_probes,
  * permitted set.  Out-of-range sources give empty rows.  When every remaining edge has its reverse (and
  * no vertex has more than 64 out-edges) the rows are taken from the
  * connected components of the permitted subgraph, which on such a graph is
- * the same set (PV_OPT_REACH_KERNEL).
+ * the same set (PV_OPT_REACH_KERNEL).  The call enqueues on `stream`; with
+ * the component path enabled, the other path's kernels (which return at
+ * once on a symmetric graph) run on a side stream of the context that
+ * `stream` waits for before the call returns (created on the first call).
  * Errors: PV_EINVAL (V == 0, V > 16384, words_per_row too small or not a
  * multiple of 4, NULL pointers); PV_ENOMEM (scratch).
  * ------------------------------------------------------------------------- */

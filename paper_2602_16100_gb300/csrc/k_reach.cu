@@ -595,6 +595,11 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
     }
     uint16_t *lab = (uint16_t *)(base + o_lab);   // [num_masks][V] (component path only)
     PV_TRY_CUDA(ctx, reach_smem_limits(), "reach shared-memory limits");
+    if (comp && !ctx->reach_side) {   // first call: the sweep path's side stream
+        PV_TRY_CUDA(ctx, cudaStreamCreateWithFlags(&ctx->reach_side, cudaStreamNonBlocking), "reach side stream");
+        PV_TRY_CUDA(ctx, cudaEventCreateWithFlags(&ctx->reach_fork, cudaEventDisableTiming), "reach fork event");
+        PV_TRY_CUDA(ctx, cudaEventCreateWithFlags(&ctx->reach_join, cudaEventDisableTiming), "reach join event");
+    }
     PV_TRY_CUDA(ctx, cudaMemsetAsync(indeg, 0, (size_t)(V + 1) * 4, st), "indeg clear");
     if (comp) {
         PV_TRY_CUDA(ctx, cudaMemsetAsync(ctx->d_reach_asym, 0, 4, st), "symmetry flag clear");
@@ -612,9 +617,17 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
         reach_symcheck_kernel<<<wgrid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, ctx->d_reach_asym, pairs,
                                                               npairs, indeg + V);
         launches += 3;
+        // Both paths are launched and the symmetry flag picks the one that
+        // works: on the component path's calls the sweep path's kernels go to
+        // the side stream (they need only the in-degrees and the flag), so
+        // their launches overlap the labels and rows kernels instead of
+        // queueing behind them; the caller's stream joins it at the end.
+        PV_TRY_CUDA(ctx, cudaEventRecord(ctx->reach_fork, st), "reach fork");
+        PV_TRY_CUDA(ctx, cudaStreamWaitEvent(ctx->reach_side, ctx->reach_fork, 0), "reach fork");
     }
-    reach_scan_kernel<<<1, 1024, 0, st>>>(V, indeg, in_offs, cursor, sym_flag);
-    reach_fill_kernel<<<grid, kGridThreads, 0, st>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, sym_flag,
+    cudaStream_t sw = comp ? ctx->reach_side : st;   // the sweep path's stream
+    reach_scan_kernel<<<1, 1024, 0, sw>>>(V, indeg, in_offs, cursor, sym_flag);
+    reach_fill_kernel<<<grid, kGridThreads, 0, sw>>>(V, num_edges, d_offs, d_cols, cursor, in_cols, sym_flag,
                                                      indeg + V);
     if (comp) {
         reach_labels_kernel<<<num_masks, kLabelThreads, lab_smem, st>>>(V, pairs, npairs, d_region, d_masks, lab,
@@ -634,9 +647,13 @@ extern "C" int pv_compliant_reach(pv_ctx *ctx, uint32_t V, const uint32_t *d_off
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bfs_per_sm, reach_msbfs_kernel, kReachThreads, smem);
     const uint64_t items = (uint64_t)((num_src + 63) / 64) * num_masks;
     const uint32_t g2 = (uint32_t)std::min<uint64_t>(items, (uint64_t)std::max(bfs_per_sm, 1) * ctx->num_sms);
-    reach_msbfs_kernel<<<g2, kReachThreads, smem, st>>>(V, in_offs, in_cols, d_region, num_src, d_src, num_masks,
+    reach_msbfs_kernel<<<g2, kReachThreads, smem, sw>>>(V, in_offs, in_cols, d_region, num_src, d_src, num_masks,
                                                        d_masks, d_reach, words_per_row,
                                                        comp ? ctx->d_reach_asym : nullptr);
+    if (comp) {
+        PV_TRY_CUDA(ctx, cudaEventRecord(ctx->reach_join, ctx->reach_side), "reach join");
+        PV_TRY_CUDA(ctx, cudaStreamWaitEvent(st, ctx->reach_join, 0), "reach join");
+    }
     pv_prof_stop(ctx, st, pr, launches);
     return pv_check_launch(ctx, "reach kernels");
 }

@@ -284,6 +284,9 @@ extern "C" void pv_destroy(pv_ctx *ctx) {
     cudaEventDestroy(ctx->retire_from);
     cudaStreamDestroy(ctx->load_stream);
     cudaStreamDestroy(ctx->retire_stream);
+    if (ctx->reach_side) cudaStreamDestroy(ctx->reach_side);
+    if (ctx->reach_fork) cudaEventDestroy(ctx->reach_fork);
+    if (ctx->reach_join) cudaEventDestroy(ctx->reach_join);
     cudaMemPoolDestroy(ctx->pool);
     for (cudaEvent_t e : ctx->prof.pool) cudaEventDestroy(e);
     pv_device_free(ctx->scratch);

@@ -105,6 +105,10 @@ struct pv_ctx {
     cudaMemPool_t pool = nullptr;
     cudaEvent_t last_use = nullptr;   // recorded by every call that reads loaded state
     cudaEvent_t load_done = nullptr;  // recorded at the end of every load (its device work)
+    // compliant reach: the sweep path's kernels run on a side stream forked
+    // from the caller's (created on the first call)
+    cudaStream_t reach_side = nullptr;
+    cudaEvent_t reach_fork = nullptr, reach_join = nullptr;
     pv_prof_state prof;
     int num_sms = 0;
     size_t max_smem_optin = 0;
