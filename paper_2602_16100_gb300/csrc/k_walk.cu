@@ -1425,19 +1425,39 @@ __device__ __forceinline__ uint32_t first_match_lane(const uint8_t *sm, const Bl
     while (__any_sync(PV_FULL_MASK, !done)) {
         uint32_t seg = 0xFFFFFFFFu;
         if (!done) {
-            for (; i < i1; ++i) {
-                const uint32_t it = items[i];
-                if (it & kSegItem) {
-                    seg = it & 0x7FFFu;
+            // two items per step, both rules loaded before either is tested
+            // (a segment token's slot loads rule 0, unused)
+            auto hit = [&](uint4 a, uint2 bb) {
+                const uint32_t diff =
+                    ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
+                return diff == 0 && dport >= (bb.x & 0xFFFFu) && dport <= (bb.x >> 16);
+            };
+            for (; i < i1; i += 2) {
+                const uint32_t it0 = items[i];
+                const bool has1 = i + 1 < i1;
+                const uint32_t it1 = has1 ? items[i + 1] : 0u;
+                const uint32_t r0 = (it0 & kSegItem) ? 0u : it0, r1 = (it1 & kSegItem) ? 0u : it1;
+                const uint4 a0 = sA[r0], a1 = sA[r1];
+                const uint2 b0 = sB[r0], b1 = sB[r1];
+                if (it0 & kSegItem) {
+                    seg = it0 & 0x7FFFu;
                     break;
                 }
                 if (kStats) ++tests;
-                const uint4 a = sA[it];
-                const uint2 bb = sB[it];
-                const uint32_t diff =
-                    ((src ^ a.x) & a.y) | ((dst ^ a.z) & a.w) | ((in_port ^ bb.y) & ((bb.y >> 8) & 0xFFu));
-                if (diff == 0 && dport >= (bb.x & 0xFFFFu) && dport <= (bb.x >> 16)) {
-                    result = kWinFound | (bb.y >> 16);
+                if (hit(a0, b0)) {
+                    result = kWinFound | (b0.y >> 16);
+                    done = true;
+                    break;
+                }
+                if (!has1) break;
+                if (it1 & kSegItem) {
+                    seg = it1 & 0x7FFFu;
+                    ++i;   // i names the token, so a segment miss resumes after it
+                    break;
+                }
+                if (kStats) ++tests;
+                if (hit(a1, b1)) {
+                    result = kWinFound | (b1.y >> 16);
                     done = true;
                     break;
                 }
