@@ -608,11 +608,14 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
         bool any = false, aok = false;
         auto finish = [&](uint4 acc, uint32_t q) {
             const uint32_t w0 = q * 4;
-            clip_rows4(acc, w0, N);
+            if (w0 + 4 > (N >> 5)) clip_rows4(acc, w0, N);   // only chunks reaching node N - 1 or past it
             out[q] = acc;
             any = any || (acc.x | acc.y | acc.z | acc.w) != 0;
-            const uint32_t *aw = &acc.x;
-            if (a < N && (a >> 5) >= w0 && (a >> 5) < w0 + 4) aok = (aw[(a >> 5) - w0] >> (a & 31)) & 1u;
+            if (a < N && (a >> 7) == q) {   // the assigned node's word is in this chunk
+                const uint32_t wsel = (a >> 5) & 3u;
+                const uint32_t word = wsel == 0 ? acc.x : wsel == 1 ? acc.y : wsel == 2 ? acc.z : acc.w;
+                aok = (word >> (a & 31)) & 1u;
+            }
         };
         if (resolved) {
             // a lane takes chunks q and q + 32 of each 64-chunk span, so one
