@@ -526,7 +526,10 @@ int pv_install_path_rules(pv_ctx *ctx, uint32_t num_slots, const pv_rule *d_rule
  *   in_port) it already held is in a forwarding cycle (its header is fixed,
  *   so its walk repeats); it walks only to the cycle position of hop
  *   hop_cap - 1 and is finished there with the PV_LOOP result the full walk
- *   gives (checkpoints at hops 4, 8, 16, ...); 1 = walk every hop to the cap.
+ *   gives (checkpoints at hops 4, 8, 16, ...).  When every switch port's
+ *   peer port leads back to it, a probe that leaves two switches in a row by
+ *   the port it came in by (two bounces) is in a two-switch cycle and is
+ *   finished at the second bounce.  1 = walk every hop to the cap.
  *   Both give the same results; PV_STAT_WALK_LIVE_TOTAL differs.
  * PV_OPT_WALK_TAIL_HOP: with the indexed kernel, the walk's hops from this
  *   one on (0 = none) run in a single launch, one thread per probe still

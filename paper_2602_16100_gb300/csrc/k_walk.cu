@@ -1063,6 +1063,18 @@ __device__ __forceinline__ uint32_t entry_switch(uint32_t loc) { return (loc >> 
 // probe walks only (cap - 1 - h) mod p more hops and is then finished with
 // exactly the result the full walk gives.
 constexpr uint32_t kCycleCheckFrom = 4;
+// Bits 24..31 of a list entry's location hold the visit after which a probe
+// in a known forwarding cycle finishes (1 .. cap - 1), 0, or kBounced: the
+// probe left its last switch by the port it had entered through (a bounce).
+// With symmetric cabling a bounce at the next switch too proves a two-switch
+// cycle: state (switch, in_port) after the second bounce equals the state
+// before the first, and the walk is a function of that state, so the visits
+// alternate between the two switches until the hop cap.
+constexpr uint32_t kBounced = 0xFFu;
+__device__ __forceinline__ uint32_t loc_finish(uint32_t loc) {
+    const uint32_t f = loc >> 24;
+    return f == kBounced ? 0u : f;
+}
 
 // One block per list slice: per-switch histogram of the live probes.
 __global__ void __launch_bounds__(kGridThreads) walk_hist_kernel(const uint2 *__restrict__ list,
@@ -1208,6 +1220,7 @@ struct HopArgs {
     uint32_t *hop_live;  // [cap]: live probes processed at each hop (statistics)
     uint32_t *ck;        // [M]: cycle-detection checkpoint location per probe
     uint32_t cycles;     // 1: finish probes caught in forwarding cycles early
+    uint32_t bounce;     // 1: finish two-switch cycles at their second bounce (symmetric cabling)
     PolicyArgs pa;       // path constraints (used by the kPolicy kernels)
     uint32_t *hist_next; // per-switch counts of the next hop's list (null: a separate pass counts)
     uint32_t hist_off;   // byte offset of the block's count array in dynamic shared memory
@@ -1662,7 +1675,7 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
                 if (at_pos) e.y = src_port;
             }
             // a probe in a known forwarding cycle that has reached its finish hop
-            const uint32_t fin = e.y >> 24;
+            const uint32_t fin = loc_finish(e.y);
             const bool fin_now = lane < cnt && fin != 0 && fin - 1 == g.hop;
             const uint32_t fin_lanes = __ballot_sync(PV_FULL_MASK, fin_now);
             uint32_t my_status = fin_now ? (uint32_t)PV_LOOP : kAlive, my_next = 0, my_fm = 0;
@@ -1729,12 +1742,18 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
                 if (my_status == kAlive && switch_listed(g.pa.sw + ph.x, ph.y, my_next >> 8))
                     my_status = kViolationNext;   // the next switch is forbidden to this flow
             }
-            if (lane < cnt && my_status != kAlive) {
+            // a bounce right after a bounce: a two-switch cycle, whose visit
+            // cap - 1 (the walk's last) is at s or at the next switch by parity
+            const bool bounce = g.bounce && lane < cnt && my_status == kAlive && (my_fm & 0xFFFFu) == (e.y & 0xFFu);
+            const bool pingpong = bounce && (e.y >> 24) == kBounced;
+            if (lane < cnt && (my_status != kAlive || pingpong)) {
                 const bool at_next = my_status == kViolationNext;
-                put_result(g.out, pid, at_next ? (uint32_t)PV_VIOLATION : my_status,
-                           fin_now ? g.cap : g.hop + (at_next ? 2u : 1u), at_next ? (my_next >> 8) : s);
+                const uint32_t last = pingpong ? (((g.cap - 1u - g.hop) & 1u) ? (my_next >> 8) : s)
+                                               : at_next ? (my_next >> 8) : s;
+                put_result(g.out, pid, pingpong ? (uint32_t)PV_LOOP : at_next ? (uint32_t)PV_VIOLATION : my_status,
+                           fin_now || pingpong ? g.cap : g.hop + (at_next ? 2u : 1u), last);
             }
-            const bool live = lane < cnt && my_status == kAlive;
+            const bool live = lane < cnt && my_status == kAlive && !pingpong;
             uint32_t nloc = my_next;
             if (live) {
                 uint32_t nfin = fin;
@@ -1747,6 +1766,8 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
                         nfin = h1 + (g.cap - 1u - h1) % period + 1u;
                     }
                 }
+                if (nfin >= g.cap) nfin = 0;   // finishing at visit cap - 1 is the plain walk's end
+                if (nfin == 0 && bounce) nfin = kBounced;
                 nloc = my_next | (nfin << 24);
             }
             const uint32_t slot = warp_reserve(live, &s_count);
@@ -1855,7 +1876,7 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                 if (!live) break;
                 if (lane == 0) atomicAdd(&g.hop_live[h], (uint32_t)__popc(live));
                 if (!active) continue;
-                const uint32_t s = (loc >> 8) & 0xFFFFu, in_port = loc & 0xFFu, fin = loc >> 24;
+                const uint32_t s = (loc >> 8) & 0xFFFFu, in_port = loc & 0xFFu, fin = loc_finish(loc);
                 uint32_t *out = reinterpret_cast<uint32_t *>(g.out) + pid;   // {status, hops, last_switch}
                 if (fin != 0 && fin - 1 == h) {   // finished at its cycle position
                     *out = (uint32_t)PV_LOOP | g.cap << 8 | s << 16;
@@ -1894,6 +1915,12 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                     active = false;
                     continue;
                 }
+                const bool bounce = g.bounce && (fm & 0xFFFFu) == in_port;
+                if (bounce && (loc >> 24) == kBounced) {   // two bounces in a row: a two-switch cycle
+                    *out = (uint32_t)PV_LOOP | g.cap << 8 | (((g.cap - 1u - h) & 1u) ? (next >> 8) : s) << 16;
+                    active = false;
+                    continue;
+                }
                 uint32_t nfin = fin;
                 const uint32_t h1 = h + 1;
                 if (g.cycles && nfin == 0 && h1 >= kCycleCheckFrom) {
@@ -1904,6 +1931,8 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                         nfin = h1 + (g.cap - 1u - h1) % period + 1u;
                     }
                 }
+                if (nfin >= g.cap) nfin = 0;
+                if (nfin == 0 && bounce) nfin = kBounced;
                 loc = next | (nfin << 24);
             }
         }
@@ -2115,6 +2144,18 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
         if (e2 == cudaSuccess)
             e2 = cudaMemcpyAsync(t.d_in_links, links.data(), links.size() * 4, cudaMemcpyHostToDevice, ls);
         t.num_links = in_offs[S];
+        // symmetric cabling (port p of u leads to port q of v exactly when q
+        // of v leads back to p of u) lets a walk recognise a two-switch
+        // forwarding cycle from two bounces in a row (walk_hop_kernel)
+        bool sym = true;
+        for (uint32_t u = 0; u < S && sym; ++u)
+            for (uint32_t p = port_offs[u]; p < port_offs[u + 1] && sym; ++p) {
+                const int32_t peer = port_peer[p];
+                if (peer < 0 || (peer & PV_PEER_HOST)) continue;
+                const uint32_t v = (uint32_t)peer >> 8, q = (uint32_t)peer & 0xFFu;
+                sym = port_peer[port_offs[v] + q] == (int32_t)(u << 8 | (p - port_offs[u]));
+            }
+        t.links_symmetric = sym;
 
         if (e2 != cudaSuccess) {
             free_temps();
@@ -2494,6 +2535,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     g.hop_live = ctx->d_walk_live;
     g.ck = (uint32_t *)(base + o_ck);
     g.cycles = cycles ? 1u : 0u;
+    g.bounce = ctx->opt_walk_cycles == 0 && ctx->tb.links_symmetric ? 1u : 0u;   // any cap: no checkpoints needed
     g.pa = pol ? *pa : no_policy;
     g.hist_next = nullptr;
     g.hist_off = (uint32_t)hist_off;

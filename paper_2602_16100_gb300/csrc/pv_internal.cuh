@@ -54,6 +54,7 @@ struct pv_table_state {
     uint32_t *d_in_offs = nullptr;    // [S + 1]
     uint32_t *d_in_links = nullptr;   // [links]
     uint32_t num_links = 0;           // switch-to-switch links
+    bool links_symmetric = false;     // every switch port's peer port leads back to it
     pv_rule *d_raw = nullptr;         // [rules] as loaded (for rule installation)
 };
 

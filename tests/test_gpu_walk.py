@@ -338,6 +338,125 @@ def test_forwarding_cycles_finish_with_the_full_walk_result(validator):
     assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) < full // 2
 
 
+def _bounce_network(kinds=("pingpong", "once", "region")):
+    """Components of a tail of t switches, then A, B and C: A sends
+    everything to B (with kind "once", what comes back from B goes to C
+    instead), B sends everything back to A (a bounce: out by the port it
+    came in by), C delivers to its host.  With kind "pingpong" A bounces
+    too, so the walk alternates A, B from its first bounce on; with
+    "region" B lies in region 1.  The source host sits at the head switch."""
+    nports, links, hosts, region, rules, comps = [], [], [], [], [], []
+    for kind in kinds:
+        for t in (0, 1, 2, 3, 5, 9):
+            base = len(nports)
+            for i in range(t):                         # tail: 0 in, 1 out, 2 host (head only)
+                nports.append(3)
+                region.append(0)
+                rules.append([rule(100, 0, 0, 1)])
+            a, b, c = base + t, base + t + 1, base + t + 2
+            nports += [4, 1, 2]                        # A: 0 in, 1 to B, 2 host (head), 3 to C; B: 0; C: 0, 1 host
+            region += [0, 1 if kind == "region" else 0, 0]
+            ra = [rule(100, 0, 0, 1)]
+            if kind == "once":
+                ra = [rule(200, 0, 0, 3, in_port=1)] + ra
+            rules += [ra, [rule(100, 0, 0, 0)], [rule(100, 0, 0, 1)]]
+            for i in range(t - 1):
+                links.append((base + i, 1, base + i + 1, 0))
+            if t:
+                links.append((base + t - 1, 1, a, 0))
+            links += [(a, 1, b, 0), (a, 3, c, 0)]
+            head = base if t else a
+            src = len(hosts)
+            hosts.append((head, 2, ip(10, len(comps), 0, 1)))
+            hosts.append((c, 1, ip(10, len(comps), 0, 2)))
+            comps.append((kind, t, src))
+    return make_net(nports, links, hosts, region, rules), comps
+
+
+def _bounce_probes(comps):
+    pr = [probe(src, ip(10, c, 0, 1), ip(10, c, 0, 2), m, dport=c) for c, (_, _, src) in enumerate(comps)
+          for m in (1, 3)]
+    return np.concatenate(pr)
+
+
+BOUNCE_CAPS = (1, 2, 3, 4, 5, 6, 7, 8, 9, 10, 15, 16, 17, 31, 32, 33, 100, 254, 255)
+
+
+@pytest.mark.parametrize("tail", [-1, 0, 1, 3])
+def test_two_switch_cycles_finish_at_the_second_bounce(validator, tail):
+    """A probe that leaves two switches in a row by the port it entered
+    through is in a two-switch cycle (symmetric cabling): its walk ends
+    there with the full walk's result (LOOP, the hop cap, the switch of the
+    last visit by parity), for every cap, both first-match kernels, any tail
+    switch-over hop and with the cycle shortcuts off."""
+    net, comps = _bounce_network()
+    pr = _bounce_probes(comps)
+    validator.set_option(B.PV_OPT_WALK_TAIL_HOP, tail)
+    try:
+        for cap in BOUNCE_CAPS:
+            o = oracle.verify_probes(net, pr, cap)
+            for cyc in (0, 1):
+                validator.set_option(B.PV_OPT_WALK_CYCLES, cyc)
+                for kernel in KERNELS:
+                    assert _same(_gpu_walk(validator, net, pr, cap, kernel), o), (cap, cyc, kernel)
+            validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
+            if cap == 255:
+                kinds = np.repeat([k for k, _, _ in comps], 2)
+                assert (o["status"][kinds == "pingpong"] == W.ST_LOOP).all()
+                assert (o["status"][kinds == "once"] == W.ST_COMPLIANT).all()
+        # pure ping-pong components: each probe enters its tail, A, B and A
+        # again, and no further switch
+        pnet, pcomps = _bounce_network(("pingpong",))
+        ppr = _bounce_probes(pcomps)
+        for cap in (3, 4, 8, 32, 255):
+            o = oracle.verify_probes(pnet, ppr, cap)
+            assert _same(_gpu_walk(validator, pnet, ppr, cap, 2), o)
+            want = sum(2 * min(cap, t + 3) for _, t, _ in pcomps)
+            assert B.pv_get_stat(validator.ctx, B.PV_STAT_WALK_LIVE_TOTAL) == want, cap
+    finally:
+        validator.set_option(B.PV_OPT_WALK_TAIL_HOP, -1)
+        validator.set_option(B.PV_OPT_WALK_CYCLES, 0)
+
+
+def test_bounces_on_asymmetric_cabling_are_walked_out(validator):
+    """With cabling that is not symmetric two bounces in a row prove no
+    two-switch cycle: X, Y and Z each send everything out of port 0, which
+    leads X -> Y -> Z -> X, so every hop after the first is a bounce and the
+    period is 3.  The walk must take every visit (one ping-pong component on
+    symmetric links shares the tables) and still match the oracle."""
+    nports = [2, 1, 1]
+    rules = [[rule(100, 0, 0, 0)], [rule(100, 0, 0, 0)], [rule(100, 0, 0, 0)]]
+    net0, comps = _bounce_network(("pingpong",))
+    base = net0.num_switches
+    nports_all = list(np.diff(net0.port_offs).astype(int)) + nports
+    rules_all = [[net0.rules[j:j + 1] for j in range(int(net0.rule_offs[s]), int(net0.rule_offs[s + 1]))]
+                 for s in range(base)] + rules
+    links = []
+    for s in range(base):
+        for p in range(int(net0.port_offs[s]), int(net0.port_offs[s + 1])):
+            peer = int(net0.port_peer[p])
+            if peer >= 0 and not peer & W.HOST_BIT and (s, p - int(net0.port_offs[s])) < (peer >> 8, peer & 0xFF):
+                links.append((s, p - int(net0.port_offs[s]), peer >> 8, peer & 0xFF))
+    hosts = [(int(net0.host_switch[h]), int(net0.host_port[h]), int(net0.host_ip[h]))
+             for h in range(net0.num_hosts)] + [(base, 1, ip(10, 200, 0, 1))]
+    region = list(net0.switch_region) + [0, 0, 0]
+    net = make_net(nports_all, links, hosts, region, rules_all)
+    x, y, z = base, base + 1, base + 2
+    po = net.port_offs
+    net.port_peer[po[x]] = (y << 8) | 0
+    net.port_peer[po[y]] = (z << 8) | 0
+    net.port_peer[po[z]] = (x << 8) | 0
+    pr = np.concatenate([_bounce_probes(comps),
+                         probe(len(hosts) - 1, ip(10, 200, 0, 1), ip(99, 0, 0, 1), 1),
+                         probe(len(hosts) - 1, ip(10, 200, 0, 1), ip(99, 0, 0, 1), 3, dport=7)])
+    for cap in BOUNCE_CAPS:
+        o = oracle.verify_probes(net, pr, cap)
+        for kernel in KERNELS:
+            assert _same(_gpu_walk(validator, net, pr, cap, kernel), o), (cap, kernel)
+        if cap == 255:
+            assert o["status"][-1] == W.ST_LOOP and o["last_switch"][-1] == [x, y, z][254 % 3]
+
+
 @pytest.mark.parametrize("kernel", KERNELS)
 def test_stalled_staging_wait_times_out_and_context_recovers(validator, kernel):
     """A staging barrier that expects bytes no copy delivers: each hop block's
