@@ -1742,16 +1742,17 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
                 if (my_status == kAlive && switch_listed(g.pa.sw + ph.x, ph.y, my_next >> 8))
                     my_status = kViolationNext;   // the next switch is forbidden to this flow
             }
-            // a bounce right after a bounce: a two-switch cycle, whose visit
-            // cap - 1 (the walk's last) is at s or at the next switch by parity
-            const bool bounce = g.bounce && lane < cnt && my_status == kAlive && (my_fm & 0xFFFFu) == (e.y & 0xFFu);
-            const bool pingpong = bounce && (e.y >> 24) == kBounced;
-            if (lane < cnt && (my_status != kAlive || pingpong)) {
+            // a bounce (out by the port it came in by) right after a bounce: a
+            // two-switch cycle, whose visit cap - 1 (the walk's last) is at s
+            // or at the next switch by parity
+            const bool bounce = (my_fm & 0xFFFFu) == (e.y & 0xFFu);
+            const bool pingpong = (e.y >> 24) == kBounced && lane < cnt && my_status == kAlive && bounce;
+            if (lane < cnt && my_status != kAlive) {
                 const bool at_next = my_status == kViolationNext;
-                const uint32_t last = pingpong ? (((g.cap - 1u - g.hop) & 1u) ? (my_next >> 8) : s)
-                                               : at_next ? (my_next >> 8) : s;
-                put_result(g.out, pid, pingpong ? (uint32_t)PV_LOOP : at_next ? (uint32_t)PV_VIOLATION : my_status,
-                           fin_now || pingpong ? g.cap : g.hop + (at_next ? 2u : 1u), last);
+                put_result(g.out, pid, at_next ? (uint32_t)PV_VIOLATION : my_status,
+                           fin_now ? g.cap : g.hop + (at_next ? 2u : 1u), at_next ? (my_next >> 8) : s);
+            } else if (pingpong) {
+                put_result(g.out, pid, PV_LOOP, g.cap, ((g.cap - 1u - g.hop) & 1u) ? (my_next >> 8) : s);
             }
             const bool live = lane < cnt && my_status == kAlive && !pingpong;
             uint32_t nloc = my_next;
@@ -1764,10 +1765,10 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
                     } else if (g.ck[e.x] == my_next) {
                         const uint32_t period = h1 - (1u << (31 - __clz(h1)));
                         nfin = h1 + (g.cap - 1u - h1) % period + 1u;
+                        if (nfin >= g.cap) nfin = 0;   // finishing at visit cap - 1 is the plain walk's end
                     }
                 }
-                if (nfin >= g.cap) nfin = 0;   // finishing at visit cap - 1 is the plain walk's end
-                if (nfin == 0 && bounce) nfin = kBounced;
+                if (nfin == 0 && g.bounce && bounce) nfin = kBounced;
                 nloc = my_next | (nfin << 24);
             }
             const uint32_t slot = warp_reserve(live, &s_count);
@@ -1929,9 +1930,9 @@ __global__ void __launch_bounds__(256) walk_tail_kernel(HopArgs g, const uint2 *
                     } else if (g.ck[e.x] == next) {
                         const uint32_t period = h1 - (1u << (31 - __clz(h1)));
                         nfin = h1 + (g.cap - 1u - h1) % period + 1u;
+                        if (nfin >= g.cap) nfin = 0;
                     }
                 }
-                if (nfin >= g.cap) nfin = 0;
                 if (nfin == 0 && bounce) nfin = kBounced;
                 loc = next | (nfin << 24);
             }
