@@ -1563,7 +1563,10 @@ __device__ __forceinline__ void hop_outcome_staged(const HopArgs &g, const uint2
     }
 }
 
-template <bool kIndexed, bool kPolicy, bool kStats, bool kRec>
+// kFirst: the walk's first hop, where every entry's finish field is 0, its
+// in_port is the source host's port (so a live probe never bounces) and no
+// cycle check is due, so all of that is left out.
+template <bool kIndexed, bool kPolicy, bool kStats, bool kRec, bool kFirst>
 __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
     extern __shared__ __align__(128) uint8_t s_raw[];
     __shared__ uint64_t s_bar;
@@ -1675,9 +1678,9 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
                 if (at_pos) e.y = src_port;
             }
             // a probe in a known forwarding cycle that has reached its finish hop
-            const uint32_t fin = loc_finish(e.y);
-            const bool fin_now = lane < cnt && fin != 0 && fin - 1 == g.hop;
-            const uint32_t fin_lanes = __ballot_sync(PV_FULL_MASK, fin_now);
+            const uint32_t fin = kFirst ? 0u : loc_finish(e.y);
+            const bool fin_now = !kFirst && lane < cnt && fin != 0 && fin - 1 == g.hop;
+            const uint32_t fin_lanes = kFirst ? 0u : __ballot_sync(PV_FULL_MASK, fin_now);
             uint32_t my_status = fin_now ? (uint32_t)PV_LOOP : kAlive, my_next = 0, my_fm = 0;
             // Every listed probe is permitted at s (checked when it was handed
             // on).  Lane-per-probe when every candidate list of the batch is short.
@@ -1745,8 +1748,8 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
             // a bounce (out by the port it came in by) right after a bounce: a
             // two-switch cycle, whose visit cap - 1 (the walk's last) is at s
             // or at the next switch by parity
-            const bool bounce = (my_fm & 0xFFFFu) == (e.y & 0xFFu);
-            const bool pingpong = (e.y >> 24) == kBounced && lane < cnt && my_status == kAlive && bounce;
+            const bool bounce = !kFirst && (my_fm & 0xFFFFu) == (e.y & 0xFFu);
+            const bool pingpong = !kFirst && (e.y >> 24) == kBounced && lane < cnt && my_status == kAlive && bounce;
             if (lane < cnt && my_status != kAlive) {
                 const bool at_next = my_status == kViolationNext;
                 put_result(g.out, pid, at_next ? (uint32_t)PV_VIOLATION : my_status,
@@ -1759,7 +1762,7 @@ __global__ void __launch_bounds__(kHopThreads, 4) walk_hop_kernel(HopArgs g) {
             if (live) {
                 uint32_t nfin = fin;
                 const uint32_t h1 = g.hop + 1;   // hop of the next visit (< cap)
-                if (g.cycles && nfin == 0 && h1 >= kCycleCheckFrom) {
+                if (!kFirst && g.cycles && nfin == 0 && h1 >= kCycleCheckFrom) {
                     if ((h1 & (h1 - 1u)) == 0) {
                         g.ck[e.x] = my_next;   // new checkpoint
                     } else if (g.ck[e.x] == my_next) {
@@ -2367,14 +2370,23 @@ namespace {
 using HopKernel = void (*)(HopArgs);
 using TailKernel = void (*)(HopArgs, const uint2 *, const uint2 *, uint32_t, uint32_t);
 
+// first: the kernel for the walk's first hop (the statistics kernels serve
+// every hop with the general form)
+template <bool kRec, bool kFirst>
+HopKernel pick_hop_form(bool indexed, bool pol) {
+    if (indexed)
+        return pol ? walk_hop_kernel<true, true, false, kRec, kFirst> : walk_hop_kernel<true, false, false, kRec, kFirst>;
+    return pol ? walk_hop_kernel<false, true, false, kRec, kFirst> : walk_hop_kernel<false, false, false, kRec, kFirst>;
+}
+
 template <bool kRec>
-HopKernel pick_hop(bool indexed, bool pol, bool stats) {
+HopKernel pick_hop(bool indexed, bool pol, bool stats, bool first) {
     if (stats) {
-        if (indexed) return pol ? walk_hop_kernel<true, true, true, kRec> : walk_hop_kernel<true, false, true, kRec>;
-        return pol ? walk_hop_kernel<false, true, true, kRec> : walk_hop_kernel<false, false, true, kRec>;
+        if (indexed)
+            return pol ? walk_hop_kernel<true, true, true, kRec, false> : walk_hop_kernel<true, false, true, kRec, false>;
+        return pol ? walk_hop_kernel<false, true, true, kRec, false> : walk_hop_kernel<false, false, true, kRec, false>;
     }
-    if (indexed) return pol ? walk_hop_kernel<true, true, false, kRec> : walk_hop_kernel<true, false, false, kRec>;
-    return pol ? walk_hop_kernel<false, true, false, kRec> : walk_hop_kernel<false, false, false, kRec>;
+    return first ? pick_hop_form<kRec, true>(indexed, pol) : pick_hop_form<kRec, false>(indexed, pol);
 }
 
 template <bool kRec>
@@ -2414,9 +2426,13 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     // compact flows with one path constraint per group are placed directly
     // (and walked through walk records)
     const bool direct = ba && (!pol || (pa->probe_pol == nullptr && (pa->per == 0 || pa->per % ba->ppg == 0)));
-    const HopKernel hop_fn = direct ? pick_hop<true>(indexed, pol, stats) : pick_hop<false>(indexed, pol, stats);
+    const HopKernel hop_fn = direct ? pick_hop<true>(indexed, pol, stats, false) : pick_hop<false>(indexed, pol, stats, false);
+    const HopKernel hop_fn0 = direct ? pick_hop<true>(indexed, pol, stats, true) : pick_hop<false>(indexed, pol, stats, true);
     const TailKernel tail_fn = direct ? pick_tail<true>(pol, stats) : pick_tail<false>(pol, stats);
     PV_TRY_CUDA(ctx, cudaFuncSetAttribute((const void *)hop_fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)hop_smem),
+                "walk_hop_kernel smem");
+    PV_TRY_CUDA(ctx, cudaFuncSetAttribute((const void *)hop_fn0, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                           (int)hop_smem),
                 "walk_hop_kernel smem");
     cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, (const void *)hop_fn, kHopThreads, hop_smem);
@@ -2574,7 +2590,7 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         g.next_list = nxt;
         g.next_desc = dnxt;
         pr = pv_prof_start(ctx, st, PV_K_WALK_HOP);
-        hop_fn<<<hop_grid, kHopThreads, hop_smem, st>>>(g);
+        (h == 0 ? hop_fn0 : hop_fn)<<<hop_grid, kHopThreads, hop_smem, st>>>(g);
         pv_prof_stop(ctx, st, pr, 1);
         in_slices = hop_grid;
     }
