@@ -2181,12 +2181,13 @@ int tables_begin(pv_ctx *ctx, pv_table_load &L, uint32_t S, const uint32_t *rule
                                                              d_rule_a, d_rule_b, d_bad);
             e = cudaGetLastError();
         }
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(index_build_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)ism.bytes);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(index_build_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)ism.bytes);
+        if (e == cudaSuccess &&
+            (pv_smem_limit(ctx, (const void *)index_build_kernel<false>, "index_build_kernel smem") ||
+             pv_smem_limit(ctx, (const void *)index_build_kernel<true>, "index_build_kernel smem"))) {
+            free_temps();
+            pv_free_tables(ctx, t);
+            return PV_ECUDA;
+        }
         if (e == cudaSuccess) {
             index_build_kernel<false><<<S, kIndexThreads, ism.bytes, ls>>>(d_rule_offs, d_tab_offs, d_rule_a,
                                                                            d_rule_b, d_sizes, nullptr, nullptr, ism);
@@ -2299,9 +2300,13 @@ int tables_end(pv_ctx *ctx, pv_table_load &L) {
         pv_free_tables(ctx, t);
         return pv_fail(ctx, PV_EINVAL, "largest flow table needs %u bytes of shared memory", max_linear);
     }
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_scatter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)(2 * kSmemHistMax * 4)),
-                "walk_scatter_kernel smem");
+    {
+        const int rc3 = pv_smem_limit(ctx, (const void *)walk_scatter_kernel, "walk_scatter_kernel smem");
+        if (rc3) {
+            pv_free_tables(ctx, t);
+            return rc3;
+        }
+    }
     // host copy for rule installation
     pv_table_host &h = ctx->tbh;
     h.rule_offs.assign(rule_offs, rule_offs + S + 1);
@@ -2429,13 +2434,9 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
     const HopKernel hop_fn = direct ? pick_hop<true>(indexed, pol, stats, false) : pick_hop<false>(indexed, pol, stats, false);
     const HopKernel hop_fn0 = direct ? pick_hop<true>(indexed, pol, stats, true) : pick_hop<false>(indexed, pol, stats, true);
     const TailKernel tail_fn = direct ? pick_tail<true>(pol, stats) : pick_tail<false>(pol, stats);
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute((const void *)hop_fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)hop_smem),
-                "walk_hop_kernel smem");
-    PV_TRY_CUDA(ctx, cudaFuncSetAttribute((const void *)hop_fn0, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)hop_smem),
-                "walk_hop_kernel smem");
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&hop_blocks_per_sm, (const void *)hop_fn, kHopThreads, hop_smem);
+    if (int rc = pv_smem_limit(ctx, (const void *)hop_fn, "walk_hop_kernel smem")) return rc;
+    if (int rc = pv_smem_limit(ctx, (const void *)hop_fn0, "walk_hop_kernel smem")) return rc;
+    hop_blocks_per_sm = pv_blocks_per_sm(ctx, (const void *)hop_fn, kHopThreads, hop_smem);
     const uint32_t hop_grid = (uint32_t)ctx->num_sms * (uint32_t)std::max(1, hop_blocks_per_sm);
     const uint32_t init_grid = (uint32_t)ctx->num_sms * 8;
     const uint32_t max_desc = std::max(hop_grid, init_grid);
@@ -2491,12 +2492,9 @@ int walk_probes(pv_ctx *ctx, uint32_t M, const pv_probe *d_probes, uint32_t hop_
         const bool by_group = ba->pods <= kGroupInitMaxPods && gsm <= kGroupInitSmem && groups <= 0x7FFFFFFFull;
         const uint64_t wait_ns = ctx->opt_test_stall_staging ? 50ull * 1000 * 1000 : 2ull * 1000 * 1000 * 1000;
         if (by_group) {
-            PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_init_group_kernel<true>,
-                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGroupInitSmem),
-                        "walk_init_group_kernel smem");
-            PV_TRY_CUDA(ctx, cudaFuncSetAttribute(walk_init_group_kernel<false>,
-                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGroupInitSmem),
-                        "walk_init_group_kernel smem");
+            const int rc2 = pol ? pv_smem_limit(ctx, (const void *)walk_init_group_kernel<true>, "walk_init_group_kernel smem")
+                                : pv_smem_limit(ctx, (const void *)walk_init_group_kernel<false>, "walk_init_group_kernel smem");
+            if (rc2) return rc2;
         }
         if (by_group && pol)
             walk_init_group_kernel<true><<<groups32, kGroupInitThreads, gsm, st>>>(

@@ -2,7 +2,10 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <mutex>
 #include <new>
+#include <utility>
+#include <vector>
 
 #include "pv_internal.cuh"
 
@@ -85,6 +88,39 @@ int pv_check_launch(pv_ctx *ctx, const char *what) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return pv_cuda_fail(ctx, e, what);
     return PV_OK;
+}
+
+int pv_smem_limit(pv_ctx *ctx, const void *fn, const char *what) {
+    static std::mutex mu;
+    static std::vector<std::pair<int, const void *>> done;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return pv_cuda_fail(ctx, e, what);
+    std::lock_guard<std::mutex> lock(mu);
+    for (const auto &d : done)
+        if (d.first == dev && d.second == fn) return PV_OK;
+    // the dynamic limit plus the kernel's static shared memory may not exceed
+    // the device's opt-in maximum
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, fn);
+    if (e != cudaSuccess) return pv_cuda_fail(ctx, e, what);
+    const size_t lim = ctx->max_smem_optin > fa.sharedSizeBytes ? ctx->max_smem_optin - fa.sharedSizeBytes : 0;
+    e = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)lim);
+    if (e != cudaSuccess) return pv_cuda_fail(ctx, e, what);
+    done.emplace_back(dev, fn);
+    return PV_OK;
+}
+
+int pv_blocks_per_sm(pv_ctx *ctx, const void *fn, int threads, size_t smem) {
+    for (const auto &o : ctx->occ)
+        if (o.fn == fn && o.threads == threads && o.smem == smem) return o.blocks;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, fn, threads, smem) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+    }
+    ctx->occ.push_back({fn, threads, smem, n});
+    return n;
 }
 
 void *pv_scratch(pv_ctx *ctx, size_t bytes) {

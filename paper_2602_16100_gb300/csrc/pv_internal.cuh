@@ -111,6 +111,10 @@ struct pv_ctx {
     cudaStream_t reach_side = nullptr;
     cudaEvent_t reach_fork = nullptr, reach_join = nullptr;
     pv_prof_state prof;
+    // blocks per SM by (kernel, block size, dynamic shared memory): the
+    // occupancy query runs once per combination
+    struct occ_entry { const void *fn; int threads; size_t smem; int blocks; };
+    std::vector<occ_entry> occ;
     int num_sms = 0;
     size_t max_smem_optin = 0;
     std::string err;
@@ -168,6 +172,16 @@ int pv_load_end(pv_ctx *ctx);
 void pv_use_begin(pv_ctx *ctx, cudaStream_t st);
 void pv_mark_use(pv_ctx *ctx, cudaStream_t st);
 int pv_check_launch(pv_ctx *ctx, const char *what);
+// Raises a kernel's dynamic shared-memory limit to the device maximum (less
+// the kernel's static shared memory), once
+// per (device, kernel).  The limit is a process-wide permission, not a
+// reservation (occupancy follows each launch's own size), so one setting at
+// the maximum serves every launch, and no thread lowers it between another
+// thread's setting and launch; later calls only look the pair up.
+int pv_smem_limit(pv_ctx *ctx, const void *fn, const char *what);
+// Resident blocks per SM of fn at this block size and dynamic shared memory
+// (0 when the query fails), cached in the context.
+int pv_blocks_per_sm(pv_ctx *ctx, const void *fn, int threads, size_t smem);
 // Kernel-group timing: no-ops unless profiling is enabled.  Returns the pair
 // index to pass to pv_prof_stop (or -1).
 int pv_prof_start(pv_ctx *ctx, cudaStream_t st, int group);
