@@ -542,6 +542,48 @@ __device__ __forceinline__ void and_resolved2(const ResolvedExprs &rx, uint32_t 
     }
 }
 
+// ANDs resolved expression e's node set into a 160-word span's accumulators
+// of one lane: chunk q (four words, loaded when l0) and word w (loaded when
+// l1); words past the rows read 0 before the complement.
+__device__ __forceinline__ void and_resolved5(const ResolvedExprs &rx, uint32_t warp, uint32_t e,
+                                              const uint32_t *__restrict__ rows, uint32_t q, uint32_t w, bool l0,
+                                              bool l1, uint4 &a0, uint32_t &a1) {
+    const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = meta >> 8;
+    uint4 v0 = make_uint4(0, 0, 0, 0);
+    uint32_t v1 = 0;
+    uint32_t j = 0;
+    for (; j + 1 < n; j += 2) {   // two rows per step: four loads in flight
+        const uint32_t *rp = rows + rx.off[warp][e][j], *rq = rows + rx.off[warp][e][j + 1];
+        uint4 x0 = make_uint4(0, 0, 0, 0), y0 = x0;
+        uint32_t x1 = 0, y1 = 0;
+        if (l0) {
+            x0 = __ldg(reinterpret_cast<const uint4 *>(rp) + q);
+            y0 = __ldg(reinterpret_cast<const uint4 *>(rq) + q);
+        }
+        if (l1) {
+            x1 = __ldg(rp + w);
+            y1 = __ldg(rq + w);
+        }
+        v0.x |= x0.x | y0.x; v0.y |= x0.y | y0.y; v0.z |= x0.z | y0.z; v0.w |= x0.w | y0.w;
+        v1 |= x1 | y1;
+    }
+    if (j < n) {
+        const uint32_t *rp = rows + rx.off[warp][e][j];
+        if (l0) {
+            const uint4 x = __ldg(reinterpret_cast<const uint4 *>(rp) + q);
+            v0.x |= x.x; v0.y |= x.y; v0.z |= x.z; v0.w |= x.w;
+        }
+        if (l1) v1 |= __ldg(rp + w);
+    }
+    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) {
+        a0.x &= ~v0.x; a0.y &= ~v0.y; a0.z &= ~v0.z; a0.w &= ~v0.w;
+        a1 &= ~v1;
+    } else {
+        a0.x &= v0.x; a0.y &= v0.y; a0.z &= v0.z; a0.w &= v0.w;
+        a1 &= v1;
+    }
+}
+
 // Clears the bits of nodes >= N in the four words from w0.
 __device__ __forceinline__ void clip_rows4(uint4 &acc, uint32_t w0, uint32_t N) {
     const uint32_t full_words = N >> 5, tail_bits = N & 31;
@@ -618,26 +660,36 @@ __global__ void __launch_bounds__(kRowsThreads) sel_rows_kernel(
             }
         };
         if (resolved) {
-            // a lane takes chunks q and q + 32 of each 64-chunk span, so one
-            // pass over the resolved rows (offsets, loop steps) serves both
-            for (uint32_t qb = 0; qb < W / 4; qb += 64) {
-                const uint32_t q0 = qb + lane, q1 = q0 + 32;
-                const bool h0 = q0 < W / 4, h1 = q1 < W / 4;
-                const bool l0 = h0 && q0 * 4 < row_words, l1 = h1 && q1 * 4 < row_words;
-                uint4 a0 = make_uint4(~0u, ~0u, ~0u, ~0u), a1 = a0;
+            // of each 160-word span a lane takes chunk lane (words 4 lane ..
+            // 4 lane + 3) and word 128 + lane: five words per lane, so a row
+            // of up to 5,120 nodes keeps every lane busy in one pass over the
+            // resolved rows
+            for (uint32_t sb = 0; sb < W; sb += 160) {
+                const uint32_t q = sb / 4 + lane, w = sb + 128 + lane;
+                const bool h0 = q * 4 < W, h1 = w < W;
+                const bool l0 = h0 && q * 4 < row_words, l1 = h1 && w < row_words;
+                uint4 a0 = make_uint4(~0u, ~0u, ~0u, ~0u);
+                uint32_t a1 = ~0u;
                 for (uint32_t i = 0; i < E; ++i) {
-                    and_resolved2(rx, warp, rx.order[warp][i], rows, q0, q1, l0, l1, a0, a1);
+                    and_resolved5(rx, warp, rx.order[warp][i], rows, q, w, l0, l1, a0, a1);
                     // every node of the span rejected: the remaining sets
-                    // cannot add any back (chunks past the rows hold no nodes)
-                    const bool nz = (l0 && (a0.x | a0.y | a0.z | a0.w)) || (l1 && (a1.x | a1.y | a1.z | a1.w));
+                    // cannot add any back (words past the rows hold no nodes)
+                    const bool nz = (l0 && (a0.x | a0.y | a0.z | a0.w)) || (l1 && a1);
                     if (!__any_sync(PV_FULL_MASK, nz)) {
                         a0 = make_uint4(0, 0, 0, 0);
-                        a1 = a0;
+                        a1 = 0;
                         break;
                     }
                 }
-                if (h0) finish(a0, q0);
-                if (h1) finish(a1, q1);
+                if (h0) finish(a0, q);
+                if (h1) {
+                    const uint32_t full_words = N >> 5, tail_bits = N & 31;
+                    if (w > full_words || (w == full_words && tail_bits == 0)) a1 = 0;
+                    else if (w == full_words) a1 &= (1u << tail_bits) - 1u;
+                    bits[(size_t)pc * W + w] = a1;
+                    any = any || a1 != 0;
+                    if (a < N && (a >> 5) == w) aok = (a1 >> (a & 31)) & 1u;
+                }
             }
         } else {
             for (uint32_t q = lane; q < W / 4; q += 32) {
