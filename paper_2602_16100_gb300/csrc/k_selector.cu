@@ -498,50 +498,6 @@ __device__ __forceinline__ uint32_t resolve_slots(ResolvedExprs &rx, uint32_t wa
     return (bad ? 1u : 0u) | (unknown ? 2u : 0u);
 }
 
-// ANDs resolved expression e's node set into the accumulators of chunks q0
-// and q1 (loaded when l0 / l1: words past the rows read 0 before the
-// complement).
-__device__ __forceinline__ void and_resolved2(const ResolvedExprs &rx, uint32_t warp, uint32_t e,
-                                              const uint32_t *__restrict__ rows, uint32_t q0, uint32_t q1, bool l0,
-                                              bool l1, uint4 &a0, uint4 &a1) {
-    const uint32_t meta = rx.meta[warp][e], op = meta & 0xFFu, n = meta >> 8;
-    uint4 v0 = make_uint4(0, 0, 0, 0), v1 = v0;
-    uint32_t j = 0;
-    for (; j + 1 < n; j += 2) {   // two rows per step: four loads in flight
-        const uint4 *rp = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j]);
-        const uint4 *rq = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j + 1]);
-        uint4 x0 = make_uint4(0, 0, 0, 0), y0 = x0, x1 = x0, y1 = x0;
-        if (l0) {
-            x0 = __ldg(rp + q0);
-            y0 = __ldg(rq + q0);
-        }
-        if (l1) {
-            x1 = __ldg(rp + q1);
-            y1 = __ldg(rq + q1);
-        }
-        v0.x |= x0.x | y0.x; v0.y |= x0.y | y0.y; v0.z |= x0.z | y0.z; v0.w |= x0.w | y0.w;
-        v1.x |= x1.x | y1.x; v1.y |= x1.y | y1.y; v1.z |= x1.z | y1.z; v1.w |= x1.w | y1.w;
-    }
-    if (j < n) {
-        const uint4 *rp = reinterpret_cast<const uint4 *>(rows + rx.off[warp][e][j]);
-        if (l0) {
-            const uint4 x = __ldg(rp + q0);
-            v0.x |= x.x; v0.y |= x.y; v0.z |= x.z; v0.w |= x.w;
-        }
-        if (l1) {
-            const uint4 x = __ldg(rp + q1);
-            v1.x |= x.x; v1.y |= x.y; v1.z |= x.z; v1.w |= x.w;
-        }
-    }
-    if (op == PV_NOTIN || op == PV_DOESNOTEXIST) {
-        a0.x &= ~v0.x; a0.y &= ~v0.y; a0.z &= ~v0.z; a0.w &= ~v0.w;
-        a1.x &= ~v1.x; a1.y &= ~v1.y; a1.z &= ~v1.z; a1.w &= ~v1.w;
-    } else {
-        a0.x &= v0.x; a0.y &= v0.y; a0.z &= v0.z; a0.w &= v0.w;
-        a1.x &= v1.x; a1.y &= v1.y; a1.z &= v1.z; a1.w &= v1.w;
-    }
-}
-
 // ANDs resolved expression e's node set into a 160-word span's accumulators
 // of one lane: chunk q (four words, loaded when l0) and word w (loaded when
 // l1); words past the rows read 0 before the complement.
@@ -754,28 +710,40 @@ __global__ void __launch_bounds__(kRowsThreads) sel_terms_kernel(
         bool any = false, aok = false;
         auto finish = [&](uint4 res, uint32_t q) {
             const uint32_t w0 = q * 4;
-            clip_rows4(res, w0, N);
+            if (w0 + 4 > (N >> 5)) clip_rows4(res, w0, N);   // only chunks reaching node N - 1 or past it
             out[q] = res;
             any = any || (res.x | res.y | res.z | res.w) != 0;
-            const uint32_t *aw = &res.x;
-            if (a < N && (a >> 5) >= w0 && (a >> 5) < w0 + 4) aok = (aw[(a >> 5) - w0] >> (a & 31)) & 1u;
+            if (a < N && (a >> 7) == q) {   // the assigned node's word is in this chunk
+                const uint32_t wsel = (a >> 5) & 3u;
+                const uint32_t word = wsel == 0 ? res.x : wsel == 1 ? res.y : wsel == 2 ? res.z : res.w;
+                aok = (word >> (a & 31)) & 1u;
+            }
         };
         const uint4 none = make_uint4(0, 0, 0, 0), all = make_uint4(~0u, ~0u, ~0u, ~0u);
-        if (resolved) {   // chunks q and q + 32 per lane, as in sel_rows_kernel
-            for (uint32_t qb = 0; qb < W / 4; qb += 64) {
-                const uint32_t q0 = qb + lane, q1 = q0 + 32;
-                const bool h0 = q0 < W / 4, h1 = q1 < W / 4;
-                const bool l0 = h0 && q0 * 4 < row_words, l1 = h1 && q1 * 4 < row_words;
-                uint4 r0 = t0 == t1 ? all : none, r1 = r0;
+        if (resolved) {   // a 160-word span per pass, five words per lane, as in sel_rows_kernel
+            for (uint32_t sb = 0; sb < W; sb += 160) {
+                const uint32_t q = sb / 4 + lane, w = sb + 128 + lane;
+                const bool h0 = q * 4 < W, h1 = w < W;
+                const bool l0 = h0 && q * 4 < row_words, l1 = h1 && w < row_words;
+                uint4 r0 = t0 == t1 ? all : none;
+                uint32_t r1 = t0 == t1 ? ~0u : 0u;
                 for (uint32_t t = t0; t < t1; ++t) {
                     const uint32_t lo = term_offs[t] - e0, hi = term_offs[t + 1] - e0;
-                    uint4 a0 = hi > lo ? all : none, a1 = a0;
-                    for (uint32_t e = lo; e < hi; ++e) and_resolved2(rx, warp, e, rows, q0, q1, l0, l1, a0, a1);
+                    uint4 a0 = hi > lo ? all : none;
+                    uint32_t a1 = hi > lo ? ~0u : 0u;
+                    for (uint32_t e = lo; e < hi; ++e) and_resolved5(rx, warp, e, rows, q, w, l0, l1, a0, a1);
                     r0.x |= a0.x; r0.y |= a0.y; r0.z |= a0.z; r0.w |= a0.w;
-                    r1.x |= a1.x; r1.y |= a1.y; r1.z |= a1.z; r1.w |= a1.w;
+                    r1 |= a1;
                 }
-                if (h0) finish(r0, q0);
-                if (h1) finish(r1, q1);
+                if (h0) finish(r0, q);
+                if (h1) {
+                    const uint32_t full_words = N >> 5, tail_bits = N & 31;
+                    if (w > full_words || (w == full_words && tail_bits == 0)) r1 = 0;
+                    else if (w == full_words) r1 &= (1u << tail_bits) - 1u;
+                    bits[(size_t)p * W + w] = r1;
+                    any = any || r1 != 0;
+                    if (a < N && (a >> 5) == w) aok = (r1 >> (a & 31)) & 1u;
+                }
             }
         } else {
             for (uint32_t q = lane; q < W / 4; q += 32) {
