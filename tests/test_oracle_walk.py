@@ -213,3 +213,98 @@ def test_walks_equal_recursive_trace_fat_tree_and_random_graph():
     pr["src_host"] = np.arange(len(pr)) % e.network.num_hosts
     pr["src_ip"] = e.network.host_ip[pr["src_host"]]
     _check_against_trace(e.network, pr, e.probes.hop_cap)
+
+
+# ---------------------------------------------------------------------------
+# two bounces in a row (the walk's two-switch cycle shortcut)
+# ---------------------------------------------------------------------------
+def _symmetric(net):
+    po, pp = net.port_offs, net.port_peer
+    for u in range(net.num_switches):
+        for p in range(int(po[u]), int(po[u + 1])):
+            peer = int(pp[p])
+            if peer < 0 or peer & W.HOST_BIT:
+                continue
+            v, q = peer >> 8, peer & 0xFF
+            if int(pp[int(po[v]) + q]) != (u << 8 | (p - int(po[u]))):
+                return False
+    return True
+
+
+def _first_double_bounce(net, pr, cap):
+    """Follow the probe's (switch, in_port) states while it is handed to
+    switches (masks that permit every region); return (h, s_h, s_h+1) for the
+    first visit h >= 1 at which it leaves by its in_port right after leaving
+    the previous switch by that switch's in_port, with h + 1 < cap; else None."""
+    hdr = (int(pr["src_ip"]), int(pr["dst_ip"]), int(pr["dport"]))
+    s, p = int(net.host_switch[int(pr["src_host"])]), int(net.host_port[int(pr["src_host"])])
+    prev_bounce = False
+    for h in range(cap - 1):
+        rs = net.rules[net.rule_offs[s]:net.rule_offs[s + 1]]
+        i = first_match_sorted(rs, p, *hdr)
+        if i < 0 or int(rs[i]["action"]) == W.DROP:
+            return None
+        port = int(rs[i]["action"])
+        if port >= int(net.port_offs[s + 1] - net.port_offs[s]):
+            return None
+        peer = int(net.port_peer[net.port_offs[s] + port])
+        if peer < 0 or peer & W.HOST_BIT:
+            return None
+        bounce = port == p
+        if bounce and prev_bounce:
+            return h, s, peer >> 8
+        prev_bounce = bounce
+        s, p = peer >> 8, peer & 0xFF
+    return None
+
+
+def test_two_bounces_in_a_row_prove_a_two_switch_cycle():
+    """With symmetric cabling, a probe that leaves two switches in a row by
+    the port it came in by walks back and forth between them until the hop
+    cap: the full walk ends PV_LOOP with hops = cap at the switch of visit
+    cap - 1, which is s_h when cap - 1 - h is even and s_h+1 otherwise.
+    Checked against the oracle's full walks on every probe that shows the
+    pattern, at several caps."""
+    cases = []
+    e = W.end_to_end(seed=9, num_switches=24, num_intents=8, probes_per_intent=40, rules_per_switch=80)
+    pr = e.probes.probes.copy()
+    pr["src_host"] = np.arange(len(pr)) % e.network.num_hosts
+    pr["src_ip"] = e.network.host_ip[pr["src_host"]]
+    cases.append((e.network, pr))
+    d = W.fat_tree(seed=7, k=4, rules_per_switch=120, num_probes=600, hop_cap=12)
+    cases.append((d["network"], d["probes"].probes.copy()))
+    checked = 0
+    for net, pr in cases:
+        assert _symmetric(net)
+        pr["allowed_mask"] = 0xFFFFFFFF
+        for cap in (4, 7, 12, 31, 32):
+            res = oracle.verify_probes(net, pr, cap)
+            for k in range(len(pr)):
+                hit = _first_double_bounce(net, pr[k], cap)
+                if hit is None:
+                    continue
+                h, s0, s1 = hit
+                want = (W.ST_LOOP, cap, s0 if (cap - 1 - h) % 2 == 0 else s1)
+                got = tuple(int(x) for x in (res[k]["status"], res[k]["hops"], res[k]["last_switch"]))
+                assert got == want, (cap, k, got, want)
+                checked += 1
+    assert checked > 50
+
+
+def test_two_bounces_on_asymmetric_cabling_prove_nothing():
+    """Port 0 of X, Y and Z leads X -> Y -> Z -> X (not back), every switch
+    sends everything out of port 0: every hop after the first is a bounce,
+    yet the walk has period 3, so the parity rule fails (cap 5: visit 4 is at
+    Y, the rule would say Z)."""
+    net = make_net([2, 1, 1], [], [(0, 1, ip(10, 0, 0, 1))], [0, 0, 0],
+                   [[rule(100, 0, 0, 0)], [rule(100, 0, 0, 0)], [rule(100, 0, 0, 0)]])
+    net.port_peer[net.port_offs[0]] = (1 << 8) | 0
+    net.port_peer[net.port_offs[1]] = (2 << 8) | 0
+    net.port_peer[net.port_offs[2]] = (0 << 8) | 0
+    assert not _symmetric(net)
+    pr = probe(0, ip(10, 0, 0, 1), ip(99, 0, 0, 1), 1)
+    h, s0, s1 = _first_double_bounce(net, pr[0], 5)
+    assert (h, s0, s1) == (2, 2, 0)
+    res = oracle.verify_probes(net, pr, 5)
+    assert (int(res[0]["status"]), int(res[0]["hops"]), int(res[0]["last_switch"])) == (W.ST_LOOP, 5, 1)
+    assert int(res[0]["last_switch"]) != (s0 if (5 - 1 - h) % 2 == 0 else s1)
