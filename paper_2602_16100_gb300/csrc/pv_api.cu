@@ -119,6 +119,7 @@ int pv_blocks_per_sm(pv_ctx *ctx, const void *fn, int threads, size_t smem) {
         cudaGetLastError();
         n = 0;
     }
+    if (ctx->occ.size() >= 64) ctx->occ.clear();   // table sets of many shapes: start over
     ctx->occ.push_back({fn, threads, smem, n});
     return n;
 }
